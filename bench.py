@@ -1,0 +1,319 @@
+"""Benchmark of one MeBP LoRA training step (Algorithm 1) on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config C] [--impl gb300|reference]
+
+A step = embed -> checkpointed forward loop over all blocks -> LM-head cross-entropy
+(forward + backward, vocabulary-chunked) -> reverse loop of block recompute + backward,
+producing the loss and every LoRA gradient (mebp_lora_step).  The default workload is the
+full Qwen2.5-0.5B-shaped model (24 blocks, vocab 151936, batch 1 x seq 512, LoRA r8 on
+q/k/v/o, 4-bit group-64 base weights).  Prints one JSON line (rank 0).
+
+--impl reference times the CPU oracle (plain numpy fp64) on the host cores, on a bounded
+sample of the same workload (one block's forward + recompute + backward and an LM-head
+token sample), extrapolated to the step.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+from workload import synth  # noqa: E402
+
+METRIC = "train tokens/s per LoRA step (1 GB300); fused dequant-GEMM % of BF16 tensor peak"
+
+
+def workload_name(d) -> str:
+    return (f"{d.name}: {d.n_layers} blocks (D {d.hidden}, H {d.n_heads}/KV {d.n_kv_heads}, hd {d.head_dim}, "
+            f"I {d.intermediate}, {d.act}), vocab {d.vocab}, batch {d.batch} x seq {d.seq}, "
+            f"LoRA r{d.rank} on {'/'.join(d.targets)}, 4-bit g64 fp16-scale base weights"
+            + (", checkpoints spilled to pinned host" if d.spill else ""))
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return p, "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+# ----------------------------------------------------------------------------- CPU oracle sample
+def oracle_sample(d, lm_tokens: int = 32):
+    """Time the oracle on one block (forward, recompute, backward) and an LM-head token
+    sample; return (tokens/s extrapolated to the whole step, description)."""
+    from oracle import model as OM
+    from oracle import quant
+
+    W = synth.block_weights(d, 0)
+    L = OM.lora64(synth.lora_weights(d, 0))
+    x = synth.hidden_input(d).astype(np.float64)
+    G = synth.upstream_grad(d).astype(np.float64)
+    t0 = time.perf_counter()
+    pm = OM.PackedModel.compress([W])
+    Wd = pm.decompress_block(0)
+    OM.block_objective(x, Wd, L, G, d)
+    t_block = time.perf_counter() - t0
+    t_lm = 0.0
+    if d.vocab:
+        E, gf = synth.embedding(d)
+        qE = quant.compress(E)
+        t1 = time.perf_counter()
+        Ed = quant.dequant(*qE)
+        t_deq = time.perf_counter() - t1
+        h = x[:lm_tokens]
+        tg = synth.token_ids(d).reshape(-1)[:lm_tokens].astype(np.int64)
+        t2 = time.perf_counter()
+        OM.lm_head_ce(h, gf.astype(np.float64), Ed, tg, d.eps)
+        t_lm = t_deq + (time.perf_counter() - t2) * d.tokens / lm_tokens
+    t_step = d.n_layers * t_block + t_lm
+    desc = (f"oracle (numpy fp64) on 1 of {d.n_layers} blocks at the full {d.tokens} tokens (compress + decompress + "
+            f"forward + recompute + backward) and the LM head on {lm_tokens} of {d.tokens} tokens, extrapolated "
+            f"linearly to the step")
+    return d.tokens / t_step, desc
+
+
+# ----------------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.p = None
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                       "-i", str(gpu_index), "-lms", "100"], stdout=subprocess.PIPE,
+                                      stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.p = None
+
+    def stop(self):
+        if self.p is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.p.terminate()
+        try:
+            out, _ = self.p.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.p.kill()
+            out, _ = self.p.communicate()
+        sm, smax, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- GPU arm
+def build_model(ctx, d, device):
+    import torch
+
+    from paper_2510_03425_gb300.model import DeviceBlock, DeviceModel, PackedLinear, compress
+    big = d.n_layers * d.hidden * d.intermediate > 2e8
+    blocks = []
+    for i in range(d.n_layers):
+        if big:
+            W = synth.torch_block_weights(d, i, device=device)
+        else:
+            W = {k: torch.from_numpy(v).to(device) for k, v in synth.block_weights(d, i).items()}
+        blocks.append(DeviceBlock(ctx, W))
+        del W
+    if big:
+        E, gf = synth.torch_embedding(d, device=device)
+    else:
+        En, gfn = synth.embedding(d)
+        E, gf = torch.from_numpy(En).to(device), torch.from_numpy(gfn).to(device)
+    emb = PackedLinear(*compress(ctx, E))
+    del E
+    torch.cuda.empty_cache()
+    return DeviceModel(blocks, emb, gf)
+
+
+def run_gpu(args, d, rank, world, local_rank):
+    import torch
+
+    from paper_2510_03425_gb300 import mebp as M
+    from paper_2510_03425_gb300.model import Context, LoraSet
+
+    device = torch.device("cuda", local_rank)
+    torch.cuda.set_device(device)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    ctx = Context(d, device=local_rank)
+    model = build_model(ctx, d, device)
+    ls = LoraSet([synth.lora_weights(d, i) for i in range(d.n_layers)], device=device)
+    ids_host = torch.from_numpy(synth.token_ids(d, seed=2 + rank)).pin_memory()
+    ids = ids_host.to(device)
+    loss = torch.zeros(1, device=device)
+    loss_host = torch.zeros(1).pin_memory()
+    mstruct = model.struct()
+    st = torch.cuda.current_stream(device)
+
+    def step():
+        M.mebp_lora_step(ctx.handle, mstruct, ls.lora_array(), ids, loss, ls.grads_array(), False, st)
+
+    gpu_index = local_rank
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis and vis.split(",")[local_rank].strip().isdigit():
+        gpu_index = int(vis.split(",")[local_rank])
+    clocks = ClockSampler(gpu_index)
+    for _ in range(args.warmup):
+        step()
+    ctx.sync()
+    # ---- timed region: K steps, inputs resident in HBM
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    n0 = M.mebp_kernel_launches()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(st)
+    for _ in range(args.steps):
+        step()
+    e1.record(st)
+    torch.cuda.synchronize()
+    launches = M.mebp_kernel_launches() - n0
+    if dist:
+        dist.barrier()
+    clk = clocks.stop()
+    ctx.sync()
+    t = e0.elapsed_time(e1) / 1e3
+    if dist:
+        tt = torch.tensor([t], device=device)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        t = float(tt.item())
+    value = world * d.tokens * args.steps / t
+
+    # ---- GEMM roofline: CUDA events around every fused dequant-GEMM launch of K more steps
+    M.mebp_profile_begin(ctx.handle)
+    for _ in range(args.steps):
+        step()
+    prof = M.mebp_profile_end(ctx.handle)
+
+    # ---- end to end through the public API: ids host->device, step, loss device->host
+    ctx.sync()
+    h2d = ids_host.numel() * ids_host.element_size()
+    d2h = loss.numel() * loss.element_size()
+    e2, e3 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e2.record(st)
+    for _ in range(args.steps):
+        ids.copy_(ids_host, non_blocking=True)
+        step()
+        loss_host.copy_(loss, non_blocking=True)
+    e3.record(st)
+    torch.cuda.synchronize()
+    te = e2.elapsed_time(e3) / 1e3
+    if dist:
+        tt = torch.tensor([te], device=device)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        te = float(tt.item())
+    ctx.sync()
+
+    if rank != 0:
+        if dist:
+            dist.destroy_process_group()
+        return None
+    pk, src = peaks()
+    long_step = t / args.steps > 1.0
+    peak = pk["bf16_tflops_sustained"] if long_step else pk["bf16_tflops"]
+    achieved = prof.gemm_flops / (prof.gemm_ms / 1e3) / 1e12 if prof.gemm_ms > 0 else None
+    weights_mb = sum(b.qkv.qpack.numel() + b.o.qpack.numel() + b.gate_up.qpack.numel() + b.down.qpack.numel()
+                     for b in model.blocks) / 2**20 * (1 + 1 / 16)
+    out = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * t / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": workload_name(d), "config_index": args.config, "global_batch": world * d.batch,
+                   "seq_len": d.seq, "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                   "l2": f"inputs larger than L2: {weights_mb:.0f} MB of packed block weights plus the "
+                         f"{d.vocab}x{d.hidden} packed LM head are streamed every step"},
+        "roofline": {"kernel": "dequant_gemm_kernel (fused 4-bit dequant GEMM, tcgen05)", "bound": "tensor",
+                     "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": (achieved / peak) if achieved else None, "traffic": None,
+                     "peak_source": f"{src} {'sustained' if long_step else 'burst'} bf16 (MEASURED_PEAKS.json)",
+                     "launches_per_step": prof.gemm_launches / args.steps,
+                     "share_of_step": (prof.gemm_ms / 1e3) / t if t > 0 else None,
+                     "fwd_tflops": prof.fwd_flops / max(prof.fwd_ms, 1e-9) / 1e9,
+                     "dx_tflops": prof.dx_flops / max(prof.dx_ms, 1e-9) / 1e9},
+        "e2e": {"value": world * d.tokens * args.steps / te, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": int(launches),
+        "clocks": clk,
+    }
+    ctx.close()
+    if dist:
+        dist.destroy_process_group()
+    return out
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--config", type=int, default=1, help="workload preset 0..4 (default 1)")
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(3, args.warmup)
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    d = synth.preset(args.config)
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        cores = os.cpu_count()
+        vals = []
+        for i in range(args.warmup + args.steps):
+            v, desc = oracle_sample(d)
+            if i >= args.warmup:
+                vals.append(v)
+        v = statistics.mean(vals)
+        print(json.dumps({
+            "metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * d.tokens / v, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": workload_name(d), "config_index": args.config, "global_batch": d.batch,
+                       "seq_len": d.seq, "parallelism": "host cores"},
+            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": desc},
+            "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        }), flush=True)
+        return
+
+    out = run_gpu(args, d, rank, world, local_rank)
+    if out is None:
+        return
+    if world == 1 and not args.no_cpu_baseline:
+        v, desc = oracle_sample(d)
+        out["cpu_baseline"] = {"value": v, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+                               "sample": desc}
+    print(json.dumps(out), flush=True)
+
+
+if __name__ == "__main__":
+    main()

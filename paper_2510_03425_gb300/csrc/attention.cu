@@ -1,0 +1,416 @@
+// Causal grouped-query attention of the decoder block, forward and backward, as tiled
+// warp-level tensor-core kernels (mma.sync m16n8k16, bf16 in / fp32 accumulate).
+//
+//   forward : o = softmax(q k^T / sqrt(hd) + causal) v, per (sequence, query head); query head h
+//             reads key/value head h / (H/KV).  Saves lse = log-sum-exp of each score row.
+//   backward: dP = dO v^T, dS = P (dP - rowsum(dO o)), dq = dS k / sqrt(hd),
+//             dk = dS^T q / sqrt(hd), dv = P^T dO; dk, dv summed over the query heads of a
+//             group.  P is recomputed from q, k and lse.  dk/dv (one CTA per key block and
+//             kv head, looping over the group's query heads) and dq (one CTA per query block)
+//             are separate passes so every output element is written exactly once
+//             (deterministic, no atomics).
+// q, k, v live in the fused projection buffer [T, (H + 2 KV) hd] (q heads, k heads, v heads);
+// token t = b*S + s.
+#include "kernels.h"
+#include "mma.cuh"
+
+namespace mebp {
+namespace attn {
+
+constexpr int BQ = 64, BKV = 64;
+constexpr float kLog2e = 1.4426950408889634f;
+
+template <int HD>
+__device__ __forceinline__ void load_tile(uint16_t* dst, const uint16_t* base, int64_t ld, int64_t tok0, int r0,
+                                          int S, int col, int tid) {
+  constexpr int LD = HD + 8, CH = HD / 8;
+  for (int c = tid; c < 64 * CH; c += 128) {
+    const int r = c / CH, cc = c % CH;
+    const bool v = r0 + r < S;
+    const uint16_t* src = v ? base + (tok0 + r0 + r) * ld + col + cc * 8 : base;
+    cp_async16(smem_u32(dst + r * LD + cc * 8), src, v);
+  }
+}
+
+// S (16 rows of this warp x 64 columns) = A_rows . B_rows^T over HD, both row-major [row][d] in smem.
+template <int HD>
+__device__ __forceinline__ void qk_tile(float (&s)[8][4], uint32_t abase, uint32_t bbase, int warp, int lane) {
+  constexpr int LD = HD + 8;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) s[i][0] = s[i][1] = s[i][2] = s[i][3] = 0.0f;
+#pragma unroll
+  for (int kk = 0; kk < HD; kk += 16) {
+    uint32_t a[4];
+    ldsm_x4(a, frag_a_addr(abase, LD, warp * 16, kk, lane));
+#pragma unroll
+    for (int nt = 0; nt < 8; nt += 2) {
+      uint32_t b[4];
+      ldsm_x4(b, frag_bn_addr(bbase, LD, nt * 8, kk, lane));
+      mma16816(s[nt], a, b[0], b[1]);
+      mma16816(s[nt + 1], a, b[2], b[3]);
+    }
+  }
+}
+
+// acc (16 x NC*8) += P (16 x 64, accumulator layout) . B[64][d0 .. d0 + NC*8) with B row-major [k][d].
+template <int HD, int NC>
+__device__ __forceinline__ void pv_tile(float (&acc)[NC][4], const float (&p)[8][4], uint32_t bbase, int d0,
+                                        int lane) {
+  constexpr int LD = HD + 8;
+#pragma unroll
+  for (int kq = 0; kq < 4; ++kq) {
+    uint32_t a[4];
+    a[0] = pack_bf16x2(p[2 * kq][0], p[2 * kq][1]);
+    a[1] = pack_bf16x2(p[2 * kq][2], p[2 * kq][3]);
+    a[2] = pack_bf16x2(p[2 * kq + 1][0], p[2 * kq + 1][1]);
+    a[3] = pack_bf16x2(p[2 * kq + 1][2], p[2 * kq + 1][3]);
+#pragma unroll
+    for (int dt = 0; dt < NC; dt += 2) {
+      uint32_t b[4];
+      ldsm_x4_t(b, frag_bk_addr(bbase, LD, d0 + dt * 8, kq * 16, lane));
+      mma16816(acc[dt], a, b[0], b[1]);
+      mma16816(acc[dt + 1], a, b[2], b[3]);
+    }
+  }
+}
+
+// ------------------------------------------------------------------------------------ forward
+template <int HD>
+__global__ void __launch_bounds__(128, 1) fwd_kernel(const uint16_t* __restrict__ qkv, int64_t ld, int S, int H,
+                                                     int KV, uint16_t* __restrict__ o, int64_t ldo,
+                                                     float* __restrict__ lse) {
+  constexpr int LD = HD + 8, NO = HD / 8;
+  extern __shared__ __align__(16) uint16_t sm[];
+  uint16_t* qs = sm;
+  uint16_t* ks = qs + BQ * LD;
+  uint16_t* vs = ks + BKV * LD;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int qb = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int kvh = h / (H / KV);
+  const int64_t tok0 = static_cast<int64_t>(b) * S;
+  const int q0 = qb * BQ;
+  const float sc = kLog2e * rsqrtf(static_cast<float>(HD));
+
+  load_tile<HD>(qs, qkv, ld, tok0, q0, S, h * HD, tid);
+  cp_async_commit();
+
+  float oacc[NO][4];
+#pragma unroll
+  for (int i = 0; i < NO; ++i) oacc[i][0] = oacc[i][1] = oacc[i][2] = oacc[i][3] = 0.0f;
+  float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.0f, 0.0f};
+  const int ra = q0 + warp * 16 + (lane >> 2);
+  const int nkb = min((q0 + BQ - 1) / BKV + 1, (S + BKV - 1) / BKV);
+
+  for (int kb = 0; kb < nkb; ++kb) {
+    const int k0 = kb * BKV;
+    load_tile<HD>(ks, qkv, ld, tok0, k0, S, (H + kvh) * HD, tid);
+    load_tile<HD>(vs, qkv, ld, tok0, k0, S, (H + KV + kvh) * HD, tid);
+    cp_async_commit();
+    cp_async_wait<0>();
+    __syncthreads();
+
+    float s[8][4];
+    qk_tile<HD>(s, smem_u32(qs), smem_u32(ks), warp, lane);
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int col = k0 + nt * 8 + 2 * (lane & 3) + (e & 1);
+        const int row = ra + ((e >> 1) << 3);
+        s[nt][e] = (col > row || col >= S) ? -INFINITY : s[nt][e] * sc;
+      }
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      float mx = -INFINITY;
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt) mx = fmaxf(mx, fmaxf(s[nt][2 * i], s[nt][2 * i + 1]));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+      const float mnew = fmaxf(mrow[i], mx);
+      const float alpha = (mnew == -INFINITY) ? 1.0f : exp2f(mrow[i] - mnew);
+      float rs = 0.0f;
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt) {
+        const float p0 = (mnew == -INFINITY) ? 0.0f : exp2f(s[nt][2 * i] - mnew);
+        const float p1 = (mnew == -INFINITY) ? 0.0f : exp2f(s[nt][2 * i + 1] - mnew);
+        s[nt][2 * i] = p0;
+        s[nt][2 * i + 1] = p1;
+        rs += p0 + p1;
+      }
+      rs += __shfl_xor_sync(0xffffffffu, rs, 1);
+      rs += __shfl_xor_sync(0xffffffffu, rs, 2);
+      lrow[i] = lrow[i] * alpha + rs;
+      mrow[i] = mnew;
+#pragma unroll
+      for (int dt = 0; dt < NO; ++dt) {
+        oacc[dt][2 * i] *= alpha;
+        oacc[dt][2 * i + 1] *= alpha;
+      }
+    }
+    pv_tile<HD, NO>(oacc, s, smem_u32(vs), 0, lane);
+    __syncthreads();
+  }
+
+  const int c = 2 * (lane & 3);
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const int row = ra + 8 * i;
+    if (row >= S) continue;
+    const float inv = 1.0f / lrow[i];
+    uint16_t* orow = o + (tok0 + row) * ldo + h * HD;
+#pragma unroll
+    for (int dt = 0; dt < NO; ++dt)
+      *reinterpret_cast<uint32_t*>(orow + dt * 8 + c) = pack_bf16x2(oacc[dt][2 * i] * inv, oacc[dt][2 * i + 1] * inv);
+    if ((lane & 3) == 0) lse[(static_cast<int64_t>(b) * H + h) * S + row] = (mrow[i] + log2f(lrow[i])) / kLog2e;
+  }
+}
+
+// ------------------------------------------------------------------------------------ backward
+// dvec[b, h, s] = sum_d dO[t, h, d] * o[t, h, d]
+__global__ void dvec_kernel(const uint16_t* __restrict__ o, const uint16_t* __restrict__ dout, int64_t ldo, int B,
+                            int S, int H, int HD, float* __restrict__ dvec) {
+  const int64_t w = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (w >= static_cast<int64_t>(B) * S * H) return;
+  const int h = static_cast<int>(w % H);
+  const int64_t t = w / H;
+  const uint32_t* a = reinterpret_cast<const uint32_t*>(o + t * ldo + h * HD);
+  const uint32_t* d = reinterpret_cast<const uint32_t*>(dout + t * ldo + h * HD);
+  float s = 0.0f;
+  for (int i = lane; i < HD / 2; i += 32) {
+    const uint32_t x = a[i], y = d[i];
+    s += bf16_lo(x) * bf16_lo(y) + bf16_hi(x) * bf16_hi(y);
+  }
+  s = warp_sum(s);
+  if (lane == 0) {
+    const int64_t b = t / S, sidx = t % S;
+    dvec[(b * H + h) * S + sidx] = s;
+  }
+}
+
+// dK, dV for one key block of one kv head, output columns d0 .. d0 + DC.
+template <int HD, int DC>
+__global__ void __launch_bounds__(128, 1) dkdv_kernel(const uint16_t* __restrict__ qkv, int64_t ld,
+                                                      const uint16_t* __restrict__ dout, int64_t ldo,
+                                                      const float* __restrict__ lse, const float* __restrict__ dvec,
+                                                      int S, int H, int KV, uint16_t* __restrict__ dqkv) {
+  constexpr int LD = HD + 8, NC = DC / 8, NCH = HD / DC;
+  extern __shared__ __align__(16) uint16_t sm[];
+  uint16_t* ks = sm;
+  uint16_t* vs = ks + BKV * LD;
+  uint16_t* qs = vs + BKV * LD;
+  uint16_t* dos = qs + BQ * LD;
+  float* lse_s = reinterpret_cast<float*>(dos + BQ * LD);
+  float* dv_s = lse_s + BQ;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int kb = blockIdx.x, kvh = blockIdx.y;
+  const int b = blockIdx.z / NCH, d0 = (blockIdx.z % NCH) * DC;
+  const int grp = H / KV;
+  const int64_t tok0 = static_cast<int64_t>(b) * S;
+  const int k0 = kb * BKV;
+  const float sc = kLog2e * rsqrtf(static_cast<float>(HD));
+
+  load_tile<HD>(ks, qkv, ld, tok0, k0, S, (H + kvh) * HD, tid);
+  load_tile<HD>(vs, qkv, ld, tok0, k0, S, (H + KV + kvh) * HD, tid);
+  cp_async_commit();
+
+  float dk[NC][4], dv[NC][4];
+#pragma unroll
+  for (int i = 0; i < NC; ++i) {
+    dk[i][0] = dk[i][1] = dk[i][2] = dk[i][3] = 0.0f;
+    dv[i][0] = dv[i][1] = dv[i][2] = dv[i][3] = 0.0f;
+  }
+  const int key_a = k0 + warp * 16 + (lane >> 2);
+  const int nqb = (S + BQ - 1) / BQ;
+
+  for (int hh = 0; hh < grp; ++hh) {
+    const int h = kvh * grp + hh;
+    for (int qb = kb; qb < nqb; ++qb) {
+      const int q0 = qb * BQ;
+      load_tile<HD>(qs, qkv, ld, tok0, q0, S, h * HD, tid);
+      load_tile<HD>(dos, dout, ldo, tok0, q0, S, h * HD, tid);
+      cp_async_commit();
+      for (int i = tid; i < BQ; i += 128) {
+        const int q = q0 + i;
+        const int64_t li = (static_cast<int64_t>(b) * H + h) * S + q;
+        lse_s[i] = q < S ? lse[li] * kLog2e : 0.0f;
+        dv_s[i] = q < S ? dvec[li] : 0.0f;
+      }
+      cp_async_wait<0>();
+      __syncthreads();
+
+      // P^T (16 keys x 64 queries)
+      float pt[8][4];
+      qk_tile<HD>(pt, smem_u32(ks), smem_u32(qs), warp, lane);
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int key = key_a + ((e >> 1) << 3);
+          const int qi = nt * 8 + 2 * (lane & 3) + (e & 1);
+          const int q = q0 + qi;
+          pt[nt][e] = (key <= q && q < S && key < S) ? exp2f(pt[nt][e] * sc - lse_s[qi]) : 0.0f;
+        }
+      // dV += P^T dO
+      pv_tile<HD, NC>(dv, pt, smem_u32(dos), d0, lane);
+      // dP^T = V dO^T ; dS^T = P^T (dP^T - dvec)
+      float dpt[8][4];
+      qk_tile<HD>(dpt, smem_u32(vs), smem_u32(dos), warp, lane);
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int qi = nt * 8 + 2 * (lane & 3) + (e & 1);
+          dpt[nt][e] = pt[nt][e] * (dpt[nt][e] - dv_s[qi]);
+        }
+      // dK += dS^T Q
+      pv_tile<HD, NC>(dk, dpt, smem_u32(qs), d0, lane);
+      __syncthreads();
+    }
+  }
+  const float inv = rsqrtf(static_cast<float>(HD));
+  const int c = 2 * (lane & 3);
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const int key = key_a + 8 * i;
+    if (key >= S) continue;
+    uint16_t* krow = dqkv + (tok0 + key) * ld + (H + kvh) * HD + d0;
+    uint16_t* vrow = dqkv + (tok0 + key) * ld + (H + KV + kvh) * HD + d0;
+#pragma unroll
+    for (int dt = 0; dt < NC; ++dt) {
+      *reinterpret_cast<uint32_t*>(krow + dt * 8 + c) = pack_bf16x2(dk[dt][2 * i] * inv, dk[dt][2 * i + 1] * inv);
+      *reinterpret_cast<uint32_t*>(vrow + dt * 8 + c) = pack_bf16x2(dv[dt][2 * i], dv[dt][2 * i + 1]);
+    }
+  }
+}
+
+// dQ for one query block of one head, output columns d0 .. d0 + DC.
+template <int HD, int DC>
+__global__ void __launch_bounds__(128, 1) dq_kernel(const uint16_t* __restrict__ qkv, int64_t ld,
+                                                    const uint16_t* __restrict__ dout, int64_t ldo,
+                                                    const float* __restrict__ lse, const float* __restrict__ dvec,
+                                                    int S, int H, int KV, uint16_t* __restrict__ dqkv) {
+  constexpr int LD = HD + 8, NC = DC / 8, NCH = HD / DC;
+  extern __shared__ __align__(16) uint16_t sm[];
+  uint16_t* qs = sm;
+  uint16_t* dos = qs + BQ * LD;
+  uint16_t* ks = dos + BQ * LD;
+  uint16_t* vs = ks + BKV * LD;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int qb = blockIdx.x, h = blockIdx.y;
+  const int b = blockIdx.z / NCH, d0 = (blockIdx.z % NCH) * DC;
+  const int kvh = h / (H / KV);
+  const int64_t tok0 = static_cast<int64_t>(b) * S;
+  const int q0 = qb * BQ;
+  const float sc = kLog2e * rsqrtf(static_cast<float>(HD));
+
+  load_tile<HD>(qs, qkv, ld, tok0, q0, S, h * HD, tid);
+  load_tile<HD>(dos, dout, ldo, tok0, q0, S, h * HD, tid);
+  cp_async_commit();
+  const int ra = q0 + warp * 16 + (lane >> 2);
+  float lse2[2], dvv[2];
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const int row = ra + 8 * i;
+    const int64_t li = (static_cast<int64_t>(b) * H + h) * S + row;
+    lse2[i] = row < S ? lse[li] * kLog2e : 0.0f;
+    dvv[i] = row < S ? dvec[li] : 0.0f;
+  }
+  float dq[NC][4];
+#pragma unroll
+  for (int i = 0; i < NC; ++i) dq[i][0] = dq[i][1] = dq[i][2] = dq[i][3] = 0.0f;
+
+  for (int kb = 0; kb <= qb; ++kb) {
+    const int k0 = kb * BKV;
+    load_tile<HD>(ks, qkv, ld, tok0, k0, S, (H + kvh) * HD, tid);
+    load_tile<HD>(vs, qkv, ld, tok0, k0, S, (H + KV + kvh) * HD, tid);
+    cp_async_commit();
+    cp_async_wait<0>();
+    __syncthreads();
+    float p[8][4];
+    qk_tile<HD>(p, smem_u32(qs), smem_u32(ks), warp, lane);
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int col = k0 + nt * 8 + 2 * (lane & 3) + (e & 1);
+        const int i = e >> 1;
+        const int row = ra + 8 * i;
+        p[nt][e] = (col <= row && col < S && row < S) ? exp2f(p[nt][e] * sc - lse2[i]) : 0.0f;
+      }
+    float dp[8][4];
+    qk_tile<HD>(dp, smem_u32(dos), smem_u32(vs), warp, lane);
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) dp[nt][e] = p[nt][e] * (dp[nt][e] - dvv[e >> 1]);
+    pv_tile<HD, NC>(dq, dp, smem_u32(ks), d0, lane);
+    __syncthreads();
+  }
+  const float inv = rsqrtf(static_cast<float>(HD));
+  const int c = 2 * (lane & 3);
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const int row = ra + 8 * i;
+    if (row >= S) continue;
+    uint16_t* qrow = dqkv + (tok0 + row) * ld + h * HD + d0;
+#pragma unroll
+    for (int dt = 0; dt < NC; ++dt)
+      *reinterpret_cast<uint32_t*>(qrow + dt * 8 + c) = pack_bf16x2(dq[dt][2 * i] * inv, dq[dt][2 * i + 1] * inv);
+  }
+}
+
+template <int HD>
+void fwd_launch(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uint16_t* o, int64_t ldo, float* lse,
+                cudaStream_t st) {
+  constexpr int smem = 3 * 64 * (HD + 8) * 2;
+  static bool init = false;
+  if (!init) {
+    cudaFuncSetAttribute(fwd_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    init = true;
+  }
+  dim3 grid((S + BQ - 1) / BQ, H, B);
+  count_launch();
+  fwd_kernel<HD><<<grid, 128, smem, st>>>(qkv, ld, S, H, KV, o, ldo, lse);
+}
+
+template <int HD, int DC>
+void bwd_launch(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t ldo, const float* lse,
+                const float* dvec, int B, int S, int H, int KV, uint16_t* dqkv, cudaStream_t st) {
+  constexpr int smem = 4 * 64 * (HD + 8) * 2 + 2 * 64 * 4;
+  static bool init = false;
+  if (!init) {
+    cudaFuncSetAttribute(dkdv_kernel<HD, DC>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(dq_kernel<HD, DC>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    init = true;
+  }
+  constexpr int NCH = HD / DC;
+  dim3 g1((S + BKV - 1) / BKV, KV, B * NCH);
+  count_launch();
+  dkdv_kernel<HD, DC><<<g1, 128, smem, st>>>(qkv, ld, dout, ldo, lse, dvec, S, H, KV, dqkv);
+  dim3 g2((S + BQ - 1) / BQ, H, B * NCH);
+  count_launch();
+  dq_kernel<HD, DC><<<g2, 128, smem, st>>>(qkv, ld, dout, ldo, lse, dvec, S, H, KV, dqkv);
+}
+
+}  // namespace attn
+
+void launch_attn_fwd(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, int hd, uint16_t* o, int64_t ldo,
+                     float* lse, cudaStream_t st) {
+  if (hd == 64) attn::fwd_launch<64>(qkv, ld, B, S, H, KV, o, ldo, lse, st);
+  else if (hd == 128) attn::fwd_launch<128>(qkv, ld, B, S, H, KV, o, ldo, lse, st);
+  else attn::fwd_launch<256>(qkv, ld, B, S, H, KV, o, ldo, lse, st);
+}
+
+void launch_attn_bwd(const uint16_t* qkv, int64_t ld, const uint16_t* o, const uint16_t* dout, int64_t ldo,
+                     const float* lse, int B, int S, int H, int KV, int hd, float* dvec, uint16_t* dqkv,
+                     cudaStream_t st) {
+  const int64_t nw = static_cast<int64_t>(B) * S * H;
+  count_launch();
+  attn::dvec_kernel<<<static_cast<unsigned>((nw * 32 + 255) / 256), 256, 0, st>>>(o, dout, ldo, B, S, H, hd, dvec);
+  if (hd == 64) attn::bwd_launch<64, 64>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, st);
+  else if (hd == 128) attn::bwd_launch<128, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, st);
+  else attn::bwd_launch<256, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, st);
+}
+
+}  // namespace mebp

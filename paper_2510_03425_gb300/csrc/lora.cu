@@ -1,0 +1,268 @@
+// LoRA kernels (Section 3: only LoRA weights are trainable; the compressed base is frozen).
+//
+//  * skinny_gemm:  U_s = s * X A^T  (and dU = s * dY B) — the rank-r down-projections whose
+//    bf16 result feeds the fused GEMM's extra K-block.  HBM-bound on X.
+//  * tall_reduce:  dB = dY^T U_s and dA = dU^T X — reductions over all T tokens, done as
+//    warp-level tensor-core tiles over a token split, then summed in a fixed order
+//    (deterministic; no floating-point atomics).
+//  * lora_shadow:  bf16 operand copies of the fp32 masters, with the targets of a fused
+//    linear (q|k|v or gate|up) laid side by side along the rank axis:
+//      A_cat [kx, K]  rows ro_t .. ro_t+r-1 = A_t
+//      B_cat [N, kx]  block-diagonal: rows of target t, columns ro_t .. ro_t+r-1 = B_t
+//      Bt_cat [kx, N] = B_cat^T
+#include "kernels.h"
+#include "mma.cuh"
+
+namespace mebp {
+
+// ------------------------------------------------------------------------------------ skinny
+template <int NT>
+__global__ void __launch_bounds__(128) skinny_gemm_kernel(const uint16_t* __restrict__ X, int64_t ldx, int64_t M,
+                                                          int64_t K, const uint16_t* __restrict__ W, int64_t ldw,
+                                                          float alpha, uint16_t* __restrict__ out, int64_t ldo) {
+  constexpr int BMs = 64, BKs = 64, LDS = BKs + 8, JR = NT * 8;
+  __shared__ __align__(16) uint16_t xs[2][BMs * LDS];
+  __shared__ __align__(16) uint16_t ws[2][JR * LDS];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int64_t m0 = static_cast<int64_t>(blockIdx.x) * BMs;
+  float acc[NT][4];
+#pragma unroll
+  for (int i = 0; i < NT; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.0f;
+
+  auto load = [&](int stage, int64_t k0) {
+    for (int c = tid; c < BMs * 8; c += 128) {
+      const int r = c >> 3, cc = c & 7;
+      const int64_t gm = m0 + r;
+      const bool v = gm < M;
+      cp_async16(smem_u32(&xs[stage][r * LDS + cc * 8]), X + (v ? gm : 0) * ldx + k0 + cc * 8, v);
+    }
+    for (int c = tid; c < JR * 8; c += 128) {
+      const int r = c >> 3, cc = c & 7;
+      cp_async16(smem_u32(&ws[stage][r * LDS + cc * 8]), W + r * ldw + k0 + cc * 8, true);
+    }
+    cp_async_commit();
+  };
+  const int nk = static_cast<int>(K / BKs);
+  load(0, 0);
+  for (int kt = 0; kt < nk; ++kt) {
+    if (kt + 1 < nk) {
+      load((kt + 1) & 1, static_cast<int64_t>(kt + 1) * BKs);
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
+    __syncthreads();
+    const int s = kt & 1;
+    const uint32_t xb = smem_u32(xs[s]), wb = smem_u32(ws[s]);
+#pragma unroll
+    for (int kk = 0; kk < BKs; kk += 16) {
+      uint32_t a[4];
+      ldsm_x4(a, frag_a_addr(xb, LDS, warp * 16, kk, lane));
+#pragma unroll
+      for (int nt = 0; nt < NT; nt += 2) {
+        uint32_t b[4];
+        ldsm_x4(b, frag_bn_addr(wb, LDS, nt * 8, kk, lane));
+        mma16816(acc[nt], a, b[0], b[1]);
+        mma16816(acc[nt + 1], a, b[2], b[3]);
+      }
+    }
+    __syncthreads();
+  }
+  const int r = lane >> 2, c = (lane & 3) * 2;
+  const int64_t row0 = m0 + warp * 16 + r;
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) {
+    const int col = nt * 8 + c;
+    if (row0 < M)
+      *reinterpret_cast<uint32_t*>(out + row0 * ldo + col) = pack_bf16x2(alpha * acc[nt][0], alpha * acc[nt][1]);
+    if (row0 + 8 < M)
+      *reinterpret_cast<uint32_t*>(out + (row0 + 8) * ldo + col) =
+          pack_bf16x2(alpha * acc[nt][2], alpha * acc[nt][3]);
+  }
+}
+
+void launch_skinny_gemm(const uint16_t* X, int64_t ldx, int64_t M, int64_t K, const uint16_t* W, int64_t ldw, int J,
+                        float alpha, uint16_t* out, int64_t ldo, cudaStream_t st) {
+  (void)J;  // W holds ldo rows (zero beyond the used ranks), so every output column is written
+  if (M <= 0) return;
+  const unsigned grid = static_cast<unsigned>((M + 63) / 64);
+  switch (ldo) {
+    case 16: count_launch(); skinny_gemm_kernel<2><<<grid, 128, 0, st>>>(X, ldx, M, K, W, ldw, alpha, out, ldo); break;
+    case 32: count_launch(); skinny_gemm_kernel<4><<<grid, 128, 0, st>>>(X, ldx, M, K, W, ldw, alpha, out, ldo); break;
+    case 48: count_launch(); skinny_gemm_kernel<6><<<grid, 128, 0, st>>>(X, ldx, M, K, W, ldw, alpha, out, ldo); break;
+    case 64: count_launch(); skinny_gemm_kernel<8><<<grid, 128, 0, st>>>(X, ldx, M, K, W, ldw, alpha, out, ldo); break;
+    default: count_launch(); skinny_gemm_kernel<12><<<grid, 128, 0, st>>>(X, ldx, M, K, W, ldw, alpha, out, ldo); break;
+  }
+}
+
+// ------------------------------------------------------------------------------------ tall reduce
+// part[z][p][q] = sum_{m in split z} P[m, p] Q[m, q]   (p < Pw, q < Qw)
+template <int NQ>
+__global__ void __launch_bounds__(128) tall_reduce_kernel(const uint16_t* __restrict__ P, int64_t ldp,
+                                                          const uint16_t* __restrict__ Q, int64_t ldq, int64_t M,
+                                                          int Pw, int Qw, int64_t m_per_split,
+                                                          float* __restrict__ part) {
+  constexpr int BP = 64, BMr = 64, QT = NQ * 8, LDP = BP + 8, LDQ = QT + 8;
+  __shared__ __align__(16) uint16_t ps[2][BMr * LDP];
+  __shared__ __align__(16) uint16_t qs[2][BMr * LDQ];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int p0 = blockIdx.x * BP, q0 = blockIdx.y * QT;
+  const int64_t mb = static_cast<int64_t>(blockIdx.z) * m_per_split;
+  const int64_t me = min(M, mb + m_per_split);
+  float acc[NQ][4];
+#pragma unroll
+  for (int i = 0; i < NQ; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.0f;
+
+  auto load = [&](int stage, int64_t m) {
+    for (int c = tid; c < BMr * 8; c += 128) {
+      const int r = c >> 3, cc = c & 7;
+      const bool v = (m + r < me) && (p0 + cc * 8 < Pw);
+      const uint16_t* src = v ? P + (m + r) * ldp + p0 + cc * 8 : P;
+      cp_async16(smem_u32(&ps[stage][r * LDP + cc * 8]), src, v);
+    }
+    for (int c = tid; c < BMr * NQ; c += 128) {
+      const int r = c / NQ, cc = c % NQ;
+      const bool v = (m + r < me) && (q0 + cc * 8 < Qw);
+      const uint16_t* src = v ? Q + (m + r) * ldq + q0 + cc * 8 : Q;
+      cp_async16(smem_u32(&qs[stage][r * LDQ + cc * 8]), src, v);
+    }
+    cp_async_commit();
+  };
+  const int64_t ntile = (me - mb + BMr - 1) / BMr;
+  if (ntile > 0) load(0, mb);
+  for (int64_t it = 0; it < ntile; ++it) {
+    if (it + 1 < ntile) {
+      load(static_cast<int>((it + 1) & 1), mb + (it + 1) * BMr);
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
+    __syncthreads();
+    const int s = static_cast<int>(it & 1);
+    const uint32_t pb = smem_u32(ps[s]), qb = smem_u32(qs[s]);
+#pragma unroll
+    for (int kk = 0; kk < BMr; kk += 16) {
+      uint32_t a[4];
+      ldsm_x4_t(a, frag_at_addr(pb, LDP, warp * 16, kk, lane));
+#pragma unroll
+      for (int nq = 0; nq < NQ; nq += 2) {
+        uint32_t b[4];
+        ldsm_x4_t(b, frag_bk_addr(qb, LDQ, nq * 8, kk, lane));
+        mma16816(acc[nq], a, b[0], b[1]);
+        mma16816(acc[nq + 1], a, b[2], b[3]);
+      }
+    }
+    __syncthreads();
+  }
+  const int r = lane >> 2, c = (lane & 3) * 2;
+  float* out = part + static_cast<int64_t>(blockIdx.z) * Pw * Qw;
+  const int pr = p0 + warp * 16 + r;
+#pragma unroll
+  for (int nq = 0; nq < NQ; ++nq) {
+    const int qc = q0 + nq * 8 + c;
+    if (qc >= Qw) continue;
+    if (pr < Pw) *reinterpret_cast<float2*>(out + static_cast<int64_t>(pr) * Qw + qc) = make_float2(acc[nq][0], acc[nq][1]);
+    if (pr + 8 < Pw)
+      *reinterpret_cast<float2*>(out + static_cast<int64_t>(pr + 8) * Qw + qc) = make_float2(acc[nq][2], acc[nq][3]);
+  }
+}
+
+// C[p * sp + q * sq] (+)= sum_z part[z][p][q]  in split order.
+__global__ void split_sum_kernel(const float* __restrict__ part, int splits, int Pw, int Qw, float* __restrict__ C,
+                                 int64_t sp, int64_t sq, int accumulate) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  const int64_t n = static_cast<int64_t>(Pw) * Qw;
+  if (i >= n) return;
+  float s = 0.0f;
+  for (int z = 0; z < splits; ++z) s += part[z * n + i];
+  const int64_t p = i / Qw, q = i % Qw;
+  float* dst = C + p * sp + q * sq;
+  *dst = accumulate ? *dst + s : s;
+}
+
+int64_t tall_reduce_scratch_floats(int64_t M, int Pw, int Qw) {
+  (void)M;
+  return static_cast<int64_t>(Pw) * Qw * 16;
+}
+
+// C is written with strides (sp, sq) = (ldc, 1) for ldc > 0, and (1, -ldc) for ldc < 0
+// (transposed output).
+int launch_tall_reduce(const uint16_t* P, int64_t ldp, const uint16_t* Q, int64_t ldq, int64_t M, int Pw, int Qw,
+                       float* C, int64_t ldc, bool accumulate, float* scratch, int64_t scratch_floats,
+                       cudaStream_t st) {
+  if (Pw <= 0 || Qw <= 0) return MEBP_OK;
+  if ((Pw % 8) || (Qw % 8) || Qw > 96) return MEBP_ERR_UNSUPPORTED;
+  const int nq = Qw <= 32 ? 4 : (Qw <= 64 ? 8 : 12);
+  const int gx = (Pw + 63) / 64, gy = (Qw + nq * 8 - 1) / (nq * 8);
+  int64_t splits = (4 * 152 + gx * gy - 1) / (gx * gy);
+  splits = std::min<int64_t>(splits, std::max<int64_t>(1, M / 256));
+  splits = std::min<int64_t>(splits, scratch_floats / (static_cast<int64_t>(Pw) * Qw));
+  if (splits < 1) return MEBP_ERR_INVALID_ARG;
+  int64_t mps = (M + splits - 1) / splits;
+  mps = (mps + 63) / 64 * 64;
+  splits = std::max<int64_t>(1, (M + mps - 1) / mps);
+  dim3 grid(gx, gy, static_cast<unsigned>(splits));
+  switch (nq) {
+    case 4: count_launch(); tall_reduce_kernel<4><<<grid, 128, 0, st>>>(P, ldp, Q, ldq, M, Pw, Qw, mps, scratch); break;
+    case 8: count_launch(); tall_reduce_kernel<8><<<grid, 128, 0, st>>>(P, ldp, Q, ldq, M, Pw, Qw, mps, scratch); break;
+    default: count_launch(); tall_reduce_kernel<12><<<grid, 128, 0, st>>>(P, ldp, Q, ldq, M, Pw, Qw, mps, scratch); break;
+  }
+  const int64_t n = static_cast<int64_t>(Pw) * Qw;
+  const int64_t sp = ldc > 0 ? ldc : 1, sq = ldc > 0 ? 1 : -ldc;
+  count_launch();
+  split_sum_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(scratch, static_cast<int>(splits), Pw, Qw,
+                                                                           C, sp, sq, accumulate ? 1 : 0);
+  return MEBP_OK;
+}
+
+// ------------------------------------------------------------------------------------ shadows
+struct ShadowArgs {
+  const float* A[3];
+  const float* B[3];
+  int ro[3];     // rank offset of target t in the concatenated rank axis
+  int no[3];     // first output row of target t
+  int nl[3];     // output rows of target t
+  int nt;
+};
+
+__global__ void lora_shadow_kernel(ShadowArgs a, int r, int K, int N, int kx, uint16_t* __restrict__ A_cat,
+                                   uint16_t* __restrict__ B_cat, uint16_t* __restrict__ Bt_cat) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  const int64_t na = static_cast<int64_t>(kx) * K, nb = static_cast<int64_t>(N) * kx;
+  if (i < na) {
+    const int j = static_cast<int>(i / K), k = static_cast<int>(i % K);
+    float v = 0.0f;
+    for (int t = 0; t < a.nt; ++t)
+      if (j >= a.ro[t] && j < a.ro[t] + r) v = a.A[t][static_cast<int64_t>(j - a.ro[t]) * K + k];
+    A_cat[i] = f_to_bf16(v);
+  }
+  if (i < nb) {
+    const int n = static_cast<int>(i / kx), j = static_cast<int>(i % kx);
+    float v = 0.0f;
+    for (int t = 0; t < a.nt; ++t)
+      if (j >= a.ro[t] && j < a.ro[t] + r && n >= a.no[t] && n < a.no[t] + a.nl[t])
+        v = a.B[t][static_cast<int64_t>(n - a.no[t]) * r + (j - a.ro[t])];
+    const uint16_t b = f_to_bf16(v);
+    B_cat[i] = b;
+    Bt_cat[static_cast<int64_t>(j) * N + n] = b;
+  }
+}
+
+void launch_lora_shadow(const float* const* A, const float* const* B, int nt, const int* ranks_off, const int* n_off,
+                        const int* n_len, int r, int K, int N, int kx, uint16_t* A_cat, uint16_t* B_cat,
+                        uint16_t* Bt_cat, cudaStream_t st) {
+  ShadowArgs a{};
+  a.nt = nt;
+  for (int t = 0; t < nt && t < 3; ++t) {
+    a.A[t] = A[t];
+    a.B[t] = B[t];
+    a.ro[t] = ranks_off[t];
+    a.no[t] = n_off[t];
+    a.nl[t] = n_len[t];
+  }
+  const int64_t n = std::max(static_cast<int64_t>(kx) * K, static_cast<int64_t>(N) * kx);
+  count_launch();
+  lora_shadow_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(a, r, K, N, kx, A_cat, B_cat, Bt_cat);
+}
+
+}  // namespace mebp

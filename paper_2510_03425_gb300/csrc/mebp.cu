@@ -1,0 +1,880 @@
+// C ABI of the MeBP training step (include/mebp.h): context and workspace, the decoder block's
+// recompute-forward and backward, the LM-head cross-entropy and Algorithm 1.
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "common.cuh"
+#include "kernels.h"
+
+using namespace mebp;
+
+namespace {
+
+enum { LIN_QKV = 0, LIN_O = 1, LIN_GU = 2, LIN_DOWN = 3 };
+
+struct Lin {
+  int N = 0, K = 0;
+  int nt = 0;        // number of LoRA targets carried by this fused linear
+  int tgt[3] = {0, 0, 0};
+  int ro[3] = {0, 0, 0};  // rank offset in the concatenated rank axis
+  int no[3] = {0, 0, 0};  // first output row of the target
+  int nl[3] = {0, 0, 0};  // output rows of the target
+  int kx = 0, kxp = 0;    // used / padded width of the rank axis
+};
+
+constexpr int kCkptSlots = 3;
+
+struct ProfRec {
+  cudaEvent_t a, b;
+  double flops;
+  bool trans;
+};
+
+}  // namespace
+
+std::atomic<long long> mebp::g_launches{0};
+
+struct mebp_ctx {
+  mebp_model_cfg cfg{};
+  int device = 0;
+  std::string err_msg = "ok";
+  int* d_err = nullptr;
+  int D = 0, H = 0, KV = 0, hd = 0, I = 0, V = 0, L = 0, Nqkv = 0, Na = 0, r = 0;
+  float s = 1.0f;
+  int64_t Tmax = 0;
+  Lin lin[4];
+  std::vector<void*> dev_allocs;
+  int64_t ws_bytes = 0;
+
+  float2* rope_cs = nullptr;
+  // one block's intermediates
+  uint16_t *a = nullptr, *qkv = nullptr, *o = nullptr, *b = nullptr, *gu = nullptr, *m = nullptr;
+  float *r1 = nullptr, *r2 = nullptr, *lse_attn = nullptr, *h1 = nullptr;
+  uint16_t* us[4] = {nullptr, nullptr, nullptr, nullptr};
+  uint16_t* du[4] = {nullptr, nullptr, nullptr, nullptr};
+  uint16_t *A_cat[4] = {}, *B_cat[4] = {}, *Bt_cat[4] = {};
+  // backward
+  uint16_t *dqkv = nullptr, *dout = nullptr, *dgu = nullptr, *dh1_bf = nullptr, *dy_bf[2] = {nullptr, nullptr};
+  float *dm = nullptr, *dtmp = nullptr, *dh1 = nullptr, *dvec = nullptr, *gbuf[2] = {nullptr, nullptr};
+  float* red = nullptr;
+  int64_t red_floats = 0;
+  // LM head
+  uint16_t *hf = nullptr, *dz = nullptr;
+  float *rf = nullptr, *part = nullptr, *zt = nullptr, *lse_tok = nullptr, *tok_loss = nullptr, *inv_n = nullptr,
+        *dhf = nullptr;
+  int32_t* targets = nullptr;
+  int nparts = 0, vchunk = 0;
+  // checkpoints
+  float* ckpt = nullptr;       // device: (L+1) x Tmax x D, or kCkptSlots slots when spilling
+  float* h_ckpt = nullptr;     // pinned host (spill)
+  cudaStream_t copy_stream = nullptr;
+  cudaEvent_t slot_free[kCkptSlots] = {};
+  cudaEvent_t slot_ready[kCkptSlots] = {};
+  // GEMM event profiling
+  bool prof = false;
+  std::vector<ProfRec> recs;
+  std::vector<cudaEvent_t> evpool;
+  size_t evnext = 0;
+  // intermediates tag
+  int saved_layer = -1;
+  const float* saved_x = nullptr;
+  int64_t saved_T = -1;
+};
+
+namespace {
+
+int fail(mebp_ctx* c, int code, const std::string& msg) {
+  if (c) c->err_msg = msg;
+  return code;
+}
+
+int cuda_check(mebp_ctx* c, const char* where) {
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return fail(c, MEBP_ERR_CUDA, std::string(where) + ": " + cudaGetErrorString(e));
+  return MEBP_OK;
+}
+
+template <typename T>
+int dalloc(mebp_ctx* c, T** p, int64_t count) {
+  *p = nullptr;
+  if (count <= 0) return MEBP_OK;
+  const size_t bytes = static_cast<size_t>(count) * sizeof(T);
+  void* q = nullptr;
+  if (cudaMalloc(&q, bytes) != cudaSuccess) {
+    cudaGetLastError();
+    return fail(c, MEBP_ERR_OOM, "device allocation of " + std::to_string(bytes) + " bytes failed");
+  }
+  c->dev_allocs.push_back(q);
+  c->ws_bytes += static_cast<int64_t>(bytes);
+  *p = static_cast<T*>(q);
+  return MEBP_OK;
+}
+
+cudaStream_t S(void* st) { return static_cast<cudaStream_t>(st); }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+int check_packed(mebp_ctx* c, const mebp_packed* w, int64_t rows, int64_t cols, const char* what) {
+  if (!w || !w->qpack || !w->scales) return fail(c, MEBP_ERR_INVALID_ARG, std::string(what) + ": NULL weight");
+  if (w->rows != rows || w->cols != cols)
+    return fail(c, MEBP_ERR_INVALID_ARG,
+                std::string(what) + ": expected [" + std::to_string(rows) + ", " + std::to_string(cols) + "]");
+  if (!aligned16(w->qpack) || !aligned16(w->scales))
+    return fail(c, MEBP_ERR_INVALID_ARG, std::string(what) + ": weight pointers must be 16-byte aligned");
+  return MEBP_OK;
+}
+
+void setup_lin(mebp_ctx* c) {
+  const int H = c->H, KV = c->KV, hd = c->hd, D = c->D, I = c->I, r = c->r;
+  const uint32_t m = c->cfg.lora_targets;
+  Lin* L = c->lin;
+  L[LIN_QKV].N = (H + 2 * KV) * hd;
+  L[LIN_QKV].K = D;
+  L[LIN_O].N = D;
+  L[LIN_O].K = H * hd;
+  L[LIN_GU].N = 2 * I;
+  L[LIN_GU].K = D;
+  L[LIN_DOWN].N = D;
+  L[LIN_DOWN].K = I;
+  struct Part { int lin, tgt, no, nl; };
+  const Part parts[7] = {{LIN_QKV, MEBP_T_Q, 0, H * hd},           {LIN_QKV, MEBP_T_K, H * hd, KV * hd},
+                         {LIN_QKV, MEBP_T_V, (H + KV) * hd, KV * hd}, {LIN_O, MEBP_T_O, 0, D},
+                         {LIN_GU, MEBP_T_GATE, 0, I},               {LIN_GU, MEBP_T_UP, I, I},
+                         {LIN_DOWN, MEBP_T_DOWN, 0, D}};
+  for (const Part& p : parts) {
+    if (!(m & (1u << p.tgt)) || r <= 0) continue;
+    Lin& l = L[p.lin];
+    l.tgt[l.nt] = p.tgt;
+    l.ro[l.nt] = l.kx;
+    l.no[l.nt] = p.no;
+    l.nl[l.nt] = p.nl;
+    l.kx += r;
+    l.nt++;
+  }
+  for (int i = 0; i < 4; ++i) L[i].kxp = L[i].kx ? (L[i].kx + 15) / 16 * 16 : 0;
+}
+
+// ------------------------------------------------------------------------------------ GEMM glue
+GemmArgs gemm_fwd(const uint16_t* X, int64_t ldx, int64_t M, const mebp_packed& W, int N, int K) {
+  GemmArgs g;
+  g.trans = false;
+  g.A = X;
+  g.lda = ldx;
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  g.qpack = W.qpack;
+  g.scales = W.scales;
+  g.scale_pitch = W.rows;
+  return g;
+}
+// dX = dY deq(W) for W [N_w, K_w] stored packed: GEMM K = N_w (reduction), N = K_w (output).
+GemmArgs gemm_dx(const uint16_t* dY, int64_t ldy, int64_t M, const mebp_packed& W) {
+  GemmArgs g;
+  g.trans = true;
+  g.A = dY;
+  g.lda = ldy;
+  g.M = M;
+  g.N = W.cols;
+  g.K = W.rows;
+  g.qpack = W.qpack;
+  g.scales = W.scales;
+  g.scale_pitch = W.rows;
+  return g;
+}
+
+cudaEvent_t pool_event(mebp_ctx* c) {
+  if (c->evnext == c->evpool.size()) {
+    cudaEvent_t e;
+    cudaEventCreate(&e);
+    c->evpool.push_back(e);
+  }
+  return c->evpool[c->evnext++];
+}
+
+int run_gemm(mebp_ctx* c, GemmArgs& g, cudaStream_t st, const char* what) {
+  g.err = c->d_err;
+  ProfRec pr{};
+  if (c->prof) {
+    pr.a = pool_event(c);
+    pr.b = pool_event(c);
+    pr.trans = g.trans;
+    pr.flops = 2.0 * g.M * g.N * g.K + (g.Ax ? 2.0 * g.M * g.N * g.kx : 0.0);
+    cudaEventRecord(pr.a, st);
+  }
+  const int rc = launch_dequant_gemm(g, st);
+  if (c->prof) {
+    cudaEventRecord(pr.b, st);
+    c->recs.push_back(pr);
+  }
+  if (rc) return fail(c, rc, std::string(what) + ": fused GEMM launch failed (" + std::to_string(rc) + ")");
+  return MEBP_OK;
+}
+
+// bf16 shadows of one fused linear's LoRA masters.
+void build_shadow(mebp_ctx* c, int li, const mebp_lora* lora, cudaStream_t st) {
+  const Lin& l = c->lin[li];
+  if (!l.kx) return;
+  const float* A[3];
+  const float* B[3];
+  for (int t = 0; t < l.nt; ++t) {
+    A[t] = lora->A[l.tgt[t]];
+    B[t] = lora->B[l.tgt[t]];
+  }
+  launch_lora_shadow(A, B, l.nt, l.ro, l.no, l.nl, c->r, l.K, l.N, l.kxp, c->A_cat[li], c->B_cat[li], c->Bt_cat[li],
+                     st);
+}
+
+int check_lora(mebp_ctx* c, const mebp_lora* lora) {
+  for (int li = 0; li < 4; ++li)
+    for (int t = 0; t < c->lin[li].nt; ++t) {
+      const int tg = c->lin[li].tgt[t];
+      if (!lora || !lora->A[tg] || !lora->B[tg])
+        return fail(c, MEBP_ERR_INVALID_ARG, "LoRA weights missing for target " + std::to_string(tg));
+    }
+  return MEBP_OK;
+}
+
+// y = F(x) for one block.  with_down == false stops after the MLP activation (what the
+// backward consumes), so y is not produced.
+int block_forward(mebp_ctx* c, int layer, const mebp_block_weights* w, const mebp_lora* lora, const float* x, float* y,
+                  int B, int Sq, bool with_down, cudaStream_t st) {
+  const int64_t T = static_cast<int64_t>(B) * Sq;
+  const int D = c->D, I = c->I;
+  int rc;
+  for (int li = 0; li < 4; ++li) build_shadow(c, li, lora, st);
+  // attention sub-block
+  launch_rmsnorm_fwd(x, w->norm1, T, D, c->cfg.rms_eps, c->a, c->r1, st);
+  const Lin& lq = c->lin[LIN_QKV];
+  GemmArgs g = gemm_fwd(c->a, D, T, w->qkv, lq.N, lq.K);
+  if (lq.kx) {
+    launch_skinny_gemm(c->a, D, T, D, c->A_cat[LIN_QKV], D, lq.kx, c->s, c->us[LIN_QKV], lq.kxp, st);
+    g.Ax = c->us[LIN_QKV]; g.ldax = lq.kxp; g.kx = lq.kxp; g.Bx = c->B_cat[LIN_QKV]; g.ldbx = lq.kxp;
+  }
+  g.epi = EPI_BF16; g.C = c->qkv; g.ldc = lq.N;
+  if ((rc = run_gemm(c, g, st, "qkv"))) return rc;
+  launch_rope(c->qkv, T, Sq, c->H, c->KV, c->hd, c->rope_cs, false, st);
+  launch_attn_fwd(c->qkv, lq.N, B, Sq, c->H, c->KV, c->hd, c->o, c->Na, c->lse_attn, st);
+  const Lin& lo = c->lin[LIN_O];
+  g = gemm_fwd(c->o, c->Na, T, w->o, lo.N, lo.K);
+  if (lo.kx) {
+    launch_skinny_gemm(c->o, c->Na, T, c->Na, c->A_cat[LIN_O], c->Na, lo.kx, c->s, c->us[LIN_O], lo.kxp, st);
+    g.Ax = c->us[LIN_O]; g.ldax = lo.kxp; g.kx = lo.kxp; g.Bx = c->B_cat[LIN_O]; g.ldbx = lo.kxp;
+  }
+  g.epi = EPI_F32; g.C = c->h1; g.ldc = D; g.R = x; g.ldr = D;
+  if ((rc = run_gemm(c, g, st, "o_proj"))) return rc;
+  // MLP sub-block
+  launch_rmsnorm_fwd(c->h1, w->norm2, T, D, c->cfg.rms_eps, c->b, c->r2, st);
+  const Lin& lg = c->lin[LIN_GU];
+  g = gemm_fwd(c->b, D, T, w->gate_up, lg.N, lg.K);
+  if (lg.kx) {
+    launch_skinny_gemm(c->b, D, T, D, c->A_cat[LIN_GU], D, lg.kx, c->s, c->us[LIN_GU], lg.kxp, st);
+    g.Ax = c->us[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = c->B_cat[LIN_GU]; g.ldbx = lg.kxp;
+  }
+  g.epi = EPI_BF16; g.C = c->gu; g.ldc = lg.N;
+  if ((rc = run_gemm(c, g, st, "gate_up"))) return rc;
+  launch_glu_fwd(c->gu, T, I, c->cfg.act, c->m, st);
+  const Lin& ld = c->lin[LIN_DOWN];
+  if (ld.kx) launch_skinny_gemm(c->m, I, T, I, c->A_cat[LIN_DOWN], I, ld.kx, c->s, c->us[LIN_DOWN], ld.kxp, st);
+  if (with_down) {
+    g = gemm_fwd(c->m, I, T, w->down, ld.N, ld.K);
+    if (ld.kx) {
+      g.Ax = c->us[LIN_DOWN]; g.ldax = ld.kxp; g.kx = ld.kxp; g.Bx = c->B_cat[LIN_DOWN]; g.ldbx = ld.kxp;
+    }
+    g.epi = EPI_F32; g.C = y; g.ldc = D; g.R = c->h1; g.ldr = D;
+    if ((rc = run_gemm(c, g, st, "down"))) return rc;
+  }
+  c->saved_layer = layer;
+  c->saved_x = x;
+  c->saved_T = T;
+  return cuda_check(c, "block forward");
+}
+
+// LoRA gradients of one fused linear: dB_t = dY[:, rows_t]^T U_s[:, ranks_t], dA_t = dU[:, ranks_t]^T X.
+int lin_grads(mebp_ctx* c, int li, const uint16_t* dY, int64_t ldy, const uint16_t* X, int64_t ldx, int64_t T,
+              const mebp_lora_grads* grads, bool acc, cudaStream_t st) {
+  const Lin& l = c->lin[li];
+  for (int t = 0; t < l.nt; ++t) {
+    const int tg = l.tgt[t];
+    if (!grads) break;
+    if (grads->dB[tg]) {
+      const int rc = launch_tall_reduce(dY + l.no[t], ldy, c->us[li] + l.ro[t], l.kxp, T, l.nl[t], c->r, grads->dB[tg],
+                                        c->r, acc, c->red, c->red_floats, st);
+      if (rc) return fail(c, rc, "LoRA dB reduction");
+    }
+    if (grads->dA[tg]) {
+      const int rc = launch_tall_reduce(X, ldx, c->du[li] + l.ro[t], l.kxp, T, l.K, c->r, grads->dA[tg], -l.K, acc,
+                                        c->red, c->red_floats, st);
+      if (rc) return fail(c, rc, "LoRA dA reduction");
+    }
+  }
+  return MEBP_OK;
+}
+
+// dE/dx and LoRA grads of one block from its input checkpoint x and dE/dy.
+// dy_bf: bf16 copy of dy (or null -> made here).  dx / dx_bf may be null.
+int block_backward(mebp_ctx* c, int layer, const mebp_block_weights* w, const mebp_lora* lora, const float* x,
+                   const float* dy, const uint16_t* dy_bf, float* dx, uint16_t* dx_bf, const mebp_lora_grads* grads,
+                   int B, int Sq, bool acc, cudaStream_t st) {
+  const int64_t T = static_cast<int64_t>(B) * Sq;
+  const int D = c->D, I = c->I;
+  int rc;
+  if (!(c->saved_layer == layer && c->saved_x == x && c->saved_T == T)) {
+    if ((rc = block_forward(c, layer, w, lora, x, nullptr, B, Sq, false, st))) return rc;
+  }
+  c->saved_layer = -1;  // the workspace is reused below
+  if (!dy_bf) {
+    launch_cast_bf16(dy, T * D, c->dy_bf[1], st);
+    dy_bf = c->dy_bf[1];
+  }
+  // ---- down projection: y = h1 + m Wd^T (+ s (m Ad^T) Bd^T)
+  const Lin& ld = c->lin[LIN_DOWN];
+  GemmArgs g = gemm_dx(dy_bf, D, T, w->down);
+  if (ld.kx) {
+    launch_skinny_gemm(dy_bf, D, T, D, c->Bt_cat[LIN_DOWN], D, ld.kx, c->s, c->du[LIN_DOWN], ld.kxp, st);
+    g.Ax = c->du[LIN_DOWN]; g.ldax = ld.kxp; g.kx = ld.kxp; g.Bx = c->A_cat[LIN_DOWN]; g.ldbx = I;
+  }
+  g.epi = EPI_F32; g.C = c->dm; g.ldc = I;
+  if ((rc = run_gemm(c, g, st, "down dX"))) return rc;
+  if ((rc = lin_grads(c, LIN_DOWN, dy_bf, D, c->m, I, T, grads, acc, st))) return rc;
+  // ---- gated MLP
+  launch_glu_bwd(c->dm, c->gu, T, I, c->cfg.act, c->dgu, st);
+  const Lin& lg = c->lin[LIN_GU];
+  g = gemm_dx(c->dgu, 2 * I, T, w->gate_up);
+  if (lg.kx) {
+    launch_skinny_gemm(c->dgu, 2 * I, T, 2 * I, c->Bt_cat[LIN_GU], 2 * I, lg.kx, c->s, c->du[LIN_GU], lg.kxp, st);
+    g.Ax = c->du[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = c->A_cat[LIN_GU]; g.ldbx = D;
+  }
+  g.epi = EPI_F32; g.C = c->dtmp; g.ldc = D;
+  if ((rc = run_gemm(c, g, st, "gate_up dX"))) return rc;
+  if ((rc = lin_grads(c, LIN_GU, c->dgu, 2 * I, c->b, D, T, grads, acc, st))) return rc;
+  // dh1 = dy + RMSNorm2^T(db)
+  launch_rmsnorm_bwd(c->dtmp, c->h1, w->norm2, c->r2, dy, T, D, c->dh1, c->dh1_bf, st);
+  // ---- o projection
+  const Lin& lo = c->lin[LIN_O];
+  g = gemm_dx(c->dh1_bf, D, T, w->o);
+  if (lo.kx) {
+    launch_skinny_gemm(c->dh1_bf, D, T, D, c->Bt_cat[LIN_O], D, lo.kx, c->s, c->du[LIN_O], lo.kxp, st);
+    g.Ax = c->du[LIN_O]; g.ldax = lo.kxp; g.kx = lo.kxp; g.Bx = c->A_cat[LIN_O]; g.ldbx = c->Na;
+  }
+  g.epi = EPI_BF16; g.C = c->dout; g.ldc = c->Na;
+  if ((rc = run_gemm(c, g, st, "o dX"))) return rc;
+  if ((rc = lin_grads(c, LIN_O, c->dh1_bf, D, c->o, c->Na, T, grads, acc, st))) return rc;
+  // ---- attention, RoPE
+  const Lin& lq = c->lin[LIN_QKV];
+  launch_attn_bwd(c->qkv, lq.N, c->o, c->dout, c->Na, c->lse_attn, B, Sq, c->H, c->KV, c->hd, c->dvec, c->dqkv, st);
+  launch_rope(c->dqkv, T, Sq, c->H, c->KV, c->hd, c->rope_cs, true, st);
+  // ---- q, k, v projections
+  if (lq.kx)
+    launch_skinny_gemm(c->dqkv, lq.N, T, lq.N, c->Bt_cat[LIN_QKV], lq.N, lq.kx, c->s, c->du[LIN_QKV], lq.kxp, st);
+  if ((rc = lin_grads(c, LIN_QKV, c->dqkv, lq.N, c->a, D, T, grads, acc, st))) return rc;
+  if (dx) {
+    g = gemm_dx(c->dqkv, lq.N, T, w->qkv);
+    if (lq.kx) {
+      g.Ax = c->du[LIN_QKV]; g.ldax = lq.kxp; g.kx = lq.kxp; g.Bx = c->A_cat[LIN_QKV]; g.ldbx = D;
+    }
+    g.epi = EPI_F32; g.C = c->dtmp; g.ldc = D;
+    if ((rc = run_gemm(c, g, st, "qkv dX"))) return rc;
+    launch_rmsnorm_bwd(c->dtmp, x, w->norm1, c->r1, c->dh1, T, D, dx, dx_bf, st);
+  }
+  return cuda_check(c, "block backward");
+}
+
+int lmhead(mebp_ctx* c, const mebp_packed* E, const float* gf, const float* h, const int32_t* targets, int64_t T,
+           float* loss, float* dh, uint16_t* dh_bf, float* tok_loss, cudaStream_t st) {
+  const int D = c->D, V = c->V;
+  int rc;
+  launch_rmsnorm_fwd(h, gf, T, D, c->cfg.rms_eps, c->hf, c->rf, st);
+  GemmArgs g = gemm_fwd(c->hf, D, T, *E, V, D);
+  g.epi = EPI_LSE; g.targets = targets; g.col_offset = 0; g.n_valid = V; g.part = c->part; g.nparts = c->nparts;
+  g.zt = c->zt;
+  if ((rc = run_gemm(c, g, st, "LM head (log-sum-exp pass)"))) return rc;
+  float* tl = tok_loss ? tok_loss : c->tok_loss;
+  launch_lse_combine(c->part, c->nparts, c->zt, targets, T, c->lse_tok, tl, st);
+  launch_loss_reduce(tl, targets, T, loss, c->inv_n, st);
+  for (int c0 = 0; c0 < V; c0 += c->vchunk) {
+    const int n = std::min(c->vchunk, V - c0);
+    mebp_packed Ec = *E;
+    Ec.qpack = E->qpack + static_cast<int64_t>(c0) * (D / 2);
+    Ec.scales = E->scales + c0;
+    Ec.rows = n;
+    g = gemm_fwd(c->hf, D, T, Ec, n, D);
+    g.scale_pitch = V;
+    g.epi = EPI_CEGRAD; g.C = c->dz; g.ldc = c->vchunk; g.targets = targets; g.col_offset = c0; g.n_valid = n;
+    g.lse = c->lse_tok; g.inv_n = c->inv_n;
+    if ((rc = run_gemm(c, g, st, "LM head (gradient pass)"))) return rc;
+    GemmArgs t;
+    t.trans = true;
+    t.A = c->dz; t.lda = c->vchunk; t.M = T; t.N = D; t.K = n;
+    t.qpack = Ec.qpack; t.scales = Ec.scales; t.scale_pitch = V;
+    t.epi = EPI_F32; t.C = c->dhf; t.ldc = D; t.R = c0 ? c->dhf : nullptr; t.ldr = D;
+    if ((rc = run_gemm(c, t, st, "LM head (dH pass)"))) return rc;
+  }
+  launch_rmsnorm_bwd(c->dhf, h, gf, c->rf, nullptr, T, D, dh, dh_bf, st);
+  return cuda_check(c, "LM head");
+}
+
+__global__ void targets_kernel(const int32_t* ids, int B, int Sq, int32_t* tg) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= static_cast<int64_t>(B) * Sq) return;
+  const int s = static_cast<int>(i % Sq);
+  tg[i] = (s < Sq - 1) ? ids[i + 1] : -1;
+}
+
+int check_block_ptrs(mebp_ctx* c, const mebp_block_weights* w) {
+  int rc;
+  if (!w) return fail(c, MEBP_ERR_INVALID_ARG, "NULL block weights");
+  if ((rc = check_packed(c, &w->qkv, c->lin[LIN_QKV].N, c->D, "qkv"))) return rc;
+  if ((rc = check_packed(c, &w->o, c->D, c->Na, "o"))) return rc;
+  if ((rc = check_packed(c, &w->gate_up, 2 * c->I, c->D, "gate_up"))) return rc;
+  if ((rc = check_packed(c, &w->down, c->D, c->I, "down"))) return rc;
+  if (!w->norm1 || !w->norm2) return fail(c, MEBP_ERR_INVALID_ARG, "NULL norm gain");
+  return MEBP_OK;
+}
+
+int check_tokens(mebp_ctx* c, int B, int Sq) {
+  if (B <= 0 || Sq <= 0) return fail(c, MEBP_ERR_INVALID_ARG, "batch and seq must be positive");
+  if (static_cast<int64_t>(B) * Sq > c->Tmax) return fail(c, MEBP_ERR_INVALID_ARG, "batch*seq exceeds max_tokens");
+  if (Sq > c->cfg.max_seq) return fail(c, MEBP_ERR_INVALID_ARG, "seq exceeds max_seq");
+  return MEBP_OK;
+}
+
+}  // namespace
+
+// ===================================================================================== C ABI
+extern "C" {
+
+int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
+  if (!cfg || !out) return MEBP_ERR_INVALID_ARG;
+  *out = nullptr;
+  const mebp_model_cfg& f = *cfg;
+  if (f.hidden <= 0 || f.hidden % 64 || f.n_heads <= 0 || f.n_kv_heads <= 0 || f.n_heads % f.n_kv_heads ||
+      f.intermediate <= 0 || f.intermediate % 64 || f.n_layers <= 0 || f.max_tokens <= 0 || f.max_seq <= 0 ||
+      f.vocab < 0 || f.vocab % 64 || f.lora_rank < 0 || f.lora_rank > 32)
+    return MEBP_ERR_INVALID_ARG;
+  if (!(f.head_dim == 64 || f.head_dim == 128 || f.head_dim == 256)) return MEBP_ERR_UNSUPPORTED;
+  if (f.lora_targets && (f.lora_rank % 8)) return MEBP_ERR_UNSUPPORTED;
+  if (f.act != MEBP_ACT_SILU && f.act != MEBP_ACT_GELU_TANH) return MEBP_ERR_INVALID_ARG;
+  if (f.vocab_chunk < 0 || f.vocab_chunk % 256) return MEBP_ERR_INVALID_ARG;
+  if (cudaSetDevice(device) != cudaSuccess) {
+    cudaGetLastError();
+    return MEBP_ERR_CUDA;
+  }
+  mebp_ctx* c = new mebp_ctx();
+  c->cfg = f;
+  c->device = device;
+  c->D = f.hidden; c->H = f.n_heads; c->KV = f.n_kv_heads; c->hd = f.head_dim; c->I = f.intermediate;
+  c->V = f.vocab; c->L = f.n_layers; c->r = f.lora_targets ? f.lora_rank : 0; c->s = f.lora_scale;
+  c->Tmax = f.max_tokens;
+  c->Na = c->H * c->hd;
+  setup_lin(c);
+  c->Nqkv = c->lin[LIN_QKV].N;
+  if (c->Na % 64) {
+    delete c;
+    return MEBP_ERR_UNSUPPORTED;
+  }
+  const int64_t T = c->Tmax, D = c->D, I = c->I;
+  int rc = MEBP_OK;
+  auto A = [&](auto** p, int64_t n) {
+    if (rc == MEBP_OK) rc = dalloc(c, p, n);
+  };
+  A(&c->d_err, 4);
+  A(&c->rope_cs, static_cast<int64_t>(f.max_seq) * (c->hd / 2));
+  A(&c->a, T * D); A(&c->b, T * D); A(&c->qkv, T * c->Nqkv); A(&c->o, T * c->Na); A(&c->gu, T * 2 * I);
+  A(&c->m, T * I); A(&c->r1, T); A(&c->r2, T); A(&c->lse_attn, T * c->H); A(&c->h1, T * D);
+  for (int li = 0; li < 4; ++li) {
+    const Lin& l = c->lin[li];
+    if (!l.kx) continue;
+    A(&c->us[li], T * l.kxp); A(&c->du[li], T * l.kxp);
+    A(&c->A_cat[li], static_cast<int64_t>(l.kxp) * l.K);
+    A(&c->B_cat[li], static_cast<int64_t>(l.N) * l.kxp);
+    A(&c->Bt_cat[li], static_cast<int64_t>(l.N) * l.kxp);
+  }
+  A(&c->dqkv, T * c->Nqkv); A(&c->dout, T * c->Na); A(&c->dgu, T * 2 * I); A(&c->dh1_bf, T * D);
+  A(&c->dy_bf[0], T * D); A(&c->dy_bf[1], T * D);
+  A(&c->dm, T * I); A(&c->dtmp, T * D); A(&c->dh1, T * D); A(&c->dvec, T * c->H);
+  A(&c->gbuf[0], T * D); A(&c->gbuf[1], T * D);
+  c->red_floats = std::max<int64_t>(tall_reduce_scratch_floats(T, std::max<int64_t>(2 * I, c->Nqkv), 32),
+                                    tall_reduce_scratch_floats(T, std::max<int64_t>(I, D), 32));
+  A(&c->red, c->red_floats);
+  if (c->V > 0) {
+    c->nparts = 2 * ((c->V + 255) / 256);
+    int64_t vc = f.vocab_chunk;
+    if (vc == 0) {
+      vc = (int64_t(1) << 30) / (2 * T);
+      vc = std::max<int64_t>(4096, vc / 256 * 256);
+    }
+    c->vchunk = static_cast<int>(std::min<int64_t>(vc, (c->V + 255) / 256 * 256));
+    A(&c->hf, T * D); A(&c->rf, T); A(&c->part, T * c->nparts * 2); A(&c->zt, T); A(&c->lse_tok, T);
+    A(&c->tok_loss, T); A(&c->inv_n, 4); A(&c->dz, T * c->vchunk); A(&c->dhf, T * D); A(&c->targets, T);
+  }
+  const int64_t nslots = f.spill_ckpts ? kCkptSlots : (c->L + 1);
+  A(&c->ckpt, nslots * T * D);
+  if (rc == MEBP_OK && f.spill_ckpts) {
+    const size_t hb = static_cast<size_t>(c->L + 1) * T * D * sizeof(float);
+    if (cudaHostAlloc(reinterpret_cast<void**>(&c->h_ckpt), hb, cudaHostAllocDefault) != cudaSuccess) {
+      cudaGetLastError();
+      c->h_ckpt = nullptr;
+      rc = MEBP_ERR_OOM;
+    }
+    if (rc == MEBP_OK && cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking) != cudaSuccess) rc = MEBP_ERR_CUDA;
+    for (int i = 0; rc == MEBP_OK && i < kCkptSlots; ++i)
+      if (cudaEventCreateWithFlags(&c->slot_free[i], cudaEventDisableTiming) != cudaSuccess ||
+          cudaEventCreateWithFlags(&c->slot_ready[i], cudaEventDisableTiming) != cudaSuccess)
+        rc = MEBP_ERR_CUDA;
+  }
+  if (rc != MEBP_OK) {
+    mebp_ctx_destroy(c);
+    return rc;
+  }
+  // RoPE table: angle(p, j) = p * theta^(-2j/hd), evaluated in double precision on the host.
+  {
+    const int half = c->hd / 2;
+    std::vector<float2> cs(static_cast<size_t>(f.max_seq) * half);
+    for (int p = 0; p < f.max_seq; ++p)
+      for (int j = 0; j < half; ++j) {
+        const double ang = p * std::pow(static_cast<double>(f.rope_theta), -2.0 * j / c->hd);
+        cs[static_cast<size_t>(p) * half + j] = make_float2(static_cast<float>(std::cos(ang)),
+                                                            static_cast<float>(std::sin(ang)));
+      }
+    cudaMemcpy(c->rope_cs, cs.data(), cs.size() * sizeof(float2), cudaMemcpyHostToDevice);
+  }
+  cudaMemset(c->d_err, 0, 16);
+  for (int li = 0; li < 4; ++li) {
+    const Lin& l = c->lin[li];
+    if (!l.kx) continue;
+    cudaMemset(c->us[li], 0, T * l.kxp * 2);
+    cudaMemset(c->du[li], 0, T * l.kxp * 2);
+  }
+  if (cudaDeviceSynchronize() != cudaSuccess || cudaGetLastError() != cudaSuccess) {
+    mebp_ctx_destroy(c);
+    return MEBP_ERR_CUDA;
+  }
+  *out = c;
+  return MEBP_OK;
+}
+
+void mebp_ctx_destroy(mebp_ctx* c) {
+  if (!c) return;
+  cudaSetDevice(c->device);
+  cudaDeviceSynchronize();
+  for (void* p : c->dev_allocs) cudaFree(p);
+  for (cudaEvent_t e : c->evpool) cudaEventDestroy(e);
+  if (c->h_ckpt) cudaFreeHost(c->h_ckpt);
+  for (int i = 0; i < kCkptSlots; ++i) {
+    if (c->slot_free[i]) cudaEventDestroy(c->slot_free[i]);
+    if (c->slot_ready[i]) cudaEventDestroy(c->slot_ready[i]);
+  }
+  if (c->copy_stream) cudaStreamDestroy(c->copy_stream);
+  cudaGetLastError();
+  delete c;
+}
+
+const char* mebp_last_error(const mebp_ctx* c) { return c ? c->err_msg.c_str() : "NULL context"; }
+
+int64_t mebp_workspace_bytes(const mebp_ctx* c) { return c ? c->ws_bytes : 0; }
+
+int mebp_sync(mebp_ctx* c, void* stream) {
+  if (!c) return MEBP_ERR_INVALID_ARG;
+  if (cudaStreamSynchronize(S(stream)) != cudaSuccess) return fail(c, MEBP_ERR_CUDA, cudaGetErrorString(cudaGetLastError()));
+  int h = 0;
+  if (cudaMemcpy(&h, c->d_err, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return fail(c, MEBP_ERR_CUDA, cudaGetErrorString(cudaGetLastError()));
+  if (h) {
+    cudaMemset(c->d_err, 0, sizeof(int));
+    return fail(c, h, h == MEBP_ERR_TIMEOUT ? "a device-side bounded wait expired"
+                                            : "a kernel flagged invalid input (e.g. token id out of range)");
+  }
+  return MEBP_OK;
+}
+
+int64_t mebp_kernel_launches(void) { return g_launches.load(); }
+
+int mebp_profile_begin(mebp_ctx* c) {
+  if (!c) return MEBP_ERR_INVALID_ARG;
+  c->recs.clear();
+  c->evnext = 0;
+  c->prof = true;
+  return MEBP_OK;
+}
+
+int mebp_profile_end(mebp_ctx* c, mebp_profile* out) {
+  if (!c || !out) return MEBP_ERR_INVALID_ARG;
+  c->prof = false;
+  mebp_profile p{};
+  for (const ProfRec& r : c->recs) {
+    if (cudaEventSynchronize(r.b) != cudaSuccess) return fail(c, MEBP_ERR_CUDA, cudaGetErrorString(cudaGetLastError()));
+    float ms = 0.0f;
+    cudaEventElapsedTime(&ms, r.a, r.b);
+    p.gemm_launches++;
+    p.gemm_ms += ms;
+    p.gemm_flops += r.flops;
+    if (r.trans) {
+      p.dx_ms += ms;
+      p.dx_flops += r.flops;
+    } else {
+      p.fwd_ms += ms;
+      p.fwd_flops += r.flops;
+    }
+  }
+  c->recs.clear();
+  c->evnext = 0;
+  *out = p;
+  return cuda_check(c, "profile");
+}
+
+int mebp_compress_weights(mebp_ctx* c, const float* W, int64_t rows, int64_t cols, int group, uint8_t* qpack,
+                          uint16_t* scales, void* stream) {
+  if (!c) return MEBP_ERR_INVALID_ARG;
+  if (!W || !qpack || !scales) return fail(c, MEBP_ERR_INVALID_ARG, "NULL pointer");
+  if (group != 64) return fail(c, MEBP_ERR_UNSUPPORTED, "group must be 64");
+  if (rows <= 0 || cols <= 0 || cols % 64) return fail(c, MEBP_ERR_INVALID_ARG, "cols must be a positive multiple of 64");
+  if (reinterpret_cast<uintptr_t>(W) & 7) return fail(c, MEBP_ERR_INVALID_ARG, "W must be 8-byte aligned");
+  launch_compress(W, rows, cols, qpack, scales, S(stream));
+  return cuda_check(c, "compress");
+}
+
+int mebp_decode_weights(mebp_ctx* c, const mebp_packed* w, uint16_t* out, void* stream) {
+  if (!c) return MEBP_ERR_INVALID_ARG;
+  if (!w || !w->qpack || !w->scales || !out) return fail(c, MEBP_ERR_INVALID_ARG, "NULL pointer");
+  if (w->rows <= 0 || w->cols <= 0 || w->cols % 64) return fail(c, MEBP_ERR_INVALID_ARG, "bad shape");
+  if (!aligned16(w->qpack) || !aligned16(out)) return fail(c, MEBP_ERR_INVALID_ARG, "pointers must be 16-byte aligned");
+  launch_decode(w->qpack, w->scales, w->rows, w->cols, out, S(stream));
+  return cuda_check(c, "decode");
+}
+
+int mebp_embed(mebp_ctx* c, const mebp_packed* E, const int32_t* ids, int64_t n, float* x0, void* stream) {
+  if (!c) return MEBP_ERR_INVALID_ARG;
+  if (!E || !E->qpack || !E->scales || !ids || !x0) return fail(c, MEBP_ERR_INVALID_ARG, "NULL pointer");
+  if (E->cols % 64 || E->rows <= 0) return fail(c, MEBP_ERR_INVALID_ARG, "bad embedding shape");
+  if (!aligned16(x0) || (reinterpret_cast<uintptr_t>(E->qpack) & 3))
+    return fail(c, MEBP_ERR_INVALID_ARG, "misaligned pointer");
+  if (n <= 0) return MEBP_OK;
+  launch_embed(E->qpack, E->scales, E->rows, E->cols, ids, n, x0, c->d_err, S(stream));
+  return cuda_check(c, "embed");
+}
+
+// One standalone LoRA linear (uses stream-ordered temporaries for the bf16 shadows).
+static int linear_common(mebp_ctx* c, bool dx_mode, const uint16_t* X, int64_t M, const mebp_packed* W,
+                         const float* A, const float* Bm, int r, float s, const float* R, float* y32, uint16_t* y16,
+                         cudaStream_t st) {
+  if (!W || !W->qpack || !W->scales || !X) return fail(c, MEBP_ERR_INVALID_ARG, "NULL pointer");
+  const int64_t N = W->rows, K = W->cols;
+  if (N % 64 || K % 64 || N <= 0 || K <= 0) return fail(c, MEBP_ERR_INVALID_ARG, "W dims must be multiples of 64");
+  if (!aligned16(X) || !aligned16(W->qpack) || !aligned16(W->scales))
+    return fail(c, MEBP_ERR_INVALID_ARG, "pointers must be 16-byte aligned");
+  if ((A == nullptr) != (Bm == nullptr)) return fail(c, MEBP_ERR_INVALID_ARG, "A and B must both be set or both NULL");
+  if (A && (r <= 0 || r > 32 || r % 8)) return fail(c, MEBP_ERR_UNSUPPORTED, "rank must be 8, 16, 24 or 32");
+  if (M <= 0) return MEBP_OK;
+  const int kxp = A ? (r + 15) / 16 * 16 : 0;
+  uint16_t *Ac = nullptr, *Bc = nullptr, *Btc = nullptr, *u = nullptr;
+  if (A) {
+    const size_t bytes = (static_cast<size_t>(kxp) * K + 2 * static_cast<size_t>(N) * kxp + M * kxp) * 2;
+    void* base = nullptr;
+    if (cudaMallocAsync(&base, bytes, st) != cudaSuccess) {
+      cudaGetLastError();
+      return fail(c, MEBP_ERR_OOM, "temporary allocation failed");
+    }
+    Ac = static_cast<uint16_t*>(base);
+    Bc = Ac + static_cast<size_t>(kxp) * K;
+    Btc = Bc + static_cast<size_t>(N) * kxp;
+    u = Btc + static_cast<size_t>(N) * kxp;
+    const float* As[1] = {A};
+    const float* Bs[1] = {Bm};
+    const int ro[1] = {0}, no[1] = {0};
+    const int nl[1] = {static_cast<int>(N)};
+    launch_lora_shadow(As, Bs, 1, ro, no, nl, r, static_cast<int>(K), static_cast<int>(N), kxp, Ac, Bc, Btc, st);
+  }
+  GemmArgs g;
+  if (!dx_mode) {
+    g = gemm_fwd(X, K, M, *W, static_cast<int>(N), static_cast<int>(K));
+    if (A) {
+      launch_skinny_gemm(X, K, M, K, Ac, K, r, s, u, kxp, st);
+      g.Ax = u; g.ldax = kxp; g.kx = kxp; g.Bx = Bc; g.ldbx = kxp;
+    }
+    if (y32) {
+      g.epi = EPI_F32; g.C = y32; g.ldc = N; g.R = R; g.ldr = N;
+    } else {
+      g.epi = EPI_BF16; g.C = y16; g.ldc = N;
+    }
+  } else {
+    g = gemm_dx(X, N, M, *W);
+    if (A) {
+      launch_skinny_gemm(X, N, M, N, Btc, N, r, s, u, kxp, st);
+      g.Ax = u; g.ldax = kxp; g.kx = kxp; g.Bx = Ac; g.ldbx = K;
+    }
+    g.epi = EPI_F32; g.C = y32; g.ldc = K; g.R = R; g.ldr = K;
+  }
+  int rc = run_gemm(c, g, st, dx_mode ? "linear dX" : "linear forward");
+  if (A) cudaFreeAsync(Ac, st);
+  if (rc) return rc;
+  return cuda_check(c, "linear");
+}
+
+int mebp_linear_fwd(mebp_ctx* c, const uint16_t* X, int64_t M, const mebp_packed* W, const float* A, const float* B,
+                    int r, float s, const float* R, float* y_f32, uint16_t* y_bf16, void* stream) {
+  if (!c) return MEBP_ERR_INVALID_ARG;
+  if (!y_f32 && !y_bf16) return fail(c, MEBP_ERR_INVALID_ARG, "no output");
+  return linear_common(c, false, X, M, W, A, B, r, s, R, y_f32, y_bf16, S(stream));
+}
+
+int mebp_linear_dx(mebp_ctx* c, const uint16_t* dY, int64_t M, const mebp_packed* W, const float* A, const float* B,
+                   int r, float s, const float* R, float* dx, void* stream) {
+  if (!c) return MEBP_ERR_INVALID_ARG;
+  if (!dx) return fail(c, MEBP_ERR_INVALID_ARG, "no output");
+  return linear_common(c, true, dY, M, W, A, B, r, s, R, dx, nullptr, S(stream));
+}
+
+int mebp_block_recompute_fwd(mebp_ctx* c, int layer, const mebp_block_weights* w, const mebp_lora* lora,
+                             const float* x, float* y, int B, int Sq, int save_for_bwd, void* stream) {
+  if (!c) return MEBP_ERR_INVALID_ARG;
+  int rc;
+  if ((rc = check_tokens(c, B, Sq)) || (rc = check_block_ptrs(c, w)) || (rc = check_lora(c, lora))) return rc;
+  if (!x || !y || !aligned16(x) || !aligned16(y)) return fail(c, MEBP_ERR_INVALID_ARG, "x / y must be 16-byte aligned");
+  if (x == y) return fail(c, MEBP_ERR_INVALID_ARG, "x and y must not alias");
+  rc = block_forward(c, layer, w, lora, x, y, B, Sq, true, S(stream));
+  if (!save_for_bwd) c->saved_layer = -1;
+  return rc;
+}
+
+int mebp_block_bwd(mebp_ctx* c, int layer, const mebp_block_weights* w, const mebp_lora* lora, const float* x,
+                   const float* dy, float* dx, const mebp_lora_grads* grads, int B, int Sq, int accumulate,
+                   void* stream) {
+  if (!c) return MEBP_ERR_INVALID_ARG;
+  int rc;
+  if ((rc = check_tokens(c, B, Sq)) || (rc = check_block_ptrs(c, w)) || (rc = check_lora(c, lora))) return rc;
+  if (!x || !dy || !aligned16(x) || !aligned16(dy) || (dx && !aligned16(dx)))
+    return fail(c, MEBP_ERR_INVALID_ARG, "x / dy / dx must be 16-byte aligned");
+  return block_backward(c, layer, w, lora, x, dy, nullptr, dx, nullptr, grads, B, Sq, accumulate != 0, S(stream));
+}
+
+int mebp_lmhead_ce_fwd_bwd(mebp_ctx* c, const mebp_packed* E, const float* gf, const float* h, const int32_t* targets,
+                           int64_t T, float* loss, float* dh, float* token_loss, void* stream) {
+  if (!c) return MEBP_ERR_INVALID_ARG;
+  if (c->V <= 0) return fail(c, MEBP_ERR_INVALID_ARG, "context has no vocabulary");
+  int rc;
+  if ((rc = check_packed(c, E, c->V, c->D, "embedding"))) return rc;
+  if (!gf || !h || !targets || !loss || !dh) return fail(c, MEBP_ERR_INVALID_ARG, "NULL pointer");
+  if (T <= 0 || T > c->Tmax) return fail(c, MEBP_ERR_INVALID_ARG, "n_tokens out of range");
+  if (!aligned16(h) || !aligned16(dh)) return fail(c, MEBP_ERR_INVALID_ARG, "h / dh must be 16-byte aligned");
+  return lmhead(c, E, gf, h, targets, T, loss, dh, nullptr, token_loss, S(stream));
+}
+
+int mebp_lora_step(mebp_ctx* c, const mebp_model_weights* model, const mebp_lora* lora, const int32_t* ids, int B,
+                   int Sq, float* loss, const mebp_lora_grads* grads, int accumulate, void* stream) {
+  if (!c) return MEBP_ERR_INVALID_ARG;
+  int rc;
+  if (!model || !model->blocks || !lora || !ids || !loss) return fail(c, MEBP_ERR_INVALID_ARG, "NULL pointer");
+  if (c->V <= 0) return fail(c, MEBP_ERR_INVALID_ARG, "context has no vocabulary");
+  if ((rc = check_tokens(c, B, Sq))) return rc;
+  if ((rc = check_packed(c, &model->embed, c->V, c->D, "embedding"))) return rc;
+  if (!model->final_norm) return fail(c, MEBP_ERR_INVALID_ARG, "NULL final norm");
+  for (int i = 0; i < c->L; ++i)
+    if ((rc = check_block_ptrs(c, &model->blocks[i])) || (rc = check_lora(c, &lora[i]))) return rc;
+  cudaStream_t st = S(stream);
+  const int64_t T = static_cast<int64_t>(B) * Sq, D = c->D;
+  const int L = c->L;
+  const bool spill = c->cfg.spill_ckpts != 0;
+  count_launch();
+  targets_kernel<<<static_cast<unsigned>((T + 255) / 256), 256, 0, st>>>(ids, B, Sq, c->targets);
+  // Checkpoint placement (Algorithm 1's ckpts_storage): HBM slot i, or, when spilling, a ring
+  // of kCkptSlots device slots whose contents are copied to / from pinned host memory on a
+  // side stream (the stand-in for memory-mapped checkpoints).
+  if (L + 1 > 4096) return fail(c, MEBP_ERR_UNSUPPORTED, "too many layers");
+  std::vector<int> slot_of(L + 1, -1);
+  int holds[kCkptSlots];
+  for (int k = 0; k < kCkptSlots; ++k) holds[k] = -1;
+  auto dev_ckpt = [&](int slot) { return c->ckpt + static_cast<int64_t>(slot) * c->Tmax * D; };
+  auto host_ckpt = [&](int i) { return c->h_ckpt + static_cast<int64_t>(i) * c->Tmax * D; };
+  // A free slot, else the one holding the lowest-index checkpoint other than `avoid` (every
+  // checkpoint below L also lives on the host, so evicting it loses nothing).
+  auto take_slot = [&](int i, int avoid) {
+    int sl = -1;
+    for (int k = 0; k < kCkptSlots && sl < 0; ++k)
+      if (holds[k] < 0) sl = k;
+    if (sl < 0)
+      for (int k = 0; k < kCkptSlots; ++k)
+        if (holds[k] != avoid && (sl < 0 || holds[k] < holds[sl])) sl = k;
+    if (holds[sl] >= 0) slot_of[holds[sl]] = -1;
+    holds[sl] = i;
+    slot_of[i] = sl;
+    return sl;
+  };
+  auto release = [&](int i) {
+    if (slot_of[i] >= 0) holds[slot_of[i]] = -1;
+    slot_of[i] = -1;
+  };
+  // device -> host copy of checkpoint i once the main stream has produced it
+  auto spill_out = [&](int i) {
+    const int sl = slot_of[i];
+    cudaEventRecord(c->slot_ready[sl], st);
+    cudaStreamWaitEvent(c->copy_stream, c->slot_ready[sl], 0);
+    cudaMemcpyAsync(host_ckpt(i), dev_ckpt(sl), T * D * sizeof(float), cudaMemcpyDeviceToHost, c->copy_stream);
+    cudaEventRecord(c->slot_free[sl], c->copy_stream);
+  };
+  // host -> device copy of checkpoint i into a slot the main stream no longer reads
+  auto fetch_in = [&](int i, int avoid) {
+    const int sl = take_slot(i, avoid);
+    cudaEventRecord(c->slot_ready[sl], st);
+    cudaStreamWaitEvent(c->copy_stream, c->slot_ready[sl], 0);
+    cudaMemcpyAsync(dev_ckpt(sl), host_ckpt(i), T * D * sizeof(float), cudaMemcpyHostToDevice, c->copy_stream);
+    cudaEventRecord(c->slot_free[sl], c->copy_stream);
+  };
+
+  float* x0 = dev_ckpt(0);
+  if (spill) {
+    const int sl = take_slot(0, -1);
+    cudaStreamWaitEvent(st, c->slot_free[sl], 0);
+    x0 = dev_ckpt(sl);
+  }
+  launch_embed(model->embed.qpack, model->embed.scales, c->V, D, ids, T, x0, c->d_err, st);
+  if (spill) spill_out(0);
+  // ---- forward loop: store only block-boundary checkpoints
+  for (int i = 0; i < L; ++i) {
+    const float* xin = spill ? dev_ckpt(slot_of[i]) : dev_ckpt(i);
+    float* yout = dev_ckpt(i + 1);
+    if (spill) {
+      const int sl = take_slot(i + 1, i);
+      cudaStreamWaitEvent(st, c->slot_free[sl], 0);  // its previous contents reached the host
+      yout = dev_ckpt(sl);
+    }
+    if ((rc = block_forward(c, i, &model->blocks[i], &lora[i], xin, yout, B, Sq, true, st))) return rc;
+    if (spill && i + 1 < L) spill_out(i + 1);
+  }
+  // ---- loss subgraph: final norm + LM head + CE
+  const float* hL = spill ? dev_ckpt(slot_of[L]) : dev_ckpt(L);
+  int cur = 0;
+  if ((rc = lmhead(c, &model->embed, model->final_norm, hL, c->targets, T, loss, c->gbuf[cur], c->dy_bf[cur], nullptr,
+                   st)))
+    return rc;
+  if (spill) release(L);
+  // ---- backward loop in reverse order: recompute block i from ckpt_i, apply its VJP
+  for (int i = L - 1; i >= 0; --i) {
+    if (spill) {
+      if (slot_of[i] < 0) {
+        fetch_in(i, i + 1);
+        cudaStreamWaitEvent(st, c->slot_free[slot_of[i]], 0);
+      }
+      if (i > 0 && slot_of[i - 1] < 0) fetch_in(i - 1, i);  // prefetch while block i runs
+    }
+    const float* xin = spill ? dev_ckpt(slot_of[i]) : dev_ckpt(i);
+    const int nxt = cur ^ 1;
+    if ((rc = block_backward(c, i, &model->blocks[i], &lora[i], xin, c->gbuf[cur], c->dy_bf[cur],
+                             i > 0 ? c->gbuf[nxt] : nullptr, i > 0 ? c->dy_bf[nxt] : nullptr, &grads[i], B, Sq,
+                             accumulate != 0, st)))
+      return rc;
+    if (spill) {
+      release(i);  // the checkpoint is removed once its backward has consumed it
+      if (i > 0) cudaStreamWaitEvent(st, c->slot_free[slot_of[i - 1]], 0);
+    }
+    cur = nxt;
+  }
+  c->saved_layer = -1;
+  return cuda_check(c, "lora step");
+}
+
+}  // extern "C"

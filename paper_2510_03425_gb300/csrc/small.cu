@@ -1,0 +1,282 @@
+// Bandwidth-bound kernels of the block: RMSNorm forward/backward, RoPE, gated-MLP activation
+// forward/backward, casts, and the LM-head's log-sum-exp combine and loss reduction.
+// Every kernel streams rows with 16-byte vector accesses, one warp per row where a row
+// reduction is needed.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace mebp {
+
+// ------------------------------------------------------------------------------------ RMSNorm
+// y = x / sqrt(mean(x^2) + eps) * g  ->  bf16 (the GEMM operand); rstd saved for the backward.
+__global__ void rmsnorm_fwd_kernel(const float* __restrict__ x, const float* __restrict__ g, int64_t T, int D,
+                                   float eps, uint16_t* __restrict__ y, float* __restrict__ rstd) {
+  const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (row >= T) return;
+  const float4* xr = reinterpret_cast<const float4*>(x + row * D);
+  const int n4 = D >> 2;
+  float ss = 0.0f;
+  for (int i = lane; i < n4; i += 32) {
+    const float4 v = xr[i];
+    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  }
+  ss = warp_sum(ss);
+  const float r = rsqrtf(ss / static_cast<float>(D) + eps);
+  if (lane == 0 && rstd) rstd[row] = r;
+  const float4* gr = reinterpret_cast<const float4*>(g);
+  uint2* yr = reinterpret_cast<uint2*>(y + row * D);
+  for (int i = lane; i < n4; i += 32) {
+    const float4 v = xr[i], w = gr[i];
+    yr[i] = make_uint2(pack_bf16x2(v.x * r * w.x, v.y * r * w.y), pack_bf16x2(v.z * r * w.z, v.w * r * w.w));
+  }
+}
+
+// dx = resid + r (g*dy) - x r^3 / D * sum(g*dy*x)
+__global__ void rmsnorm_bwd_kernel(const float* __restrict__ dy, const float* __restrict__ x,
+                                   const float* __restrict__ g, const float* __restrict__ rstd,
+                                   const float* __restrict__ resid, int64_t T, int D, float* __restrict__ dx,
+                                   uint16_t* __restrict__ dxb) {
+  const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (row >= T) return;
+  const int n4 = D >> 2;
+  const float4* dr = reinterpret_cast<const float4*>(dy + row * D);
+  const float4* xr = reinterpret_cast<const float4*>(x + row * D);
+  const float4* gr = reinterpret_cast<const float4*>(g);
+  float dot = 0.0f;
+  for (int i = lane; i < n4; i += 32) {
+    const float4 a = dr[i], b = xr[i], w = gr[i];
+    dot += a.x * w.x * b.x + a.y * w.y * b.y + a.z * w.z * b.z + a.w * w.w * b.w;
+  }
+  dot = warp_sum(dot);
+  const float r = rstd[row];
+  const float c = r * r * r * dot / static_cast<float>(D);
+  const float4* rr = resid ? reinterpret_cast<const float4*>(resid + row * D) : nullptr;
+  float4* outr = reinterpret_cast<float4*>(dx + row * D);
+  uint2* outb = dxb ? reinterpret_cast<uint2*>(dxb + row * D) : nullptr;
+  for (int i = lane; i < n4; i += 32) {
+    const float4 a = dr[i], b = xr[i], w = gr[i];
+    float4 o = make_float4(r * w.x * a.x - b.x * c, r * w.y * a.y - b.y * c, r * w.z * a.z - b.z * c,
+                           r * w.w * a.w - b.w * c);
+    if (rr) {
+      const float4 q = rr[i];
+      o.x += q.x; o.y += q.y; o.z += q.z; o.w += q.w;
+    }
+    outr[i] = o;
+    if (outb) outb[i] = make_uint2(pack_bf16x2(o.x, o.y), pack_bf16x2(o.z, o.w));
+  }
+}
+
+void launch_rmsnorm_fwd(const float* x, const float* g, int64_t T, int D, float eps, uint16_t* y, float* rstd,
+                        cudaStream_t st) {
+  if (T <= 0) return;
+  count_launch();
+  rmsnorm_fwd_kernel<<<static_cast<unsigned>((T * 32 + 255) / 256), 256, 0, st>>>(x, g, T, D, eps, y, rstd);
+}
+void launch_rmsnorm_bwd(const float* dy, const float* x, const float* g, const float* rstd, const float* resid,
+                        int64_t T, int D, float* dx, uint16_t* dxb, cudaStream_t st) {
+  if (T <= 0) return;
+  count_launch();
+  rmsnorm_bwd_kernel<<<static_cast<unsigned>((T * 32 + 255) / 256), 256, 0, st>>>(dy, x, g, rstd, resid, T, D, dx,
+                                                                                   dxb);
+}
+
+// ------------------------------------------------------------------------------------ RoPE
+// Half-split rotation: (x1, x2) -> (x1 c - x2 s, x2 c + x1 s) with (c, s) = table[pos][j];
+// inverse rotates by -angle (the VJP).  One thread per (token, head, pair of j).
+__global__ void rope_kernel(uint16_t* __restrict__ qkv, int64_t T, int S, int nheads, int ld, int hd,
+                            const float2* __restrict__ cs, int inverse) {
+  const int half = hd >> 1, pairs = half >> 1;
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= T * nheads * pairs) return;
+  const int jp = static_cast<int>(i % pairs);
+  const int64_t th = i / pairs;
+  const int head = static_cast<int>(th % nheads);
+  const int64_t t = th / nheads;
+  const int pos = static_cast<int>(t % S);
+  uint16_t* base = qkv + t * ld + static_cast<int64_t>(head) * hd;
+  uint32_t* p1 = reinterpret_cast<uint32_t*>(base + 2 * jp);
+  uint32_t* p2 = reinterpret_cast<uint32_t*>(base + half + 2 * jp);
+  const uint32_t a = *p1, b = *p2;
+  const float2 c0 = cs[static_cast<int64_t>(pos) * half + 2 * jp];
+  const float2 c1 = cs[static_cast<int64_t>(pos) * half + 2 * jp + 1];
+  const float sg = inverse ? -1.0f : 1.0f;
+  const float x1a = bf16_lo(a), x1b = bf16_hi(a), x2a = bf16_lo(b), x2b = bf16_hi(b);
+  const float s0 = sg * c0.y, s1 = sg * c1.y;
+  *p1 = pack_bf16x2(x1a * c0.x - x2a * s0, x1b * c1.x - x2b * s1);
+  *p2 = pack_bf16x2(x2a * c0.x + x1a * s0, x2b * c1.x + x1b * s1);
+}
+
+void launch_rope(uint16_t* qkv, int64_t T, int S, int H, int KV, int hd, const float2* cs, bool inverse,
+                 cudaStream_t st) {
+  const int nheads = H + KV;  // q heads then k heads
+  const int64_t n = T * nheads * (hd / 4);
+  if (n <= 0) return;
+  count_launch();
+  rope_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(qkv, T, S, nheads, (H + 2 * KV) * hd, hd, cs,
+                                                                      inverse ? 1 : 0);
+}
+
+// ------------------------------------------------------------------------------------ gated MLP
+__device__ __forceinline__ float act_f(float x, int act) {
+  if (act == MEBP_ACT_SILU) return x / (1.0f + __expf(-x));
+  const float k0 = 0.7978845608028654f;  // sqrt(2/pi)
+  return 0.5f * x * (1.0f + tanhf(k0 * (x + 0.044715f * x * x * x)));
+}
+__device__ __forceinline__ float act_grad(float x, int act) {
+  if (act == MEBP_ACT_SILU) {
+    const float sg = 1.0f / (1.0f + __expf(-x));
+    return sg * (1.0f + x * (1.0f - sg));
+  }
+  const float k0 = 0.7978845608028654f;
+  const float th = tanhf(k0 * (x + 0.044715f * x * x * x));
+  return 0.5f * (1.0f + th) + 0.5f * x * (1.0f - th * th) * k0 * (1.0f + 3.0f * 0.044715f * x * x);
+}
+
+// m = act(g) * u; gu row = [g (I) | u (I)].  8 elements per thread.
+__global__ void glu_fwd_kernel(const uint16_t* __restrict__ gu, int64_t T, int I, int act, uint16_t* __restrict__ m) {
+  const int per = I / 8;
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= T * per) return;
+  const int64_t t = i / per;
+  const int c = static_cast<int>(i % per) * 8;
+  const uint4 gv = *reinterpret_cast<const uint4*>(gu + t * 2 * I + c);
+  const uint4 uv = *reinterpret_cast<const uint4*>(gu + t * 2 * I + I + c);
+  const uint32_t ga[4] = {gv.x, gv.y, gv.z, gv.w}, ua[4] = {uv.x, uv.y, uv.z, uv.w};
+  uint32_t o[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k)
+    o[k] = pack_bf16x2(act_f(bf16_lo(ga[k]), act) * bf16_lo(ua[k]), act_f(bf16_hi(ga[k]), act) * bf16_hi(ua[k]));
+  *reinterpret_cast<uint4*>(m + t * I + c) = make_uint4(o[0], o[1], o[2], o[3]);
+}
+
+// dg = dm * u * act'(g), du = dm * act(g)
+__global__ void glu_bwd_kernel(const float* __restrict__ dm, const uint16_t* __restrict__ gu, int64_t T, int I, int act,
+                               uint16_t* __restrict__ dgu) {
+  const int per = I / 8;
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= T * per) return;
+  const int64_t t = i / per;
+  const int c = static_cast<int>(i % per) * 8;
+  const uint4 gv = *reinterpret_cast<const uint4*>(gu + t * 2 * I + c);
+  const uint4 uv = *reinterpret_cast<const uint4*>(gu + t * 2 * I + I + c);
+  const float4 d0 = *reinterpret_cast<const float4*>(dm + t * I + c);
+  const float4 d1 = *reinterpret_cast<const float4*>(dm + t * I + c + 4);
+  const float dd[8] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
+  const uint32_t ga[4] = {gv.x, gv.y, gv.z, gv.w}, ua[4] = {uv.x, uv.y, uv.z, uv.w};
+  uint32_t og[4], ou[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const float g0 = bf16_lo(ga[k]), g1 = bf16_hi(ga[k]), u0 = bf16_lo(ua[k]), u1 = bf16_hi(ua[k]);
+    og[k] = pack_bf16x2(dd[2 * k] * u0 * act_grad(g0, act), dd[2 * k + 1] * u1 * act_grad(g1, act));
+    ou[k] = pack_bf16x2(dd[2 * k] * act_f(g0, act), dd[2 * k + 1] * act_f(g1, act));
+  }
+  *reinterpret_cast<uint4*>(dgu + t * 2 * I + c) = make_uint4(og[0], og[1], og[2], og[3]);
+  *reinterpret_cast<uint4*>(dgu + t * 2 * I + I + c) = make_uint4(ou[0], ou[1], ou[2], ou[3]);
+}
+
+void launch_glu_fwd(const uint16_t* gu, int64_t T, int I, int act, uint16_t* m, cudaStream_t st) {
+  const int64_t n = T * (I / 8);
+  if (n <= 0) return;
+  count_launch();
+  glu_fwd_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(gu, T, I, act, m);
+}
+void launch_glu_bwd(const float* dm, const uint16_t* gu, int64_t T, int I, int act, uint16_t* dgu, cudaStream_t st) {
+  const int64_t n = T * (I / 8);
+  if (n <= 0) return;
+  count_launch();
+  glu_bwd_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(dm, gu, T, I, act, dgu);
+}
+
+// ------------------------------------------------------------------------------------ casts
+__global__ void cast_bf16_kernel(const float* __restrict__ x, int64_t n4, uint16_t* __restrict__ y) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= n4) return;
+  const float4 v = reinterpret_cast<const float4*>(x)[i];
+  reinterpret_cast<uint2*>(y)[i] = make_uint2(pack_bf16x2(v.x, v.y), pack_bf16x2(v.z, v.w));
+}
+__global__ void fill_kernel(float* __restrict__ x, int64_t n, float v) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i < n) x[i] = v;
+}
+void launch_cast_bf16(const float* x, int64_t n, uint16_t* y, cudaStream_t st) {
+  const int64_t n4 = n / 4;
+  if (n4 <= 0) return;
+  count_launch();
+  cast_bf16_kernel<<<static_cast<unsigned>((n4 + 255) / 256), 256, 0, st>>>(x, n4, y);
+}
+void launch_fill_f32(float* x, int64_t n, float v, cudaStream_t st) {
+  if (n <= 0) return;
+  count_launch();
+  fill_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(x, n, v);
+}
+
+// ------------------------------------------------------------------------------------ LM head
+// lse[t] = M + log(sum_i l_i exp(m_i - M)) over the per-tile partials (m_i, l_i);
+// tok_loss[t] = lse[t] - z_target[t] for valid targets, else 0.
+__global__ void lse_combine_kernel(const float2* __restrict__ part, int nparts, const float* __restrict__ zt,
+                                   const int32_t* __restrict__ targets, int64_t T, float* __restrict__ lse,
+                                   float* __restrict__ tok_loss) {
+  const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (row >= T) return;
+  const float2* pr = part + row * nparts;
+  float mx = -INFINITY;
+  for (int i = lane; i < nparts; i += 32) mx = fmaxf(mx, pr[i].x);
+  mx = warp_max(mx);
+  float s = 0.0f;
+  for (int i = lane; i < nparts; i += 32) {
+    const float2 v = pr[i];
+    if (v.x > -INFINITY) s += v.y * expf(v.x - mx);
+  }
+  s = warp_sum(s);
+  if (lane == 0) {
+    const float l = mx + logf(s);
+    lse[row] = l;
+    tok_loss[row] = targets[row] >= 0 ? l - zt[row] : 0.0f;
+  }
+}
+
+// loss = sum(tok_loss) / n_valid, inv_n = 1 / n_valid: one block, fixed reduction order.
+__global__ void loss_reduce_kernel(const float* __restrict__ tok_loss, const int32_t* __restrict__ targets, int64_t T,
+                                   float* __restrict__ loss, float* __restrict__ inv_n) {
+  __shared__ double ssum[1024];
+  __shared__ int scnt[1024];
+  double s = 0.0;
+  int c = 0;
+  for (int64_t i = threadIdx.x; i < T; i += blockDim.x) {
+    s += static_cast<double>(tok_loss[i]);
+    c += targets[i] >= 0 ? 1 : 0;
+  }
+  ssum[threadIdx.x] = s;
+  scnt[threadIdx.x] = c;
+  __syncthreads();
+  for (int w = blockDim.x / 2; w > 0; w >>= 1) {
+    if (threadIdx.x < w) {
+      ssum[threadIdx.x] += ssum[threadIdx.x + w];
+      scnt[threadIdx.x] += scnt[threadIdx.x + w];
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    const int n = scnt[0];
+    *loss = n > 0 ? static_cast<float>(ssum[0] / n) : 0.0f;
+    *inv_n = n > 0 ? 1.0f / static_cast<float>(n) : 0.0f;
+  }
+}
+
+void launch_lse_combine(const float* part, int nparts, const float* zt, const int32_t* targets, int64_t T, float* lse,
+                        float* tok_loss, cudaStream_t st) {
+  if (T <= 0) return;
+  count_launch();
+  lse_combine_kernel<<<static_cast<unsigned>((T * 32 + 255) / 256), 256, 0, st>>>(
+      reinterpret_cast<const float2*>(part), nparts, zt, targets, T, lse, tok_loss);
+}
+void launch_loss_reduce(const float* tok_loss, const int32_t* targets, int64_t T, float* loss, float* inv_n,
+                        cudaStream_t st) {
+  count_launch();
+  loss_reduce_kernel<<<1, 1024, 0, st>>>(tok_loss, targets, T, loss, inv_n);
+}
+
+}  // namespace mebp

@@ -1,0 +1,128 @@
+"""Block-level parity (forward_i / backward_i of Algorithm 1) of the CUDA path against the
+oracle: the single Qwen2.5-0.5B-shaped block (batch 1 x seq 128, objective sum(G*y)) and
+smaller blocks covering head dims 128 / 256, grouped-query attention, GeGLU, every LoRA
+target, ranks 8-32 and sequence lengths that leave ragged tiles."""
+import numpy as np
+import pytest
+
+from oracle import model as OM
+from oracle import quant
+from workload import synth
+
+from .helpers import np_of, rel_fro, to_gpu
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+if not torch.cuda.is_available():
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+from paper_2510_03425_gb300 import mebp as M  # noqa: E402
+from paper_2510_03425_gb300.model import Context, DeviceBlock, LoraSet  # noqa: E402
+
+TOL = 2e-2  # relative Frobenius error of gradients (bf16 operands, fp32 accumulate)
+
+
+def oracle_dense(W):
+    """The oracle's own decode of the oracle's own compression of W."""
+    out = {n: quant.dequant(*quant.compress(W[n])) for n in OM.LINEARS}
+    out["norm1"] = W["norm1"].astype(np.float64)
+    out["norm2"] = W["norm2"].astype(np.float64)
+    return out
+
+
+def run_block(dims, jitter=0.0, zero_b=False, x_scale=1.0):
+    W = synth.block_weights(dims, 0, norm_jitter=jitter)
+    L = synth.lora_weights(dims, 0, zero_b=zero_b)
+    x = synth.hidden_input(dims) * np.float32(x_scale)
+    G = synth.upstream_grad(dims)
+    ctx = Context(dims)
+    blk = DeviceBlock(ctx, {k: to_gpu(v) for k, v in W.items()})
+    ls = LoraSet([L])
+    xg, Gg = to_gpu(x), to_gpu(G)
+    y = torch.empty_like(xg)
+    dx = torch.empty_like(xg)
+    M.mebp_block_recompute_fwd(ctx.handle, 0, blk.struct(), ls.layer(0), xg, y, dims.batch, dims.seq, False)
+    M.mebp_block_bwd(ctx.handle, 0, blk.struct(), ls.layer(0), xg, Gg, dx, ls.layer_grads(0), dims.batch, dims.seq)
+    ctx.sync()
+    gpu = dict(y=np_of(y), dx=np_of(dx), grads={n: (np_of(a), np_of(b)) for n, (a, b) in ls.grads[0].items()})
+    # oracle
+    Wd = oracle_dense(W)
+    Lo = OM.lora64(L)
+    xo = x.astype(np.float64)
+    yo, _ = OM.block_forward(xo, Wd, Lo, dims)
+    _, dxo, go = OM.block_objective(xo, Wd, Lo, G.astype(np.float64), dims)
+    ref = dict(y=yo, dx=dxo, grads=go, x=xo)
+    return gpu, ref, (ctx, blk, ls, xg, Gg)
+
+
+def check(gpu, ref, tol=TOL):
+    assert rel_fro(gpu["y"] - ref["x"], ref["y"] - ref["x"]) < tol
+    assert rel_fro(gpu["dx"], ref["dx"]) < tol
+    for n, (dA, dB) in ref["grads"].items():
+        ga, gb = gpu["grads"][n]
+        assert rel_fro(gb, dB) < tol, (n, "dB", rel_fro(gb, dB))
+        if np.linalg.norm(dA) > 0:
+            assert rel_fro(ga, dA) < tol, (n, "dA", rel_fro(ga, dA))
+
+
+def test_qwen05b_block_matches_oracle():
+    gpu, ref, _ = run_block(synth.preset(0))
+    check(gpu, ref)
+
+
+@pytest.mark.parametrize("kw", [
+    dict(hidden=256, n_heads=4, n_kv_heads=2, head_dim=128, intermediate=512, act="silu", batch=2, seq=80,
+         rank=16, alpha=32.0, targets=synth.TARGETS),
+    dict(hidden=512, n_heads=2, n_kv_heads=1, head_dim=256, intermediate=768, act="gelu_tanh", batch=1, seq=200,
+         rank=32, alpha=64.0, targets=synth.TARGETS),
+    dict(hidden=192, n_heads=3, n_kv_heads=3, head_dim=64, intermediate=320, act="gelu_tanh", batch=3, seq=33,
+         rank=8, alpha=16.0, targets=("q", "v", "up", "down")),
+])
+def test_block_variants_match_oracle(kw):
+    dims = synth.tiny(n_layers=1, vocab=0, **kw)
+    gpu, ref, _ = run_block(dims, jitter=0.1)
+    check(gpu, ref)
+
+
+def test_lora_b_zero_block_equals_base_block_and_da_is_zero():
+    dims = synth.preset(0)
+    gpu, ref, (ctx, blk, ls, xg, Gg) = run_block(dims, zero_b=True)
+    for n, (dA, dB) in gpu["grads"].items():
+        assert np.all(dA == 0), n
+        assert np.any(dB != 0), n
+    # base block (no LoRA targets) is bit-identical to LoRA with B = 0
+    base = dims.with_(targets=())
+    ctx0 = Context(base)
+    W = synth.block_weights(dims, 0)
+    blk0 = DeviceBlock(ctx0, {k: to_gpu(v) for k, v in W.items()})
+    y0 = torch.empty_like(xg)
+    M.mebp_block_recompute_fwd(ctx0.handle, 0, blk0.struct(), M.Lora(), xg, y0, dims.batch, dims.seq, False)
+    ctx0.sync()
+    np.testing.assert_array_equal(np_of(y0), gpu["y"])
+
+
+def test_saved_intermediates_give_the_same_backward_as_recompute():
+    dims = synth.preset(0)
+    gpu, _, (ctx, blk, ls, xg, Gg) = run_block(dims)
+    y = torch.empty_like(xg)
+    dx = torch.empty_like(xg)
+    M.mebp_block_recompute_fwd(ctx.handle, 0, blk.struct(), ls.layer(0), xg, y, dims.batch, dims.seq, True)
+    M.mebp_block_bwd(ctx.handle, 0, blk.struct(), ls.layer(0), xg, Gg, dx, ls.layer_grads(0), dims.batch, dims.seq)
+    ctx.sync()
+    np.testing.assert_array_equal(np_of(dx), gpu["dx"])
+    for n, (a, b) in ls.grads[0].items():
+        np.testing.assert_array_equal(np_of(a), gpu["grads"][n][0])
+        np.testing.assert_array_equal(np_of(b), gpu["grads"][n][1])
+
+
+def test_gradient_accumulation_adds():
+    dims = synth.preset(0)
+    gpu, _, (ctx, blk, ls, xg, Gg) = run_block(dims)
+    dx = torch.empty_like(xg)
+    M.mebp_block_bwd(ctx.handle, 0, blk.struct(), ls.layer(0), xg, Gg, dx, ls.layer_grads(0), dims.batch, dims.seq,
+                     accumulate=True)
+    ctx.sync()
+    for n, (a, b) in ls.grads[0].items():
+        np.testing.assert_array_equal(np_of(a), 2 * gpu["grads"][n][0])
+        np.testing.assert_array_equal(np_of(b), 2 * gpu["grads"][n][1])

@@ -1,0 +1,182 @@
+"""Kernel-level parity of the CUDA path (through the C ABI) against the CPU oracle:
+compression and decode bit-exact, embedding gather exact, and the fused dequant-GEMMs
+(forward and transposed) against fp64 references built from the oracle's decode."""
+import numpy as np
+import pytest
+
+from oracle import quant
+from workload import synth
+
+from .helpers import bf16_round, np_of, rel_fro, to_gpu
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+if not torch.cuda.is_available():
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+from paper_2510_03425_gb300 import mebp as M  # noqa: E402
+from paper_2510_03425_gb300.model import Context, compress  # noqa: E402
+
+
+@pytest.fixture(scope="module")
+def ctx():
+    c = Context(synth.tiny(), max_tokens=4096, max_seq=64)
+    yield c
+    c.close()
+
+
+def _w(rows, cols, seed, std=0.02):
+    W = (np.random.default_rng(seed).standard_normal((rows, cols)) * std).astype(np.float32)
+    W[min(3, rows - 1), 64:128 if cols >= 128 else 64] *= 500.0  # a loud group
+    if rows > 5:
+        W[5, :64] = 0.0                                            # an all-zero group
+    return W
+
+
+@pytest.mark.parametrize("rows,cols", [(1, 64), (7, 192), (256, 896), (1152, 896), (333, 4864)])
+def test_compress_bit_exact(ctx, rows, cols):
+    W = _w(rows, cols, rows + cols)
+    q, s = compress(ctx, to_gpu(W))
+    ctx.sync()
+    qo, so = quant.compress(W)
+    np.testing.assert_array_equal(np_of(q), qo)
+    np.testing.assert_array_equal(s.cpu().numpy().view(np.uint16), so.view(np.uint16))
+
+
+def test_decode_bit_exact(ctx):
+    W = _w(320, 1024, 5, std=0.3)
+    qo, so = quant.compress(W)
+    out = torch.empty((320, 1024), dtype=torch.int16, device="cuda")
+    M.mebp_decode_weights(ctx.handle, M.packed(to_gpu(qo), to_gpu(so)), out)
+    ctx.sync()
+    np.testing.assert_array_equal(out.cpu().numpy().view(np.uint16), quant.dequant_bf16_bits(qo, so))
+
+
+def test_embedding_gather_exact(ctx):
+    V, D = 1000, 256
+    E = _w(V, D, 9, std=0.5)
+    qo, so = quant.compress(E)
+    ids = np.random.default_rng(1).integers(0, V, 777).astype(np.int32)
+    x0 = torch.empty((777, D), dtype=torch.float32, device="cuda")
+    M.mebp_embed(ctx.handle, M.packed(to_gpu(qo), to_gpu(so)), to_gpu(ids), x0)
+    ctx.sync()
+    np.testing.assert_array_equal(np_of(x0).astype(np.float64), quant.dequant_rows(qo, so, ids))
+
+
+def test_embedding_bad_id_flags_device_error(ctx):
+    V, D = 128, 64
+    qo, so = quant.compress(_w(V, D, 3))
+    ids = to_gpu(np.array([1, 2, V + 5], np.int32))
+    x0 = torch.full((3, D), 7.0, device="cuda")
+    M.mebp_embed(ctx.handle, M.packed(to_gpu(qo), to_gpu(so)), ids, x0)
+    with pytest.raises(M.MebpError) as ei:
+        ctx.sync()
+    assert ei.value.code == M.ERR_DEVICE
+    assert (x0[2] == 0).all()
+    ctx.sync()  # the error word was cleared
+
+
+SHAPES = [(200, 320, 192), (128, 256, 64), (1, 64, 64), (300, 1152, 896), (513, 512, 1024)]
+
+
+def _x(M_, K, seed, scale=1.0):
+    x = (np.random.default_rng(seed).standard_normal((M_, K)) * scale).astype(np.float32)
+    return bf16_round(x)
+
+
+@pytest.mark.parametrize("Mr,N,K", SHAPES)
+def test_linear_fwd_matches_exact_operand_product(ctx, Mr, N, K):
+    """No LoRA: Y must equal X_bf16 . bf16(deq(W))^T up to fp32 accumulation."""
+    W = _w(N, K, N + K)
+    qo, so = quant.compress(W)
+    X = _x(Mr, K, 1)
+    ref = X @ quant.bf16_bits_to_f64(quant.dequant_bf16_bits(qo, so)).T
+    Xg = to_gpu(X.astype(np.float32)).to(torch.bfloat16)
+    Wp = M.packed(to_gpu(qo), to_gpu(so))
+    y = torch.empty((Mr, N), dtype=torch.float32, device="cuda")
+    yb = torch.empty((Mr, N), dtype=torch.bfloat16, device="cuda")
+    M.mebp_linear_fwd(ctx.handle, Xg, Wp, y_f32=y)
+    M.mebp_linear_fwd(ctx.handle, Xg, Wp, y_bf16=yb)
+    ctx.sync()
+    scale = np.abs(ref).max()
+    assert np.abs(np_of(y) - ref).max() <= 2e-5 * scale + 1e-6
+    assert np.abs(np_of(yb) - ref).max() <= 8e-3 * scale + 1e-6
+
+
+@pytest.mark.parametrize("Mr,N,K", SHAPES)
+def test_linear_dx_matches_exact_operand_product(ctx, Mr, N, K):
+    """No LoRA: dX = dY_bf16 . bf16(deq(W)) up to fp32 accumulation (W is [N, K])."""
+    W = _w(N, K, N + 2 * K)
+    qo, so = quant.compress(W)
+    dY = _x(Mr, N, 2)
+    ref = dY @ quant.bf16_bits_to_f64(quant.dequant_bf16_bits(qo, so))
+    dx = torch.empty((Mr, K), dtype=torch.float32, device="cuda")
+    M.mebp_linear_dx(ctx.handle, to_gpu(dY.astype(np.float32)).to(torch.bfloat16), M.packed(to_gpu(qo), to_gpu(so)),
+                     dx=dx)
+    ctx.sync()
+    assert np.abs(np_of(dx) - ref).max() <= 2e-5 * np.abs(ref).max() + 1e-6
+
+
+@pytest.mark.parametrize("r", [8, 16, 32])
+@pytest.mark.parametrize("Mr,N,K", [(200, 320, 192), (300, 1152, 896)])
+def test_linear_with_lora_against_oracle(ctx, r, Mr, N, K):
+    """Y = X deq(W)^T + s (X A^T) B^T (+R) and dX = dY deq(W) + s (dY B) A against fp64."""
+    s = 2.0
+    rng = np.random.default_rng(r)
+    W = _w(N, K, 11)
+    qo, so = quant.compress(W)
+    Wd = quant.dequant(qo, so)
+    A = (rng.standard_normal((r, K)) * 0.05).astype(np.float32)
+    B = (rng.standard_normal((N, r)) * 0.05).astype(np.float32)
+    X = _x(Mr, K, 3)
+    R = rng.standard_normal((Mr, N)).astype(np.float32)
+    ref = X @ Wd.T + s * (X @ A.T.astype(np.float64)) @ B.T.astype(np.float64) + R
+    Wp = M.packed(to_gpu(qo), to_gpu(so))
+    y = torch.empty((Mr, N), dtype=torch.float32, device="cuda")
+    Ag, Bg = to_gpu(A), to_gpu(B)
+    M.mebp_linear_fwd(ctx.handle, to_gpu(X.astype(np.float32)).to(torch.bfloat16), Wp, Ag, Bg, r, s, R=to_gpu(R), y_f32=y)
+    dY = _x(Mr, N, 4)
+    ref_dx = dY @ Wd + s * (dY @ B.astype(np.float64)) @ A.astype(np.float64)
+    dx = torch.empty((Mr, K), dtype=torch.float32, device="cuda")
+    M.mebp_linear_dx(ctx.handle, to_gpu(dY.astype(np.float32)).to(torch.bfloat16), Wp, Ag, Bg, r, s, dx=dx)
+    ctx.sync()
+    assert rel_fro(np_of(y) - R, ref - R) < 1e-2
+    assert rel_fro(np_of(dx), ref_dx) < 1e-2
+    # the LoRA term itself is carried (not just the base product)
+    base = X @ Wd.T
+    lora_term = ref - R - base
+    got_term = np_of(y).astype(np.float64) - R - base
+    assert rel_fro(got_term, lora_term) < 5e-2
+
+
+def test_lora_b_zero_is_bit_identical_to_base(ctx):
+    Mr, N, K, r = 257, 512, 384, 16
+    W = _w(N, K, 21)
+    qo, so = quant.compress(W)
+    Wp = M.packed(to_gpu(qo), to_gpu(so))
+    X = to_gpu(_x(Mr, K, 5).astype(np.float32)).to(torch.bfloat16)
+    A = to_gpu((np.random.default_rng(0).standard_normal((r, K)) * 0.1).astype(np.float32))
+    B0 = torch.zeros((N, r), device="cuda")
+    y0 = torch.empty((Mr, N), device="cuda")
+    y1 = torch.empty((Mr, N), device="cuda")
+    M.mebp_linear_fwd(ctx.handle, X, Wp, y_f32=y0)
+    M.mebp_linear_fwd(ctx.handle, X, Wp, A, B0, r, 2.0, y_f32=y1)
+    dY = to_gpu(_x(Mr, N, 6).astype(np.float32)).to(torch.bfloat16)
+    d0 = torch.empty((Mr, K), device="cuda")
+    d1 = torch.empty((Mr, K), device="cuda")
+    M.mebp_linear_dx(ctx.handle, dY, Wp, dx=d0)
+    M.mebp_linear_dx(ctx.handle, dY, Wp, A, B0, r, 2.0, dx=d1)
+    ctx.sync()
+    assert torch.equal(y0, y1)
+    assert torch.equal(d0, d1)
+
+
+def test_linear_rejects_bad_shapes(ctx):
+    q = torch.zeros((64, 48), dtype=torch.uint8, device="cuda")   # cols = 96: not a multiple of 64
+    s = torch.zeros((1, 64), dtype=torch.float16, device="cuda")
+    X = torch.zeros((4, 96), dtype=torch.bfloat16, device="cuda")
+    y = torch.empty((4, 64), device="cuda")
+    with pytest.raises(M.MebpError) as ei:
+        M.mebp_linear_fwd(ctx.handle, X, M.packed(q, s), y_f32=y)
+    assert ei.value.code == M.ERR_INVALID_ARG

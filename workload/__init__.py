@@ -6,5 +6,6 @@ oracle and the CUDA path receive what it produces as plain arrays.
 """
 from .synth import (  # noqa: F401
     PRESETS, TARGETS, ModelDims, preset, tiny, linear_shapes, block_weights,
-    embedding, lora_weights, hidden_input, token_ids, upstream_grad,
+    embedding, lora_weights, hidden_input, token_ids, upstream_grad, torch_block_weights,
+    torch_embedding,
 )

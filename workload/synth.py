@@ -89,7 +89,7 @@ def tiny(**kw) -> ModelDims:
     """A small model for oracle self-tests (finite differences etc.)."""
     base = dict(name="tiny", hidden=64, n_heads=2, n_kv_heads=1, head_dim=32,
                 intermediate=128, act="silu", n_layers=2, vocab=97, batch=2, seq=8,
-                rank=4, alpha=8.0, targets=_ALL7)
+                rank=8, alpha=16.0, targets=_ALL7)
     base.update(kw)
     return ModelDims(**base)
 
@@ -161,3 +161,28 @@ def token_ids(d: ModelDims, seed: int = 2) -> np.ndarray:
 def upstream_grad(d: ModelDims, seed: int = 3) -> np.ndarray:
     """Upstream gradient G = dE/dy [B*S, D] ~ N(0, 1) for the single-block objective E = sum(G * y)."""
     return _normal(seed, (0,), (d.tokens, d.hidden), 1.0)
+
+
+# ----------------------------------------------------------------------------- device-side draws
+# Large presets (billions of weights) are drawn directly on the GPU with torch's seeded
+# Philox generator: same distributions, a different (but equally seeded) stream from the
+# numpy draws above.  Used by the benchmark; parity tests use the numpy draws.
+
+def _torch_normal(shape, std, seed, key, device):
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed(int(np.random.SeedSequence([seed, *key]).generate_state(1, np.uint64)[0] & 0x7FFFFFFFFFFFFFFF))
+    return torch.randn(shape, generator=g, device=device, dtype=torch.float32) * std
+
+
+def torch_block_weights(d: ModelDims, layer: int, seed: int = 0, device="cuda", std: float = 0.02):
+    import torch
+    out = {name: _torch_normal(shp, std, seed, (layer, i), device) for i, (name, shp) in enumerate(linear_shapes(d).items())}
+    out["norm1"] = torch.ones(d.hidden, device=device)
+    out["norm2"] = torch.ones(d.hidden, device=device)
+    return out
+
+
+def torch_embedding(d: ModelDims, seed: int = 0, device="cuda", std: float = 0.02):
+    import torch
+    return _torch_normal((d.vocab, d.hidden), std, seed, (10_000, 0), device), torch.ones(d.hidden, device=device)
