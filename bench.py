@@ -245,7 +245,7 @@ def run_gpu(args, d, rank, world, local_rank):
     out = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1e3 * t / args.steps, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "scaling": "weak", "vs_baseline": None, "dtype": "f16", "data": "synthetic",
         "config": {"workload": workload_name(d), "config_index": args.config, "global_batch": world * d.batch,
                    "seq_len": d.seq, "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                    "l2": f"inputs larger than L2: {weights_mb:.0f} MB of packed block weights plus the "
@@ -253,7 +253,8 @@ def run_gpu(args, d, rank, world, local_rank):
         "roofline": {"kernel": "dequant_gemm_kernel (fused 4-bit dequant GEMM, tcgen05)", "bound": "tensor",
                      "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": (achieved / peak) if achieved else None, "traffic": None,
-                     "peak_source": f"{src} {'sustained' if long_step else 'burst'} bf16 (MEASURED_PEAKS.json)",
+                     "peak_source": f"{src} {'sustained' if long_step else 'burst'} dense bf16 GEMM rate "
+                                    "(MEASURED_PEAKS.json); fp16 and bf16 share the kind::f16 rate (nominal ratio 1)",
                      "launches_per_step": prof.gemm_launches / args.steps,
                      "share_of_step": (prof.gemm_ms / 1e3) / t if t > 0 else None,
                      "fwd_tflops": prof.fwd_flops / max(prof.fwd_ms, 1e-9) / 1e9,

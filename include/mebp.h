@@ -73,7 +73,7 @@ typedef struct {
  *   qpack  uint8 [rows, cols/2]: column 2j in the low nibble of byte j, 2j+1 in the high one;
  *   scales fp16 bits [cols/64, rows] (group-major: the scales of one column group are
  *          contiguous over rows).
- * deq(W)[n, k] = (u - 8) * scales[k/64, n]; the tensor cores consume bf16_rne(deq).
+ * deq(W)[n, k] = (u - 8) * scales[k/64, n]; the tensor cores consume fp16_rne(deq) (IEEE half).
  * Both pointers must be 16-byte aligned. */
 typedef struct {
   const uint8_t* qpack;
@@ -137,9 +137,9 @@ int64_t mebp_workspace_bytes(const mebp_ctx* ctx);
 int mebp_compress_weights(mebp_ctx* ctx, const float* W, int64_t rows, int64_t cols, int group,
                           uint8_t* qpack, uint16_t* scales, void* stream);
 
-/* Debug decode: out bf16 bits [rows, cols] = bf16_rne(q * s), produced by the same device
+/* Debug decode: out fp16 bits [rows, cols] = fp16_rne(q * s), produced by the same device
  * function that feeds the fused GEMM's shared-memory operand. */
-int mebp_decode_weights(mebp_ctx* ctx, const mebp_packed* w, uint16_t* out_bf16, void* stream);
+int mebp_decode_weights(mebp_ctx* ctx, const mebp_packed* w, uint16_t* out_f16, void* stream);
 
 /* Embedding gather + dequant: x0[t, :] = deq(E)[ids[t], :] (fp32 [n_tokens, D], exact).
  * An id outside [0, V) writes zeros and sets MEBP_ERR_DEVICE. */
@@ -149,14 +149,14 @@ int mebp_embed(mebp_ctx* ctx, const mebp_packed* embed, const int32_t* ids, int6
 /* ---- one LoRA linear with just-in-time dequantised base weight (Algorithm 1,
  * LazyLoadAndDecompressWeights, with the decompression fused into the GEMM mainloop).
  * mebp_linear_fwd:  Y [M, N] = X [M, K] deq(W)^T + s (X A^T) B^T  (+ R if R != NULL)
- *   X bf16 [M, K] (bits), W packed [N, K], A fp32 [r, K] / B fp32 [N, r] or both NULL,
- *   Y fp32 [M, N] when y_f32 != NULL else bf16 bits into y_bf16.  R fp32 [M, N] may alias y_f32.
+ *   X fp16 [M, K] (bits), W packed [N, K], A fp32 [r, K] / B fp32 [N, r] or both NULL,
+ *   Y fp32 [M, N] when y_f32 != NULL else fp16 bits into y_f16.  R fp32 [M, N] may alias y_f32.
  * mebp_linear_dx:   dX [M, K] = dY [M, N] deq(W) + s (dY B) A  (+ R if R != NULL)
- *   dY bf16 [M, N] (bits), same W / A / B, dX fp32 [M, K].
+ *   dY fp16 [M, N] (bits), same W / A / B, dX fp32 [M, K].
  * Both use the tcgen05 fused dequant-GEMM kernels; r <= 32. */
 int mebp_linear_fwd(mebp_ctx* ctx, const uint16_t* X, int64_t M, const mebp_packed* W,
                     const float* A, const float* B, int r, float s, const float* R,
-                    float* y_f32, uint16_t* y_bf16, void* stream);
+                    float* y_f32, uint16_t* y_f16, void* stream);
 int mebp_linear_dx(mebp_ctx* ctx, const uint16_t* dY, int64_t M, const mebp_packed* W,
                    const float* A, const float* B, int r, float s, const float* R,
                    float* dx, void* stream);

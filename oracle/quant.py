@@ -17,9 +17,9 @@ Storage: ``qpack[n, j] = u[n, 2j] | u[n, 2j+1] << 4`` (uint8 [rows, cols/2]) and
 ``scales[g, n]`` (fp16 [cols/64, rows], group-major).
 
 Decode: ``deq = q * s`` — exact in fp32 (a 4-bit integer times an 11-bit
-significand).  The GPU feeds its tensor cores ``bf16_rne(q * s)``; the function
-``dequant_bf16_bits`` states that value so the GPU's operand can be compared bit
-for bit.
+significand).  The GPU feeds its tensor cores the IEEE-half rounding
+``fp16_rne(q * s)``; the function ``dequant_f16_bits`` states that value so the GPU's
+operand can be compared bit for bit.
 
 The code and scale decisions are taken in fp32 because that is the precision
 the GPU kernel takes them in (a quantised code is an integer decided by
@@ -82,18 +82,12 @@ def dequant_rows(qpack: np.ndarray, scales: np.ndarray, rows: np.ndarray, group:
     return q * s
 
 
-def bf16_rne_bits(x: np.ndarray) -> np.ndarray:
-    """uint16 bit patterns of bf16 round-to-nearest-even of finite fp32 values."""
-    b = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
-    lsb = (b >> 16) & 1
-    return ((b + 0x7FFF + lsb) >> 16).astype(np.uint16)
+def dequant_f16_bits(qpack: np.ndarray, scales: np.ndarray, group: int = GROUP) -> np.ndarray:
+    """uint16 bits of fp16_rne(q * s) [rows, cols]: the tensor-core operand value
+    (numpy's float32 -> float16 conversion rounds to nearest, ties to even)."""
+    deq32 = unpack_codes(qpack).astype(np.float32) * row_scales(scales, group)
+    return deq32.astype(np.float16).view(np.uint16)
 
 
-def dequant_bf16_bits(qpack: np.ndarray, scales: np.ndarray, group: int = GROUP) -> np.ndarray:
-    """bf16 bits of bf16_rne(q * s) [rows, cols]: the tensor-core operand value."""
-    deq32 = (unpack_codes(qpack).astype(np.float32) * row_scales(scales, group))
-    return bf16_rne_bits(deq32)
-
-
-def bf16_bits_to_f64(bits: np.ndarray) -> np.ndarray:
-    return (bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+def f16_bits_to_f64(bits: np.ndarray) -> np.ndarray:
+    return np.ascontiguousarray(bits, np.uint16).view(np.float16).astype(np.float64)

@@ -1,5 +1,5 @@
 // Causal grouped-query attention of the decoder block, forward and backward, as tiled
-// warp-level tensor-core kernels (mma.sync m16n8k16, bf16 in / fp32 accumulate).
+// warp-level tensor-core kernels (mma.sync m16n8k16, fp16 in / fp32 accumulate).
 //
 //   forward : o = softmax(q k^T / sqrt(hd) + causal) v, per (sequence, query head); query head h
 //             reads key/value head h / (H/KV).  Saves lse = log-sum-exp of each score row.
@@ -60,10 +60,10 @@ __device__ __forceinline__ void pv_tile(float (&acc)[NC][4], const float (&p)[8]
 #pragma unroll
   for (int kq = 0; kq < 4; ++kq) {
     uint32_t a[4];
-    a[0] = pack_bf16x2(p[2 * kq][0], p[2 * kq][1]);
-    a[1] = pack_bf16x2(p[2 * kq][2], p[2 * kq][3]);
-    a[2] = pack_bf16x2(p[2 * kq + 1][0], p[2 * kq + 1][1]);
-    a[3] = pack_bf16x2(p[2 * kq + 1][2], p[2 * kq + 1][3]);
+    a[0] = pack_half2(p[2 * kq][0], p[2 * kq][1]);
+    a[1] = pack_half2(p[2 * kq][2], p[2 * kq][3]);
+    a[2] = pack_half2(p[2 * kq + 1][0], p[2 * kq + 1][1]);
+    a[3] = pack_half2(p[2 * kq + 1][2], p[2 * kq + 1][3]);
 #pragma unroll
     for (int dt = 0; dt < NC; dt += 2) {
       uint32_t b[4];
@@ -160,7 +160,7 @@ __global__ void __launch_bounds__(128, 1) fwd_kernel(const uint16_t* __restrict_
     uint16_t* orow = o + (tok0 + row) * ldo + h * HD;
 #pragma unroll
     for (int dt = 0; dt < NO; ++dt)
-      *reinterpret_cast<uint32_t*>(orow + dt * 8 + c) = pack_bf16x2(oacc[dt][2 * i] * inv, oacc[dt][2 * i + 1] * inv);
+      *reinterpret_cast<uint32_t*>(orow + dt * 8 + c) = pack_half2(oacc[dt][2 * i] * inv, oacc[dt][2 * i + 1] * inv);
     if ((lane & 3) == 0) lse[(static_cast<int64_t>(b) * H + h) * S + row] = (mrow[i] + log2f(lrow[i])) / kLog2e;
   }
 }
@@ -179,7 +179,7 @@ __global__ void dvec_kernel(const uint16_t* __restrict__ o, const uint16_t* __re
   float s = 0.0f;
   for (int i = lane; i < HD / 2; i += 32) {
     const uint32_t x = a[i], y = d[i];
-    s += bf16_lo(x) * bf16_lo(y) + bf16_hi(x) * bf16_hi(y);
+    s += h2_lo(x) * h2_lo(y) + h2_hi(x) * h2_hi(y);
   }
   s = warp_sum(s);
   if (lane == 0) {
@@ -278,8 +278,8 @@ __global__ void __launch_bounds__(128, 1) dkdv_kernel(const uint16_t* __restrict
     uint16_t* vrow = dqkv + (tok0 + key) * ld + (H + KV + kvh) * HD + d0;
 #pragma unroll
     for (int dt = 0; dt < NC; ++dt) {
-      *reinterpret_cast<uint32_t*>(krow + dt * 8 + c) = pack_bf16x2(dk[dt][2 * i] * inv, dk[dt][2 * i + 1] * inv);
-      *reinterpret_cast<uint32_t*>(vrow + dt * 8 + c) = pack_bf16x2(dv[dt][2 * i], dv[dt][2 * i + 1]);
+      *reinterpret_cast<uint32_t*>(krow + dt * 8 + c) = pack_half2(dk[dt][2 * i] * inv, dk[dt][2 * i + 1] * inv);
+      *reinterpret_cast<uint32_t*>(vrow + dt * 8 + c) = pack_half2(dv[dt][2 * i], dv[dt][2 * i + 1]);
     }
   }
 }
@@ -356,7 +356,7 @@ __global__ void __launch_bounds__(128, 1) dq_kernel(const uint16_t* __restrict__
     uint16_t* qrow = dqkv + (tok0 + row) * ld + h * HD + d0;
 #pragma unroll
     for (int dt = 0; dt < NC; ++dt)
-      *reinterpret_cast<uint32_t*>(qrow + dt * 8 + c) = pack_bf16x2(dq[dt][2 * i] * inv, dq[dt][2 * i + 1] * inv);
+      *reinterpret_cast<uint32_t*>(qrow + dt * 8 + c) = pack_half2(dq[dt][2 * i] * inv, dq[dt][2 * i + 1] * inv);
   }
 }
 

@@ -1,7 +1,6 @@
-// Shared device helpers: bf16 packing, bounded mbarrier waits, TMA and tcgen05 inline PTX.
+// Shared device helpers: fp16 packing, bounded mbarrier waits, TMA and tcgen05 inline PTX.
 #pragma once
 #include <cuda.h>
-#include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -31,19 +30,18 @@ MEBP_DEV uint64_t globaltimer_ns() {
 
 MEBP_DEV uint32_t smem_u32(const void* p) { return static_cast<uint32_t>(__cvta_generic_to_shared(p)); }
 
-MEBP_DEV uint32_t pack_bf16x2(float lo, float hi) {
-  // cvt.rn.bf16x2.f32 d, a, b puts a in the upper half, b in the lower half.
+// Tensor-core operands and stored activations are IEEE fp16 (kind::f16 runs fp16 and fp16 at
+// the same rate; fp16 keeps 3 more mantissa bits, see deq_consts in dequant.cuh).
+MEBP_DEV uint32_t pack_half2(float lo, float hi) {
+  // cvt.rn.f16x2.f32 d, a, b puts a in the upper half, b in the lower half.
   uint32_t r;
-  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
   return r;
 }
-
-MEBP_DEV float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
-MEBP_DEV float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
-MEBP_DEV float bf16_to_f(uint16_t v) { return __uint_as_float(static_cast<uint32_t>(v) << 16); }
-MEBP_DEV uint16_t f_to_bf16(float f) {
-  return __bfloat16_as_ushort(__float2bfloat16_rn(f));
-}
+MEBP_DEV float h2_lo(uint32_t v) { return __half2float(__ushort_as_half(static_cast<uint16_t>(v & 0xFFFFu))); }
+MEBP_DEV float h2_hi(uint32_t v) { return __half2float(__ushort_as_half(static_cast<uint16_t>(v >> 16))); }
+MEBP_DEV float h_to_f(uint16_t v) { return __half2float(__ushort_as_half(v)); }
+MEBP_DEV uint16_t f_to_h(float f) { return __half_as_ushort(__float2half_rn(f)); }
 
 // ------------------------------------------------------------------------------------ mbarrier
 MEBP_DEV void mbar_init(uint64_t* bar, uint32_t count) {
@@ -115,8 +113,8 @@ MEBP_DEV void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
 MEBP_DEV void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 MEBP_DEV void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
-// D[tmem] (+)= A[smem desc] * B[smem desc]^T, kind::f16 (bf16 inputs, fp32 accumulate).
-MEBP_DEV void tc_mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc, uint32_t accumulate) {
+// D[tmem] (+)= A[smem desc] * B[smem desc]^T, kind::f16 (fp16 inputs, fp32 accumulate).
+MEBP_DEV void tc_mma_f16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc, uint32_t accumulate) {
   asm volatile(
       "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
       "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
@@ -156,11 +154,11 @@ MEBP_DEV uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
   return d;
 }
 
-// Instruction descriptor, kind::f16 with bf16 A/B, fp32 D, dense.
-__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, bool b_mn_major) {
+// Instruction descriptor, kind::f16 with fp16 A/B, fp32 D, dense.
+__host__ __device__ constexpr uint32_t idesc_f16_f32(int M, int N, bool b_mn_major) {
   return (1u << 4)                        // D format f32
-         | (1u << 7)                      // A format bf16
-         | (1u << 10)                     // B format bf16
+         | (0u << 7)                      // A format f16
+         | (0u << 10)                     // B format f16
          | ((b_mn_major ? 1u : 0u) << 16) // B major-ness
          | (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(M >> 4) << 24);
 }

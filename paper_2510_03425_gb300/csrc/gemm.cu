@@ -7,7 +7,7 @@
 //
 // This is the decompression of Algorithm 1's LazyLoadAndDecompressWeights fused into the GEMM:
 // TMA brings the packed 4-bit tile and its fp16 scales into shared memory, eight converter
-// warps turn them into the bf16 operand (bit-exact bf16_rne(q*s), see dequant.cuh) in the
+// warps turn them into the fp16 operand (bit-exact fp16_rne(q*s), see dequant.cuh) in the
 // 128-byte-swizzled layout tcgen05 reads, one thread issues tcgen05.mma into a 128x256 fp32
 // TMEM accumulator, and the same eight warps run the epilogue out of TMEM.
 //
@@ -22,8 +22,8 @@ namespace mebp {
 namespace gemm {
 
 constexpr int BM = 128, BN = 256, BK = 64, STAGES = 3;
-constexpr int B_OFF = 0;                      // bf16 operand B: 256 x 64   = 32 KB
-constexpr int A_OFF = 32768;                  // bf16 operand A: 128 x 64   = 16 KB
+constexpr int B_OFF = 0;                      // fp16 operand B: 256 x 64   = 32 KB
+constexpr int A_OFF = 32768;                  // fp16 operand A: 128 x 64   = 16 KB
 constexpr int P_OFF = 49152;                  // packed nibbles            =  8 KB
 constexpr int S_OFF = 57344;                  // fp16 scales (256)         = 512 B
 constexpr int STAGE_STRIDE = 58368;           // 57 KB, multiple of 1024
@@ -41,6 +41,7 @@ struct Params {
   int64_t ldc;
   const float* R;      // fp32 residual / accumulation source (EPI_F32), may alias C
   int64_t ldr;
+  float alpha;         // EPI_F32: C = alpha * acc (+ R)
   // LM-head epilogues
   const int32_t* targets;  // [M]
   int col_offset;          // global vocabulary index of GEMM column 0
@@ -49,7 +50,7 @@ struct Params {
   int nparts;
   float* zt;               // EPI_LSE: target logit [M]
   const float* lse;        // EPI_CEGRAD: [M]
-  const float* inv_n;      // EPI_CEGRAD: device scalar 1 / N_valid
+  const float* ce_w;       // EPI_CEGRAD: device scalar weight of a valid row
   int* err;
 };
 
@@ -139,7 +140,7 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
   if (p.epi == EPI_CEGRAD) {
     const float lse = row_ok ? p.lse[row] : 0.0f;
     const int tgt = row_ok ? p.targets[row] : -1;
-    const float w = (tgt >= 0) ? *p.inv_n : 0.0f;
+    const float w = (tgt >= 0) ? *p.ce_w : 0.0f;
     const int tl = tgt - p.col_offset;
     uint16_t* C = static_cast<uint16_t*>(p.C);
 #pragma unroll 1
@@ -155,7 +156,7 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
         float b = (c0 + i + 1 < p.n_valid) ? __expf(v[i + 1] - lse) * w : 0.0f;
         if (c0 + i == tl) a -= w;
         if (c0 + i + 1 == tl) b -= w;
-        o[i / 2] = pack_bf16x2(a, b);
+        o[i / 2] = pack_half2(a, b);
       }
       uint4* dst = reinterpret_cast<uint4*>(C + static_cast<int64_t>(row) * p.ldc + c0);
 #pragma unroll
@@ -171,14 +172,14 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
     tmem_ld32(tbase + 32 * cc, v);
     const int c0 = cbase + 32 * cc;
     if (!row_ok || c0 >= p.N) continue;
-    if (p.epi == EPI_BF16) {
+    if (p.epi == EPI_F16) {
       uint16_t* C = static_cast<uint16_t*>(p.C);
       uint4* dst = reinterpret_cast<uint4*>(C + static_cast<int64_t>(row) * p.ldc + c0);
 #pragma unroll
       for (int i = 0; i < 4; ++i)
         if (c0 + 8 * i < p.N)
-          dst[i] = make_uint4(pack_bf16x2(v[8 * i], v[8 * i + 1]), pack_bf16x2(v[8 * i + 2], v[8 * i + 3]),
-                              pack_bf16x2(v[8 * i + 4], v[8 * i + 5]), pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
+          dst[i] = make_uint4(pack_half2(v[8 * i], v[8 * i + 1]), pack_half2(v[8 * i + 2], v[8 * i + 3]),
+                              pack_half2(v[8 * i + 4], v[8 * i + 5]), pack_half2(v[8 * i + 6], v[8 * i + 7]));
     } else {  // EPI_F32 (+ residual)
       float* C = static_cast<float*>(p.C);
       float4* dst = reinterpret_cast<float4*>(C + static_cast<int64_t>(row) * p.ldc + c0);
@@ -186,7 +187,8 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         if (c0 + 4 * i >= p.N) break;
-        float4 o = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+        float4 o = make_float4(p.alpha * v[4 * i], p.alpha * v[4 * i + 1], p.alpha * v[4 * i + 2],
+                               p.alpha * v[4 * i + 3]);
         if (res) {
           const float4 r = res[i];
           o.x += r.x; o.y += r.y; o.z += r.z; o.w += r.w;
@@ -278,7 +280,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   } else if (warp == 9) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, TRANS);
+      constexpr uint32_t idesc = idesc_f16_f32(BM, BN, TRANS);
       for (int it = 0; it < total; ++it) {
         const int s = it % STAGES;
         if (!mbar_wait(&full[s], mbar_phase(it), abort_flag, p.err)) break;
@@ -291,7 +293,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           const uint64_t ad = smem_desc_sw128(a_base + kk * 32, 16, 1024);
           const uint64_t bd = TRANS ? smem_desc_sw128(b_base + kk * 2048, 8192, 1024)
                                     : smem_desc_sw128(b_base + kk * 32, 16, 1024);
-          tc_mma_bf16(tmem, ad, bd, idesc, (it > 0 || kk > 0) ? 1u : 0u);
+          tc_mma_f16(tmem, ad, bd, idesc, (it > 0 || kk > 0) ? 1u : 0u);
         }
         tc_commit(&empty[s]);
       }
@@ -381,8 +383,8 @@ int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st) {
 
   CUtensorMap tA, tP, tS, tAx, tBx;
   int rc;
-  // A: bf16 [M, K], row pitch lda elements.
-  if ((rc = make_tmap_2d(&tA, g.A, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, g.K, g.M, g.lda * 2, 64, BM,
+  // A: fp16 [M, K], row pitch lda elements.
+  if ((rc = make_tmap_2d(&tA, g.A, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, g.K, g.M, g.lda * 2, 64, BM,
                          CU_TENSOR_MAP_SWIZZLE_128B)))
     return rc;
   if (!g.trans) {
@@ -405,15 +407,15 @@ int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st) {
   int kx_steps = 0;
   if (g.Ax && g.kx > 0) {
     kx_steps = (g.kx + 15) / 16;
-    if ((rc = make_tmap_2d(&tAx, g.Ax, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, g.kx, g.M, g.ldax * 2, 64, BM,
+    if ((rc = make_tmap_2d(&tAx, g.Ax, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, g.kx, g.M, g.ldax * 2, 64, BM,
                            CU_TENSOR_MAP_SWIZZLE_128B)))
       return rc;
     if (!g.trans) {
-      if ((rc = make_tmap_2d(&tBx, g.Bx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, g.kx, g.N, g.ldbx * 2, 64, BN,
+      if ((rc = make_tmap_2d(&tBx, g.Bx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, g.kx, g.N, g.ldbx * 2, 64, BN,
                              CU_TENSOR_MAP_SWIZZLE_128B)))
         return rc;
     } else {
-      if ((rc = make_tmap_2d(&tBx, g.Bx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, g.N, g.kx, g.ldbx * 2, 64, 64,
+      if ((rc = make_tmap_2d(&tBx, g.Bx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, g.N, g.kx, g.ldbx * 2, 64, 64,
                              CU_TENSOR_MAP_SWIZZLE_128B)))
         return rc;
     }
@@ -438,7 +440,8 @@ int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st) {
   p.nparts = g.nparts;
   p.zt = g.zt;
   p.lse = g.lse;
-  p.inv_n = g.inv_n;
+  p.ce_w = g.ce_w;
+  p.alpha = g.alpha;
   p.err = g.err;
   dim3 grid(static_cast<unsigned>((g.N + BN - 1) / BN), static_cast<unsigned>((g.M + BM - 1) / BM));
   count_launch();

@@ -12,26 +12,27 @@ namespace mebp {
 extern std::atomic<long long> g_launches;
 inline void count_launch(int n = 1) { g_launches.fetch_add(n, std::memory_order_relaxed); }
 
-enum GemmEpi { EPI_BF16 = 0, EPI_F32 = 1, EPI_LSE = 2, EPI_CEGRAD = 3 };
+enum GemmEpi { EPI_F16 = 0, EPI_F32 = 1, EPI_LSE = 2, EPI_CEGRAD = 3 };
 
 struct GemmArgs {
   bool trans = false;            // false: C = A deq(W)^T (W [N,K]);  true: C = A deq(W) (W [K,N])
-  const void* A = nullptr;       // bf16 [M, K]
+  const void* A = nullptr;       // fp16 [M, K]
   int64_t lda = 0;
   int64_t M = 0, N = 0, K = 0;
   const uint8_t* qpack = nullptr;
   const uint16_t* scales = nullptr;
   int64_t scale_pitch = 0;       // elements between consecutive scale rows (groups)
-  const void* Ax = nullptr;      // bf16 [M, kx] extra (LoRA) operand, or null
+  const void* Ax = nullptr;      // fp16 [M, kx] extra (LoRA) operand, or null
   int64_t ldax = 0;
   int64_t kx = 0;
-  const void* Bx = nullptr;      // FWD: bf16 [N, kx];  TRANS: bf16 [kx, N]
+  const void* Bx = nullptr;      // FWD: fp16 [N, kx];  TRANS: fp16 [kx, N]
   int64_t ldbx = 0;
-  int epi = EPI_BF16;
+  int epi = EPI_F16;
   void* C = nullptr;
   int64_t ldc = 0;
   const float* R = nullptr;
   int64_t ldr = 0;
+  float alpha = 1.0f;            // EPI_F32: C = alpha * acc (+ R)
   const int32_t* targets = nullptr;
   int col_offset = 0;
   int n_valid = 0;
@@ -39,7 +40,7 @@ struct GemmArgs {
   int nparts = 0;
   float* zt = nullptr;
   const float* lse = nullptr;
-  const float* inv_n = nullptr;
+  const float* ce_w = nullptr;   // EPI_CEGRAD: device scalar weight of a valid row
   int* err = nullptr;
 };
 
@@ -52,36 +53,44 @@ void launch_decode(const uint8_t* qpack, const uint16_t* scales, int64_t rows, i
 void launch_embed(const uint8_t* qpack, const uint16_t* scales, int64_t V, int64_t D, const int32_t* ids, int64_t T,
                   float* x0, int* err, cudaStream_t st);
 
-// RMSNorm: y_bf16 = x * rstd * g (rstd saved); backward: dx = resid + rstd (g dy) - x rstd^3/D sum(g dy x)
+// RMSNorm: y_f16 = x * rstd * g (rstd saved); backward: dx = resid + rstd (g dy) - x rstd^3/D sum(g dy x)
 void launch_rmsnorm_fwd(const float* x, const float* g, int64_t T, int D, float eps, uint16_t* y, float* rstd,
                         cudaStream_t st);
+// dx = (resid + ...) * (*out_mult) (out_mult may be null = 1); dx_h = fp16(resid + ...) (unmultiplied).
 void launch_rmsnorm_bwd(const float* dy, const float* x, const float* g, const float* rstd, const float* resid,
-                        int64_t T, int D, float* dx, uint16_t* dx_bf16, cudaStream_t st);
-// RoPE (half-split) on the q and k heads of a fused [T, (H+2KV)*hd] bf16 buffer, in place.
+                        int64_t T, int D, const float* out_mult, float* dx, uint16_t* dx_h, cudaStream_t st);
+// RoPE (half-split) on the q and k heads of a fused [T, (H+2KV)*hd] fp16 buffer, in place.
 void launch_rope(uint16_t* qkv, int64_t T, int S, int H, int KV, int hd, const float2* cs, bool inverse,
                  cudaStream_t st);
-// Gated MLP: m = act(g) * u from gu = [g | u] (bf16 [T, 2I]); backward writes dgu bf16 [T, 2I].
+// Gated MLP: m = act(g) * u from gu = [g | u] (fp16 [T, 2I]); backward writes dgu fp16 [T, 2I].
 void launch_glu_fwd(const uint16_t* gu, int64_t T, int I, int act, uint16_t* m, cudaStream_t st);
 void launch_glu_bwd(const float* dm, const uint16_t* gu, int64_t T, int I, int act, uint16_t* dgu, cudaStream_t st);
-void launch_cast_bf16(const float* x, int64_t n, uint16_t* y, cudaStream_t st);
+// y32 = x * (*scale), y16 = fp16(x * (*scale)); scale may be null (= 1), y32 may be null.
+void launch_scale_cast(const float* x, int64_t n, const float* scale, float* y32, uint16_t* y16, cudaStream_t st);
+// scal[0] = sigma = 2^-floor(log2(max|x|)) (1 if x == 0), scal[1] = 1/sigma; uses scal[2] as scratch.
+void launch_grad_scale(const float* x, int64_t n, float* scal, cudaStream_t st);
 void launch_fill_f32(float* x, int64_t n, float v, cudaStream_t st);
 
 // LM head helpers.
 void launch_lse_combine(const float* part, int nparts, const float* zt, const int32_t* targets, int64_t T,
                         float* lse, float* tok_loss, cudaStream_t st);
-void launch_loss_reduce(const float* tok_loss, const int32_t* targets, int64_t T, float* loss, float* inv_n,
+// loss = sum(tok_loss) / n_valid; scal[0] = sigma = 2^ceil(log2(n_valid)), scal[1] = 1/sigma,
+// scal[2] = sigma * kCeShift / n_valid (weight of a valid row of the scaled CE gradient).
+constexpr float kCeShift = 4096.0f;
+void launch_loss_reduce(const float* tok_loss, const int32_t* targets, int64_t T, float* loss, float* scal,
                         cudaStream_t st);
 
 // LoRA helpers.
-// out[m, j] = alpha * sum_k X[m, k] W[j, k]  (bf16 in, bf16 out with columns J..ldo-1 zeroed)
+// out[m, j] = alpha * sum_k X[m, k] W[j, k]  (fp16 in, fp16 out with columns J..ldo-1 zeroed)
 void launch_skinny_gemm(const uint16_t* X, int64_t ldx, int64_t M, int64_t K, const uint16_t* W, int64_t ldw, int J,
                         float alpha, uint16_t* out, int64_t ldo, cudaStream_t st);
 // C[p, q] (+)= sum_m P[m, p0 + p] Q[m, q0 + q], p < Pw, q < Qw; deterministic split over m.
+// The sum is multiplied by *mult (mult may be null = 1) before it is written / added.
 int launch_tall_reduce(const uint16_t* P, int64_t ldp, const uint16_t* Q, int64_t ldq, int64_t M, int Pw, int Qw,
-                       float* C, int64_t ldc, bool accumulate, float* scratch, int64_t scratch_floats,
-                       cudaStream_t st);
+                       float* C, int64_t ldc, bool accumulate, const float* mult, float* scratch,
+                       int64_t scratch_floats, cudaStream_t st);
 int64_t tall_reduce_scratch_floats(int64_t M, int Pw, int Qw);
-// bf16 shadows of the LoRA masters, see lora.cu.
+// fp16 shadows of the LoRA masters, see lora.cu.
 void launch_lora_shadow(const float* const* A, const float* const* B, int nt, const int* ranks_off,
                         const int* n_off, const int* n_len, int r, int K, int N, int kx, uint16_t* A_cat,
                         uint16_t* B_cat, uint16_t* Bt_cat, cudaStream_t st);

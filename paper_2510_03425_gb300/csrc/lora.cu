@@ -1,11 +1,11 @@
 // LoRA kernels (Section 3: only LoRA weights are trainable; the compressed base is frozen).
 //
 //  * skinny_gemm:  U_s = s * X A^T  (and dU = s * dY B) — the rank-r down-projections whose
-//    bf16 result feeds the fused GEMM's extra K-block.  HBM-bound on X.
+//    fp16 result feeds the fused GEMM's extra K-block.  HBM-bound on X.
 //  * tall_reduce:  dB = dY^T U_s and dA = dU^T X — reductions over all T tokens, done as
 //    warp-level tensor-core tiles over a token split, then summed in a fixed order
 //    (deterministic; no floating-point atomics).
-//  * lora_shadow:  bf16 operand copies of the fp32 masters, with the targets of a fused
+//  * lora_shadow:  fp16 operand copies of the fp32 masters, with the targets of a fused
 //    linear (q|k|v or gate|up) laid side by side along the rank axis:
 //      A_cat [kx, K]  rows ro_t .. ro_t+r-1 = A_t
 //      B_cat [N, kx]  block-diagonal: rows of target t, columns ro_t .. ro_t+r-1 = B_t
@@ -74,10 +74,10 @@ __global__ void __launch_bounds__(128) skinny_gemm_kernel(const uint16_t* __rest
   for (int nt = 0; nt < NT; ++nt) {
     const int col = nt * 8 + c;
     if (row0 < M)
-      *reinterpret_cast<uint32_t*>(out + row0 * ldo + col) = pack_bf16x2(alpha * acc[nt][0], alpha * acc[nt][1]);
+      *reinterpret_cast<uint32_t*>(out + row0 * ldo + col) = pack_half2(alpha * acc[nt][0], alpha * acc[nt][1]);
     if (row0 + 8 < M)
       *reinterpret_cast<uint32_t*>(out + (row0 + 8) * ldo + col) =
-          pack_bf16x2(alpha * acc[nt][2], alpha * acc[nt][3]);
+          pack_half2(alpha * acc[nt][2], alpha * acc[nt][3]);
   }
 }
 
@@ -167,14 +167,15 @@ __global__ void __launch_bounds__(128) tall_reduce_kernel(const uint16_t* __rest
   }
 }
 
-// C[p * sp + q * sq] (+)= sum_z part[z][p][q]  in split order.
+// C[p * sp + q * sq] (+)= mult * sum_z part[z][p][q]  in split order.
 __global__ void split_sum_kernel(const float* __restrict__ part, int splits, int Pw, int Qw, float* __restrict__ C,
-                                 int64_t sp, int64_t sq, int accumulate) {
+                                 int64_t sp, int64_t sq, int accumulate, const float* __restrict__ mult) {
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   const int64_t n = static_cast<int64_t>(Pw) * Qw;
   if (i >= n) return;
   float s = 0.0f;
   for (int z = 0; z < splits; ++z) s += part[z * n + i];
+  if (mult) s *= *mult;
   const int64_t p = i / Qw, q = i % Qw;
   float* dst = C + p * sp + q * sq;
   *dst = accumulate ? *dst + s : s;
@@ -188,8 +189,8 @@ int64_t tall_reduce_scratch_floats(int64_t M, int Pw, int Qw) {
 // C is written with strides (sp, sq) = (ldc, 1) for ldc > 0, and (1, -ldc) for ldc < 0
 // (transposed output).
 int launch_tall_reduce(const uint16_t* P, int64_t ldp, const uint16_t* Q, int64_t ldq, int64_t M, int Pw, int Qw,
-                       float* C, int64_t ldc, bool accumulate, float* scratch, int64_t scratch_floats,
-                       cudaStream_t st) {
+                       float* C, int64_t ldc, bool accumulate, const float* mult, float* scratch,
+                       int64_t scratch_floats, cudaStream_t st) {
   if (Pw <= 0 || Qw <= 0) return MEBP_OK;
   if ((Pw % 8) || (Qw % 8) || Qw > 96) return MEBP_ERR_UNSUPPORTED;
   const int nq = Qw <= 32 ? 4 : (Qw <= 64 ? 8 : 12);
@@ -211,7 +212,7 @@ int launch_tall_reduce(const uint16_t* P, int64_t ldp, const uint16_t* Q, int64_
   const int64_t sp = ldc > 0 ? ldc : 1, sq = ldc > 0 ? 1 : -ldc;
   count_launch();
   split_sum_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(scratch, static_cast<int>(splits), Pw, Qw,
-                                                                           C, sp, sq, accumulate ? 1 : 0);
+                                                                           C, sp, sq, accumulate ? 1 : 0, mult);
   return MEBP_OK;
 }
 
@@ -234,7 +235,7 @@ __global__ void lora_shadow_kernel(ShadowArgs a, int r, int K, int N, int kx, ui
     float v = 0.0f;
     for (int t = 0; t < a.nt; ++t)
       if (j >= a.ro[t] && j < a.ro[t] + r) v = a.A[t][static_cast<int64_t>(j - a.ro[t]) * K + k];
-    A_cat[i] = f_to_bf16(v);
+    A_cat[i] = f_to_h(v);
   }
   if (i < nb) {
     const int n = static_cast<int>(i / kx), j = static_cast<int>(i % kx);
@@ -242,7 +243,7 @@ __global__ void lora_shadow_kernel(ShadowArgs a, int r, int K, int N, int kx, ui
     for (int t = 0; t < a.nt; ++t)
       if (j >= a.ro[t] && j < a.ro[t] + r && n >= a.no[t] && n < a.no[t] + a.nl[t])
         v = a.B[t][static_cast<int64_t>(n - a.no[t]) * r + (j - a.ro[t])];
-    const uint16_t b = f_to_bf16(v);
+    const uint16_t b = f_to_h(v);
     B_cat[i] = b;
     Bt_cat[static_cast<int64_t>(j) * N + n] = b;
   }

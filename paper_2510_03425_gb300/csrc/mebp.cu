@@ -43,6 +43,10 @@ struct mebp_ctx {
   int device = 0;
   std::string err_msg = "ok";
   int* d_err = nullptr;
+  // device scalars: [0] sigma of the backward working scale, [1] 1/sigma, [2] CE row weight
+  // (all written by the loss reduction); [4] / [5] sigma / 1/sigma of a standalone block
+  // backward, [6] scratch.
+  float* scal = nullptr;
   int D = 0, H = 0, KV = 0, hd = 0, I = 0, V = 0, L = 0, Nqkv = 0, Na = 0, r = 0;
   float s = 1.0f;
   int64_t Tmax = 0;
@@ -58,13 +62,13 @@ struct mebp_ctx {
   uint16_t* du[4] = {nullptr, nullptr, nullptr, nullptr};
   uint16_t *A_cat[4] = {}, *B_cat[4] = {}, *Bt_cat[4] = {};
   // backward
-  uint16_t *dqkv = nullptr, *dout = nullptr, *dgu = nullptr, *dh1_bf = nullptr, *dy_bf[2] = {nullptr, nullptr};
+  uint16_t *dqkv = nullptr, *dout = nullptr, *dgu = nullptr, *dh1_h = nullptr, *dy_h[2] = {nullptr, nullptr};
   float *dm = nullptr, *dtmp = nullptr, *dh1 = nullptr, *dvec = nullptr, *gbuf[2] = {nullptr, nullptr};
   float* red = nullptr;
   int64_t red_floats = 0;
   // LM head
   uint16_t *hf = nullptr, *dz = nullptr;
-  float *rf = nullptr, *part = nullptr, *zt = nullptr, *lse_tok = nullptr, *tok_loss = nullptr, *inv_n = nullptr,
+  float *rf = nullptr, *part = nullptr, *zt = nullptr, *lse_tok = nullptr, *tok_loss = nullptr,
         *dhf = nullptr;
   int32_t* targets = nullptr;
   int nparts = 0, vchunk = 0;
@@ -215,7 +219,7 @@ int run_gemm(mebp_ctx* c, GemmArgs& g, cudaStream_t st, const char* what) {
   return MEBP_OK;
 }
 
-// bf16 shadows of one fused linear's LoRA masters.
+// fp16 shadows of one fused linear's LoRA masters.
 void build_shadow(mebp_ctx* c, int li, const mebp_lora* lora, cudaStream_t st) {
   const Lin& l = c->lin[li];
   if (!l.kx) return;
@@ -255,7 +259,7 @@ int block_forward(mebp_ctx* c, int layer, const mebp_block_weights* w, const meb
     launch_skinny_gemm(c->a, D, T, D, c->A_cat[LIN_QKV], D, lq.kx, c->s, c->us[LIN_QKV], lq.kxp, st);
     g.Ax = c->us[LIN_QKV]; g.ldax = lq.kxp; g.kx = lq.kxp; g.Bx = c->B_cat[LIN_QKV]; g.ldbx = lq.kxp;
   }
-  g.epi = EPI_BF16; g.C = c->qkv; g.ldc = lq.N;
+  g.epi = EPI_F16; g.C = c->qkv; g.ldc = lq.N;
   if ((rc = run_gemm(c, g, st, "qkv"))) return rc;
   launch_rope(c->qkv, T, Sq, c->H, c->KV, c->hd, c->rope_cs, false, st);
   launch_attn_fwd(c->qkv, lq.N, B, Sq, c->H, c->KV, c->hd, c->o, c->Na, c->lse_attn, st);
@@ -275,7 +279,7 @@ int block_forward(mebp_ctx* c, int layer, const mebp_block_weights* w, const meb
     launch_skinny_gemm(c->b, D, T, D, c->A_cat[LIN_GU], D, lg.kx, c->s, c->us[LIN_GU], lg.kxp, st);
     g.Ax = c->us[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = c->B_cat[LIN_GU]; g.ldbx = lg.kxp;
   }
-  g.epi = EPI_BF16; g.C = c->gu; g.ldc = lg.N;
+  g.epi = EPI_F16; g.C = c->gu; g.ldc = lg.N;
   if ((rc = run_gemm(c, g, st, "gate_up"))) return rc;
   launch_glu_fwd(c->gu, T, I, c->cfg.act, c->m, st);
   const Lin& ld = c->lin[LIN_DOWN];
@@ -296,30 +300,33 @@ int block_forward(mebp_ctx* c, int layer, const mebp_block_weights* w, const meb
 
 // LoRA gradients of one fused linear: dB_t = dY[:, rows_t]^T U_s[:, ranks_t], dA_t = dU[:, ranks_t]^T X.
 int lin_grads(mebp_ctx* c, int li, const uint16_t* dY, int64_t ldy, const uint16_t* X, int64_t ldx, int64_t T,
-              const mebp_lora_grads* grads, bool acc, cudaStream_t st) {
+              const mebp_lora_grads* grads, bool acc, const float* grad_mult, cudaStream_t st) {
   const Lin& l = c->lin[li];
   for (int t = 0; t < l.nt; ++t) {
     const int tg = l.tgt[t];
     if (!grads) break;
     if (grads->dB[tg]) {
       const int rc = launch_tall_reduce(dY + l.no[t], ldy, c->us[li] + l.ro[t], l.kxp, T, l.nl[t], c->r, grads->dB[tg],
-                                        c->r, acc, c->red, c->red_floats, st);
+                                        c->r, acc, grad_mult, c->red, c->red_floats, st);
       if (rc) return fail(c, rc, "LoRA dB reduction");
     }
     if (grads->dA[tg]) {
       const int rc = launch_tall_reduce(X, ldx, c->du[li] + l.ro[t], l.kxp, T, l.K, c->r, grads->dA[tg], -l.K, acc,
-                                        c->red, c->red_floats, st);
+                                        grad_mult, c->red, c->red_floats, st);
       if (rc) return fail(c, rc, "LoRA dA reduction");
     }
   }
   return MEBP_OK;
 }
 
-// dE/dx and LoRA grads of one block from its input checkpoint x and dE/dy.
-// dy_bf: bf16 copy of dy (or null -> made here).  dx / dx_bf may be null.
+// dE/dx and LoRA grads of one block from its input checkpoint x and dE/dy.  dy (fp32) and its
+// fp16 copy dy_h are in the backward's working scale sigma (a power of two that keeps the fp16
+// operands in range); the LoRA gradients are written times *grad_mult and dx times *dx_mult
+// (null = 1), so grad_mult = dx_mult = 1/sigma gives true gradients.  dx_h = fp16(sigma dE/dx).
+// dx / dx_h may be null.
 int block_backward(mebp_ctx* c, int layer, const mebp_block_weights* w, const mebp_lora* lora, const float* x,
-                   const float* dy, const uint16_t* dy_bf, float* dx, uint16_t* dx_bf, const mebp_lora_grads* grads,
-                   int B, int Sq, bool acc, cudaStream_t st) {
+                   const float* dy, const uint16_t* dy_h, float* dx, uint16_t* dx_h, const mebp_lora_grads* grads,
+                   int B, int Sq, bool acc, const float* grad_mult, const float* dx_mult, cudaStream_t st) {
   const int64_t T = static_cast<int64_t>(B) * Sq;
   const int D = c->D, I = c->I;
   int rc;
@@ -327,20 +334,16 @@ int block_backward(mebp_ctx* c, int layer, const mebp_block_weights* w, const me
     if ((rc = block_forward(c, layer, w, lora, x, nullptr, B, Sq, false, st))) return rc;
   }
   c->saved_layer = -1;  // the workspace is reused below
-  if (!dy_bf) {
-    launch_cast_bf16(dy, T * D, c->dy_bf[1], st);
-    dy_bf = c->dy_bf[1];
-  }
   // ---- down projection: y = h1 + m Wd^T (+ s (m Ad^T) Bd^T)
   const Lin& ld = c->lin[LIN_DOWN];
-  GemmArgs g = gemm_dx(dy_bf, D, T, w->down);
+  GemmArgs g = gemm_dx(dy_h, D, T, w->down);
   if (ld.kx) {
-    launch_skinny_gemm(dy_bf, D, T, D, c->Bt_cat[LIN_DOWN], D, ld.kx, c->s, c->du[LIN_DOWN], ld.kxp, st);
+    launch_skinny_gemm(dy_h, D, T, D, c->Bt_cat[LIN_DOWN], D, ld.kx, c->s, c->du[LIN_DOWN], ld.kxp, st);
     g.Ax = c->du[LIN_DOWN]; g.ldax = ld.kxp; g.kx = ld.kxp; g.Bx = c->A_cat[LIN_DOWN]; g.ldbx = I;
   }
   g.epi = EPI_F32; g.C = c->dm; g.ldc = I;
   if ((rc = run_gemm(c, g, st, "down dX"))) return rc;
-  if ((rc = lin_grads(c, LIN_DOWN, dy_bf, D, c->m, I, T, grads, acc, st))) return rc;
+  if ((rc = lin_grads(c, LIN_DOWN, dy_h, D, c->m, I, T, grads, acc, grad_mult, st))) return rc;
   // ---- gated MLP
   launch_glu_bwd(c->dm, c->gu, T, I, c->cfg.act, c->dgu, st);
   const Lin& lg = c->lin[LIN_GU];
@@ -351,19 +354,19 @@ int block_backward(mebp_ctx* c, int layer, const mebp_block_weights* w, const me
   }
   g.epi = EPI_F32; g.C = c->dtmp; g.ldc = D;
   if ((rc = run_gemm(c, g, st, "gate_up dX"))) return rc;
-  if ((rc = lin_grads(c, LIN_GU, c->dgu, 2 * I, c->b, D, T, grads, acc, st))) return rc;
+  if ((rc = lin_grads(c, LIN_GU, c->dgu, 2 * I, c->b, D, T, grads, acc, grad_mult, st))) return rc;
   // dh1 = dy + RMSNorm2^T(db)
-  launch_rmsnorm_bwd(c->dtmp, c->h1, w->norm2, c->r2, dy, T, D, c->dh1, c->dh1_bf, st);
+  launch_rmsnorm_bwd(c->dtmp, c->h1, w->norm2, c->r2, dy, T, D, nullptr, c->dh1, c->dh1_h, st);
   // ---- o projection
   const Lin& lo = c->lin[LIN_O];
-  g = gemm_dx(c->dh1_bf, D, T, w->o);
+  g = gemm_dx(c->dh1_h, D, T, w->o);
   if (lo.kx) {
-    launch_skinny_gemm(c->dh1_bf, D, T, D, c->Bt_cat[LIN_O], D, lo.kx, c->s, c->du[LIN_O], lo.kxp, st);
+    launch_skinny_gemm(c->dh1_h, D, T, D, c->Bt_cat[LIN_O], D, lo.kx, c->s, c->du[LIN_O], lo.kxp, st);
     g.Ax = c->du[LIN_O]; g.ldax = lo.kxp; g.kx = lo.kxp; g.Bx = c->A_cat[LIN_O]; g.ldbx = c->Na;
   }
-  g.epi = EPI_BF16; g.C = c->dout; g.ldc = c->Na;
+  g.epi = EPI_F16; g.C = c->dout; g.ldc = c->Na;
   if ((rc = run_gemm(c, g, st, "o dX"))) return rc;
-  if ((rc = lin_grads(c, LIN_O, c->dh1_bf, D, c->o, c->Na, T, grads, acc, st))) return rc;
+  if ((rc = lin_grads(c, LIN_O, c->dh1_h, D, c->o, c->Na, T, grads, acc, grad_mult, st))) return rc;
   // ---- attention, RoPE
   const Lin& lq = c->lin[LIN_QKV];
   launch_attn_bwd(c->qkv, lq.N, c->o, c->dout, c->Na, c->lse_attn, B, Sq, c->H, c->KV, c->hd, c->dvec, c->dqkv, st);
@@ -371,7 +374,7 @@ int block_backward(mebp_ctx* c, int layer, const mebp_block_weights* w, const me
   // ---- q, k, v projections
   if (lq.kx)
     launch_skinny_gemm(c->dqkv, lq.N, T, lq.N, c->Bt_cat[LIN_QKV], lq.N, lq.kx, c->s, c->du[LIN_QKV], lq.kxp, st);
-  if ((rc = lin_grads(c, LIN_QKV, c->dqkv, lq.N, c->a, D, T, grads, acc, st))) return rc;
+  if ((rc = lin_grads(c, LIN_QKV, c->dqkv, lq.N, c->a, D, T, grads, acc, grad_mult, st))) return rc;
   if (dx) {
     g = gemm_dx(c->dqkv, lq.N, T, w->qkv);
     if (lq.kx) {
@@ -379,13 +382,15 @@ int block_backward(mebp_ctx* c, int layer, const mebp_block_weights* w, const me
     }
     g.epi = EPI_F32; g.C = c->dtmp; g.ldc = D;
     if ((rc = run_gemm(c, g, st, "qkv dX"))) return rc;
-    launch_rmsnorm_bwd(c->dtmp, x, w->norm1, c->r1, c->dh1, T, D, dx, dx_bf, st);
+    launch_rmsnorm_bwd(c->dtmp, x, w->norm1, c->r1, c->dh1, T, D, dx_mult, dx, dx_h, st);
   }
   return cuda_check(c, "block backward");
 }
 
+// Final RMSNorm + LM head + CE.  dh (fp32) is the true gradient when unscale_dh, else it is
+// sigma * dloss/dh (the backward working scale, see loss_reduce_kernel); dh_h = fp16(sigma dloss/dh).
 int lmhead(mebp_ctx* c, const mebp_packed* E, const float* gf, const float* h, const int32_t* targets, int64_t T,
-           float* loss, float* dh, uint16_t* dh_bf, float* tok_loss, cudaStream_t st) {
+           float* loss, float* dh, uint16_t* dh_h, float* tok_loss, bool unscale_dh, cudaStream_t st) {
   const int D = c->D, V = c->V;
   int rc;
   launch_rmsnorm_fwd(h, gf, T, D, c->cfg.rms_eps, c->hf, c->rf, st);
@@ -395,7 +400,7 @@ int lmhead(mebp_ctx* c, const mebp_packed* E, const float* gf, const float* h, c
   if ((rc = run_gemm(c, g, st, "LM head (log-sum-exp pass)"))) return rc;
   float* tl = tok_loss ? tok_loss : c->tok_loss;
   launch_lse_combine(c->part, c->nparts, c->zt, targets, T, c->lse_tok, tl, st);
-  launch_loss_reduce(tl, targets, T, loss, c->inv_n, st);
+  launch_loss_reduce(tl, targets, T, loss, c->scal, st);
   for (int c0 = 0; c0 < V; c0 += c->vchunk) {
     const int n = std::min(c->vchunk, V - c0);
     mebp_packed Ec = *E;
@@ -405,16 +410,16 @@ int lmhead(mebp_ctx* c, const mebp_packed* E, const float* gf, const float* h, c
     g = gemm_fwd(c->hf, D, T, Ec, n, D);
     g.scale_pitch = V;
     g.epi = EPI_CEGRAD; g.C = c->dz; g.ldc = c->vchunk; g.targets = targets; g.col_offset = c0; g.n_valid = n;
-    g.lse = c->lse_tok; g.inv_n = c->inv_n;
+    g.lse = c->lse_tok; g.ce_w = c->scal + 2;
     if ((rc = run_gemm(c, g, st, "LM head (gradient pass)"))) return rc;
     GemmArgs t;
     t.trans = true;
     t.A = c->dz; t.lda = c->vchunk; t.M = T; t.N = D; t.K = n;
     t.qpack = Ec.qpack; t.scales = Ec.scales; t.scale_pitch = V;
-    t.epi = EPI_F32; t.C = c->dhf; t.ldc = D; t.R = c0 ? c->dhf : nullptr; t.ldr = D;
+    t.epi = EPI_F32; t.C = c->dhf; t.ldc = D; t.R = c0 ? c->dhf : nullptr; t.ldr = D; t.alpha = 1.0f / kCeShift;
     if ((rc = run_gemm(c, t, st, "LM head (dH pass)"))) return rc;
   }
-  launch_rmsnorm_bwd(c->dhf, h, gf, c->rf, nullptr, T, D, dh, dh_bf, st);
+  launch_rmsnorm_bwd(c->dhf, h, gf, c->rf, nullptr, T, D, unscale_dh ? c->scal + 1 : nullptr, dh, dh_h, st);
   return cuda_check(c, "LM head");
 }
 
@@ -483,6 +488,7 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
     if (rc == MEBP_OK) rc = dalloc(c, p, n);
   };
   A(&c->d_err, 4);
+  A(&c->scal, 8);
   A(&c->rope_cs, static_cast<int64_t>(f.max_seq) * (c->hd / 2));
   A(&c->a, T * D); A(&c->b, T * D); A(&c->qkv, T * c->Nqkv); A(&c->o, T * c->Na); A(&c->gu, T * 2 * I);
   A(&c->m, T * I); A(&c->r1, T); A(&c->r2, T); A(&c->lse_attn, T * c->H); A(&c->h1, T * D);
@@ -494,8 +500,8 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
     A(&c->B_cat[li], static_cast<int64_t>(l.N) * l.kxp);
     A(&c->Bt_cat[li], static_cast<int64_t>(l.N) * l.kxp);
   }
-  A(&c->dqkv, T * c->Nqkv); A(&c->dout, T * c->Na); A(&c->dgu, T * 2 * I); A(&c->dh1_bf, T * D);
-  A(&c->dy_bf[0], T * D); A(&c->dy_bf[1], T * D);
+  A(&c->dqkv, T * c->Nqkv); A(&c->dout, T * c->Na); A(&c->dgu, T * 2 * I); A(&c->dh1_h, T * D);
+  A(&c->dy_h[0], T * D); A(&c->dy_h[1], T * D);
   A(&c->dm, T * I); A(&c->dtmp, T * D); A(&c->dh1, T * D); A(&c->dvec, T * c->H);
   A(&c->gbuf[0], T * D); A(&c->gbuf[1], T * D);
   c->red_floats = std::max<int64_t>(tall_reduce_scratch_floats(T, std::max<int64_t>(2 * I, c->Nqkv), 32),
@@ -510,7 +516,7 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
     }
     c->vchunk = static_cast<int>(std::min<int64_t>(vc, (c->V + 255) / 256 * 256));
     A(&c->hf, T * D); A(&c->rf, T); A(&c->part, T * c->nparts * 2); A(&c->zt, T); A(&c->lse_tok, T);
-    A(&c->tok_loss, T); A(&c->inv_n, 4); A(&c->dz, T * c->vchunk); A(&c->dhf, T * D); A(&c->targets, T);
+    A(&c->tok_loss, T); A(&c->dz, T * c->vchunk); A(&c->dhf, T * D); A(&c->targets, T);
   }
   const int64_t nslots = f.spill_ckpts ? kCkptSlots : (c->L + 1);
   A(&c->ckpt, nslots * T * D);
@@ -544,6 +550,7 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
     cudaMemcpy(c->rope_cs, cs.data(), cs.size() * sizeof(float2), cudaMemcpyHostToDevice);
   }
   cudaMemset(c->d_err, 0, 16);
+  cudaMemset(c->scal, 0, 8 * sizeof(float));
   for (int li = 0; li < 4; ++li) {
     const Lin& l = c->lin[li];
     if (!l.kx) continue;
@@ -658,7 +665,7 @@ int mebp_embed(mebp_ctx* c, const mebp_packed* E, const int32_t* ids, int64_t n,
   return cuda_check(c, "embed");
 }
 
-// One standalone LoRA linear (uses stream-ordered temporaries for the bf16 shadows).
+// One standalone LoRA linear (uses stream-ordered temporaries for the fp16 shadows).
 static int linear_common(mebp_ctx* c, bool dx_mode, const uint16_t* X, int64_t M, const mebp_packed* W,
                          const float* A, const float* Bm, int r, float s, const float* R, float* y32, uint16_t* y16,
                          cudaStream_t st) {
@@ -699,7 +706,7 @@ static int linear_common(mebp_ctx* c, bool dx_mode, const uint16_t* X, int64_t M
     if (y32) {
       g.epi = EPI_F32; g.C = y32; g.ldc = N; g.R = R; g.ldr = N;
     } else {
-      g.epi = EPI_BF16; g.C = y16; g.ldc = N;
+      g.epi = EPI_F16; g.C = y16; g.ldc = N;
     }
   } else {
     g = gemm_dx(X, N, M, *W);
@@ -716,10 +723,10 @@ static int linear_common(mebp_ctx* c, bool dx_mode, const uint16_t* X, int64_t M
 }
 
 int mebp_linear_fwd(mebp_ctx* c, const uint16_t* X, int64_t M, const mebp_packed* W, const float* A, const float* B,
-                    int r, float s, const float* R, float* y_f32, uint16_t* y_bf16, void* stream) {
+                    int r, float s, const float* R, float* y_f32, uint16_t* y_f16, void* stream) {
   if (!c) return MEBP_ERR_INVALID_ARG;
-  if (!y_f32 && !y_bf16) return fail(c, MEBP_ERR_INVALID_ARG, "no output");
-  return linear_common(c, false, X, M, W, A, B, r, s, R, y_f32, y_bf16, S(stream));
+  if (!y_f32 && !y_f16) return fail(c, MEBP_ERR_INVALID_ARG, "no output");
+  return linear_common(c, false, X, M, W, A, B, r, s, R, y_f32, y_f16, S(stream));
 }
 
 int mebp_linear_dx(mebp_ctx* c, const uint16_t* dY, int64_t M, const mebp_packed* W, const float* A, const float* B,
@@ -749,7 +756,13 @@ int mebp_block_bwd(mebp_ctx* c, int layer, const mebp_block_weights* w, const me
   if ((rc = check_tokens(c, B, Sq)) || (rc = check_block_ptrs(c, w)) || (rc = check_lora(c, lora))) return rc;
   if (!x || !dy || !aligned16(x) || !aligned16(dy) || (dx && !aligned16(dx)))
     return fail(c, MEBP_ERR_INVALID_ARG, "x / dy / dx must be 16-byte aligned");
-  return block_backward(c, layer, w, lora, x, dy, nullptr, dx, nullptr, grads, B, Sq, accumulate != 0, S(stream));
+  cudaStream_t st = S(stream);
+  const int64_t n = static_cast<int64_t>(B) * Sq * c->D;
+  // working scale for this call: sigma = 2^-floor(log2(max|dy|)); the outputs are scaled back
+  launch_grad_scale(dy, n, c->scal + 4, st);
+  launch_scale_cast(dy, n, c->scal + 4, c->gbuf[0], c->dy_h[1], st);
+  return block_backward(c, layer, w, lora, x, c->gbuf[0], c->dy_h[1], dx, nullptr, grads, B, Sq, accumulate != 0,
+                        c->scal + 5, c->scal + 5, st);
 }
 
 int mebp_lmhead_ce_fwd_bwd(mebp_ctx* c, const mebp_packed* E, const float* gf, const float* h, const int32_t* targets,
@@ -761,7 +774,7 @@ int mebp_lmhead_ce_fwd_bwd(mebp_ctx* c, const mebp_packed* E, const float* gf, c
   if (!gf || !h || !targets || !loss || !dh) return fail(c, MEBP_ERR_INVALID_ARG, "NULL pointer");
   if (T <= 0 || T > c->Tmax) return fail(c, MEBP_ERR_INVALID_ARG, "n_tokens out of range");
   if (!aligned16(h) || !aligned16(dh)) return fail(c, MEBP_ERR_INVALID_ARG, "h / dh must be 16-byte aligned");
-  return lmhead(c, E, gf, h, targets, T, loss, dh, nullptr, token_loss, S(stream));
+  return lmhead(c, E, gf, h, targets, T, loss, dh, nullptr, token_loss, true, S(stream));
 }
 
 int mebp_lora_step(mebp_ctx* c, const mebp_model_weights* model, const mebp_lora* lora, const int32_t* ids, int B,
@@ -848,8 +861,8 @@ int mebp_lora_step(mebp_ctx* c, const mebp_model_weights* model, const mebp_lora
   // ---- loss subgraph: final norm + LM head + CE
   const float* hL = spill ? dev_ckpt(slot_of[L]) : dev_ckpt(L);
   int cur = 0;
-  if ((rc = lmhead(c, &model->embed, model->final_norm, hL, c->targets, T, loss, c->gbuf[cur], c->dy_bf[cur], nullptr,
-                   st)))
+  if ((rc = lmhead(c, &model->embed, model->final_norm, hL, c->targets, T, loss, c->gbuf[cur], c->dy_h[cur], nullptr,
+                   false, st)))
     return rc;
   if (spill) release(L);
   // ---- backward loop in reverse order: recompute block i from ckpt_i, apply its VJP
@@ -863,9 +876,9 @@ int mebp_lora_step(mebp_ctx* c, const mebp_model_weights* model, const mebp_lora
     }
     const float* xin = spill ? dev_ckpt(slot_of[i]) : dev_ckpt(i);
     const int nxt = cur ^ 1;
-    if ((rc = block_backward(c, i, &model->blocks[i], &lora[i], xin, c->gbuf[cur], c->dy_bf[cur],
-                             i > 0 ? c->gbuf[nxt] : nullptr, i > 0 ? c->dy_bf[nxt] : nullptr, &grads[i], B, Sq,
-                             accumulate != 0, st)))
+    if ((rc = block_backward(c, i, &model->blocks[i], &lora[i], xin, c->gbuf[cur], c->dy_h[cur],
+                             i > 0 ? c->gbuf[nxt] : nullptr, i > 0 ? c->dy_h[nxt] : nullptr, &grads[i], B, Sq,
+                             accumulate != 0, c->scal + 1, nullptr, st)))
       return rc;
     if (spill) {
       release(i);  // the checkpoint is removed once its backward has consumed it

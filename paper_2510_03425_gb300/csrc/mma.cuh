@@ -1,4 +1,4 @@
-// Warp-level bf16 tensor-core fragments (mma.sync m16n8k16) and cp.async helpers for the
+// Warp-level fp16 tensor-core fragments (mma.sync m16n8k16) and cp.async helpers for the
 // small contractions (LoRA down-projections, LoRA gradient reductions, attention tiles).
 #pragma once
 #include "common.cuh"
@@ -18,7 +18,7 @@ MEBP_DEV void ldsm_x4_t(uint32_t (&r)[4], uint32_t addr) {
 // d += a * b  (A 16x16 row-major, B 16x8 "col", fp32 accumulate)
 MEBP_DEV void mma16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
   asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
       "{%0, %1, %2, %3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));

@@ -2,13 +2,15 @@
 // forward/backward, casts, and the LM-head's log-sum-exp combine and loss reduction.
 // Every kernel streams rows with 16-byte vector accesses, one warp per row where a row
 // reduction is needed.
+#include <algorithm>
+
 #include "common.cuh"
 #include "kernels.h"
 
 namespace mebp {
 
 // ------------------------------------------------------------------------------------ RMSNorm
-// y = x / sqrt(mean(x^2) + eps) * g  ->  bf16 (the GEMM operand); rstd saved for the backward.
+// y = x / sqrt(mean(x^2) + eps) * g  ->  fp16 (the GEMM operand); rstd saved for the backward.
 __global__ void rmsnorm_fwd_kernel(const float* __restrict__ x, const float* __restrict__ g, int64_t T, int D,
                                    float eps, uint16_t* __restrict__ y, float* __restrict__ rstd) {
   const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
@@ -28,15 +30,15 @@ __global__ void rmsnorm_fwd_kernel(const float* __restrict__ x, const float* __r
   uint2* yr = reinterpret_cast<uint2*>(y + row * D);
   for (int i = lane; i < n4; i += 32) {
     const float4 v = xr[i], w = gr[i];
-    yr[i] = make_uint2(pack_bf16x2(v.x * r * w.x, v.y * r * w.y), pack_bf16x2(v.z * r * w.z, v.w * r * w.w));
+    yr[i] = make_uint2(pack_half2(v.x * r * w.x, v.y * r * w.y), pack_half2(v.z * r * w.z, v.w * r * w.w));
   }
 }
 
-// dx = resid + r (g*dy) - x r^3 / D * sum(g*dy*x)
+// v = resid + r (g*dy) - x r^3 / D * sum(g*dy*x);  dx = v * mult,  dxb = fp16(v)
 __global__ void rmsnorm_bwd_kernel(const float* __restrict__ dy, const float* __restrict__ x,
                                    const float* __restrict__ g, const float* __restrict__ rstd,
-                                   const float* __restrict__ resid, int64_t T, int D, float* __restrict__ dx,
-                                   uint16_t* __restrict__ dxb) {
+                                   const float* __restrict__ resid, int64_t T, int D, const float* __restrict__ mult,
+                                   float* __restrict__ dx, uint16_t* __restrict__ dxb) {
   const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (row >= T) return;
@@ -52,6 +54,7 @@ __global__ void rmsnorm_bwd_kernel(const float* __restrict__ dy, const float* __
   dot = warp_sum(dot);
   const float r = rstd[row];
   const float c = r * r * r * dot / static_cast<float>(D);
+  const float mu = mult ? *mult : 1.0f;
   const float4* rr = resid ? reinterpret_cast<const float4*>(resid + row * D) : nullptr;
   float4* outr = reinterpret_cast<float4*>(dx + row * D);
   uint2* outb = dxb ? reinterpret_cast<uint2*>(dxb + row * D) : nullptr;
@@ -63,8 +66,8 @@ __global__ void rmsnorm_bwd_kernel(const float* __restrict__ dy, const float* __
       const float4 q = rr[i];
       o.x += q.x; o.y += q.y; o.z += q.z; o.w += q.w;
     }
-    outr[i] = o;
-    if (outb) outb[i] = make_uint2(pack_bf16x2(o.x, o.y), pack_bf16x2(o.z, o.w));
+    if (outb) outb[i] = make_uint2(pack_half2(o.x, o.y), pack_half2(o.z, o.w));
+    outr[i] = make_float4(o.x * mu, o.y * mu, o.z * mu, o.w * mu);
   }
 }
 
@@ -75,11 +78,11 @@ void launch_rmsnorm_fwd(const float* x, const float* g, int64_t T, int D, float 
   rmsnorm_fwd_kernel<<<static_cast<unsigned>((T * 32 + 255) / 256), 256, 0, st>>>(x, g, T, D, eps, y, rstd);
 }
 void launch_rmsnorm_bwd(const float* dy, const float* x, const float* g, const float* rstd, const float* resid,
-                        int64_t T, int D, float* dx, uint16_t* dxb, cudaStream_t st) {
+                        int64_t T, int D, const float* out_mult, float* dx, uint16_t* dxb, cudaStream_t st) {
   if (T <= 0) return;
   count_launch();
-  rmsnorm_bwd_kernel<<<static_cast<unsigned>((T * 32 + 255) / 256), 256, 0, st>>>(dy, x, g, rstd, resid, T, D, dx,
-                                                                                   dxb);
+  rmsnorm_bwd_kernel<<<static_cast<unsigned>((T * 32 + 255) / 256), 256, 0, st>>>(dy, x, g, rstd, resid, T, D,
+                                                                                   out_mult, dx, dxb);
 }
 
 // ------------------------------------------------------------------------------------ RoPE
@@ -102,10 +105,10 @@ __global__ void rope_kernel(uint16_t* __restrict__ qkv, int64_t T, int S, int nh
   const float2 c0 = cs[static_cast<int64_t>(pos) * half + 2 * jp];
   const float2 c1 = cs[static_cast<int64_t>(pos) * half + 2 * jp + 1];
   const float sg = inverse ? -1.0f : 1.0f;
-  const float x1a = bf16_lo(a), x1b = bf16_hi(a), x2a = bf16_lo(b), x2b = bf16_hi(b);
+  const float x1a = h2_lo(a), x1b = h2_hi(a), x2a = h2_lo(b), x2b = h2_hi(b);
   const float s0 = sg * c0.y, s1 = sg * c1.y;
-  *p1 = pack_bf16x2(x1a * c0.x - x2a * s0, x1b * c1.x - x2b * s1);
-  *p2 = pack_bf16x2(x2a * c0.x + x1a * s0, x2b * c1.x + x1b * s1);
+  *p1 = pack_half2(x1a * c0.x - x2a * s0, x1b * c1.x - x2b * s1);
+  *p2 = pack_half2(x2a * c0.x + x1a * s0, x2b * c1.x + x1b * s1);
 }
 
 void launch_rope(uint16_t* qkv, int64_t T, int S, int H, int KV, int hd, const float2* cs, bool inverse,
@@ -147,7 +150,7 @@ __global__ void glu_fwd_kernel(const uint16_t* __restrict__ gu, int64_t T, int I
   uint32_t o[4];
 #pragma unroll
   for (int k = 0; k < 4; ++k)
-    o[k] = pack_bf16x2(act_f(bf16_lo(ga[k]), act) * bf16_lo(ua[k]), act_f(bf16_hi(ga[k]), act) * bf16_hi(ua[k]));
+    o[k] = pack_half2(act_f(h2_lo(ga[k]), act) * h2_lo(ua[k]), act_f(h2_hi(ga[k]), act) * h2_hi(ua[k]));
   *reinterpret_cast<uint4*>(m + t * I + c) = make_uint4(o[0], o[1], o[2], o[3]);
 }
 
@@ -168,9 +171,9 @@ __global__ void glu_bwd_kernel(const float* __restrict__ dm, const uint16_t* __r
   uint32_t og[4], ou[4];
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
-    const float g0 = bf16_lo(ga[k]), g1 = bf16_hi(ga[k]), u0 = bf16_lo(ua[k]), u1 = bf16_hi(ua[k]);
-    og[k] = pack_bf16x2(dd[2 * k] * u0 * act_grad(g0, act), dd[2 * k + 1] * u1 * act_grad(g1, act));
-    ou[k] = pack_bf16x2(dd[2 * k] * act_f(g0, act), dd[2 * k + 1] * act_f(g1, act));
+    const float g0 = h2_lo(ga[k]), g1 = h2_hi(ga[k]), u0 = h2_lo(ua[k]), u1 = h2_hi(ua[k]);
+    og[k] = pack_half2(dd[2 * k] * u0 * act_grad(g0, act), dd[2 * k + 1] * u1 * act_grad(g1, act));
+    ou[k] = pack_half2(dd[2 * k] * act_f(g0, act), dd[2 * k + 1] * act_f(g1, act));
   }
   *reinterpret_cast<uint4*>(dgu + t * 2 * I + c) = make_uint4(og[0], og[1], og[2], og[3]);
   *reinterpret_cast<uint4*>(dgu + t * 2 * I + I + c) = make_uint4(ou[0], ou[1], ou[2], ou[3]);
@@ -190,21 +193,51 @@ void launch_glu_bwd(const float* dm, const uint16_t* gu, int64_t T, int I, int a
 }
 
 // ------------------------------------------------------------------------------------ casts
-__global__ void cast_bf16_kernel(const float* __restrict__ x, int64_t n4, uint16_t* __restrict__ y) {
+__global__ void scale_cast_kernel(const float* __restrict__ x, int64_t n4, const float* __restrict__ scale,
+                                  float* __restrict__ y32, uint16_t* __restrict__ y16) {
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (i >= n4) return;
-  const float4 v = reinterpret_cast<const float4*>(x)[i];
-  reinterpret_cast<uint2*>(y)[i] = make_uint2(pack_bf16x2(v.x, v.y), pack_bf16x2(v.z, v.w));
+  const float sc = scale ? *scale : 1.0f;
+  float4 v = reinterpret_cast<const float4*>(x)[i];
+  v.x *= sc; v.y *= sc; v.z *= sc; v.w *= sc;
+  if (y32) reinterpret_cast<float4*>(y32)[i] = v;
+  reinterpret_cast<uint2*>(y16)[i] = make_uint2(pack_half2(v.x, v.y), pack_half2(v.z, v.w));
+}
+// max |x| into *amax_bits (as the bit pattern of a non-negative float; atomicMax on the
+// integer view is order independent, so the result is deterministic).
+__global__ void amax_kernel(const float* __restrict__ x, int64_t n, unsigned int* __restrict__ amax_bits) {
+  float m = 0.0f;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x)
+    m = fmaxf(m, fabsf(x[i]));
+  m = warp_max(m);
+  if ((threadIdx.x & 31) == 0) atomicMax(amax_bits, __float_as_uint(m));
+}
+// sigma = 2^-floor(log2(amax)) so that max|x * sigma| lies in [1, 2); 1 when amax is 0 or not finite.
+__global__ void sigma_kernel(float* scal) {
+  const float amax = __uint_as_float(reinterpret_cast<unsigned int*>(scal)[2]);
+  float sg = 1.0f;
+  if (amax > 0.0f && amax < INFINITY) sg = exp2f(-floorf(log2f(amax)));
+  scal[0] = sg;
+  scal[1] = 1.0f / sg;
+}
+void launch_scale_cast(const float* x, int64_t n, const float* scale, float* y32, uint16_t* y16, cudaStream_t st) {
+  const int64_t n4 = n / 4;
+  if (n4 <= 0) return;
+  count_launch();
+  scale_cast_kernel<<<static_cast<unsigned>((n4 + 255) / 256), 256, 0, st>>>(x, n4, scale, y32, y16);
+}
+void launch_grad_scale(const float* x, int64_t n, float* scal, cudaStream_t st) {
+  cudaMemsetAsync(scal + 2, 0, sizeof(float), st);
+  count_launch(2);
+  const int64_t blocks = std::min<int64_t>(1184, (n + 255) / 256);
+  amax_kernel<<<static_cast<unsigned>(std::max<int64_t>(1, blocks)), 256, 0, st>>>(
+      x, n, reinterpret_cast<unsigned int*>(scal + 2));
+  sigma_kernel<<<1, 1, 0, st>>>(scal);
 }
 __global__ void fill_kernel(float* __restrict__ x, int64_t n, float v) {
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (i < n) x[i] = v;
-}
-void launch_cast_bf16(const float* x, int64_t n, uint16_t* y, cudaStream_t st) {
-  const int64_t n4 = n / 4;
-  if (n4 <= 0) return;
-  count_launch();
-  cast_bf16_kernel<<<static_cast<unsigned>((n4 + 255) / 256), 256, 0, st>>>(x, n4, y);
 }
 void launch_fill_f32(float* x, int64_t n, float v, cudaStream_t st) {
   if (n <= 0) return;
@@ -238,9 +271,11 @@ __global__ void lse_combine_kernel(const float2* __restrict__ part, int nparts, 
   }
 }
 
-// loss = sum(tok_loss) / n_valid, inv_n = 1 / n_valid: one block, fixed reduction order.
+// loss = sum(tok_loss) / n_valid: one block, fixed reduction order.  Also the backward's
+// power-of-two working scale sigma = 2^ceil(log2(n_valid)) (the gradient of the mean loss times
+// sigma keeps fp16 operands in range), 1/sigma, and the CE-gradient row weight sigma*shift/n.
 __global__ void loss_reduce_kernel(const float* __restrict__ tok_loss, const int32_t* __restrict__ targets, int64_t T,
-                                   float* __restrict__ loss, float* __restrict__ inv_n) {
+                                   float* __restrict__ loss, float* __restrict__ scal) {
   __shared__ double ssum[1024];
   __shared__ int scnt[1024];
   double s = 0.0;
@@ -262,7 +297,11 @@ __global__ void loss_reduce_kernel(const float* __restrict__ tok_loss, const int
   if (threadIdx.x == 0) {
     const int n = scnt[0];
     *loss = n > 0 ? static_cast<float>(ssum[0] / n) : 0.0f;
-    *inv_n = n > 0 ? 1.0f / static_cast<float>(n) : 0.0f;
+    float sg = 1.0f;
+    while (sg < static_cast<float>(n)) sg *= 2.0f;
+    scal[0] = sg;
+    scal[1] = 1.0f / sg;
+    scal[2] = n > 0 ? static_cast<float>(static_cast<double>(sg) * kCeShift / n) : 0.0f;
   }
 }
 
@@ -273,10 +312,10 @@ void launch_lse_combine(const float* part, int nparts, const float* zt, const in
   lse_combine_kernel<<<static_cast<unsigned>((T * 32 + 255) / 256), 256, 0, st>>>(
       reinterpret_cast<const float2*>(part), nparts, zt, targets, T, lse, tok_loss);
 }
-void launch_loss_reduce(const float* tok_loss, const int32_t* targets, int64_t T, float* loss, float* inv_n,
+void launch_loss_reduce(const float* tok_loss, const int32_t* targets, int64_t T, float* loss, float* scal,
                         cudaStream_t st) {
   count_launch();
-  loss_reduce_kernel<<<1, 1024, 0, st>>>(tok_loss, targets, T, loss, inv_n);
+  loss_reduce_kernel<<<1, 1024, 0, st>>>(tok_loss, targets, T, loss, scal);
 }
 
 }  // namespace mebp

@@ -211,9 +211,9 @@ def mebp_embed(ctx, E: Packed, ids, x0, stream=None):
     _check(ctx, _lib.mebp_embed(ctx, ctypes.byref(E), _ptr(ids), ids.numel(), _ptr(x0), _stream(stream)))
 
 
-def mebp_linear_fwd(ctx, X, W: Packed, A=None, B=None, r=0, s=1.0, R=None, y_f32=None, y_bf16=None, stream=None):
+def mebp_linear_fwd(ctx, X, W: Packed, A=None, B=None, r=0, s=1.0, R=None, y_f32=None, y_f16=None, stream=None):
     _check(ctx, _lib.mebp_linear_fwd(ctx, _ptr(X), X.shape[0], ctypes.byref(W), _ptr(A), _ptr(B), r, s, _ptr(R),
-                                     _ptr(y_f32), _ptr(y_bf16), _stream(stream)))
+                                     _ptr(y_f32), _ptr(y_f16), _stream(stream)))
 
 
 def mebp_linear_dx(ctx, dY, W: Packed, A=None, B=None, r=0, s=1.0, R=None, dx=None, stream=None):

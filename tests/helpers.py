@@ -13,11 +13,9 @@ def rel_fro(a, b) -> float:
     return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-30))
 
 
-def bf16_round(x: np.ndarray) -> np.ndarray:
-    """Values of x rounded to bf16 (as float64), via torch's RNE conversion."""
-    import torch
-    t = torch.from_numpy(np.ascontiguousarray(x, np.float32)).to(torch.bfloat16)
-    return t.to(torch.float32).numpy().astype(np.float64)
+def f16_round(x: np.ndarray) -> np.ndarray:
+    """Values of x rounded to IEEE half (as float64)."""
+    return np.ascontiguousarray(x, np.float32).astype(np.float16).astype(np.float64)
 
 
 def to_gpu(x, dtype=None):
@@ -30,7 +28,7 @@ def to_gpu(x, dtype=None):
 
 def np_of(t):
     import torch
-    if t.dtype == torch.bfloat16:
+    if t.dtype in (torch.bfloat16, torch.float16):
         t = t.float()
     return t.detach().cpu().numpy()
 

@@ -20,7 +20,7 @@ if not torch.cuda.is_available():
 from paper_2510_03425_gb300 import mebp as M  # noqa: E402
 from paper_2510_03425_gb300.model import Context, DeviceBlock, LoraSet  # noqa: E402
 
-TOL = 2e-2  # relative Frobenius error of gradients (bf16 operands, fp32 accumulate)
+TOL = 2e-2  # relative Frobenius error of gradients (stated bound; fp16 operands, fp32 accumulate)
 
 
 def oracle_dense(W):

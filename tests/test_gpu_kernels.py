@@ -7,7 +7,7 @@ import pytest
 from oracle import quant
 from workload import synth
 
-from .helpers import bf16_round, np_of, rel_fro, to_gpu
+from .helpers import f16_round, np_of, rel_fro, to_gpu
 
 pytestmark = pytest.mark.gpu
 
@@ -21,7 +21,7 @@ from paper_2510_03425_gb300.model import Context, compress  # noqa: E402
 
 @pytest.fixture(scope="module")
 def ctx():
-    c = Context(synth.tiny(), max_tokens=4096, max_seq=64)
+    c = Context(synth.tiny(vocab=0, head_dim=64), max_tokens=4096, max_seq=64)
     yield c
     c.close()
 
@@ -50,7 +50,7 @@ def test_decode_bit_exact(ctx):
     out = torch.empty((320, 1024), dtype=torch.int16, device="cuda")
     M.mebp_decode_weights(ctx.handle, M.packed(to_gpu(qo), to_gpu(so)), out)
     ctx.sync()
-    np.testing.assert_array_equal(out.cpu().numpy().view(np.uint16), quant.dequant_bf16_bits(qo, so))
+    np.testing.assert_array_equal(out.cpu().numpy().view(np.uint16), quant.dequant_f16_bits(qo, so))
 
 
 def test_embedding_gather_exact(ctx):
@@ -82,37 +82,37 @@ SHAPES = [(200, 320, 192), (128, 256, 64), (1, 64, 64), (300, 1152, 896), (513, 
 
 def _x(M_, K, seed, scale=1.0):
     x = (np.random.default_rng(seed).standard_normal((M_, K)) * scale).astype(np.float32)
-    return bf16_round(x)
+    return f16_round(x)
 
 
 @pytest.mark.parametrize("Mr,N,K", SHAPES)
 def test_linear_fwd_matches_exact_operand_product(ctx, Mr, N, K):
-    """No LoRA: Y must equal X_bf16 . bf16(deq(W))^T up to fp32 accumulation."""
+    """No LoRA: Y must equal X_f16 . fp16(deq(W))^T up to fp32 accumulation."""
     W = _w(N, K, N + K)
     qo, so = quant.compress(W)
     X = _x(Mr, K, 1)
-    ref = X @ quant.bf16_bits_to_f64(quant.dequant_bf16_bits(qo, so)).T
-    Xg = to_gpu(X.astype(np.float32)).to(torch.bfloat16)
+    ref = X @ quant.f16_bits_to_f64(quant.dequant_f16_bits(qo, so)).T
+    Xg = to_gpu(X.astype(np.float32)).to(torch.float16)
     Wp = M.packed(to_gpu(qo), to_gpu(so))
     y = torch.empty((Mr, N), dtype=torch.float32, device="cuda")
-    yb = torch.empty((Mr, N), dtype=torch.bfloat16, device="cuda")
+    yb = torch.empty((Mr, N), dtype=torch.float16, device="cuda")
     M.mebp_linear_fwd(ctx.handle, Xg, Wp, y_f32=y)
-    M.mebp_linear_fwd(ctx.handle, Xg, Wp, y_bf16=yb)
+    M.mebp_linear_fwd(ctx.handle, Xg, Wp, y_f16=yb)
     ctx.sync()
     scale = np.abs(ref).max()
     assert np.abs(np_of(y) - ref).max() <= 2e-5 * scale + 1e-6
-    assert np.abs(np_of(yb) - ref).max() <= 8e-3 * scale + 1e-6
+    assert np.abs(np_of(yb) - ref).max() <= 1e-3 * scale + 1e-6
 
 
 @pytest.mark.parametrize("Mr,N,K", SHAPES)
 def test_linear_dx_matches_exact_operand_product(ctx, Mr, N, K):
-    """No LoRA: dX = dY_bf16 . bf16(deq(W)) up to fp32 accumulation (W is [N, K])."""
+    """No LoRA: dX = dY_f16 . fp16(deq(W)) up to fp32 accumulation (W is [N, K])."""
     W = _w(N, K, N + 2 * K)
     qo, so = quant.compress(W)
     dY = _x(Mr, N, 2)
-    ref = dY @ quant.bf16_bits_to_f64(quant.dequant_bf16_bits(qo, so))
+    ref = dY @ quant.f16_bits_to_f64(quant.dequant_f16_bits(qo, so))
     dx = torch.empty((Mr, K), dtype=torch.float32, device="cuda")
-    M.mebp_linear_dx(ctx.handle, to_gpu(dY.astype(np.float32)).to(torch.bfloat16), M.packed(to_gpu(qo), to_gpu(so)),
+    M.mebp_linear_dx(ctx.handle, to_gpu(dY.astype(np.float32)).to(torch.float16), M.packed(to_gpu(qo), to_gpu(so)),
                      dx=dx)
     ctx.sync()
     assert np.abs(np_of(dx) - ref).max() <= 2e-5 * np.abs(ref).max() + 1e-6
@@ -135,19 +135,19 @@ def test_linear_with_lora_against_oracle(ctx, r, Mr, N, K):
     Wp = M.packed(to_gpu(qo), to_gpu(so))
     y = torch.empty((Mr, N), dtype=torch.float32, device="cuda")
     Ag, Bg = to_gpu(A), to_gpu(B)
-    M.mebp_linear_fwd(ctx.handle, to_gpu(X.astype(np.float32)).to(torch.bfloat16), Wp, Ag, Bg, r, s, R=to_gpu(R), y_f32=y)
+    M.mebp_linear_fwd(ctx.handle, to_gpu(X.astype(np.float32)).to(torch.float16), Wp, Ag, Bg, r, s, R=to_gpu(R), y_f32=y)
     dY = _x(Mr, N, 4)
     ref_dx = dY @ Wd + s * (dY @ B.astype(np.float64)) @ A.astype(np.float64)
     dx = torch.empty((Mr, K), dtype=torch.float32, device="cuda")
-    M.mebp_linear_dx(ctx.handle, to_gpu(dY.astype(np.float32)).to(torch.bfloat16), Wp, Ag, Bg, r, s, dx=dx)
+    M.mebp_linear_dx(ctx.handle, to_gpu(dY.astype(np.float32)).to(torch.float16), Wp, Ag, Bg, r, s, dx=dx)
     ctx.sync()
-    assert rel_fro(np_of(y) - R, ref - R) < 1e-2
-    assert rel_fro(np_of(dx), ref_dx) < 1e-2
+    assert rel_fro(np_of(y) - R, ref - R) < 2e-3
+    assert rel_fro(np_of(dx), ref_dx) < 2e-3
     # the LoRA term itself is carried (not just the base product)
     base = X @ Wd.T
     lora_term = ref - R - base
     got_term = np_of(y).astype(np.float64) - R - base
-    assert rel_fro(got_term, lora_term) < 5e-2
+    assert rel_fro(got_term, lora_term) < 1e-2
 
 
 def test_lora_b_zero_is_bit_identical_to_base(ctx):
@@ -155,14 +155,14 @@ def test_lora_b_zero_is_bit_identical_to_base(ctx):
     W = _w(N, K, 21)
     qo, so = quant.compress(W)
     Wp = M.packed(to_gpu(qo), to_gpu(so))
-    X = to_gpu(_x(Mr, K, 5).astype(np.float32)).to(torch.bfloat16)
+    X = to_gpu(_x(Mr, K, 5).astype(np.float32)).to(torch.float16)
     A = to_gpu((np.random.default_rng(0).standard_normal((r, K)) * 0.1).astype(np.float32))
     B0 = torch.zeros((N, r), device="cuda")
     y0 = torch.empty((Mr, N), device="cuda")
     y1 = torch.empty((Mr, N), device="cuda")
     M.mebp_linear_fwd(ctx.handle, X, Wp, y_f32=y0)
     M.mebp_linear_fwd(ctx.handle, X, Wp, A, B0, r, 2.0, y_f32=y1)
-    dY = to_gpu(_x(Mr, N, 6).astype(np.float32)).to(torch.bfloat16)
+    dY = to_gpu(_x(Mr, N, 6).astype(np.float32)).to(torch.float16)
     d0 = torch.empty((Mr, K), device="cuda")
     d1 = torch.empty((Mr, K), device="cuda")
     M.mebp_linear_dx(ctx.handle, dY, Wp, dx=d0)
@@ -175,7 +175,7 @@ def test_lora_b_zero_is_bit_identical_to_base(ctx):
 def test_linear_rejects_bad_shapes(ctx):
     q = torch.zeros((64, 48), dtype=torch.uint8, device="cuda")   # cols = 96: not a multiple of 64
     s = torch.zeros((1, 64), dtype=torch.float16, device="cuda")
-    X = torch.zeros((4, 96), dtype=torch.bfloat16, device="cuda")
+    X = torch.zeros((4, 96), dtype=torch.float16, device="cuda")
     y = torch.empty((4, 64), device="cuda")
     with pytest.raises(M.MebpError) as ei:
         M.mebp_linear_fwd(ctx.handle, X, M.packed(q, s), y_f32=y)

@@ -39,7 +39,7 @@ def run(dims, T, chunk, ignore_every=7, h_scale=1.0, seed=0):
 
 @pytest.mark.parametrize("V,chunk,T", [(1088, 256, 100), (1088, 0, 100), (4096, 1024, 300), (64, 256, 5)])
 def test_lmhead_matches_oracle(V, chunk, T):
-    dims = synth.tiny(hidden=128, vocab=V)
+    dims = synth.tiny(hidden=128, head_dim=64, vocab=V)
     loss, dh, tok, lo, dho, toko, tg = run(dims, T, chunk)
     assert abs(loss - lo) < 1e-3
     np.testing.assert_allclose(tok, toko, atol=2e-3)
@@ -49,7 +49,7 @@ def test_lmhead_matches_oracle(V, chunk, T):
 
 
 def test_lmhead_chunking_does_not_change_the_result_beyond_rounding():
-    dims = synth.tiny(hidden=128, vocab=4096)
+    dims = synth.tiny(hidden=128, head_dim=64, vocab=4096)
     a = run(dims, 300, 256)
     b = run(dims, 300, 4096)
     assert abs(a[0] - b[0]) < 1e-5
@@ -57,7 +57,7 @@ def test_lmhead_chunking_does_not_change_the_result_beyond_rounding():
 
 
 def test_lmhead_uniform_logits_give_log_v():
-    dims = synth.tiny(hidden=64, vocab=512)
+    dims = synth.tiny(hidden=64, head_dim=64, vocab=512)
     T = 40
     ctx = Context(dims, max_tokens=T)
     Ep = PackedLinear(*compress(ctx, torch.zeros((512, 64), device="cuda")))

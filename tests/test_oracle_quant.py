@@ -1,7 +1,7 @@
 """Pins of the oracle's 4-bit compression (Section 3, 'Base model weights compression').
 
 The oracle is checked against a hand-worked example, the round-trip error
-bound, idempotence on its own decode, range facts and (for the bf16 operand
+bound, idempotence on its own decode, range facts and (for the fp16 operand
 value) torch's own round-to-nearest-even conversion.
 """
 import json
@@ -85,14 +85,16 @@ def test_scale_saturates_to_fp16_max():
     assert quant.unpack_codes(qpack)[0, 0] == 7     # clamped code
 
 
-def test_bf16_operand_bits_match_torch_rne():
+def test_f16_operand_bits_match_torch_rne():
     torch = pytest.importorskip("torch")
     W = _rand(16, 256, 11, std=0.5)
+    W[0, :64] *= 1e-6          # scales in the fp16 subnormal range
     qpack, scales = quant.compress(W)
-    bits = quant.dequant_bf16_bits(qpack, scales)
+    bits = quant.dequant_f16_bits(qpack, scales)
     deq32 = torch.from_numpy(quant.dequant(qpack, scales).astype(np.float32))
-    tb = deq32.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    tb = deq32.to(torch.float16).view(torch.int16).numpy().view(np.uint16)
     np.testing.assert_array_equal(bits, tb)
+    np.testing.assert_array_equal(quant.f16_bits_to_f64(bits), tb.view(np.float16).astype(np.float64))
 
 
 def test_rejects_ragged_groups():
