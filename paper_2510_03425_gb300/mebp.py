@@ -139,9 +139,12 @@ def _check(ctx, rc: int):
 
 
 def packed(qpack, scales) -> Packed:
+    """Descriptor of a compressed weight; it keeps the two tensors alive while it exists."""
     rows = qpack.shape[0]
     cols = qpack.shape[1] * 2
-    return Packed(_ptr(qpack), _ptr(scales), rows, cols)
+    p = Packed(_ptr(qpack), _ptr(scales), rows, cols)
+    p._keep = (qpack, scales)
+    return p
 
 
 def lora_struct(tensors: dict) -> Lora:
