@@ -51,8 +51,9 @@ def test_gemm_rows_at_full_size(name, N, K):
     dYr = np_of(dY[rows]).astype(np.float64)
     ref_y = Xr @ Wh.T
     ref_dx = dYr @ Wh
-    assert np.abs(np_of(Y[rows]) - ref_y).max() <= 2e-5 * np.abs(ref_y).max()
-    assert np.abs(np_of(dX[rows]) - ref_dx).max() <= 2e-5 * np.abs(ref_dx).max()
+    # fp32 accumulation over the reduction: the bound grows with sqrt(reduction length)
+    assert np.abs(np_of(Y[rows]) - ref_y).max() <= 2e-5 * max(1.0, np.sqrt(K / 2560)) * np.abs(ref_y).max()
+    assert np.abs(np_of(dX[rows]) - ref_dx).max() <= 2e-5 * max(1.0, np.sqrt(N / 2560)) * np.abs(ref_dx).max()
 
 
 @pytest.mark.parametrize("cfg", [2, 3, 4])
