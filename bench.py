@@ -270,6 +270,64 @@ def run_gpu(args, d, rank, world, local_rank):
     return out
 
 
+def gemm_bench(config: int, m_tokens=None, reps: int = 10, warmup: int = 3, shapes_only=None):
+    """The fused dequant-GEMMs alone (forward Y = X deq(W)^T and transposed dX = dY deq(W)) at
+    the four projection shapes of a workload, M = its token count.  Returns a dict."""
+    import torch
+
+    from paper_2510_03425_gb300 import mebp as M
+    from paper_2510_03425_gb300.model import Context, compress
+    d = synth.preset(config)
+    Mr = m_tokens or d.tokens
+    shapes = synth.linear_shapes(d)
+    mats = {"qkv": (shapes["q"][0] + 2 * shapes["k"][0], d.hidden), "o": shapes["o"],
+            "gate_up": (2 * d.intermediate, d.hidden), "down": shapes["down"]}
+    if shapes_only:
+        mats = {k: v for k, v in mats.items() if k in shapes_only}
+    ctx = Context(synth.tiny(vocab=0, head_dim=64), max_tokens=64, max_seq=64)
+    g = torch.Generator(device="cuda")
+    g.manual_seed(7)
+    res, tot_flops, tot_ms = {}, 0.0, 0.0
+    for name, (N, K) in mats.items():
+        W = torch.randn(N, K, device="cuda", generator=g) * 0.02
+        q, sc = compress(ctx, W)
+        del W
+        Wp = M.packed(q, sc)
+        X = torch.randn(Mr, K, device="cuda", generator=g).half()
+        Y = torch.empty(Mr, N, device="cuda", dtype=torch.float16)
+        dY = torch.randn(Mr, N, device="cuda", generator=g).half()
+        dX = torch.empty(Mr, K, device="cuda")
+        for mode in ("fwd", "dx"):
+            def f():
+                if mode == "fwd":
+                    M.mebp_linear_fwd(ctx.handle, X, Wp, y_f16=Y)
+                else:
+                    M.mebp_linear_dx(ctx.handle, dY, Wp, dx=dX)
+            for _ in range(warmup):
+                f()
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            for _ in range(reps):
+                f()
+            e1.record()
+            torch.cuda.synchronize()
+            ms = e0.elapsed_time(e1) / reps
+            fl = 2.0 * Mr * N * K
+            res[f"{name}_{mode}"] = {"M": Mr, "N": N if mode == "fwd" else K, "K": K if mode == "fwd" else N,
+                                     "us": 1e3 * ms, "tflops": fl / ms / 1e9}
+            tot_flops += fl
+            tot_ms += ms
+        del X, Y, dY, dX, q, sc, Wp
+    ctx.sync()
+    ctx.close()
+    pk, src = peaks()
+    tf = tot_flops / tot_ms / 1e9
+    return {"workload": f"projection GEMMs of {d.name}, M = {Mr} tokens, 4-bit g64 weights, fp16 operands",
+            "tflops": tf, "peak": pk["bf16_tflops"], "frac": tf / pk["bf16_tflops"],
+            "peak_source": f"{src} burst dense bf16 GEMM rate (fp16 shares it)", "per_gemm": res}
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -278,12 +336,22 @@ def main():
     ap.add_argument("--config", type=int, default=1, help="workload preset 0..4 (default 1)")
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--gemm-bench", action="store_true",
+                    help="time only the fused dequant-GEMMs at the config's projection shapes")
+    ap.add_argument("--gemm-m", type=int, default=None, help="token count M for --gemm-bench")
+    ap.add_argument("--gemm-shapes", default=None, help="comma list of qkv,o,gate_up,down for --gemm-bench")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     d = synth.preset(args.config)
+
+    if args.gemm_bench:
+        out = gemm_bench(args.config, args.gemm_m, reps=args.steps, warmup=args.warmup,
+                         shapes_only=args.gemm_shapes.split(",") if args.gemm_shapes else None)
+        print(json.dumps(out), flush=True)
+        return
 
     if args.impl == "reference":
         if rank != 0:
@@ -309,6 +377,9 @@ def main():
     out = run_gpu(args, d, rank, world, local_rank)
     if out is None:
         return
+    if world == 1:
+        # second half of the metric: the fused dequant-GEMM alone at the largest workload's shapes
+        out["fused_gemm_isolated"] = gemm_bench(4)
     if world == 1 and not args.no_cpu_baseline:
         v, desc = oracle_sample(d)
         out["cpu_baseline"] = {"value": v, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
