@@ -171,7 +171,9 @@ def run_gpu(args, d, rank, world, local_rank):
     loss = torch.zeros(1, device=device)
     loss_host = torch.zeros(1).pin_memory()
     mstruct = model.struct()
-    st = torch.cuda.current_stream(device)
+    # a dedicated stream: mebp_lora_step replays a captured CUDA graph on non-default streams
+    st = torch.cuda.Stream(device)
+    torch.cuda.set_stream(st)
 
     def step():
         M.mebp_lora_step(ctx.handle, mstruct, ls.lora_array(), ids, loss, ls.grads_array(), False, st)

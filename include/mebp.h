@@ -70,7 +70,9 @@ typedef struct {
  * A dense W [rows, cols] (cols % 64 == 0) quantised per group of 64 consecutive
  * columns of a row: s = fp16(min(amax/7, 65504)), q = clamp(rint(w/s), -7, 7),
  * stored as offset-binary nibbles u = q + 8:
- *   qpack  uint8 [rows, cols/2]: column 2j in the low nibble of byte j, 2j+1 in the high one;
+ *   qpack  uint8 [rows, cols/2]: every run of 8 columns is one little-endian 32-bit word with
+ *          column 8w+2j in bits 4j..4j+3 and column 8w+2j+1 in bits 16+4j..16+4j+3 (even
+ *          columns in the low half-word, odd ones in the high half-word);
  *   scales fp16 bits [cols/64, rows] (group-major: the scales of one column group are
  *          contiguous over rows).
  * deq(W)[n, k] = (u - 8) * scales[k/64, n]; the tensor cores consume fp16_rne(deq) (IEEE half).
@@ -189,7 +191,11 @@ int mebp_lmhead_ce_fwd_bwd(mebp_ctx* ctx, const mebp_packed* embed, const float*
 /* ---- Algorithm 1, Backpropagation(x): embed ids [batch, seq], forward loop storing only
  * block-boundary checkpoints (HBM, or pinned host when cfg.spill_ckpts), LM head + CE with
  * targets ids[b, s+1] (last position ignored), then the reverse loop of recompute + VJP.
- * lora / grads are HOST arrays of n_layers descriptors.  loss: device fp32 scalar. */
+ * lora / grads are HOST arrays of n_layers descriptors.  loss: device fp32 scalar.
+ * On a non-NULL stream (and unless disabled with mebp_enable_graphs) the step is replayed as
+ * a CUDA graph: the first call with a given set of pointers, sizes, stream and accumulate
+ * flag runs eagerly, the second captures the launch sequence, later ones replay it.  Data
+ * behind the pointers may change between calls; any pointer change re-captures. */
 int mebp_lora_step(mebp_ctx* ctx, const mebp_model_weights* model, const mebp_lora* lora,
                    const int32_t* ids, int batch, int seq, float* loss,
                    const mebp_lora_grads* grads, int accumulate, void* stream);
@@ -208,6 +214,8 @@ typedef struct {
   double dx_ms, dx_flops;
 } mebp_profile;
 int64_t mebp_kernel_launches(void);
+/* Turn CUDA-graph replay of mebp_lora_step on (default) or off; drops any captured graph. */
+int mebp_enable_graphs(mebp_ctx* ctx, int on);
 int mebp_profile_begin(mebp_ctx* ctx);
 int mebp_profile_end(mebp_ctx* ctx, mebp_profile* out);
 

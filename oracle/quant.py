@@ -13,8 +13,11 @@ For every row n of W [rows, cols] and every group g of 64 consecutive columns:
           = clamp(rint(w / s), -7, 7)         otherwise (fp32 division, ties to even)
     u     = q + 8                             (offset-binary nibble, 1..15)
 
-Storage: ``qpack[n, j] = u[n, 2j] | u[n, 2j+1] << 4`` (uint8 [rows, cols/2]) and
-``scales[g, n]`` (fp16 [cols/64, rows], group-major).
+Storage: ``qpack`` uint8 [rows, cols/2] holds each run of 8 consecutive columns in one
+little-endian 32-bit word, even columns in the low half-word and odd columns in the high
+half-word: element 8w + 2j sits in bits 4j..4j+3 of word w and element 8w + 2j + 1 in bits
+16 + 4j..16 + 4j + 3 (j = 0..3).  As bytes: (u0 | u2 << 4), (u4 | u6 << 4), (u1 | u3 << 4),
+(u5 | u7 << 4).  ``scales[g, n]`` (fp16 [cols/64, rows], group-major).
 
 Decode: ``deq = q * s`` — exact in fp32 (a 4-bit integer times an 11-bit
 significand).  The GPU feeds its tensor cores the IEEE-half rounding
@@ -38,7 +41,7 @@ def compress(W: np.ndarray, group: int = GROUP):
     """Quantise W (fp32 [rows, cols], cols % group == 0) -> (qpack uint8 [rows, cols/2], scales fp16 [cols/group, rows])."""
     W = np.ascontiguousarray(W, dtype=np.float32)
     rows, cols = W.shape
-    if cols % group or group % 2:
+    if cols % group or group % 8:
         raise ValueError("cols must be a multiple of the group size")
     Wg = W.reshape(rows, cols // group, group)
     amax = np.abs(Wg).max(axis=2)                                   # fp32
@@ -48,21 +51,23 @@ def compress(W: np.ndarray, group: int = GROUP):
         ratio = Wg / sf[:, :, None]                                 # fp32 division
     q = np.clip(np.rint(ratio), -QMAX, QMAX)
     q = np.where(sf[:, :, None] == 0, 0.0, q).astype(np.int8).reshape(rows, cols)
-    u = (q.astype(np.int16) + 8).astype(np.uint8)
-    qpack = (u[:, 0::2] | (u[:, 1::2] << 4)).astype(np.uint8)
+    u = (q.astype(np.int16) + 8).astype(np.uint8).reshape(rows, cols // 8, 8)
+    words = np.stack([u[:, :, 0] | (u[:, :, 2] << 4), u[:, :, 4] | (u[:, :, 6] << 4),
+                      u[:, :, 1] | (u[:, :, 3] << 4), u[:, :, 5] | (u[:, :, 7] << 4)], axis=2)
+    qpack = np.ascontiguousarray(words.reshape(rows, cols // 2)).astype(np.uint8)
     scales = np.ascontiguousarray(s16.T)                            # [cols/group, rows]
     return qpack, scales
 
 
 def unpack_codes(qpack: np.ndarray) -> np.ndarray:
     """Signed codes q (int8 [rows, cols]) from packed nibbles."""
-    lo = (qpack & 0x0F).astype(np.int16) - 8
-    hi = (qpack >> 4).astype(np.int16) - 8
     rows, half = qpack.shape
-    q = np.empty((rows, 2 * half), np.int8)
-    q[:, 0::2] = lo
-    q[:, 1::2] = hi
-    return q
+    b = qpack.reshape(rows, half // 4, 4).astype(np.int16)
+    u = np.empty((rows, half // 4, 8), np.int16)
+    for k, (lo, hi) in enumerate(((0, 2), (4, 6), (1, 3), (5, 7))):
+        u[:, :, lo] = b[:, :, k] & 0x0F
+        u[:, :, hi] = b[:, :, k] >> 4
+    return (u - 8).astype(np.int8).reshape(rows, 2 * half)
 
 
 def row_scales(scales: np.ndarray, group: int = GROUP) -> np.ndarray:

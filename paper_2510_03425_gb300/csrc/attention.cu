@@ -188,12 +188,16 @@ __global__ void dvec_kernel(const uint16_t* __restrict__ o, const uint16_t* __re
   }
 }
 
-// dK, dV for one key block of one kv head, output columns d0 .. d0 + DC.
+// dK, dV for one key block, output columns d0 .. d0 + DC.  Grouped mode (part == null): one CTA
+// per kv head loops over the query heads of its group and writes fp16 dK, dV.  Per-head mode
+// (small grids): blockIdx.y is a query head; the CTA writes its head's fp32 contribution to
+// part ([2][B*S][H][HD]: dK then dV) and dkdv_group_sum adds the heads of each group.
 template <int HD, int DC>
 __global__ void __launch_bounds__(128, 1) dkdv_kernel(const uint16_t* __restrict__ qkv, int64_t ld,
                                                       const uint16_t* __restrict__ dout, int64_t ldo,
                                                       const float* __restrict__ lse, const float* __restrict__ dvec,
-                                                      int S, int H, int KV, uint16_t* __restrict__ dqkv) {
+                                                      int S, int H, int KV, uint16_t* __restrict__ dqkv,
+                                                      float* __restrict__ part, int64_t T) {
   constexpr int LD = HD + 8, NC = DC / 8, NCH = HD / DC;
   extern __shared__ __align__(16) uint16_t sm[];
   uint16_t* ks = sm;
@@ -203,9 +207,12 @@ __global__ void __launch_bounds__(128, 1) dkdv_kernel(const uint16_t* __restrict
   float* lse_s = reinterpret_cast<float*>(dos + BQ * LD);
   float* dv_s = lse_s + BQ;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int kb = blockIdx.x, kvh = blockIdx.y;
-  const int b = blockIdx.z / NCH, d0 = (blockIdx.z % NCH) * DC;
   const int grp = H / KV;
+  const bool perhead = part != nullptr;
+  const int kb = blockIdx.x;
+  const int kvh = perhead ? blockIdx.y / grp : blockIdx.y;
+  const int h_first = perhead ? blockIdx.y : kvh * grp, h_count = perhead ? 1 : grp;
+  const int b = blockIdx.z / NCH, d0 = (blockIdx.z % NCH) * DC;
   const int64_t tok0 = static_cast<int64_t>(b) * S;
   const int k0 = kb * BKV;
   const float sc = kLog2e * rsqrtf(static_cast<float>(HD));
@@ -223,8 +230,8 @@ __global__ void __launch_bounds__(128, 1) dkdv_kernel(const uint16_t* __restrict
   const int key_a = k0 + warp * 16 + (lane >> 2);
   const int nqb = (S + BQ - 1) / BQ;
 
-  for (int hh = 0; hh < grp; ++hh) {
-    const int h = kvh * grp + hh;
+  for (int hh = 0; hh < h_count; ++hh) {
+    const int h = h_first + hh;
     for (int qb = kb; qb < nqb; ++qb) {
       const int q0 = qb * BQ;
       load_tile<HD>(qs, qkv, ld, tok0, q0, S, h * HD, tid);
@@ -270,6 +277,21 @@ __global__ void __launch_bounds__(128, 1) dkdv_kernel(const uint16_t* __restrict
   }
   const float inv = rsqrtf(static_cast<float>(HD));
   const int c = 2 * (lane & 3);
+  if (perhead) {
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int key = key_a + 8 * i;
+      if (key >= S) continue;
+      float* krow = part + ((tok0 + key) * H + h_first) * HD + d0;
+      float* vrow = krow + T * H * HD;
+#pragma unroll
+      for (int dt = 0; dt < NC; ++dt) {
+        *reinterpret_cast<float2*>(krow + dt * 8 + c) = make_float2(dk[dt][2 * i] * inv, dk[dt][2 * i + 1] * inv);
+        *reinterpret_cast<float2*>(vrow + dt * 8 + c) = make_float2(dv[dt][2 * i], dv[dt][2 * i + 1]);
+      }
+    }
+    return;
+  }
 #pragma unroll
   for (int i = 0; i < 2; ++i) {
     const int key = key_a + 8 * i;
@@ -374,9 +396,31 @@ void fwd_launch(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, ui
   fwd_kernel<HD><<<grid, 128, smem, st>>>(qkv, ld, S, H, KV, o, ldo, lse);
 }
 
+// dK, dV of kv head j = sum over the query heads of group j of the per-head partials (fixed order).
+__global__ void dkdv_group_sum(const float* __restrict__ part, int64_t T, int H, int KV, int HD, int64_t ld,
+                               uint16_t* __restrict__ dqkv) {
+  const int64_t n2 = T * KV * HD / 2;
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= 2 * n2) return;
+  const int which = i >= n2;  // 0: dK, 1: dV
+  const int64_t r = (which ? i - n2 : i) * 2;
+  const int d = static_cast<int>(r % HD);
+  const int j = static_cast<int>((r / HD) % KV);
+  const int64_t t = r / (static_cast<int64_t>(HD) * KV);
+  const int grp = H / KV;
+  const float* src = part + which * T * H * HD + (t * H + j * grp) * HD + d;
+  float a = 0.0f, b2 = 0.0f;
+  for (int hh = 0; hh < grp; ++hh) {
+    a += src[hh * HD];
+    b2 += src[hh * HD + 1];
+  }
+  *reinterpret_cast<uint32_t*>(dqkv + t * ld + (H + which * KV + j) * HD + d) = pack_half2(a, b2);
+}
+
 template <int HD, int DC>
 void bwd_launch(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t ldo, const float* lse,
-                const float* dvec, int B, int S, int H, int KV, uint16_t* dqkv, cudaStream_t st) {
+                const float* dvec, int B, int S, int H, int KV, uint16_t* dqkv, float* part, int64_t part_floats,
+                cudaStream_t st) {
   constexpr int smem = 4 * 64 * (HD + 8) * 2 + 2 * 64 * 4;
   static bool init = false;
   if (!init) {
@@ -385,9 +429,20 @@ void bwd_launch(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t l
     init = true;
   }
   constexpr int NCH = HD / DC;
-  dim3 g1((S + BKV - 1) / BKV, KV, B * NCH);
+  const int64_t T = static_cast<int64_t>(B) * S;
+  const int nkb = (S + BKV - 1) / BKV;
+  // One CTA per query head when one per kv head leaves most of the 152 SMs idle.
+  const bool perhead = H > KV && part && static_cast<int64_t>(nkb) * KV * B * NCH < 2 * 152 &&
+                       2 * T * H * HD <= part_floats;
+  dim3 g1(nkb, perhead ? H : KV, B * NCH);
   count_launch();
-  dkdv_kernel<HD, DC><<<g1, 128, smem, st>>>(qkv, ld, dout, ldo, lse, dvec, S, H, KV, dqkv);
+  dkdv_kernel<HD, DC><<<g1, 128, smem, st>>>(qkv, ld, dout, ldo, lse, dvec, S, H, KV, dqkv, perhead ? part : nullptr,
+                                             T);
+  if (perhead) {
+    const int64_t n = T * KV * HD;
+    count_launch();
+    dkdv_group_sum<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(part, T, H, KV, HD, ld, dqkv);
+  }
   dim3 g2((S + BQ - 1) / BQ, H, B * NCH);
   count_launch();
   dq_kernel<HD, DC><<<g2, 128, smem, st>>>(qkv, ld, dout, ldo, lse, dvec, S, H, KV, dqkv);
@@ -404,13 +459,14 @@ void launch_attn_fwd(const uint16_t* qkv, int64_t ld, int B, int S, int H, int K
 
 void launch_attn_bwd(const uint16_t* qkv, int64_t ld, const uint16_t* o, const uint16_t* dout, int64_t ldo,
                      const float* lse, int B, int S, int H, int KV, int hd, float* dvec, uint16_t* dqkv,
-                     cudaStream_t st) {
+                     float* part, int64_t part_floats, cudaStream_t st) {
   const int64_t nw = static_cast<int64_t>(B) * S * H;
   count_launch();
   attn::dvec_kernel<<<static_cast<unsigned>((nw * 32 + 255) / 256), 256, 0, st>>>(o, dout, ldo, B, S, H, hd, dvec);
-  if (hd == 64) attn::bwd_launch<64, 64>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, st);
-  else if (hd == 128) attn::bwd_launch<128, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, st);
-  else attn::bwd_launch<256, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, st);
+  if (hd == 64) attn::bwd_launch<64, 64>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, part, part_floats, st);
+  else if (hd == 128)
+    attn::bwd_launch<128, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, part, part_floats, st);
+  else attn::bwd_launch<256, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, part, part_floats, st);
 }
 
 }  // namespace mebp

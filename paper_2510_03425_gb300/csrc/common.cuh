@@ -31,7 +31,7 @@ MEBP_DEV uint64_t globaltimer_ns() {
 MEBP_DEV uint32_t smem_u32(const void* p) { return static_cast<uint32_t>(__cvta_generic_to_shared(p)); }
 
 // Tensor-core operands and stored activations are IEEE fp16 (kind::f16 runs fp16 and fp16 at
-// the same rate; fp16 keeps 3 more mantissa bits, see deq_consts in dequant.cuh).
+// the same rate; fp16 keeps 3 more mantissa bits).
 MEBP_DEV uint32_t pack_half2(float lo, float hi) {
   // cvt.rn.f16x2.f32 d, a, b puts a in the upper half, b in the lower half.
   uint32_t r;

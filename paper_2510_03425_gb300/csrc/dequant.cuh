@@ -1,59 +1,49 @@
 // Just-in-time decode of the 4-bit weight format into fp16 tensor-core operands.
 //
 // Format (Section 3, "Base model weights compression", read as symmetric INT4 with group 64
-// and fp16 scales): element k of a row sits in nibble k of the row's packed bytes
-// (low nibble = even k) as u = q + 8; deq = q * s, s = fp16 scale of the group.
+// and fp16 scales): u = q + 8 (offset binary).  Each run of 8 consecutive columns of a row is
+// one little-endian 32-bit word: column 8w + 2j in bits 4j..4j+3 (low half-word), column
+// 8w + 2j + 1 in bits 16 + 4j..16 + 4j + 3 (high half-word), j = 0..3.
 //
-// The operand must equal fp16_rne(q * s) bit for bit.  q * s is exact in fp32 (4-bit integer
-// times an 11-bit significand), so one correctly rounded FMA that reaches it exactly and one
-// RNE conversion give that value:
-//   m   = float_from_bits(0x3F800000 | (u << p)) = 1 + u * 2^(p-23)     (exact, p in {8,12,16})
-//   S_p = s * 2^(23-p),  C_p = -s * (2^(23-p) + 8)                      (both exact in fp32)
-//   fma(m, S_p, C_p) = s * 2^(23-p) + u*s - s * 2^(23-p) - 8s = (u - 8) s  (exact -> no rounding)
-// C_p is exact because 2^(23-p) + 8 has at most 13 significant bits for p >= 8 and s has 11.
-// Each nibble is moved into bit position 8, 12 or 16 with at most one shift per word.
+// The operand must equal fp16_rne(q * s) bit for bit.  With that word order one mask selects
+// an (even, odd) column pair already in operand order:
+//   t   = ((w >> 4j) & 0x000F000F) | 0x64006400    fp16 pair (1024 + u_2j, 1024 + u_2j+1), exact
+//   q   = t - (1032, 1032)                          exact small integers
+//   out = q * (s, s)                                one IEEE fp16 multiplication = fp16_rne(q * s)
+// i.e. 1 shift, 1 LOP3 and 2 half2 FP ops per two elements, and the scale is used as the
+// fp16 bits it is stored in.
 #pragma once
 #include "common.cuh"
 
 namespace mebp {
 
-struct DeqConsts {
-  float s8, c8, s12, c12, s16, c16;
-};
+// (s, s) as an fp16x2 register from the stored scale bits.
+MEBP_DEV uint32_t scale_pair(uint16_t s_bits) { return static_cast<uint32_t>(s_bits) * 0x00010001u; }
 
-MEBP_DEV DeqConsts deq_consts(float s) {
-  DeqConsts c;
-  c.s8 = s * 32768.0f;
-  c.c8 = -(s * 32776.0f);
-  c.s12 = s * 2048.0f;
-  c.c12 = -(s * 2056.0f);
-  c.s16 = s * 128.0f;
-  c.c16 = -(s * 136.0f);
-  return c;
+MEBP_DEV uint32_t hsub2_u32(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+MEBP_DEV uint32_t hmul2_u32(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("mul.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
 }
 
-MEBP_DEV float magic_nib(uint32_t w, uint32_t mask) { return __uint_as_float((w & mask) | 0x3F800000u); }
-
-// 8 nibbles of `w` (element i at bits 4i..4i+3) -> 4 fp16x2 words, element 2i in the low half
-// of out[i].
-MEBP_DEV void dequant_word(uint32_t w, const DeqConsts& c, uint32_t (&out)[4]) {
-  const uint32_t y = w << 8;   // nibbles 0,1 -> bits 8..11, 12..15
-  const uint32_t z = w >> 12;  // nibbles 5,6,7 -> bits 8..11, 12..15, 16..19
-  const float v0 = __fmaf_rn(magic_nib(y, 0x00000F00u), c.s8, c.c8);
-  const float v1 = __fmaf_rn(magic_nib(y, 0x0000F000u), c.s12, c.c12);
-  const float v2 = __fmaf_rn(magic_nib(w, 0x00000F00u), c.s8, c.c8);
-  const float v3 = __fmaf_rn(magic_nib(w, 0x0000F000u), c.s12, c.c12);
-  const float v4 = __fmaf_rn(magic_nib(w, 0x000F0000u), c.s16, c.c16);
-  const float v5 = __fmaf_rn(magic_nib(z, 0x00000F00u), c.s8, c.c8);
-  const float v6 = __fmaf_rn(magic_nib(z, 0x0000F000u), c.s12, c.c12);
-  const float v7 = __fmaf_rn(magic_nib(z, 0x000F0000u), c.s16, c.c16);
-  out[0] = pack_half2(v0, v1);
-  out[1] = pack_half2(v2, v3);
-  out[2] = pack_half2(v4, v5);
-  out[3] = pack_half2(v6, v7);
+// 8 nibbles of `w` -> 4 fp16x2 words: out[j] = (column 2j, column 2j+1) of the 8-column run.
+MEBP_DEV void dequant_word(uint32_t w, uint32_t s2, uint32_t (&out)[4]) {
+  constexpr uint32_t kMask = 0x000F000Fu, kMagic = 0x64006400u, kBias = 0x64086408u;  // 1024, 1032
+  out[0] = hmul2_u32(hsub2_u32((w & kMask) | kMagic, kBias), s2);
+  out[1] = hmul2_u32(hsub2_u32(((w >> 4) & kMask) | kMagic, kBias), s2);
+  out[2] = hmul2_u32(hsub2_u32(((w >> 8) & kMask) | kMagic, kBias), s2);
+  out[3] = hmul2_u32(hsub2_u32(((w >> 12) & kMask) | kMagic, kBias), s2);
 }
 
-// fp32 value of one element (used where the exact fp32 value is wanted, e.g. the embedding).
+// Nibble of column e (0..7) of a word, per the layout above.
+MEBP_DEV uint32_t word_nibble(uint32_t w, int e) { return (w >> ((e & 1) * 16 + (e >> 1) * 4)) & 0xFu; }
+
+// fp32 value of one element (the exact q * s, used by the embedding gather).
 MEBP_DEV float dequant_f32(uint32_t u, float s) { return static_cast<float>(static_cast<int>(u) - 8) * s; }
 
 }  // namespace mebp

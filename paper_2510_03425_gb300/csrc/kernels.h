@@ -41,6 +41,8 @@ struct GemmArgs {
   float* zt = nullptr;
   const float* lse = nullptr;
   const float* ce_w = nullptr;   // EPI_CEGRAD: device scalar weight of a valid row
+  float* split_ws = nullptr;     // fp32 workspace for split-K partial tiles (EPI_F32 / EPI_F16), or null
+  int64_t split_ws_floats = 0;
   int* err = nullptr;
 };
 
@@ -98,8 +100,9 @@ void launch_lora_shadow(const float* const* A, const float* const* B, int nt, co
 // Attention (causal GQA).  q/k/v live inside the fused qkv buffer (row pitch ld).
 void launch_attn_fwd(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, int hd, uint16_t* o, int64_t ldo,
                      float* lse, cudaStream_t st);
+// part: fp32 scratch (>= 2 * B*S * H * hd floats for the per-head dK/dV mode), may be null.
 void launch_attn_bwd(const uint16_t* qkv, int64_t ld, const uint16_t* o, const uint16_t* dout, int64_t ldo,
                      const float* lse, int B, int S, int H, int KV, int hd, float* dvec, uint16_t* dqkv,
-                     cudaStream_t st);
+                     float* part, int64_t part_floats, cudaStream_t st);
 
 }  // namespace mebp

@@ -66,6 +66,8 @@ struct mebp_ctx {
   float *dm = nullptr, *dtmp = nullptr, *dh1 = nullptr, *dvec = nullptr, *gbuf[2] = {nullptr, nullptr};
   float* red = nullptr;
   int64_t red_floats = 0;
+  float* split_ws = nullptr;   // split-K partial tiles of the fused GEMMs
+  int64_t split_ws_floats = 0;
   // LM head
   uint16_t *hf = nullptr, *dz = nullptr;
   float *rf = nullptr, *part = nullptr, *zt = nullptr, *lse_tok = nullptr, *tok_loss = nullptr,
@@ -78,6 +80,13 @@ struct mebp_ctx {
   cudaStream_t copy_stream = nullptr;
   cudaEvent_t slot_free[kCkptSlots] = {};
   cudaEvent_t slot_ready[kCkptSlots] = {};
+  // CUDA-graph replay of mebp_lora_step (key = every pointer and size the step depends on)
+  bool graphs = true;
+  std::vector<uintptr_t> graph_key;
+  cudaGraphExec_t graph_exec = nullptr;
+  long long graph_launches = 0;
+  int graph_eager_runs = 0;
+  cudaEvent_t copy_join = nullptr;
   // GEMM event profiling
   bool prof = false;
   std::vector<ProfRec> recs;
@@ -202,6 +211,8 @@ cudaEvent_t pool_event(mebp_ctx* c) {
 
 int run_gemm(mebp_ctx* c, GemmArgs& g, cudaStream_t st, const char* what) {
   g.err = c->d_err;
+  g.split_ws = c->split_ws;
+  g.split_ws_floats = c->split_ws_floats;
   ProfRec pr{};
   if (c->prof) {
     pr.a = pool_event(c);
@@ -369,7 +380,8 @@ int block_backward(mebp_ctx* c, int layer, const mebp_block_weights* w, const me
   if ((rc = lin_grads(c, LIN_O, c->dh1_h, D, c->o, c->Na, T, grads, acc, grad_mult, st))) return rc;
   // ---- attention, RoPE
   const Lin& lq = c->lin[LIN_QKV];
-  launch_attn_bwd(c->qkv, lq.N, c->o, c->dout, c->Na, c->lse_attn, B, Sq, c->H, c->KV, c->hd, c->dvec, c->dqkv, st);
+  launch_attn_bwd(c->qkv, lq.N, c->o, c->dout, c->Na, c->lse_attn, B, Sq, c->H, c->KV, c->hd, c->dvec, c->dqkv,
+                  c->split_ws, c->split_ws_floats, st);
   launch_rope(c->dqkv, T, Sq, c->H, c->KV, c->hd, c->rope_cs, true, st);
   // ---- q, k, v projections
   if (lq.kx)
@@ -507,6 +519,8 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
   c->red_floats = std::max<int64_t>(tall_reduce_scratch_floats(T, std::max<int64_t>(2 * I, c->Nqkv), 32),
                                     tall_reduce_scratch_floats(T, std::max<int64_t>(I, D), 32));
   A(&c->red, c->red_floats);
+  c->split_ws_floats = int64_t(16) << 20;
+  A(&c->split_ws, c->split_ws_floats);
   if (c->V > 0) {
     c->nparts = 2 * ((c->V + 255) / 256);
     int64_t vc = f.vocab_chunk;
@@ -532,6 +546,8 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
       if (cudaEventCreateWithFlags(&c->slot_free[i], cudaEventDisableTiming) != cudaSuccess ||
           cudaEventCreateWithFlags(&c->slot_ready[i], cudaEventDisableTiming) != cudaSuccess)
         rc = MEBP_ERR_CUDA;
+    if (rc == MEBP_OK && cudaEventCreateWithFlags(&c->copy_join, cudaEventDisableTiming) != cudaSuccess)
+      rc = MEBP_ERR_CUDA;
   }
   if (rc != MEBP_OK) {
     mebp_ctx_destroy(c);
@@ -571,6 +587,8 @@ void mebp_ctx_destroy(mebp_ctx* c) {
   cudaDeviceSynchronize();
   for (void* p : c->dev_allocs) cudaFree(p);
   for (cudaEvent_t e : c->evpool) cudaEventDestroy(e);
+  if (c->graph_exec) cudaGraphExecDestroy(c->graph_exec);
+  if (c->copy_join) cudaEventDestroy(c->copy_join);
   if (c->h_ckpt) cudaFreeHost(c->h_ckpt);
   for (int i = 0; i < kCkptSlots; ++i) {
     if (c->slot_free[i]) cudaEventDestroy(c->slot_free[i]);
@@ -600,6 +618,16 @@ int mebp_sync(mebp_ctx* c, void* stream) {
 }
 
 int64_t mebp_kernel_launches(void) { return g_launches.load(); }
+
+int mebp_enable_graphs(mebp_ctx* c, int on) {
+  if (!c) return MEBP_ERR_INVALID_ARG;
+  c->graphs = on != 0;
+  if (c->graph_exec) cudaGraphExecDestroy(c->graph_exec);
+  c->graph_exec = nullptr;
+  c->graph_key.clear();
+  c->graph_eager_runs = 0;
+  return MEBP_OK;
+}
 
 int mebp_profile_begin(mebp_ctx* c) {
   if (!c) return MEBP_ERR_INVALID_ARG;
@@ -777,17 +805,9 @@ int mebp_lmhead_ce_fwd_bwd(mebp_ctx* c, const mebp_packed* E, const float* gf, c
   return lmhead(c, E, gf, h, targets, T, loss, dh, nullptr, token_loss, true, S(stream));
 }
 
-int mebp_lora_step(mebp_ctx* c, const mebp_model_weights* model, const mebp_lora* lora, const int32_t* ids, int B,
-                   int Sq, float* loss, const mebp_lora_grads* grads, int accumulate, void* stream) {
-  if (!c) return MEBP_ERR_INVALID_ARG;
+static int lora_step_body(mebp_ctx* c, const mebp_model_weights* model, const mebp_lora* lora, const int32_t* ids,
+                          int B, int Sq, float* loss, const mebp_lora_grads* grads, int accumulate, void* stream) {
   int rc;
-  if (!model || !model->blocks || !lora || !ids || !loss) return fail(c, MEBP_ERR_INVALID_ARG, "NULL pointer");
-  if (c->V <= 0) return fail(c, MEBP_ERR_INVALID_ARG, "context has no vocabulary");
-  if ((rc = check_tokens(c, B, Sq))) return rc;
-  if ((rc = check_packed(c, &model->embed, c->V, c->D, "embedding"))) return rc;
-  if (!model->final_norm) return fail(c, MEBP_ERR_INVALID_ARG, "NULL final norm");
-  for (int i = 0; i < c->L; ++i)
-    if ((rc = check_block_ptrs(c, &model->blocks[i])) || (rc = check_lora(c, &lora[i]))) return rc;
   cudaStream_t st = S(stream);
   const int64_t T = static_cast<int64_t>(B) * Sq, D = c->D;
   const int L = c->L;
@@ -803,6 +823,9 @@ int mebp_lora_step(mebp_ctx* c, const mebp_model_weights* model, const mebp_lora
   for (int k = 0; k < kCkptSlots; ++k) holds[k] = -1;
   auto dev_ckpt = [&](int slot) { return c->ckpt + static_cast<int64_t>(slot) * c->Tmax * D; };
   auto host_ckpt = [&](int i) { return c->h_ckpt + static_cast<int64_t>(i) * c->Tmax * D; };
+  // Events recorded during THIS step only (a captured step must not wait on earlier events;
+  // work of earlier steps is already ordered before this one on the stream).
+  bool freed_rec[kCkptSlots] = {false, false, false};
   // A free slot, else the one holding the lowest-index checkpoint other than `avoid` (every
   // checkpoint below L also lives on the host, so evicting it loses nothing).
   auto take_slot = [&](int i, int avoid) {
@@ -828,6 +851,10 @@ int mebp_lora_step(mebp_ctx* c, const mebp_model_weights* model, const mebp_lora
     cudaStreamWaitEvent(c->copy_stream, c->slot_ready[sl], 0);
     cudaMemcpyAsync(host_ckpt(i), dev_ckpt(sl), T * D * sizeof(float), cudaMemcpyDeviceToHost, c->copy_stream);
     cudaEventRecord(c->slot_free[sl], c->copy_stream);
+    freed_rec[sl] = true;
+  };
+  auto wait_free = [&](int sl) {
+    if (freed_rec[sl]) cudaStreamWaitEvent(st, c->slot_free[sl], 0);
   };
   // host -> device copy of checkpoint i into a slot the main stream no longer reads
   auto fetch_in = [&](int i, int avoid) {
@@ -836,12 +863,13 @@ int mebp_lora_step(mebp_ctx* c, const mebp_model_weights* model, const mebp_lora
     cudaStreamWaitEvent(c->copy_stream, c->slot_ready[sl], 0);
     cudaMemcpyAsync(dev_ckpt(sl), host_ckpt(i), T * D * sizeof(float), cudaMemcpyHostToDevice, c->copy_stream);
     cudaEventRecord(c->slot_free[sl], c->copy_stream);
+    freed_rec[sl] = true;
   };
 
   float* x0 = dev_ckpt(0);
   if (spill) {
     const int sl = take_slot(0, -1);
-    cudaStreamWaitEvent(st, c->slot_free[sl], 0);
+    wait_free(sl);
     x0 = dev_ckpt(sl);
   }
   launch_embed(model->embed.qpack, model->embed.scales, c->V, D, ids, T, x0, c->d_err, st);
@@ -852,7 +880,7 @@ int mebp_lora_step(mebp_ctx* c, const mebp_model_weights* model, const mebp_lora
     float* yout = dev_ckpt(i + 1);
     if (spill) {
       const int sl = take_slot(i + 1, i);
-      cudaStreamWaitEvent(st, c->slot_free[sl], 0);  // its previous contents reached the host
+      wait_free(sl);  // its previous contents reached the host
       yout = dev_ckpt(sl);
     }
     if ((rc = block_forward(c, i, &model->blocks[i], &lora[i], xin, yout, B, Sq, true, st))) return rc;
@@ -870,7 +898,7 @@ int mebp_lora_step(mebp_ctx* c, const mebp_model_weights* model, const mebp_lora
     if (spill) {
       if (slot_of[i] < 0) {
         fetch_in(i, i + 1);
-        cudaStreamWaitEvent(st, c->slot_free[slot_of[i]], 0);
+        wait_free(slot_of[i]);
       }
       if (i > 0 && slot_of[i - 1] < 0) fetch_in(i - 1, i);  // prefetch while block i runs
     }
@@ -882,12 +910,86 @@ int mebp_lora_step(mebp_ctx* c, const mebp_model_weights* model, const mebp_lora
       return rc;
     if (spill) {
       release(i);  // the checkpoint is removed once its backward has consumed it
-      if (i > 0) cudaStreamWaitEvent(st, c->slot_free[slot_of[i - 1]], 0);
+      if (i > 0) wait_free(slot_of[i - 1]);
     }
     cur = nxt;
+  }
+  if (spill) {  // every copy of this step is complete when the stream reaches this point
+    cudaEventRecord(c->copy_join, c->copy_stream);
+    cudaStreamWaitEvent(st, c->copy_join, 0);
   }
   c->saved_layer = -1;
   return cuda_check(c, "lora step");
 }
+
+int mebp_lora_step(mebp_ctx* c, const mebp_model_weights* model, const mebp_lora* lora, const int32_t* ids, int B,
+                   int Sq, float* loss, const mebp_lora_grads* grads, int accumulate, void* stream) {
+  if (!c) return MEBP_ERR_INVALID_ARG;
+  int rc;
+  if (!model || !model->blocks || !lora || !ids || !loss) return fail(c, MEBP_ERR_INVALID_ARG, "NULL pointer");
+  if (c->V <= 0) return fail(c, MEBP_ERR_INVALID_ARG, "context has no vocabulary");
+  if ((rc = check_tokens(c, B, Sq))) return rc;
+  if ((rc = check_packed(c, &model->embed, c->V, c->D, "embedding"))) return rc;
+  if (!model->final_norm) return fail(c, MEBP_ERR_INVALID_ARG, "NULL final norm");
+  for (int i = 0; i < c->L; ++i)
+    if ((rc = check_block_ptrs(c, &model->blocks[i])) || (rc = check_lora(c, &lora[i]))) return rc;
+  cudaStream_t st = S(stream);
+  // CUDA-graph replay: the first call with a given set of pointers runs eagerly, the second
+  // captures the identical launch sequence, later calls replay it (values behind the
+  // pointers may change freely between calls).
+  std::vector<uintptr_t> key;
+  key.reserve(16 + static_cast<size_t>(c->L) * 40);
+  auto K = [&](const void* p) { key.push_back(reinterpret_cast<uintptr_t>(p)); };
+  K(stream); K(ids); K(loss); K(model->final_norm); K(model->embed.qpack); K(model->embed.scales);
+  key.push_back(static_cast<uintptr_t>(B)); key.push_back(static_cast<uintptr_t>(Sq));
+  key.push_back(static_cast<uintptr_t>(accumulate != 0));
+  for (int i = 0; i < c->L; ++i) {
+    const mebp_block_weights& w = model->blocks[i];
+    K(w.qkv.qpack); K(w.qkv.scales); K(w.o.qpack); K(w.o.scales); K(w.gate_up.qpack); K(w.gate_up.scales);
+    K(w.down.qpack); K(w.down.scales); K(w.norm1); K(w.norm2);
+    for (int t = 0; t < MEBP_N_TARGETS; ++t) {
+      K(lora[i].A[t]); K(lora[i].B[t]);
+      K(grads ? grads[i].dA[t] : nullptr); K(grads ? grads[i].dB[t] : nullptr);
+    }
+  }
+  const bool can_graph = c->graphs && stream != nullptr && !c->prof;
+  if (key != c->graph_key) {
+    if (c->graph_exec) cudaGraphExecDestroy(c->graph_exec);
+    c->graph_exec = nullptr;
+    c->graph_key = key;
+    c->graph_eager_runs = 0;
+  }
+  if (can_graph && c->graph_exec) {
+    if (cudaGraphLaunch(c->graph_exec, st) != cudaSuccess) return cuda_check(c, "graph launch");
+    g_launches.fetch_add(c->graph_launches);
+    return MEBP_OK;
+  }
+  if (can_graph && c->graph_eager_runs >= 1) {
+    const long long n0 = g_launches.load();
+    if (cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal) != cudaSuccess)
+      return cuda_check(c, "begin capture");
+    rc = lora_step_body(c, model, lora, ids, B, Sq, loss, grads, accumulate, stream);
+    cudaGraph_t graph = nullptr;
+    const cudaError_t ce = cudaStreamEndCapture(st, &graph);
+    if (rc != MEBP_OK || ce != cudaSuccess) {
+      if (graph) cudaGraphDestroy(graph);
+      cudaGetLastError();
+      return rc != MEBP_OK ? rc : fail(c, MEBP_ERR_CUDA, "stream capture of the step failed");
+    }
+    const cudaError_t ie = cudaGraphInstantiate(&c->graph_exec, graph, 0);
+    cudaGraphDestroy(graph);
+    if (ie != cudaSuccess) {
+      c->graph_exec = nullptr;
+      return cuda_check(c, "graph instantiate");
+    }
+    c->graph_launches = g_launches.load() - n0;  // kernels in the graph (counted once per replay)
+    if (cudaGraphLaunch(c->graph_exec, st) != cudaSuccess) return cuda_check(c, "graph launch");
+    return MEBP_OK;
+  }
+  rc = lora_step_body(c, model, lora, ids, B, Sq, loss, grads, accumulate, stream);
+  if (rc == MEBP_OK) c->graph_eager_runs++;
+  return rc;
+}
+
 
 }  // extern "C"

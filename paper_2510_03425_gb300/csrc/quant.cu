@@ -4,9 +4,11 @@
 
 namespace mebp {
 
-// One warp per (row, group of 64 columns).  Lane l handles columns 2l, 2l+1 and writes byte l.
+// One warp per (row, group of 64 columns).  Lane l writes byte l of the group: byte p of word
+// w = l/4 packs columns (c_lo, c_hi) = 8w + {(0,2), (4,6), (1,3), (5,7)}[p] as
+// (u_lo | u_hi << 4), the word layout of dequant.cuh.
 // s = fp16_satfinite_rne(amax / 7) (IEEE fp32 division), q = clamp(rint(w / s), -7, 7), q = 0
-// when s == 0; byte = (q0 + 8) | (q1 + 8) << 4.
+// when s == 0, u = q + 8.
 __global__ void compress_kernel(const float* __restrict__ W, int64_t rows, int64_t cols,
                                 uint8_t* __restrict__ qpack, uint16_t* __restrict__ scales) {
   const int64_t groups = cols / 64;
@@ -14,8 +16,12 @@ __global__ void compress_kernel(const float* __restrict__ W, int64_t rows, int64
   const int lane = threadIdx.x & 31;
   if (gw >= rows * groups) return;
   const int64_t r = gw / groups, g = gw % groups;
-  const float2 w = reinterpret_cast<const float2*>(W + r * cols + g * 64)[lane];
-  const float amax = warp_max(fmaxf(fabsf(w.x), fabsf(w.y)));
+  const float* grp = W + r * cols + g * 64;
+  const float2 pairv = reinterpret_cast<const float2*>(grp)[lane];  // columns 2l, 2l+1 for the max
+  const float amax = warp_max(fmaxf(fabsf(pairv.x), fabsf(pairv.y)));
+  const int wi = lane >> 2, pos = lane & 3;
+  const int c_lo = 8 * wi + ((pos & 1) ? 4 : 0) + ((pos & 2) ? 1 : 0);
+  const float2 w = make_float2(grp[c_lo], grp[c_lo + 2]);
   const float sq = __fdiv_rn(amax, 7.0f);
   uint16_t sbits;
   asm("cvt.rn.satfinite.f16.f32 %0, %1;" : "=h"(sbits) : "f"(sq));
@@ -29,7 +35,7 @@ __global__ void compress_kernel(const float* __restrict__ W, int64_t rows, int64
   if (lane == 0) scales[g * rows + r] = sbits;
 }
 
-// Decode every 8-element word with the GEMM's operand transform.
+// Decode every 8-column word with the GEMM's operand transform.
 __global__ void decode_kernel(const uint8_t* __restrict__ qpack, const uint16_t* __restrict__ scales, int64_t rows,
                               int64_t cols, uint16_t* __restrict__ out) {
   const int64_t words_per_row = cols / 8;
@@ -37,9 +43,8 @@ __global__ void decode_kernel(const uint8_t* __restrict__ qpack, const uint16_t*
   if (i >= rows * words_per_row) return;
   const int64_t r = i / words_per_row, j = i % words_per_row;
   const uint32_t w = reinterpret_cast<const uint32_t*>(qpack + r * (cols / 2))[j];
-  const float s = __half2float(__ushort_as_half(scales[(j / 8) * rows + r]));
   uint32_t o[4];
-  dequant_word(w, deq_consts(s), o);
+  dequant_word(w, scale_pair(scales[(j / 8) * rows + r]), o);
   reinterpret_cast<uint4*>(out + r * cols)[j] = make_uint4(o[0], o[1], o[2], o[3]);
 }
 
@@ -63,7 +68,7 @@ __global__ void embed_kernel(const uint8_t* __restrict__ qpack, const uint16_t* 
     const float s = __half2float(__ushort_as_half(scales[(j / 8) * V + id]));
     float v[8];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) v[e] = dequant_f32((w >> (4 * e)) & 0xFu, s);
+    for (int e = 0; e < 8; ++e) v[e] = dequant_f32(word_nibble(w, e), s);
     reinterpret_cast<float4*>(dst + j * 8)[0] = make_float4(v[0], v[1], v[2], v[3]);
     reinterpret_cast<float4*>(dst + j * 8)[1] = make_float4(v[4], v[5], v[6], v[7]);
   }

@@ -84,6 +84,7 @@ _SIGS = {
     "mebp_lmhead_ce_fwd_bwd": (c_int, [c_void_p, POINTER(Packed), c_void_p, c_void_p, c_void_p, c_int64, c_void_p,
                                        c_void_p, c_void_p, c_void_p]),
     "mebp_kernel_launches": (c_int64, []),
+    "mebp_enable_graphs": (c_int, [c_void_p, c_int]),
     "mebp_profile_begin": (c_int, [c_void_p]),
     "mebp_profile_end": (c_int, [c_void_p, POINTER(Profile)]),
     "mebp_lora_step": (c_int, [c_void_p, POINTER(ModelWeights), POINTER(Lora), c_void_p, c_int, c_int, c_void_p,
@@ -262,3 +263,7 @@ def mebp_profile_end(ctx) -> Profile:
     p = Profile()
     _check(ctx, _lib.mebp_profile_end(ctx, ctypes.byref(p)))
     return p
+
+
+def mebp_enable_graphs(ctx, on: bool = True):
+    _check(ctx, _lib.mebp_enable_graphs(ctx, int(on)))

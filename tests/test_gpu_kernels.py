@@ -77,7 +77,9 @@ def test_embedding_bad_id_flags_device_error(ctx):
     ctx.sync()  # the error word was cleared
 
 
-SHAPES = [(200, 320, 192), (128, 256, 64), (1, 64, 64), (300, 1152, 896), (513, 512, 1024)]
+# (M, N, K): ragged tiles, a single tile, split-K (small grids), and two-accumulator tiles (M >= 2048)
+SHAPES = [(200, 320, 192), (128, 256, 64), (1, 64, 64), (300, 1152, 896), (513, 512, 1024), (512, 896, 4864),
+          (2048, 256, 128), (2304 + 77, 576, 640)]
 
 
 def _x(M_, K, seed, scale=1.0):
@@ -119,7 +121,7 @@ def test_linear_dx_matches_exact_operand_product(ctx, Mr, N, K):
 
 
 @pytest.mark.parametrize("r", [8, 16, 32])
-@pytest.mark.parametrize("Mr,N,K", [(200, 320, 192), (300, 1152, 896)])
+@pytest.mark.parametrize("Mr,N,K", [(200, 320, 192), (300, 1152, 896), (2304 + 77, 576, 640)])
 def test_linear_with_lora_against_oracle(ctx, r, Mr, N, K):
     """Y = X deq(W)^T + s (X A^T) B^T (+R) and dX = dY deq(W) + s (dY B) A against fp64."""
     s = 2.0

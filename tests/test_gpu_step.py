@@ -107,3 +107,35 @@ def test_step_gradient_accumulation_doubles():
     for g0, g1 in zip(once, ls.grads):
         for n in g0:
             assert torch.equal(2 * g0[n][0], g1[n][0]) and torch.equal(2 * g0[n][1], g1[n][1])
+
+
+@pytest.mark.parametrize("spill", [False, True])
+def test_graph_replay_is_bit_identical_to_eager(spill):
+    """On a non-default stream the step is run eagerly once, captured on the second call and
+    replayed afterwards; every call must give the eager result bit for bit."""
+    dims, blocks, E, gf, loras, ids = _small()
+    idg = to_gpu(ids)
+    ctx, model = build(dims, blocks, E, gf, spill=spill)
+    ls = LoraSet(loras)
+    mstruct = model.struct()
+    loss = torch.zeros(1, device="cuda")
+    s = torch.cuda.Stream()
+    results = []
+    with torch.cuda.stream(s):
+        for _ in range(4):
+            n0 = M.mebp_kernel_launches()
+            M.mebp_lora_step(ctx.handle, mstruct, ls.lora_array(), idg, loss, ls.grads_array())
+            ctx.sync()
+            results.append((float(loss.item()), [{n: (a.clone(), b.clone()) for n, (a, b) in g.items()}
+                                                 for g in ls.grads], M.mebp_kernel_launches() - n0))
+    M.mebp_enable_graphs(ctx.handle, False)
+    with torch.cuda.stream(s):
+        M.mebp_lora_step(ctx.handle, mstruct, ls.lora_array(), idg, loss, ls.grads_array())
+        ctx.sync()
+    ref = (float(loss.item()), ls.grads)
+    for lo, gr, launches in results:
+        assert lo == ref[0]
+        assert launches == results[0][2]          # a replay counts the kernels it runs
+        for g0, g1 in zip(gr, ref[1]):
+            for n in g0:
+                assert torch.equal(g0[n][0], g1[n][0]) and torch.equal(g0[n][1], g1[n][1])

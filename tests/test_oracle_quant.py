@@ -29,16 +29,29 @@ def test_hand_worked_example():
     qpack, scales = quant.compress(W)
     assert qpack.shape == (2, 64) and scales.shape == (2, 2)
     assert scales.view(np.uint16).tolist() == g["scales_fp16_bits_group_major"]
-    assert qpack[0, :3].tolist() == g["qpack_row0_head"]
-    assert qpack[1, :3].tolist() == g["qpack_row1_head"]
-    assert qpack[1, 32:35].tolist() == g["qpack_row1_group1_head"]
+    assert qpack[0, :4].tolist() == g["qpack_row0_head"]
+    assert qpack[1, :4].tolist() == g["qpack_row1_head"]
+    assert qpack[1, 32:36].tolist() == g["qpack_row1_group1_head"]
     q = quant.unpack_codes(qpack)
     expect = np.zeros_like(q)
     for e in g["codes_nonzero"]:
         expect[e["row"], e["col"]] = e["q"]
     np.testing.assert_array_equal(q, expect)
     # every untouched byte is the zero code (u = 8 in both nibbles)
-    assert (qpack[0, 3:] == 0x88).all()
+    assert (qpack[0, 4:] == 0x88).all()
+
+
+def test_word_layout_is_even_columns_low_half_odd_columns_high_half():
+    """Element 8w+2j sits in bits 4j..4j+3 of little-endian word w, element 8w+2j+1 in bits 16+4j.."""
+    W = np.zeros((1, 64), np.float32)
+    W[0, :8] = [-7, -5, -3, -1, 1, 3, 5, 7]
+    W[0, 8] = 7.0
+    qpack, scales = quant.compress(W)
+    assert float(scales[0, 0]) == 1.0
+    word = int(qpack[0, :4].view("<u4")[0])
+    u = [(word >> (4 * j)) & 0xF for j in range(4)] + [(word >> (16 + 4 * j)) & 0xF for j in range(4)]
+    assert u == [1, 5, 9, 13, 3, 7, 11, 15]          # even columns 0,2,4,6 then odd 1,3,5,7
+    np.testing.assert_array_equal(quant.unpack_codes(qpack)[0, :8], [-7, -5, -3, -1, 1, 3, 5, 7])
 
 
 def _rand(rows, cols, seed, std=0.02):
