@@ -37,7 +37,9 @@ enum {
   MEBP_ERR_OOM = 3,          /* device or pinned-host allocation failed                          */
   MEBP_ERR_TIMEOUT = 4,      /* a device-side bounded wait expired (kernel returned early)       */
   MEBP_ERR_UNSUPPORTED = 5,  /* configuration outside what the kernels implement                 */
-  MEBP_ERR_DEVICE = 6        /* a kernel flagged bad input (e.g. token id out of range)          */
+  MEBP_ERR_DEVICE = 6,       /* a kernel flagged bad input (e.g. token id out of range)          */
+  MEBP_ERR_SCRATCH = 7       /* mebp_linear_fwd_noalloc: the request needs more than the fixed
+                                scratch array (MEBP_NOALLOC_SCRATCH_BYTES) holds                  */
 };
 
 /* LoRA target index (bit i of mebp_model_cfg.lora_targets). */
@@ -162,6 +164,27 @@ int mebp_linear_fwd(mebp_ctx* ctx, const uint16_t* X, int64_t M, const mebp_pack
 int mebp_linear_dx(mebp_ctx* ctx, const uint16_t* dY, int64_t M, const mebp_packed* W,
                    const float* A, const float* B, int r, float s, const float* R,
                    float* dx, void* stream);
+
+/* ---- mebp_linear_fwd without any device allocation (the paper has no counterpart; this is a
+ * deployment convenience).  For callers that may not call cudaMalloc/cudaFree at the point where
+ * the layer runs — e.g. a host program whose device memory belongs to an external pool, or code
+ * that must keep the process's allocations fixed — and so cannot create a mebp_ctx either.
+ * Same arguments and result as mebp_linear_fwd minus the context; the work runs on the device
+ * that is current when called.  Its scratch (the fp16 LoRA shadows, the rank-r product and an
+ * error word) lives in one static device array of MEBP_NOALLOC_SCRATCH_BYTES per GPU that loads
+ * the library, kept until the process exits:
+ *   - the first call on a device looks up that array's address (cudaGetSymbolAddress) and must
+ *     happen before any stream capture on that device;
+ *   - every call shares the array and leaves its contents behind: calls that can overlap on the
+ *     GPU (different streams without ordering) race on it;
+ *   - a request whose scratch (about 2 * (kx*K + 2*N*kx + M*kx) bytes, kx = r rounded up to 16;
+ *     none without LoRA) exceeds the array returns MEBP_ERR_SCRATCH before doing anything;
+ *   - device-side wait timeouts are not reported (there is no context to read them from).
+ * Allocates nothing: no cudaMalloc, cudaFree or allocating library call. */
+#define MEBP_NOALLOC_SCRATCH_BYTES (8u << 20)
+int mebp_linear_fwd_noalloc(const uint16_t* X, int64_t M, const mebp_packed* W, const float* A,
+                            const float* B, int r, float s, const float* R, float* y_f32,
+                            uint16_t* y_f16, void* stream);
 
 /* ---- forward_i of Algorithm 1: y [T, D] = F(x [T, D]) for block `layer`, T = batch*seq.
  * save_for_bwd != 0 keeps the block's intermediates in the context workspace so that a

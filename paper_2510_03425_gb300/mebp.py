@@ -17,7 +17,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "libmebp.so")
 HEADER = os.path.join(os.path.dirname(HERE), "include", "mebp.h")
 
-OK, ERR_INVALID_ARG, ERR_CUDA, ERR_OOM, ERR_TIMEOUT, ERR_UNSUPPORTED, ERR_DEVICE = range(7)
+OK, ERR_INVALID_ARG, ERR_CUDA, ERR_OOM, ERR_TIMEOUT, ERR_UNSUPPORTED, ERR_DEVICE, ERR_SCRATCH = range(8)
+NOALLOC_SCRATCH_BYTES = 8 << 20
 T_Q, T_K, T_V, T_O, T_GATE, T_UP, T_DOWN = range(7)
 TARGET_NAMES = ("q", "k", "v", "o", "gate", "up", "down")
 ACT = {"silu": 0, "gelu_tanh": 1}
@@ -83,6 +84,8 @@ _SIGS = {
                                POINTER(LoraGrads), c_int, c_int, c_int, c_void_p]),
     "mebp_lmhead_ce_fwd_bwd": (c_int, [c_void_p, POINTER(Packed), c_void_p, c_void_p, c_void_p, c_int64, c_void_p,
                                        c_void_p, c_void_p, c_void_p]),
+    "mebp_linear_fwd_noalloc": (c_int, [c_void_p, c_int64, POINTER(Packed), c_void_p, c_void_p, c_int, c_float,
+                                        c_void_p, c_void_p, c_void_p, c_void_p]),
     "mebp_kernel_launches": (c_int64, []),
     "mebp_enable_graphs": (c_int, [c_void_p, c_int]),
     "mebp_profile_begin": (c_int, [c_void_p]),
@@ -267,3 +270,11 @@ def mebp_profile_end(ctx) -> Profile:
 
 def mebp_enable_graphs(ctx, on: bool = True):
     _check(ctx, _lib.mebp_enable_graphs(ctx, int(on)))
+
+
+def mebp_linear_fwd_noalloc(X, W: Packed, A=None, B=None, r=0, s=1.0, R=None, y_f32=None, y_f16=None, stream=None):
+    """mebp_linear_fwd without a context or any device allocation (fixed static scratch)."""
+    rc = _lib.mebp_linear_fwd_noalloc(_ptr(X), X.shape[0], ctypes.byref(W), _ptr(A), _ptr(B), r, s, _ptr(R),
+                                      _ptr(y_f32), _ptr(y_f16), _stream(stream))
+    if rc != OK:
+        raise MebpError(rc, "mebp_linear_fwd_noalloc failed")
