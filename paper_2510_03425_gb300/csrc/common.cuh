@@ -163,6 +163,36 @@ __host__ __device__ constexpr uint32_t idesc_f16_f32(int M, int N, bool b_mn_maj
          | (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(M >> 4) << 24);
 }
 
+// ------------------------------------------------------------------------------------ clusters
+// Barrier over every thread of every CTA in the cluster; release/acquire orders the shared-memory
+// writes before it against the distributed-shared-memory reads after it.
+MEBP_DEV void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+}
+// Address of the same shared-memory location in CTA `rank` of this cluster.
+MEBP_DEV uint32_t dsmem_addr(uint32_t local, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
+  return r;
+}
+MEBP_DEV float4 ld_dsmem_f4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
+}
+
+// ------------------------------------------------------------------------------------ PDL
+// Programmatic dependent launch: a kernel launched with programmatic stream serialization may
+// start while its predecessor in the stream still runs.  griddep_wait() blocks until every
+// prerequisite grid has completed and its memory is visible (a no-op for a normal launch);
+// everything that reads a predecessor's output or writes memory a predecessor may read comes
+// after it.  griddep_launch() lets the dependents of this grid start early.
+MEBP_DEV void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+MEBP_DEV void griddep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // ------------------------------------------------------------------------------------ misc
 MEBP_DEV float warp_sum(float v) {
 #pragma unroll

@@ -14,8 +14,12 @@
 // CTA: 320 threads.  warps 0-7 convert + epilogue, warp 8 issues TMA, warp 9 issues MMA and
 // owns the TMEM allocation.  Tile (128*NACC) x 256 x 64: NACC 128-row A tiles share every
 // decoded 256-row B tile (NACC = 2 halves the decode work per flop and fills all 512 TMEM
-// columns).  3-stage smem ring.  Small grids split K over blockIdx.z into fp32 partial tiles
-// that a second kernel sums in a fixed order and finishes with the real epilogue.
+// columns).  Two shared-memory rings: a TMA ring (A tile(s) + packed nibbles + scales, with
+// separate barriers for the weight half and the activation half, so weights can be fetched and
+// decoded before the previous kernel has finished) and a ring of decoded B tiles written by the
+// converters (which also copy the LoRA B tile there).  Small grids split K over a thread-block
+// cluster along z and reduce the fp32 partial tiles through distributed shared memory
+// (deterministic, no workspace, no extra launch).
 #include <cudaTypedefs.h>
 
 #include <algorithm>
@@ -26,40 +30,48 @@
 namespace mebp {
 namespace gemm {
 
-constexpr int BM = 128, BN = 256, BK = 64, STAGES = 3, THREADS = 320;
+constexpr int BM = 128, BN = 256, BK = 64, THREADS = 320;
 constexpr int B_BYTES = BN * BK * 2, A_BYTES = BM * BK * 2, P_BYTES = BN * BK / 2, S_BYTES = 512;
 
-// Shared-memory stage layout for NACC accumulators (all tiles 1024-byte aligned).
+// Shared-memory layout for NACC accumulators (tiles 1024-byte aligned).
 template <int NACC>
 struct Layout {
-  static constexpr int B_OFF = 0;                                   // fp16 B: 256 x 64
-  static constexpr int A_OFF = B_BYTES;                             // fp16 A: NACC x 128 x 64
-  static constexpr int P_OFF = A_OFF + NACC * A_BYTES;              // packed nibbles
+  static constexpr int TSTG = NACC == 1 ? 4 : 3;                    // TMA ring depth
+  static constexpr int BSTG = NACC == 1 ? 3 : 2;                    // decoded-B ring depth
+  static constexpr int A_OFF = 0;                                   // fp16 A: NACC x 128 x 64
+  static constexpr int P_OFF = NACC * A_BYTES;                      // packed nibbles
   static constexpr int S_OFF = P_OFF + P_BYTES;                     // fp16 scales
-  static constexpr int STRIDE = (S_OFF + S_BYTES + 1023) / 1024 * 1024;
-  static constexpr int BAR_OFF = STAGES * STRIDE;
-  static constexpr int SMEM = BAR_OFF + 256 + 1024;                 // + barriers + alignment slack
+  static constexpr int T_STRIDE = (S_OFF + S_BYTES + 1023) / 1024 * 1024;
+  static constexpr int B_BASE = TSTG * T_STRIDE;                    // decoded fp16 B ring
+  static constexpr int BAR_OFF = B_BASE + BSTG * B_BYTES;
+  static constexpr int SMEM = BAR_OFF + 512 + 1024;                 // + barriers + alignment slack
   static constexpr uint32_t TMEM_COLS = 256 * NACC;
 };
-static_assert(Layout<2>::SMEM <= 232448, "shared memory budget");
-
-enum { EPI_PARTIAL = 100 };  // split-K: fp32 partial tile into Params::C + z * M * ldc
+static_assert(Layout<1>::SMEM <= 232448 && Layout<2>::SMEM <= 232448, "shared memory budget");
+// One CTA per SM (no two GEMM CTAs ever share an SM's TMEM), and the split-K partial tile fits in
+// the idle rings.
+static_assert(Layout<1>::SMEM > 232448 / 2 && Layout<2>::SMEM > 232448 / 2, "one CTA per SM");
+static_assert(Layout<1>::BAR_OFF >= BM * BN * 4, "partial tile fits below the barriers");
 
 struct Params {
   int M, N, K;
   int kx_steps;        // 16-wide MMA steps of the extra (LoRA) block; 0 = none
+  int kx;              // LoRA block width (columns of A_x / B_x, multiple of 16)
+  const uint16_t* Bx;  // LoRA B operand (FWD [N, kx], TRANS [kx, N]), row pitch ldbx
+  int64_t ldbx;
   int kt_split;        // main 64-wide K tiles per split (blockIdx.z)
-  int epi;             // GemmEpi or EPI_PARTIAL
+  int epi;             // GemmEpi
   void* C;
   int64_t ldc;
   const float* R;      // fp32 residual / accumulation source (EPI_F32), may alias C
   int64_t ldr;
   float alpha;         // EPI_F32: C = alpha * acc (+ R)
+  int w_ready;         // packed weights are not written by any kernel that may still run
   // LM-head epilogues
   const int32_t* targets;  // [M]
   int col_offset;          // global vocabulary index of GEMM column 0
   int n_valid;             // GEMM columns >= n_valid are outside the vocabulary
-  float* part;             // EPI_LSE: float2 [M, nparts]
+  float* lse_part;         // EPI_LSE: float2 [M, nparts]
   int nparts;
   float* zt;               // EPI_LSE: target logit [M]
   const float* lse;        // EPI_CEGRAD: [M]
@@ -67,18 +79,14 @@ struct Params {
   int* err;
 };
 
-__device__ __forceinline__ int mbar_phase(int it) { return (it / STAGES) & 1; }
-
 // ---------------------------------------------------------------------------------- convert
 // FWD: packed tile [256 rows][32 B] (plain), scales [256]; thread t converts row t (one group)
 // into the K-major SW128 B tile (row t at t*128 B, 16-byte chunk j stored at chunk j ^ (t&7)).
-template <int NACC>
-__device__ __forceinline__ void convert_fwd(uint8_t* stage, int t) {
-  using Ly = Layout<NACC>;
-  const uint4* src = reinterpret_cast<const uint4*>(stage + Ly::P_OFF + t * 32);
+__device__ __forceinline__ void convert_fwd(const uint8_t* pk, const uint8_t* sc, uint8_t* bt, int t) {
+  const uint4* src = reinterpret_cast<const uint4*>(pk + t * 32);
   const uint4 p0 = src[0], p1 = src[1];
-  const uint32_t s2 = scale_pair(reinterpret_cast<const uint16_t*>(stage + Ly::S_OFF)[t]);
-  uint8_t* row = stage + Ly::B_OFF + t * 128;
+  const uint32_t s2 = scale_pair(reinterpret_cast<const uint16_t*>(sc)[t]);
+  uint8_t* row = bt + t * 128;
   const uint32_t words[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
@@ -92,21 +100,46 @@ __device__ __forceinline__ void convert_fwd(uint8_t* stage, int t) {
 // chunk c ^ (k&7)), scales [4 groups][64 k-rows].  Thread t: group g = t/64 (64 output
 // columns), row k = t%64; its 8 words become chunks 0..7 of row k of MN-major atom g
 // (atom = 64 columns x 64 k-rows, 128 B per k-row, chunk c stored at c ^ (k&7)).
-template <int NACC>
-__device__ __forceinline__ void convert_trans(uint8_t* stage, int t) {
-  using Ly = Layout<NACC>;
+__device__ __forceinline__ void convert_trans(const uint8_t* pk, const uint8_t* sc, uint8_t* bt, int t) {
   const int g = t >> 6, k = t & 63;
-  const uint8_t* prow = stage + Ly::P_OFF + k * 128;
+  const uint8_t* prow = pk + k * 128;
   const uint4 p0 = *reinterpret_cast<const uint4*>(prow + (((2 * g) ^ (k & 7)) << 4));
   const uint4 p1 = *reinterpret_cast<const uint4*>(prow + (((2 * g + 1) ^ (k & 7)) << 4));
-  const uint32_t s2 = scale_pair(reinterpret_cast<const uint16_t*>(stage + Ly::S_OFF)[g * 64 + k]);
-  uint8_t* row = stage + Ly::B_OFF + g * 8192 + k * 128;
+  const uint32_t s2 = scale_pair(reinterpret_cast<const uint16_t*>(sc)[g * 64 + k]);
+  uint8_t* row = bt + g * 8192 + k * 128;
   const uint32_t words[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
     uint32_t o[4];
     dequant_word(words[j], s2, o);
     *reinterpret_cast<uint4*>(row + ((j ^ (k & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
+// LoRA block e: copy the 64-wide slice of B_x into the B slot in the layout the MMA reads,
+// zero outside [0, kx) x [0, N).  The operand is a few tens of KB and stays in L2.
+template <bool TRANS>
+__device__ __forceinline__ void copy_lora_b(const Params& p, int e, int n0, uint8_t* bt, int t) {
+  const uint4 zero = make_uint4(0, 0, 0, 0);
+  if (!TRANS) {  // K-major: row n = t, chunk j = 8 columns of the rank axis
+    const int n = n0 + t;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int col = e * 64 + 8 * j;
+      uint4 v = zero;
+      if (n < p.N && col < p.kx) v = *reinterpret_cast<const uint4*>(p.Bx + static_cast<int64_t>(n) * p.ldbx + col);
+      *reinterpret_cast<uint4*>(bt + t * 128 + ((j ^ (t & 7)) << 4)) = v;
+    }
+  } else {       // MN-major: atom g (64 output columns), row k of the rank axis
+    const int g = t >> 6, k = t & 63;
+    const int rr = e * 64 + k;
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      const int col = n0 + 64 * g + 8 * c;
+      uint4 v = zero;
+      if (rr < p.kx && col < p.N) v = *reinterpret_cast<const uint4*>(p.Bx + static_cast<int64_t>(rr) * p.ldbx + col);
+      *reinterpret_cast<uint4*>(bt + g * 8192 + k * 128 + ((c ^ (k & 7)) << 4)) = v;
+    }
   }
 }
 
@@ -149,7 +182,7 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
       }
     }
     if (row_ok) {
-      float2* pr = reinterpret_cast<float2*>(p.part) + static_cast<int64_t>(row) * p.nparts + blockIdx.x * 2;
+      float2* pr = reinterpret_cast<float2*>(p.lse_part) + static_cast<int64_t>(row) * p.nparts + blockIdx.x * 2;
       if (NACC == 2) {
         pr[0] = make_float2(mx, sum);
         pr[1] = make_float2(-INFINITY, 0.0f);
@@ -190,8 +223,6 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
     return;
   }
 
-  float* Cp = static_cast<float*>(p.C);
-  if (p.epi == EPI_PARTIAL) Cp += static_cast<int64_t>(blockIdx.z) * p.M * p.ldc;
 #pragma unroll 1
   for (int cc = 0; cc < NCH; ++cc) {
     float v[32];
@@ -206,16 +237,14 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
         if (c0 + 8 * i < p.N)
           dst[i] = make_uint4(pack_half2(v[8 * i], v[8 * i + 1]), pack_half2(v[8 * i + 2], v[8 * i + 3]),
                               pack_half2(v[8 * i + 4], v[8 * i + 5]), pack_half2(v[8 * i + 6], v[8 * i + 7]));
-    } else {  // EPI_F32 (+ residual) or EPI_PARTIAL
-      const bool part = p.epi == EPI_PARTIAL;
-      const float al = part ? 1.0f : p.alpha;
-      float4* dst = reinterpret_cast<float4*>(Cp + static_cast<int64_t>(row) * p.ldc + c0);
-      const float4* res =
-          (!part && p.R) ? reinterpret_cast<const float4*>(p.R + static_cast<int64_t>(row) * p.ldr + c0) : nullptr;
+    } else {  // EPI_F32 (+ residual)
+      float4* dst = reinterpret_cast<float4*>(static_cast<float*>(p.C) + static_cast<int64_t>(row) * p.ldc + c0);
+      const float4* res = p.R ? reinterpret_cast<const float4*>(p.R + static_cast<int64_t>(row) * p.ldr + c0) : nullptr;
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         if (c0 + 4 * i >= p.N) break;
-        float4 o = make_float4(al * v[4 * i], al * v[4 * i + 1], al * v[4 * i + 2], al * v[4 * i + 3]);
+        float4 o = make_float4(p.alpha * v[4 * i], p.alpha * v[4 * i + 1], p.alpha * v[4 * i + 2],
+                               p.alpha * v[4 * i + 3]);
         if (res) {
           const float4 r = res[i];
           o.x += r.x; o.y += r.y; o.z += r.z; o.w += r.w;
@@ -226,22 +255,93 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
   }
 }
 
+// ---------------------------------------------------------------------------------- split-K
+// The splits of one output tile run as one thread-block cluster along z.  Each CTA parks its fp32
+// accumulator tile in its own shared memory (the rings are idle once the accumulator is final):
+// row r at r * 1 KB, 16-byte chunk c at chunk c ^ (r & 31), conflict-free for the row-per-thread
+// writes and the chunk-per-thread reads.  After a cluster barrier CTA z sums rows
+// [z * ceil(128/S), ...) of all S partials over distributed shared memory in split order
+// (deterministic) and applies the epilogue.
+__device__ __forceinline__ void stash_partial(uint32_t tmem, bool valid, int warp, int lane, uint8_t* smem) {
+  const int q = warp & 3, h = warp >> 2;
+  const int r = 32 * q + lane;
+  const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * q) << 16) + 128 * h;
+  uint8_t* row = smem + r * 1024;
+#pragma unroll 1
+  for (int cc = 0; cc < 4; ++cc) {
+    float v[32];
+    if (valid) {
+      tmem_ld32(tbase + 32 * cc, v);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 32; ++i) v[i] = 0.0f;
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int c = 32 * h + 8 * cc + i;
+      *reinterpret_cast<float4*>(row + ((c ^ (r & 31)) << 4)) =
+          make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+    }
+  }
+}
+
+__device__ __forceinline__ void split_reduce(const Params& p, const uint8_t* smem, int m0, int n0) {
+  const int S = gridDim.z, z = blockIdx.z;
+  const int rpc = (BM + S - 1) / S;
+  const int r0 = z * rpc, r1 = min(BM, r0 + rpc);
+  const uint32_t base = smem_u32(smem);
+  for (int i = threadIdx.x; i < (r1 - r0) * 64; i += THREADS) {
+    const int r = r0 + (i >> 6), c = i & 63;
+    const int64_t row = m0 + r, col = n0 + 4 * c;
+    if (row >= p.M || col >= p.N) continue;
+    const uint32_t off = base + r * 1024 + ((c ^ (r & 31)) << 4);
+    float4 v[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      if (j < S) v[j] = ld_dsmem_f4(dsmem_addr(off, j));
+    float4 s = v[0];
+#pragma unroll
+    for (int j = 1; j < 8; ++j)
+      if (j < S) {
+        s.x += v[j].x; s.y += v[j].y; s.z += v[j].z; s.w += v[j].w;
+      }
+    if (p.epi == EPI_F16) {
+      *reinterpret_cast<uint2*>(static_cast<uint16_t*>(p.C) + row * p.ldc + col) =
+          make_uint2(pack_half2(s.x, s.y), pack_half2(s.z, s.w));
+    } else {
+      float4 o = make_float4(p.alpha * s.x, p.alpha * s.y, p.alpha * s.z, p.alpha * s.w);
+      if (p.R) {
+        const float4 rr = *reinterpret_cast<const float4*>(p.R + row * p.ldr + col);
+        o.x += rr.x; o.y += rr.y; o.z += rr.z; o.w += rr.w;
+      }
+      *reinterpret_cast<float4*>(static_cast<float*>(p.C) + row * p.ldc + col) = o;
+    }
+  }
+}
+
 // ---------------------------------------------------------------------------------- kernel
+// Launched with programmatic stream serialization: the prologue, and (when p.w_ready) the
+// weight loads and decodes of the first ring slots, overlap the previous kernel; everything that
+// reads an activation or writes memory waits in griddep_wait() first.
 template <bool TRANS, int NACC>
 __global__ void __launch_bounds__(THREADS, 1)
     dequant_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmP,
                         const __grid_constant__ CUtensorMap tmS, const __grid_constant__ CUtensorMap tmAx,
-                        const __grid_constant__ CUtensorMap tmBx, const Params p) {
+                        const Params p) {
   using Ly = Layout<NACC>;
+  constexpr int TSTG = Ly::TSTG, BSTG = Ly::BSTG;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + Ly::BAR_OFF);
-  uint64_t* conv = full + STAGES;
-  uint64_t* empty = conv + STAGES;
-  uint64_t* accf = empty + STAGES;
+  uint64_t* wfull = reinterpret_cast<uint64_t*>(smem + Ly::BAR_OFF);  // TMA ring: packed W + scales landed
+  uint64_t* afull = wfull + TSTG;                                      // TMA ring: A tile landed
+  uint64_t* empty = afull + TSTG;                                      // TMA ring: MMA done with slot
+  uint64_t* bfull = empty + TSTG;                                      // B ring: tile decoded
+  uint64_t* bempty = bfull + BSTG;                                     // B ring: MMA done with slot
+  uint64_t* accf = bempty + BSTG;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accf + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
+  griddep_launch();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM * NACC;
   // K range of this split: main tiles [kt0, kt1); the LoRA block rides with the last split.
@@ -249,15 +349,20 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int kt0 = blockIdx.z * p.kt_split;
   const int kt1 = min(num_k, kt0 + p.kt_split);
   const int num_main = max(0, kt1 - kt0);
+  const bool split = gridDim.z > 1;  // NACC == 1 only (host)
   const bool last_split = blockIdx.z == gridDim.z - 1;
   const int num_x = last_split ? (p.kx_steps + 3) / 4 : 0;
   const int total = num_main + num_x;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&conv[s], 8);
+    for (int s = 0; s < TSTG; ++s) {
+      mbar_init(&wfull[s], 1);
+      mbar_init(&afull[s], 1);
       mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < BSTG; ++b) {
+      mbar_init(&bfull[b], 8);
+      mbar_init(&bempty[b], 1);
     }
     mbar_init(accf, 1);
     *abort_flag = 0;
@@ -275,53 +380,50 @@ __global__ void __launch_bounds__(THREADS, 1)
       tma_prefetch_desc(&tmA);
       tma_prefetch_desc(&tmP);
       tma_prefetch_desc(&tmS);
-      int issued = 0;
-      for (int it = 0; it < total; ++it) {
-        const int s = it % STAGES;
-        if (!mbar_wait(&empty[s], mbar_phase(it) ^ 1, abort_flag, p.err)) break;
-        uint8_t* st = smem + s * Ly::STRIDE;
-        if (it < num_main) {
-          const int kt = kt0 + it;
-          mbar_arrive_expect_tx(&full[s], NACC * A_BYTES + P_BYTES + S_BYTES);
-          tma_load_2d(st + Ly::A_OFF, &tmA, &full[s], kt * BK, m0);
-          if (!TRANS) {
-            tma_load_2d(st + Ly::P_OFF, &tmP, &full[s], kt * (BK / 2), n0);  // packed [N, K/2]
-            tma_load_2d(st + Ly::S_OFF, &tmS, &full[s], n0, kt);             // scales [K/64, N]
-          } else {
-            tma_load_2d(st + Ly::P_OFF, &tmP, &full[s], n0 / 2, kt * BK);    // packed [K, N/2]
-            tma_load_2d(st + Ly::S_OFF, &tmS, &full[s], kt * BK, n0 / 64);   // scales [N/64, K]
-          }
+      auto load_w = [&](int it) {
+        const int s = it % TSTG, kt = kt0 + it;
+        uint8_t* st = smem + s * Ly::T_STRIDE;
+        mbar_arrive_expect_tx(&wfull[s], P_BYTES + S_BYTES);
+        if (!TRANS) {
+          tma_load_2d(st + Ly::P_OFF, &tmP, &wfull[s], kt * (BK / 2), n0);  // packed [N, K/2]
+          tma_load_2d(st + Ly::S_OFF, &tmS, &wfull[s], n0, kt);             // scales [K/64, N]
         } else {
-          const int e = it - num_main;
-          mbar_arrive_expect_tx(&full[s], NACC * A_BYTES + B_BYTES);
-          tma_load_2d(st + Ly::A_OFF, &tmAx, &full[s], e * BK, m0);
-          if (!TRANS) {
-            tma_load_2d(st + Ly::B_OFF, &tmBx, &full[s], e * BK, n0);        // B_x [N, Kx], K-major
-          } else {
-#pragma unroll
-            for (int a = 0; a < 4; ++a)                                        // B_x [Kx, N], MN-major atoms
-              tma_load_2d(st + Ly::B_OFF + a * 8192, &tmBx, &full[s], n0 + 64 * a, e * BK);
-          }
+          tma_load_2d(st + Ly::P_OFF, &tmP, &wfull[s], n0 / 2, kt * BK);    // packed [K, N/2]
+          tma_load_2d(st + Ly::S_OFF, &tmS, &wfull[s], kt * BK, n0 / 64);   // scales [N/64, K]
         }
-        issued = it + 1;
+      };
+      int w_issued = 0, a_issued = 0;
+      if (p.w_ready)
+        for (; w_issued < min(TSTG, num_main); ++w_issued) load_w(w_issued);
+      griddep_wait();
+      for (int it = 0; it < total; ++it) {
+        const int s = it % TSTG;
+        if (it >= TSTG && !mbar_wait(&empty[s], ((it / TSTG) & 1) ^ 1, abort_flag, p.err)) break;
+        if (it < num_main && it >= w_issued) load_w(w_issued++);
+        uint8_t* st = smem + s * Ly::T_STRIDE;
+        mbar_arrive_expect_tx(&afull[s], NACC * A_BYTES);
+        if (it < num_main) tma_load_2d(st + Ly::A_OFF, &tmA, &afull[s], (kt0 + it) * BK, m0);
+        else tma_load_2d(st + Ly::A_OFF, &tmAx, &afull[s], (it - num_main) * BK, m0);
+        a_issued = it + 1;
       }
-      // Never leave the CTA with copies in flight: wait (bounded) for the last stages issued.
-      for (int it = (issued > STAGES ? issued - STAGES : 0); it < issued; ++it) {
-        int dummy = 0;
-        mbar_wait(&full[it % STAGES], mbar_phase(it), &dummy, p.err);
-      }
+      // Never leave the CTA with copies in flight: wait (bounded) for the last loads issued.
+      int dummy = 0;
+      for (int it = (w_issued > TSTG ? w_issued - TSTG : 0); it < w_issued; ++it)
+        mbar_wait(&wfull[it % TSTG], (it / TSTG) & 1, &dummy, p.err);
+      for (int it = (a_issued > TSTG ? a_issued - TSTG : 0); it < a_issued; ++it)
+        mbar_wait(&afull[it % TSTG], (it / TSTG) & 1, &dummy, p.err);
     }
   } else if (warp == 9) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_f16_f32(BM, BN, TRANS);
       for (int it = 0; it < total; ++it) {
-        const int s = it % STAGES;
-        if (!mbar_wait(&full[s], mbar_phase(it), abort_flag, p.err)) break;
-        if (!mbar_wait(&conv[s], mbar_phase(it), abort_flag, p.err)) break;
+        const int s = it % TSTG, b = it % BSTG;
+        if (!mbar_wait(&afull[s], (it / TSTG) & 1, abort_flag, p.err)) break;
+        if (!mbar_wait(&bfull[b], (it / BSTG) & 1, abort_flag, p.err)) break;
         tc_fence_after();
-        uint8_t* st = smem + s * Ly::STRIDE;
-        const uint32_t a_base = smem_u32(st + Ly::A_OFF), b_base = smem_u32(st + Ly::B_OFF);
+        const uint32_t a_base = smem_u32(smem + s * Ly::T_STRIDE + Ly::A_OFF);
+        const uint32_t b_base = smem_u32(smem + Ly::B_BASE + b * B_BYTES);
         const int nk = (it < num_main) ? 4 : min(4, p.kx_steps - 4 * (it - num_main));
         for (int kk = 0; kk < nk; ++kk) {
           const uint64_t bd = TRANS ? smem_desc_sw128(b_base + kk * 2048, 8192, 1024)
@@ -333,6 +435,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
         }
         tc_commit(&empty[s]);
+        tc_commit(&bempty[b]);
       }
       tc_commit(accf);
     }
@@ -340,21 +443,27 @@ __global__ void __launch_bounds__(THREADS, 1)
     // ------------------------------------------------------------ converters, then epilogue
     const int t = threadIdx.x;  // 0..255
     for (int it = 0; it < total; ++it) {
-      const int s = it % STAGES;
-      if (!mbar_wait(&full[s], mbar_phase(it), abort_flag, p.err)) break;
+      const int s = it % TSTG, b = it % BSTG;
+      if (!mbar_wait(&bempty[b], ((it / BSTG) & 1) ^ 1, abort_flag, p.err)) break;
+      uint8_t* bt = smem + Ly::B_BASE + b * B_BYTES;
       if (it < num_main) {
-        uint8_t* st = smem + s * Ly::STRIDE;
-        if (TRANS) convert_trans<NACC>(st, t);
-        else convert_fwd<NACC>(st, t);
-        fence_proxy_async_smem();
+        if (!mbar_wait(&wfull[s], (it / TSTG) & 1, abort_flag, p.err)) break;
+        const uint8_t* st = smem + s * Ly::T_STRIDE;
+        if (TRANS) convert_trans(st + Ly::P_OFF, st + Ly::S_OFF, bt, t);
+        else convert_fwd(st + Ly::P_OFF, st + Ly::S_OFF, bt, t);
+      } else {
+        griddep_wait();  // the LoRA operand comes from an earlier kernel
+        copy_lora_b<TRANS>(p, it - num_main, n0, bt, t);
       }
+      fence_proxy_async_smem();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&conv[s]);
+      if (lane == 0) mbar_arrive(&bfull[b]);
     }
-    if (mbar_wait(accf, 0, abort_flag, p.err)) {
-      tc_fence_after();
-      if (total > 0) epilogue<NACC>(p, tmem, warp, lane, m0, n0);
-    }
+    griddep_wait();
+    const bool acc_ok = __all_sync(0xffffffffu, mbar_wait(accf, 0, abort_flag, p.err));
+    tc_fence_after();
+    if (split) stash_partial(tmem, acc_ok && total > 0, warp, lane, smem);
+    else if (acc_ok && total > 0) epilogue<NACC>(p, tmem, warp, lane, m0, n0);
   }
 
   tc_fence_before();
@@ -368,32 +477,12 @@ __global__ void __launch_bounds__(THREADS, 1)
     tc_fence_after();
     tmem_dealloc(tmem, Ly::TMEM_COLS);
   }
-}
-
-// Split-K finish: C = epilogue(sum_z part[z]) in split order.  EPI_F32: alpha * sum (+ R); EPI_F16.
-__global__ void splitk_reduce_kernel(const float* __restrict__ part, int splits, int M, int N, int epi, void* C,
-                                     int64_t ldc, const float* R, int64_t ldr, float alpha) {
-  const int64_t n4 = static_cast<int64_t>(M) * (N / 4);
-  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (i >= n4) return;
-  const int64_t row = i / (N / 4), c = (i % (N / 4)) * 4;
-  const int64_t stride = static_cast<int64_t>(M) * N;
-  float4 s = make_float4(0, 0, 0, 0);
-  for (int z = 0; z < splits; ++z) {
-    const float4 v = *reinterpret_cast<const float4*>(part + z * stride + row * N + c);
-    s.x += v.x; s.y += v.y; s.z += v.z; s.w += v.w;
+  if (split) {  // every thread of every CTA of the cluster passes both barriers
+    griddep_wait();
+    cluster_sync_all();
+    split_reduce(p, smem, m0, n0);
+    cluster_sync_all();
   }
-  if (epi == EPI_F16) {
-    *reinterpret_cast<uint2*>(static_cast<uint16_t*>(C) + row * ldc + c) =
-        make_uint2(pack_half2(s.x, s.y), pack_half2(s.z, s.w));
-    return;
-  }
-  float4 o = make_float4(alpha * s.x, alpha * s.y, alpha * s.z, alpha * s.w);
-  if (R) {
-    const float4 r = *reinterpret_cast<const float4*>(R + row * ldr + c);
-    o.x += r.x; o.y += r.y; o.z += r.z; o.w += r.w;
-  }
-  *reinterpret_cast<float4*>(static_cast<float*>(C) + row * ldc + c) = o;
 }
 
 }  // namespace gemm
@@ -427,22 +516,74 @@ int make_tmap_2d(CUtensorMap* m, const void* base, CUtensorMapDataType dt, int e
   return r == CUDA_SUCCESS ? MEBP_OK : MEBP_ERR_INVALID_ARG;
 }
 
-int gemm_smem_bytes() { return gemm::Layout<2>::SMEM; }
+int gemm_smem_bytes() { return gemm::Layout<1>::SMEM; }
 
 namespace {
 template <bool TRANS, int NACC>
-int launch_variant(dim3 grid, const CUtensorMap& tA, const CUtensorMap& tP, const CUtensorMap& tS,
-                   const CUtensorMap& tAx, const CUtensorMap& tBx, const gemm::Params& p, cudaStream_t st) {
-  using Ly = gemm::Layout<NACC>;
+bool set_smem_attr() {
   static bool attr = false;
-  if (!attr) {
-    if (cudaFuncSetAttribute(gemm::dequant_gemm_kernel<TRANS, NACC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             Ly::SMEM) != cudaSuccess)
-      return MEBP_ERR_CUDA;
-    attr = true;
+  if (!attr)
+    attr = cudaFuncSetAttribute(gemm::dequant_gemm_kernel<TRANS, NACC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                gemm::Layout<NACC>::SMEM) == cudaSuccess;
+  return attr;
+}
+
+// Clusters of `s` CTAs (along z) of the one-accumulator kernel that can be resident at once;
+// 0 when the cluster shape cannot be scheduled.  Queried once per size.
+template <bool TRANS>
+int max_active_clusters(int s) {
+  static int cache[9] = {-1, -1, -1, -1, -1, -1, -1, -1, -1};
+  if (s < 1 || s > 8) return 0;
+  if (cache[s] < 0) {
+    int n = 0;
+    if (set_smem_attr<TRANS, 1>()) {
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(1, 1, s);
+      cfg.blockDim = dim3(gemm::THREADS);
+      cfg.dynamicSmemBytes = gemm::Layout<1>::SMEM;
+      cudaLaunchAttribute at[1];
+      at[0].id = cudaLaunchAttributeClusterDimension;
+      at[0].val.clusterDim.x = 1;
+      at[0].val.clusterDim.y = 1;
+      at[0].val.clusterDim.z = s;
+      cfg.attrs = at;
+      cfg.numAttrs = 1;
+      if (cudaOccupancyMaxActiveClusters(&n, gemm::dequant_gemm_kernel<TRANS, 1>, &cfg) != cudaSuccess) {
+        cudaGetLastError();
+        n = 0;
+      }
+    }
+    cache[s] = n;
   }
+  return cache[s];
+}
+
+template <bool TRANS, int NACC>
+int launch_variant(dim3 grid, const CUtensorMap& tA, const CUtensorMap& tP, const CUtensorMap& tS,
+                   const CUtensorMap& tAx, const gemm::Params& p, cudaStream_t st) {
+  if (!set_smem_attr<TRANS, NACC>()) return MEBP_ERR_CUDA;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(gemm::THREADS);
+  cfg.dynamicSmemBytes = gemm::Layout<NACC>::SMEM;
+  cfg.stream = st;
+  cudaLaunchAttribute at[2];
+  int na = 0;
+  at[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[na].val.programmaticStreamSerializationAllowed = 1;
+  ++na;
+  if (grid.z > 1) {
+    at[na].id = cudaLaunchAttributeClusterDimension;
+    at[na].val.clusterDim.x = 1;
+    at[na].val.clusterDim.y = 1;
+    at[na].val.clusterDim.z = grid.z;
+    ++na;
+  }
+  cfg.attrs = at;
+  cfg.numAttrs = na;
   count_launch();
-  gemm::dequant_gemm_kernel<TRANS, NACC><<<grid, gemm::THREADS, Ly::SMEM, st>>>(tA, tP, tS, tAx, tBx, p);
+  if (cudaLaunchKernelEx(&cfg, gemm::dequant_gemm_kernel<TRANS, NACC>, tA, tP, tS, tAx, p) != cudaSuccess)
+    return MEBP_ERR_CUDA;
   return MEBP_OK;
 }
 }  // namespace
@@ -455,7 +596,7 @@ int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st) {
   const int nacc = (g.M >= 2048) ? 2 : 1;
   const int bm = BM * nacc;
 
-  CUtensorMap tA, tP, tS, tAx, tBx;
+  CUtensorMap tA, tP, tS, tAx;
   int rc;
   // A: fp16 [M, K], row pitch lda elements.
   if ((rc = make_tmap_2d(&tA, g.A, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, g.K, g.M, g.lda * 2, 64, bm,
@@ -478,26 +619,20 @@ int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st) {
                            CU_TENSOR_MAP_SWIZZLE_NONE)))
       return rc;
   }
+  Params p{};
   int kx_steps = 0;
   if (g.Ax && g.kx > 0) {
-    kx_steps = static_cast<int>((g.kx + 15) / 16);
+    if ((g.kx % 16) || (reinterpret_cast<uintptr_t>(g.Bx) & 15) || (g.ldbx % 8)) return MEBP_ERR_INVALID_ARG;
+    kx_steps = static_cast<int>(g.kx / 16);
     if ((rc = make_tmap_2d(&tAx, g.Ax, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, g.kx, g.M, g.ldax * 2, 64, bm,
                            CU_TENSOR_MAP_SWIZZLE_128B)))
       return rc;
-    if (!g.trans) {
-      if ((rc = make_tmap_2d(&tBx, g.Bx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, g.kx, g.N, g.ldbx * 2, 64, BN,
-                             CU_TENSOR_MAP_SWIZZLE_128B)))
-        return rc;
-    } else {
-      if ((rc = make_tmap_2d(&tBx, g.Bx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, g.N, g.kx, g.ldbx * 2, 64, 64,
-                             CU_TENSOR_MAP_SWIZZLE_128B)))
-        return rc;
-    }
+    p.Bx = static_cast<const uint16_t*>(g.Bx);
+    p.ldbx = g.ldbx;
+    p.kx = static_cast<int>(g.kx);
   } else {
     tAx = tA;
-    tBx = tA;
   }
-  Params p{};
   p.M = static_cast<int>(g.M);
   p.N = static_cast<int>(g.N);
   p.K = static_cast<int>(g.K);
@@ -511,46 +646,41 @@ int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st) {
   p.targets = g.targets;
   p.col_offset = g.col_offset;
   p.n_valid = g.n_valid > 0 ? g.n_valid : static_cast<int>(g.N);
-  p.part = g.part;
+  p.lse_part = g.part;
   p.nparts = g.nparts;
   p.zt = g.zt;
   p.lse = g.lse;
   p.ce_w = g.ce_w;
   p.err = g.err;
 
+  p.w_ready = g.w_ready ? 1 : 0;
+
   const int tiles_n = static_cast<int>((g.N + BN - 1) / BN), tiles_m = static_cast<int>((g.M + bm - 1) / bm);
   const int num_k = static_cast<int>(g.K / BK);
-  // Split K when the output tiles cannot fill the GPU (152 SMs, one CTA each) and each split
-  // keeps >= 4 K tiles; partial tiles go to the caller's workspace.
+  // Split K when the output tiles leave at least half of the 152 SMs idle: the largest cluster
+  // size S <= 8 with >= 2 K tiles per split whose clusters all fit on the GPU at once.
   int splits = 1;
   const int grid_mn = tiles_n * tiles_m;
-  if ((g.epi == EPI_F32 || g.epi == EPI_F16) && g.split_ws && grid_mn < 120 && num_k >= 8) {
-    splits = std::min({num_k / 4, (2 * 152 + grid_mn - 1) / grid_mn, 16});
-    const int64_t need = g.M * g.N;
-    while (splits > 1 && splits * need > g.split_ws_floats) --splits;
+  if ((g.epi == EPI_F32 || g.epi == EPI_F16) && nacc == 1 && grid_mn <= 76 && num_k >= 4) {
+    for (int s = std::min(8, num_k / 2); s >= 2; --s) {
+      const int mac = g.trans ? max_active_clusters<true>(s) : max_active_clusters<false>(s);
+      if (grid_mn <= mac) {
+        splits = s;
+        break;
+      }
+    }
   }
   const int kt_split = (num_k + splits - 1) / splits;
-  splits = (num_k + kt_split - 1) / kt_split;
+  splits = (num_k + kt_split - 1) / kt_split;  // every split gets >= 1 K tile
   p.kt_split = kt_split;
-  if (splits > 1) {
-    p.epi = EPI_PARTIAL;
-    p.C = g.split_ws;
-    p.ldc = g.N;
-  }
   dim3 grid(tiles_n, tiles_m, splits);
   if (g.trans)
-    rc = nacc == 2 ? launch_variant<true, 2>(grid, tA, tP, tS, tAx, tBx, p, st)
-                   : launch_variant<true, 1>(grid, tA, tP, tS, tAx, tBx, p, st);
+    rc = nacc == 2 ? launch_variant<true, 2>(grid, tA, tP, tS, tAx, p, st)
+                   : launch_variant<true, 1>(grid, tA, tP, tS, tAx, p, st);
   else
-    rc = nacc == 2 ? launch_variant<false, 2>(grid, tA, tP, tS, tAx, tBx, p, st)
-                   : launch_variant<false, 1>(grid, tA, tP, tS, tAx, tBx, p, st);
+    rc = nacc == 2 ? launch_variant<false, 2>(grid, tA, tP, tS, tAx, p, st)
+                   : launch_variant<false, 1>(grid, tA, tP, tS, tAx, p, st);
   if (rc) return rc;
-  if (splits > 1) {
-    const int64_t n4 = g.M * (g.N / 4);
-    count_launch();
-    splitk_reduce_kernel<<<static_cast<unsigned>((n4 + 255) / 256), 256, 0, st>>>(
-        g.split_ws, splits, static_cast<int>(g.M), static_cast<int>(g.N), g.epi, g.C, g.ldc, g.R, g.ldr, g.alpha);
-  }
   return cudaGetLastError() == cudaSuccess ? MEBP_OK : MEBP_ERR_CUDA;
 }
 

@@ -41,8 +41,11 @@ struct GemmArgs {
   float* zt = nullptr;
   const float* lse = nullptr;
   const float* ce_w = nullptr;   // EPI_CEGRAD: device scalar weight of a valid row
-  float* split_ws = nullptr;     // fp32 workspace for split-K partial tiles (EPI_F32 / EPI_F16), or null
-  int64_t split_ws_floats = 0;
+  // The packed weights are not written by any kernel that may still be running when this GEMM
+  // starts, so they may be fetched and decoded before the previous kernel in the stream finishes.
+  // Holds whenever the kernel launched before the GEMM was itself launched normally after the
+  // weights were written (every entry point starts with such a kernel, or clears the flag).
+  bool w_ready = false;
   int* err = nullptr;
 };
 

@@ -96,12 +96,20 @@ void launch_skinny_gemm(const uint16_t* X, int64_t ldx, int64_t M, int64_t K, co
 }
 
 // ------------------------------------------------------------------------------------ tall reduce
+// Direct output of a single-split reduction: C[p * sp + q * sq] (+)= mult * sum.
+struct Direct {
+  float* C;
+  int64_t sp, sq;
+  int accumulate;
+  const float* mult;
+};
+
 // part[z][p][q] = sum_{m in split z} P[m, p] Q[m, q]   (p < Pw, q < Qw)
 template <int NQ>
 __global__ void __launch_bounds__(128) tall_reduce_kernel(const uint16_t* __restrict__ P, int64_t ldp,
                                                           const uint16_t* __restrict__ Q, int64_t ldq, int64_t M,
                                                           int Pw, int Qw, int64_t m_per_split,
-                                                          float* __restrict__ part) {
+                                                          float* __restrict__ part, Direct dw) {
   constexpr int BP = 64, BMr = 64, QT = NQ * 8, LDP = BP + 8, LDQ = QT + 8;
   __shared__ __align__(16) uint16_t ps[2][BMr * LDP];
   __shared__ __align__(16) uint16_t qs[2][BMr * LDQ];
@@ -155,8 +163,22 @@ __global__ void __launch_bounds__(128) tall_reduce_kernel(const uint16_t* __rest
     __syncthreads();
   }
   const int r = lane >> 2, c = (lane & 3) * 2;
-  float* out = part + static_cast<int64_t>(blockIdx.z) * Pw * Qw;
   const int pr = p0 + warp * 16 + r;
+  if (dw.C) {  // a single split: finish here (C (+)= mult * sum)
+    const float mu = dw.mult ? *dw.mult : 1.0f;
+#pragma unroll
+    for (int nq = 0; nq < NQ; ++nq) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int pp = pr + ((e >> 1) << 3), qq = q0 + nq * 8 + c + (e & 1);
+        if (pp >= Pw || qq >= Qw) continue;
+        float* dst = dw.C + pp * dw.sp + qq * dw.sq;
+        *dst = dw.accumulate ? *dst + mu * acc[nq][e] : mu * acc[nq][e];
+      }
+    }
+    return;
+  }
+  float* out = part + static_cast<int64_t>(blockIdx.z) * Pw * Qw;
 #pragma unroll
   for (int nq = 0; nq < NQ; ++nq) {
     const int qc = q0 + nq * 8 + c;
@@ -196,20 +218,23 @@ int launch_tall_reduce(const uint16_t* P, int64_t ldp, const uint16_t* Q, int64_
   const int nq = Qw <= 32 ? 4 : (Qw <= 64 ? 8 : 12);
   const int gx = (Pw + 63) / 64, gy = (Qw + nq * 8 - 1) / (nq * 8);
   int64_t splits = (4 * 152 + gx * gy - 1) / (gx * gy);
-  splits = std::min<int64_t>(splits, std::max<int64_t>(1, M / 256));
+  splits = std::min<int64_t>(splits, std::max<int64_t>(1, M / 1024));  // short token ranges: one pass, no second kernel
   splits = std::min<int64_t>(splits, scratch_floats / (static_cast<int64_t>(Pw) * Qw));
   if (splits < 1) return MEBP_ERR_INVALID_ARG;
   int64_t mps = (M + splits - 1) / splits;
   mps = (mps + 63) / 64 * 64;
   splits = std::max<int64_t>(1, (M + mps - 1) / mps);
   dim3 grid(gx, gy, static_cast<unsigned>(splits));
-  switch (nq) {
-    case 4: count_launch(); tall_reduce_kernel<4><<<grid, 128, 0, st>>>(P, ldp, Q, ldq, M, Pw, Qw, mps, scratch); break;
-    case 8: count_launch(); tall_reduce_kernel<8><<<grid, 128, 0, st>>>(P, ldp, Q, ldq, M, Pw, Qw, mps, scratch); break;
-    default: count_launch(); tall_reduce_kernel<12><<<grid, 128, 0, st>>>(P, ldp, Q, ldq, M, Pw, Qw, mps, scratch); break;
-  }
-  const int64_t n = static_cast<int64_t>(Pw) * Qw;
   const int64_t sp = ldc > 0 ? ldc : 1, sq = ldc > 0 ? 1 : -ldc;
+  Direct dw{nullptr, sp, sq, accumulate ? 1 : 0, mult};
+  if (splits == 1) dw.C = C;
+  switch (nq) {
+    case 4: count_launch(); tall_reduce_kernel<4><<<grid, 128, 0, st>>>(P, ldp, Q, ldq, M, Pw, Qw, mps, scratch, dw); break;
+    case 8: count_launch(); tall_reduce_kernel<8><<<grid, 128, 0, st>>>(P, ldp, Q, ldq, M, Pw, Qw, mps, scratch, dw); break;
+    default: count_launch(); tall_reduce_kernel<12><<<grid, 128, 0, st>>>(P, ldp, Q, ldq, M, Pw, Qw, mps, scratch, dw); break;
+  }
+  if (dw.C) return MEBP_OK;
+  const int64_t n = static_cast<int64_t>(Pw) * Qw;
   count_launch();
   split_sum_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(scratch, static_cast<int>(splits), Pw, Qw,
                                                                            C, sp, sq, accumulate ? 1 : 0, mult);

@@ -66,7 +66,7 @@ struct mebp_ctx {
   float *dm = nullptr, *dtmp = nullptr, *dh1 = nullptr, *dvec = nullptr, *gbuf[2] = {nullptr, nullptr};
   float* red = nullptr;
   int64_t red_floats = 0;
-  float* split_ws = nullptr;   // split-K partial tiles of the fused GEMMs
+  float* split_ws = nullptr;   // fp32 per-head partials of the attention backward
   int64_t split_ws_floats = 0;
   // LM head
   uint16_t *hf = nullptr, *dz = nullptr;
@@ -183,6 +183,7 @@ GemmArgs gemm_fwd(const uint16_t* X, int64_t ldx, int64_t M, const mebp_packed& 
   g.qpack = W.qpack;
   g.scales = W.scales;
   g.scale_pitch = W.rows;
+  g.w_ready = true;  // model weights: written only by mebp_compress_weights, before any step
   return g;
 }
 // dX = dY deq(W) for W [N_w, K_w] stored packed: GEMM K = N_w (reduction), N = K_w (output).
@@ -197,6 +198,7 @@ GemmArgs gemm_dx(const uint16_t* dY, int64_t ldy, int64_t M, const mebp_packed& 
   g.qpack = W.qpack;
   g.scales = W.scales;
   g.scale_pitch = W.rows;
+  g.w_ready = true;  // model weights: written only by mebp_compress_weights, before any step
   return g;
 }
 
@@ -211,8 +213,6 @@ cudaEvent_t pool_event(mebp_ctx* c) {
 
 int run_gemm(mebp_ctx* c, GemmArgs& g, cudaStream_t st, const char* what) {
   g.err = c->d_err;
-  g.split_ws = c->split_ws;
-  g.split_ws_floats = c->split_ws_floats;
   ProfRec pr{};
   if (c->prof) {
     pr.a = pool_event(c);
@@ -429,6 +429,7 @@ int lmhead(mebp_ctx* c, const mebp_packed* E, const float* gf, const float* h, c
     t.A = c->dz; t.lda = c->vchunk; t.M = T; t.N = D; t.K = n;
     t.qpack = Ec.qpack; t.scales = Ec.scales; t.scale_pitch = V;
     t.epi = EPI_F32; t.C = c->dhf; t.ldc = D; t.R = c0 ? c->dhf : nullptr; t.ldr = D; t.alpha = 1.0f / kCeShift;
+    t.w_ready = true;
     if ((rc = run_gemm(c, t, st, "LM head (dH pass)"))) return rc;
   }
   launch_rmsnorm_bwd(c->dhf, h, gf, c->rf, nullptr, T, D, unscale_dh ? c->scal + 1 : nullptr, dh, dh_h, st);
@@ -744,6 +745,7 @@ static int linear_common(mebp_ctx* c, bool dx_mode, const uint16_t* X, int64_t M
     }
     g.epi = EPI_F32; g.C = y32; g.ldc = K; g.R = R; g.ldr = K;
   }
+  g.w_ready = false;  // the caller may have written W with the kernel just before this one
   int rc = run_gemm(c, g, st, dx_mode ? "linear dX" : "linear forward");
   if (A) cudaFreeAsync(Ac, st);
   if (rc) return rc;
