@@ -79,6 +79,8 @@ template <int HD>
 __global__ void __launch_bounds__(128, 1) fwd_kernel(const uint16_t* __restrict__ qkv, int64_t ld, int S, int H,
                                                      int KV, uint16_t* __restrict__ o, int64_t ldo,
                                                      float* __restrict__ lse) {
+  griddep_wait();
+  griddep_launch();
   constexpr int LD = HD + 8, NO = HD / 8;
   extern __shared__ __align__(16) uint16_t sm[];
   uint16_t* qs = sm;
@@ -169,6 +171,8 @@ __global__ void __launch_bounds__(128, 1) fwd_kernel(const uint16_t* __restrict_
 // dvec[b, h, s] = sum_d dO[t, h, d] * o[t, h, d]
 __global__ void dvec_kernel(const uint16_t* __restrict__ o, const uint16_t* __restrict__ dout, int64_t ldo, int B,
                             int S, int H, int HD, float* __restrict__ dvec) {
+  griddep_wait();
+  griddep_launch();
   const int64_t w = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (w >= static_cast<int64_t>(B) * S * H) return;
@@ -198,6 +202,8 @@ __global__ void __launch_bounds__(128, 1) dkdv_kernel(const uint16_t* __restrict
                                                       const float* __restrict__ lse, const float* __restrict__ dvec,
                                                       int S, int H, int KV, uint16_t* __restrict__ dqkv,
                                                       float* __restrict__ part, int64_t T) {
+  griddep_wait();
+  griddep_launch();
   constexpr int LD = HD + 8, NC = DC / 8, NCH = HD / DC;
   extern __shared__ __align__(16) uint16_t sm[];
   uint16_t* ks = sm;
@@ -312,6 +318,8 @@ __global__ void __launch_bounds__(128, 1) dq_kernel(const uint16_t* __restrict__
                                                     const uint16_t* __restrict__ dout, int64_t ldo,
                                                     const float* __restrict__ lse, const float* __restrict__ dvec,
                                                     int S, int H, int KV, uint16_t* __restrict__ dqkv) {
+  griddep_wait();
+  griddep_launch();
   constexpr int LD = HD + 8, NC = DC / 8, NCH = HD / DC;
   extern __shared__ __align__(16) uint16_t sm[];
   uint16_t* qs = sm;
@@ -392,13 +400,14 @@ void fwd_launch(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, ui
     init = true;
   }
   dim3 grid((S + BQ - 1) / BQ, H, B);
-  count_launch();
-  fwd_kernel<HD><<<grid, 128, smem, st>>>(qkv, ld, S, H, KV, o, ldo, lse);
+  launch_k(fwd_kernel<HD>, grid, 128, smem, st, qkv, ld, S, H, KV, o, ldo, lse);
 }
 
 // dK, dV of kv head j = sum over the query heads of group j of the per-head partials (fixed order).
 __global__ void dkdv_group_sum(const float* __restrict__ part, int64_t T, int H, int KV, int HD, int64_t ld,
                                uint16_t* __restrict__ dqkv) {
+  griddep_wait();
+  griddep_launch();
   const int64_t n2 = T * KV * HD / 2;
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (i >= 2 * n2) return;
@@ -435,17 +444,14 @@ void bwd_launch(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t l
   const bool perhead = H > KV && part && static_cast<int64_t>(nkb) * KV * B * NCH < 2 * 152 &&
                        2 * T * H * HD <= part_floats;
   dim3 g1(nkb, perhead ? H : KV, B * NCH);
-  count_launch();
-  dkdv_kernel<HD, DC><<<g1, 128, smem, st>>>(qkv, ld, dout, ldo, lse, dvec, S, H, KV, dqkv, perhead ? part : nullptr,
-                                             T);
+  launch_k(dkdv_kernel<HD, DC>, g1, 128, smem, st, qkv, ld, dout, ldo, lse, dvec, S, H, KV, dqkv,
+           perhead ? part : nullptr, T);
   if (perhead) {
     const int64_t n = T * KV * HD;
-    count_launch();
-    dkdv_group_sum<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(part, T, H, KV, HD, ld, dqkv);
+    launch_k(dkdv_group_sum, static_cast<unsigned>((n + 255) / 256), 256, 0, st, part, T, H, KV, HD, ld, dqkv);
   }
   dim3 g2((S + BQ - 1) / BQ, H, B * NCH);
-  count_launch();
-  dq_kernel<HD, DC><<<g2, 128, smem, st>>>(qkv, ld, dout, ldo, lse, dvec, S, H, KV, dqkv);
+  launch_k(dq_kernel<HD, DC>, g2, 128, smem, st, qkv, ld, dout, ldo, lse, dvec, S, H, KV, dqkv);
 }
 
 }  // namespace attn
@@ -461,8 +467,8 @@ void launch_attn_bwd(const uint16_t* qkv, int64_t ld, const uint16_t* o, const u
                      const float* lse, int B, int S, int H, int KV, int hd, float* dvec, uint16_t* dqkv,
                      float* part, int64_t part_floats, cudaStream_t st) {
   const int64_t nw = static_cast<int64_t>(B) * S * H;
-  count_launch();
-  attn::dvec_kernel<<<static_cast<unsigned>((nw * 32 + 255) / 256), 256, 0, st>>>(o, dout, ldo, B, S, H, hd, dvec);
+  launch_k(attn::dvec_kernel, static_cast<unsigned>((nw * 32 + 255) / 256), 256, 0, st, o, dout, ldo, B, S, H, hd,
+           dvec);
   if (hd == 64) attn::bwd_launch<64, 64>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, part, part_floats, st);
   else if (hd == 128)
     attn::bwd_launch<128, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, part, part_floats, st);

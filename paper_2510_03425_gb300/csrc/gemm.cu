@@ -66,7 +66,6 @@ struct Params {
   const float* R;      // fp32 residual / accumulation source (EPI_F32), may alias C
   int64_t ldr;
   float alpha;         // EPI_F32: C = alpha * acc (+ R)
-  int w_ready;         // packed weights are not written by any kernel that may still run
   // LM-head epilogues
   const int32_t* targets;  // [M]
   int col_offset;          // global vocabulary index of GEMM column 0
@@ -320,9 +319,9 @@ __device__ __forceinline__ void split_reduce(const Params& p, const uint8_t* sme
 }
 
 // ---------------------------------------------------------------------------------- kernel
-// Launched with programmatic stream serialization: the prologue, and (when p.w_ready) the
-// weight loads and decodes of the first ring slots, overlap the previous kernel; everything that
-// reads an activation or writes memory waits in griddep_wait() first.
+// Launched with programmatic stream serialization: the prologue and the weight loads and decodes
+// of the first ring slots overlap the previous kernel; everything that reads an activation or
+// writes memory waits in griddep_wait() first.
 template <bool TRANS, int NACC>
 __global__ void __launch_bounds__(THREADS, 1)
     dequant_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmP,
@@ -392,9 +391,10 @@ __global__ void __launch_bounds__(THREADS, 1)
           tma_load_2d(st + Ly::S_OFF, &tmS, &wfull[s], kt * BK, n0 / 64);   // scales [N/64, K]
         }
       };
+      // The packed weights are never written by a kernel of the same call (and the first kernel
+      // of a call is a normal launch), so the first slots' weights load before the wait.
       int w_issued = 0, a_issued = 0;
-      if (p.w_ready)
-        for (; w_issued < min(TSTG, num_main); ++w_issued) load_w(w_issued);
+      for (; w_issued < min(TSTG, num_main); ++w_issued) load_w(w_issued);
       griddep_wait();
       for (int it = 0; it < total; ++it) {
         const int s = it % TSTG;
@@ -569,9 +569,11 @@ int launch_variant(dim3 grid, const CUtensorMap& tA, const CUtensorMap& tP, cons
   cfg.stream = st;
   cudaLaunchAttribute at[2];
   int na = 0;
-  at[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  at[na].val.programmaticStreamSerializationAllowed = 1;
-  ++na;
+  if (pdl_take()) {
+    at[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+  }
   if (grid.z > 1) {
     at[na].id = cudaLaunchAttributeClusterDimension;
     at[na].val.clusterDim.x = 1;
@@ -652,8 +654,6 @@ int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st) {
   p.lse = g.lse;
   p.ce_w = g.ce_w;
   p.err = g.err;
-
-  p.w_ready = g.w_ready ? 1 : 0;
 
   const int tiles_n = static_cast<int>((g.N + BN - 1) / BN), tiles_m = static_cast<int>((g.M + bm - 1) / bm);
   const int num_k = static_cast<int>(g.K / BK);

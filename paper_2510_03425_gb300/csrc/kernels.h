@@ -5,12 +5,40 @@
 #include <stdint.h>
 
 #include <atomic>
+#include <utility>
 
 namespace mebp {
 
 // Process-wide count of kernel launches issued by the library (reported by mebp_kernel_launches).
 extern std::atomic<long long> g_launches;
 inline void count_launch(int n = 1) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+
+// Programmatic dependent launch (PDL).  Every kernel of the library starts with griddep_wait()
+// (and then griddep_launch()), so a kernel may be launched while its predecessor in the stream
+// still runs: its launch latency and prologue overlap the predecessor, and its first access to
+// memory still waits for the predecessor to complete.  The first kernel an entry point launches
+// is a normal launch (pdl_entry() marks it), so no kernel of one call overlaps an earlier call:
+// the fused GEMM may then read the packed weights before its wait (they are written only by
+// mebp_compress_weights, a separate call).
+void pdl_entry();   // the calling thread's next launch is a normal launch
+bool pdl_take();    // may this launch use PDL? (consumes the entry mark)
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                            Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = pdl_take() ? 1 : 0;
+  count_launch();
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 enum GemmEpi { EPI_F16 = 0, EPI_F32 = 1, EPI_LSE = 2, EPI_CEGRAD = 3 };
 
@@ -41,11 +69,6 @@ struct GemmArgs {
   float* zt = nullptr;
   const float* lse = nullptr;
   const float* ce_w = nullptr;   // EPI_CEGRAD: device scalar weight of a valid row
-  // The packed weights are not written by any kernel that may still be running when this GEMM
-  // starts, so they may be fetched and decoded before the previous kernel in the stream finishes.
-  // Holds whenever the kernel launched before the GEMM was itself launched normally after the
-  // weights were written (every entry point starts with such a kernel, or clears the flag).
-  bool w_ready = false;
   int* err = nullptr;
 };
 

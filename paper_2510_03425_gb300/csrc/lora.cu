@@ -20,6 +20,8 @@ template <int NT>
 __global__ void __launch_bounds__(128) skinny_gemm_kernel(const uint16_t* __restrict__ X, int64_t ldx, int64_t M,
                                                           int64_t K, const uint16_t* __restrict__ W, int64_t ldw,
                                                           float alpha, uint16_t* __restrict__ out, int64_t ldo) {
+  griddep_wait();
+  griddep_launch();
   constexpr int BMs = 64, BKs = 64, LDS = BKs + 8, JR = NT * 8;
   __shared__ __align__(16) uint16_t xs[2][BMs * LDS];
   __shared__ __align__(16) uint16_t ws[2][JR * LDS];
@@ -87,11 +89,11 @@ void launch_skinny_gemm(const uint16_t* X, int64_t ldx, int64_t M, int64_t K, co
   if (M <= 0) return;
   const unsigned grid = static_cast<unsigned>((M + 63) / 64);
   switch (ldo) {
-    case 16: count_launch(); skinny_gemm_kernel<2><<<grid, 128, 0, st>>>(X, ldx, M, K, W, ldw, alpha, out, ldo); break;
-    case 32: count_launch(); skinny_gemm_kernel<4><<<grid, 128, 0, st>>>(X, ldx, M, K, W, ldw, alpha, out, ldo); break;
-    case 48: count_launch(); skinny_gemm_kernel<6><<<grid, 128, 0, st>>>(X, ldx, M, K, W, ldw, alpha, out, ldo); break;
-    case 64: count_launch(); skinny_gemm_kernel<8><<<grid, 128, 0, st>>>(X, ldx, M, K, W, ldw, alpha, out, ldo); break;
-    default: count_launch(); skinny_gemm_kernel<12><<<grid, 128, 0, st>>>(X, ldx, M, K, W, ldw, alpha, out, ldo); break;
+    case 16: launch_k(skinny_gemm_kernel<2>, grid, 128, 0, st, X, ldx, M, K, W, ldw, alpha, out, ldo); break;
+    case 32: launch_k(skinny_gemm_kernel<4>, grid, 128, 0, st, X, ldx, M, K, W, ldw, alpha, out, ldo); break;
+    case 48: launch_k(skinny_gemm_kernel<6>, grid, 128, 0, st, X, ldx, M, K, W, ldw, alpha, out, ldo); break;
+    case 64: launch_k(skinny_gemm_kernel<8>, grid, 128, 0, st, X, ldx, M, K, W, ldw, alpha, out, ldo); break;
+    default: launch_k(skinny_gemm_kernel<12>, grid, 128, 0, st, X, ldx, M, K, W, ldw, alpha, out, ldo); break;
   }
 }
 
@@ -110,6 +112,8 @@ __global__ void __launch_bounds__(128) tall_reduce_kernel(const uint16_t* __rest
                                                           const uint16_t* __restrict__ Q, int64_t ldq, int64_t M,
                                                           int Pw, int Qw, int64_t m_per_split,
                                                           float* __restrict__ part, Direct dw) {
+  griddep_wait();
+  griddep_launch();
   constexpr int BP = 64, BMr = 64, QT = NQ * 8, LDP = BP + 8, LDQ = QT + 8;
   __shared__ __align__(16) uint16_t ps[2][BMr * LDP];
   __shared__ __align__(16) uint16_t qs[2][BMr * LDQ];
@@ -192,6 +196,8 @@ __global__ void __launch_bounds__(128) tall_reduce_kernel(const uint16_t* __rest
 // C[p * sp + q * sq] (+)= mult * sum_z part[z][p][q]  in split order.
 __global__ void split_sum_kernel(const float* __restrict__ part, int splits, int Pw, int Qw, float* __restrict__ C,
                                  int64_t sp, int64_t sq, int accumulate, const float* __restrict__ mult) {
+  griddep_wait();
+  griddep_launch();
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   const int64_t n = static_cast<int64_t>(Pw) * Qw;
   if (i >= n) return;
@@ -229,15 +235,14 @@ int launch_tall_reduce(const uint16_t* P, int64_t ldp, const uint16_t* Q, int64_
   Direct dw{nullptr, sp, sq, accumulate ? 1 : 0, mult};
   if (splits == 1) dw.C = C;
   switch (nq) {
-    case 4: count_launch(); tall_reduce_kernel<4><<<grid, 128, 0, st>>>(P, ldp, Q, ldq, M, Pw, Qw, mps, scratch, dw); break;
-    case 8: count_launch(); tall_reduce_kernel<8><<<grid, 128, 0, st>>>(P, ldp, Q, ldq, M, Pw, Qw, mps, scratch, dw); break;
-    default: count_launch(); tall_reduce_kernel<12><<<grid, 128, 0, st>>>(P, ldp, Q, ldq, M, Pw, Qw, mps, scratch, dw); break;
+    case 4: launch_k(tall_reduce_kernel<4>, grid, 128, 0, st, P, ldp, Q, ldq, M, Pw, Qw, mps, scratch, dw); break;
+    case 8: launch_k(tall_reduce_kernel<8>, grid, 128, 0, st, P, ldp, Q, ldq, M, Pw, Qw, mps, scratch, dw); break;
+    default: launch_k(tall_reduce_kernel<12>, grid, 128, 0, st, P, ldp, Q, ldq, M, Pw, Qw, mps, scratch, dw); break;
   }
   if (dw.C) return MEBP_OK;
   const int64_t n = static_cast<int64_t>(Pw) * Qw;
-  count_launch();
-  split_sum_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(scratch, static_cast<int>(splits), Pw, Qw,
-                                                                           C, sp, sq, accumulate ? 1 : 0, mult);
+  launch_k(split_sum_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, st, scratch, static_cast<int>(splits), Pw,
+           Qw, C, sp, sq, accumulate ? 1 : 0, mult);
   return MEBP_OK;
 }
 
@@ -253,6 +258,8 @@ struct ShadowArgs {
 
 __global__ void lora_shadow_kernel(ShadowArgs a, int r, int K, int N, int kx, uint16_t* __restrict__ A_cat,
                                    uint16_t* __restrict__ B_cat, uint16_t* __restrict__ Bt_cat) {
+  griddep_wait();
+  griddep_launch();
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   const int64_t na = static_cast<int64_t>(kx) * K, nb = static_cast<int64_t>(N) * kx;
   if (i < na) {
@@ -287,8 +294,8 @@ void launch_lora_shadow(const float* const* A, const float* const* B, int nt, co
     a.nl[t] = n_len[t];
   }
   const int64_t n = std::max(static_cast<int64_t>(kx) * K, static_cast<int64_t>(N) * kx);
-  count_launch();
-  lora_shadow_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(a, r, K, N, kx, A_cat, B_cat, Bt_cat);
+  launch_k(lora_shadow_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, st, a, r, K, N, kx, A_cat, B_cat,
+           Bt_cat);
 }
 
 }  // namespace mebp

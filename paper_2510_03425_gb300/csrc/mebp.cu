@@ -37,6 +37,15 @@ struct ProfRec {
 }  // namespace
 
 std::atomic<long long> mebp::g_launches{0};
+namespace {
+thread_local bool t_pdl_entry = false;
+}
+void mebp::pdl_entry() { t_pdl_entry = true; }
+bool mebp::pdl_take() {
+  const bool ok = !t_pdl_entry;
+  t_pdl_entry = false;
+  return ok;
+}
 
 struct mebp_ctx {
   mebp_model_cfg cfg{};
@@ -183,7 +192,6 @@ GemmArgs gemm_fwd(const uint16_t* X, int64_t ldx, int64_t M, const mebp_packed& 
   g.qpack = W.qpack;
   g.scales = W.scales;
   g.scale_pitch = W.rows;
-  g.w_ready = true;  // model weights: written only by mebp_compress_weights, before any step
   return g;
 }
 // dX = dY deq(W) for W [N_w, K_w] stored packed: GEMM K = N_w (reduction), N = K_w (output).
@@ -198,7 +206,6 @@ GemmArgs gemm_dx(const uint16_t* dY, int64_t ldy, int64_t M, const mebp_packed& 
   g.qpack = W.qpack;
   g.scales = W.scales;
   g.scale_pitch = W.rows;
-  g.w_ready = true;  // model weights: written only by mebp_compress_weights, before any step
   return g;
 }
 
@@ -429,7 +436,6 @@ int lmhead(mebp_ctx* c, const mebp_packed* E, const float* gf, const float* h, c
     t.A = c->dz; t.lda = c->vchunk; t.M = T; t.N = D; t.K = n;
     t.qpack = Ec.qpack; t.scales = Ec.scales; t.scale_pitch = V;
     t.epi = EPI_F32; t.C = c->dhf; t.ldc = D; t.R = c0 ? c->dhf : nullptr; t.ldr = D; t.alpha = 1.0f / kCeShift;
-    t.w_ready = true;
     if ((rc = run_gemm(c, t, st, "LM head (dH pass)"))) return rc;
   }
   launch_rmsnorm_bwd(c->dhf, h, gf, c->rf, nullptr, T, D, unscale_dh ? c->scal + 1 : nullptr, dh, dh_h, st);
@@ -437,6 +443,8 @@ int lmhead(mebp_ctx* c, const mebp_packed* E, const float* gf, const float* h, c
 }
 
 __global__ void targets_kernel(const int32_t* ids, int B, int Sq, int32_t* tg) {
+  griddep_wait();
+  griddep_launch();
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (i >= static_cast<int64_t>(B) * Sq) return;
   const int s = static_cast<int>(i % Sq);
@@ -670,6 +678,7 @@ int mebp_compress_weights(mebp_ctx* c, const float* W, int64_t rows, int64_t col
   if (group != 64) return fail(c, MEBP_ERR_UNSUPPORTED, "group must be 64");
   if (rows <= 0 || cols <= 0 || cols % 64) return fail(c, MEBP_ERR_INVALID_ARG, "cols must be a positive multiple of 64");
   if (reinterpret_cast<uintptr_t>(W) & 7) return fail(c, MEBP_ERR_INVALID_ARG, "W must be 8-byte aligned");
+  pdl_entry();
   launch_compress(W, rows, cols, qpack, scales, S(stream));
   return cuda_check(c, "compress");
 }
@@ -679,6 +688,7 @@ int mebp_decode_weights(mebp_ctx* c, const mebp_packed* w, uint16_t* out, void* 
   if (!w || !w->qpack || !w->scales || !out) return fail(c, MEBP_ERR_INVALID_ARG, "NULL pointer");
   if (w->rows <= 0 || w->cols <= 0 || w->cols % 64) return fail(c, MEBP_ERR_INVALID_ARG, "bad shape");
   if (!aligned16(w->qpack) || !aligned16(out)) return fail(c, MEBP_ERR_INVALID_ARG, "pointers must be 16-byte aligned");
+  pdl_entry();
   launch_decode(w->qpack, w->scales, w->rows, w->cols, out, S(stream));
   return cuda_check(c, "decode");
 }
@@ -690,6 +700,7 @@ int mebp_embed(mebp_ctx* c, const mebp_packed* E, const int32_t* ids, int64_t n,
   if (!aligned16(x0) || (reinterpret_cast<uintptr_t>(E->qpack) & 3))
     return fail(c, MEBP_ERR_INVALID_ARG, "misaligned pointer");
   if (n <= 0) return MEBP_OK;
+  pdl_entry();
   launch_embed(E->qpack, E->scales, E->rows, E->cols, ids, n, x0, c->d_err, S(stream));
   return cuda_check(c, "embed");
 }
@@ -707,6 +718,7 @@ static int linear_common(mebp_ctx* c, bool dx_mode, const uint16_t* X, int64_t M
   if (A && (r <= 0 || r > 32 || r % 8)) return fail(c, MEBP_ERR_UNSUPPORTED, "rank must be 8, 16, 24 or 32");
   if (M <= 0) return MEBP_OK;
   const int kxp = A ? (r + 15) / 16 * 16 : 0;
+  pdl_entry();
   uint16_t *Ac = nullptr, *Bc = nullptr, *Btc = nullptr, *u = nullptr;
   if (A) {
     const size_t bytes = (static_cast<size_t>(kxp) * K + 2 * static_cast<size_t>(N) * kxp + M * kxp) * 2;
@@ -745,7 +757,6 @@ static int linear_common(mebp_ctx* c, bool dx_mode, const uint16_t* X, int64_t M
     }
     g.epi = EPI_F32; g.C = y32; g.ldc = K; g.R = R; g.ldr = K;
   }
-  g.w_ready = false;  // the caller may have written W with the kernel just before this one
   int rc = run_gemm(c, g, st, dx_mode ? "linear dX" : "linear forward");
   if (A) cudaFreeAsync(Ac, st);
   if (rc) return rc;
@@ -773,6 +784,7 @@ int mebp_block_recompute_fwd(mebp_ctx* c, int layer, const mebp_block_weights* w
   if ((rc = check_tokens(c, B, Sq)) || (rc = check_block_ptrs(c, w)) || (rc = check_lora(c, lora))) return rc;
   if (!x || !y || !aligned16(x) || !aligned16(y)) return fail(c, MEBP_ERR_INVALID_ARG, "x / y must be 16-byte aligned");
   if (x == y) return fail(c, MEBP_ERR_INVALID_ARG, "x and y must not alias");
+  pdl_entry();
   rc = block_forward(c, layer, w, lora, x, y, B, Sq, true, S(stream));
   if (!save_for_bwd) c->saved_layer = -1;
   return rc;
@@ -789,6 +801,7 @@ int mebp_block_bwd(mebp_ctx* c, int layer, const mebp_block_weights* w, const me
   cudaStream_t st = S(stream);
   const int64_t n = static_cast<int64_t>(B) * Sq * c->D;
   // working scale for this call: sigma = 2^-floor(log2(max|dy|)); the outputs are scaled back
+  pdl_entry();
   launch_grad_scale(dy, n, c->scal + 4, st);
   launch_scale_cast(dy, n, c->scal + 4, c->gbuf[0], c->dy_h[1], st);
   return block_backward(c, layer, w, lora, x, c->gbuf[0], c->dy_h[1], dx, nullptr, grads, B, Sq, accumulate != 0,
@@ -804,6 +817,7 @@ int mebp_lmhead_ce_fwd_bwd(mebp_ctx* c, const mebp_packed* E, const float* gf, c
   if (!gf || !h || !targets || !loss || !dh) return fail(c, MEBP_ERR_INVALID_ARG, "NULL pointer");
   if (T <= 0 || T > c->Tmax) return fail(c, MEBP_ERR_INVALID_ARG, "n_tokens out of range");
   if (!aligned16(h) || !aligned16(dh)) return fail(c, MEBP_ERR_INVALID_ARG, "h / dh must be 16-byte aligned");
+  pdl_entry();
   return lmhead(c, E, gf, h, targets, T, loss, dh, nullptr, token_loss, true, S(stream));
 }
 
@@ -814,8 +828,8 @@ static int lora_step_body(mebp_ctx* c, const mebp_model_weights* model, const me
   const int64_t T = static_cast<int64_t>(B) * Sq, D = c->D;
   const int L = c->L;
   const bool spill = c->cfg.spill_ckpts != 0;
-  count_launch();
-  targets_kernel<<<static_cast<unsigned>((T + 255) / 256), 256, 0, st>>>(ids, B, Sq, c->targets);
+  pdl_entry();
+  launch_k(targets_kernel, static_cast<unsigned>((T + 255) / 256), 256, 0, st, ids, B, Sq, c->targets);
   // Checkpoint placement (Algorithm 1's ckpts_storage): HBM slot i, or, when spilling, a ring
   // of kCkptSlots device slots whose contents are copied to / from pinned host memory on a
   // side stream (the stand-in for memory-mapped checkpoints).

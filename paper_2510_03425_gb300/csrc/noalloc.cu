@@ -79,6 +79,7 @@ extern "C" int mebp_linear_fwd_noalloc(const uint16_t* X, int64_t M, const mebp_
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   int* err = reinterpret_cast<int*>(scratch);
   cudaMemsetAsync(err, 0, sizeof(int), st);  // the only scratch that must start at zero
+  pdl_entry();  // no kernel of this call overlaps work issued before it
 
   GemmArgs g;
   g.trans = false;

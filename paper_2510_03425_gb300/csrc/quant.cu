@@ -11,6 +11,8 @@ namespace mebp {
 // when s == 0, u = q + 8.
 __global__ void compress_kernel(const float* __restrict__ W, int64_t rows, int64_t cols,
                                 uint8_t* __restrict__ qpack, uint16_t* __restrict__ scales) {
+  griddep_wait();
+  griddep_launch();
   const int64_t groups = cols / 64;
   const int64_t gw = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
@@ -38,6 +40,8 @@ __global__ void compress_kernel(const float* __restrict__ W, int64_t rows, int64
 // Decode every 8-column word with the GEMM's operand transform.
 __global__ void decode_kernel(const uint8_t* __restrict__ qpack, const uint16_t* __restrict__ scales, int64_t rows,
                               int64_t cols, uint16_t* __restrict__ out) {
+  griddep_wait();
+  griddep_launch();
   const int64_t words_per_row = cols / 8;
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (i >= rows * words_per_row) return;
@@ -52,6 +56,8 @@ __global__ void decode_kernel(const uint8_t* __restrict__ qpack, const uint16_t*
 __global__ void embed_kernel(const uint8_t* __restrict__ qpack, const uint16_t* __restrict__ scales, int64_t V,
                              int64_t D, const int32_t* __restrict__ ids, int64_t T, float* __restrict__ x0,
                              int* err) {
+  griddep_wait();
+  griddep_launch();
   const int64_t t = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (t >= T) return;
@@ -77,22 +83,19 @@ __global__ void embed_kernel(const uint8_t* __restrict__ qpack, const uint16_t* 
 void launch_compress(const float* W, int64_t rows, int64_t cols, uint8_t* qpack, uint16_t* scales, cudaStream_t st) {
   const int64_t warps = rows * (cols / 64);
   const int64_t blocks = (warps * 32 + 255) / 256;
-  count_launch();
-  compress_kernel<<<static_cast<unsigned>(blocks), 256, 0, st>>>(W, rows, cols, qpack, scales);
+  launch_k(compress_kernel, static_cast<unsigned>(blocks), 256, 0, st, W, rows, cols, qpack, scales);
 }
 
 void launch_decode(const uint8_t* qpack, const uint16_t* scales, int64_t rows, int64_t cols, uint16_t* out,
                    cudaStream_t st) {
   const int64_t n = rows * (cols / 8);
-  count_launch();
-  decode_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(qpack, scales, rows, cols, out);
+  launch_k(decode_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, st, qpack, scales, rows, cols, out);
 }
 
 void launch_embed(const uint8_t* qpack, const uint16_t* scales, int64_t V, int64_t D, const int32_t* ids, int64_t T,
                   float* x0, int* err, cudaStream_t st) {
   const int64_t blocks = (T * 32 + 255) / 256;
-  count_launch();
-  embed_kernel<<<static_cast<unsigned>(blocks), 256, 0, st>>>(qpack, scales, V, D, ids, T, x0, err);
+  launch_k(embed_kernel, static_cast<unsigned>(blocks), 256, 0, st, qpack, scales, V, D, ids, T, x0, err);
 }
 
 }  // namespace mebp

@@ -13,6 +13,8 @@ namespace mebp {
 // y = x / sqrt(mean(x^2) + eps) * g  ->  fp16 (the GEMM operand); rstd saved for the backward.
 __global__ void rmsnorm_fwd_kernel(const float* __restrict__ x, const float* __restrict__ g, int64_t T, int D,
                                    float eps, uint16_t* __restrict__ y, float* __restrict__ rstd) {
+  griddep_wait();
+  griddep_launch();
   const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (row >= T) return;
@@ -39,6 +41,8 @@ __global__ void rmsnorm_bwd_kernel(const float* __restrict__ dy, const float* __
                                    const float* __restrict__ g, const float* __restrict__ rstd,
                                    const float* __restrict__ resid, int64_t T, int D, const float* __restrict__ mult,
                                    float* __restrict__ dx, uint16_t* __restrict__ dxb) {
+  griddep_wait();
+  griddep_launch();
   const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (row >= T) return;
@@ -74,15 +78,13 @@ __global__ void rmsnorm_bwd_kernel(const float* __restrict__ dy, const float* __
 void launch_rmsnorm_fwd(const float* x, const float* g, int64_t T, int D, float eps, uint16_t* y, float* rstd,
                         cudaStream_t st) {
   if (T <= 0) return;
-  count_launch();
-  rmsnorm_fwd_kernel<<<static_cast<unsigned>((T * 32 + 255) / 256), 256, 0, st>>>(x, g, T, D, eps, y, rstd);
+  launch_k(rmsnorm_fwd_kernel, static_cast<unsigned>((T * 32 + 255) / 256), 256, 0, st, x, g, T, D, eps, y, rstd);
 }
 void launch_rmsnorm_bwd(const float* dy, const float* x, const float* g, const float* rstd, const float* resid,
                         int64_t T, int D, const float* out_mult, float* dx, uint16_t* dxb, cudaStream_t st) {
   if (T <= 0) return;
-  count_launch();
-  rmsnorm_bwd_kernel<<<static_cast<unsigned>((T * 32 + 255) / 256), 256, 0, st>>>(dy, x, g, rstd, resid, T, D,
-                                                                                   out_mult, dx, dxb);
+  launch_k(rmsnorm_bwd_kernel, static_cast<unsigned>((T * 32 + 255) / 256), 256, 0, st, dy, x, g, rstd, resid, T, D,
+           out_mult, dx, dxb);
 }
 
 // ------------------------------------------------------------------------------------ RoPE
@@ -90,6 +92,8 @@ void launch_rmsnorm_bwd(const float* dy, const float* x, const float* g, const f
 // inverse rotates by -angle (the VJP).  One thread per (token, head, pair of j).
 __global__ void rope_kernel(uint16_t* __restrict__ qkv, int64_t T, int S, int nheads, int ld, int hd,
                             const float2* __restrict__ cs, int inverse) {
+  griddep_wait();
+  griddep_launch();
   const int half = hd >> 1, pairs = half >> 1;
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (i >= T * nheads * pairs) return;
@@ -116,9 +120,8 @@ void launch_rope(uint16_t* qkv, int64_t T, int S, int H, int KV, int hd, const f
   const int nheads = H + KV;  // q heads then k heads
   const int64_t n = T * nheads * (hd / 4);
   if (n <= 0) return;
-  count_launch();
-  rope_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(qkv, T, S, nheads, (H + 2 * KV) * hd, hd, cs,
-                                                                      inverse ? 1 : 0);
+  launch_k(rope_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, st, qkv, T, S, nheads, (H + 2 * KV) * hd, hd,
+           cs, inverse ? 1 : 0);
 }
 
 // ------------------------------------------------------------------------------------ gated MLP
@@ -139,6 +142,8 @@ __device__ __forceinline__ float act_grad(float x, int act) {
 
 // m = act(g) * u; gu row = [g (I) | u (I)].  8 elements per thread.
 __global__ void glu_fwd_kernel(const uint16_t* __restrict__ gu, int64_t T, int I, int act, uint16_t* __restrict__ m) {
+  griddep_wait();
+  griddep_launch();
   const int per = I / 8;
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (i >= T * per) return;
@@ -157,6 +162,8 @@ __global__ void glu_fwd_kernel(const uint16_t* __restrict__ gu, int64_t T, int I
 // dg = dm * u * act'(g), du = dm * act(g)
 __global__ void glu_bwd_kernel(const float* __restrict__ dm, const uint16_t* __restrict__ gu, int64_t T, int I, int act,
                                uint16_t* __restrict__ dgu) {
+  griddep_wait();
+  griddep_launch();
   const int per = I / 8;
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (i >= T * per) return;
@@ -182,19 +189,19 @@ __global__ void glu_bwd_kernel(const float* __restrict__ dm, const uint16_t* __r
 void launch_glu_fwd(const uint16_t* gu, int64_t T, int I, int act, uint16_t* m, cudaStream_t st) {
   const int64_t n = T * (I / 8);
   if (n <= 0) return;
-  count_launch();
-  glu_fwd_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(gu, T, I, act, m);
+  launch_k(glu_fwd_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, st, gu, T, I, act, m);
 }
 void launch_glu_bwd(const float* dm, const uint16_t* gu, int64_t T, int I, int act, uint16_t* dgu, cudaStream_t st) {
   const int64_t n = T * (I / 8);
   if (n <= 0) return;
-  count_launch();
-  glu_bwd_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(dm, gu, T, I, act, dgu);
+  launch_k(glu_bwd_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, st, dm, gu, T, I, act, dgu);
 }
 
 // ------------------------------------------------------------------------------------ casts
 __global__ void scale_cast_kernel(const float* __restrict__ x, int64_t n4, const float* __restrict__ scale,
                                   float* __restrict__ y32, uint16_t* __restrict__ y16) {
+  griddep_wait();
+  griddep_launch();
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (i >= n4) return;
   const float sc = scale ? *scale : 1.0f;
@@ -206,6 +213,8 @@ __global__ void scale_cast_kernel(const float* __restrict__ x, int64_t n4, const
 // max |x| into *amax_bits (as the bit pattern of a non-negative float; atomicMax on the
 // integer view is order independent, so the result is deterministic).
 __global__ void amax_kernel(const float* __restrict__ x, int64_t n, unsigned int* __restrict__ amax_bits) {
+  griddep_wait();
+  griddep_launch();
   float m = 0.0f;
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x)
@@ -215,6 +224,8 @@ __global__ void amax_kernel(const float* __restrict__ x, int64_t n, unsigned int
 }
 // sigma = 2^-floor(log2(amax)) so that max|x * sigma| lies in [1, 2); 1 when amax is 0 or not finite.
 __global__ void sigma_kernel(float* scal) {
+  griddep_wait();
+  griddep_launch();
   const float amax = __uint_as_float(reinterpret_cast<unsigned int*>(scal)[2]);
   float sg = 1.0f;
   if (amax > 0.0f && amax < INFINITY) sg = exp2f(-floorf(log2f(amax)));
@@ -224,25 +235,24 @@ __global__ void sigma_kernel(float* scal) {
 void launch_scale_cast(const float* x, int64_t n, const float* scale, float* y32, uint16_t* y16, cudaStream_t st) {
   const int64_t n4 = n / 4;
   if (n4 <= 0) return;
-  count_launch();
-  scale_cast_kernel<<<static_cast<unsigned>((n4 + 255) / 256), 256, 0, st>>>(x, n4, scale, y32, y16);
+  launch_k(scale_cast_kernel, static_cast<unsigned>((n4 + 255) / 256), 256, 0, st, x, n4, scale, y32, y16);
 }
 void launch_grad_scale(const float* x, int64_t n, float* scal, cudaStream_t st) {
   cudaMemsetAsync(scal + 2, 0, sizeof(float), st);
-  count_launch(2);
   const int64_t blocks = std::min<int64_t>(1184, (n + 255) / 256);
-  amax_kernel<<<static_cast<unsigned>(std::max<int64_t>(1, blocks)), 256, 0, st>>>(
-      x, n, reinterpret_cast<unsigned int*>(scal + 2));
-  sigma_kernel<<<1, 1, 0, st>>>(scal);
+  launch_k(amax_kernel, static_cast<unsigned>(std::max<int64_t>(1, blocks)), 256, 0, st, x, n,
+           reinterpret_cast<unsigned int*>(scal + 2));
+  launch_k(sigma_kernel, 1, 1, 0, st, scal);
 }
 __global__ void fill_kernel(float* __restrict__ x, int64_t n, float v) {
+  griddep_wait();
+  griddep_launch();
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (i < n) x[i] = v;
 }
 void launch_fill_f32(float* x, int64_t n, float v, cudaStream_t st) {
   if (n <= 0) return;
-  count_launch();
-  fill_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(x, n, v);
+  launch_k(fill_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, st, x, n, v);
 }
 
 // ------------------------------------------------------------------------------------ LM head
@@ -251,6 +261,8 @@ void launch_fill_f32(float* x, int64_t n, float v, cudaStream_t st) {
 __global__ void lse_combine_kernel(const float2* __restrict__ part, int nparts, const float* __restrict__ zt,
                                    const int32_t* __restrict__ targets, int64_t T, float* __restrict__ lse,
                                    float* __restrict__ tok_loss) {
+  griddep_wait();
+  griddep_launch();
   const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (row >= T) return;
@@ -276,6 +288,8 @@ __global__ void lse_combine_kernel(const float2* __restrict__ part, int nparts, 
 // sigma keeps fp16 operands in range), 1/sigma, and the CE-gradient row weight sigma*shift/n.
 __global__ void loss_reduce_kernel(const float* __restrict__ tok_loss, const int32_t* __restrict__ targets, int64_t T,
                                    float* __restrict__ loss, float* __restrict__ scal) {
+  griddep_wait();
+  griddep_launch();
   __shared__ double ssum[1024];
   __shared__ int scnt[1024];
   double s = 0.0;
@@ -308,14 +322,12 @@ __global__ void loss_reduce_kernel(const float* __restrict__ tok_loss, const int
 void launch_lse_combine(const float* part, int nparts, const float* zt, const int32_t* targets, int64_t T, float* lse,
                         float* tok_loss, cudaStream_t st) {
   if (T <= 0) return;
-  count_launch();
-  lse_combine_kernel<<<static_cast<unsigned>((T * 32 + 255) / 256), 256, 0, st>>>(
-      reinterpret_cast<const float2*>(part), nparts, zt, targets, T, lse, tok_loss);
+  launch_k(lse_combine_kernel, static_cast<unsigned>((T * 32 + 255) / 256), 256, 0, st,
+           reinterpret_cast<const float2*>(part), nparts, zt, targets, T, lse, tok_loss);
 }
 void launch_loss_reduce(const float* tok_loss, const int32_t* targets, int64_t T, float* loss, float* scal,
                         cudaStream_t st) {
-  count_launch();
-  loss_reduce_kernel<<<1, 1024, 0, st>>>(tok_loss, targets, T, loss, scal);
+  launch_k(loss_reduce_kernel, 1, 1024, 0, st, tok_loss, targets, T, loss, scal);
 }
 
 }  // namespace mebp
