@@ -47,6 +47,20 @@ bool mebp::pdl_take() {
   return ok;
 }
 
+// One block's forward intermediates (what the backward consumes) and the fp16 LoRA shadows they
+// were computed with.  The step keeps two sets so that the recompute of block i-1 can run on a
+// second stream while the backward of block i reads the other set.
+struct Acts {
+  uint16_t *a = nullptr, *qkv = nullptr, *o = nullptr, *b = nullptr, *gu = nullptr, *m = nullptr;
+  float *r1 = nullptr, *r2 = nullptr, *lse_attn = nullptr, *h1 = nullptr;
+  uint16_t* us[4] = {nullptr, nullptr, nullptr, nullptr};
+  uint16_t *A_cat[4] = {}, *B_cat[4] = {}, *Bt_cat[4] = {};
+  // which block / input / token count the set currently holds (-1: none)
+  int layer = -1;
+  const float* x = nullptr;
+  int64_t T = -1;
+};
+
 struct mebp_ctx {
   mebp_model_cfg cfg{};
   int device = 0;
@@ -64,12 +78,13 @@ struct mebp_ctx {
   int64_t ws_bytes = 0;
 
   float2* rope_cs = nullptr;
-  // one block's intermediates
-  uint16_t *a = nullptr, *qkv = nullptr, *o = nullptr, *b = nullptr, *gu = nullptr, *m = nullptr;
-  float *r1 = nullptr, *r2 = nullptr, *lse_attn = nullptr, *h1 = nullptr;
-  uint16_t* us[4] = {nullptr, nullptr, nullptr, nullptr};
+  // forward intermediates: set 0 always, set 1 when the step overlaps recompute and backward
+  Acts act[2];
+  int nsets = 1;
+  cudaStream_t fstream = nullptr;  // recompute stream of the overlapped backward
+  cudaEvent_t ev_main = nullptr;   // main-stream progress, waited on by the recompute stream
+  cudaEvent_t ev_fwd[2] = {};      // recompute into set k finished
   uint16_t* du[4] = {nullptr, nullptr, nullptr, nullptr};
-  uint16_t *A_cat[4] = {}, *B_cat[4] = {}, *Bt_cat[4] = {};
   // backward
   uint16_t *dqkv = nullptr, *dout = nullptr, *dgu = nullptr, *dh1_h = nullptr, *dy_h[2] = {nullptr, nullptr};
   float *dm = nullptr, *dtmp = nullptr, *dh1 = nullptr, *dvec = nullptr, *gbuf[2] = {nullptr, nullptr};
@@ -101,10 +116,6 @@ struct mebp_ctx {
   std::vector<ProfRec> recs;
   std::vector<cudaEvent_t> evpool;
   size_t evnext = 0;
-  // intermediates tag
-  int saved_layer = -1;
-  const float* saved_x = nullptr;
-  int64_t saved_T = -1;
 };
 
 namespace {
@@ -238,16 +249,16 @@ int run_gemm(mebp_ctx* c, GemmArgs& g, cudaStream_t st, const char* what) {
 }
 
 // fp16 shadows of one fused linear's LoRA masters.
-void build_shadow(mebp_ctx* c, int li, const mebp_lora* lora, cudaStream_t st) {
+void build_shadow(mebp_ctx* c, Acts& A, int li, const mebp_lora* lora, cudaStream_t st) {
   const Lin& l = c->lin[li];
   if (!l.kx) return;
-  const float* A[3];
-  const float* B[3];
+  const float* As[3];
+  const float* Bs[3];
   for (int t = 0; t < l.nt; ++t) {
-    A[t] = lora->A[l.tgt[t]];
-    B[t] = lora->B[l.tgt[t]];
+    As[t] = lora->A[l.tgt[t]];
+    Bs[t] = lora->B[l.tgt[t]];
   }
-  launch_lora_shadow(A, B, l.nt, l.ro, l.no, l.nl, c->r, l.K, l.N, l.kxp, c->A_cat[li], c->B_cat[li], c->Bt_cat[li],
+  launch_lora_shadow(As, Bs, l.nt, l.ro, l.no, l.nl, c->r, l.K, l.N, l.kxp, A.A_cat[li], A.B_cat[li], A.Bt_cat[li],
                      st);
 }
 
@@ -263,68 +274,69 @@ int check_lora(mebp_ctx* c, const mebp_lora* lora) {
 
 // y = F(x) for one block.  with_down == false stops after the MLP activation (what the
 // backward consumes), so y is not produced.
-int block_forward(mebp_ctx* c, int layer, const mebp_block_weights* w, const mebp_lora* lora, const float* x, float* y,
-                  int B, int Sq, bool with_down, cudaStream_t st) {
+int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, const mebp_lora* lora, const float* x,
+                  float* y, int B, int Sq, bool with_down, cudaStream_t st) {
+  Acts& A = c->act[set];
   const int64_t T = static_cast<int64_t>(B) * Sq;
   const int D = c->D, I = c->I;
   int rc;
-  for (int li = 0; li < 4; ++li) build_shadow(c, li, lora, st);
+  for (int li = 0; li < 4; ++li) build_shadow(c, A, li, lora, st);
   // attention sub-block
-  launch_rmsnorm_fwd(x, w->norm1, T, D, c->cfg.rms_eps, c->a, c->r1, st);
+  launch_rmsnorm_fwd(x, w->norm1, T, D, c->cfg.rms_eps, A.a, A.r1, st);
   const Lin& lq = c->lin[LIN_QKV];
-  GemmArgs g = gemm_fwd(c->a, D, T, w->qkv, lq.N, lq.K);
+  GemmArgs g = gemm_fwd(A.a, D, T, w->qkv, lq.N, lq.K);
   if (lq.kx) {
-    launch_skinny_gemm(c->a, D, T, D, c->A_cat[LIN_QKV], D, lq.kx, c->s, c->us[LIN_QKV], lq.kxp, st);
-    g.Ax = c->us[LIN_QKV]; g.ldax = lq.kxp; g.kx = lq.kxp; g.Bx = c->B_cat[LIN_QKV]; g.ldbx = lq.kxp;
+    launch_skinny_gemm(A.a, D, T, D, A.A_cat[LIN_QKV], D, lq.kx, c->s, A.us[LIN_QKV], lq.kxp, st);
+    g.Ax = A.us[LIN_QKV]; g.ldax = lq.kxp; g.kx = lq.kxp; g.Bx = A.B_cat[LIN_QKV]; g.ldbx = lq.kxp;
   }
-  g.epi = EPI_F16; g.C = c->qkv; g.ldc = lq.N;
+  g.epi = EPI_F16; g.C = A.qkv; g.ldc = lq.N;
   if ((rc = run_gemm(c, g, st, "qkv"))) return rc;
-  launch_rope(c->qkv, T, Sq, c->H, c->KV, c->hd, c->rope_cs, false, st);
-  launch_attn_fwd(c->qkv, lq.N, B, Sq, c->H, c->KV, c->hd, c->o, c->Na, c->lse_attn, st);
+  launch_rope(A.qkv, T, Sq, c->H, c->KV, c->hd, c->rope_cs, false, st);
+  launch_attn_fwd(A.qkv, lq.N, B, Sq, c->H, c->KV, c->hd, A.o, c->Na, A.lse_attn, st);
   const Lin& lo = c->lin[LIN_O];
-  g = gemm_fwd(c->o, c->Na, T, w->o, lo.N, lo.K);
+  g = gemm_fwd(A.o, c->Na, T, w->o, lo.N, lo.K);
   if (lo.kx) {
-    launch_skinny_gemm(c->o, c->Na, T, c->Na, c->A_cat[LIN_O], c->Na, lo.kx, c->s, c->us[LIN_O], lo.kxp, st);
-    g.Ax = c->us[LIN_O]; g.ldax = lo.kxp; g.kx = lo.kxp; g.Bx = c->B_cat[LIN_O]; g.ldbx = lo.kxp;
+    launch_skinny_gemm(A.o, c->Na, T, c->Na, A.A_cat[LIN_O], c->Na, lo.kx, c->s, A.us[LIN_O], lo.kxp, st);
+    g.Ax = A.us[LIN_O]; g.ldax = lo.kxp; g.kx = lo.kxp; g.Bx = A.B_cat[LIN_O]; g.ldbx = lo.kxp;
   }
-  g.epi = EPI_F32; g.C = c->h1; g.ldc = D; g.R = x; g.ldr = D;
+  g.epi = EPI_F32; g.C = A.h1; g.ldc = D; g.R = x; g.ldr = D;
   if ((rc = run_gemm(c, g, st, "o_proj"))) return rc;
   // MLP sub-block
-  launch_rmsnorm_fwd(c->h1, w->norm2, T, D, c->cfg.rms_eps, c->b, c->r2, st);
+  launch_rmsnorm_fwd(A.h1, w->norm2, T, D, c->cfg.rms_eps, A.b, A.r2, st);
   const Lin& lg = c->lin[LIN_GU];
-  g = gemm_fwd(c->b, D, T, w->gate_up, lg.N, lg.K);
+  g = gemm_fwd(A.b, D, T, w->gate_up, lg.N, lg.K);
   if (lg.kx) {
-    launch_skinny_gemm(c->b, D, T, D, c->A_cat[LIN_GU], D, lg.kx, c->s, c->us[LIN_GU], lg.kxp, st);
-    g.Ax = c->us[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = c->B_cat[LIN_GU]; g.ldbx = lg.kxp;
+    launch_skinny_gemm(A.b, D, T, D, A.A_cat[LIN_GU], D, lg.kx, c->s, A.us[LIN_GU], lg.kxp, st);
+    g.Ax = A.us[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = A.B_cat[LIN_GU]; g.ldbx = lg.kxp;
   }
-  g.epi = EPI_F16; g.C = c->gu; g.ldc = lg.N;
+  g.epi = EPI_F16; g.C = A.gu; g.ldc = lg.N;
   if ((rc = run_gemm(c, g, st, "gate_up"))) return rc;
-  launch_glu_fwd(c->gu, T, I, c->cfg.act, c->m, st);
+  launch_glu_fwd(A.gu, T, I, c->cfg.act, A.m, st);
   const Lin& ld = c->lin[LIN_DOWN];
-  if (ld.kx) launch_skinny_gemm(c->m, I, T, I, c->A_cat[LIN_DOWN], I, ld.kx, c->s, c->us[LIN_DOWN], ld.kxp, st);
+  if (ld.kx) launch_skinny_gemm(A.m, I, T, I, A.A_cat[LIN_DOWN], I, ld.kx, c->s, A.us[LIN_DOWN], ld.kxp, st);
   if (with_down) {
-    g = gemm_fwd(c->m, I, T, w->down, ld.N, ld.K);
+    g = gemm_fwd(A.m, I, T, w->down, ld.N, ld.K);
     if (ld.kx) {
-      g.Ax = c->us[LIN_DOWN]; g.ldax = ld.kxp; g.kx = ld.kxp; g.Bx = c->B_cat[LIN_DOWN]; g.ldbx = ld.kxp;
+      g.Ax = A.us[LIN_DOWN]; g.ldax = ld.kxp; g.kx = ld.kxp; g.Bx = A.B_cat[LIN_DOWN]; g.ldbx = ld.kxp;
     }
-    g.epi = EPI_F32; g.C = y; g.ldc = D; g.R = c->h1; g.ldr = D;
+    g.epi = EPI_F32; g.C = y; g.ldc = D; g.R = A.h1; g.ldr = D;
     if ((rc = run_gemm(c, g, st, "down"))) return rc;
   }
-  c->saved_layer = layer;
-  c->saved_x = x;
-  c->saved_T = T;
+  A.layer = layer;
+  A.x = x;
+  A.T = T;
   return cuda_check(c, "block forward");
 }
 
 // LoRA gradients of one fused linear: dB_t = dY[:, rows_t]^T U_s[:, ranks_t], dA_t = dU[:, ranks_t]^T X.
-int lin_grads(mebp_ctx* c, int li, const uint16_t* dY, int64_t ldy, const uint16_t* X, int64_t ldx, int64_t T,
-              const mebp_lora_grads* grads, bool acc, const float* grad_mult, cudaStream_t st) {
+int lin_grads(mebp_ctx* c, const Acts& A, int li, const uint16_t* dY, int64_t ldy, const uint16_t* X, int64_t ldx,
+              int64_t T, const mebp_lora_grads* grads, bool acc, const float* grad_mult, cudaStream_t st) {
   const Lin& l = c->lin[li];
   for (int t = 0; t < l.nt; ++t) {
     const int tg = l.tgt[t];
     if (!grads) break;
     if (grads->dB[tg]) {
-      const int rc = launch_tall_reduce(dY + l.no[t], ldy, c->us[li] + l.ro[t], l.kxp, T, l.nl[t], c->r, grads->dB[tg],
+      const int rc = launch_tall_reduce(dY + l.no[t], ldy, A.us[li] + l.ro[t], l.kxp, T, l.nl[t], c->r, grads->dB[tg],
                                         c->r, acc, grad_mult, c->red, c->red_floats, st);
       if (rc) return fail(c, rc, "LoRA dB reduction");
     }
@@ -342,66 +354,68 @@ int lin_grads(mebp_ctx* c, int li, const uint16_t* dY, int64_t ldy, const uint16
 // operands in range); the LoRA gradients are written times *grad_mult and dx times *dx_mult
 // (null = 1), so grad_mult = dx_mult = 1/sigma gives true gradients.  dx_h = fp16(sigma dE/dx).
 // dx / dx_h may be null.
-int block_backward(mebp_ctx* c, int layer, const mebp_block_weights* w, const mebp_lora* lora, const float* x,
-                   const float* dy, const uint16_t* dy_h, float* dx, uint16_t* dx_h, const mebp_lora_grads* grads,
-                   int B, int Sq, bool acc, const float* grad_mult, const float* dx_mult, cudaStream_t st) {
+int block_backward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, const mebp_lora* lora,
+                   const float* x, const float* dy, const uint16_t* dy_h, float* dx, uint16_t* dx_h,
+                   const mebp_lora_grads* grads, int B, int Sq, bool acc, const float* grad_mult,
+                   const float* dx_mult, cudaStream_t st) {
+  Acts& A = c->act[set];
   const int64_t T = static_cast<int64_t>(B) * Sq;
   const int D = c->D, I = c->I;
   int rc;
-  if (!(c->saved_layer == layer && c->saved_x == x && c->saved_T == T)) {
-    if ((rc = block_forward(c, layer, w, lora, x, nullptr, B, Sq, false, st))) return rc;
+  if (!(A.layer == layer && A.x == x && A.T == T)) {
+    if ((rc = block_forward(c, set, layer, w, lora, x, nullptr, B, Sq, false, st))) return rc;
   }
-  c->saved_layer = -1;  // the workspace is reused below
+  A.layer = -1;  // the set is consumed below
   // ---- down projection: y = h1 + m Wd^T (+ s (m Ad^T) Bd^T)
   const Lin& ld = c->lin[LIN_DOWN];
   GemmArgs g = gemm_dx(dy_h, D, T, w->down);
   if (ld.kx) {
-    launch_skinny_gemm(dy_h, D, T, D, c->Bt_cat[LIN_DOWN], D, ld.kx, c->s, c->du[LIN_DOWN], ld.kxp, st);
-    g.Ax = c->du[LIN_DOWN]; g.ldax = ld.kxp; g.kx = ld.kxp; g.Bx = c->A_cat[LIN_DOWN]; g.ldbx = I;
+    launch_skinny_gemm(dy_h, D, T, D, A.Bt_cat[LIN_DOWN], D, ld.kx, c->s, c->du[LIN_DOWN], ld.kxp, st);
+    g.Ax = c->du[LIN_DOWN]; g.ldax = ld.kxp; g.kx = ld.kxp; g.Bx = A.A_cat[LIN_DOWN]; g.ldbx = I;
   }
   g.epi = EPI_F32; g.C = c->dm; g.ldc = I;
   if ((rc = run_gemm(c, g, st, "down dX"))) return rc;
-  if ((rc = lin_grads(c, LIN_DOWN, dy_h, D, c->m, I, T, grads, acc, grad_mult, st))) return rc;
+  if ((rc = lin_grads(c, A, LIN_DOWN, dy_h, D, A.m, I, T, grads, acc, grad_mult, st))) return rc;
   // ---- gated MLP
-  launch_glu_bwd(c->dm, c->gu, T, I, c->cfg.act, c->dgu, st);
+  launch_glu_bwd(c->dm, A.gu, T, I, c->cfg.act, c->dgu, st);
   const Lin& lg = c->lin[LIN_GU];
   g = gemm_dx(c->dgu, 2 * I, T, w->gate_up);
   if (lg.kx) {
-    launch_skinny_gemm(c->dgu, 2 * I, T, 2 * I, c->Bt_cat[LIN_GU], 2 * I, lg.kx, c->s, c->du[LIN_GU], lg.kxp, st);
-    g.Ax = c->du[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = c->A_cat[LIN_GU]; g.ldbx = D;
+    launch_skinny_gemm(c->dgu, 2 * I, T, 2 * I, A.Bt_cat[LIN_GU], 2 * I, lg.kx, c->s, c->du[LIN_GU], lg.kxp, st);
+    g.Ax = c->du[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = A.A_cat[LIN_GU]; g.ldbx = D;
   }
   g.epi = EPI_F32; g.C = c->dtmp; g.ldc = D;
   if ((rc = run_gemm(c, g, st, "gate_up dX"))) return rc;
-  if ((rc = lin_grads(c, LIN_GU, c->dgu, 2 * I, c->b, D, T, grads, acc, grad_mult, st))) return rc;
+  if ((rc = lin_grads(c, A, LIN_GU, c->dgu, 2 * I, A.b, D, T, grads, acc, grad_mult, st))) return rc;
   // dh1 = dy + RMSNorm2^T(db)
-  launch_rmsnorm_bwd(c->dtmp, c->h1, w->norm2, c->r2, dy, T, D, nullptr, c->dh1, c->dh1_h, st);
+  launch_rmsnorm_bwd(c->dtmp, A.h1, w->norm2, A.r2, dy, T, D, nullptr, c->dh1, c->dh1_h, st);
   // ---- o projection
   const Lin& lo = c->lin[LIN_O];
   g = gemm_dx(c->dh1_h, D, T, w->o);
   if (lo.kx) {
-    launch_skinny_gemm(c->dh1_h, D, T, D, c->Bt_cat[LIN_O], D, lo.kx, c->s, c->du[LIN_O], lo.kxp, st);
-    g.Ax = c->du[LIN_O]; g.ldax = lo.kxp; g.kx = lo.kxp; g.Bx = c->A_cat[LIN_O]; g.ldbx = c->Na;
+    launch_skinny_gemm(c->dh1_h, D, T, D, A.Bt_cat[LIN_O], D, lo.kx, c->s, c->du[LIN_O], lo.kxp, st);
+    g.Ax = c->du[LIN_O]; g.ldax = lo.kxp; g.kx = lo.kxp; g.Bx = A.A_cat[LIN_O]; g.ldbx = c->Na;
   }
   g.epi = EPI_F16; g.C = c->dout; g.ldc = c->Na;
   if ((rc = run_gemm(c, g, st, "o dX"))) return rc;
-  if ((rc = lin_grads(c, LIN_O, c->dh1_h, D, c->o, c->Na, T, grads, acc, grad_mult, st))) return rc;
+  if ((rc = lin_grads(c, A, LIN_O, c->dh1_h, D, A.o, c->Na, T, grads, acc, grad_mult, st))) return rc;
   // ---- attention, RoPE
   const Lin& lq = c->lin[LIN_QKV];
-  launch_attn_bwd(c->qkv, lq.N, c->o, c->dout, c->Na, c->lse_attn, B, Sq, c->H, c->KV, c->hd, c->dvec, c->dqkv,
+  launch_attn_bwd(A.qkv, lq.N, A.o, c->dout, c->Na, A.lse_attn, B, Sq, c->H, c->KV, c->hd, c->dvec, c->dqkv,
                   c->split_ws, c->split_ws_floats, st);
   launch_rope(c->dqkv, T, Sq, c->H, c->KV, c->hd, c->rope_cs, true, st);
   // ---- q, k, v projections
   if (lq.kx)
-    launch_skinny_gemm(c->dqkv, lq.N, T, lq.N, c->Bt_cat[LIN_QKV], lq.N, lq.kx, c->s, c->du[LIN_QKV], lq.kxp, st);
-  if ((rc = lin_grads(c, LIN_QKV, c->dqkv, lq.N, c->a, D, T, grads, acc, grad_mult, st))) return rc;
+    launch_skinny_gemm(c->dqkv, lq.N, T, lq.N, A.Bt_cat[LIN_QKV], lq.N, lq.kx, c->s, c->du[LIN_QKV], lq.kxp, st);
+  if ((rc = lin_grads(c, A, LIN_QKV, c->dqkv, lq.N, A.a, D, T, grads, acc, grad_mult, st))) return rc;
   if (dx) {
     g = gemm_dx(c->dqkv, lq.N, T, w->qkv);
     if (lq.kx) {
-      g.Ax = c->du[LIN_QKV]; g.ldax = lq.kxp; g.kx = lq.kxp; g.Bx = c->A_cat[LIN_QKV]; g.ldbx = D;
+      g.Ax = c->du[LIN_QKV]; g.ldax = lq.kxp; g.kx = lq.kxp; g.Bx = A.A_cat[LIN_QKV]; g.ldbx = D;
     }
     g.epi = EPI_F32; g.C = c->dtmp; g.ldc = D;
     if ((rc = run_gemm(c, g, st, "qkv dX"))) return rc;
-    launch_rmsnorm_bwd(c->dtmp, x, w->norm1, c->r1, c->dh1, T, D, dx_mult, dx, dx_h, st);
+    launch_rmsnorm_bwd(c->dtmp, x, w->norm1, A.r1, c->dh1, T, D, dx_mult, dx, dx_h, st);
   }
   return cuda_check(c, "block backward");
 }
@@ -511,15 +525,32 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
   A(&c->d_err, 4);
   A(&c->scal, 8);
   A(&c->rope_cs, static_cast<int64_t>(f.max_seq) * (c->hd / 2));
-  A(&c->a, T * D); A(&c->b, T * D); A(&c->qkv, T * c->Nqkv); A(&c->o, T * c->Na); A(&c->gu, T * 2 * I);
-  A(&c->m, T * I); A(&c->r1, T); A(&c->r2, T); A(&c->lse_attn, T * c->H); A(&c->h1, T * D);
-  for (int li = 0; li < 4; ++li) {
-    const Lin& l = c->lin[li];
-    if (!l.kx) continue;
-    A(&c->us[li], T * l.kxp); A(&c->du[li], T * l.kxp);
-    A(&c->A_cat[li], static_cast<int64_t>(l.kxp) * l.K);
-    A(&c->B_cat[li], static_cast<int64_t>(l.N) * l.kxp);
-    A(&c->Bt_cat[li], static_cast<int64_t>(l.N) * l.kxp);
+  // a second intermediate set lets the step overlap recompute and backward (not when spilling:
+  // then device memory is the constraint)
+  c->nsets = (!f.spill_ckpts && c->L > 1) ? 2 : 1;
+  for (int k = 0; k < c->nsets; ++k) {
+    Acts& s = c->act[k];
+    A(&s.a, T * D); A(&s.b, T * D); A(&s.qkv, T * c->Nqkv); A(&s.o, T * c->Na); A(&s.gu, T * 2 * I);
+    A(&s.m, T * I); A(&s.r1, T); A(&s.r2, T); A(&s.lse_attn, T * c->H); A(&s.h1, T * D);
+    for (int li = 0; li < 4; ++li) {
+      const Lin& l = c->lin[li];
+      if (!l.kx) continue;
+      A(&s.us[li], T * l.kxp);
+      A(&s.A_cat[li], static_cast<int64_t>(l.kxp) * l.K);
+      A(&s.B_cat[li], static_cast<int64_t>(l.N) * l.kxp);
+      A(&s.Bt_cat[li], static_cast<int64_t>(l.N) * l.kxp);
+    }
+  }
+  for (int li = 0; li < 4; ++li)
+    if (c->lin[li].kx) A(&c->du[li], T * c->lin[li].kxp);
+  if (rc == MEBP_OK && c->nsets == 2) {
+    if (cudaStreamCreateWithFlags(&c->fstream, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaEventCreateWithFlags(&c->ev_main, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&c->ev_fwd[0], cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&c->ev_fwd[1], cudaEventDisableTiming) != cudaSuccess) {
+      cudaGetLastError();
+      rc = MEBP_ERR_CUDA;
+    }
   }
   A(&c->dqkv, T * c->Nqkv); A(&c->dout, T * c->Na); A(&c->dgu, T * 2 * I); A(&c->dh1_h, T * D);
   A(&c->dy_h[0], T * D); A(&c->dy_h[1], T * D);
@@ -579,7 +610,7 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
   for (int li = 0; li < 4; ++li) {
     const Lin& l = c->lin[li];
     if (!l.kx) continue;
-    cudaMemset(c->us[li], 0, T * l.kxp * 2);
+    for (int k = 0; k < c->nsets; ++k) cudaMemset(c->act[k].us[li], 0, T * l.kxp * 2);
     cudaMemset(c->du[li], 0, T * l.kxp * 2);
   }
   if (cudaDeviceSynchronize() != cudaSuccess || cudaGetLastError() != cudaSuccess) {
@@ -604,6 +635,10 @@ void mebp_ctx_destroy(mebp_ctx* c) {
     if (c->slot_ready[i]) cudaEventDestroy(c->slot_ready[i]);
   }
   if (c->copy_stream) cudaStreamDestroy(c->copy_stream);
+  if (c->ev_main) cudaEventDestroy(c->ev_main);
+  for (cudaEvent_t e : c->ev_fwd)
+    if (e) cudaEventDestroy(e);
+  if (c->fstream) cudaStreamDestroy(c->fstream);
   cudaGetLastError();
   delete c;
 }
@@ -785,8 +820,8 @@ int mebp_block_recompute_fwd(mebp_ctx* c, int layer, const mebp_block_weights* w
   if (!x || !y || !aligned16(x) || !aligned16(y)) return fail(c, MEBP_ERR_INVALID_ARG, "x / y must be 16-byte aligned");
   if (x == y) return fail(c, MEBP_ERR_INVALID_ARG, "x and y must not alias");
   pdl_entry();
-  rc = block_forward(c, layer, w, lora, x, y, B, Sq, true, S(stream));
-  if (!save_for_bwd) c->saved_layer = -1;
+  rc = block_forward(c, 0, layer, w, lora, x, y, B, Sq, true, S(stream));
+  if (!save_for_bwd) c->act[0].layer = -1;
   return rc;
 }
 
@@ -804,7 +839,7 @@ int mebp_block_bwd(mebp_ctx* c, int layer, const mebp_block_weights* w, const me
   pdl_entry();
   launch_grad_scale(dy, n, c->scal + 4, st);
   launch_scale_cast(dy, n, c->scal + 4, c->gbuf[0], c->dy_h[1], st);
-  return block_backward(c, layer, w, lora, x, c->gbuf[0], c->dy_h[1], dx, nullptr, grads, B, Sq, accumulate != 0,
+  return block_backward(c, 0, layer, w, lora, x, c->gbuf[0], c->dy_h[1], dx, nullptr, grads, B, Sq, accumulate != 0,
                         c->scal + 5, c->scal + 5, st);
 }
 
@@ -899,7 +934,7 @@ static int lora_step_body(mebp_ctx* c, const mebp_model_weights* model, const me
       wait_free(sl);  // its previous contents reached the host
       yout = dev_ckpt(sl);
     }
-    if ((rc = block_forward(c, i, &model->blocks[i], &lora[i], xin, yout, B, Sq, true, st))) return rc;
+    if ((rc = block_forward(c, i % c->nsets, i, &model->blocks[i], &lora[i], xin, yout, B, Sq, true, st))) return rc;
     if (spill && i + 1 < L) spill_out(i + 1);
   }
   // ---- loss subgraph: final norm + LM head + CE
@@ -909,7 +944,12 @@ static int lora_step_body(mebp_ctx* c, const mebp_model_weights* model, const me
                    false, st)))
     return rc;
   if (spill) release(L);
-  // ---- backward loop in reverse order: recompute block i from ckpt_i, apply its VJP
+  // ---- backward loop in reverse order: recompute block i from ckpt_i, apply its VJP.  With two
+  // intermediate sets (no spilling) the recompute of block i-1 runs on the recompute stream while
+  // the backward of block i runs on the main stream: block i-1's recompute needs only ckpt_{i-1}
+  // and a set the backward of block i+1 has finished reading.  Block L-1's intermediates are
+  // still in place from the forward loop.
+  const bool overlap = c->nsets == 2 && !spill && L > 1;
   for (int i = L - 1; i >= 0; --i) {
     if (spill) {
       if (slot_of[i] < 0) {
@@ -919,8 +959,21 @@ static int lora_step_body(mebp_ctx* c, const mebp_model_weights* model, const me
       if (i > 0 && slot_of[i - 1] < 0) fetch_in(i - 1, i);  // prefetch while block i runs
     }
     const float* xin = spill ? dev_ckpt(slot_of[i]) : dev_ckpt(i);
+    const int set = i % c->nsets;
+    if (overlap && i > 0) {
+      cudaEventRecord(c->ev_main, st);  // the backward of block i+1 has been issued
+      cudaStreamWaitEvent(c->fstream, c->ev_main, 0);
+      const int ps = (i - 1) % 2;
+      const Acts& P = c->act[ps];
+      if (!(P.layer == i - 1 && P.x == dev_ckpt(i - 1) && P.T == T) &&  // block L-2: kept from the forward loop
+          (rc = block_forward(c, ps, i - 1, &model->blocks[i - 1], &lora[i - 1], dev_ckpt(i - 1), nullptr, B, Sq,
+                              false, c->fstream)))
+        return rc;
+      cudaEventRecord(c->ev_fwd[ps], c->fstream);
+    }
+    if (overlap && i < L - 1) cudaStreamWaitEvent(st, c->ev_fwd[set], 0);
     const int nxt = cur ^ 1;
-    if ((rc = block_backward(c, i, &model->blocks[i], &lora[i], xin, c->gbuf[cur], c->dy_h[cur],
+    if ((rc = block_backward(c, set, i, &model->blocks[i], &lora[i], xin, c->gbuf[cur], c->dy_h[cur],
                              i > 0 ? c->gbuf[nxt] : nullptr, i > 0 ? c->dy_h[nxt] : nullptr, &grads[i], B, Sq,
                              accumulate != 0, c->scal + 1, nullptr, st)))
       return rc;
@@ -934,7 +987,7 @@ static int lora_step_body(mebp_ctx* c, const mebp_model_weights* model, const me
     cudaEventRecord(c->copy_join, c->copy_stream);
     cudaStreamWaitEvent(st, c->copy_join, 0);
   }
-  c->saved_layer = -1;
+  for (int k = 0; k < c->nsets; ++k) c->act[k].layer = -1;
   return cuda_check(c, "lora step");
 }
 
