@@ -61,6 +61,12 @@ struct Acts {
   int64_t T = -1;
 };
 
+// Backward intermediates that the LoRA-gradient reductions read besides the forward set.
+struct Grads2 {
+  uint16_t *dqkv = nullptr, *dgu = nullptr, *dh1_h = nullptr;
+  uint16_t* du[4] = {nullptr, nullptr, nullptr, nullptr};
+};
+
 struct mebp_ctx {
   mebp_model_cfg cfg{};
   int device = 0;
@@ -84,9 +90,14 @@ struct mebp_ctx {
   cudaStream_t fstream = nullptr;  // recompute stream of the overlapped backward
   cudaEvent_t ev_main = nullptr;   // main-stream progress, waited on by the recompute stream
   cudaEvent_t ev_fwd[2] = {};      // recompute into set k finished
-  uint16_t* du[4] = {nullptr, nullptr, nullptr, nullptr};
   // backward
-  uint16_t *dqkv = nullptr, *dout = nullptr, *dgu = nullptr, *dh1_h = nullptr, *dy_h[2] = {nullptr, nullptr};
+  // backward operands of the LoRA-gradient reductions, one copy per layer parity (the reductions
+  // of block i run on the gradient stream while the backward of block i-1 runs)
+  Grads2 bw[2];
+  cudaStream_t gstream = nullptr;  // LoRA-gradient reductions of the overlapped backward
+  cudaEvent_t ev_bwd = nullptr;    // backward of the current block issued (main stream)
+  cudaEvent_t ev_grad[2] = {};     // reductions of a block of parity k finished
+  uint16_t *dout = nullptr, *dy_h[3] = {nullptr, nullptr, nullptr};
   float *dm = nullptr, *dtmp = nullptr, *dh1 = nullptr, *dvec = nullptr, *gbuf[2] = {nullptr, nullptr};
   float* red = nullptr;
   int64_t red_floats = 0;
@@ -329,8 +340,9 @@ int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, 
 }
 
 // LoRA gradients of one fused linear: dB_t = dY[:, rows_t]^T U_s[:, ranks_t], dA_t = dU[:, ranks_t]^T X.
-int lin_grads(mebp_ctx* c, const Acts& A, int li, const uint16_t* dY, int64_t ldy, const uint16_t* X, int64_t ldx,
-              int64_t T, const mebp_lora_grads* grads, bool acc, const float* grad_mult, cudaStream_t st) {
+int lin_grads(mebp_ctx* c, const Acts& A, const uint16_t* du, int li, const uint16_t* dY, int64_t ldy,
+              const uint16_t* X, int64_t ldx, int64_t T, const mebp_lora_grads* grads, bool acc,
+              const float* grad_mult, cudaStream_t st) {
   const Lin& l = c->lin[li];
   for (int t = 0; t < l.nt; ++t) {
     const int tg = l.tgt[t];
@@ -341,7 +353,7 @@ int lin_grads(mebp_ctx* c, const Acts& A, int li, const uint16_t* dY, int64_t ld
       if (rc) return fail(c, rc, "LoRA dB reduction");
     }
     if (grads->dA[tg]) {
-      const int rc = launch_tall_reduce(X, ldx, c->du[li] + l.ro[t], l.kxp, T, l.K, c->r, grads->dA[tg], -l.K, acc,
+      const int rc = launch_tall_reduce(X, ldx, du + l.ro[t], l.kxp, T, l.K, c->r, grads->dA[tg], -l.K, acc,
                                         grad_mult, c->red, c->red_floats, st);
       if (rc) return fail(c, rc, "LoRA dA reduction");
     }
@@ -354,11 +366,13 @@ int lin_grads(mebp_ctx* c, const Acts& A, int li, const uint16_t* dY, int64_t ld
 // operands in range); the LoRA gradients are written times *grad_mult and dx times *dx_mult
 // (null = 1), so grad_mult = dx_mult = 1/sigma gives true gradients.  dx_h = fp16(sigma dE/dx).
 // dx / dx_h may be null.
-int block_backward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, const mebp_lora* lora,
+int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_weights* w, const mebp_lora* lora,
                    const float* x, const float* dy, const uint16_t* dy_h, float* dx, uint16_t* dx_h,
                    const mebp_lora_grads* grads, int B, int Sq, bool acc, const float* grad_mult,
                    const float* dx_mult, cudaStream_t st) {
   Acts& A = c->act[set];
+  Grads2& G = c->bw[bset];
+  uint16_t* const* du = G.du;
   const int64_t T = static_cast<int64_t>(B) * Sq;
   const int D = c->D, I = c->I;
   int rc;
@@ -370,54 +384,68 @@ int block_backward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w,
   const Lin& ld = c->lin[LIN_DOWN];
   GemmArgs g = gemm_dx(dy_h, D, T, w->down);
   if (ld.kx) {
-    launch_skinny_gemm(dy_h, D, T, D, A.Bt_cat[LIN_DOWN], D, ld.kx, c->s, c->du[LIN_DOWN], ld.kxp, st);
-    g.Ax = c->du[LIN_DOWN]; g.ldax = ld.kxp; g.kx = ld.kxp; g.Bx = A.A_cat[LIN_DOWN]; g.ldbx = I;
+    launch_skinny_gemm(dy_h, D, T, D, A.Bt_cat[LIN_DOWN], D, ld.kx, c->s, du[LIN_DOWN], ld.kxp, st);
+    g.Ax = du[LIN_DOWN]; g.ldax = ld.kxp; g.kx = ld.kxp; g.Bx = A.A_cat[LIN_DOWN]; g.ldbx = I;
   }
   g.epi = EPI_F32; g.C = c->dm; g.ldc = I;
   if ((rc = run_gemm(c, g, st, "down dX"))) return rc;
-  if ((rc = lin_grads(c, A, LIN_DOWN, dy_h, D, A.m, I, T, grads, acc, grad_mult, st))) return rc;
+  if ((rc = lin_grads(c, A, du[LIN_DOWN], LIN_DOWN, dy_h, D, A.m, I, T, grads, acc, grad_mult, st))) return rc;
   // ---- gated MLP
-  launch_glu_bwd(c->dm, A.gu, T, I, c->cfg.act, c->dgu, st);
+  launch_glu_bwd(c->dm, A.gu, T, I, c->cfg.act, G.dgu, st);
   const Lin& lg = c->lin[LIN_GU];
-  g = gemm_dx(c->dgu, 2 * I, T, w->gate_up);
+  g = gemm_dx(G.dgu, 2 * I, T, w->gate_up);
   if (lg.kx) {
-    launch_skinny_gemm(c->dgu, 2 * I, T, 2 * I, A.Bt_cat[LIN_GU], 2 * I, lg.kx, c->s, c->du[LIN_GU], lg.kxp, st);
-    g.Ax = c->du[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = A.A_cat[LIN_GU]; g.ldbx = D;
+    launch_skinny_gemm(G.dgu, 2 * I, T, 2 * I, A.Bt_cat[LIN_GU], 2 * I, lg.kx, c->s, du[LIN_GU], lg.kxp, st);
+    g.Ax = du[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = A.A_cat[LIN_GU]; g.ldbx = D;
   }
   g.epi = EPI_F32; g.C = c->dtmp; g.ldc = D;
   if ((rc = run_gemm(c, g, st, "gate_up dX"))) return rc;
-  if ((rc = lin_grads(c, A, LIN_GU, c->dgu, 2 * I, A.b, D, T, grads, acc, grad_mult, st))) return rc;
+  if ((rc = lin_grads(c, A, du[LIN_GU], LIN_GU, G.dgu, 2 * I, A.b, D, T, grads, acc, grad_mult, st))) return rc;
   // dh1 = dy + RMSNorm2^T(db)
-  launch_rmsnorm_bwd(c->dtmp, A.h1, w->norm2, A.r2, dy, T, D, nullptr, c->dh1, c->dh1_h, st);
+  launch_rmsnorm_bwd(c->dtmp, A.h1, w->norm2, A.r2, dy, T, D, nullptr, c->dh1, G.dh1_h, st);
   // ---- o projection
   const Lin& lo = c->lin[LIN_O];
-  g = gemm_dx(c->dh1_h, D, T, w->o);
+  g = gemm_dx(G.dh1_h, D, T, w->o);
   if (lo.kx) {
-    launch_skinny_gemm(c->dh1_h, D, T, D, A.Bt_cat[LIN_O], D, lo.kx, c->s, c->du[LIN_O], lo.kxp, st);
-    g.Ax = c->du[LIN_O]; g.ldax = lo.kxp; g.kx = lo.kxp; g.Bx = A.A_cat[LIN_O]; g.ldbx = c->Na;
+    launch_skinny_gemm(G.dh1_h, D, T, D, A.Bt_cat[LIN_O], D, lo.kx, c->s, du[LIN_O], lo.kxp, st);
+    g.Ax = du[LIN_O]; g.ldax = lo.kxp; g.kx = lo.kxp; g.Bx = A.A_cat[LIN_O]; g.ldbx = c->Na;
   }
   g.epi = EPI_F16; g.C = c->dout; g.ldc = c->Na;
   if ((rc = run_gemm(c, g, st, "o dX"))) return rc;
-  if ((rc = lin_grads(c, A, LIN_O, c->dh1_h, D, A.o, c->Na, T, grads, acc, grad_mult, st))) return rc;
+  if ((rc = lin_grads(c, A, du[LIN_O], LIN_O, G.dh1_h, D, A.o, c->Na, T, grads, acc, grad_mult, st))) return rc;
   // ---- attention, RoPE
   const Lin& lq = c->lin[LIN_QKV];
-  launch_attn_bwd(A.qkv, lq.N, A.o, c->dout, c->Na, A.lse_attn, B, Sq, c->H, c->KV, c->hd, c->dvec, c->dqkv,
+  launch_attn_bwd(A.qkv, lq.N, A.o, c->dout, c->Na, A.lse_attn, B, Sq, c->H, c->KV, c->hd, c->dvec, G.dqkv,
                   c->split_ws, c->split_ws_floats, st);
-  launch_rope(c->dqkv, T, Sq, c->H, c->KV, c->hd, c->rope_cs, true, st);
+  launch_rope(G.dqkv, T, Sq, c->H, c->KV, c->hd, c->rope_cs, true, st);
   // ---- q, k, v projections
   if (lq.kx)
-    launch_skinny_gemm(c->dqkv, lq.N, T, lq.N, A.Bt_cat[LIN_QKV], lq.N, lq.kx, c->s, c->du[LIN_QKV], lq.kxp, st);
-  if ((rc = lin_grads(c, A, LIN_QKV, c->dqkv, lq.N, A.a, D, T, grads, acc, grad_mult, st))) return rc;
+    launch_skinny_gemm(G.dqkv, lq.N, T, lq.N, A.Bt_cat[LIN_QKV], lq.N, lq.kx, c->s, du[LIN_QKV], lq.kxp, st);
+  if ((rc = lin_grads(c, A, du[LIN_QKV], LIN_QKV, G.dqkv, lq.N, A.a, D, T, grads, acc, grad_mult, st))) return rc;
   if (dx) {
-    g = gemm_dx(c->dqkv, lq.N, T, w->qkv);
+    g = gemm_dx(G.dqkv, lq.N, T, w->qkv);
     if (lq.kx) {
-      g.Ax = c->du[LIN_QKV]; g.ldax = lq.kxp; g.kx = lq.kxp; g.Bx = A.A_cat[LIN_QKV]; g.ldbx = D;
+      g.Ax = du[LIN_QKV]; g.ldax = lq.kxp; g.kx = lq.kxp; g.Bx = A.A_cat[LIN_QKV]; g.ldbx = D;
     }
     g.epi = EPI_F32; g.C = c->dtmp; g.ldc = D;
     if ((rc = run_gemm(c, g, st, "qkv dX"))) return rc;
     launch_rmsnorm_bwd(c->dtmp, x, w->norm1, A.r1, c->dh1, T, D, dx_mult, dx, dx_h, st);
   }
   return cuda_check(c, "block backward");
+}
+
+// The LoRA-gradient reductions of one block whose backward (block_backward with grads = null)
+// has been issued: the same operands the inline reductions read.
+int block_lora_grads(mebp_ctx* c, int set, int bset, const uint16_t* dy_h, int64_t T, const mebp_lora_grads* grads,
+                     bool acc, const float* grad_mult, cudaStream_t st) {
+  const Acts& A = c->act[set];
+  const Grads2& G = c->bw[bset];
+  const int D = c->D, I = c->I;
+  int rc;
+  if ((rc = lin_grads(c, A, G.du[LIN_DOWN], LIN_DOWN, dy_h, D, A.m, I, T, grads, acc, grad_mult, st))) return rc;
+  if ((rc = lin_grads(c, A, G.du[LIN_GU], LIN_GU, G.dgu, 2 * I, A.b, D, T, grads, acc, grad_mult, st))) return rc;
+  if ((rc = lin_grads(c, A, G.du[LIN_O], LIN_O, G.dh1_h, D, A.o, c->Na, T, grads, acc, grad_mult, st))) return rc;
+  return lin_grads(c, A, G.du[LIN_QKV], LIN_QKV, G.dqkv, c->lin[LIN_QKV].N, A.a, D, T, grads, acc, grad_mult, st);
 }
 
 // Final RMSNorm + LM head + CE.  dh (fp32) is the true gradient when unscale_dh, else it is
@@ -541,19 +569,27 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
       A(&s.Bt_cat[li], static_cast<int64_t>(l.N) * l.kxp);
     }
   }
-  for (int li = 0; li < 4; ++li)
-    if (c->lin[li].kx) A(&c->du[li], T * c->lin[li].kxp);
+  for (int k = 0; k < c->nsets; ++k) {
+    Grads2& g = c->bw[k];
+    A(&g.dqkv, T * c->Nqkv); A(&g.dgu, T * 2 * I); A(&g.dh1_h, T * D);
+    for (int li = 0; li < 4; ++li)
+      if (c->lin[li].kx) A(&g.du[li], T * c->lin[li].kxp);
+  }
   if (rc == MEBP_OK && c->nsets == 2) {
     if (cudaStreamCreateWithFlags(&c->fstream, cudaStreamNonBlocking) != cudaSuccess ||
         cudaEventCreateWithFlags(&c->ev_main, cudaEventDisableTiming) != cudaSuccess ||
         cudaEventCreateWithFlags(&c->ev_fwd[0], cudaEventDisableTiming) != cudaSuccess ||
-        cudaEventCreateWithFlags(&c->ev_fwd[1], cudaEventDisableTiming) != cudaSuccess) {
+        cudaEventCreateWithFlags(&c->ev_fwd[1], cudaEventDisableTiming) != cudaSuccess ||
+        cudaStreamCreateWithFlags(&c->gstream, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaEventCreateWithFlags(&c->ev_bwd, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&c->ev_grad[0], cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&c->ev_grad[1], cudaEventDisableTiming) != cudaSuccess) {
       cudaGetLastError();
       rc = MEBP_ERR_CUDA;
     }
   }
-  A(&c->dqkv, T * c->Nqkv); A(&c->dout, T * c->Na); A(&c->dgu, T * 2 * I); A(&c->dh1_h, T * D);
-  A(&c->dy_h[0], T * D); A(&c->dy_h[1], T * D);
+  A(&c->dout, T * c->Na);
+  for (int k = 0; k < (c->nsets == 2 ? 3 : 2); ++k) A(&c->dy_h[k], T * D);
   A(&c->dm, T * I); A(&c->dtmp, T * D); A(&c->dh1, T * D); A(&c->dvec, T * c->H);
   A(&c->gbuf[0], T * D); A(&c->gbuf[1], T * D);
   c->red_floats = std::max<int64_t>(tall_reduce_scratch_floats(T, std::max<int64_t>(2 * I, c->Nqkv), 32),
@@ -611,7 +647,7 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
     const Lin& l = c->lin[li];
     if (!l.kx) continue;
     for (int k = 0; k < c->nsets; ++k) cudaMemset(c->act[k].us[li], 0, T * l.kxp * 2);
-    cudaMemset(c->du[li], 0, T * l.kxp * 2);
+    for (int k = 0; k < c->nsets; ++k) cudaMemset(c->bw[k].du[li], 0, T * l.kxp * 2);
   }
   if (cudaDeviceSynchronize() != cudaSuccess || cudaGetLastError() != cudaSuccess) {
     mebp_ctx_destroy(c);
@@ -639,6 +675,10 @@ void mebp_ctx_destroy(mebp_ctx* c) {
   for (cudaEvent_t e : c->ev_fwd)
     if (e) cudaEventDestroy(e);
   if (c->fstream) cudaStreamDestroy(c->fstream);
+  if (c->ev_bwd) cudaEventDestroy(c->ev_bwd);
+  for (cudaEvent_t e : c->ev_grad)
+    if (e) cudaEventDestroy(e);
+  if (c->gstream) cudaStreamDestroy(c->gstream);
   cudaGetLastError();
   delete c;
 }
@@ -839,7 +879,7 @@ int mebp_block_bwd(mebp_ctx* c, int layer, const mebp_block_weights* w, const me
   pdl_entry();
   launch_grad_scale(dy, n, c->scal + 4, st);
   launch_scale_cast(dy, n, c->scal + 4, c->gbuf[0], c->dy_h[1], st);
-  return block_backward(c, 0, layer, w, lora, x, c->gbuf[0], c->dy_h[1], dx, nullptr, grads, B, Sq, accumulate != 0,
+  return block_backward(c, 0, 0, layer, w, lora, x, c->gbuf[0], c->dy_h[1], dx, nullptr, grads, B, Sq, accumulate != 0,
                         c->scal + 5, c->scal + 5, st);
 }
 
@@ -945,11 +985,14 @@ static int lora_step_body(mebp_ctx* c, const mebp_model_weights* model, const me
     return rc;
   if (spill) release(L);
   // ---- backward loop in reverse order: recompute block i from ckpt_i, apply its VJP.  With two
-  // intermediate sets (no spilling) the recompute of block i-1 runs on the recompute stream while
-  // the backward of block i runs on the main stream: block i-1's recompute needs only ckpt_{i-1}
-  // and a set the backward of block i+1 has finished reading.  Block L-1's intermediates are
-  // still in place from the forward loop.
+  // intermediate sets (no spilling) three streams share the work: the recompute of block i-1
+  // (recompute stream) and the LoRA-gradient reductions of block i+1 (gradient stream) run while
+  // the main stream computes the input gradients of block i.  Buffers alternate by block parity
+  // (fp16 upstream gradients over three blocks), so a set is rewritten only after the stream
+  // that reads it has finished with it.  Block L-1's intermediates are still in place from the
+  // forward loop, and so are block L-2's.
   const bool overlap = c->nsets == 2 && !spill && L > 1;
+  auto dyh = [&](int i) { return c->dy_h[(L - 1 - i) % 3]; };  // fp16 dE/dy of block i (overlap)
   for (int i = L - 1; i >= 0; --i) {
     if (spill) {
       if (slot_of[i] < 0) {
@@ -960,28 +1003,46 @@ static int lora_step_body(mebp_ctx* c, const mebp_model_weights* model, const me
     }
     const float* xin = spill ? dev_ckpt(slot_of[i]) : dev_ckpt(i);
     const int set = i % c->nsets;
-    if (overlap && i > 0) {
-      cudaEventRecord(c->ev_main, st);  // the backward of block i+1 has been issued
-      cudaStreamWaitEvent(c->fstream, c->ev_main, 0);
-      const int ps = (i - 1) % 2;
-      const Acts& P = c->act[ps];
-      if (!(P.layer == i - 1 && P.x == dev_ckpt(i - 1) && P.T == T) &&  // block L-2: kept from the forward loop
-          (rc = block_forward(c, ps, i - 1, &model->blocks[i - 1], &lora[i - 1], dev_ckpt(i - 1), nullptr, B, Sq,
-                              false, c->fstream)))
-        return rc;
-      cudaEventRecord(c->ev_fwd[ps], c->fstream);
-    }
-    if (overlap && i < L - 1) cudaStreamWaitEvent(st, c->ev_fwd[set], 0);
     const int nxt = cur ^ 1;
-    if ((rc = block_backward(c, set, i, &model->blocks[i], &lora[i], xin, c->gbuf[cur], c->dy_h[cur],
-                             i > 0 ? c->gbuf[nxt] : nullptr, i > 0 ? c->dy_h[nxt] : nullptr, &grads[i], B, Sq,
-                             accumulate != 0, c->scal + 1, nullptr, st)))
-      return rc;
+    if (!overlap) {
+      if ((rc = block_backward(c, set, 0, i, &model->blocks[i], &lora[i], xin, c->gbuf[cur], c->dy_h[cur],
+                               i > 0 ? c->gbuf[nxt] : nullptr, i > 0 ? c->dy_h[nxt] : nullptr, &grads[i], B, Sq,
+                               accumulate != 0, c->scal + 1, nullptr, st)))
+        return rc;
+    } else {
+      if (i > 0) {  // recompute block i-1 into the other set once its readers are done with it
+        const int ps = (i - 1) % 2;
+        cudaEventRecord(c->ev_main, st);  // the backward of block i+1 has been issued
+        cudaStreamWaitEvent(c->fstream, c->ev_main, 0);
+        if (i + 1 < L) cudaStreamWaitEvent(c->fstream, c->ev_grad[ps], 0);  // reductions of block i+1
+        const Acts& P = c->act[ps];
+        if (!(P.layer == i - 1 && P.x == dev_ckpt(i - 1) && P.T == T) &&
+            (rc = block_forward(c, ps, i - 1, &model->blocks[i - 1], &lora[i - 1], dev_ckpt(i - 1), nullptr, B, Sq,
+                                false, c->fstream)))
+          return rc;
+        cudaEventRecord(c->ev_fwd[ps], c->fstream);
+      }
+      if (i < L - 1) cudaStreamWaitEvent(st, c->ev_fwd[set], 0);
+      if (i + 2 < L) cudaStreamWaitEvent(st, c->ev_grad[set], 0);  // reductions of block i+2
+      if ((rc = block_backward(c, set, set, i, &model->blocks[i], &lora[i], xin, c->gbuf[cur], dyh(i),
+                               i > 0 ? c->gbuf[nxt] : nullptr, i > 0 ? dyh(i - 1) : nullptr, nullptr, B, Sq,
+                               accumulate != 0, c->scal + 1, nullptr, st)))
+        return rc;
+      cudaEventRecord(c->ev_bwd, st);
+      cudaStreamWaitEvent(c->gstream, c->ev_bwd, 0);
+      if ((rc = block_lora_grads(c, set, set, dyh(i), T, &grads[i], accumulate != 0, c->scal + 1, c->gstream)))
+        return rc;
+      cudaEventRecord(c->ev_grad[set], c->gstream);
+    }
     if (spill) {
       release(i);  // the checkpoint is removed once its backward has consumed it
       if (i > 0) wait_free(slot_of[i - 1]);
     }
     cur = nxt;
+  }
+  if (overlap) {  // join the gradient stream
+    cudaStreamWaitEvent(st, c->ev_grad[0], 0);
+    cudaStreamWaitEvent(st, c->ev_grad[1], 0);
   }
   if (spill) {  // every copy of this step is complete when the stream reaches this point
     cudaEventRecord(c->copy_join, c->copy_stream);
