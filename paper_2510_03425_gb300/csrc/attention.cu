@@ -75,7 +75,9 @@ __device__ __forceinline__ void pv_tile(float (&acc)[NC][4], const float (&p)[8]
 }
 
 // ------------------------------------------------------------------------------------ forward
-template <int HD>
+// NB key/value buffers: 2 overlaps the next block's load with this one; 1 leaves room for two
+// CTAs per SM at head_dim 256.
+template <int HD, int NB>
 __global__ void __launch_bounds__(128, 1) fwd_kernel(const uint16_t* __restrict__ qkv, int64_t ld, int S, int H,
                                                      int KV, uint16_t* __restrict__ o, int64_t ldo,
                                                      float* __restrict__ lse) {
@@ -83,9 +85,9 @@ __global__ void __launch_bounds__(128, 1) fwd_kernel(const uint16_t* __restrict_
   griddep_launch();
   constexpr int LD = HD + 8, NO = HD / 8;
   extern __shared__ __align__(16) uint16_t sm[];
-  uint16_t* qs = sm;
-  uint16_t* ks = qs + BQ * LD;
-  uint16_t* vs = ks + BKV * LD;
+  uint16_t* qs = sm;  // then NB (K, V) buffers
+  auto ks = [&](int buf) { return qs + (1 + 2 * buf) * BQ * LD; };
+  auto vs = [&](int buf) { return qs + (2 + 2 * buf) * BQ * LD; };
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int qb = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int kvh = h / (H / KV);
@@ -94,6 +96,10 @@ __global__ void __launch_bounds__(128, 1) fwd_kernel(const uint16_t* __restrict_
   const float sc = kLog2e * rsqrtf(static_cast<float>(HD));
 
   load_tile<HD>(qs, qkv, ld, tok0, q0, S, h * HD, tid);
+  if (NB == 2) {
+    load_tile<HD>(ks(0), qkv, ld, tok0, 0, S, (H + kvh) * HD, tid);
+    load_tile<HD>(vs(0), qkv, ld, tok0, 0, S, (H + KV + kvh) * HD, tid);
+  }
   cp_async_commit();
 
   float oacc[NO][4];
@@ -104,15 +110,24 @@ __global__ void __launch_bounds__(128, 1) fwd_kernel(const uint16_t* __restrict_
   const int nkb = min((q0 + BQ - 1) / BKV + 1, (S + BKV - 1) / BKV);
 
   for (int kb = 0; kb < nkb; ++kb) {
-    const int k0 = kb * BKV;
-    load_tile<HD>(ks, qkv, ld, tok0, k0, S, (H + kvh) * HD, tid);
-    load_tile<HD>(vs, qkv, ld, tok0, k0, S, (H + KV + kvh) * HD, tid);
-    cp_async_commit();
-    cp_async_wait<0>();
+    const int k0 = kb * BKV, buf = NB == 2 ? kb & 1 : 0;
+    if (NB == 1) {
+      load_tile<HD>(ks(0), qkv, ld, tok0, k0, S, (H + kvh) * HD, tid);
+      load_tile<HD>(vs(0), qkv, ld, tok0, k0, S, (H + KV + kvh) * HD, tid);
+      cp_async_commit();
+      cp_async_wait<0>();
+    } else if (kb + 1 < nkb) {
+      load_tile<HD>(ks(buf ^ 1), qkv, ld, tok0, k0 + BKV, S, (H + kvh) * HD, tid);
+      load_tile<HD>(vs(buf ^ 1), qkv, ld, tok0, k0 + BKV, S, (H + KV + kvh) * HD, tid);
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
     __syncthreads();
 
     float s[8][4];
-    qk_tile<HD>(s, smem_u32(qs), smem_u32(ks), warp, lane);
+    qk_tile<HD>(s, smem_u32(qs), smem_u32(ks(buf)), warp, lane);
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt)
 #pragma unroll
@@ -149,8 +164,8 @@ __global__ void __launch_bounds__(128, 1) fwd_kernel(const uint16_t* __restrict_
         oacc[dt][2 * i + 1] *= alpha;
       }
     }
-    pv_tile<HD, NO>(oacc, s, smem_u32(vs), 0, lane);
-    __syncthreads();
+    pv_tile<HD, NO>(oacc, s, smem_u32(vs(buf)), 0, lane);
+    __syncthreads();  // every warp is done with this buffer before it is refilled
   }
 
   const int c = 2 * (lane & 3);
@@ -208,10 +223,11 @@ __global__ void __launch_bounds__(128, 1) dkdv_kernel(const uint16_t* __restrict
   extern __shared__ __align__(16) uint16_t sm[];
   uint16_t* ks = sm;
   uint16_t* vs = ks + BKV * LD;
-  uint16_t* qs = vs + BKV * LD;
-  uint16_t* dos = qs + BQ * LD;
-  float* lse_s = reinterpret_cast<float*>(dos + BQ * LD);
-  float* dv_s = lse_s + BQ;
+  // two (Q, dO, lse, dvec) buffers: the next query block loads while this one is used
+  auto qs = [&](int buf) { return vs + (1 + 2 * buf) * BQ * LD; };
+  auto dos = [&](int buf) { return vs + (2 + 2 * buf) * BQ * LD; };
+  auto lse_s = [&](int buf) { return reinterpret_cast<float*>(vs + 5 * BQ * LD) + buf * 2 * BQ; };
+  auto dv_s = [&](int buf) { return lse_s(buf) + BQ; };
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int grp = H / KV;
   const bool perhead = part != nullptr;
@@ -223,10 +239,6 @@ __global__ void __launch_bounds__(128, 1) dkdv_kernel(const uint16_t* __restrict
   const int k0 = kb * BKV;
   const float sc = kLog2e * rsqrtf(static_cast<float>(HD));
 
-  load_tile<HD>(ks, qkv, ld, tok0, k0, S, (H + kvh) * HD, tid);
-  load_tile<HD>(vs, qkv, ld, tok0, k0, S, (H + KV + kvh) * HD, tid);
-  cp_async_commit();
-
   float dk[NC][4], dv[NC][4];
 #pragma unroll
   for (int i = 0; i < NC; ++i) {
@@ -235,51 +247,66 @@ __global__ void __launch_bounds__(128, 1) dkdv_kernel(const uint16_t* __restrict
   }
   const int key_a = k0 + warp * 16 + (lane >> 2);
   const int nqb = (S + BQ - 1) / BQ;
-
-  for (int hh = 0; hh < h_count; ++hh) {
-    const int h = h_first + hh;
-    for (int qb = kb; qb < nqb; ++qb) {
-      const int q0 = qb * BQ;
-      load_tile<HD>(qs, qkv, ld, tok0, q0, S, h * HD, tid);
-      load_tile<HD>(dos, dout, ldo, tok0, q0, S, h * HD, tid);
-      cp_async_commit();
-      for (int i = tid; i < BQ; i += 128) {
-        const int q = q0 + i;
-        const int64_t li = (static_cast<int64_t>(b) * H + h) * S + q;
-        lse_s[i] = q < S ? lse[li] * kLog2e : 0.0f;
-        dv_s[i] = q < S ? dvec[li] : 0.0f;
-      }
-      cp_async_wait<0>();
-      __syncthreads();
-
-      // P^T (16 keys x 64 queries)
-      float pt[8][4];
-      qk_tile<HD>(pt, smem_u32(ks), smem_u32(qs), warp, lane);
-#pragma unroll
-      for (int nt = 0; nt < 8; ++nt)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int key = key_a + ((e >> 1) << 3);
-          const int qi = nt * 8 + 2 * (lane & 3) + (e & 1);
-          const int q = q0 + qi;
-          pt[nt][e] = (key <= q && q < S && key < S) ? exp2f(pt[nt][e] * sc - lse_s[qi]) : 0.0f;
-        }
-      // dV += P^T dO
-      pv_tile<HD, NC>(dv, pt, smem_u32(dos), d0, lane);
-      // dP^T = V dO^T ; dS^T = P^T (dP^T - dvec)
-      float dpt[8][4];
-      qk_tile<HD>(dpt, smem_u32(vs), smem_u32(dos), warp, lane);
-#pragma unroll
-      for (int nt = 0; nt < 8; ++nt)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int qi = nt * 8 + 2 * (lane & 3) + (e & 1);
-          dpt[nt][e] = pt[nt][e] * (dpt[nt][e] - dv_s[qi]);
-        }
-      // dK += dS^T Q
-      pv_tile<HD, NC>(dk, dpt, smem_u32(qs), d0, lane);
-      __syncthreads();
+  const int per_head = nqb - kb;            // query blocks kb .. nqb-1 see this key block
+  const int n_it = h_count * per_head;
+  // query block of iteration it -> (head, first query) and its loads into buffer buf
+  auto fetch = [&](int it, int buf) {
+    const int h = h_first + it / per_head, q0 = (kb + it % per_head) * BQ;
+    load_tile<HD>(qs(buf), qkv, ld, tok0, q0, S, h * HD, tid);
+    load_tile<HD>(dos(buf), dout, ldo, tok0, q0, S, h * HD, tid);
+    for (int i = tid; i < BQ; i += 128) {
+      const int q = q0 + i;
+      const int64_t li = (static_cast<int64_t>(b) * H + h) * S + q;
+      lse_s(buf)[i] = q < S ? lse[li] * kLog2e : 0.0f;
+      dv_s(buf)[i] = q < S ? dvec[li] : 0.0f;
     }
+  };
+  load_tile<HD>(ks, qkv, ld, tok0, k0, S, (H + kvh) * HD, tid);
+  load_tile<HD>(vs, qkv, ld, tok0, k0, S, (H + KV + kvh) * HD, tid);
+  if (n_it > 0) fetch(0, 0);
+  cp_async_commit();
+
+  for (int it = 0; it < n_it; ++it) {
+    const int buf = it & 1;
+    const int q0 = (kb + it % per_head) * BQ;
+    if (it + 1 < n_it) {
+      fetch(it + 1, buf ^ 1);
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
+    __syncthreads();
+    const float* lsb = lse_s(buf);
+    const float* dvb = dv_s(buf);
+
+    // P^T (16 keys x 64 queries)
+    float pt[8][4];
+    qk_tile<HD>(pt, smem_u32(ks), smem_u32(qs(buf)), warp, lane);
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int key = key_a + ((e >> 1) << 3);
+        const int qi = nt * 8 + 2 * (lane & 3) + (e & 1);
+        const int q = q0 + qi;
+        pt[nt][e] = (key <= q && q < S && key < S) ? exp2f(pt[nt][e] * sc - lsb[qi]) : 0.0f;
+      }
+    // dV += P^T dO
+    pv_tile<HD, NC>(dv, pt, smem_u32(dos(buf)), d0, lane);
+    // dP^T = V dO^T ; dS^T = P^T (dP^T - dvec)
+    float dpt[8][4];
+    qk_tile<HD>(dpt, smem_u32(vs), smem_u32(dos(buf)), warp, lane);
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int qi = nt * 8 + 2 * (lane & 3) + (e & 1);
+        dpt[nt][e] = pt[nt][e] * (dpt[nt][e] - dvb[qi]);
+      }
+    // dK += dS^T Q
+    pv_tile<HD, NC>(dk, dpt, smem_u32(qs(buf)), d0, lane);
+    __syncthreads();  // every warp is done with this buffer before it is refilled
   }
   const float inv = rsqrtf(static_cast<float>(HD));
   const int c = 2 * (lane & 3);
@@ -324,8 +351,9 @@ __global__ void __launch_bounds__(128, 1) dq_kernel(const uint16_t* __restrict__
   extern __shared__ __align__(16) uint16_t sm[];
   uint16_t* qs = sm;
   uint16_t* dos = qs + BQ * LD;
-  uint16_t* ks = dos + BQ * LD;
-  uint16_t* vs = ks + BKV * LD;
+  // two (K, V) buffers: the next key block loads while this one is used
+  auto ks = [&](int buf) { return dos + (1 + 2 * buf) * BQ * LD; };
+  auto vs = [&](int buf) { return dos + (2 + 2 * buf) * BQ * LD; };
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int qb = blockIdx.x, h = blockIdx.y;
   const int b = blockIdx.z / NCH, d0 = (blockIdx.z % NCH) * DC;
@@ -336,6 +364,8 @@ __global__ void __launch_bounds__(128, 1) dq_kernel(const uint16_t* __restrict__
 
   load_tile<HD>(qs, qkv, ld, tok0, q0, S, h * HD, tid);
   load_tile<HD>(dos, dout, ldo, tok0, q0, S, h * HD, tid);
+  load_tile<HD>(ks(0), qkv, ld, tok0, 0, S, (H + kvh) * HD, tid);
+  load_tile<HD>(vs(0), qkv, ld, tok0, 0, S, (H + KV + kvh) * HD, tid);
   cp_async_commit();
   const int ra = q0 + warp * 16 + (lane >> 2);
   float lse2[2], dvv[2];
@@ -351,14 +381,18 @@ __global__ void __launch_bounds__(128, 1) dq_kernel(const uint16_t* __restrict__
   for (int i = 0; i < NC; ++i) dq[i][0] = dq[i][1] = dq[i][2] = dq[i][3] = 0.0f;
 
   for (int kb = 0; kb <= qb; ++kb) {
-    const int k0 = kb * BKV;
-    load_tile<HD>(ks, qkv, ld, tok0, k0, S, (H + kvh) * HD, tid);
-    load_tile<HD>(vs, qkv, ld, tok0, k0, S, (H + KV + kvh) * HD, tid);
-    cp_async_commit();
-    cp_async_wait<0>();
+    const int k0 = kb * BKV, buf = kb & 1;
+    if (kb < qb) {
+      load_tile<HD>(ks(buf ^ 1), qkv, ld, tok0, k0 + BKV, S, (H + kvh) * HD, tid);
+      load_tile<HD>(vs(buf ^ 1), qkv, ld, tok0, k0 + BKV, S, (H + KV + kvh) * HD, tid);
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
     __syncthreads();
     float p[8][4];
-    qk_tile<HD>(p, smem_u32(qs), smem_u32(ks), warp, lane);
+    qk_tile<HD>(p, smem_u32(qs), smem_u32(ks(buf)), warp, lane);
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt)
 #pragma unroll
@@ -369,13 +403,13 @@ __global__ void __launch_bounds__(128, 1) dq_kernel(const uint16_t* __restrict__
         p[nt][e] = (col <= row && col < S && row < S) ? exp2f(p[nt][e] * sc - lse2[i]) : 0.0f;
       }
     float dp[8][4];
-    qk_tile<HD>(dp, smem_u32(dos), smem_u32(vs), warp, lane);
+    qk_tile<HD>(dp, smem_u32(dos), smem_u32(vs(buf)), warp, lane);
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt)
 #pragma unroll
       for (int e = 0; e < 4; ++e) dp[nt][e] = p[nt][e] * (dp[nt][e] - dvv[e >> 1]);
-    pv_tile<HD, NC>(dq, dp, smem_u32(ks), d0, lane);
-    __syncthreads();
+    pv_tile<HD, NC>(dq, dp, smem_u32(ks(buf)), d0, lane);
+    __syncthreads();  // every warp is done with this buffer before it is refilled
   }
   const float inv = rsqrtf(static_cast<float>(HD));
   const int c = 2 * (lane & 3);
@@ -390,17 +424,27 @@ __global__ void __launch_bounds__(128, 1) dq_kernel(const uint16_t* __restrict__
   }
 }
 
-template <int HD>
-void fwd_launch(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uint16_t* o, int64_t ldo, float* lse,
-                cudaStream_t st) {
-  constexpr int smem = 3 * 64 * (HD + 8) * 2;
+template <int HD, int NB>
+void fwd_launch_nb(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uint16_t* o, int64_t ldo, float* lse,
+                   cudaStream_t st) {
+  constexpr int smem = (1 + 2 * NB) * 64 * (HD + 8) * 2;  // Q, NB x (K, V)
   static bool init = false;
   if (!init) {
-    cudaFuncSetAttribute(fwd_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(fwd_kernel<HD, NB>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     init = true;
   }
   dim3 grid((S + BQ - 1) / BQ, H, B);
-  launch_k(fwd_kernel<HD>, grid, 128, smem, st, qkv, ld, S, H, KV, o, ldo, lse);
+  launch_k(fwd_kernel<HD, NB>, grid, 128, smem, st, qkv, ld, S, H, KV, o, ldo, lse);
+}
+
+// Double-buffered key/value loads, except at head_dim 256 with more than two waves of CTAs: there
+// the single-buffered kernel fits two CTAs per SM, which hides the loads better.
+template <int HD>
+void fwd_launch(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uint16_t* o, int64_t ldo, float* lse,
+                cudaStream_t st) {
+  const int64_t ctas = static_cast<int64_t>((S + BQ - 1) / BQ) * H * B;
+  if (HD == 256 && ctas > 2 * 152) fwd_launch_nb<HD, 1>(qkv, ld, B, S, H, KV, o, ldo, lse, st);
+  else fwd_launch_nb<HD, 2>(qkv, ld, B, S, H, KV, o, ldo, lse, st);
 }
 
 // dK, dV of kv head j = sum over the query heads of group j of the per-head partials (fixed order).
@@ -430,7 +474,8 @@ template <int HD, int DC>
 void bwd_launch(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t ldo, const float* lse,
                 const float* dvec, int B, int S, int H, int KV, uint16_t* dqkv, float* part, int64_t part_floats,
                 cudaStream_t st) {
-  constexpr int smem = 4 * 64 * (HD + 8) * 2 + 2 * 64 * 4;
+  constexpr int smem = 6 * 64 * (HD + 8) * 2 + 4 * 64 * 4;  // 6 tiles (2 of them double-buffered) + lse, dvec x 2
+  static_assert(smem <= 232448, "attention backward shared memory");
   static bool init = false;
   if (!init) {
     cudaFuncSetAttribute(dkdv_kernel<HD, DC>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);

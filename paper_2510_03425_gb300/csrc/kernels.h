@@ -40,6 +40,35 @@ inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, siz
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
+// launch_k with a thread-block cluster of cluster.x * cluster.y * cluster.z CTAs (1: none).
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_k_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                                    dim3 cluster, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute at[2];
+  int na = 0;
+  if (pdl_take()) {
+    at[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+  }
+  if (cluster.x * cluster.y * cluster.z > 1) {
+    at[na].id = cudaLaunchAttributeClusterDimension;
+    at[na].val.clusterDim.x = cluster.x;
+    at[na].val.clusterDim.y = cluster.y;
+    at[na].val.clusterDim.z = cluster.z;
+    ++na;
+  }
+  cfg.attrs = at;
+  cfg.numAttrs = na;
+  count_launch();
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 enum GemmEpi { EPI_F16 = 0, EPI_F32 = 1, EPI_LSE = 2, EPI_CEGRAD = 3 };
 
 struct GemmArgs {
@@ -119,6 +148,13 @@ int launch_tall_reduce(const uint16_t* P, int64_t ldp, const uint16_t* Q, int64_
                        int64_t scratch_floats, cudaStream_t st);
 int64_t tall_reduce_scratch_floats(int64_t M, int Pw, int Qw);
 // fp16 shadows of the LoRA masters, see lora.cu.
+// fp16 LoRA shadows of n_layers layers at once: target t of layer l reads A[3 l + t], B[3 l + t];
+// layer l's outputs start at l * stride_a (A_cat) and l * stride_b (B_cat, Bt_cat).
+constexpr int kShadowMaxLayers = 64;  // layers per launch
+void launch_lora_shadow_layers(int n_layers, const float* const* A, const float* const* B, int nt,
+                               const int* ranks_off, const int* n_off, const int* n_len, int r, int K, int N, int kx,
+                               uint16_t* A_cat, uint16_t* B_cat, uint16_t* Bt_cat, int64_t stride_a, int64_t stride_b,
+                               cudaStream_t st);
 void launch_lora_shadow(const float* const* A, const float* const* B, int nt, const int* ranks_off,
                         const int* n_off, const int* n_len, int r, int K, int N, int kx, uint16_t* A_cat,
                         uint16_t* B_cat, uint16_t* Bt_cat, cudaStream_t st);

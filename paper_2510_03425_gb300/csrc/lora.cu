@@ -10,21 +10,32 @@
 //      A_cat [kx, K]  rows ro_t .. ro_t+r-1 = A_t
 //      B_cat [N, kx]  block-diagonal: rows of target t, columns ro_t .. ro_t+r-1 = B_t
 //      Bt_cat [kx, N] = B_cat^T
+#include <algorithm>
+
 #include "kernels.h"
 #include "mma.cuh"
 
 namespace mebp {
 
 // ------------------------------------------------------------------------------------ skinny
+// CTA (blockIdx.x, blockIdx.y): rows m0 .. m0+63, K tiles of split blockIdx.y.  With more than
+// one split (gridDim.y > 1) the splits of a row block form one cluster: each parks its fp32
+// partial [64][JR] in shared memory and CTA z sums rows z*ceil(64/S) .. of all S partials over
+// distributed shared memory in split order (deterministic).
 template <int NT>
 __global__ void __launch_bounds__(128) skinny_gemm_kernel(const uint16_t* __restrict__ X, int64_t ldx, int64_t M,
                                                           int64_t K, const uint16_t* __restrict__ W, int64_t ldw,
-                                                          float alpha, uint16_t* __restrict__ out, int64_t ldo) {
+                                                          float alpha, uint16_t* __restrict__ out, int64_t ldo,
+                                                          int kt_split) {
   griddep_wait();
   griddep_launch();
-  constexpr int BMs = 64, BKs = 64, LDS = BKs + 8, JR = NT * 8;
-  __shared__ __align__(16) uint16_t xs[2][BMs * LDS];
-  __shared__ __align__(16) uint16_t ws[2][JR * LDS];
+  constexpr int BMs = 64, BKs = 64, LDS = BKs + 8, JR = NT * 8, LDP = JR + 4;
+  constexpr int XS_BYTES = 2 * BMs * LDS * 2, WS_BYTES = 2 * JR * LDS * 2;
+  static_assert(BMs * LDP * 4 <= XS_BYTES + WS_BYTES, "partial fits in the staging buffers");
+  __shared__ __align__(16) uint8_t smraw[XS_BYTES + WS_BYTES];
+  uint16_t (*xs)[BMs * LDS] = reinterpret_cast<uint16_t (*)[BMs * LDS]>(smraw);
+  uint16_t (*ws)[JR * LDS] = reinterpret_cast<uint16_t (*)[JR * LDS]>(smraw + XS_BYTES);
+  float* part = reinterpret_cast<float*>(smraw);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int64_t m0 = static_cast<int64_t>(blockIdx.x) * BMs;
   float acc[NT][4];
@@ -44,11 +55,13 @@ __global__ void __launch_bounds__(128) skinny_gemm_kernel(const uint16_t* __rest
     }
     cp_async_commit();
   };
-  const int nk = static_cast<int>(K / BKs);
-  load(0, 0);
+  const int nk_all = static_cast<int>(K / BKs);
+  const int kt0 = blockIdx.y * kt_split;
+  const int nk = max(0, min(nk_all, kt0 + kt_split) - kt0);
+  if (nk > 0) load(0, static_cast<int64_t>(kt0) * BKs);
   for (int kt = 0; kt < nk; ++kt) {
     if (kt + 1 < nk) {
-      load((kt + 1) & 1, static_cast<int64_t>(kt + 1) * BKs);
+      load((kt + 1) & 1, static_cast<int64_t>(kt0 + kt + 1) * BKs);
       cp_async_wait<1>();
     } else {
       cp_async_wait<0>();
@@ -71,29 +84,78 @@ __global__ void __launch_bounds__(128) skinny_gemm_kernel(const uint16_t* __rest
     __syncthreads();
   }
   const int r = lane >> 2, c = (lane & 3) * 2;
-  const int64_t row0 = m0 + warp * 16 + r;
+  if (gridDim.y == 1) {
+    const int64_t row0 = m0 + warp * 16 + r;
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+      const int col = nt * 8 + c;
+      if (row0 < M)
+        *reinterpret_cast<uint32_t*>(out + row0 * ldo + col) = pack_half2(alpha * acc[nt][0], alpha * acc[nt][1]);
+      if (row0 + 8 < M)
+        *reinterpret_cast<uint32_t*>(out + (row0 + 8) * ldo + col) =
+            pack_half2(alpha * acc[nt][2], alpha * acc[nt][3]);
+    }
+    return;
+  }
+  // split K: partial tile into own shared memory (the staging buffers are idle after the loop)
+  const int pr = warp * 16 + r;
 #pragma unroll
   for (int nt = 0; nt < NT; ++nt) {
-    const int col = nt * 8 + c;
-    if (row0 < M)
-      *reinterpret_cast<uint32_t*>(out + row0 * ldo + col) = pack_half2(alpha * acc[nt][0], alpha * acc[nt][1]);
-    if (row0 + 8 < M)
-      *reinterpret_cast<uint32_t*>(out + (row0 + 8) * ldo + col) =
-          pack_half2(alpha * acc[nt][2], alpha * acc[nt][3]);
+    *reinterpret_cast<float2*>(part + pr * LDP + nt * 8 + c) = make_float2(acc[nt][0], acc[nt][1]);
+    *reinterpret_cast<float2*>(part + (pr + 8) * LDP + nt * 8 + c) = make_float2(acc[nt][2], acc[nt][3]);
   }
+  cluster_sync_all();
+  const int S = gridDim.y, z = blockIdx.y;
+  const int rpc = (BMs + S - 1) / S;
+  const int r0 = z * rpc, r1 = min(BMs, r0 + rpc);
+  constexpr int C4 = JR / 4;
+  const uint32_t base = smem_u32(part);
+  for (int i = tid; i < (r1 - r0) * C4; i += 128) {
+    const int rr = r0 + i / C4, cc = (i % C4) * 4;
+    const int64_t row = m0 + rr;
+    if (row >= M) continue;
+    const uint32_t off = base + (rr * LDP + cc) * 4;
+    float4 v[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      if (j < S) v[j] = ld_dsmem_f4(dsmem_addr(off, j));
+    float4 sum = v[0];
+#pragma unroll
+    for (int j = 1; j < 8; ++j)
+      if (j < S) {
+        sum.x += v[j].x; sum.y += v[j].y; sum.z += v[j].z; sum.w += v[j].w;
+      }
+    *reinterpret_cast<uint2*>(out + row * ldo + cc) =
+        make_uint2(pack_half2(alpha * sum.x, alpha * sum.y), pack_half2(alpha * sum.z, alpha * sum.w));
+  }
+  cluster_sync_all();  // no CTA leaves while its partial is being read
+}
+
+template <int NT>
+void skinny_launch(const uint16_t* X, int64_t ldx, int64_t M, int64_t K, const uint16_t* W, int64_t ldw, float alpha,
+                   uint16_t* out, int64_t ldo, cudaStream_t st) {
+  const int gx = static_cast<int>((M + 63) / 64);
+  const int nk = static_cast<int>(K / 64);
+  // Split K over a cluster when the row blocks alone leave most of the SMs idle: up to 8 splits
+  // of >= 2 K tiles, at most ~2 CTAs per SM in total.
+  int splits = 1;
+  if (gx < 152) splits = std::max(1, std::min({8, nk / 2, (2 * 152) / gx}));
+  const int kt_split = (nk + splits - 1) / splits;
+  splits = std::max(1, (nk + kt_split - 1) / kt_split);
+  launch_k_cluster(skinny_gemm_kernel<NT>, dim3(gx, splits), 128, 0, st, dim3(1, splits, 1), X, ldx, M, K, W, ldw,
+                   alpha, out, ldo, kt_split);
 }
 
 void launch_skinny_gemm(const uint16_t* X, int64_t ldx, int64_t M, int64_t K, const uint16_t* W, int64_t ldw, int J,
                         float alpha, uint16_t* out, int64_t ldo, cudaStream_t st) {
   (void)J;  // W holds ldo rows (zero beyond the used ranks), so every output column is written
   if (M <= 0) return;
-  const unsigned grid = static_cast<unsigned>((M + 63) / 64);
   switch (ldo) {
-    case 16: launch_k(skinny_gemm_kernel<2>, grid, 128, 0, st, X, ldx, M, K, W, ldw, alpha, out, ldo); break;
-    case 32: launch_k(skinny_gemm_kernel<4>, grid, 128, 0, st, X, ldx, M, K, W, ldw, alpha, out, ldo); break;
-    case 48: launch_k(skinny_gemm_kernel<6>, grid, 128, 0, st, X, ldx, M, K, W, ldw, alpha, out, ldo); break;
-    case 64: launch_k(skinny_gemm_kernel<8>, grid, 128, 0, st, X, ldx, M, K, W, ldw, alpha, out, ldo); break;
-    default: launch_k(skinny_gemm_kernel<12>, grid, 128, 0, st, X, ldx, M, K, W, ldw, alpha, out, ldo); break;
+    case 16: skinny_launch<2>(X, ldx, M, K, W, ldw, alpha, out, ldo, st); break;
+    case 32: skinny_launch<4>(X, ldx, M, K, W, ldw, alpha, out, ldo, st); break;
+    case 48: skinny_launch<6>(X, ldx, M, K, W, ldw, alpha, out, ldo, st); break;
+    case 64: skinny_launch<8>(X, ldx, M, K, W, ldw, alpha, out, ldo, st); break;
+    default: skinny_launch<12>(X, ldx, M, K, W, ldw, alpha, out, ldo, st); break;
   }
 }
 
@@ -247,26 +309,36 @@ int launch_tall_reduce(const uint16_t* P, int64_t ldp, const uint16_t* Q, int64_
 }
 
 // ------------------------------------------------------------------------------------ shadows
-struct ShadowArgs {
-  const float* A[3];
-  const float* B[3];
+// Per-layer LoRA masters of one fused linear (up to 3 targets side by side).
+struct ShadowTable {
+  const float* A[kShadowMaxLayers][3];
+  const float* B[kShadowMaxLayers][3];
   int ro[3];     // rank offset of target t in the concatenated rank axis
   int no[3];     // first output row of target t
   int nl[3];     // output rows of target t
   int nt;
 };
 
-__global__ void lora_shadow_kernel(ShadowArgs a, int r, int K, int N, int kx, uint16_t* __restrict__ A_cat,
-                                   uint16_t* __restrict__ B_cat, uint16_t* __restrict__ Bt_cat) {
+// Layer blockIdx.y: A_cat [kx, K], B_cat [N, kx], Bt_cat [kx, N] at offsets layer * (stride_a,
+// stride_b, stride_b).
+__global__ void lora_shadow_kernel(ShadowTable a, int r, int K, int N, int kx, uint16_t* __restrict__ A_cat,
+                                   uint16_t* __restrict__ B_cat, uint16_t* __restrict__ Bt_cat, int64_t stride_a,
+                                   int64_t stride_b) {
   griddep_wait();
   griddep_launch();
+  const int layer = blockIdx.y;
+  const float* const* As = a.A[layer];
+  const float* const* Bs = a.B[layer];
+  A_cat += layer * stride_a;
+  B_cat += layer * stride_b;
+  Bt_cat += layer * stride_b;
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   const int64_t na = static_cast<int64_t>(kx) * K, nb = static_cast<int64_t>(N) * kx;
   if (i < na) {
     const int j = static_cast<int>(i / K), k = static_cast<int>(i % K);
     float v = 0.0f;
     for (int t = 0; t < a.nt; ++t)
-      if (j >= a.ro[t] && j < a.ro[t] + r) v = a.A[t][static_cast<int64_t>(j - a.ro[t]) * K + k];
+      if (j >= a.ro[t] && j < a.ro[t] + r) v = As[t][static_cast<int64_t>(j - a.ro[t]) * K + k];
     A_cat[i] = f_to_h(v);
   }
   if (i < nb) {
@@ -274,28 +346,47 @@ __global__ void lora_shadow_kernel(ShadowArgs a, int r, int K, int N, int kx, ui
     float v = 0.0f;
     for (int t = 0; t < a.nt; ++t)
       if (j >= a.ro[t] && j < a.ro[t] + r && n >= a.no[t] && n < a.no[t] + a.nl[t])
-        v = a.B[t][static_cast<int64_t>(n - a.no[t]) * r + (j - a.ro[t])];
+        v = Bs[t][static_cast<int64_t>(n - a.no[t]) * r + (j - a.ro[t])];
     const uint16_t b = f_to_h(v);
     B_cat[i] = b;
     Bt_cat[static_cast<int64_t>(j) * N + n] = b;
   }
 }
 
+void launch_lora_shadow_layers(int n_layers, const float* const* A, const float* const* B, int nt,
+                               const int* ranks_off, const int* n_off, const int* n_len, int r, int K, int N, int kx,
+                               uint16_t* A_cat, uint16_t* B_cat, uint16_t* Bt_cat, int64_t stride_a, int64_t stride_b,
+                               cudaStream_t st) {
+  const int64_t n = std::max(static_cast<int64_t>(kx) * K, static_cast<int64_t>(N) * kx);
+  for (int l0 = 0; l0 < n_layers; l0 += kShadowMaxLayers) {
+    const int nl_batch = std::min(kShadowMaxLayers, n_layers - l0);
+    ShadowTable a{};
+    a.nt = nt;
+    for (int t = 0; t < nt && t < 3; ++t) {
+      a.ro[t] = ranks_off[t];
+      a.no[t] = n_off[t];
+      a.nl[t] = n_len[t];
+      for (int l = 0; l < nl_batch; ++l) {
+        a.A[l][t] = A[(l0 + l) * 3 + t];
+        a.B[l][t] = B[(l0 + l) * 3 + t];
+      }
+    }
+    launch_k(lora_shadow_kernel, dim3(static_cast<unsigned>((n + 255) / 256), static_cast<unsigned>(nl_batch)), 256,
+             0, st, a, r, K, N, kx, A_cat + l0 * stride_a, B_cat + l0 * stride_b, Bt_cat + l0 * stride_b, stride_a,
+             stride_b);
+  }
+}
+
 void launch_lora_shadow(const float* const* A, const float* const* B, int nt, const int* ranks_off, const int* n_off,
                         const int* n_len, int r, int K, int N, int kx, uint16_t* A_cat, uint16_t* B_cat,
                         uint16_t* Bt_cat, cudaStream_t st) {
-  ShadowArgs a{};
-  a.nt = nt;
+  const float* Al[3] = {nullptr, nullptr, nullptr};
+  const float* Bl[3] = {nullptr, nullptr, nullptr};
   for (int t = 0; t < nt && t < 3; ++t) {
-    a.A[t] = A[t];
-    a.B[t] = B[t];
-    a.ro[t] = ranks_off[t];
-    a.no[t] = n_off[t];
-    a.nl[t] = n_len[t];
+    Al[t] = A[t];
+    Bl[t] = B[t];
   }
-  const int64_t n = std::max(static_cast<int64_t>(kx) * K, static_cast<int64_t>(N) * kx);
-  launch_k(lora_shadow_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, st, a, r, K, N, kx, A_cat, B_cat,
-           Bt_cat);
+  launch_lora_shadow_layers(1, Al, Bl, nt, ranks_off, n_off, n_len, r, K, N, kx, A_cat, B_cat, Bt_cat, 0, 0, st);
 }
 
 }  // namespace mebp

@@ -50,11 +50,17 @@ bool mebp::pdl_take() {
 // One block's forward intermediates (what the backward consumes) and the fp16 LoRA shadows they
 // were computed with.  The step keeps two sets so that the recompute of block i-1 can run on a
 // second stream while the backward of block i reads the other set.
+// fp16 LoRA shadows of one block's fused linears: A_cat [kxp, K], B_cat [N, kxp], Bt_cat [kxp, N].
+struct Shadow {
+  uint16_t *A_cat[4] = {}, *B_cat[4] = {}, *Bt_cat[4] = {};
+};
+
 struct Acts {
   uint16_t *a = nullptr, *qkv = nullptr, *o = nullptr, *b = nullptr, *gu = nullptr, *m = nullptr;
   float *r1 = nullptr, *r2 = nullptr, *lse_attn = nullptr, *h1 = nullptr;
   uint16_t* us[4] = {nullptr, nullptr, nullptr, nullptr};
-  uint16_t *A_cat[4] = {}, *B_cat[4] = {}, *Bt_cat[4] = {};
+  Shadow own;                  // shadows built by the forward itself
+  const Shadow* sh = nullptr;  // the shadows the set was computed with
   // which block / input / token count the set currently holds (-1: none)
   int layer = -1;
   const float* x = nullptr;
@@ -87,6 +93,7 @@ struct mebp_ctx {
   // forward intermediates: set 0 always, set 1 when the step overlaps recompute and backward
   Acts act[2];
   int nsets = 1;
+  std::vector<Shadow> layer_sh;  // the step's shadows, built for every block at once
   cudaStream_t fstream = nullptr;  // recompute stream of the overlapped backward
   cudaEvent_t ev_main = nullptr;   // main-stream progress, waited on by the recompute stream
   cudaEvent_t ev_fwd[2] = {};      // recompute into set k finished
@@ -260,7 +267,7 @@ int run_gemm(mebp_ctx* c, GemmArgs& g, cudaStream_t st, const char* what) {
 }
 
 // fp16 shadows of one fused linear's LoRA masters.
-void build_shadow(mebp_ctx* c, Acts& A, int li, const mebp_lora* lora, cudaStream_t st) {
+void build_shadow(mebp_ctx* c, Shadow& A, int li, const mebp_lora* lora, cudaStream_t st) {
   const Lin& l = c->lin[li];
   if (!l.kx) return;
   const float* As[3];
@@ -286,19 +293,23 @@ int check_lora(mebp_ctx* c, const mebp_lora* lora) {
 // y = F(x) for one block.  with_down == false stops after the MLP activation (what the
 // backward consumes), so y is not produced.
 int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, const mebp_lora* lora, const float* x,
-                  float* y, int B, int Sq, bool with_down, cudaStream_t st) {
+                  float* y, int B, int Sq, bool with_down, cudaStream_t st, const Shadow* sh = nullptr) {
   Acts& A = c->act[set];
   const int64_t T = static_cast<int64_t>(B) * Sq;
   const int D = c->D, I = c->I;
   int rc;
-  for (int li = 0; li < 4; ++li) build_shadow(c, A, li, lora, st);
+  if (!sh) {
+    for (int li = 0; li < 4; ++li) build_shadow(c, A.own, li, lora, st);
+    sh = &A.own;
+  }
+  A.sh = sh;
   // attention sub-block
   launch_rmsnorm_fwd(x, w->norm1, T, D, c->cfg.rms_eps, A.a, A.r1, st);
   const Lin& lq = c->lin[LIN_QKV];
   GemmArgs g = gemm_fwd(A.a, D, T, w->qkv, lq.N, lq.K);
   if (lq.kx) {
-    launch_skinny_gemm(A.a, D, T, D, A.A_cat[LIN_QKV], D, lq.kx, c->s, A.us[LIN_QKV], lq.kxp, st);
-    g.Ax = A.us[LIN_QKV]; g.ldax = lq.kxp; g.kx = lq.kxp; g.Bx = A.B_cat[LIN_QKV]; g.ldbx = lq.kxp;
+    launch_skinny_gemm(A.a, D, T, D, A.sh->A_cat[LIN_QKV], D, lq.kx, c->s, A.us[LIN_QKV], lq.kxp, st);
+    g.Ax = A.us[LIN_QKV]; g.ldax = lq.kxp; g.kx = lq.kxp; g.Bx = A.sh->B_cat[LIN_QKV]; g.ldbx = lq.kxp;
   }
   g.epi = EPI_F16; g.C = A.qkv; g.ldc = lq.N;
   if ((rc = run_gemm(c, g, st, "qkv"))) return rc;
@@ -307,8 +318,8 @@ int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, 
   const Lin& lo = c->lin[LIN_O];
   g = gemm_fwd(A.o, c->Na, T, w->o, lo.N, lo.K);
   if (lo.kx) {
-    launch_skinny_gemm(A.o, c->Na, T, c->Na, A.A_cat[LIN_O], c->Na, lo.kx, c->s, A.us[LIN_O], lo.kxp, st);
-    g.Ax = A.us[LIN_O]; g.ldax = lo.kxp; g.kx = lo.kxp; g.Bx = A.B_cat[LIN_O]; g.ldbx = lo.kxp;
+    launch_skinny_gemm(A.o, c->Na, T, c->Na, A.sh->A_cat[LIN_O], c->Na, lo.kx, c->s, A.us[LIN_O], lo.kxp, st);
+    g.Ax = A.us[LIN_O]; g.ldax = lo.kxp; g.kx = lo.kxp; g.Bx = A.sh->B_cat[LIN_O]; g.ldbx = lo.kxp;
   }
   g.epi = EPI_F32; g.C = A.h1; g.ldc = D; g.R = x; g.ldr = D;
   if ((rc = run_gemm(c, g, st, "o_proj"))) return rc;
@@ -317,18 +328,18 @@ int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, 
   const Lin& lg = c->lin[LIN_GU];
   g = gemm_fwd(A.b, D, T, w->gate_up, lg.N, lg.K);
   if (lg.kx) {
-    launch_skinny_gemm(A.b, D, T, D, A.A_cat[LIN_GU], D, lg.kx, c->s, A.us[LIN_GU], lg.kxp, st);
-    g.Ax = A.us[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = A.B_cat[LIN_GU]; g.ldbx = lg.kxp;
+    launch_skinny_gemm(A.b, D, T, D, A.sh->A_cat[LIN_GU], D, lg.kx, c->s, A.us[LIN_GU], lg.kxp, st);
+    g.Ax = A.us[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = A.sh->B_cat[LIN_GU]; g.ldbx = lg.kxp;
   }
   g.epi = EPI_F16; g.C = A.gu; g.ldc = lg.N;
   if ((rc = run_gemm(c, g, st, "gate_up"))) return rc;
   launch_glu_fwd(A.gu, T, I, c->cfg.act, A.m, st);
   const Lin& ld = c->lin[LIN_DOWN];
-  if (ld.kx) launch_skinny_gemm(A.m, I, T, I, A.A_cat[LIN_DOWN], I, ld.kx, c->s, A.us[LIN_DOWN], ld.kxp, st);
+  if (ld.kx) launch_skinny_gemm(A.m, I, T, I, A.sh->A_cat[LIN_DOWN], I, ld.kx, c->s, A.us[LIN_DOWN], ld.kxp, st);
   if (with_down) {
     g = gemm_fwd(A.m, I, T, w->down, ld.N, ld.K);
     if (ld.kx) {
-      g.Ax = A.us[LIN_DOWN]; g.ldax = ld.kxp; g.kx = ld.kxp; g.Bx = A.B_cat[LIN_DOWN]; g.ldbx = ld.kxp;
+      g.Ax = A.us[LIN_DOWN]; g.ldax = ld.kxp; g.kx = ld.kxp; g.Bx = A.sh->B_cat[LIN_DOWN]; g.ldbx = ld.kxp;
     }
     g.epi = EPI_F32; g.C = y; g.ldc = D; g.R = A.h1; g.ldr = D;
     if ((rc = run_gemm(c, g, st, "down"))) return rc;
@@ -369,7 +380,7 @@ int lin_grads(mebp_ctx* c, const Acts& A, const uint16_t* du, int li, const uint
 int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_weights* w, const mebp_lora* lora,
                    const float* x, const float* dy, const uint16_t* dy_h, float* dx, uint16_t* dx_h,
                    const mebp_lora_grads* grads, int B, int Sq, bool acc, const float* grad_mult,
-                   const float* dx_mult, cudaStream_t st) {
+                   const float* dx_mult, cudaStream_t st, const Shadow* sh = nullptr) {
   Acts& A = c->act[set];
   Grads2& G = c->bw[bset];
   uint16_t* const* du = G.du;
@@ -377,15 +388,15 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   const int D = c->D, I = c->I;
   int rc;
   if (!(A.layer == layer && A.x == x && A.T == T)) {
-    if ((rc = block_forward(c, set, layer, w, lora, x, nullptr, B, Sq, false, st))) return rc;
+    if ((rc = block_forward(c, set, layer, w, lora, x, nullptr, B, Sq, false, st, sh))) return rc;
   }
   A.layer = -1;  // the set is consumed below
   // ---- down projection: y = h1 + m Wd^T (+ s (m Ad^T) Bd^T)
   const Lin& ld = c->lin[LIN_DOWN];
   GemmArgs g = gemm_dx(dy_h, D, T, w->down);
   if (ld.kx) {
-    launch_skinny_gemm(dy_h, D, T, D, A.Bt_cat[LIN_DOWN], D, ld.kx, c->s, du[LIN_DOWN], ld.kxp, st);
-    g.Ax = du[LIN_DOWN]; g.ldax = ld.kxp; g.kx = ld.kxp; g.Bx = A.A_cat[LIN_DOWN]; g.ldbx = I;
+    launch_skinny_gemm(dy_h, D, T, D, A.sh->Bt_cat[LIN_DOWN], D, ld.kx, c->s, du[LIN_DOWN], ld.kxp, st);
+    g.Ax = du[LIN_DOWN]; g.ldax = ld.kxp; g.kx = ld.kxp; g.Bx = A.sh->A_cat[LIN_DOWN]; g.ldbx = I;
   }
   g.epi = EPI_F32; g.C = c->dm; g.ldc = I;
   if ((rc = run_gemm(c, g, st, "down dX"))) return rc;
@@ -395,8 +406,8 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   const Lin& lg = c->lin[LIN_GU];
   g = gemm_dx(G.dgu, 2 * I, T, w->gate_up);
   if (lg.kx) {
-    launch_skinny_gemm(G.dgu, 2 * I, T, 2 * I, A.Bt_cat[LIN_GU], 2 * I, lg.kx, c->s, du[LIN_GU], lg.kxp, st);
-    g.Ax = du[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = A.A_cat[LIN_GU]; g.ldbx = D;
+    launch_skinny_gemm(G.dgu, 2 * I, T, 2 * I, A.sh->Bt_cat[LIN_GU], 2 * I, lg.kx, c->s, du[LIN_GU], lg.kxp, st);
+    g.Ax = du[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = A.sh->A_cat[LIN_GU]; g.ldbx = D;
   }
   g.epi = EPI_F32; g.C = c->dtmp; g.ldc = D;
   if ((rc = run_gemm(c, g, st, "gate_up dX"))) return rc;
@@ -407,8 +418,8 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   const Lin& lo = c->lin[LIN_O];
   g = gemm_dx(G.dh1_h, D, T, w->o);
   if (lo.kx) {
-    launch_skinny_gemm(G.dh1_h, D, T, D, A.Bt_cat[LIN_O], D, lo.kx, c->s, du[LIN_O], lo.kxp, st);
-    g.Ax = du[LIN_O]; g.ldax = lo.kxp; g.kx = lo.kxp; g.Bx = A.A_cat[LIN_O]; g.ldbx = c->Na;
+    launch_skinny_gemm(G.dh1_h, D, T, D, A.sh->Bt_cat[LIN_O], D, lo.kx, c->s, du[LIN_O], lo.kxp, st);
+    g.Ax = du[LIN_O]; g.ldax = lo.kxp; g.kx = lo.kxp; g.Bx = A.sh->A_cat[LIN_O]; g.ldbx = c->Na;
   }
   g.epi = EPI_F16; g.C = c->dout; g.ldc = c->Na;
   if ((rc = run_gemm(c, g, st, "o dX"))) return rc;
@@ -420,12 +431,12 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   launch_rope(G.dqkv, T, Sq, c->H, c->KV, c->hd, c->rope_cs, true, st);
   // ---- q, k, v projections
   if (lq.kx)
-    launch_skinny_gemm(G.dqkv, lq.N, T, lq.N, A.Bt_cat[LIN_QKV], lq.N, lq.kx, c->s, du[LIN_QKV], lq.kxp, st);
+    launch_skinny_gemm(G.dqkv, lq.N, T, lq.N, A.sh->Bt_cat[LIN_QKV], lq.N, lq.kx, c->s, du[LIN_QKV], lq.kxp, st);
   if ((rc = lin_grads(c, A, du[LIN_QKV], LIN_QKV, G.dqkv, lq.N, A.a, D, T, grads, acc, grad_mult, st))) return rc;
   if (dx) {
     g = gemm_dx(G.dqkv, lq.N, T, w->qkv);
     if (lq.kx) {
-      g.Ax = du[LIN_QKV]; g.ldax = lq.kxp; g.kx = lq.kxp; g.Bx = A.A_cat[LIN_QKV]; g.ldbx = D;
+      g.Ax = du[LIN_QKV]; g.ldax = lq.kxp; g.kx = lq.kxp; g.Bx = A.sh->A_cat[LIN_QKV]; g.ldbx = D;
     }
     g.epi = EPI_F32; g.C = c->dtmp; g.ldc = D;
     if ((rc = run_gemm(c, g, st, "qkv dX"))) return rc;
@@ -564,9 +575,24 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
       const Lin& l = c->lin[li];
       if (!l.kx) continue;
       A(&s.us[li], T * l.kxp);
-      A(&s.A_cat[li], static_cast<int64_t>(l.kxp) * l.K);
-      A(&s.B_cat[li], static_cast<int64_t>(l.N) * l.kxp);
-      A(&s.Bt_cat[li], static_cast<int64_t>(l.N) * l.kxp);
+      A(&s.own.A_cat[li], static_cast<int64_t>(l.kxp) * l.K);
+      A(&s.own.B_cat[li], static_cast<int64_t>(l.N) * l.kxp);
+      A(&s.own.Bt_cat[li], static_cast<int64_t>(l.N) * l.kxp);
+    }
+  }
+  // the step's per-block shadows (one allocation per linear, blocks back to back)
+  c->layer_sh.assign(c->L, Shadow{});
+  for (int li = 0; li < 4; ++li) {
+    const Lin& l = c->lin[li];
+    if (!l.kx) continue;
+    uint16_t *pa = nullptr, *pb = nullptr, *pbt = nullptr;
+    const int64_t na = static_cast<int64_t>(l.kxp) * l.K, nb = static_cast<int64_t>(l.N) * l.kxp;
+    A(&pa, na * c->L); A(&pb, nb * c->L); A(&pbt, nb * c->L);
+    if (rc != MEBP_OK) break;
+    for (int i = 0; i < c->L; ++i) {
+      c->layer_sh[i].A_cat[li] = pa + i * na;
+      c->layer_sh[i].B_cat[li] = pb + i * nb;
+      c->layer_sh[i].Bt_cat[li] = pbt + i * nb;
     }
   }
   for (int k = 0; k < c->nsets; ++k) {
@@ -905,6 +931,21 @@ static int lora_step_body(mebp_ctx* c, const mebp_model_weights* model, const me
   const bool spill = c->cfg.spill_ckpts != 0;
   pdl_entry();
   launch_k(targets_kernel, static_cast<unsigned>((T + 255) / 256), 256, 0, st, ids, B, Sq, c->targets);
+  // fp16 shadows of every block's LoRA masters, one launch per fused linear
+  for (int li = 0; li < 4; ++li) {
+    const Lin& l = c->lin[li];
+    if (!l.kx) continue;
+    std::vector<const float*> As(3 * static_cast<size_t>(L), nullptr), Bs(3 * static_cast<size_t>(L), nullptr);
+    for (int i = 0; i < L; ++i)
+      for (int t = 0; t < l.nt; ++t) {
+        As[3 * i + t] = lora[i].A[l.tgt[t]];
+        Bs[3 * i + t] = lora[i].B[l.tgt[t]];
+      }
+    const Shadow& s0 = c->layer_sh[0];
+    launch_lora_shadow_layers(L, As.data(), Bs.data(), l.nt, l.ro, l.no, l.nl, c->r, l.K, l.N, l.kxp, s0.A_cat[li],
+                              s0.B_cat[li], s0.Bt_cat[li], static_cast<int64_t>(l.kxp) * l.K,
+                              static_cast<int64_t>(l.N) * l.kxp, st);
+  }
   // Checkpoint placement (Algorithm 1's ckpts_storage): HBM slot i, or, when spilling, a ring
   // of kCkptSlots device slots whose contents are copied to / from pinned host memory on a
   // side stream (the stand-in for memory-mapped checkpoints).
@@ -974,7 +1015,9 @@ static int lora_step_body(mebp_ctx* c, const mebp_model_weights* model, const me
       wait_free(sl);  // its previous contents reached the host
       yout = dev_ckpt(sl);
     }
-    if ((rc = block_forward(c, i % c->nsets, i, &model->blocks[i], &lora[i], xin, yout, B, Sq, true, st))) return rc;
+    if ((rc = block_forward(c, i % c->nsets, i, &model->blocks[i], &lora[i], xin, yout, B, Sq, true, st,
+                            &c->layer_sh[i])))
+      return rc;
     if (spill && i + 1 < L) spill_out(i + 1);
   }
   // ---- loss subgraph: final norm + LM head + CE
@@ -1007,7 +1050,7 @@ static int lora_step_body(mebp_ctx* c, const mebp_model_weights* model, const me
     if (!overlap) {
       if ((rc = block_backward(c, set, 0, i, &model->blocks[i], &lora[i], xin, c->gbuf[cur], c->dy_h[cur],
                                i > 0 ? c->gbuf[nxt] : nullptr, i > 0 ? c->dy_h[nxt] : nullptr, &grads[i], B, Sq,
-                               accumulate != 0, c->scal + 1, nullptr, st)))
+                               accumulate != 0, c->scal + 1, nullptr, st, &c->layer_sh[i])))
         return rc;
     } else {
       if (i > 0) {  // recompute block i-1 into the other set once its readers are done with it
@@ -1018,7 +1061,7 @@ static int lora_step_body(mebp_ctx* c, const mebp_model_weights* model, const me
         const Acts& P = c->act[ps];
         if (!(P.layer == i - 1 && P.x == dev_ckpt(i - 1) && P.T == T) &&
             (rc = block_forward(c, ps, i - 1, &model->blocks[i - 1], &lora[i - 1], dev_ckpt(i - 1), nullptr, B, Sq,
-                                false, c->fstream)))
+                                false, c->fstream, &c->layer_sh[i - 1])))
           return rc;
         cudaEventRecord(c->ev_fwd[ps], c->fstream);
       }
