@@ -272,6 +272,36 @@ def run_gpu(args, d, rank, world, local_rank):
     return out
 
 
+def launch_list_step(args, d):
+    """Warm-up steps, then one step run eagerly (no graph replay) inside an NVTX range, so a
+    profiler can list exactly the kernels of one step."""
+    import torch
+
+    from paper_2510_03425_gb300 import mebp as M
+    from paper_2510_03425_gb300.model import Context, LoraSet
+    device = torch.device("cuda", 0)
+    ctx = Context(d, device=0)
+    model = build_model(ctx, d, device)
+    ls = LoraSet([synth.lora_weights(d, i) for i in range(d.n_layers)], device=device)
+    ids = torch.from_numpy(synth.token_ids(d)).to(device)
+    loss = torch.zeros(1, device=device)
+    mstruct = model.struct()
+    st = torch.cuda.Stream(device)
+    torch.cuda.set_stream(st)
+    for _ in range(args.warmup):
+        M.mebp_lora_step(ctx.handle, mstruct, ls.lora_array(), ids, loss, ls.grads_array(), False, st)
+    ctx.sync()
+    M.mebp_enable_graphs(ctx.handle, False)
+    n0 = M.mebp_kernel_launches()
+    torch.cuda.nvtx.range_push("mebp_step")
+    M.mebp_lora_step(ctx.handle, mstruct, ls.lora_array(), ids, loss, ls.grads_array(), False, st)
+    torch.cuda.nvtx.range_pop()
+    ctx.sync()
+    print(json.dumps({"launch_list_step": workload_name(d), "kernels": M.mebp_kernel_launches() - n0,
+                      "loss": float(loss.item())}), flush=True)
+    ctx.close()
+
+
 def gemm_bench(config: int, m_tokens=None, reps: int = 10, warmup: int = 3, shapes_only=None):
     """The fused dequant-GEMMs alone (forward Y = X deq(W)^T and transposed dX = dY deq(W)) at
     the four projection shapes of a workload, M = its token count.  Returns a dict."""
@@ -333,7 +363,7 @@ def gemm_bench(config: int, m_tokens=None, reps: int = 10, warmup: int = 3, shap
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=150)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--config", type=int, default=1, help="workload preset 0..4 (default 1)")
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
@@ -342,6 +372,9 @@ def main():
                     help="time only the fused dequant-GEMMs at the config's projection shapes")
     ap.add_argument("--gemm-m", type=int, default=None, help="token count M for --gemm-bench")
     ap.add_argument("--gemm-shapes", default=None, help="comma list of qkv,o,gate_up,down for --gemm-bench")
+    ap.add_argument("--launch-list", action="store_true",
+                    help="no timing: after the warm-up run one eager step inside the NVTX range "
+                         "'mebp_step' (for ncu --nvtx --nvtx-include mebp_step/)")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     rank = int(os.environ.get("RANK", "0"))
@@ -353,6 +386,10 @@ def main():
         out = gemm_bench(args.config, args.gemm_m, reps=args.steps, warmup=args.warmup,
                          shapes_only=args.gemm_shapes.split(",") if args.gemm_shapes else None)
         print(json.dumps(out), flush=True)
+        return
+
+    if args.launch_list:
+        launch_list_step(args, d)
         return
 
     if args.impl == "reference":
