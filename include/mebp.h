@@ -51,7 +51,7 @@ enum { MEBP_ACT_SILU = 0, MEBP_ACT_GELU_TANH = 1 };
 typedef struct {
   int32_t hidden;        /* D                                                                   */
   int32_t n_heads;       /* H   (query heads)                                                   */
-  int32_t n_kv_heads;    /* KV  (key/value heads; H % KV == 0)                                  */
+  int32_t n_kv_heads;    /* KV  (key/value heads; H % KV == 0, H / KV <= 8)                     */
   int32_t head_dim;      /* hd  in {64, 128, 256}                                               */
   int32_t intermediate;  /* I   (gated-MLP width)                                               */
   int32_t vocab;         /* V   (tied embedding / LM head rows; 0 = no LM head)                 */

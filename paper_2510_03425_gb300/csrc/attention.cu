@@ -5,10 +5,11 @@
 //             reads key/value head h / (H/KV).  Saves lse = log-sum-exp of each score row.
 //   backward: dP = dO v^T, dS = P (dP - rowsum(dO o)), dq = dS k / sqrt(hd),
 //             dk = dS^T q / sqrt(hd), dv = P^T dO; dk, dv summed over the query heads of a
-//             group.  P is recomputed from q, k and lse.  dk/dv (one CTA per key block and
-//             kv head, looping over the group's query heads) and dq (one CTA per query block)
-//             are separate passes so every output element is written exactly once
-//             (deterministic, no atomics).
+//             group.  P is recomputed from q, k and lse.  One launch holds two kinds of work
+//             item: dk/dv (one CTA per key block and query head; the query heads of a kv head
+//             form a thread-block cluster that sums their partials over distributed shared
+//             memory) and dq (one CTA per query block and head), so every output element is
+//             written exactly once (deterministic, no atomics).
 // q, k, v live in the fused projection buffer [T, (H + 2 KV) hd] (q heads, k heads, v heads);
 // token t = b*S + s.
 #include "kernels.h"
@@ -207,20 +208,37 @@ __global__ void dvec_kernel(const uint16_t* __restrict__ o, const uint16_t* __re
   }
 }
 
-// dK, dV for one key block, output columns d0 .. d0 + DC.  Grouped mode (part == null): one CTA
-// per kv head loops over the query heads of its group and writes fp16 dK, dV.  Per-head mode
-// (small grids): blockIdx.y is a query head; the CTA writes its head's fp32 contribution to
-// part ([2][B*S][H][HD]: dK then dV) and dkdv_group_sum adds the heads of each group.
-template <int HD, int DC>
-__global__ void __launch_bounds__(128, 1) dkdv_kernel(const uint16_t* __restrict__ qkv, int64_t ld,
-                                                      const uint16_t* __restrict__ dout, int64_t ldo,
-                                                      const float* __restrict__ lse, const float* __restrict__ dvec,
-                                                      int S, int H, int KV, uint16_t* __restrict__ dqkv,
-                                                      float* __restrict__ part, int64_t T) {
-  griddep_wait();
-  griddep_launch();
+struct BwdArgs {
+  const uint16_t* qkv;
+  int64_t ld;
+  const uint16_t* dout;
+  int64_t ldo;
+  const float* lse;
+  const float* dvec;
+  int S, H, KV, B;
+  int n_kv;  // dK/dV work items (blocks [0, n_kv)); dQ items follow
+  uint16_t* dqkv;
+};
+
+// dK, dV of one key block kb (output columns d0 .. d0 + DC), accumulated over the query blocks
+// kb .. that see the block.  Every dK/dV element is written once (no atomics, deterministic):
+//   CL = true : one item per query head h; the grp = H/KV query heads of a kv head form one
+//               thread-block cluster (rank j = head kvh*grp + j) whose fp32 partials are summed
+//               over distributed shared memory in head order (small grids);
+//   CL = false: one item per kv head, looping over its grp query heads (large grids).
+template <int HD, int DC, bool CL>
+__device__ __forceinline__ void dkdv_item(const BwdArgs& a, int idx, uint16_t* sm) {
   constexpr int LD = HD + 8, NC = DC / 8, NCH = HD / DC;
-  extern __shared__ __align__(16) uint16_t sm[];
+  const int S = a.S, H = a.H, KV = a.KV;
+  const int grp = H / KV;
+  const int j = CL ? idx % grp : 0;
+  int rest = CL ? idx / grp : idx;
+  const int kvh = rest % KV;
+  rest /= KV;
+  const int nkb = (S + BKV - 1) / BKV;
+  const int kb = rest % nkb, bz = rest / nkb;
+  const int b = bz / NCH, d0 = (bz % NCH) * DC;
+  const int h_first = kvh * grp + j, h_count = CL ? 1 : grp;
   uint16_t* ks = sm;
   uint16_t* vs = ks + BKV * LD;
   // two (Q, dO, lse, dvec) buffers: the next query block loads while this one is used
@@ -229,12 +247,6 @@ __global__ void __launch_bounds__(128, 1) dkdv_kernel(const uint16_t* __restrict
   auto lse_s = [&](int buf) { return reinterpret_cast<float*>(vs + 5 * BQ * LD) + buf * 2 * BQ; };
   auto dv_s = [&](int buf) { return lse_s(buf) + BQ; };
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int grp = H / KV;
-  const bool perhead = part != nullptr;
-  const int kb = blockIdx.x;
-  const int kvh = perhead ? blockIdx.y / grp : blockIdx.y;
-  const int h_first = perhead ? blockIdx.y : kvh * grp, h_count = perhead ? 1 : grp;
-  const int b = blockIdx.z / NCH, d0 = (blockIdx.z % NCH) * DC;
   const int64_t tok0 = static_cast<int64_t>(b) * S;
   const int k0 = kb * BKV;
   const float sc = kLog2e * rsqrtf(static_cast<float>(HD));
@@ -247,22 +259,21 @@ __global__ void __launch_bounds__(128, 1) dkdv_kernel(const uint16_t* __restrict
   }
   const int key_a = k0 + warp * 16 + (lane >> 2);
   const int nqb = (S + BQ - 1) / BQ;
-  const int per_head = nqb - kb;            // query blocks kb .. nqb-1 see this key block
+  const int per_head = nqb - kb;  // query blocks kb .. nqb-1 see this key block
   const int n_it = h_count * per_head;
-  // query block of iteration it -> (head, first query) and its loads into buffer buf
   auto fetch = [&](int it, int buf) {
     const int h = h_first + it / per_head, q0 = (kb + it % per_head) * BQ;
-    load_tile<HD>(qs(buf), qkv, ld, tok0, q0, S, h * HD, tid);
-    load_tile<HD>(dos(buf), dout, ldo, tok0, q0, S, h * HD, tid);
+    load_tile<HD>(qs(buf), a.qkv, a.ld, tok0, q0, S, h * HD, tid);
+    load_tile<HD>(dos(buf), a.dout, a.ldo, tok0, q0, S, h * HD, tid);
     for (int i = tid; i < BQ; i += 128) {
       const int q = q0 + i;
       const int64_t li = (static_cast<int64_t>(b) * H + h) * S + q;
-      lse_s(buf)[i] = q < S ? lse[li] * kLog2e : 0.0f;
-      dv_s(buf)[i] = q < S ? dvec[li] : 0.0f;
+      lse_s(buf)[i] = q < S ? a.lse[li] * kLog2e : 0.0f;
+      dv_s(buf)[i] = q < S ? a.dvec[li] : 0.0f;
     }
   };
-  load_tile<HD>(ks, qkv, ld, tok0, k0, S, (H + kvh) * HD, tid);
-  load_tile<HD>(vs, qkv, ld, tok0, k0, S, (H + KV + kvh) * HD, tid);
+  load_tile<HD>(ks, a.qkv, a.ld, tok0, k0, S, (H + kvh) * HD, tid);
+  load_tile<HD>(vs, a.qkv, a.ld, tok0, k0, S, (H + KV + kvh) * HD, tid);
   if (n_it > 0) fetch(0, 0);
   cp_async_commit();
 
@@ -279,7 +290,6 @@ __global__ void __launch_bounds__(128, 1) dkdv_kernel(const uint16_t* __restrict
     __syncthreads();
     const float* lsb = lse_s(buf);
     const float* dvb = dv_s(buf);
-
     // P^T (16 keys x 64 queries)
     float pt[8][4];
     qk_tile<HD>(pt, smem_u32(ks), smem_u32(qs(buf)), warp, lane);
@@ -308,64 +318,92 @@ __global__ void __launch_bounds__(128, 1) dkdv_kernel(const uint16_t* __restrict
     pv_tile<HD, NC>(dk, dpt, smem_u32(qs(buf)), d0, lane);
     __syncthreads();  // every warp is done with this buffer before it is refilled
   }
+
   const float inv = rsqrtf(static_cast<float>(HD));
   const int c = 2 * (lane & 3);
-  if (perhead) {
+  if (!CL || grp == 1) {
 #pragma unroll
     for (int i = 0; i < 2; ++i) {
       const int key = key_a + 8 * i;
       if (key >= S) continue;
-      float* krow = part + ((tok0 + key) * H + h_first) * HD + d0;
-      float* vrow = krow + T * H * HD;
+      uint16_t* krow = a.dqkv + (tok0 + key) * a.ld + (H + kvh) * HD + d0;
+      uint16_t* vrow = a.dqkv + (tok0 + key) * a.ld + (H + KV + kvh) * HD + d0;
 #pragma unroll
       for (int dt = 0; dt < NC; ++dt) {
-        *reinterpret_cast<float2*>(krow + dt * 8 + c) = make_float2(dk[dt][2 * i] * inv, dk[dt][2 * i + 1] * inv);
-        *reinterpret_cast<float2*>(vrow + dt * 8 + c) = make_float2(dv[dt][2 * i], dv[dt][2 * i + 1]);
+        *reinterpret_cast<uint32_t*>(krow + dt * 8 + c) = pack_half2(dk[dt][2 * i] * inv, dk[dt][2 * i + 1] * inv);
+        *reinterpret_cast<uint32_t*>(vrow + dt * 8 + c) = pack_half2(dv[dt][2 * i], dv[dt][2 * i + 1]);
       }
     }
     return;
   }
+  // partials [64 keys][DC] for dK then dV, fp32, in the idle tile buffers
+  constexpr int LDP = DC + 4;
+  static_assert(2 * BKV * LDP * 4 <= 6 * 64 * LD * 2, "partials fit in the tile buffers");
+  float* pk = reinterpret_cast<float*>(sm);
+  float* pv = pk + BKV * LDP;
 #pragma unroll
   for (int i = 0; i < 2; ++i) {
-    const int key = key_a + 8 * i;
-    if (key >= S) continue;
-    uint16_t* krow = dqkv + (tok0 + key) * ld + (H + kvh) * HD + d0;
-    uint16_t* vrow = dqkv + (tok0 + key) * ld + (H + KV + kvh) * HD + d0;
+    const int kr = warp * 16 + (lane >> 2) + 8 * i;
 #pragma unroll
     for (int dt = 0; dt < NC; ++dt) {
-      *reinterpret_cast<uint32_t*>(krow + dt * 8 + c) = pack_half2(dk[dt][2 * i] * inv, dk[dt][2 * i + 1] * inv);
-      *reinterpret_cast<uint32_t*>(vrow + dt * 8 + c) = pack_half2(dv[dt][2 * i], dv[dt][2 * i + 1]);
+      *reinterpret_cast<float2*>(pk + kr * LDP + dt * 8 + c) = make_float2(dk[dt][2 * i], dk[dt][2 * i + 1]);
+      *reinterpret_cast<float2*>(pv + kr * LDP + dt * 8 + c) = make_float2(dv[dt][2 * i], dv[dt][2 * i + 1]);
     }
   }
+  cluster_sync_all();
+  const int rpc = (BKV + grp - 1) / grp;
+  const int r0 = j * rpc, r1 = min(BKV, r0 + rpc);
+  constexpr int C4 = DC / 4;
+  const uint32_t base = smem_u32(sm);
+  for (int i = tid; i < 2 * (r1 - r0) * C4; i += 128) {
+    const int which = i / ((r1 - r0) * C4);  // 0: dK, 1: dV
+    const int e = i % ((r1 - r0) * C4);
+    const int kr = r0 + e / C4, cc = (e % C4) * 4;
+    const int key = k0 + kr;
+    if (key >= S) continue;
+    const uint32_t off = base + ((which * BKV + kr) * LDP + cc) * 4;
+    float4 v[8];
+#pragma unroll
+    for (int t = 0; t < 8; ++t)
+      if (t < grp) v[t] = ld_dsmem_f4(dsmem_addr(off, t));
+    float4 sum = v[0];
+#pragma unroll
+    for (int t = 1; t < 8; ++t)
+      if (t < grp) {
+        sum.x += v[t].x; sum.y += v[t].y; sum.z += v[t].z; sum.w += v[t].w;
+      }
+    const float m = which ? 1.0f : inv;
+    uint16_t* dst = a.dqkv + (tok0 + key) * a.ld + (H + which * KV + kvh) * HD + d0 + cc;
+    *reinterpret_cast<uint2*>(dst) = make_uint2(pack_half2(sum.x * m, sum.y * m), pack_half2(sum.z * m, sum.w * m));
+  }
+  cluster_sync_all();  // no CTA leaves while its partials are being read
 }
 
 // dQ for one query block of one head, output columns d0 .. d0 + DC.
 template <int HD, int DC>
-__global__ void __launch_bounds__(128, 1) dq_kernel(const uint16_t* __restrict__ qkv, int64_t ld,
-                                                    const uint16_t* __restrict__ dout, int64_t ldo,
-                                                    const float* __restrict__ lse, const float* __restrict__ dvec,
-                                                    int S, int H, int KV, uint16_t* __restrict__ dqkv) {
-  griddep_wait();
-  griddep_launch();
+__device__ __forceinline__ void dq_item(const BwdArgs& a, int idx, uint16_t* sm) {
   constexpr int LD = HD + 8, NC = DC / 8, NCH = HD / DC;
-  extern __shared__ __align__(16) uint16_t sm[];
+  const int S = a.S, H = a.H, KV = a.KV;
+  const int h = idx % H;
+  const int rest = idx / H;
+  const int nqb = (S + BQ - 1) / BQ;
+  const int qb = rest % nqb, bz = rest / nqb;
+  const int b = bz / NCH, d0 = (bz % NCH) * DC;
   uint16_t* qs = sm;
   uint16_t* dos = qs + BQ * LD;
   // two (K, V) buffers: the next key block loads while this one is used
   auto ks = [&](int buf) { return dos + (1 + 2 * buf) * BQ * LD; };
   auto vs = [&](int buf) { return dos + (2 + 2 * buf) * BQ * LD; };
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int qb = blockIdx.x, h = blockIdx.y;
-  const int b = blockIdx.z / NCH, d0 = (blockIdx.z % NCH) * DC;
   const int kvh = h / (H / KV);
   const int64_t tok0 = static_cast<int64_t>(b) * S;
   const int q0 = qb * BQ;
   const float sc = kLog2e * rsqrtf(static_cast<float>(HD));
 
-  load_tile<HD>(qs, qkv, ld, tok0, q0, S, h * HD, tid);
-  load_tile<HD>(dos, dout, ldo, tok0, q0, S, h * HD, tid);
-  load_tile<HD>(ks(0), qkv, ld, tok0, 0, S, (H + kvh) * HD, tid);
-  load_tile<HD>(vs(0), qkv, ld, tok0, 0, S, (H + KV + kvh) * HD, tid);
+  load_tile<HD>(qs, a.qkv, a.ld, tok0, q0, S, h * HD, tid);
+  load_tile<HD>(dos, a.dout, a.ldo, tok0, q0, S, h * HD, tid);
+  load_tile<HD>(ks(0), a.qkv, a.ld, tok0, 0, S, (H + kvh) * HD, tid);
+  load_tile<HD>(vs(0), a.qkv, a.ld, tok0, 0, S, (H + KV + kvh) * HD, tid);
   cp_async_commit();
   const int ra = q0 + warp * 16 + (lane >> 2);
   float lse2[2], dvv[2];
@@ -373,8 +411,8 @@ __global__ void __launch_bounds__(128, 1) dq_kernel(const uint16_t* __restrict__
   for (int i = 0; i < 2; ++i) {
     const int row = ra + 8 * i;
     const int64_t li = (static_cast<int64_t>(b) * H + h) * S + row;
-    lse2[i] = row < S ? lse[li] * kLog2e : 0.0f;
-    dvv[i] = row < S ? dvec[li] : 0.0f;
+    lse2[i] = row < S ? a.lse[li] * kLog2e : 0.0f;
+    dvv[i] = row < S ? a.dvec[li] : 0.0f;
   }
   float dq[NC][4];
 #pragma unroll
@@ -383,8 +421,8 @@ __global__ void __launch_bounds__(128, 1) dq_kernel(const uint16_t* __restrict__
   for (int kb = 0; kb <= qb; ++kb) {
     const int k0 = kb * BKV, buf = kb & 1;
     if (kb < qb) {
-      load_tile<HD>(ks(buf ^ 1), qkv, ld, tok0, k0 + BKV, S, (H + kvh) * HD, tid);
-      load_tile<HD>(vs(buf ^ 1), qkv, ld, tok0, k0 + BKV, S, (H + KV + kvh) * HD, tid);
+      load_tile<HD>(ks(buf ^ 1), a.qkv, a.ld, tok0, k0 + BKV, S, (H + kvh) * HD, tid);
+      load_tile<HD>(vs(buf ^ 1), a.qkv, a.ld, tok0, k0 + BKV, S, (H + KV + kvh) * HD, tid);
       cp_async_commit();
       cp_async_wait<1>();
     } else {
@@ -417,11 +455,39 @@ __global__ void __launch_bounds__(128, 1) dq_kernel(const uint16_t* __restrict__
   for (int i = 0; i < 2; ++i) {
     const int row = ra + 8 * i;
     if (row >= S) continue;
-    uint16_t* qrow = dqkv + (tok0 + row) * ld + h * HD + d0;
+    uint16_t* qrow = a.dqkv + (tok0 + row) * a.ld + h * HD + d0;
 #pragma unroll
     for (int dt = 0; dt < NC; ++dt)
       *reinterpret_cast<uint32_t*>(qrow + dt * 8 + c) = pack_half2(dq[dt][2 * i] * inv, dq[dt][2 * i + 1] * inv);
   }
+}
+
+// Small grids: one launch for both backward passes; blocks [0, n_kv) are dK/dV items (clusters
+// of the grp query heads of a kv head), the rest dQ items, and the two kinds run concurrently.
+// n_kv is a multiple of grp, so no cluster mixes the kinds.
+template <int HD, int DC>
+__global__ void __launch_bounds__(128, 1) bwd_kernel(const BwdArgs a) {
+  griddep_wait();
+  griddep_launch();
+  extern __shared__ __align__(16) uint16_t sm[];
+  if (static_cast<int>(blockIdx.x) < a.n_kv) dkdv_item<HD, DC, true>(a, blockIdx.x, sm);
+  else dq_item<HD, DC>(a, blockIdx.x - a.n_kv, sm);
+}
+
+// Large grids: dK/dV with one CTA per kv head, then dQ, as two launches.
+template <int HD, int DC>
+__global__ void __launch_bounds__(128, 1) dkdv_kernel(const BwdArgs a) {
+  griddep_wait();
+  griddep_launch();
+  extern __shared__ __align__(16) uint16_t sm[];
+  dkdv_item<HD, DC, false>(a, blockIdx.x, sm);
+}
+template <int HD, int DC>
+__global__ void __launch_bounds__(128, 1) dq_kernel(const BwdArgs a) {
+  griddep_wait();
+  griddep_launch();
+  extern __shared__ __align__(16) uint16_t sm[];
+  dq_item<HD, DC>(a, blockIdx.x, sm);
 }
 
 template <int HD, int NB>
@@ -447,56 +513,32 @@ void fwd_launch(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, ui
   else fwd_launch_nb<HD, 2>(qkv, ld, B, S, H, KV, o, ldo, lse, st);
 }
 
-// dK, dV of kv head j = sum over the query heads of group j of the per-head partials (fixed order).
-__global__ void dkdv_group_sum(const float* __restrict__ part, int64_t T, int H, int KV, int HD, int64_t ld,
-                               uint16_t* __restrict__ dqkv) {
-  griddep_wait();
-  griddep_launch();
-  const int64_t n2 = T * KV * HD / 2;
-  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (i >= 2 * n2) return;
-  const int which = i >= n2;  // 0: dK, 1: dV
-  const int64_t r = (which ? i - n2 : i) * 2;
-  const int d = static_cast<int>(r % HD);
-  const int j = static_cast<int>((r / HD) % KV);
-  const int64_t t = r / (static_cast<int64_t>(HD) * KV);
-  const int grp = H / KV;
-  const float* src = part + which * T * H * HD + (t * H + j * grp) * HD + d;
-  float a = 0.0f, b2 = 0.0f;
-  for (int hh = 0; hh < grp; ++hh) {
-    a += src[hh * HD];
-    b2 += src[hh * HD + 1];
-  }
-  *reinterpret_cast<uint32_t*>(dqkv + t * ld + (H + which * KV + j) * HD + d) = pack_half2(a, b2);
-}
-
 template <int HD, int DC>
 void bwd_launch(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t ldo, const float* lse,
-                const float* dvec, int B, int S, int H, int KV, uint16_t* dqkv, float* part, int64_t part_floats,
-                cudaStream_t st) {
+                const float* dvec, int B, int S, int H, int KV, uint16_t* dqkv, cudaStream_t st) {
   constexpr int smem = 6 * 64 * (HD + 8) * 2 + 4 * 64 * 4;  // 6 tiles (2 of them double-buffered) + lse, dvec x 2
   static_assert(smem <= 232448, "attention backward shared memory");
   static bool init = false;
   if (!init) {
+    cudaFuncSetAttribute(bwd_kernel<HD, DC>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     cudaFuncSetAttribute(dkdv_kernel<HD, DC>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     cudaFuncSetAttribute(dq_kernel<HD, DC>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     init = true;
   }
   constexpr int NCH = HD / DC;
-  const int64_t T = static_cast<int64_t>(B) * S;
-  const int nkb = (S + BKV - 1) / BKV;
-  // One CTA per query head when one per kv head leaves most of the 152 SMs idle.
-  const bool perhead = H > KV && part && static_cast<int64_t>(nkb) * KV * B * NCH < 2 * 152 &&
-                       2 * T * H * HD <= part_floats;
-  dim3 g1(nkb, perhead ? H : KV, B * NCH);
-  launch_k(dkdv_kernel<HD, DC>, g1, 128, smem, st, qkv, ld, dout, ldo, lse, dvec, S, H, KV, dqkv,
-           perhead ? part : nullptr, T);
-  if (perhead) {
-    const int64_t n = T * KV * HD;
-    launch_k(dkdv_group_sum, static_cast<unsigned>((n + 255) / 256), 256, 0, st, part, T, H, KV, HD, ld, dqkv);
+  const int nkb = (S + BKV - 1) / BKV, nqb = (S + BQ - 1) / BQ;
+  const int grp = H / KV;
+  BwdArgs a{qkv, ld, dout, ldo, lse, dvec, S, H, KV, B, 0, dqkv};
+  const int n_q = nqb * H * B * NCH;      // a multiple of grp (H is)
+  const int n_grouped = nkb * KV * B * NCH;
+  if (n_grouped >= 2 * 152) {             // the per-kv-head items alone fill the GPU twice
+    a.n_kv = n_grouped;
+    launch_k(dkdv_kernel<HD, DC>, dim3(a.n_kv), 128, smem, st, a);
+    launch_k(dq_kernel<HD, DC>, dim3(n_q), 128, smem, st, a);
+    return;
   }
-  dim3 g2((S + BQ - 1) / BQ, H, B * NCH);
-  launch_k(dq_kernel<HD, DC>, g2, 128, smem, st, qkv, ld, dout, ldo, lse, dvec, S, H, KV, dqkv);
+  a.n_kv = nkb * H * B * NCH;             // one item per (key block, query head, batch, column chunk)
+  launch_k_cluster(bwd_kernel<HD, DC>, dim3(a.n_kv + n_q), 128, smem, st, dim3(grp, 1, 1), a);
 }
 
 }  // namespace attn
@@ -510,14 +552,14 @@ void launch_attn_fwd(const uint16_t* qkv, int64_t ld, int B, int S, int H, int K
 
 void launch_attn_bwd(const uint16_t* qkv, int64_t ld, const uint16_t* o, const uint16_t* dout, int64_t ldo,
                      const float* lse, int B, int S, int H, int KV, int hd, float* dvec, uint16_t* dqkv,
-                     float* part, int64_t part_floats, cudaStream_t st) {
+                     cudaStream_t st) {
   const int64_t nw = static_cast<int64_t>(B) * S * H;
   launch_k(attn::dvec_kernel, static_cast<unsigned>((nw * 32 + 255) / 256), 256, 0, st, o, dout, ldo, B, S, H, hd,
            dvec);
-  if (hd == 64) attn::bwd_launch<64, 64>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, part, part_floats, st);
+  if (hd == 64) attn::bwd_launch<64, 64>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, st);
   else if (hd == 128)
-    attn::bwd_launch<128, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, part, part_floats, st);
-  else attn::bwd_launch<256, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, part, part_floats, st);
+    attn::bwd_launch<128, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, st);
+  else attn::bwd_launch<256, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, st);
 }
 
 }  // namespace mebp

@@ -165,6 +165,6 @@ void launch_attn_fwd(const uint16_t* qkv, int64_t ld, int B, int S, int H, int K
 // part: fp32 scratch (>= 2 * B*S * H * hd floats for the per-head dK/dV mode), may be null.
 void launch_attn_bwd(const uint16_t* qkv, int64_t ld, const uint16_t* o, const uint16_t* dout, int64_t ldo,
                      const float* lse, int B, int S, int H, int KV, int hd, float* dvec, uint16_t* dqkv,
-                     float* part, int64_t part_floats, cudaStream_t st);
+                     cudaStream_t st);
 
 }  // namespace mebp

@@ -108,8 +108,6 @@ struct mebp_ctx {
   float *dm = nullptr, *dtmp = nullptr, *dh1 = nullptr, *dvec = nullptr, *gbuf[2] = {nullptr, nullptr};
   float* red = nullptr;
   int64_t red_floats = 0;
-  float* split_ws = nullptr;   // fp32 per-head partials of the attention backward
-  int64_t split_ws_floats = 0;
   // LM head
   uint16_t *hf = nullptr, *dz = nullptr;
   float *rf = nullptr, *part = nullptr, *zt = nullptr, *lse_tok = nullptr, *tok_loss = nullptr,
@@ -426,8 +424,7 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   if ((rc = lin_grads(c, A, du[LIN_O], LIN_O, G.dh1_h, D, A.o, c->Na, T, grads, acc, grad_mult, st))) return rc;
   // ---- attention, RoPE
   const Lin& lq = c->lin[LIN_QKV];
-  launch_attn_bwd(A.qkv, lq.N, A.o, c->dout, c->Na, A.lse_attn, B, Sq, c->H, c->KV, c->hd, c->dvec, G.dqkv,
-                  c->split_ws, c->split_ws_floats, st);
+  launch_attn_bwd(A.qkv, lq.N, A.o, c->dout, c->Na, A.lse_attn, B, Sq, c->H, c->KV, c->hd, c->dvec, G.dqkv, st);
   launch_rope(G.dqkv, T, Sq, c->H, c->KV, c->hd, c->rope_cs, true, st);
   // ---- q, k, v projections
   if (lq.kx)
@@ -536,6 +533,7 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
       f.vocab < 0 || f.vocab % 64 || f.lora_rank < 0 || f.lora_rank > 32)
     return MEBP_ERR_INVALID_ARG;
   if (!(f.head_dim == 64 || f.head_dim == 128 || f.head_dim == 256)) return MEBP_ERR_UNSUPPORTED;
+  if (f.n_heads / f.n_kv_heads > 8) return MEBP_ERR_UNSUPPORTED;  // query heads per kv head: one cluster
   if (f.lora_targets && (f.lora_rank % 8)) return MEBP_ERR_UNSUPPORTED;
   if (f.act != MEBP_ACT_SILU && f.act != MEBP_ACT_GELU_TANH) return MEBP_ERR_INVALID_ARG;
   if (f.vocab_chunk < 0 || f.vocab_chunk % 256) return MEBP_ERR_INVALID_ARG;
@@ -621,8 +619,6 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
   c->red_floats = std::max<int64_t>(tall_reduce_scratch_floats(T, std::max<int64_t>(2 * I, c->Nqkv), 32),
                                     tall_reduce_scratch_floats(T, std::max<int64_t>(I, D), 32));
   A(&c->red, c->red_floats);
-  c->split_ws_floats = int64_t(16) << 20;
-  A(&c->split_ws, c->split_ws_floats);
   if (c->V > 0) {
     c->nparts = 2 * ((c->V + 255) / 256);
     int64_t vc = f.vocab_chunk;
