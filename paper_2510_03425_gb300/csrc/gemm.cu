@@ -6,13 +6,13 @@
 //   (FWD: A_x = s X A^T, B_x = B [N, Kx];  TRANS: A_x = s dY B, B_x = A [Kx, N]).
 //
 // This is the decompression of Algorithm 1's LazyLoadAndDecompressWeights fused into the GEMM:
-// TMA brings the packed 4-bit tile and its fp16 scales into shared memory, eight converter
+// TMA brings the packed 4-bit tile and its fp16 scales into shared memory, sixteen converter
 // warps turn them into the fp16 operand (bit-exact fp16_rne(q*s), see dequant.cuh) in the
 // 128-byte-swizzled layout tcgen05 reads, one thread issues tcgen05.mma into fp32 TMEM
-// accumulators, and the same eight warps run the epilogue out of TMEM.
+// accumulators, and the same sixteen warps run the epilogue out of TMEM.
 //
-// CTA: 320 threads.  warps 0-7 convert + epilogue, warp 8 issues TMA, warp 9 issues MMA and
-// owns the TMEM allocation.  Tile (128*NACC) x 256 x 64: NACC 128-row A tiles share every
+// CTA: 16 (NACC 1) or 8 (NACC 2) converter warps that also run the epilogue, then one warp that
+// issues TMA and one that issues MMA and owns the TMEM allocation.  Tile (128*NACC) x 256 x 64: NACC 128-row A tiles share every
 // decoded 256-row B tile (NACC = 2 halves the decode work per flop and fills all 512 TMEM
 // columns).  Two shared-memory rings: a TMA ring (A tile(s) + packed nibbles + scales, with
 // separate barriers for the weight half and the activation half, so weights can be fetched and
@@ -30,7 +30,18 @@
 namespace mebp {
 namespace gemm {
 
-constexpr int BM = 128, BN = 256, BK = 64, THREADS = 320;
+constexpr int BM = 128, BN = 256, BK = 64;
+// Decode + epilogue warps: 16 (two threads per decoded row) when one 128-row accumulator uses
+// each decoded tile, so the decode keeps pace with the tensor pipe; 8 with two accumulators,
+// where the decode is not the limit and fewer warps compete with the MMA-issuing thread.
+template <int NACC>
+struct Warps {
+  static constexpr int CONV = NACC == 1 ? 16 : 8;
+  static constexpr int TPR = CONV / 8;  // converter threads per decoded 256-row tile row
+  static constexpr int CONV_THREADS = CONV * 32;
+  static constexpr int TMA = CONV, MMA = CONV + 1;
+  static constexpr int THREADS = CONV_THREADS + 64;
+};
 constexpr int B_BYTES = BN * BK * 2, A_BYTES = BM * BK * 2, P_BYTES = BN * BK / 2, S_BYTES = 512;
 
 // Shared-memory layout for NACC accumulators (tiles 1024-byte aligned).
@@ -79,61 +90,81 @@ struct Params {
 };
 
 // ---------------------------------------------------------------------------------- convert
-// FWD: packed tile [256 rows][32 B] (plain), scales [256]; thread t converts row t (one group)
-// into the K-major SW128 B tile (row t at t*128 B, 16-byte chunk j stored at chunk j ^ (t&7)).
+// TPR converter threads per decoded row (1 or 2): thread t handles part h of its row's 8 words.
+// FWD: packed tile [256 rows][32 B] (plain), scales [256]; row r = t / TPR goes to the K-major
+// SW128 B tile (row r at r*128 B, 16-byte chunk j stored at chunk j ^ (r&7)).
+template <int TPR>
 __device__ __forceinline__ void convert_fwd(const uint8_t* pk, const uint8_t* sc, uint8_t* bt, int t) {
-  const uint4* src = reinterpret_cast<const uint4*>(pk + t * 32);
-  const uint4 p0 = src[0], p1 = src[1];
-  const uint32_t s2 = scale_pair(reinterpret_cast<const uint16_t*>(sc)[t]);
-  uint8_t* row = bt + t * 128;
-  const uint32_t words[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
+  constexpr int NW = 8 / TPR;
+  const int r = t / TPR, h = t % TPR;
+  const uint4* src = reinterpret_cast<const uint4*>(pk + r * 32) + h * (NW / 4);
+  uint32_t words[NW];
 #pragma unroll
-  for (int j = 0; j < 8; ++j) {
+  for (int i = 0; i < NW / 4; ++i) {
+    const uint4 p = src[i];
+    words[4 * i] = p.x; words[4 * i + 1] = p.y; words[4 * i + 2] = p.z; words[4 * i + 3] = p.w;
+  }
+  const uint32_t s2 = scale_pair(reinterpret_cast<const uint16_t*>(sc)[r]);
+  uint8_t* row = bt + r * 128;
+#pragma unroll
+  for (int w = 0; w < NW; ++w) {
+    const int j = NW * h + w;
     uint32_t o[4];
-    dequant_word(words[j], s2, o);
-    *reinterpret_cast<uint4*>(row + ((j ^ (t & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
+    dequant_word(words[w], s2, o);
+    *reinterpret_cast<uint4*>(row + ((j ^ (r & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
   }
 }
 
 // TRANS: packed tile [64 k-rows][128 B] loaded with the 128-byte swizzle (chunk c of row k at
-// chunk c ^ (k&7)), scales [4 groups][64 k-rows].  Thread t: group g = t/64 (64 output
-// columns), row k = t%64; its 8 words become chunks 0..7 of row k of MN-major atom g
-// (atom = 64 columns x 64 k-rows, 128 B per k-row, chunk c stored at c ^ (k&7)).
+// chunk c ^ (k&7)), scales [4 groups][64 k-rows].  Thread t: row k = t & 63, group g =
+// (t >> 6) & 3 (64 output columns), part h = t >> 8; packed chunks 2g .. 2g+1 (part h of them)
+// become chunks of row k of MN-major atom g (atom = 64 columns x 64 k-rows, 128 B per k-row,
+// chunk c stored at c ^ (k&7)).  Consecutive threads take consecutive k: conflict-free.
+template <int TPR>
 __device__ __forceinline__ void convert_trans(const uint8_t* pk, const uint8_t* sc, uint8_t* bt, int t) {
-  const int g = t >> 6, k = t & 63;
+  constexpr int NW = 8 / TPR;
+  const int k = t & 63, g = (t >> 6) & 3, h = t >> 8;
   const uint8_t* prow = pk + k * 128;
-  const uint4 p0 = *reinterpret_cast<const uint4*>(prow + (((2 * g) ^ (k & 7)) << 4));
-  const uint4 p1 = *reinterpret_cast<const uint4*>(prow + (((2 * g + 1) ^ (k & 7)) << 4));
+  uint32_t words[NW];
+#pragma unroll
+  for (int i = 0; i < NW / 4; ++i) {
+    const int c = 2 * g + h * (NW / 4) + i;
+    const uint4 p = *reinterpret_cast<const uint4*>(prow + ((c ^ (k & 7)) << 4));
+    words[4 * i] = p.x; words[4 * i + 1] = p.y; words[4 * i + 2] = p.z; words[4 * i + 3] = p.w;
+  }
   const uint32_t s2 = scale_pair(reinterpret_cast<const uint16_t*>(sc)[g * 64 + k]);
   uint8_t* row = bt + g * 8192 + k * 128;
-  const uint32_t words[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
 #pragma unroll
-  for (int j = 0; j < 8; ++j) {
+  for (int w = 0; w < NW; ++w) {
+    const int j = NW * h + w;
     uint32_t o[4];
-    dequant_word(words[j], s2, o);
+    dequant_word(words[w], s2, o);
     *reinterpret_cast<uint4*>(row + ((j ^ (k & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
   }
 }
 
 // LoRA block e: copy the 64-wide slice of B_x into the B slot in the layout the MMA reads,
 // zero outside [0, kx) x [0, N).  The operand is a few tens of KB and stays in L2.
-template <bool TRANS>
+template <bool TRANS, int TPR>
 __device__ __forceinline__ void copy_lora_b(const Params& p, int e, int n0, uint8_t* bt, int t) {
+  constexpr int NW = 8 / TPR;
   const uint4 zero = make_uint4(0, 0, 0, 0);
-  if (!TRANS) {  // K-major: row n = t, chunk j = 8 columns of the rank axis
-    const int n = n0 + t;
+  if (!TRANS) {  // K-major: row r, chunk j = 8 columns of the rank axis
+    const int r = t / TPR, h = t % TPR, n = n0 + r;
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
+    for (int w = 0; w < NW; ++w) {
+      const int j = NW * h + w;
       const int col = e * 64 + 8 * j;
       uint4 v = zero;
       if (n < p.N && col < p.kx) v = *reinterpret_cast<const uint4*>(p.Bx + static_cast<int64_t>(n) * p.ldbx + col);
-      *reinterpret_cast<uint4*>(bt + t * 128 + ((j ^ (t & 7)) << 4)) = v;
+      *reinterpret_cast<uint4*>(bt + r * 128 + ((j ^ (r & 7)) << 4)) = v;
     }
   } else {       // MN-major: atom g (64 output columns), row k of the rank axis
-    const int g = t >> 6, k = t & 63;
+    const int k = t & 63, g = (t >> 6) & 3, h = t >> 8;
     const int rr = e * 64 + k;
 #pragma unroll
-    for (int c = 0; c < 8; ++c) {
+    for (int w = 0; w < NW; ++w) {
+      const int c = NW * h + w;
       const int col = n0 + 64 * g + 8 * c;
       uint4 v = zero;
       if (rr < p.kx && col < p.N) v = *reinterpret_cast<const uint4*>(p.Bx + static_cast<int64_t>(rr) * p.ldbx + col);
@@ -143,17 +174,23 @@ __device__ __forceinline__ void copy_lora_b(const Params& p, int e, int n0, uint
 }
 
 // ---------------------------------------------------------------------------------- epilogue
-// NACC = 1: warp w owns TMEM lanes 32*(w&3) .. +31 (tile rows) and columns 128*(w>>2) .. +127.
-// NACC = 2: warp w owns lanes 32*(w&3) .. +31 of accumulator w>>2 (tile rows 128*(w>>2) + ...)
-//           and all 256 columns.
+// Warp w reads TMEM lanes 32*(w&3) .. +31 (a warp may only touch its lane quarter); the warps
+// of a quarter split the NACC x 256 accumulator columns into column groups cg = w >> 2:
+// NACC = 1 (16 warps): columns 64*cg .. +63 of the single accumulator;
+// NACC = 2 (8 warps):  accumulator cg (tile rows 128*cg + ...), all 256 columns.
 template <int NACC>
 __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int warp, int lane, int m0, int n0) {
-  const int q = warp & 3, h = warp >> 2;
-  constexpr int NCH = (NACC == 2) ? 8 : 4;  // 32-column chunks per thread
-  const int row = m0 + (NACC == 2 ? 128 * h : 0) + 32 * q + lane;
+  const int q = warp & 3, cg = warp >> 2;
+  constexpr int NCG = Warps<NACC>::CONV / 4;            // column groups
+  constexpr int COLS = NACC * 256 / NCG;                // columns per group
+  constexpr int NCH = COLS / 32;                        // 32-column chunks per thread
+  static_assert(COLS <= 256 && 256 % COLS == 0, "a column group stays in one accumulator");
+  const int acc = (cg * COLS) / 256;
+  const int col0 = (cg * COLS) % 256;
+  const int row = m0 + 128 * acc + 32 * q + lane;
   const bool row_ok = row < p.M;
-  const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * q) << 16) + (NACC == 2 ? 256 * h : 128 * h);
-  const int cbase = n0 + (NACC == 2 ? 0 : 128 * h);  // first GEMM column of this thread's range
+  const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * q) << 16) + 256 * acc + col0;
+  const int cbase = n0 + col0;  // first GEMM column of this thread's range
 
   if (p.epi == EPI_LSE) {
     float mx = -INFINITY, sum = 0.0f, zt = 0.0f;
@@ -180,14 +217,13 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
         mx = nm;
       }
     }
-    if (row_ok) {
-      float2* pr = reinterpret_cast<float2*>(p.lse_part) + static_cast<int64_t>(row) * p.nparts + blockIdx.x * 2;
-      if (NACC == 2) {
-        pr[0] = make_float2(mx, sum);
-        pr[1] = make_float2(-INFINITY, 0.0f);
-      } else {
-        pr[h] = make_float2(mx, sum);
-      }
+    if (row_ok) {  // four (max, sum) parts per 256-column tile and row; unused parts are empty
+      float2* pr = reinterpret_cast<float2*>(p.lse_part) + static_cast<int64_t>(row) * p.nparts + blockIdx.x * 4;
+      constexpr int GPR = 256 / COLS;      // column groups per row (1 or 4)
+      const int part = col0 / COLS;
+      pr[part] = make_float2(mx, sum);
+      if (GPR == 1)
+        for (int k = 1; k < 4; ++k) pr[k] = make_float2(-INFINITY, 0.0f);
       if (has_t) p.zt[row] = zt;
     }
     return;
@@ -262,12 +298,13 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
 // [z * ceil(128/S), ...) of all S partials over distributed shared memory in split order
 // (deterministic) and applies the epilogue.
 __device__ __forceinline__ void stash_partial(uint32_t tmem, bool valid, int warp, int lane, uint8_t* smem) {
-  const int q = warp & 3, h = warp >> 2;
+  static_assert(Warps<1>::CONV == 16, "one-accumulator kernels stash with 16 warps of 64 columns");
+  const int q = warp & 3, cg = warp >> 2;
   const int r = 32 * q + lane;
-  const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * q) << 16) + 128 * h;
+  const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * q) << 16) + 64 * cg;
   uint8_t* row = smem + r * 1024;
 #pragma unroll 1
-  for (int cc = 0; cc < 4; ++cc) {
+  for (int cc = 0; cc < 2; ++cc) {
     float v[32];
     if (valid) {
       tmem_ld32(tbase + 32 * cc, v);
@@ -277,7 +314,7 @@ __device__ __forceinline__ void stash_partial(uint32_t tmem, bool valid, int war
     }
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-      const int c = 32 * h + 8 * cc + i;
+      const int c = 16 * cg + 8 * cc + i;
       *reinterpret_cast<float4*>(row + ((c ^ (r & 31)) << 4)) =
           make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
     }
@@ -289,7 +326,7 @@ __device__ __forceinline__ void split_reduce(const Params& p, const uint8_t* sme
   const int rpc = (BM + S - 1) / S;
   const int r0 = z * rpc, r1 = min(BM, r0 + rpc);
   const uint32_t base = smem_u32(smem);
-  for (int i = threadIdx.x; i < (r1 - r0) * 64; i += THREADS) {
+  for (int i = threadIdx.x; i < (r1 - r0) * 64; i += Warps<1>::THREADS) {
     const int r = r0 + (i >> 6), c = i & 63;
     const int64_t row = m0 + r, col = n0 + 4 * c;
     if (row >= p.M || col >= p.N) continue;
@@ -323,11 +360,12 @@ __device__ __forceinline__ void split_reduce(const Params& p, const uint8_t* sme
 // of the first ring slots overlap the previous kernel; everything that reads an activation or
 // writes memory waits in griddep_wait() first.
 template <bool TRANS, int NACC>
-__global__ void __launch_bounds__(THREADS, 1)
+__global__ void __launch_bounds__(Warps<NACC>::THREADS, 1)
     dequant_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmP,
                         const __grid_constant__ CUtensorMap tmS, const __grid_constant__ CUtensorMap tmAx,
                         const Params p) {
   using Ly = Layout<NACC>;
+  using Wp = Warps<NACC>;
   constexpr int TSTG = Ly::TSTG, BSTG = Ly::BSTG;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -360,20 +398,20 @@ __global__ void __launch_bounds__(THREADS, 1)
       mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < BSTG; ++b) {
-      mbar_init(&bfull[b], 8);
+      mbar_init(&bfull[b], Wp::CONV);
       mbar_init(&bempty[b], 1);
     }
     mbar_init(accf, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
-  if (warp == 9) tmem_alloc(tmem_slot, Ly::TMEM_COLS);
+  if (warp == Wp::MMA) tmem_alloc(tmem_slot, Ly::TMEM_COLS);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (warp == 8) {
+  if (warp == Wp::TMA) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
       tma_prefetch_desc(&tmA);
@@ -413,7 +451,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       for (int it = (a_issued > TSTG ? a_issued - TSTG : 0); it < a_issued; ++it)
         mbar_wait(&afull[it % TSTG], (it / TSTG) & 1, &dummy, p.err);
     }
-  } else if (warp == 9) {
+  } else if (warp == Wp::MMA) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_f16_f32(BM, BN, TRANS);
@@ -441,7 +479,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
   } else {
     // ------------------------------------------------------------ converters, then epilogue
-    const int t = threadIdx.x;  // 0..255
+    const int t = threadIdx.x;  // 0 .. Wp::CONV_THREADS-1
     for (int it = 0; it < total; ++it) {
       const int s = it % TSTG, b = it % BSTG;
       if (!mbar_wait(&bempty[b], ((it / BSTG) & 1) ^ 1, abort_flag, p.err)) break;
@@ -449,11 +487,11 @@ __global__ void __launch_bounds__(THREADS, 1)
       if (it < num_main) {
         if (!mbar_wait(&wfull[s], (it / TSTG) & 1, abort_flag, p.err)) break;
         const uint8_t* st = smem + s * Ly::T_STRIDE;
-        if (TRANS) convert_trans(st + Ly::P_OFF, st + Ly::S_OFF, bt, t);
-        else convert_fwd(st + Ly::P_OFF, st + Ly::S_OFF, bt, t);
+        if (TRANS) convert_trans<Wp::TPR>(st + Ly::P_OFF, st + Ly::S_OFF, bt, t);
+        else convert_fwd<Wp::TPR>(st + Ly::P_OFF, st + Ly::S_OFF, bt, t);
       } else {
         griddep_wait();  // the LoRA operand comes from an earlier kernel
-        copy_lora_b<TRANS>(p, it - num_main, n0, bt, t);
+        copy_lora_b<TRANS, Wp::TPR>(p, it - num_main, n0, bt, t);
       }
       fence_proxy_async_smem();
       __syncwarp();
@@ -468,7 +506,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 
   tc_fence_before();
   __syncthreads();
-  if (warp == 9) {
+  if (warp == Wp::MMA) {
     if (lane == 0) {  // the accumulator is complete (or every issued MMA has retired) before TMEM is freed
       int dummy = 0;
       mbar_wait(accf, 0, &dummy, p.err);
@@ -539,7 +577,7 @@ int max_active_clusters(int s) {
     if (set_smem_attr<TRANS, 1>()) {
       cudaLaunchConfig_t cfg = {};
       cfg.gridDim = dim3(1, 1, s);
-      cfg.blockDim = dim3(gemm::THREADS);
+      cfg.blockDim = dim3(gemm::Warps<1>::THREADS);
       cfg.dynamicSmemBytes = gemm::Layout<1>::SMEM;
       cudaLaunchAttribute at[1];
       at[0].id = cudaLaunchAttributeClusterDimension;
@@ -564,7 +602,7 @@ int launch_variant(dim3 grid, const CUtensorMap& tA, const CUtensorMap& tP, cons
   if (!set_smem_attr<TRANS, NACC>()) return MEBP_ERR_CUDA;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
-  cfg.blockDim = dim3(gemm::THREADS);
+  cfg.blockDim = dim3(gemm::Warps<NACC>::THREADS);
   cfg.dynamicSmemBytes = gemm::Layout<NACC>::SMEM;
   cfg.stream = st;
   cudaLaunchAttribute at[2];
@@ -594,8 +632,10 @@ int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st) {
   using namespace gemm;
   if (g.M <= 0 || g.N <= 0) return MEBP_OK;
   if (g.K % 64 || g.N % 64 || g.K <= 0) return MEBP_ERR_INVALID_ARG;
-  // Two 128-row accumulators per CTA once M is large enough to fill the GPU with 256-row tiles.
-  const int nacc = (g.M >= 2048) ? 2 : 1;
+  // Two 128-row accumulators per CTA (half the decode work per flop) once 256-row tiles alone give
+  // at least two waves on the 152 SMs (large M, or a large N such as the LM head).
+  const int64_t tiles_n256 = (g.N + BN - 1) / BN;
+  const int nacc = (g.M >= 2048 || (g.M >= 256 && tiles_n256 * ((g.M + 255) / 256) >= 2 * 152)) ? 2 : 1;
   const int bm = BM * nacc;
 
   CUtensorMap tA, tP, tS, tAx;

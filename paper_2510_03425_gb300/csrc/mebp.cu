@@ -620,7 +620,7 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
                                     tall_reduce_scratch_floats(T, std::max<int64_t>(I, D), 32));
   A(&c->red, c->red_floats);
   if (c->V > 0) {
-    c->nparts = 2 * ((c->V + 255) / 256);
+    c->nparts = 4 * ((c->V + 255) / 256);  // four (max, sum) parts per 256-column tile
     int64_t vc = f.vocab_chunk;
     if (vc == 0) {
       vc = (int64_t(1) << 30) / (2 * T);

@@ -77,9 +77,10 @@ def test_embedding_bad_id_flags_device_error(ctx):
     ctx.sync()  # the error word was cleared
 
 
-# (M, N, K): ragged tiles, a single tile, split-K (small grids), and two-accumulator tiles (M >= 2048)
+# (M, N, K): ragged tiles, a single tile, split-K (small grids), two-accumulator tiles (M >= 2048, or
+# a large N: 152 256-column tiles x 2 row tiles), and a transposed pass with a 608-tile split reduction
 SHAPES = [(200, 320, 192), (128, 256, 64), (1, 64, 64), (300, 1152, 896), (513, 512, 1024), (512, 896, 4864),
-          (2048, 256, 128), (2304 + 77, 576, 640)]
+          (2048, 256, 128), (2304 + 77, 576, 640), (300, 38912, 128)]
 
 
 def _x(M_, K, seed, scale=1.0):
