@@ -9,9 +9,10 @@ computes, written from the paper's text:
   VJP of Section 3, "Gradient checkpointing compilation"), the LM-head
   cross-entropy, and Algorithm 1 (checkpointed forward loop, then reverse
   backward loop that recomputes each block from its stored input).
+* ``optim``  — the AdamW update of the LoRA weights (Section 4 trains with AdamW).
 
 Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline leg may
 import this package.  It shares no code with the CUDA path and the product
 never calls it.
 """
-from . import quant, model  # noqa: F401
+from . import quant, model, optim  # noqa: F401
