@@ -272,6 +272,48 @@ def run_gpu(args, d, rank, world, local_rank):
     return out
 
 
+def lora_params(d) -> int:
+    """Trainable LoRA parameters: r * (K_in + N_out) per targeted linear and layer."""
+    shapes = synth.linear_shapes(d)
+    return d.n_layers * sum(d.rank * (shapes[t][0] + shapes[t][1]) for t in d.targets)
+
+
+def adamw_bench(config: int = 4, reps: int = 20, warmup: int = 3):
+    """The AdamW update (mebp_adamw_step) alone over the flat LoRA buffer of a workload: reads
+    p, g, m, v and writes p, m, v, 28 bytes per parameter; HBM-bound."""
+    import torch
+
+    from paper_2510_03425_gb300 import mebp as M
+    from paper_2510_03425_gb300.model import Context
+    d = synth.preset(config)
+    n = lora_params(d)
+    ctx = Context(synth.tiny(vocab=0, head_dim=64), max_tokens=64, max_seq=64)
+    g = torch.Generator(device="cuda")
+    g.manual_seed(11)
+    p = torch.randn(n, device="cuda", generator=g)
+    gr = torch.randn(n, device="cuda", generator=g)
+    m, v = torch.zeros(n, device="cuda"), torch.zeros(n, device="cuda")
+    cfg = M.adamw_cfg(lr=1e-4)
+    for t in range(1, warmup + 1):
+        M.mebp_adamw_step(ctx.handle, p, gr, m, v, cfg, t)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for t in range(warmup + 1, warmup + reps + 1):
+        M.mebp_adamw_step(ctx.handle, p, gr, m, v, cfg, t)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    ctx.sync()
+    ctx.close()
+    pk, src = peaks()
+    gbs = 28.0 * n / (ms / 1e3) / 1e9
+    return {"workload": f"AdamW over the {n} LoRA parameters of {d.name} (r{d.rank} on {'/'.join(d.targets)}), "
+                        f"flat fp32 buffers ({28.0 * n / 1e9:.2f} GB per update, larger than L2)",
+            "bound": "hbm", "us": 1e3 * ms, "achieved": gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
+            "frac": gbs / pk["hbm_gbs"], "peak_source": f"{src} copy bandwidth"}
+
+
 def launch_list_step(args, d):
     """Warm-up steps, then one step run eagerly (no graph replay) inside an NVTX range, so a
     profiler can list exactly the kernels of one step."""
@@ -419,6 +461,7 @@ def main():
     if world == 1:
         # second half of the metric: the fused dequant-GEMM alone at the largest workload's shapes
         out["fused_gemm_isolated"] = gemm_bench(4)
+        out["adamw_isolated"] = adamw_bench(4)
     if world == 1 and not args.no_cpu_baseline:
         v, desc = oracle_sample(d)
         out["cpu_baseline"] = {"value": v, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",

@@ -223,6 +223,27 @@ int mebp_lora_step(mebp_ctx* ctx, const mebp_model_weights* model, const mebp_lo
                    const int32_t* ids, int batch, int seq, float* loss,
                    const mebp_lora_grads* grads, int accumulate, void* stream);
 
+/* ---- optimizer step (Section 4: every model is trained with AdamW; Section 3 keeps only the LoRA
+ * weights, their gradients and the optimizer states, and accumulates gradients over the samples
+ * of a batch).  AdamW = Adam with decoupled weight decay; at step t >= 1, per element:
+ *   g = grad_scale * grad;  m = b1 m + (1-b1) g;  v = b2 v + (1-b2) g^2;
+ *   p = p - lr * ( (m / (1 - b1^t)) / (sqrt(v / (1 - b2^t)) + eps) + weight_decay * p ).
+ * grad_scale = 1/n turns a gradient summed over n micro-batches (mebp_lora_step with
+ * accumulate = 1) into their mean. */
+typedef struct {
+  float lr, beta1, beta2, eps, weight_decay;
+  float grad_scale;
+} mebp_adamw_cfg;
+
+/* One AdamW update, in place, of n fp32 parameters held in one flat device buffer (the LoRA
+ * masters of every layer back to back), with their gradients and moment buffers m, v (same
+ * length; zero before step 1).  All four pointers 16-byte aligned; params, m, v are read and
+ * written, grads only read; none may overlap another.  step >= 1 is the (host) step count t.
+ * MEBP_ERR_INVALID_ARG for NULL or misaligned pointers, n < 0, step < 1 or bad hyper-parameters;
+ * n = 0 is a no-op. */
+int mebp_adamw_step(mebp_ctx* ctx, float* params, const float* grads, float* m, float* v, int64_t n,
+                    const mebp_adamw_cfg* cfg, int64_t step, void* stream);
+
 /* ---- instrumentation (Section 4 reports per-layer time; here: device time of the fused GEMMs).
  * mebp_kernel_launches: process-wide number of kernel launches the library has issued.
  * mebp_profile_begin: from now on record a CUDA-event pair on the launching stream around every

@@ -163,6 +163,8 @@ void launch_lora_shadow(const float* const* A, const float* const* B, int nt, co
 void launch_attn_fwd(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, int hd, uint16_t* o, int64_t ldo,
                      float* lse, cudaStream_t st);
 // part: fp32 scratch (>= 2 * B*S * H * hd floats for the per-head dK/dV mode), may be null.
+void launch_adamw(float* p, const float* g, float* m, float* v, int64_t n, float lr, float b1, float b2, float eps,
+                  float wd, float gs, double bc1, double bc2, cudaStream_t st);
 void launch_attn_bwd(const uint16_t* qkv, int64_t ld, const uint16_t* o, const uint16_t* dout, int64_t ldo,
                      const float* lse, int B, int S, int H, int KV, int hd, float* dvec, uint16_t* dqkv,
                      cudaStream_t st);

@@ -1091,6 +1091,25 @@ static int lora_step_body(mebp_ctx* c, const mebp_model_weights* model, const me
   return cuda_check(c, "lora step");
 }
 
+int mebp_adamw_step(mebp_ctx* c, float* params, const float* grads, float* m, float* v, int64_t n,
+                    const mebp_adamw_cfg* cfg, int64_t step, void* stream) {
+  if (!c) return MEBP_ERR_INVALID_ARG;
+  if (!cfg || n < 0 || step < 1) return fail(c, MEBP_ERR_INVALID_ARG, "bad AdamW arguments");
+  if (n == 0) return MEBP_OK;
+  if (!params || !grads || !m || !v) return fail(c, MEBP_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(params) || !aligned16(grads) || !aligned16(m) || !aligned16(v))
+    return fail(c, MEBP_ERR_INVALID_ARG, "AdamW buffers must be 16-byte aligned");
+  if (!(cfg->lr >= 0.0f) || !(cfg->beta1 >= 0.0f && cfg->beta1 < 1.0f) || !(cfg->beta2 >= 0.0f && cfg->beta2 < 1.0f) ||
+      !(cfg->eps > 0.0f) || !(cfg->weight_decay >= 0.0f))
+    return fail(c, MEBP_ERR_INVALID_ARG, "bad AdamW hyper-parameters");
+  const double bc1 = 1.0 / (1.0 - std::pow(static_cast<double>(cfg->beta1), static_cast<double>(step)));
+  const double bc2 = 1.0 / (1.0 - std::pow(static_cast<double>(cfg->beta2), static_cast<double>(step)));
+  pdl_entry();
+  launch_adamw(params, grads, m, v, n, cfg->lr, cfg->beta1, cfg->beta2, cfg->eps, cfg->weight_decay, cfg->grad_scale,
+               bc1, bc2, S(stream));
+  return cuda_check(c, "AdamW");
+}
+
 int mebp_lora_step(mebp_ctx* c, const mebp_model_weights* model, const mebp_lora* lora, const int32_t* ids, int B,
                    int Sq, float* loss, const mebp_lora_grads* grads, int accumulate, void* stream) {
   if (!c) return MEBP_ERR_INVALID_ARG;

@@ -61,6 +61,11 @@ class Profile(ctypes.Structure):
                 ("dx_ms", ctypes.c_double), ("dx_flops", ctypes.c_double)]
 
 
+class AdamWCfg(ctypes.Structure):
+    _fields_ = [("lr", c_float), ("beta1", c_float), ("beta2", c_float), ("eps", c_float),
+                ("weight_decay", c_float), ("grad_scale", c_float)]
+
+
 class ModelWeights(ctypes.Structure):
     _fields_ = [("embed", Packed), ("final_norm", c_void_p), ("blocks", POINTER(BlockWeights))]
 
@@ -92,6 +97,8 @@ _SIGS = {
     "mebp_profile_end": (c_int, [c_void_p, POINTER(Profile)]),
     "mebp_lora_step": (c_int, [c_void_p, POINTER(ModelWeights), POINTER(Lora), c_void_p, c_int, c_int, c_void_p,
                                POINTER(LoraGrads), c_int, c_void_p]),
+    "mebp_adamw_step": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_int64, POINTER(AdamWCfg), c_int64,
+                                c_void_p]),
 }
 
 
@@ -252,6 +259,16 @@ def mebp_lora_step(ctx, model: ModelWeights, lora_array, ids, loss, grads_array,
     B, S = ids.shape
     _check(ctx, _lib.mebp_lora_step(ctx, ctypes.byref(model), lora_array, _ptr(ids), B, S, _ptr(loss), grads_array,
                                     int(accumulate), _stream(stream)))
+
+
+def adamw_cfg(lr=1e-3, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.01, grad_scale=1.0) -> AdamWCfg:
+    return AdamWCfg(lr, beta1, beta2, eps, weight_decay, grad_scale)
+
+
+def mebp_adamw_step(ctx, params, grads, m, v, cfg: AdamWCfg, step: int, stream=None):
+    """In-place AdamW update of flat fp32 buffers (params, m, v written; grads read)."""
+    _check(ctx, _lib.mebp_adamw_step(ctx, _ptr(params), _ptr(grads), _ptr(m), _ptr(v), params.numel(),
+                                     ctypes.byref(cfg), int(step), _stream(stream)))
 
 
 def mebp_kernel_launches() -> int:

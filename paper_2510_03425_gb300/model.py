@@ -90,13 +90,52 @@ def to_device(x, device="cuda") -> torch.Tensor:
 
 
 class LoraSet:
-    """LoRA masters and gradients of every layer: lora[l][name] = (A [r, K], B [N, r])."""
+    """LoRA masters and gradients of every layer: lora[l][name] = (A [r, K], B [N, r]).
+
+    All masters live in one flat fp32 buffer and all gradients in another (each tensor a view,
+    16-byte aligned), so the optimizer updates every LoRA weight in one pass."""
 
     def __init__(self, layers: List[Dict[str, Tuple]], device="cuda"):
-        self.lora = [{n: (to_device(A, device), to_device(B, device)) for n, (A, B) in L.items()} for L in layers]
-        self.grads = [{n: (torch.zeros_like(A), torch.zeros_like(B)) for n, (A, B) in L.items()} for L in self.lora]
+        import numpy as np
+        sizes = []
+        for L in layers:
+            for n, (A, B) in L.items():
+                sizes += [int(np.prod(A.shape)), int(np.prod(B.shape))]
+        offs, n = [], 0
+        for sz in sizes:
+            offs.append(n)
+            n += (sz + 3) // 4 * 4
+        self.n = n
+        self.params = torch.zeros(n, dtype=torch.float32, device=device)
+        self.grad_flat = torch.zeros(n, dtype=torch.float32, device=device)
+        self.lora, self.grads, k = [], [], 0
+        for L in layers:
+            lw, lg = {}, {}
+            for name, (A, B) in L.items():
+                views = []
+                for src in (A, B):
+                    sz, o = int(np.prod(src.shape)), offs[k]
+                    p = self.params[o:o + sz].view(*src.shape)
+                    p.copy_(to_device(src, device))
+                    views.append((p, self.grad_flat[o:o + sz].view(*src.shape)))
+                    k += 1
+                lw[name] = (views[0][0], views[1][0])
+                lg[name] = (views[0][1], views[1][1])
+            self.lora.append(lw)
+            self.grads.append(lg)
         self._la = (M.Lora * len(self.lora))(*[M.lora_struct(L) for L in self.lora])
         self._ga = (M.LoraGrads * len(self.grads))(*[M.grads_struct(G) for G in self.grads])
+        self.m = self.v = None
+        self.t = 0
+
+    def adamw(self, ctx, cfg=None, stream=None):
+        """One AdamW update of every LoRA weight from the current gradients (mebp_adamw_step)."""
+        if self.m is None:
+            self.m = torch.zeros_like(self.params)
+            self.v = torch.zeros_like(self.params)
+        self.t += 1
+        M.mebp_adamw_step(ctx.handle, self.params, self.grad_flat, self.m, self.v, cfg or M.adamw_cfg(), self.t,
+                          stream)
 
     def lora_array(self):
         return self._la
