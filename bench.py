@@ -314,6 +314,105 @@ def adamw_bench(config: int = 4, reps: int = 20, warmup: int = 3):
             "frac": gbs / pk["hbm_gbs"], "peak_source": f"{src} copy bandwidth"}
 
 
+def _time_ms(f, reps: int, warmup: int = 3) -> float:
+    import torch
+    for _ in range(warmup):
+        f()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        f()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / reps
+
+
+def table2(reps: int = 10):
+    """Analogues of the paper's Table 2 (share of each pass spent on weight decompression) and
+    Table 3 (sequence-length sweep) on GB300.
+
+    Per projection GEMM of a workload: t_fused (this library: decode inside the GEMM mainloop),
+    t_dense (cuBLAS fp16 GEMM on weights decoded beforehand: a dense model with no compression)
+    and t_decode (the standalone decode of the whole matrix: the paper's decompress-then-compute
+    design pays t_decode + t_dense).  Reported per pass: the fused path's overhead over the dense
+    GEMM, (t_fused - t_dense) / t_fused, and the decompression share of decompress-then-compute,
+    t_decode / (t_decode + t_dense) -- the quantity Table 2 reports for the iPhone."""
+    import torch
+
+    from paper_2510_03425_gb300 import mebp as M
+    from paper_2510_03425_gb300.model import Context, LoraSet, compress
+    torch.backends.cuda.matmul.allow_fp16_reduced_precision_reduction = False
+    out = {"decompression": {}, "seq_sweep": {}}
+    ctx = Context(synth.tiny(vocab=0, head_dim=64), max_tokens=64, max_seq=64)
+    g = torch.Generator(device="cuda")
+    g.manual_seed(5)
+    for cfg_i in (1, 4):
+        d = synth.preset(cfg_i)
+        Mr = d.tokens
+        shapes = synth.linear_shapes(d)
+        mats = {"qkv": (shapes["q"][0] + 2 * shapes["k"][0], d.hidden), "o": shapes["o"],
+                "gate_up": (2 * d.intermediate, d.hidden), "down": shapes["down"]}
+        rows, tot = {}, {"fused_fwd": 0.0, "dense_fwd": 0.0, "fused_dx": 0.0, "dense_dx": 0.0, "decode": 0.0}
+        for name, (N, K) in mats.items():
+            W = torch.randn(N, K, device="cuda", generator=g) * 0.02
+            q, sc = compress(ctx, W)
+            del W
+            Wp = M.packed(q, sc)
+            Wd = torch.empty((N, K), dtype=torch.int16, device="cuda")
+            X = torch.randn(Mr, K, device="cuda", generator=g).half()
+            dY = torch.randn(Mr, N, device="cuda", generator=g).half()
+            Y = torch.empty(Mr, N, device="cuda", dtype=torch.float16)
+            dX = torch.empty(Mr, K, device="cuda")
+            t_dec = _time_ms(lambda: M.mebp_decode_weights(ctx.handle, Wp, Wd), reps)
+            Wh = Wd.view(torch.float16)
+            t_ff = _time_ms(lambda: M.mebp_linear_fwd(ctx.handle, X, Wp, y_f16=Y), reps)
+            t_fd = _time_ms(lambda: M.mebp_linear_dx(ctx.handle, dY, Wp, dx=dX), reps)
+            t_df = _time_ms(lambda: torch.matmul(X, Wh.t(), out=Y), reps)
+            dXh = torch.empty(Mr, K, device="cuda", dtype=torch.float16)
+            t_dd = _time_ms(lambda: torch.matmul(dY, Wh, out=dXh), reps)
+            rows[name] = {"N": N, "K": K, "fused_fwd_us": 1e3 * t_ff, "dense_fwd_us": 1e3 * t_df,
+                          "fused_dx_us": 1e3 * t_fd, "dense_dx_us": 1e3 * t_dd, "decode_us": 1e3 * t_dec}
+            for k, v in (("fused_fwd", t_ff), ("dense_fwd", t_df), ("fused_dx", t_fd), ("dense_dx", t_dd),
+                         ("decode", t_dec)):
+                tot[k] += v
+            del q, sc, Wp, Wd, X, dY, Y, dX, dXh
+        out["decompression"][d.name] = {
+            "M": Mr, "per_gemm": rows,
+            "fused_over_dense_fwd": (tot["fused_fwd"] - tot["dense_fwd"]) / tot["fused_fwd"],
+            "fused_over_dense_dx": (tot["fused_dx"] - tot["dense_dx"]) / tot["fused_dx"],
+            "decode_share_separate_fwd": tot["decode"] / (tot["decode"] + tot["dense_fwd"]),
+            "decode_share_separate_dx": tot["decode"] / (tot["decode"] + tot["dense_dx"]),
+        }
+        torch.cuda.empty_cache()
+    ctx.close()
+    # Table 3 analogue: Qwen2.5-1.5B shape, batch 1, the paper's sequence lengths
+    base = synth.preset(3).with_(batch=1, spill=False)
+    for S in (128, 256, 512, 1024):
+        d = base.with_(seq=S)
+        c2 = Context(d)
+        model = build_model(c2, d, torch.device("cuda"))
+        ls = LoraSet([synth.lora_weights(d, i) for i in range(d.n_layers)])
+        ids = torch.from_numpy(synth.token_ids(d)).cuda()
+        loss = torch.zeros(1, device="cuda")
+        st = torch.cuda.Stream()
+        ms = model.struct()
+
+        def step():
+            M.mebp_lora_step(c2.handle, ms, ls.lora_array(), ids, loss, ls.grads_array(), False, st)
+        with torch.cuda.stream(st):
+            t = _time_ms(step, reps)
+        wb = sum(b.qkv.qpack.numel() + b.o.qpack.numel() + b.gate_up.qpack.numel() + b.down.qpack.numel()
+                 for b in model.blocks) * (1 + 1 / 16) + model.embed.qpack.numel() * (1 + 1 / 16)
+        out["seq_sweep"][S] = {"ms_per_step": t, "tokens_per_s": S / (t / 1e3),
+                               "workspace_mb": M.mebp_workspace_bytes(c2.handle) / 2**20,
+                               "packed_weights_mb": wb / 2**20, "lora_and_grads_mb": 2 * 4 * ls.n / 2**20}
+        c2.close()
+        del model, ls
+        torch.cuda.empty_cache()
+    return out
+
+
 def launch_list_step(args, d):
     """Warm-up steps, then one step run eagerly (no graph replay) inside an NVTX range, so a
     profiler can list exactly the kernels of one step."""
@@ -414,6 +513,8 @@ def main():
                     help="time only the fused dequant-GEMMs at the config's projection shapes")
     ap.add_argument("--gemm-m", type=int, default=None, help="token count M for --gemm-bench")
     ap.add_argument("--gemm-shapes", default=None, help="comma list of qkv,o,gate_up,down for --gemm-bench")
+    ap.add_argument("--table2", action="store_true",
+                    help="decompression-overhead (Table 2) and sequence-length (Table 3) analogues")
     ap.add_argument("--launch-list", action="store_true",
                     help="no timing: after the warm-up run one eager step inside the NVTX range "
                          "'mebp_step' (for ncu --nvtx --nvtx-include mebp_step/)")
@@ -432,6 +533,9 @@ def main():
 
     if args.launch_list:
         launch_list_step(args, d)
+        return
+    if args.table2:
+        print(json.dumps(table2()), flush=True)
         return
 
     if args.impl == "reference":
