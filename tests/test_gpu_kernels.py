@@ -121,8 +121,9 @@ def test_linear_dx_matches_exact_operand_product(ctx, Mr, N, K):
     assert np.abs(np_of(dx) - ref).max() <= 2e-5 * np.abs(ref).max() + 1e-6
 
 
-@pytest.mark.parametrize("r", [8, 16, 32])
-@pytest.mark.parametrize("Mr,N,K", [(200, 320, 192), (300, 1152, 896), (2304 + 77, 576, 640)])
+@pytest.mark.parametrize("r,Mr,N,K", [(r, *shape) for r in (8, 16, 32)
+                                      for shape in ((200, 320, 192), (300, 1152, 896), (2304 + 77, 576, 640))]
+                         + [(16, 4096 + 77, 1152, 1536)])  # > 152 tiles: persistent CTAs run several
 def test_linear_with_lora_against_oracle(ctx, r, Mr, N, K):
     """Y = X deq(W)^T + s (X A^T) B^T (+R) and dX = dY deq(W) + s (dY B) A against fp64."""
     s = 2.0
