@@ -460,17 +460,26 @@ __global__ void __launch_bounds__(Warps<NACC>::THREADS, 1)
         if (!mbar_wait(&afull[s], (it / TSTG) & 1, abort_flag, p.err)) break;
         if (!mbar_wait(&bfull[b], (it / BSTG) & 1, abort_flag, p.err)) break;
         tc_fence_after();
-        const uint32_t a_base = smem_u32(smem + s * Ly::T_STRIDE + Ly::A_OFF);
-        const uint32_t b_base = smem_u32(smem + Ly::B_BASE + b * B_BYTES);
-        const int nk = (it < num_main) ? 4 : min(4, p.kx_steps - 4 * (it - num_main));
-        for (int kk = 0; kk < nk; ++kk) {
-          const uint64_t bd = TRANS ? smem_desc_sw128(b_base + kk * 2048, 8192, 1024)
-                                    : smem_desc_sw128(b_base + kk * 32, 16, 1024);
+        // Descriptors of the stage's first k16 slice; later slices advance the start-address field
+        // (bits 0-13, in 16-byte units) by a constant, so the issue loop is adds and MMAs only.
+        const uint64_t ad0 = smem_desc_sw128(smem_u32(smem + s * Ly::T_STRIDE + Ly::A_OFF), 16, 1024);
+        const uint64_t bd0 = TRANS ? smem_desc_sw128(smem_u32(smem + Ly::B_BASE + b * B_BYTES), 8192, 1024)
+                                   : smem_desc_sw128(smem_u32(smem + Ly::B_BASE + b * B_BYTES), 16, 1024);
+        constexpr uint64_t A_K16 = 32 >> 4, A_ACC = A_BYTES >> 4, B_K16 = (TRANS ? 2048 : 32) >> 4;
+        if (it < num_main) {
 #pragma unroll
-          for (int a = 0; a < NACC; ++a) {
-            const uint64_t ad = smem_desc_sw128(a_base + a * A_BYTES + kk * 32, 16, 1024);
-            tc_mma_f16(tmem + 256 * a, ad, bd, idesc, (it > 0 || kk > 0) ? 1u : 0u);
-          }
+          for (int kk = 0; kk < 4; ++kk)
+#pragma unroll
+            for (int a = 0; a < NACC; ++a)
+              tc_mma_f16(tmem + 256 * a, ad0 + a * A_ACC + kk * A_K16, bd0 + kk * B_K16, idesc,
+                         (it > 0 || kk > 0) ? 1u : 0u);
+        } else {
+          const int nk = min(4, p.kx_steps - 4 * (it - num_main));
+          for (int kk = 0; kk < nk; ++kk)
+#pragma unroll
+            for (int a = 0; a < NACC; ++a)
+              tc_mma_f16(tmem + 256 * a, ad0 + a * A_ACC + kk * A_K16, bd0 + kk * B_K16, idesc,
+                         (it > 0 || kk > 0) ? 1u : 0u);
         }
         tc_commit(&empty[s]);
         tc_commit(&bempty[b]);
@@ -637,6 +646,11 @@ int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st) {
   const int64_t tiles_n256 = (g.N + BN - 1) / BN;
   const int nacc = (g.M >= 2048 || (g.M >= 256 && tiles_n256 * ((g.M + 255) / 256) >= 2 * 152)) ? 2 : 1;
   const int bm = BM * nacc;
+  // Few tokens and a short K: 128 x 256 tiles would leave most SMs idle; narrow 128 x 64 tiles
+  // instead of a K split (a long K keeps the split: its serial chain would dominate).
+  if (nacc == 1 && (g.epi == EPI_F32 || g.epi == EPI_F16) && g.K <= 2560 &&
+      ((g.N + BN - 1) / BN) * ((g.M + BM - 1) / BM) <= 76)
+    return launch_dequant_gemm_narrow(g, st);
 
   CUtensorMap tA, tP, tS, tAx;
   int rc;

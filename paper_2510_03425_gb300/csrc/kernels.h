@@ -102,6 +102,12 @@ struct GemmArgs {
 };
 
 int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st);
+// The 128 x 64-tile variant for few-token GEMMs (EPI_F16 / EPI_F32); launch_dequant_gemm routes
+// to it when the 128 x 256 tiles would leave most SMs idle.
+int launch_dequant_gemm_narrow(const GemmArgs& g, cudaStream_t st);
+// 2-D tiled TMA descriptor: dims {d0 (inner), d1}, row pitch in bytes, box {b0, b1}.
+int make_tmap_2d(CUtensorMap* m, const void* base, CUtensorMapDataType dt, int elem_bytes, uint64_t d0, uint64_t d1,
+                 uint64_t pitch_bytes, uint32_t b0, uint32_t b1, CUtensorMapSwizzle swz);
 int gemm_smem_bytes();
 
 void launch_compress(const float* W, int64_t rows, int64_t cols, uint8_t* qpack, uint16_t* scales, cudaStream_t st);
