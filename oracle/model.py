@@ -25,6 +25,13 @@ grouped-query attention -> o projection (+LoRA) + residual -> RMSNorm ->
 act(gate) * up (+LoRA) -> down projection (+LoRA) + residual, with
 act = SiLU (Qwen) or tanh-approximated GELU (Gemma).  No biases, eps = 1e-6,
 RoPE theta = 1e6, LoRA ``Y = X W^T + s (X A^T) B^T`` with ``s = alpha / r``.
+
+With ``dims.gemma_norms`` the block follows the Gemma3 architecture of the paper's Gemma models:
+per-head RMSNorm of q and k (gains q_norm, k_norm) before RoPE, RMSNorm of the attention output
+and of the MLP output before each residual add (gains post_attn_norm, post_ffn_norm; the
+pre-norms stay norm1 / norm2), and input embeddings scaled by sqrt(D).  With
+``dims.sliding_window = W > 0`` every layer except each ``global_every``-th is local: position i
+attends to j with 0 <= i - j < W, and its RoPE base is ``rope_theta_local``.
 """
 from __future__ import annotations
 
@@ -36,6 +43,7 @@ import numpy as np
 from . import quant
 
 LINEARS = ("q", "k", "v", "o", "gate", "up", "down")
+NORMS = ("norm1", "norm2", "q_norm", "k_norm", "post_attn_norm", "post_ffn_norm")
 
 
 # ----------------------------------------------------------------------------- basic ops
@@ -99,11 +107,12 @@ def rope(x: np.ndarray, ang: np.ndarray, inverse: bool = False) -> np.ndarray:
     return np.concatenate([x1 * c - x2 * s, x2 * c + x1 * s], axis=-1)
 
 
-def attention(q, k, v, batch: int, seq: int):
+def attention(q, k, v, batch: int, seq: int, window: int = 0):
     """Causal grouped-query attention.  q [T, H, hd], k/v [T, KV, hd], T = batch*seq.
 
     Query head h reads key/value head h // (H/KV); scores are scaled by 1/sqrt(hd)
-    and position i attends to positions j <= i of its own sequence.
+    and position i attends to positions j <= i of its own sequence (and, with a
+    sliding window W > 0, only to i - j < W).
     Returns o [T, H, hd], lse [batch, H, seq], P (list per (b, h)) for the VJP.
     """
     T, H, hd = q.shape
@@ -111,6 +120,8 @@ def attention(q, k, v, batch: int, seq: int):
     grp = H // KV
     scale = 1.0 / math.sqrt(hd)
     causal = np.tril(np.ones((seq, seq), dtype=bool))
+    if window > 0:
+        causal &= np.triu(np.ones((seq, seq), dtype=bool), -(window - 1))
     o = np.zeros_like(q)
     lse = np.zeros((batch, H, seq))
     probs = {}
@@ -182,38 +193,60 @@ def linear_vjp(dY, X, U, W, lora, s: float, need_dx: bool = True):
 
 # ----------------------------------------------------------------------------- the block
 
-def block_forward(x, W: Dict[str, np.ndarray], lora: Dict[str, Tuple], dims, save: bool = False):
+def block_forward(x, W: Dict[str, np.ndarray], lora: Dict[str, Tuple], dims, save: bool = False, layer: int = 0):
     """One pre-norm decoder block y = F(x, w).  x [T, D] float64; W holds dense
-    (already decompressed) matrices W[name] [N_out, K_in] and norm gains.
+    (already decompressed) matrices W[name] [N_out, K_in] and norm gains.  ``layer``
+    selects local or global attention when dims.sliding_window > 0.
     Returns y, and the saved intermediates when ``save``."""
     D, H, KV, hd = dims.hidden, dims.n_heads, dims.n_kv_heads, dims.head_dim
     T = x.shape[0]
     s = dims.lora_scale
     act, _ = ACT[dims.act]
-    pos_ang = rope_angles(dims.seq, hd, dims.rope_theta)[np.arange(T) % dims.seq]
+    gemma = getattr(dims, "gemma_norms", False)
+    local = dims.layer_is_local(layer) if hasattr(dims, "layer_is_local") else False
+    theta = dims.rope_theta_local if local else dims.rope_theta
+    window = dims.sliding_window if local else 0
+    pos_ang = rope_angles(dims.seq, hd, theta)[np.arange(T) % dims.seq]
 
     a, r1 = rmsnorm(x, W["norm1"], dims.eps)
     q, Uq = linear(a, W["q"], lora.get("q"), s)
     k, Uk = linear(a, W["k"], lora.get("k"), s)
     v, Uv = linear(a, W["v"], lora.get("v"), s)
-    q = rope(q.reshape(T, H, hd), pos_ang)
-    k = rope(k.reshape(T, KV, hd), pos_ang)
+    q_raw, k_raw = q.reshape(T, H, hd), k.reshape(T, KV, hd)
+    rq = rk = None
+    if gemma:  # QK-norm: per-head RMSNorm before the rotation
+        qn, rq = rmsnorm(q_raw, W["q_norm"], dims.eps)
+        kn, rk = rmsnorm(k_raw, W["k_norm"], dims.eps)
+    else:
+        qn, kn = q_raw, k_raw
+    q = rope(qn, pos_ang)
+    k = rope(kn, pos_ang)
     v = v.reshape(T, KV, hd)
-    o, lse, probs = attention(q, k, v, dims.batch, dims.seq)
+    o, lse, probs = attention(q, k, v, dims.batch, dims.seq, window)
     o2 = o.reshape(T, H * hd)
     ao, Uo = linear(o2, W["o"], lora.get("o"), s)
-    h1 = x + ao
+    rpa = None
+    if gemma:  # sandwich norm on the attention output
+        aon, rpa = rmsnorm(ao, W["post_attn_norm"], dims.eps)
+    else:
+        aon = ao
+    h1 = x + aon
     b, r2 = rmsnorm(h1, W["norm2"], dims.eps)
     g, Ug = linear(b, W["gate"], lora.get("gate"), s)
     u, Uu = linear(b, W["up"], lora.get("up"), s)
     m = act(g) * u
     dn, Ud = linear(m, W["down"], lora.get("down"), s)
-    y = h1 + dn
+    rpf = None
+    if gemma:  # sandwich norm on the MLP output
+        dnn, rpf = rmsnorm(dn, W["post_ffn_norm"], dims.eps)
+    else:
+        dnn = dn
+    y = h1 + dnn
     if not save:
         return y, None
     cache = dict(x=x, a=a, r1=r1, q=q, k=k, v=v, o=o, lse=lse, probs=probs, o2=o2, h1=h1,
                  b=b, r2=r2, g=g, u=u, m=m, U=dict(q=Uq, k=Uk, v=Uv, o=Uo, gate=Ug, up=Uu, down=Ud),
-                 ang=pos_ang)
+                 ang=pos_ang, gemma=gemma, q_raw=q_raw, k_raw=k_raw, rq=rq, rk=rk, ao=ao, rpa=rpa, dn=dn, rpf=rpf)
     return y, cache
 
 
@@ -233,19 +266,26 @@ def block_backward(dy, cache, W, lora, dims, need_dx: bool = True):
             grads[name] = gr
         return dX
 
-    # y = h1 + down(m)
-    dm = lin_bwd("down", dy, c["m"])
+    # y = h1 + [norm_pf](down(m))
+    ddn = rmsnorm_vjp(dy, c["dn"], W["post_ffn_norm"], c["rpf"]) if c["gemma"] else dy
+    dm = lin_bwd("down", ddn, c["m"])
     ag = act(c["g"])
     dg = dm * c["u"] * act_grad(c["g"])
     du = dm * ag
     db = lin_bwd("gate", dg, c["b"]) + lin_bwd("up", du, c["b"])
     dh1 = dy + rmsnorm_vjp(db, c["h1"], W["norm2"], c["r2"])
-    # h1 = x + o_proj(attn)
-    do2 = lin_bwd("o", dh1, c["o2"])
+    # h1 = x + [norm_pa](o_proj(attn))
+    dao = rmsnorm_vjp(dh1, c["ao"], W["post_attn_norm"], c["rpa"]) if c["gemma"] else dh1
+    do2 = lin_bwd("o", dao, c["o2"])
     dq, dk, dv = attention_vjp(do2.reshape(T, H, hd), c["q"], c["k"], c["v"], c["probs"],
                                dims.batch, dims.seq)
-    dq = rope(dq, c["ang"], inverse=True).reshape(T, H * hd)
-    dk = rope(dk, c["ang"], inverse=True).reshape(T, KV * hd)
+    dq = rope(dq, c["ang"], inverse=True)
+    dk = rope(dk, c["ang"], inverse=True)
+    if c["gemma"]:
+        dq = rmsnorm_vjp(dq, c["q_raw"], W["q_norm"], c["rq"])
+        dk = rmsnorm_vjp(dk, c["k_raw"], W["k_norm"], c["rk"])
+    dq = dq.reshape(T, H * hd)
+    dk = dk.reshape(T, KV * hd)
     dv = dv.reshape(T, KV * hd)
     da_q = lin_bwd("q", dq, c["a"], need_dx)
     da_k = lin_bwd("k", dk, c["a"], need_dx)
@@ -257,12 +297,12 @@ def block_backward(dy, cache, W, lora, dims, need_dx: bool = True):
     return dx, grads
 
 
-def block_objective(x, W, lora, G, dims):
+def block_objective(x, W, lora, G, dims, layer: int = 0):
     """Single-block objective E = sum(G * y) (the scalar of Section 3 with dE/dy = G).
     Returns E, dE/dx and the LoRA gradients, through one checkpointed recompute + backward."""
-    y, _ = block_forward(x, W, lora, dims)                 # forward pass: only the output is kept
+    y, _ = block_forward(x, W, lora, dims, layer=layer)                 # forward pass: only the output is kept
     E = float(np.sum(G * y))
-    _, cache = block_forward(x, W, lora, dims, save=True)  # recompute from the stored input
+    _, cache = block_forward(x, W, lora, dims, save=True, layer=layer)  # recompute from the stored input
     dx, grads = block_backward(G, cache, W, lora, dims)
     return E, dx, grads
 
@@ -331,8 +371,9 @@ class PackedModel:
         blocks = []
         for Wb in dense_blocks:
             pb = {n: quant.compress(Wb[n]) for n in LINEARS}
-            pb["norm1"] = np.asarray(Wb["norm1"], np.float64)
-            pb["norm2"] = np.asarray(Wb["norm2"], np.float64)
+            for nm in NORMS:
+                if nm in Wb:
+                    pb[nm] = np.asarray(Wb[nm], np.float64)
             blocks.append(pb)
         embed = quant.compress(E) if E is not None else None
         return cls(blocks, embed, None if g_f is None else np.asarray(g_f, np.float64))
@@ -341,13 +382,19 @@ class PackedModel:
         """LazyLoadAndDecompressWeights(i): dense float64 matrices of block i."""
         pb = self.blocks[i]
         W = {n: quant.dequant(*pb[n]) for n in LINEARS}
-        W["norm1"], W["norm2"] = pb["norm1"], pb["norm2"]
+        for nm in NORMS:
+            if nm in pb:
+                W[nm] = pb[nm]
         return W
 
 
-def embed_tokens(model: PackedModel, ids: np.ndarray) -> np.ndarray:
-    """x0[t] = deq(E)[id_t] (the embedding is compressed like every base matrix)."""
-    return quant.dequant_rows(*model.embed, ids.reshape(-1))
+def embed_tokens(model: PackedModel, ids: np.ndarray, dims=None) -> np.ndarray:
+    """x0[t] = deq(E)[id_t] (the embedding is compressed like every base matrix), times sqrt(D)
+    for the Gemma3 block."""
+    x0 = quant.dequant_rows(*model.embed, ids.reshape(-1))
+    if dims is not None and getattr(dims, "gemma_norms", False):
+        x0 = x0 * math.sqrt(dims.hidden)
+    return x0
 
 
 def lora64(lora_layer):
@@ -365,10 +412,10 @@ def mebp_backpropagation(model: PackedModel, lora: List[Dict], ids: np.ndarray, 
     """
     n = len(model.blocks)
     targets = next_token_targets(ids)
-    ckpts = {0: embed_tokens(model, ids)}                 # ckpts_storage <- {x}
+    ckpts = {0: embed_tokens(model, ids, dims)}           # ckpts_storage <- {x}
     for i in range(1, n + 1):                             # forward loop, checkpoints only
         W = model.decompress_block(i - 1)
-        ckpts[i], _ = block_forward(ckpts[i - 1], W, lora64(lora[i - 1]), dims)
+        ckpts[i], _ = block_forward(ckpts[i - 1], W, lora64(lora[i - 1]), dims, layer=i - 1)
     E_deq = quant.dequant(*model.embed)                   # final linear layer (tied embedding)
     loss, g, tok = lm_head_ce(ckpts[n], model.final_norm, E_deq, targets, dims.eps, want_token_loss=True)
     del E_deq
@@ -378,7 +425,7 @@ def mebp_backpropagation(model: PackedModel, lora: List[Dict], ids: np.ndarray, 
     for i in range(n, 0, -1):                             # backward loop, reverse order
         W = model.decompress_block(i - 1)
         lw = lora64(lora[i - 1])
-        _, cache = block_forward(ckpts[i - 1], W, lw, dims, save=True)   # recompute block i
+        _, cache = block_forward(ckpts[i - 1], W, lw, dims, save=True, layer=i - 1)   # recompute block i
         if want_trace:
             trace["dys"][i] = g.copy()
         g, grads[i - 1] = block_backward(g, cache, W, lw, dims, need_dx=(i > 1))
@@ -393,11 +440,11 @@ def full_backpropagation(model: PackedModel, lora: List[Dict], ids: np.ndarray, 
     of every block, then the backward from those stored intermediates."""
     n = len(model.blocks)
     targets = next_token_targets(ids)
-    x = embed_tokens(model, ids)
+    x = embed_tokens(model, ids, dims)
     caches, Ws = [], []
     for i in range(n):
         W = model.decompress_block(i)
-        x, cache = block_forward(x, W, lora64(lora[i]), dims, save=True)
+        x, cache = block_forward(x, W, lora64(lora[i]), dims, save=True, layer=i)
         caches.append(cache)
         Ws.append(W)
     E_deq = quant.dequant(*model.embed)

@@ -44,6 +44,16 @@ class ModelDims:
     rope_theta: float = 1e6
     eps: float = 1e-6
     spill: bool = False  # activation checkpoints in pinned host memory
+    # Gemma3 block fidelity (off for the benchmark presets): QK-norm, sandwich norms and the
+    # sqrt(D) embedding scale; sliding-window attention on local layers (window > 0), every
+    # global_every-th layer global, local layers with their own RoPE base.
+    gemma_norms: bool = False
+    sliding_window: int = 0
+    global_every: int = 6
+    rope_theta_local: float = 1e4
+
+    def layer_is_local(self, layer: int) -> bool:
+        return self.sliding_window > 0 and (layer + 1) % self.global_every != 0
 
     @property
     def tokens(self) -> int:
@@ -116,11 +126,18 @@ def block_weights(d: ModelDims, layer: int, seed: int = 0, norm_jitter: float = 
     out = {}
     for i, (name, shp) in enumerate(linear_shapes(d).items()):
         out[name] = _normal(seed, (layer, i), shp, std)
-    for j, name in enumerate(("norm1", "norm2")):
+    names = ("norm1", "norm2") + (("post_attn_norm", "post_ffn_norm") if d.gemma_norms else ())
+    for j, name in enumerate(names):
         g = np.ones(d.hidden, np.float32)
         if norm_jitter:
             g += _normal(seed, (layer, 100 + j), (d.hidden,), norm_jitter)
         out[name] = g
+    if d.gemma_norms:
+        for j, name in enumerate(("q_norm", "k_norm")):
+            g = np.ones(d.head_dim, np.float32)
+            if norm_jitter:
+                g += _normal(seed, (layer, 110 + j), (d.head_dim,), norm_jitter)
+            out[name] = g
     return out
 
 
@@ -178,8 +195,11 @@ def _torch_normal(shape, std, seed, key, device):
 def torch_block_weights(d: ModelDims, layer: int, seed: int = 0, device="cuda", std: float = 0.02):
     import torch
     out = {name: _torch_normal(shp, std, seed, (layer, i), device) for i, (name, shp) in enumerate(linear_shapes(d).items())}
-    out["norm1"] = torch.ones(d.hidden, device=device)
-    out["norm2"] = torch.ones(d.hidden, device=device)
+    for name in ("norm1", "norm2") + (("post_attn_norm", "post_ffn_norm") if d.gemma_norms else ()):
+        out[name] = torch.ones(d.hidden, device=device)
+    if d.gemma_norms:
+        out["q_norm"] = torch.ones(d.head_dim, device=device)
+        out["k_norm"] = torch.ones(d.head_dim, device=device)
     return out
 
 
