@@ -66,6 +66,17 @@ typedef struct {
   int32_t max_seq;       /* longest sequence (RoPE table size)                                  */
   int32_t spill_ckpts;   /* 1: mebp_lora_step keeps block checkpoints in pinned host memory     */
   int32_t vocab_chunk;   /* LM-head vocabulary chunk (multiple of 256); 0 = library default     */
+  /* Gemma3 block options (Section 4 fine-tunes Gemma3 models; all zero = the plain pre-norm block):
+   *  gemma_norms != 0: per-head RMSNorm of q and k (gains q_norm / k_norm, over head_dim) before
+   *    RoPE; RMSNorm of the attention output (post_attn_norm) and of the MLP output
+   *    (post_ffn_norm) before each residual add; input embeddings multiplied by sqrt(hidden).
+   *  sliding_window = W > 0: layer l is local iff (l + 1) % global_every != 0; a local layer's
+   *    query at position i attends to keys i - W + 1 .. i and rotates with base rope_theta_local
+   *    (global layers: causal, rope_theta).  global_every >= 1 when W > 0. */
+  int32_t gemma_norms;
+  int32_t sliding_window;
+  int32_t global_every;
+  float rope_theta_local;
 } mebp_model_cfg;
 
 /* ---- compressed base weight (Section 3, "Base model weights compression") -------------------
@@ -91,11 +102,17 @@ typedef struct {
  *   o       rows = D,  cols = H * hd
  *   gate_up rows = 2 I (gate rows, then up rows),                      cols = D
  *   down    rows = D,  cols = I
- * norm1 / norm2: fp32 [D] RMSNorm gains (before attention / before the MLP). */
+ * norm1 / norm2: fp32 [D] RMSNorm gains (before attention / before the MLP).
+ * With cfg.gemma_norms also (else ignored, may be NULL): q_norm / k_norm fp32 [hd], post_attn_norm
+ * / post_ffn_norm fp32 [D].  Every gain pointer 16-byte aligned. */
 typedef struct {
   mebp_packed qkv, o, gate_up, down;
   const float* norm1;
   const float* norm2;
+  const float* q_norm;
+  const float* k_norm;
+  const float* post_attn_norm;
+  const float* post_ffn_norm;
 } mebp_block_weights;
 
 /* LoRA masters of one block (fp32, device).  A[t] = [r, K_in], B[t] = [N_out, r];
@@ -145,7 +162,8 @@ int mebp_compress_weights(mebp_ctx* ctx, const float* W, int64_t rows, int64_t c
  * function that feeds the fused GEMM's shared-memory operand. */
 int mebp_decode_weights(mebp_ctx* ctx, const mebp_packed* w, uint16_t* out_f16, void* stream);
 
-/* Embedding gather + dequant: x0[t, :] = deq(E)[ids[t], :] (fp32 [n_tokens, D], exact).
+/* Embedding gather + dequant: x0[t, :] = deq(E)[ids[t], :] (fp32 [n_tokens, D], exact), times
+ * sqrt(D) with cfg.gemma_norms.
  * An id outside [0, V) writes zeros and sets MEBP_ERR_DEVICE. */
 int mebp_embed(mebp_ctx* ctx, const mebp_packed* embed, const int32_t* ids, int64_t n_tokens,
                float* x0, void* stream);

@@ -1,8 +1,10 @@
 // Causal grouped-query attention of the decoder block, forward and backward, as tiled
 // warp-level tensor-core kernels (mma.sync m16n8k16, fp16 in / fp32 accumulate).
 //
-//   forward : o = softmax(q k^T / sqrt(hd) + causal) v, per (sequence, query head); query head h
+//   forward : o = softmax(q k^T / sqrt(hd) + mask) v, per (sequence, query head); query head h
 //             reads key/value head h / (H/KV).  Saves lse = log-sum-exp of each score row.
+//             mask: query i sees key j iff j <= i and, with a sliding window W > 0 (the local
+//             layers of Gemma3), i - j < W; key blocks wholly outside the window are skipped.
 //   backward: dP = dO v^T, dS = P (dP - rowsum(dO o)), dq = dS k / sqrt(hd),
 //             dk = dS^T q / sqrt(hd), dv = P^T dO; dk, dv summed over the query heads of a
 //             group.  P is recomputed from q, k and lse.  One launch holds two kinds of work
@@ -81,7 +83,7 @@ __device__ __forceinline__ void pv_tile(float (&acc)[NC][4], const float (&p)[8]
 template <int HD, int NB>
 __global__ void __launch_bounds__(128, 1) fwd_kernel(const uint16_t* __restrict__ qkv, int64_t ld, int S, int H,
                                                      int KV, uint16_t* __restrict__ o, int64_t ldo,
-                                                     float* __restrict__ lse) {
+                                                     float* __restrict__ lse, int W) {
   griddep_wait();
   griddep_launch();
   constexpr int LD = HD + 8, NO = HD / 8;
@@ -96,10 +98,11 @@ __global__ void __launch_bounds__(128, 1) fwd_kernel(const uint16_t* __restrict_
   const int q0 = qb * BQ;
   const float sc = kLog2e * rsqrtf(static_cast<float>(HD));
 
+  const int kb0 = W > 0 ? max(0, q0 - W + 1) / BKV : 0;  // first key block inside the window
   load_tile<HD>(qs, qkv, ld, tok0, q0, S, h * HD, tid);
   if (NB == 2) {
-    load_tile<HD>(ks(0), qkv, ld, tok0, 0, S, (H + kvh) * HD, tid);
-    load_tile<HD>(vs(0), qkv, ld, tok0, 0, S, (H + KV + kvh) * HD, tid);
+    load_tile<HD>(ks(0), qkv, ld, tok0, kb0 * BKV, S, (H + kvh) * HD, tid);
+    load_tile<HD>(vs(0), qkv, ld, tok0, kb0 * BKV, S, (H + KV + kvh) * HD, tid);
   }
   cp_async_commit();
 
@@ -110,8 +113,8 @@ __global__ void __launch_bounds__(128, 1) fwd_kernel(const uint16_t* __restrict_
   const int ra = q0 + warp * 16 + (lane >> 2);
   const int nkb = min((q0 + BQ - 1) / BKV + 1, (S + BKV - 1) / BKV);
 
-  for (int kb = 0; kb < nkb; ++kb) {
-    const int k0 = kb * BKV, buf = NB == 2 ? kb & 1 : 0;
+  for (int kb = kb0; kb < nkb; ++kb) {
+    const int k0 = kb * BKV, buf = NB == 2 ? (kb - kb0) & 1 : 0;
     if (NB == 1) {
       load_tile<HD>(ks(0), qkv, ld, tok0, k0, S, (H + kvh) * HD, tid);
       load_tile<HD>(vs(0), qkv, ld, tok0, k0, S, (H + KV + kvh) * HD, tid);
@@ -135,7 +138,7 @@ __global__ void __launch_bounds__(128, 1) fwd_kernel(const uint16_t* __restrict_
       for (int e = 0; e < 4; ++e) {
         const int col = k0 + nt * 8 + 2 * (lane & 3) + (e & 1);
         const int row = ra + ((e >> 1) << 3);
-        s[nt][e] = (col > row || col >= S) ? -INFINITY : s[nt][e] * sc;
+        s[nt][e] = (col > row || col >= S || (W > 0 && row - col >= W)) ? -INFINITY : s[nt][e] * sc;
       }
 #pragma unroll
     for (int i = 0; i < 2; ++i) {
@@ -216,6 +219,7 @@ struct BwdArgs {
   const float* lse;
   const float* dvec;
   int S, H, KV, B;
+  int W;     // sliding window (0 = none)
   int n_kv;  // dK/dV work items (blocks [0, n_kv)); dQ items follow
   uint16_t* dqkv;
 };
@@ -259,7 +263,9 @@ __device__ __forceinline__ void dkdv_item(const BwdArgs& a, int idx, uint16_t* s
   }
   const int key_a = k0 + warp * 16 + (lane >> 2);
   const int nqb = (S + BQ - 1) / BQ;
-  const int per_head = nqb - kb;  // query blocks kb .. nqb-1 see this key block
+  // query blocks kb .. qb_end-1 see this key block (with a window, queries < k0 + BKV - 1 + W)
+  const int qb_end = a.W > 0 ? min(nqb, (k0 + BKV - 1 + a.W - 1) / BQ + 1) : nqb;
+  const int per_head = qb_end - kb;
   const int n_it = h_count * per_head;
   auto fetch = [&](int it, int buf) {
     const int h = h_first + it / per_head, q0 = (kb + it % per_head) * BQ;
@@ -300,7 +306,8 @@ __device__ __forceinline__ void dkdv_item(const BwdArgs& a, int idx, uint16_t* s
         const int key = key_a + ((e >> 1) << 3);
         const int qi = nt * 8 + 2 * (lane & 3) + (e & 1);
         const int q = q0 + qi;
-        pt[nt][e] = (key <= q && q < S && key < S) ? exp2f(pt[nt][e] * sc - lsb[qi]) : 0.0f;
+        const bool vis = key <= q && q < S && key < S && (a.W == 0 || q - key < a.W);
+        pt[nt][e] = vis ? exp2f(pt[nt][e] * sc - lsb[qi]) : 0.0f;
       }
     // dV += P^T dO
     pv_tile<HD, NC>(dv, pt, smem_u32(dos(buf)), d0, lane);
@@ -400,10 +407,11 @@ __device__ __forceinline__ void dq_item(const BwdArgs& a, int idx, uint16_t* sm)
   const int q0 = qb * BQ;
   const float sc = kLog2e * rsqrtf(static_cast<float>(HD));
 
+  const int kb0 = a.W > 0 ? max(0, q0 - a.W + 1) / BKV : 0;  // first key block inside the window
   load_tile<HD>(qs, a.qkv, a.ld, tok0, q0, S, h * HD, tid);
   load_tile<HD>(dos, a.dout, a.ldo, tok0, q0, S, h * HD, tid);
-  load_tile<HD>(ks(0), a.qkv, a.ld, tok0, 0, S, (H + kvh) * HD, tid);
-  load_tile<HD>(vs(0), a.qkv, a.ld, tok0, 0, S, (H + KV + kvh) * HD, tid);
+  load_tile<HD>(ks(0), a.qkv, a.ld, tok0, kb0 * BKV, S, (H + kvh) * HD, tid);
+  load_tile<HD>(vs(0), a.qkv, a.ld, tok0, kb0 * BKV, S, (H + KV + kvh) * HD, tid);
   cp_async_commit();
   const int ra = q0 + warp * 16 + (lane >> 2);
   float lse2[2], dvv[2];
@@ -418,8 +426,8 @@ __device__ __forceinline__ void dq_item(const BwdArgs& a, int idx, uint16_t* sm)
 #pragma unroll
   for (int i = 0; i < NC; ++i) dq[i][0] = dq[i][1] = dq[i][2] = dq[i][3] = 0.0f;
 
-  for (int kb = 0; kb <= qb; ++kb) {
-    const int k0 = kb * BKV, buf = kb & 1;
+  for (int kb = kb0; kb <= qb; ++kb) {
+    const int k0 = kb * BKV, buf = (kb - kb0) & 1;
     if (kb < qb) {
       load_tile<HD>(ks(buf ^ 1), a.qkv, a.ld, tok0, k0 + BKV, S, (H + kvh) * HD, tid);
       load_tile<HD>(vs(buf ^ 1), a.qkv, a.ld, tok0, k0 + BKV, S, (H + KV + kvh) * HD, tid);
@@ -438,7 +446,8 @@ __device__ __forceinline__ void dq_item(const BwdArgs& a, int idx, uint16_t* sm)
         const int col = k0 + nt * 8 + 2 * (lane & 3) + (e & 1);
         const int i = e >> 1;
         const int row = ra + 8 * i;
-        p[nt][e] = (col <= row && col < S && row < S) ? exp2f(p[nt][e] * sc - lse2[i]) : 0.0f;
+        const bool vis = col <= row && col < S && row < S && (a.W == 0 || row - col < a.W);
+        p[nt][e] = vis ? exp2f(p[nt][e] * sc - lse2[i]) : 0.0f;
       }
     float dp[8][4];
     qk_tile<HD>(dp, smem_u32(dos), smem_u32(vs(buf)), warp, lane);
@@ -492,7 +501,7 @@ __global__ void __launch_bounds__(128, 1) dq_kernel(const BwdArgs a) {
 
 template <int HD, int NB>
 void fwd_launch_nb(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uint16_t* o, int64_t ldo, float* lse,
-                   cudaStream_t st) {
+                   int W, cudaStream_t st) {
   constexpr int smem = (1 + 2 * NB) * 64 * (HD + 8) * 2;  // Q, NB x (K, V)
   static bool init = false;
   if (!init) {
@@ -500,22 +509,22 @@ void fwd_launch_nb(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV,
     init = true;
   }
   dim3 grid((S + BQ - 1) / BQ, H, B);
-  launch_k(fwd_kernel<HD, NB>, grid, 128, smem, st, qkv, ld, S, H, KV, o, ldo, lse);
+  launch_k(fwd_kernel<HD, NB>, grid, 128, smem, st, qkv, ld, S, H, KV, o, ldo, lse, W);
 }
 
 // Double-buffered key/value loads, except at head_dim 256 with more than two waves of CTAs: there
 // the single-buffered kernel fits two CTAs per SM, which hides the loads better.
 template <int HD>
 void fwd_launch(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uint16_t* o, int64_t ldo, float* lse,
-                cudaStream_t st) {
+                int W, cudaStream_t st) {
   const int64_t ctas = static_cast<int64_t>((S + BQ - 1) / BQ) * H * B;
-  if (HD == 256 && ctas > 2 * 152) fwd_launch_nb<HD, 1>(qkv, ld, B, S, H, KV, o, ldo, lse, st);
-  else fwd_launch_nb<HD, 2>(qkv, ld, B, S, H, KV, o, ldo, lse, st);
+  if (HD == 256 && ctas > 2 * 152) fwd_launch_nb<HD, 1>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
+  else fwd_launch_nb<HD, 2>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
 }
 
 template <int HD, int DC>
 void bwd_launch(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t ldo, const float* lse,
-                const float* dvec, int B, int S, int H, int KV, uint16_t* dqkv, cudaStream_t st) {
+                const float* dvec, int B, int S, int H, int KV, int W, uint16_t* dqkv, cudaStream_t st) {
   constexpr int smem = 6 * 64 * (HD + 8) * 2 + 4 * 64 * 4;  // 6 tiles (2 of them double-buffered) + lse, dvec x 2
   static_assert(smem <= 232448, "attention backward shared memory");
   static bool init = false;
@@ -528,7 +537,7 @@ void bwd_launch(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t l
   constexpr int NCH = HD / DC;
   const int nkb = (S + BKV - 1) / BKV, nqb = (S + BQ - 1) / BQ;
   const int grp = H / KV;
-  BwdArgs a{qkv, ld, dout, ldo, lse, dvec, S, H, KV, B, 0, dqkv};
+  BwdArgs a{qkv, ld, dout, ldo, lse, dvec, S, H, KV, B, W, 0, dqkv};
   const int n_q = nqb * H * B * NCH;      // a multiple of grp (H is)
   const int n_grouped = nkb * KV * B * NCH;
   if (n_grouped >= 2 * 152) {             // the per-kv-head items alone fill the GPU twice
@@ -544,22 +553,24 @@ void bwd_launch(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t l
 }  // namespace attn
 
 void launch_attn_fwd(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, int hd, uint16_t* o, int64_t ldo,
-                     float* lse, cudaStream_t st) {
-  if (hd == 64) attn::fwd_launch<64>(qkv, ld, B, S, H, KV, o, ldo, lse, st);
-  else if (hd == 128) attn::fwd_launch<128>(qkv, ld, B, S, H, KV, o, ldo, lse, st);
-  else attn::fwd_launch<256>(qkv, ld, B, S, H, KV, o, ldo, lse, st);
+                     float* lse, int window, cudaStream_t st) {
+  const int W = window >= S ? 0 : window;  // a window covering the sequence is plain causal
+  if (hd == 64) attn::fwd_launch<64>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
+  else if (hd == 128) attn::fwd_launch<128>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
+  else attn::fwd_launch<256>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
 }
 
 void launch_attn_bwd(const uint16_t* qkv, int64_t ld, const uint16_t* o, const uint16_t* dout, int64_t ldo,
                      const float* lse, int B, int S, int H, int KV, int hd, float* dvec, uint16_t* dqkv,
-                     cudaStream_t st) {
+                     int window, cudaStream_t st) {
+  const int W = window >= S ? 0 : window;
   const int64_t nw = static_cast<int64_t>(B) * S * H;
   launch_k(attn::dvec_kernel, static_cast<unsigned>((nw * 32 + 255) / 256), 256, 0, st, o, dout, ldo, B, S, H, hd,
            dvec);
-  if (hd == 64) attn::bwd_launch<64, 64>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, st);
+  if (hd == 64) attn::bwd_launch<64, 64>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, st);
   else if (hd == 128)
-    attn::bwd_launch<128, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, st);
-  else attn::bwd_launch<256, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, dqkv, st);
+    attn::bwd_launch<128, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, st);
+  else attn::bwd_launch<256, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, st);
 }
 
 }  // namespace mebp

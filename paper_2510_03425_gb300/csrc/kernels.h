@@ -113,18 +113,32 @@ int gemm_smem_bytes();
 void launch_compress(const float* W, int64_t rows, int64_t cols, uint8_t* qpack, uint16_t* scales, cudaStream_t st);
 void launch_decode(const uint8_t* qpack, const uint16_t* scales, int64_t rows, int64_t cols, uint16_t* out,
                    cudaStream_t st);
+// x0[t] = scale * deq(E)[ids[t]] (scale = sqrt(D) for Gemma3, else 1).
 void launch_embed(const uint8_t* qpack, const uint16_t* scales, int64_t V, int64_t D, const int32_t* ids, int64_t T,
-                  float* x0, int* err, cudaStream_t st);
+                  float* x0, int* err, float scale, cudaStream_t st);
 
 // RMSNorm: y_f16 = x * rstd * g (rstd saved); backward: dx = resid + rstd (g dy) - x rstd^3/D sum(g dy x)
 void launch_rmsnorm_fwd(const float* x, const float* g, int64_t T, int D, float eps, uint16_t* y, float* rstd,
                         cudaStream_t st);
-// dx = (resid + ...) * (*out_mult) (out_mult may be null = 1); dx_h = fp16(resid + ...) (unmultiplied).
+// dx = (resid + ...) * (*out_mult) (out_mult may be null = 1); dx_h = fp16(resid + ...) (unmultiplied);
+// either output may be null.
 void launch_rmsnorm_bwd(const float* dy, const float* x, const float* g, const float* rstd, const float* resid,
                         int64_t T, int D, const float* out_mult, float* dx, uint16_t* dx_h, cudaStream_t st);
 // RoPE (half-split) on the q and k heads of a fused [T, (H+2KV)*hd] fp16 buffer, in place.
 void launch_rope(uint16_t* qkv, int64_t T, int S, int H, int KV, int hd, const float2* cs, bool inverse,
                  cudaStream_t st);
+// Gemma3 QK-norm + RoPE on the q and k heads of the fused qkv buffer, in place; raw fp16 heads
+// [T, H+KV, hd] and their 1/rms [T, H+KV] are saved for the backward, which runs in place on dqkv.
+void launch_qknorm_rope(uint16_t* qkv, int64_t T, int S, int H, int KV, int hd, const float* qg, const float* kg,
+                        float eps, const float2* cs, uint16_t* raw, float* rstd, cudaStream_t st);
+void launch_qknorm_rope_bwd(uint16_t* dqkv, int64_t T, int S, int H, int KV, int hd, const float* qg, const float* kg,
+                            const float2* cs, const uint16_t* raw, const float* rstd, cudaStream_t st);
+// Gemma3 sandwich norms: h1 = x + norm(ao) g_pa and b = fp16(norm(h1) g2) (1/rms of ao and of h1
+// saved); y = h1 + norm(dn) g_pf (1/rms of dn saved when rpf != null; y == null computes it only).
+void launch_add_norm2(const float* ao, const float* x, const float* gpa, const float* g2, int64_t T, int D, float eps,
+                      float* h1, uint16_t* b, float* rpa, float* r2, cudaStream_t st);
+void launch_add_norm(const float* dn, const float* h1, const float* gpf, int64_t T, int D, float eps, float* y,
+                     float* rpf, cudaStream_t st);
 // Gated MLP: m = act(g) * u from gu = [g | u] (fp16 [T, 2I]); backward writes dgu fp16 [T, 2I].
 void launch_glu_fwd(const uint16_t* gu, int64_t T, int I, int act, uint16_t* m, cudaStream_t st);
 void launch_glu_bwd(const float* dm, const uint16_t* gu, int64_t T, int I, int act, uint16_t* dgu, cudaStream_t st);
@@ -166,13 +180,13 @@ void launch_lora_shadow(const float* const* A, const float* const* B, int nt, co
                         uint16_t* B_cat, uint16_t* Bt_cat, cudaStream_t st);
 
 // Attention (causal GQA).  q/k/v live inside the fused qkv buffer (row pitch ld).
+// window > 0: query i sees keys i - window + 1 .. i (sliding-window local layers); 0 = causal.
 void launch_attn_fwd(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, int hd, uint16_t* o, int64_t ldo,
-                     float* lse, cudaStream_t st);
-// part: fp32 scratch (>= 2 * B*S * H * hd floats for the per-head dK/dV mode), may be null.
+                     float* lse, int window, cudaStream_t st);
 void launch_adamw(float* p, const float* g, float* m, float* v, int64_t n, float lr, float b1, float b2, float eps,
                   float wd, float gs, double bc1, double bc2, cudaStream_t st);
 void launch_attn_bwd(const uint16_t* qkv, int64_t ld, const uint16_t* o, const uint16_t* dout, int64_t ldo,
                      const float* lse, int B, int S, int H, int KV, int hd, float* dvec, uint16_t* dqkv,
-                     cudaStream_t st);
+                     int window, cudaStream_t st);
 
 }  // namespace mebp

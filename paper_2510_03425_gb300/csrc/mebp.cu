@@ -59,6 +59,10 @@ struct Acts {
   uint16_t *a = nullptr, *qkv = nullptr, *o = nullptr, *b = nullptr, *gu = nullptr, *m = nullptr;
   float *r1 = nullptr, *r2 = nullptr, *lse_attn = nullptr, *h1 = nullptr;
   uint16_t* us[4] = {nullptr, nullptr, nullptr, nullptr};
+  // Gemma3 block only: o-proj and down-proj outputs before their sandwich norms and the norms'
+  // 1/rms, the q/k heads before QK-norm ([T, H+KV, hd]) and their 1/rms
+  float *ao = nullptr, *dn = nullptr, *rpa = nullptr, *rpf = nullptr, *rqk = nullptr;
+  uint16_t* qk_raw = nullptr;
   Shadow own;                  // shadows built by the forward itself
   const Shadow* sh = nullptr;  // the shadows the set was computed with
   // which block / input / token count the set currently holds (-1: none)
@@ -70,6 +74,7 @@ struct Acts {
 // Backward intermediates that the LoRA-gradient reductions read besides the forward set.
 struct Grads2 {
   uint16_t *dqkv = nullptr, *dgu = nullptr, *dh1_h = nullptr;
+  uint16_t* ddn_h = nullptr;  // Gemma3: gradient of the down projection's output (fp16)
   uint16_t* du[4] = {nullptr, nullptr, nullptr, nullptr};
 };
 
@@ -90,6 +95,8 @@ struct mebp_ctx {
   int64_t ws_bytes = 0;
 
   float2* rope_cs = nullptr;
+  float2* rope_cs_local = nullptr;  // RoPE table of the sliding-window layers (their own base)
+  bool gemma = false;               // Gemma3 block (QK-norm, sandwich norms, sqrt(D) embedding)
   // forward intermediates: set 0 always, set 1 when the step overlaps recompute and backward
   Acts act[2];
   int nsets = 1;
@@ -288,8 +295,18 @@ int check_lora(mebp_ctx* c, const mebp_lora* lora) {
   return MEBP_OK;
 }
 
+// Sliding window of layer `layer` (0 = global: causal over the whole sequence).
+int layer_window(const mebp_ctx* c, int layer) {
+  const int W = c->cfg.sliding_window;
+  return (W > 0 && (layer + 1) % c->cfg.global_every != 0) ? W : 0;
+}
+const float2* layer_rope(const mebp_ctx* c, int layer) {
+  return layer_window(c, layer) ? c->rope_cs_local : c->rope_cs;
+}
+
 // y = F(x) for one block.  with_down == false stops after the MLP activation (what the
-// backward consumes), so y is not produced.
+// backward consumes), so y is not produced; the Gemma3 block still runs the down projection,
+// whose output the backward of its sandwich norm reads.
 int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, const mebp_lora* lora, const float* x,
                   float* y, int B, int Sq, bool with_down, cudaStream_t st, const Shadow* sh = nullptr) {
   Acts& A = c->act[set];
@@ -311,18 +328,28 @@ int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, 
   }
   g.epi = EPI_F16; g.C = A.qkv; g.ldc = lq.N;
   if ((rc = run_gemm(c, g, st, "qkv"))) return rc;
-  launch_rope(A.qkv, T, Sq, c->H, c->KV, c->hd, c->rope_cs, false, st);
-  launch_attn_fwd(A.qkv, lq.N, B, Sq, c->H, c->KV, c->hd, A.o, c->Na, A.lse_attn, st);
+  if (c->gemma)
+    launch_qknorm_rope(A.qkv, T, Sq, c->H, c->KV, c->hd, w->q_norm, w->k_norm, c->cfg.rms_eps,
+                       layer_rope(c, layer), A.qk_raw, A.rqk, st);
+  else
+    launch_rope(A.qkv, T, Sq, c->H, c->KV, c->hd, layer_rope(c, layer), false, st);
+  launch_attn_fwd(A.qkv, lq.N, B, Sq, c->H, c->KV, c->hd, A.o, c->Na, A.lse_attn, layer_window(c, layer), st);
   const Lin& lo = c->lin[LIN_O];
   g = gemm_fwd(A.o, c->Na, T, w->o, lo.N, lo.K);
   if (lo.kx) {
     launch_skinny_gemm(A.o, c->Na, T, c->Na, A.sh->A_cat[LIN_O], c->Na, lo.kx, c->s, A.us[LIN_O], lo.kxp, st);
     g.Ax = A.us[LIN_O]; g.ldax = lo.kxp; g.kx = lo.kxp; g.Bx = A.sh->B_cat[LIN_O]; g.ldbx = lo.kxp;
   }
-  g.epi = EPI_F32; g.C = A.h1; g.ldc = D; g.R = x; g.ldr = D;
-  if ((rc = run_gemm(c, g, st, "o_proj"))) return rc;
+  if (c->gemma) {  // h1 = x + norm(ao) g_pa, b = norm(h1) g2
+    g.epi = EPI_F32; g.C = A.ao; g.ldc = D;
+    if ((rc = run_gemm(c, g, st, "o_proj"))) return rc;
+    launch_add_norm2(A.ao, x, w->post_attn_norm, w->norm2, T, D, c->cfg.rms_eps, A.h1, A.b, A.rpa, A.r2, st);
+  } else {
+    g.epi = EPI_F32; g.C = A.h1; g.ldc = D; g.R = x; g.ldr = D;
+    if ((rc = run_gemm(c, g, st, "o_proj"))) return rc;
+    launch_rmsnorm_fwd(A.h1, w->norm2, T, D, c->cfg.rms_eps, A.b, A.r2, st);
+  }
   // MLP sub-block
-  launch_rmsnorm_fwd(A.h1, w->norm2, T, D, c->cfg.rms_eps, A.b, A.r2, st);
   const Lin& lg = c->lin[LIN_GU];
   g = gemm_fwd(A.b, D, T, w->gate_up, lg.N, lg.K);
   if (lg.kx) {
@@ -334,13 +361,19 @@ int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, 
   launch_glu_fwd(A.gu, T, I, c->cfg.act, A.m, st);
   const Lin& ld = c->lin[LIN_DOWN];
   if (ld.kx) launch_skinny_gemm(A.m, I, T, I, A.sh->A_cat[LIN_DOWN], I, ld.kx, c->s, A.us[LIN_DOWN], ld.kxp, st);
-  if (with_down) {
+  if (with_down || c->gemma) {
     g = gemm_fwd(A.m, I, T, w->down, ld.N, ld.K);
     if (ld.kx) {
       g.Ax = A.us[LIN_DOWN]; g.ldax = ld.kxp; g.kx = ld.kxp; g.Bx = A.sh->B_cat[LIN_DOWN]; g.ldbx = ld.kxp;
     }
-    g.epi = EPI_F32; g.C = y; g.ldc = D; g.R = A.h1; g.ldr = D;
-    if ((rc = run_gemm(c, g, st, "down"))) return rc;
+    if (c->gemma) {  // y = h1 + norm(dn) g_pf
+      g.epi = EPI_F32; g.C = A.dn; g.ldc = D;
+      if ((rc = run_gemm(c, g, st, "down"))) return rc;
+      launch_add_norm(A.dn, A.h1, w->post_ffn_norm, T, D, c->cfg.rms_eps, with_down ? y : nullptr, A.rpf, st);
+    } else {
+      g.epi = EPI_F32; g.C = y; g.ldc = D; g.R = A.h1; g.ldr = D;
+      if ((rc = run_gemm(c, g, st, "down"))) return rc;
+    }
   }
   A.layer = layer;
   A.x = x;
@@ -389,16 +422,21 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
     if ((rc = block_forward(c, set, layer, w, lora, x, nullptr, B, Sq, false, st, sh))) return rc;
   }
   A.layer = -1;  // the set is consumed below
-  // ---- down projection: y = h1 + m Wd^T (+ s (m Ad^T) Bd^T)
+  // ---- down projection: y = h1 + m Wd^T (+ s (m Ad^T) Bd^T); Gemma3: y = h1 + norm(dn) g_pf
+  const uint16_t* ddn_h = dy_h;
+  if (c->gemma) {
+    launch_rmsnorm_bwd(dy, A.dn, w->post_ffn_norm, A.rpf, nullptr, T, D, nullptr, nullptr, G.ddn_h, st);
+    ddn_h = G.ddn_h;
+  }
   const Lin& ld = c->lin[LIN_DOWN];
-  GemmArgs g = gemm_dx(dy_h, D, T, w->down);
+  GemmArgs g = gemm_dx(ddn_h, D, T, w->down);
   if (ld.kx) {
-    launch_skinny_gemm(dy_h, D, T, D, A.sh->Bt_cat[LIN_DOWN], D, ld.kx, c->s, du[LIN_DOWN], ld.kxp, st);
+    launch_skinny_gemm(ddn_h, D, T, D, A.sh->Bt_cat[LIN_DOWN], D, ld.kx, c->s, du[LIN_DOWN], ld.kxp, st);
     g.Ax = du[LIN_DOWN]; g.ldax = ld.kxp; g.kx = ld.kxp; g.Bx = A.sh->A_cat[LIN_DOWN]; g.ldbx = I;
   }
   g.epi = EPI_F32; g.C = c->dm; g.ldc = I;
   if ((rc = run_gemm(c, g, st, "down dX"))) return rc;
-  if ((rc = lin_grads(c, A, du[LIN_DOWN], LIN_DOWN, dy_h, D, A.m, I, T, grads, acc, grad_mult, st))) return rc;
+  if ((rc = lin_grads(c, A, du[LIN_DOWN], LIN_DOWN, ddn_h, D, A.m, I, T, grads, acc, grad_mult, st))) return rc;
   // ---- gated MLP
   launch_glu_bwd(c->dm, A.gu, T, I, c->cfg.act, G.dgu, st);
   const Lin& lg = c->lin[LIN_GU];
@@ -410,8 +448,14 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   g.epi = EPI_F32; g.C = c->dtmp; g.ldc = D;
   if ((rc = run_gemm(c, g, st, "gate_up dX"))) return rc;
   if ((rc = lin_grads(c, A, du[LIN_GU], LIN_GU, G.dgu, 2 * I, A.b, D, T, grads, acc, grad_mult, st))) return rc;
-  // dh1 = dy + RMSNorm2^T(db)
-  launch_rmsnorm_bwd(c->dtmp, A.h1, w->norm2, A.r2, dy, T, D, nullptr, c->dh1, G.dh1_h, st);
+  // dh1 = dy + RMSNorm2^T(db); the o projection's output gradient is dh1 (fp16 copy in dh1_h), for
+  // Gemma3 the post-attention norm's VJP of it
+  if (c->gemma) {
+    launch_rmsnorm_bwd(c->dtmp, A.h1, w->norm2, A.r2, dy, T, D, nullptr, c->dh1, nullptr, st);
+    launch_rmsnorm_bwd(c->dh1, A.ao, w->post_attn_norm, A.rpa, nullptr, T, D, nullptr, nullptr, G.dh1_h, st);
+  } else {
+    launch_rmsnorm_bwd(c->dtmp, A.h1, w->norm2, A.r2, dy, T, D, nullptr, c->dh1, G.dh1_h, st);
+  }
   // ---- o projection
   const Lin& lo = c->lin[LIN_O];
   g = gemm_dx(G.dh1_h, D, T, w->o);
@@ -424,8 +468,13 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   if ((rc = lin_grads(c, A, du[LIN_O], LIN_O, G.dh1_h, D, A.o, c->Na, T, grads, acc, grad_mult, st))) return rc;
   // ---- attention, RoPE
   const Lin& lq = c->lin[LIN_QKV];
-  launch_attn_bwd(A.qkv, lq.N, A.o, c->dout, c->Na, A.lse_attn, B, Sq, c->H, c->KV, c->hd, c->dvec, G.dqkv, st);
-  launch_rope(G.dqkv, T, Sq, c->H, c->KV, c->hd, c->rope_cs, true, st);
+  launch_attn_bwd(A.qkv, lq.N, A.o, c->dout, c->Na, A.lse_attn, B, Sq, c->H, c->KV, c->hd, c->dvec, G.dqkv,
+                  layer_window(c, layer), st);
+  if (c->gemma)
+    launch_qknorm_rope_bwd(G.dqkv, T, Sq, c->H, c->KV, c->hd, w->q_norm, w->k_norm, layer_rope(c, layer), A.qk_raw,
+                           A.rqk, st);
+  else
+    launch_rope(G.dqkv, T, Sq, c->H, c->KV, c->hd, layer_rope(c, layer), true, st);
   // ---- q, k, v projections
   if (lq.kx)
     launch_skinny_gemm(G.dqkv, lq.N, T, lq.N, A.sh->Bt_cat[LIN_QKV], lq.N, lq.kx, c->s, du[LIN_QKV], lq.kxp, st);
@@ -450,7 +499,8 @@ int block_lora_grads(mebp_ctx* c, int set, int bset, const uint16_t* dy_h, int64
   const Grads2& G = c->bw[bset];
   const int D = c->D, I = c->I;
   int rc;
-  if ((rc = lin_grads(c, A, G.du[LIN_DOWN], LIN_DOWN, dy_h, D, A.m, I, T, grads, acc, grad_mult, st))) return rc;
+  const uint16_t* ddn_h = c->gemma ? G.ddn_h : dy_h;
+  if ((rc = lin_grads(c, A, G.du[LIN_DOWN], LIN_DOWN, ddn_h, D, A.m, I, T, grads, acc, grad_mult, st))) return rc;
   if ((rc = lin_grads(c, A, G.du[LIN_GU], LIN_GU, G.dgu, 2 * I, A.b, D, T, grads, acc, grad_mult, st))) return rc;
   if ((rc = lin_grads(c, A, G.du[LIN_O], LIN_O, G.dh1_h, D, A.o, c->Na, T, grads, acc, grad_mult, st))) return rc;
   return lin_grads(c, A, G.du[LIN_QKV], LIN_QKV, G.dqkv, c->lin[LIN_QKV].N, A.a, D, T, grads, acc, grad_mult, st);
@@ -509,8 +559,18 @@ int check_block_ptrs(mebp_ctx* c, const mebp_block_weights* w) {
   if ((rc = check_packed(c, &w->gate_up, 2 * c->I, c->D, "gate_up"))) return rc;
   if ((rc = check_packed(c, &w->down, c->D, c->I, "down"))) return rc;
   if (!w->norm1 || !w->norm2) return fail(c, MEBP_ERR_INVALID_ARG, "NULL norm gain");
+  if (c->gemma) {
+    const float* gs[4] = {w->q_norm, w->k_norm, w->post_attn_norm, w->post_ffn_norm};
+    for (const float* p : gs)
+      if (!p || !aligned16(p)) return fail(c, MEBP_ERR_INVALID_ARG, "Gemma3 norm gain NULL or not 16-byte aligned");
+  }
+  if (!aligned16(w->norm1) || !aligned16(w->norm2))
+    return fail(c, MEBP_ERR_INVALID_ARG, "norm gains must be 16-byte aligned");
   return MEBP_OK;
 }
+
+// Gemma3 scales the input embeddings by sqrt(D) (rounded to fp32 once).
+float embed_scale(const mebp_ctx* c) { return c->gemma ? static_cast<float>(std::sqrt(static_cast<double>(c->D))) : 1.0f; }
 
 int check_tokens(mebp_ctx* c, int B, int Sq) {
   if (B <= 0 || Sq <= 0) return fail(c, MEBP_ERR_INVALID_ARG, "batch and seq must be positive");
@@ -537,6 +597,8 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
   if (f.lora_targets && (f.lora_rank % 8)) return MEBP_ERR_UNSUPPORTED;
   if (f.act != MEBP_ACT_SILU && f.act != MEBP_ACT_GELU_TANH) return MEBP_ERR_INVALID_ARG;
   if (f.vocab_chunk < 0 || f.vocab_chunk % 256) return MEBP_ERR_INVALID_ARG;
+  if (f.sliding_window < 0 || (f.sliding_window > 0 && (f.global_every < 1 || !(f.rope_theta_local > 0.0f))))
+    return MEBP_ERR_INVALID_ARG;
   if (cudaSetDevice(device) != cudaSuccess) {
     cudaGetLastError();
     return MEBP_ERR_CUDA;
@@ -548,6 +610,7 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
   c->V = f.vocab; c->L = f.n_layers; c->r = f.lora_targets ? f.lora_rank : 0; c->s = f.lora_scale;
   c->Tmax = f.max_tokens;
   c->Na = c->H * c->hd;
+  c->gemma = f.gemma_norms != 0;
   setup_lin(c);
   c->Nqkv = c->lin[LIN_QKV].N;
   if (c->Na % 64) {
@@ -562,6 +625,7 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
   A(&c->d_err, 4);
   A(&c->scal, 8);
   A(&c->rope_cs, static_cast<int64_t>(f.max_seq) * (c->hd / 2));
+  if (f.sliding_window > 0) A(&c->rope_cs_local, static_cast<int64_t>(f.max_seq) * (c->hd / 2));
   // a second intermediate set lets the step overlap recompute and backward (not when spilling:
   // then device memory is the constraint)
   c->nsets = (!f.spill_ckpts && c->L > 1) ? 2 : 1;
@@ -569,6 +633,10 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
     Acts& s = c->act[k];
     A(&s.a, T * D); A(&s.b, T * D); A(&s.qkv, T * c->Nqkv); A(&s.o, T * c->Na); A(&s.gu, T * 2 * I);
     A(&s.m, T * I); A(&s.r1, T); A(&s.r2, T); A(&s.lse_attn, T * c->H); A(&s.h1, T * D);
+    if (c->gemma) {
+      A(&s.ao, T * D); A(&s.dn, T * D); A(&s.rpa, T); A(&s.rpf, T);
+      A(&s.qk_raw, T * (c->H + c->KV) * c->hd); A(&s.rqk, T * (c->H + c->KV));
+    }
     for (int li = 0; li < 4; ++li) {
       const Lin& l = c->lin[li];
       if (!l.kx) continue;
@@ -596,6 +664,7 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
   for (int k = 0; k < c->nsets; ++k) {
     Grads2& g = c->bw[k];
     A(&g.dqkv, T * c->Nqkv); A(&g.dgu, T * 2 * I); A(&g.dh1_h, T * D);
+    if (c->gemma) A(&g.ddn_h, T * D);
     for (int li = 0; li < 4; ++li)
       if (c->lin[li].kx) A(&g.du[li], T * c->lin[li].kxp);
   }
@@ -651,18 +720,20 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
     mebp_ctx_destroy(c);
     return rc;
   }
-  // RoPE table: angle(p, j) = p * theta^(-2j/hd), evaluated in double precision on the host.
-  {
+  // RoPE tables: angle(p, j) = p * theta^(-2j/hd), evaluated in double precision on the host.
+  auto rope_table = [&](float2* dst, float theta) {
     const int half = c->hd / 2;
     std::vector<float2> cs(static_cast<size_t>(f.max_seq) * half);
     for (int p = 0; p < f.max_seq; ++p)
       for (int j = 0; j < half; ++j) {
-        const double ang = p * std::pow(static_cast<double>(f.rope_theta), -2.0 * j / c->hd);
+        const double ang = p * std::pow(static_cast<double>(theta), -2.0 * j / c->hd);
         cs[static_cast<size_t>(p) * half + j] = make_float2(static_cast<float>(std::cos(ang)),
                                                             static_cast<float>(std::sin(ang)));
       }
-    cudaMemcpy(c->rope_cs, cs.data(), cs.size() * sizeof(float2), cudaMemcpyHostToDevice);
-  }
+    cudaMemcpy(dst, cs.data(), cs.size() * sizeof(float2), cudaMemcpyHostToDevice);
+  };
+  rope_table(c->rope_cs, f.rope_theta);
+  if (c->rope_cs_local) rope_table(c->rope_cs_local, f.rope_theta_local);
   cudaMemset(c->d_err, 0, 16);
   cudaMemset(c->scal, 0, 8 * sizeof(float));
   for (int li = 0; li < 4; ++li) {
@@ -798,7 +869,7 @@ int mebp_embed(mebp_ctx* c, const mebp_packed* E, const int32_t* ids, int64_t n,
     return fail(c, MEBP_ERR_INVALID_ARG, "misaligned pointer");
   if (n <= 0) return MEBP_OK;
   pdl_entry();
-  launch_embed(E->qpack, E->scales, E->rows, E->cols, ids, n, x0, c->d_err, S(stream));
+  launch_embed(E->qpack, E->scales, E->rows, E->cols, ids, n, x0, c->d_err, embed_scale(c), S(stream));
   return cuda_check(c, "embed");
 }
 
@@ -1000,7 +1071,7 @@ static int lora_step_body(mebp_ctx* c, const mebp_model_weights* model, const me
     wait_free(sl);
     x0 = dev_ckpt(sl);
   }
-  launch_embed(model->embed.qpack, model->embed.scales, c->V, D, ids, T, x0, c->d_err, st);
+  launch_embed(model->embed.qpack, model->embed.scales, c->V, D, ids, T, x0, c->d_err, embed_scale(c), st);
   if (spill) spill_out(0);
   // ---- forward loop: store only block-boundary checkpoints
   for (int i = 0; i < L; ++i) {

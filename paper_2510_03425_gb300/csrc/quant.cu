@@ -52,10 +52,11 @@ __global__ void decode_kernel(const uint8_t* __restrict__ qpack, const uint16_t*
   reinterpret_cast<uint4*>(out + r * cols)[j] = make_uint4(o[0], o[1], o[2], o[3]);
 }
 
-// x0[t, :] = deq(E)[ids[t], :] in fp32 (exact).  One warp per token, 8 elements per lane-step.
+// x0[t, :] = scale * deq(E)[ids[t], :] in fp32 (exact for scale 1).  One warp per token, 8 elements
+// per lane-step.
 __global__ void embed_kernel(const uint8_t* __restrict__ qpack, const uint16_t* __restrict__ scales, int64_t V,
                              int64_t D, const int32_t* __restrict__ ids, int64_t T, float* __restrict__ x0,
-                             int* err) {
+                             int* err, float scale) {
   griddep_wait();
   griddep_launch();
   const int64_t t = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
@@ -74,7 +75,7 @@ __global__ void embed_kernel(const uint8_t* __restrict__ qpack, const uint16_t* 
     const float s = __half2float(__ushort_as_half(scales[(j / 8) * V + id]));
     float v[8];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) v[e] = dequant_f32(word_nibble(w, e), s);
+    for (int e = 0; e < 8; ++e) v[e] = dequant_f32(word_nibble(w, e), s) * scale;
     reinterpret_cast<float4*>(dst + j * 8)[0] = make_float4(v[0], v[1], v[2], v[3]);
     reinterpret_cast<float4*>(dst + j * 8)[1] = make_float4(v[4], v[5], v[6], v[7]);
   }
@@ -93,9 +94,9 @@ void launch_decode(const uint8_t* qpack, const uint16_t* scales, int64_t rows, i
 }
 
 void launch_embed(const uint8_t* qpack, const uint16_t* scales, int64_t V, int64_t D, const int32_t* ids, int64_t T,
-                  float* x0, int* err, cudaStream_t st) {
+                  float* x0, int* err, float scale, cudaStream_t st) {
   const int64_t blocks = (T * 32 + 255) / 256;
-  launch_k(embed_kernel, static_cast<unsigned>(blocks), 256, 0, st, qpack, scales, V, D, ids, T, x0, err);
+  launch_k(embed_kernel, static_cast<unsigned>(blocks), 256, 0, st, qpack, scales, V, D, ids, T, x0, err, scale);
 }
 
 }  // namespace mebp

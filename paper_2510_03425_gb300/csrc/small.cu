@@ -71,7 +71,7 @@ __global__ void rmsnorm_bwd_kernel(const float* __restrict__ dy, const float* __
       o.x += q.x; o.y += q.y; o.z += q.z; o.w += q.w;
     }
     if (outb) outb[i] = make_uint2(pack_half2(o.x, o.y), pack_half2(o.z, o.w));
-    outr[i] = make_float4(o.x * mu, o.y * mu, o.z * mu, o.w * mu);
+    if (dx) outr[i] = make_float4(o.x * mu, o.y * mu, o.z * mu, o.w * mu);
   }
 }
 
@@ -122,6 +122,203 @@ void launch_rope(uint16_t* qkv, int64_t T, int S, int H, int KV, int hd, const f
   if (n <= 0) return;
   launch_k(rope_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, st, qkv, T, S, nheads, (H + 2 * KV) * hd, hd,
            cs, inverse ? 1 : 0);
+}
+
+// ------------------------------------------------------------------------------------ Gemma3 block
+// QK-norm then RoPE: each q or k head (token t, head h < H + KV) is RMS-normalised over its hd
+// elements with the head gain (q_norm for q heads, k_norm for k heads) and rotated in place; the
+// raw head and its 1/rms are kept for the backward.  One warp per (token, head); lane handles
+// the rotation pairs (j, j + hd/2) for j = lane + 32 i.
+template <int HD>
+__global__ void qknorm_rope_kernel(uint16_t* __restrict__ qkv, int64_t T, int S, int H, int KV, int64_t ld,
+                                   const float* __restrict__ qg, const float* __restrict__ kg, float eps,
+                                   const float2* __restrict__ cs, uint16_t* __restrict__ raw,
+                                   float* __restrict__ rstd) {
+  griddep_wait();
+  griddep_launch();
+  constexpr int HALF = HD / 2, NP = HALF / 32;
+  const int nh = H + KV;
+  const int64_t wid = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (wid >= T * nh) return;
+  const int head = static_cast<int>(wid % nh);
+  const int64_t t = wid / nh;
+  const int pos = static_cast<int>(t % S);
+  uint16_t* base = qkv + t * ld + static_cast<int64_t>(head) * HD;
+  uint16_t* rb = raw + wid * HD;
+  const float* g = head < H ? qg : kg;
+  float x1[NP], x2[NP];
+  float ss = 0.0f;
+#pragma unroll
+  for (int i = 0; i < NP; ++i) {
+    const int j = lane + 32 * i;
+    const uint16_t a = base[j], b = base[j + HALF];
+    rb[j] = a;
+    rb[j + HALF] = b;
+    x1[i] = h_to_f(a);
+    x2[i] = h_to_f(b);
+    ss += x1[i] * x1[i] + x2[i] * x2[i];
+  }
+  ss = warp_sum(ss);
+  const float r = rsqrtf(ss / static_cast<float>(HD) + eps);
+  if (lane == 0) rstd[wid] = r;
+#pragma unroll
+  for (int i = 0; i < NP; ++i) {
+    const int j = lane + 32 * i;
+    const float y1 = x1[i] * r * g[j], y2 = x2[i] * r * g[j + HALF];
+    const float2 c = cs[static_cast<int64_t>(pos) * HALF + j];
+    base[j] = f_to_h(y1 * c.x - y2 * c.y);
+    base[j + HALF] = f_to_h(y2 * c.x + y1 * c.y);
+  }
+}
+
+// Backward of qknorm_rope on dqkv in place: rotate the head gradient back (by -angle), then
+// the RMSNorm VJP dx = r (g dy) - x r^3 / hd * sum(g dy x) with the saved raw head x and r.
+template <int HD>
+__global__ void qknorm_rope_bwd_kernel(uint16_t* __restrict__ dqkv, int64_t T, int S, int H, int KV, int64_t ld,
+                                       const float* __restrict__ qg, const float* __restrict__ kg,
+                                       const float2* __restrict__ cs, const uint16_t* __restrict__ raw,
+                                       const float* __restrict__ rstd) {
+  griddep_wait();
+  griddep_launch();
+  constexpr int HALF = HD / 2, NP = HALF / 32;
+  const int nh = H + KV;
+  const int64_t wid = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (wid >= T * nh) return;
+  const int head = static_cast<int>(wid % nh);
+  const int64_t t = wid / nh;
+  const int pos = static_cast<int>(t % S);
+  uint16_t* base = dqkv + t * ld + static_cast<int64_t>(head) * HD;
+  const uint16_t* rb = raw + wid * HD;
+  const float* g = head < H ? qg : kg;
+  float gd1[NP], gd2[NP], x1[NP], x2[NP];
+  float dot = 0.0f;
+#pragma unroll
+  for (int i = 0; i < NP; ++i) {
+    const int j = lane + 32 * i;
+    const float d1 = h_to_f(base[j]), d2 = h_to_f(base[j + HALF]);
+    const float2 c = cs[static_cast<int64_t>(pos) * HALF + j];
+    gd1[i] = g[j] * (d1 * c.x + d2 * c.y);
+    gd2[i] = g[j + HALF] * (d2 * c.x - d1 * c.y);
+    x1[i] = h_to_f(rb[j]);
+    x2[i] = h_to_f(rb[j + HALF]);
+    dot += gd1[i] * x1[i] + gd2[i] * x2[i];
+  }
+  dot = warp_sum(dot);
+  const float r = rstd[wid];
+  const float cc = r * r * r * dot / static_cast<float>(HD);
+#pragma unroll
+  for (int i = 0; i < NP; ++i) {
+    const int j = lane + 32 * i;
+    base[j] = f_to_h(r * gd1[i] - x1[i] * cc);
+    base[j + HALF] = f_to_h(r * gd2[i] - x2[i] * cc);
+  }
+}
+
+void launch_qknorm_rope(uint16_t* qkv, int64_t T, int S, int H, int KV, int hd, const float* qg, const float* kg,
+                        float eps, const float2* cs, uint16_t* raw, float* rstd, cudaStream_t st) {
+  const int64_t n = T * (H + KV) * 32;
+  if (n <= 0) return;
+  const int64_t ld = static_cast<int64_t>(H + 2 * KV) * hd;
+  const unsigned grid = static_cast<unsigned>((n + 255) / 256);
+  if (hd == 64) launch_k(qknorm_rope_kernel<64>, grid, 256, 0, st, qkv, T, S, H, KV, ld, qg, kg, eps, cs, raw, rstd);
+  else if (hd == 128) launch_k(qknorm_rope_kernel<128>, grid, 256, 0, st, qkv, T, S, H, KV, ld, qg, kg, eps, cs, raw, rstd);
+  else launch_k(qknorm_rope_kernel<256>, grid, 256, 0, st, qkv, T, S, H, KV, ld, qg, kg, eps, cs, raw, rstd);
+}
+void launch_qknorm_rope_bwd(uint16_t* dqkv, int64_t T, int S, int H, int KV, int hd, const float* qg, const float* kg,
+                            const float2* cs, const uint16_t* raw, const float* rstd, cudaStream_t st) {
+  const int64_t n = T * (H + KV) * 32;
+  if (n <= 0) return;
+  const int64_t ld = static_cast<int64_t>(H + 2 * KV) * hd;
+  const unsigned grid = static_cast<unsigned>((n + 255) / 256);
+  if (hd == 64) launch_k(qknorm_rope_bwd_kernel<64>, grid, 256, 0, st, dqkv, T, S, H, KV, ld, qg, kg, cs, raw, rstd);
+  else if (hd == 128)
+    launch_k(qknorm_rope_bwd_kernel<128>, grid, 256, 0, st, dqkv, T, S, H, KV, ld, qg, kg, cs, raw, rstd);
+  else launch_k(qknorm_rope_bwd_kernel<256>, grid, 256, 0, st, dqkv, T, S, H, KV, ld, qg, kg, cs, raw, rstd);
+}
+
+// Sandwich norm after attention, residual add and the MLP pre-norm in one pass per row:
+// h1 = x + ao * r_pa * g_pa (r_pa = 1/rms(ao)), b = fp16(h1 * r2 * g2) (r2 = 1/rms(h1)).
+__global__ void add_norm2_kernel(const float* __restrict__ ao, const float* __restrict__ x,
+                                 const float* __restrict__ gpa, const float* __restrict__ g2, int64_t T, int D,
+                                 float eps, float* __restrict__ h1, uint16_t* __restrict__ b, float* __restrict__ rpa,
+                                 float* __restrict__ r2) {
+  griddep_wait();
+  griddep_launch();
+  const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (row >= T) return;
+  const int n4 = D >> 2;
+  const float4* ar = reinterpret_cast<const float4*>(ao + row * D);
+  const float4* xr = reinterpret_cast<const float4*>(x + row * D);
+  const float4* gp = reinterpret_cast<const float4*>(gpa);
+  const float4* gq = reinterpret_cast<const float4*>(g2);
+  float4* hr = reinterpret_cast<float4*>(h1 + row * D);
+  float ss = 0.0f;
+  for (int i = lane; i < n4; i += 32) {
+    const float4 v = ar[i];
+    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  }
+  const float ra = rsqrtf(warp_sum(ss) / static_cast<float>(D) + eps);
+  float sh = 0.0f;
+  for (int i = lane; i < n4; i += 32) {
+    const float4 v = ar[i], w = gp[i], xx = xr[i];
+    const float4 h = make_float4(xx.x + v.x * ra * w.x, xx.y + v.y * ra * w.y, xx.z + v.z * ra * w.z,
+                                 xx.w + v.w * ra * w.w);
+    hr[i] = h;
+    sh += h.x * h.x + h.y * h.y + h.z * h.z + h.w * h.w;
+  }
+  const float rb = rsqrtf(warp_sum(sh) / static_cast<float>(D) + eps);
+  if (lane == 0) {
+    rpa[row] = ra;
+    r2[row] = rb;
+  }
+  uint2* br = reinterpret_cast<uint2*>(b + row * D);
+  for (int i = lane; i < n4; i += 32) {  // the row this thread just wrote
+    const float4 h = hr[i], w = gq[i];
+    br[i] = make_uint2(pack_half2(h.x * rb * w.x, h.y * rb * w.y), pack_half2(h.z * rb * w.z, h.w * rb * w.w));
+  }
+}
+
+// Sandwich norm after the MLP and the residual add: y = h1 + dn * r_pf * g_pf.
+__global__ void add_norm_kernel(const float* __restrict__ dn, const float* __restrict__ h1,
+                                const float* __restrict__ gpf, int64_t T, int D, float eps, float* __restrict__ y,
+                                float* __restrict__ rpf) {
+  griddep_wait();
+  griddep_launch();
+  const int64_t row = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (row >= T) return;
+  const int n4 = D >> 2;
+  const float4* dr = reinterpret_cast<const float4*>(dn + row * D);
+  const float4* hr = reinterpret_cast<const float4*>(h1 + row * D);
+  const float4* gp = reinterpret_cast<const float4*>(gpf);
+  float4* yr = reinterpret_cast<float4*>(y ? y + row * D : nullptr);
+  float ss = 0.0f;
+  for (int i = lane; i < n4; i += 32) {
+    const float4 v = dr[i];
+    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  }
+  const float r = rsqrtf(warp_sum(ss) / static_cast<float>(D) + eps);
+  if (lane == 0 && rpf) rpf[row] = r;
+  if (!y) return;  // the backward's recompute wants the 1/rms only
+  for (int i = lane; i < n4; i += 32) {
+    const float4 v = dr[i], w = gp[i], h = hr[i];
+    yr[i] = make_float4(h.x + v.x * r * w.x, h.y + v.y * r * w.y, h.z + v.z * r * w.z, h.w + v.w * r * w.w);
+  }
+}
+
+void launch_add_norm2(const float* ao, const float* x, const float* gpa, const float* g2, int64_t T, int D, float eps,
+                      float* h1, uint16_t* b, float* rpa, float* r2, cudaStream_t st) {
+  if (T <= 0) return;
+  launch_k(add_norm2_kernel, static_cast<unsigned>((T * 32 + 255) / 256), 256, 0, st, ao, x, gpa, g2, T, D, eps, h1,
+           b, rpa, r2);
+}
+void launch_add_norm(const float* dn, const float* h1, const float* gpf, int64_t T, int D, float eps, float* y,
+                     float* rpf, cudaStream_t st) {
+  if (T <= 0) return;
+  launch_k(add_norm_kernel, static_cast<unsigned>((T * 32 + 255) / 256), 256, 0, st, dn, h1, gpf, T, D, eps, y, rpf);
 }
 
 // ------------------------------------------------------------------------------------ gated MLP

@@ -35,7 +35,8 @@ class ModelCfg(ctypes.Structure):
                 ("intermediate", c_int32), ("vocab", c_int32), ("n_layers", c_int32), ("act", c_int32),
                 ("rope_theta", c_float), ("rms_eps", c_float), ("lora_rank", c_int32), ("lora_scale", c_float),
                 ("lora_targets", c_uint32), ("max_tokens", c_int32), ("max_seq", c_int32),
-                ("spill_ckpts", c_int32), ("vocab_chunk", c_int32)]
+                ("spill_ckpts", c_int32), ("vocab_chunk", c_int32), ("gemma_norms", c_int32),
+                ("sliding_window", c_int32), ("global_every", c_int32), ("rope_theta_local", c_float)]
 
 
 class Packed(ctypes.Structure):
@@ -44,7 +45,8 @@ class Packed(ctypes.Structure):
 
 class BlockWeights(ctypes.Structure):
     _fields_ = [("qkv", Packed), ("o", Packed), ("gate_up", Packed), ("down", Packed),
-                ("norm1", c_void_p), ("norm2", c_void_p)]
+                ("norm1", c_void_p), ("norm2", c_void_p), ("q_norm", c_void_p), ("k_norm", c_void_p),
+                ("post_attn_norm", c_void_p), ("post_ffn_norm", c_void_p)]
 
 
 class Lora(ctypes.Structure):
@@ -183,7 +185,9 @@ def model_cfg(dims, max_tokens=None, max_seq=None, spill=None, vocab_chunk=0) ->
     return ModelCfg(dims.hidden, dims.n_heads, dims.n_kv_heads, dims.head_dim, dims.intermediate, dims.vocab,
                     dims.n_layers, ACT[dims.act], dims.rope_theta, dims.eps, dims.rank, dims.alpha / dims.rank,
                     mask, max_tokens or dims.batch * dims.seq, max_seq or dims.seq,
-                    int(dims.spill if spill is None else spill), vocab_chunk)
+                    int(dims.spill if spill is None else spill), vocab_chunk,
+                    int(getattr(dims, "gemma_norms", False)), int(getattr(dims, "sliding_window", 0)),
+                    int(getattr(dims, "global_every", 1)), float(getattr(dims, "rope_theta_local", 1e4)))
 
 
 # ----------------------------------------------------------------------------- C entry points

@@ -58,17 +58,22 @@ class PackedLinear:
 
 class DeviceBlock:
     def __init__(self, ctx: Context, W: Dict[str, torch.Tensor]):
-        """W: dense fp32 device tensors q, k, v, o, gate, up, down ([N, K]) and norm1, norm2."""
+        """W: dense fp32 device tensors q, k, v, o, gate, up, down ([N, K]) and norm1, norm2; for
+        the Gemma3 block also q_norm, k_norm ([head_dim]) and post_attn_norm, post_ffn_norm."""
         self.qkv = PackedLinear(*compress(ctx, torch.cat([W["q"], W["k"], W["v"]], 0)))
         self.o = PackedLinear(*compress(ctx, W["o"]))
         self.gate_up = PackedLinear(*compress(ctx, torch.cat([W["gate"], W["up"]], 0)))
         self.down = PackedLinear(*compress(ctx, W["down"]))
-        self.norm1 = W["norm1"].contiguous().float()
-        self.norm2 = W["norm2"].contiguous().float()
+        self.norms = {n: W[n].contiguous().float() for n in
+                      ("norm1", "norm2", "q_norm", "k_norm", "post_attn_norm", "post_ffn_norm") if n in W}
+        self.norm1 = self.norms["norm1"]
+        self.norm2 = self.norms["norm2"]
 
     def struct(self) -> M.BlockWeights:
+        opt = [self.norms[n].data_ptr() if n in self.norms else None
+               for n in ("q_norm", "k_norm", "post_attn_norm", "post_ffn_norm")]
         return M.BlockWeights(self.qkv.struct(), self.o.struct(), self.gate_up.struct(), self.down.struct(),
-                              self.norm1.data_ptr(), self.norm2.data_ptr())
+                              self.norm1.data_ptr(), self.norm2.data_ptr(), *opt)
 
 
 class DeviceModel:
