@@ -37,7 +37,18 @@ def workload_name(d) -> str:
     return (f"{d.name}: {d.n_layers} blocks (D {d.hidden}, H {d.n_heads}/KV {d.n_kv_heads}, hd {d.head_dim}, "
             f"I {d.intermediate}, {d.act}), vocab {d.vocab}, batch {d.batch} x seq {d.seq}, "
             f"LoRA r{d.rank} on {'/'.join(d.targets)}, 4-bit g64 fp16-scale base weights"
-            + (", checkpoints spilled to pinned host" if d.spill else ""))
+            + (", checkpoints spilled to pinned host" if d.spill else "")
+            + (f", Gemma3 block (QK-norm, sandwich norms, sqrt(D) embedding, window {d.sliding_window} on "
+               f"{d.global_every - 1} of every {d.global_every} layers, local RoPE base {d.rope_theta_local:g})"
+               if d.gemma_norms else ""))
+
+
+def gemma3_extras(d):
+    """The Gemma-shaped workload with the Gemma3 block options on: QK-norm, sandwich norms,
+    sqrt(D) embedding scale, five local layers (window 512 for the 1B shape, 1024 for the 4B
+    shape, RoPE base 1e4) per global layer."""
+    return d.with_(gemma_norms=True, sliding_window=512 if d.hidden < 2048 else 1024, global_every=6,
+                   rope_theta_local=1e4)
 
 
 def peaks():
@@ -515,6 +526,8 @@ def main():
     ap.add_argument("--gemm-shapes", default=None, help="comma list of qkv,o,gate_up,down for --gemm-bench")
     ap.add_argument("--table2", action="store_true",
                     help="decompression-overhead (Table 2) and sequence-length (Table 3) analogues")
+    ap.add_argument("--gemma3", action="store_true",
+                    help="Gemma-shaped configs (2, 4) with the Gemma3 block options on")
     ap.add_argument("--launch-list", action="store_true",
                     help="no timing: after the warm-up run one eager step inside the NVTX range "
                          "'mebp_step' (for ncu --nvtx --nvtx-include mebp_step/)")
@@ -524,6 +537,10 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     d = synth.preset(args.config)
+    if args.gemma3:
+        if d.act != "gelu_tanh":
+            ap.error("--gemma3 applies to the Gemma-shaped configs 2 and 4")
+        d = gemma3_extras(d)
 
     if args.gemm_bench:
         out = gemm_bench(args.config, args.gemm_m, reps=args.steps, warmup=args.warmup,
