@@ -80,7 +80,8 @@ __device__ __forceinline__ void pv_tile(float (&acc)[NC][4], const float (&p)[8]
 // ------------------------------------------------------------------------------------ forward
 // NB key/value buffers: 2 overlaps the next block's load with this one; 1 leaves room for two
 // CTAs per SM at head_dim 256.
-template <int HD, int NB>
+// WIN: sliding-window layer (window W); false compiles the plain causal kernel.
+template <int HD, int NB, bool WIN>
 __global__ void __launch_bounds__(128, 1) fwd_kernel(const uint16_t* __restrict__ qkv, int64_t ld, int S, int H,
                                                      int KV, uint16_t* __restrict__ o, int64_t ldo,
                                                      float* __restrict__ lse, int W) {
@@ -98,7 +99,7 @@ __global__ void __launch_bounds__(128, 1) fwd_kernel(const uint16_t* __restrict_
   const int q0 = qb * BQ;
   const float sc = kLog2e * rsqrtf(static_cast<float>(HD));
 
-  const int kb0 = W > 0 ? max(0, q0 - W + 1) / BKV : 0;  // first key block inside the window
+  const int kb0 = WIN ? max(0, q0 - W + 1) / BKV : 0;  // first key block inside the window
   load_tile<HD>(qs, qkv, ld, tok0, q0, S, h * HD, tid);
   if (NB == 2) {
     load_tile<HD>(ks(0), qkv, ld, tok0, kb0 * BKV, S, (H + kvh) * HD, tid);
@@ -138,7 +139,7 @@ __global__ void __launch_bounds__(128, 1) fwd_kernel(const uint16_t* __restrict_
       for (int e = 0; e < 4; ++e) {
         const int col = k0 + nt * 8 + 2 * (lane & 3) + (e & 1);
         const int row = ra + ((e >> 1) << 3);
-        s[nt][e] = (col > row || col >= S || (W > 0 && row - col >= W)) ? -INFINITY : s[nt][e] * sc;
+        s[nt][e] = (col > row || col >= S || (WIN && row - col >= W)) ? -INFINITY : s[nt][e] * sc;
       }
 #pragma unroll
     for (int i = 0; i < 2; ++i) {
@@ -230,7 +231,7 @@ struct BwdArgs {
 //               thread-block cluster (rank j = head kvh*grp + j) whose fp32 partials are summed
 //               over distributed shared memory in head order (small grids);
 //   CL = false: one item per kv head, looping over its grp query heads (large grids).
-template <int HD, int DC, bool CL>
+template <int HD, int DC, bool CL, bool WIN>
 __device__ __forceinline__ void dkdv_item(const BwdArgs& a, int idx, uint16_t* sm) {
   constexpr int LD = HD + 8, NC = DC / 8, NCH = HD / DC;
   const int S = a.S, H = a.H, KV = a.KV;
@@ -264,7 +265,7 @@ __device__ __forceinline__ void dkdv_item(const BwdArgs& a, int idx, uint16_t* s
   const int key_a = k0 + warp * 16 + (lane >> 2);
   const int nqb = (S + BQ - 1) / BQ;
   // query blocks kb .. qb_end-1 see this key block (with a window, queries < k0 + BKV - 1 + W)
-  const int qb_end = a.W > 0 ? min(nqb, (k0 + BKV - 1 + a.W - 1) / BQ + 1) : nqb;
+  const int qb_end = WIN ? min(nqb, (k0 + BKV - 1 + a.W - 1) / BQ + 1) : nqb;
   const int per_head = qb_end - kb;
   const int n_it = h_count * per_head;
   auto fetch = [&](int it, int buf) {
@@ -306,7 +307,7 @@ __device__ __forceinline__ void dkdv_item(const BwdArgs& a, int idx, uint16_t* s
         const int key = key_a + ((e >> 1) << 3);
         const int qi = nt * 8 + 2 * (lane & 3) + (e & 1);
         const int q = q0 + qi;
-        const bool vis = key <= q && q < S && key < S && (a.W == 0 || q - key < a.W);
+        const bool vis = key <= q && q < S && key < S && (!WIN || q - key < a.W);
         pt[nt][e] = vis ? exp2f(pt[nt][e] * sc - lsb[qi]) : 0.0f;
       }
     // dV += P^T dO
@@ -387,7 +388,7 @@ __device__ __forceinline__ void dkdv_item(const BwdArgs& a, int idx, uint16_t* s
 }
 
 // dQ for one query block of one head, output columns d0 .. d0 + DC.
-template <int HD, int DC>
+template <int HD, int DC, bool WIN>
 __device__ __forceinline__ void dq_item(const BwdArgs& a, int idx, uint16_t* sm) {
   constexpr int LD = HD + 8, NC = DC / 8, NCH = HD / DC;
   const int S = a.S, H = a.H, KV = a.KV;
@@ -407,7 +408,7 @@ __device__ __forceinline__ void dq_item(const BwdArgs& a, int idx, uint16_t* sm)
   const int q0 = qb * BQ;
   const float sc = kLog2e * rsqrtf(static_cast<float>(HD));
 
-  const int kb0 = a.W > 0 ? max(0, q0 - a.W + 1) / BKV : 0;  // first key block inside the window
+  const int kb0 = WIN ? max(0, q0 - a.W + 1) / BKV : 0;  // first key block inside the window
   load_tile<HD>(qs, a.qkv, a.ld, tok0, q0, S, h * HD, tid);
   load_tile<HD>(dos, a.dout, a.ldo, tok0, q0, S, h * HD, tid);
   load_tile<HD>(ks(0), a.qkv, a.ld, tok0, kb0 * BKV, S, (H + kvh) * HD, tid);
@@ -446,7 +447,7 @@ __device__ __forceinline__ void dq_item(const BwdArgs& a, int idx, uint16_t* sm)
         const int col = k0 + nt * 8 + 2 * (lane & 3) + (e & 1);
         const int i = e >> 1;
         const int row = ra + 8 * i;
-        const bool vis = col <= row && col < S && row < S && (a.W == 0 || row - col < a.W);
+        const bool vis = col <= row && col < S && row < S && (!WIN || row - col < a.W);
         p[nt][e] = vis ? exp2f(p[nt][e] * sc - lse2[i]) : 0.0f;
       }
     float dp[8][4];
@@ -474,42 +475,42 @@ __device__ __forceinline__ void dq_item(const BwdArgs& a, int idx, uint16_t* sm)
 // Small grids: one launch for both backward passes; blocks [0, n_kv) are dK/dV items (clusters
 // of the grp query heads of a kv head), the rest dQ items, and the two kinds run concurrently.
 // n_kv is a multiple of grp, so no cluster mixes the kinds.
-template <int HD, int DC>
+template <int HD, int DC, bool WIN>
 __global__ void __launch_bounds__(128, 1) bwd_kernel(const BwdArgs a) {
   griddep_wait();
   griddep_launch();
   extern __shared__ __align__(16) uint16_t sm[];
-  if (static_cast<int>(blockIdx.x) < a.n_kv) dkdv_item<HD, DC, true>(a, blockIdx.x, sm);
-  else dq_item<HD, DC>(a, blockIdx.x - a.n_kv, sm);
+  if (static_cast<int>(blockIdx.x) < a.n_kv) dkdv_item<HD, DC, true, WIN>(a, blockIdx.x, sm);
+  else dq_item<HD, DC, WIN>(a, blockIdx.x - a.n_kv, sm);
 }
 
 // Large grids: dK/dV with one CTA per kv head, then dQ, as two launches.
-template <int HD, int DC>
+template <int HD, int DC, bool WIN>
 __global__ void __launch_bounds__(128, 1) dkdv_kernel(const BwdArgs a) {
   griddep_wait();
   griddep_launch();
   extern __shared__ __align__(16) uint16_t sm[];
-  dkdv_item<HD, DC, false>(a, blockIdx.x, sm);
+  dkdv_item<HD, DC, false, WIN>(a, blockIdx.x, sm);
 }
-template <int HD, int DC>
+template <int HD, int DC, bool WIN>
 __global__ void __launch_bounds__(128, 1) dq_kernel(const BwdArgs a) {
   griddep_wait();
   griddep_launch();
   extern __shared__ __align__(16) uint16_t sm[];
-  dq_item<HD, DC>(a, blockIdx.x, sm);
+  dq_item<HD, DC, WIN>(a, blockIdx.x, sm);
 }
 
-template <int HD, int NB>
+template <int HD, int NB, bool WIN>
 void fwd_launch_nb(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uint16_t* o, int64_t ldo, float* lse,
                    int W, cudaStream_t st) {
   constexpr int smem = (1 + 2 * NB) * 64 * (HD + 8) * 2;  // Q, NB x (K, V)
   static bool init = false;
   if (!init) {
-    cudaFuncSetAttribute(fwd_kernel<HD, NB>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(fwd_kernel<HD, NB, WIN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     init = true;
   }
   dim3 grid((S + BQ - 1) / BQ, H, B);
-  launch_k(fwd_kernel<HD, NB>, grid, 128, smem, st, qkv, ld, S, H, KV, o, ldo, lse, W);
+  launch_k(fwd_kernel<HD, NB, WIN>, grid, 128, smem, st, qkv, ld, S, H, KV, o, ldo, lse, W);
 }
 
 // Double-buffered key/value loads, except at head_dim 256 with more than two waves of CTAs: there
@@ -518,20 +519,26 @@ template <int HD>
 void fwd_launch(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uint16_t* o, int64_t ldo, float* lse,
                 int W, cudaStream_t st) {
   const int64_t ctas = static_cast<int64_t>((S + BQ - 1) / BQ) * H * B;
-  if (HD == 256 && ctas > 2 * 152) fwd_launch_nb<HD, 1>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
-  else fwd_launch_nb<HD, 2>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
+  const bool nb1 = HD == 256 && ctas > 2 * 152;
+  if (W > 0) {
+    if (nb1) fwd_launch_nb<HD, 1, true>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
+    else fwd_launch_nb<HD, 2, true>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
+  } else {
+    if (nb1) fwd_launch_nb<HD, 1, false>(qkv, ld, B, S, H, KV, o, ldo, lse, 0, st);
+    else fwd_launch_nb<HD, 2, false>(qkv, ld, B, S, H, KV, o, ldo, lse, 0, st);
+  }
 }
 
-template <int HD, int DC>
-void bwd_launch(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t ldo, const float* lse,
+template <int HD, int DC, bool WIN>
+void bwd_launch_w(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t ldo, const float* lse,
                 const float* dvec, int B, int S, int H, int KV, int W, uint16_t* dqkv, cudaStream_t st) {
   constexpr int smem = 6 * 64 * (HD + 8) * 2 + 4 * 64 * 4;  // 6 tiles (2 of them double-buffered) + lse, dvec x 2
   static_assert(smem <= 232448, "attention backward shared memory");
   static bool init = false;
   if (!init) {
-    cudaFuncSetAttribute(bwd_kernel<HD, DC>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    cudaFuncSetAttribute(dkdv_kernel<HD, DC>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    cudaFuncSetAttribute(dq_kernel<HD, DC>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(bwd_kernel<HD, DC, WIN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(dkdv_kernel<HD, DC, WIN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(dq_kernel<HD, DC, WIN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     init = true;
   }
   constexpr int NCH = HD / DC;
@@ -542,12 +549,18 @@ void bwd_launch(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t l
   const int n_grouped = nkb * KV * B * NCH;
   if (n_grouped >= 2 * 152) {             // the per-kv-head items alone fill the GPU twice
     a.n_kv = n_grouped;
-    launch_k(dkdv_kernel<HD, DC>, dim3(a.n_kv), 128, smem, st, a);
-    launch_k(dq_kernel<HD, DC>, dim3(n_q), 128, smem, st, a);
+    launch_k(dkdv_kernel<HD, DC, WIN>, dim3(a.n_kv), 128, smem, st, a);
+    launch_k(dq_kernel<HD, DC, WIN>, dim3(n_q), 128, smem, st, a);
     return;
   }
   a.n_kv = nkb * H * B * NCH;             // one item per (key block, query head, batch, column chunk)
-  launch_k_cluster(bwd_kernel<HD, DC>, dim3(a.n_kv + n_q), 128, smem, st, dim3(grp, 1, 1), a);
+  launch_k_cluster(bwd_kernel<HD, DC, WIN>, dim3(a.n_kv + n_q), 128, smem, st, dim3(grp, 1, 1), a);
+}
+template <int HD, int DC>
+void bwd_launch(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t ldo, const float* lse,
+                const float* dvec, int B, int S, int H, int KV, int W, uint16_t* dqkv, cudaStream_t st) {
+  if (W > 0) bwd_launch_w<HD, DC, true>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, st);
+  else bwd_launch_w<HD, DC, false>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, 0, dqkv, st);
 }
 
 }  // namespace attn
