@@ -23,11 +23,13 @@ namespace attn {
 constexpr int BQ = 64, BKV = 64;
 constexpr float kLog2e = 1.4426950408889634f;
 
-template <int HD>
+// 64 rows x HD columns into shared memory (row pitch HD + 8), NT threads cooperating; rows past S
+// are zero-filled.
+template <int HD, int NT = 128>
 __device__ __forceinline__ void load_tile(uint16_t* dst, const uint16_t* base, int64_t ld, int64_t tok0, int r0,
                                           int S, int col, int tid) {
   constexpr int LD = HD + 8, CH = HD / 8;
-  for (int c = tid; c < 64 * CH; c += 128) {
+  for (int c = tid; c < 64 * CH; c += NT) {
     const int r = c / CH, cc = c % CH;
     const bool v = r0 + r < S;
     const uint16_t* src = v ? base + (tok0 + r0 + r) * ld + col + cc * 8 : base;
@@ -78,102 +80,157 @@ __device__ __forceinline__ void pv_tile(float (&acc)[NC][4], const float (&p)[8]
 }
 
 // ------------------------------------------------------------------------------------ forward
-// NB key/value buffers: 2 overlaps the next block's load with this one; 1 leaves room for two
-// CTAs per SM at head_dim 256.
-// WIN: sliding-window layer (window W); false compiles the plain causal kernel.
-template <int HD, int NB, bool WIN>
-__global__ void __launch_bounds__(128, 1) fwd_kernel(const uint16_t* __restrict__ qkv, int64_t ld, int S, int H,
-                                                     int KV, uint16_t* __restrict__ o, int64_t ldo,
-                                                     float* __restrict__ lse, int W) {
+// One CTA per (query block of 64 rows, head, sequence) with NWG warp-groups of four warps (warp r
+// of a group owns query rows 16 r .. 16 r + 15).  Warp-group g takes key blocks kb_first + g,
+// kb_first + g + NWG, ... with its own online softmax, and the groups' (max, sum, o) are merged
+// through shared memory at the end: NWG = 2 on grids of less than one CTA per SM doubles the warps
+// per scheduler and halves the serial key-block steps of the longest query block.  NB key/value
+// buffers per group: 2 overlaps the next round's loads with this one; 1 saves shared memory.
+// WIN: sliding-window layer (window W); key blocks wholly before the window are skipped.  (Masking
+// only the blocks a mask cuts measured slower than masking every block.)
+template <int HD, int NB, bool WIN, int NWG>
+__global__ void __launch_bounds__(128 * NWG, 1) fwd_kernel(const uint16_t* __restrict__ qkv, int64_t ld, int S,
+                                                           int H, int KV, uint16_t* __restrict__ o, int64_t ldo,
+                                                           float* __restrict__ lse, int W) {
   griddep_wait();
   griddep_launch();
-  constexpr int LD = HD + 8, NO = HD / 8;
+  constexpr int LD = HD + 8, NO = HD / 8, NT = 128 * NWG, TILE = BQ * LD;
   extern __shared__ __align__(16) uint16_t sm[];
-  uint16_t* qs = sm;  // then NB (K, V) buffers
-  auto ks = [&](int buf) { return qs + (1 + 2 * buf) * BQ * LD; };
-  auto vs = [&](int buf) { return qs + (2 + 2 * buf) * BQ * LD; };
+  uint16_t* qs = sm;  // then per buffer slot and group: K, V
+  auto ks = [&](int buf, int g) { return qs + (1 + 2 * (buf * NWG + g)) * TILE; };
+  auto vs = [&](int buf, int g) { return qs + (2 + 2 * (buf * NWG + g)) * TILE; };
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int wg = warp >> 2, wr = warp & 3;
   const int qb = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int kvh = h / (H / KV);
   const int64_t tok0 = static_cast<int64_t>(b) * S;
   const int q0 = qb * BQ;
   const float sc = kLog2e * rsqrtf(static_cast<float>(HD));
-
-  const int kb0 = WIN ? max(0, q0 - W + 1) / BKV : 0;  // first key block inside the window
-  load_tile<HD>(qs, qkv, ld, tok0, q0, S, h * HD, tid);
-  if (NB == 2) {
-    load_tile<HD>(ks(0), qkv, ld, tok0, kb0 * BKV, S, (H + kvh) * HD, tid);
-    load_tile<HD>(vs(0), qkv, ld, tok0, kb0 * BKV, S, (H + KV + kvh) * HD, tid);
-  }
+  // visible key blocks: kb_first .. qb (window: from the first block inside it)
+  const int kb_first = WIN ? max(0, q0 - W + 1) / BKV : 0;
+  const int nrounds = (qb - kb_first + NWG) / NWG;
+  auto fetch = [&](int t, int buf) {  // the key/value blocks of round t, one per group
+#pragma unroll
+    for (int g = 0; g < NWG; ++g) {
+      const int kb = kb_first + t * NWG + g;
+      if (kb > qb) break;
+      load_tile<HD, NT>(ks(buf, g), qkv, ld, tok0, kb * BKV, S, (H + kvh) * HD, tid);
+      load_tile<HD, NT>(vs(buf, g), qkv, ld, tok0, kb * BKV, S, (H + KV + kvh) * HD, tid);
+    }
+  };
+  load_tile<HD, NT>(qs, qkv, ld, tok0, q0, S, h * HD, tid);
+  if (NB == 2) fetch(0, 0);
   cp_async_commit();
 
   float oacc[NO][4];
 #pragma unroll
   for (int i = 0; i < NO; ++i) oacc[i][0] = oacc[i][1] = oacc[i][2] = oacc[i][3] = 0.0f;
   float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.0f, 0.0f};
-  const int ra = q0 + warp * 16 + (lane >> 2);
-  const int nkb = min((q0 + BQ - 1) / BKV + 1, (S + BKV - 1) / BKV);
+  const int ra = q0 + wr * 16 + (lane >> 2);
 
-  for (int kb = kb0; kb < nkb; ++kb) {
-    const int k0 = kb * BKV, buf = NB == 2 ? (kb - kb0) & 1 : 0;
+  for (int t = 0; t < nrounds; ++t) {
+    const int buf = NB == 2 ? t & 1 : 0;
     if (NB == 1) {
-      load_tile<HD>(ks(0), qkv, ld, tok0, k0, S, (H + kvh) * HD, tid);
-      load_tile<HD>(vs(0), qkv, ld, tok0, k0, S, (H + KV + kvh) * HD, tid);
+      fetch(t, 0);
       cp_async_commit();
       cp_async_wait<0>();
-    } else if (kb + 1 < nkb) {
-      load_tile<HD>(ks(buf ^ 1), qkv, ld, tok0, k0 + BKV, S, (H + kvh) * HD, tid);
-      load_tile<HD>(vs(buf ^ 1), qkv, ld, tok0, k0 + BKV, S, (H + KV + kvh) * HD, tid);
+    } else if (t + 1 < nrounds) {
+      fetch(t + 1, buf ^ 1);
       cp_async_commit();
       cp_async_wait<1>();
     } else {
       cp_async_wait<0>();
     }
     __syncthreads();
-
-    float s[8][4];
-    qk_tile<HD>(s, smem_u32(qs), smem_u32(ks(buf)), warp, lane);
+    const int kb = kb_first + t * NWG + wg;
+    if (kb <= qb) {  // uniform over the warp-group
+      const int k0 = kb * BKV;
+      float s[8][4];
+      qk_tile<HD>(s, smem_u32(qs), smem_u32(ks(buf, wg)), wr, lane);
 #pragma unroll
-    for (int nt = 0; nt < 8; ++nt)
+      for (int nt = 0; nt < 8; ++nt)
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int col = k0 + nt * 8 + 2 * (lane & 3) + (e & 1);
-        const int row = ra + ((e >> 1) << 3);
-        s[nt][e] = (col > row || col >= S || (WIN && row - col >= W)) ? -INFINITY : s[nt][e] * sc;
+        for (int e = 0; e < 4; ++e) {
+          const int col = k0 + nt * 8 + 2 * (lane & 3) + (e & 1);
+          const int row = ra + ((e >> 1) << 3);
+          s[nt][e] = (col > row || col >= S || (WIN && row - col >= W)) ? -INFINITY : s[nt][e] * sc;
+        }
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        float mx = -INFINITY;
+#pragma unroll
+        for (int nt = 0; nt < 8; ++nt) mx = fmaxf(mx, fmaxf(s[nt][2 * i], s[nt][2 * i + 1]));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+        const float mnew = fmaxf(mrow[i], mx);
+        const float alpha = (mnew == -INFINITY) ? 1.0f : exp2f(mrow[i] - mnew);
+        float rs = 0.0f;
+#pragma unroll
+        for (int nt = 0; nt < 8; ++nt) {
+          const float p0 = (mnew == -INFINITY) ? 0.0f : exp2f(s[nt][2 * i] - mnew);
+          const float p1 = (mnew == -INFINITY) ? 0.0f : exp2f(s[nt][2 * i + 1] - mnew);
+          s[nt][2 * i] = p0;
+          s[nt][2 * i + 1] = p1;
+          rs += p0 + p1;
+        }
+        rs += __shfl_xor_sync(0xffffffffu, rs, 1);
+        rs += __shfl_xor_sync(0xffffffffu, rs, 2);
+        lrow[i] = lrow[i] * alpha + rs;
+        mrow[i] = mnew;
+#pragma unroll
+        for (int dt = 0; dt < NO; ++dt) {
+          oacc[dt][2 * i] *= alpha;
+          oacc[dt][2 * i + 1] *= alpha;
+        }
       }
-#pragma unroll
-    for (int i = 0; i < 2; ++i) {
-      float mx = -INFINITY;
-#pragma unroll
-      for (int nt = 0; nt < 8; ++nt) mx = fmaxf(mx, fmaxf(s[nt][2 * i], s[nt][2 * i + 1]));
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-      const float mnew = fmaxf(mrow[i], mx);
-      const float alpha = (mnew == -INFINITY) ? 1.0f : exp2f(mrow[i] - mnew);
-      float rs = 0.0f;
-#pragma unroll
-      for (int nt = 0; nt < 8; ++nt) {
-        const float p0 = (mnew == -INFINITY) ? 0.0f : exp2f(s[nt][2 * i] - mnew);
-        const float p1 = (mnew == -INFINITY) ? 0.0f : exp2f(s[nt][2 * i + 1] - mnew);
-        s[nt][2 * i] = p0;
-        s[nt][2 * i + 1] = p1;
-        rs += p0 + p1;
-      }
-      rs += __shfl_xor_sync(0xffffffffu, rs, 1);
-      rs += __shfl_xor_sync(0xffffffffu, rs, 2);
-      lrow[i] = lrow[i] * alpha + rs;
-      mrow[i] = mnew;
-#pragma unroll
-      for (int dt = 0; dt < NO; ++dt) {
-        oacc[dt][2 * i] *= alpha;
-        oacc[dt][2 * i + 1] *= alpha;
-      }
+      pv_tile<HD, NO>(oacc, s, smem_u32(vs(buf, wg)), 0, lane);
     }
-    pv_tile<HD, NO>(oacc, s, smem_u32(vs(buf)), 0, lane);
-    __syncthreads();  // every warp is done with this buffer before it is refilled
+    __syncthreads();  // every warp is done with this slot before it is refilled
   }
 
   const int c = 2 * (lane & 3);
+  if constexpr (NWG > 1) {
+    // groups 1 .. NWG-1 park (o, m, l) in the idle tile buffers; group 0 merges them in group
+    // order and writes
+    constexpr int LDO = HD + 4, PART = 64 * LDO + 128;  // floats per parked group
+    static_assert((NWG - 1) * PART * 4 <= (1 + 2 * NB * NWG) * TILE * 2, "merge buffers fit");
+    float* park = reinterpret_cast<float*>(sm);
+    if (wg > 0) {
+      float* op = park + (wg - 1) * PART;
+      float2* ml = reinterpret_cast<float2*>(op + 64 * LDO);
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        const int rl = wr * 16 + (lane >> 2) + 8 * i;
+#pragma unroll
+        for (int dt = 0; dt < NO; ++dt)
+          *reinterpret_cast<float2*>(op + rl * LDO + dt * 8 + c) = make_float2(oacc[dt][2 * i], oacc[dt][2 * i + 1]);
+        if ((lane & 3) == 0) ml[rl] = make_float2(mrow[i], lrow[i]);
+      }
+    }
+    __syncthreads();
+    if (wg > 0) return;
+#pragma unroll
+    for (int g = 1; g < NWG; ++g) {
+      const float* op = park + (g - 1) * PART;
+      const float2* ml = reinterpret_cast<const float2*>(op + 64 * LDO);
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        const int rl = wr * 16 + (lane >> 2) + 8 * i;
+        const float2 p = ml[rl];
+        const float M = fmaxf(mrow[i], p.x);
+        const float a0 = mrow[i] == -INFINITY ? 0.0f : exp2f(mrow[i] - M);
+        const float a1 = p.x == -INFINITY ? 0.0f : exp2f(p.x - M);
+        lrow[i] = a0 * lrow[i] + a1 * p.y;
+        mrow[i] = M;
+#pragma unroll
+        for (int dt = 0; dt < NO; ++dt) {
+          const float2 q = *reinterpret_cast<const float2*>(op + rl * LDO + dt * 8 + c);
+          oacc[dt][2 * i] = a0 * oacc[dt][2 * i] + a1 * q.x;
+          oacc[dt][2 * i + 1] = a0 * oacc[dt][2 * i + 1] + a1 * q.y;
+        }
+      }
+    }
+  }
 #pragma unroll
   for (int i = 0; i < 2; ++i) {
     const int row = ra + 8 * i;
@@ -500,33 +557,43 @@ __global__ void __launch_bounds__(128, 1) dq_kernel(const BwdArgs a) {
   dq_item<HD, DC, WIN>(a, blockIdx.x, sm);
 }
 
-template <int HD, int NB, bool WIN>
-void fwd_launch_nb(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uint16_t* o, int64_t ldo, float* lse,
-                   int W, cudaStream_t st) {
-  constexpr int smem = (1 + 2 * NB) * 64 * (HD + 8) * 2;  // Q, NB x (K, V)
+template <int HD, int NB, bool WIN, int NWG>
+void fwd_launch_g(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uint16_t* o, int64_t ldo, float* lse,
+                  int W, cudaStream_t st) {
+  constexpr int smem = (1 + 2 * NB * NWG) * 64 * (HD + 8) * 2;  // Q, NB x NWG x (K, V)
+  static_assert(smem <= 232448, "attention forward shared memory");
   static bool init = false;
   if (!init) {
-    cudaFuncSetAttribute(fwd_kernel<HD, NB, WIN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(fwd_kernel<HD, NB, WIN, NWG>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     init = true;
   }
   dim3 grid((S + BQ - 1) / BQ, H, B);
-  launch_k(fwd_kernel<HD, NB, WIN>, grid, 128, smem, st, qkv, ld, S, H, KV, o, ldo, lse, W);
+  launch_k(fwd_kernel<HD, NB, WIN, NWG>, grid, 128 * NWG, smem, st, qkv, ld, S, H, KV, o, ldo, lse, W);
 }
 
-// Double-buffered key/value loads, except at head_dim 256 with more than two waves of CTAs: there
-// the single-buffered kernel fits two CTAs per SM, which hides the loads better.
+// Grids of at most one CTA per SM: several warp-groups per CTA — four at head_dim 64 when the
+// sequence has at least four query blocks (512 threads, 128 registers each), else two
+// (single-buffered at head_dim 256, for shared memory).  Measured at 512 tokens, 14 heads, hd 64:
+// 16.5 us with one group, 11.9 with two, 9.8 with four.  Larger grids: one group, double-buffered,
+// except at head_dim 256 with more than two waves, where the single-buffered kernel fits two CTAs
+// per SM and hides the loads better.
+template <int HD, bool WIN>
+void fwd_launch_w(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uint16_t* o, int64_t ldo, float* lse,
+                  int W, cudaStream_t st) {
+  const int nqb = (S + BQ - 1) / BQ;
+  const int64_t ctas = static_cast<int64_t>(nqb) * H * B;
+  if constexpr (HD == 64) {
+    if (ctas <= 152 && nqb >= 4) return fwd_launch_g<HD, 2, WIN, 4>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
+  }
+  if (ctas <= 152 && nqb > 1) fwd_launch_g<HD, HD == 256 ? 1 : 2, WIN, 2>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
+  else if (HD == 256 && ctas > 2 * 152) fwd_launch_g<HD, 1, WIN, 1>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
+  else fwd_launch_g<HD, 2, WIN, 1>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
+}
 template <int HD>
 void fwd_launch(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uint16_t* o, int64_t ldo, float* lse,
                 int W, cudaStream_t st) {
-  const int64_t ctas = static_cast<int64_t>((S + BQ - 1) / BQ) * H * B;
-  const bool nb1 = HD == 256 && ctas > 2 * 152;
-  if (W > 0) {
-    if (nb1) fwd_launch_nb<HD, 1, true>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
-    else fwd_launch_nb<HD, 2, true>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
-  } else {
-    if (nb1) fwd_launch_nb<HD, 1, false>(qkv, ld, B, S, H, KV, o, ldo, lse, 0, st);
-    else fwd_launch_nb<HD, 2, false>(qkv, ld, B, S, H, KV, o, ldo, lse, 0, st);
-  }
+  if (W > 0) fwd_launch_w<HD, true>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
+  else fwd_launch_w<HD, false>(qkv, ld, B, S, H, KV, o, ldo, lse, 0, st);
 }
 
 template <int HD, int DC, bool WIN>
