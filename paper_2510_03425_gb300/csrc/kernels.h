@@ -167,6 +167,25 @@ int launch_tall_reduce(const uint16_t* P, int64_t ldp, const uint16_t* Q, int64_
                        float* C, int64_t ldc, bool accumulate, const float* mult, float* scratch,
                        int64_t scratch_floats, cudaStream_t st);
 int64_t tall_reduce_scratch_floats(int64_t M, int Pw, int Qw);
+// Up to kTallMaxProbs single-pass reductions C (+)= mult * P^T Q over the same M rows in one launch
+// (Qw <= 32, Pw and Qw multiples of 8).  tall_batch_add returns false for a problem it cannot take.
+constexpr int kTallMaxProbs = 16;
+struct TallProb {
+  const uint16_t* P;
+  const uint16_t* Q;
+  float* C;
+  int64_t ldp, ldq, sp, sq;
+  int Pw, Qw, acc, ctas;
+};
+struct TallBatch {
+  TallProb p[kTallMaxProbs];
+  int n = 0;
+  int64_t M = 0;
+  const float* mult = nullptr;
+};
+bool tall_batch_add(TallBatch& b, const uint16_t* P, int64_t ldp, const uint16_t* Q, int64_t ldq, int Pw, int Qw,
+                    float* C, int64_t ldc, bool accumulate);
+void launch_tall_reduce_batched(const TallBatch& b, cudaStream_t st);
 // fp16 shadows of the LoRA masters, see lora.cu.
 // fp16 LoRA shadows of n_layers layers at once: target t of layer l reads A[3 l + t], B[3 l + t];
 // layer l's outputs start at l * stride_a (A_cat) and l * stride_b (B_cat, Bt_cat).

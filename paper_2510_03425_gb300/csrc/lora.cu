@@ -308,6 +308,107 @@ int launch_tall_reduce(const uint16_t* P, int64_t ldp, const uint16_t* Q, int64_
   return MEBP_OK;
 }
 
+// Several single-pass reductions in one launch (the LoRA gradients of a block at short token
+// counts, where each alone is a handful of CTAs): CTA -> (problem, 64-row block of its output).
+// Three-stage cp.async pipeline over the token axis; C (+)= mult * sum, written directly.
+__global__ void __launch_bounds__(128) tall_reduce_batched_kernel(const TallBatch b) {
+  griddep_wait();
+  griddep_launch();
+  constexpr int NQ = 4, BP = 64, BMr = 64, QT = NQ * 8, LDP = BP + 8, LDQ = QT + 8, NS = 3;
+  __shared__ __align__(16) uint16_t ps[NS][BMr * LDP];
+  __shared__ __align__(16) uint16_t qs[NS][BMr * LDQ];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  // this CTA's problem (fields read with compile-time indices: no local-memory copy)
+  int idx = blockIdx.x, pi = 0;
+#pragma unroll
+  for (int i = 0; i < kTallMaxProbs; ++i)
+    if (i < b.n && pi == i && idx >= b.p[i].ctas) {
+      idx -= b.p[i].ctas;
+      pi = i + 1;
+    }
+  TallProb pr;
+#pragma unroll
+  for (int i = 0; i < kTallMaxProbs; ++i)
+    if (i == pi) pr = b.p[i];
+  const int Pw = pr.Pw, Qw = pr.Qw;
+  const int p0 = idx * BP;
+  const int64_t M = b.M;
+  float acc[NQ][4];
+#pragma unroll
+  for (int i = 0; i < NQ; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.0f;
+  auto load = [&](int stage, int64_t m) {
+    for (int c = tid; c < BMr * 8; c += 128) {
+      const int r = c >> 3, cc = c & 7;
+      const bool v = (m + r < M) && (p0 + cc * 8 < Pw);
+      const uint16_t* src = v ? pr.P + (m + r) * pr.ldp + p0 + cc * 8 : pr.P;
+      cp_async16(smem_u32(&ps[stage][r * LDP + cc * 8]), src, v);
+    }
+    for (int c = tid; c < BMr * NQ; c += 128) {
+      const int r = c / NQ, cc = c % NQ;
+      const bool v = (m + r < M) && (cc * 8 < Qw);
+      const uint16_t* src = v ? pr.Q + (m + r) * pr.ldq + cc * 8 : pr.Q;
+      cp_async16(smem_u32(&qs[stage][r * LDQ + cc * 8]), src, v);
+    }
+  };
+  const int64_t ntile = (M + BMr - 1) / BMr;
+#pragma unroll
+  for (int st = 0; st < NS - 1; ++st) {
+    if (st < ntile) load(st, st * BMr);
+    cp_async_commit();
+  }
+  for (int64_t it = 0; it < ntile; ++it) {
+    if (it + NS - 1 < ntile) load(static_cast<int>((it + NS - 1) % NS), (it + NS - 1) * BMr);
+    cp_async_commit();
+    cp_async_wait<NS - 1>();
+    __syncthreads();
+    const int s = static_cast<int>(it % NS);
+    const uint32_t pb = smem_u32(ps[s]), qb = smem_u32(qs[s]);
+#pragma unroll
+    for (int kk = 0; kk < BMr; kk += 16) {
+      uint32_t a[4];
+      ldsm_x4_t(a, frag_at_addr(pb, LDP, warp * 16, kk, lane));
+#pragma unroll
+      for (int nq = 0; nq < NQ; nq += 2) {
+        uint32_t bb[4];
+        ldsm_x4_t(bb, frag_bk_addr(qb, LDQ, nq * 8, kk, lane));
+        mma16816(acc[nq], a, bb[0], bb[1]);
+        mma16816(acc[nq + 1], a, bb[2], bb[3]);
+      }
+    }
+    __syncthreads();
+  }
+  const float mu = b.mult ? *b.mult : 1.0f;
+  const int r = lane >> 2, c = (lane & 3) * 2;
+  const int prow = p0 + warp * 16 + r;
+#pragma unroll
+  for (int nq = 0; nq < NQ; ++nq)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int pp = prow + ((e >> 1) << 3), qq = nq * 8 + c + (e & 1);
+      if (pp >= Pw || qq >= Qw) continue;
+      float* dst = pr.C + pp * pr.sp + qq * pr.sq;
+      *dst = pr.acc ? *dst + mu * acc[nq][e] : mu * acc[nq][e];
+    }
+}
+
+bool tall_batch_add(TallBatch& b, const uint16_t* P, int64_t ldp, const uint16_t* Q, int64_t ldq, int Pw, int Qw,
+                    float* C, int64_t ldc, bool accumulate) {
+  if (b.n >= kTallMaxProbs || Pw <= 0 || Qw <= 0 || Qw > 32 || (Pw % 8) || (Qw % 8)) return false;
+  TallProb& p = b.p[b.n++];
+  p.P = P; p.ldp = ldp; p.Q = Q; p.ldq = ldq; p.Pw = Pw; p.Qw = Qw; p.C = C;
+  p.sp = ldc > 0 ? ldc : 1;
+  p.sq = ldc > 0 ? 1 : -ldc;
+  p.acc = accumulate ? 1 : 0;
+  p.ctas = (Pw + 63) / 64;
+  return true;
+}
+
+void launch_tall_reduce_batched(const TallBatch& b, cudaStream_t st) {
+  int ctas = 0;
+  for (int i = 0; i < b.n; ++i) ctas += b.p[i].ctas;
+  if (ctas > 0) launch_k(tall_reduce_batched_kernel, static_cast<unsigned>(ctas), 128, 0, st, b);
+}
+
 // ------------------------------------------------------------------------------------ shadows
 // Per-layer LoRA masters of one fused linear (up to 3 targets side by side).
 struct ShadowTable {

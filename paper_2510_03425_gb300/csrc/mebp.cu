@@ -381,20 +381,28 @@ int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, 
   return cuda_check(c, "block forward");
 }
 
+// Token counts below this run a block's LoRA-gradient reductions as one batched launch (each is a
+// single pass over the tokens there); larger ones launch each reduction with its token split.
+constexpr int64_t kTallBatchMaxT = 2048;
+
 // LoRA gradients of one fused linear: dB_t = dY[:, rows_t]^T U_s[:, ranks_t], dA_t = dU[:, ranks_t]^T X.
+// With tb the reductions are queued in the batch (launched by the caller) where it can take them.
 int lin_grads(mebp_ctx* c, const Acts& A, const uint16_t* du, int li, const uint16_t* dY, int64_t ldy,
               const uint16_t* X, int64_t ldx, int64_t T, const mebp_lora_grads* grads, bool acc,
-              const float* grad_mult, cudaStream_t st) {
+              const float* grad_mult, cudaStream_t st, TallBatch* tb = nullptr) {
   const Lin& l = c->lin[li];
   for (int t = 0; t < l.nt; ++t) {
     const int tg = l.tgt[t];
     if (!grads) break;
-    if (grads->dB[tg]) {
+    if (grads->dB[tg] &&
+        !(tb && tall_batch_add(*tb, dY + l.no[t], ldy, A.us[li] + l.ro[t], l.kxp, l.nl[t], c->r, grads->dB[tg], c->r,
+                               acc))) {
       const int rc = launch_tall_reduce(dY + l.no[t], ldy, A.us[li] + l.ro[t], l.kxp, T, l.nl[t], c->r, grads->dB[tg],
                                         c->r, acc, grad_mult, c->red, c->red_floats, st);
       if (rc) return fail(c, rc, "LoRA dB reduction");
     }
-    if (grads->dA[tg]) {
+    if (grads->dA[tg] &&
+        !(tb && tall_batch_add(*tb, X, ldx, du + l.ro[t], l.kxp, l.K, c->r, grads->dA[tg], -l.K, acc))) {
       const int rc = launch_tall_reduce(X, ldx, du + l.ro[t], l.kxp, T, l.K, c->r, grads->dA[tg], -l.K, acc,
                                         grad_mult, c->red, c->red_floats, st);
       if (rc) return fail(c, rc, "LoRA dA reduction");
@@ -418,6 +426,10 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   const int64_t T = static_cast<int64_t>(B) * Sq;
   const int D = c->D, I = c->I;
   int rc;
+  TallBatch batch;
+  batch.M = T;
+  batch.mult = grad_mult;
+  TallBatch* tb = T < kTallBatchMaxT ? &batch : nullptr;
   if (!(A.layer == layer && A.x == x && A.T == T)) {
     if ((rc = block_forward(c, set, layer, w, lora, x, nullptr, B, Sq, false, st, sh))) return rc;
   }
@@ -436,7 +448,7 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   }
   g.epi = EPI_F32; g.C = c->dm; g.ldc = I;
   if ((rc = run_gemm(c, g, st, "down dX"))) return rc;
-  if ((rc = lin_grads(c, A, du[LIN_DOWN], LIN_DOWN, ddn_h, D, A.m, I, T, grads, acc, grad_mult, st))) return rc;
+  if ((rc = lin_grads(c, A, du[LIN_DOWN], LIN_DOWN, ddn_h, D, A.m, I, T, grads, acc, grad_mult, st, tb))) return rc;
   // ---- gated MLP
   launch_glu_bwd(c->dm, A.gu, T, I, c->cfg.act, G.dgu, st);
   const Lin& lg = c->lin[LIN_GU];
@@ -447,7 +459,7 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   }
   g.epi = EPI_F32; g.C = c->dtmp; g.ldc = D;
   if ((rc = run_gemm(c, g, st, "gate_up dX"))) return rc;
-  if ((rc = lin_grads(c, A, du[LIN_GU], LIN_GU, G.dgu, 2 * I, A.b, D, T, grads, acc, grad_mult, st))) return rc;
+  if ((rc = lin_grads(c, A, du[LIN_GU], LIN_GU, G.dgu, 2 * I, A.b, D, T, grads, acc, grad_mult, st, tb))) return rc;
   // dh1 = dy + RMSNorm2^T(db); the o projection's output gradient is dh1 (fp16 copy in dh1_h), for
   // Gemma3 the post-attention norm's VJP of it
   if (c->gemma) {
@@ -465,7 +477,7 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   }
   g.epi = EPI_F16; g.C = c->dout; g.ldc = c->Na;
   if ((rc = run_gemm(c, g, st, "o dX"))) return rc;
-  if ((rc = lin_grads(c, A, du[LIN_O], LIN_O, G.dh1_h, D, A.o, c->Na, T, grads, acc, grad_mult, st))) return rc;
+  if ((rc = lin_grads(c, A, du[LIN_O], LIN_O, G.dh1_h, D, A.o, c->Na, T, grads, acc, grad_mult, st, tb))) return rc;
   // ---- attention, RoPE
   const Lin& lq = c->lin[LIN_QKV];
   launch_attn_bwd(A.qkv, lq.N, A.o, c->dout, c->Na, A.lse_attn, B, Sq, c->H, c->KV, c->hd, c->dvec, G.dqkv,
@@ -478,7 +490,7 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   // ---- q, k, v projections
   if (lq.kx)
     launch_skinny_gemm(G.dqkv, lq.N, T, lq.N, A.sh->Bt_cat[LIN_QKV], lq.N, lq.kx, c->s, du[LIN_QKV], lq.kxp, st);
-  if ((rc = lin_grads(c, A, du[LIN_QKV], LIN_QKV, G.dqkv, lq.N, A.a, D, T, grads, acc, grad_mult, st))) return rc;
+  if ((rc = lin_grads(c, A, du[LIN_QKV], LIN_QKV, G.dqkv, lq.N, A.a, D, T, grads, acc, grad_mult, st, tb))) return rc;
   if (dx) {
     g = gemm_dx(G.dqkv, lq.N, T, w->qkv);
     if (lq.kx) {
@@ -488,6 +500,7 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
     if ((rc = run_gemm(c, g, st, "qkv dX"))) return rc;
     launch_rmsnorm_bwd(c->dtmp, x, w->norm1, A.r1, c->dh1, T, D, dx_mult, dx, dx_h, st);
   }
+  if (batch.n) launch_tall_reduce_batched(batch, st);
   return cuda_check(c, "block backward");
 }
 
@@ -499,11 +512,19 @@ int block_lora_grads(mebp_ctx* c, int set, int bset, const uint16_t* dy_h, int64
   const Grads2& G = c->bw[bset];
   const int D = c->D, I = c->I;
   int rc;
+  TallBatch batch;
+  batch.M = T;
+  batch.mult = grad_mult;
+  TallBatch* tb = T < kTallBatchMaxT ? &batch : nullptr;
   const uint16_t* ddn_h = c->gemma ? G.ddn_h : dy_h;
-  if ((rc = lin_grads(c, A, G.du[LIN_DOWN], LIN_DOWN, ddn_h, D, A.m, I, T, grads, acc, grad_mult, st))) return rc;
-  if ((rc = lin_grads(c, A, G.du[LIN_GU], LIN_GU, G.dgu, 2 * I, A.b, D, T, grads, acc, grad_mult, st))) return rc;
-  if ((rc = lin_grads(c, A, G.du[LIN_O], LIN_O, G.dh1_h, D, A.o, c->Na, T, grads, acc, grad_mult, st))) return rc;
-  return lin_grads(c, A, G.du[LIN_QKV], LIN_QKV, G.dqkv, c->lin[LIN_QKV].N, A.a, D, T, grads, acc, grad_mult, st);
+  if ((rc = lin_grads(c, A, G.du[LIN_DOWN], LIN_DOWN, ddn_h, D, A.m, I, T, grads, acc, grad_mult, st, tb))) return rc;
+  if ((rc = lin_grads(c, A, G.du[LIN_GU], LIN_GU, G.dgu, 2 * I, A.b, D, T, grads, acc, grad_mult, st, tb))) return rc;
+  if ((rc = lin_grads(c, A, G.du[LIN_O], LIN_O, G.dh1_h, D, A.o, c->Na, T, grads, acc, grad_mult, st, tb))) return rc;
+  if ((rc = lin_grads(c, A, G.du[LIN_QKV], LIN_QKV, G.dqkv, c->lin[LIN_QKV].N, A.a, D, T, grads, acc, grad_mult, st,
+                      tb)))
+    return rc;
+  if (batch.n) launch_tall_reduce_batched(batch, st);
+  return MEBP_OK;
 }
 
 // Final RMSNorm + LM head + CE.  dh (fp32) is the true gradient when unscale_dh, else it is
