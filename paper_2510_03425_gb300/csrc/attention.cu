@@ -7,11 +7,11 @@
 //             layers of Gemma3), i - j < W; key blocks wholly outside the window are skipped.
 //   backward: dP = dO v^T, dS = P (dP - rowsum(dO o)), dq = dS k / sqrt(hd),
 //             dk = dS^T q / sqrt(hd), dv = P^T dO; dk, dv summed over the query heads of a
-//             group.  P is recomputed from q, k and lse.  One launch holds two kinds of work
-//             item: dk/dv (one CTA per key block and query head; the query heads of a kv head
-//             form a thread-block cluster that sums their partials over distributed shared
-//             memory) and dq (one CTA per query block and head), so every output element is
-//             written exactly once (deterministic, no atomics).
+//             group.  P is recomputed from q, k and lse.  Large grids: dk/dv items (key block,
+//             kv head, looping over the group's query heads) and dq items (query block, head)
+//             write dqkv directly.  Small grids: dk/dv items per query head and dq items, each
+//             cut into interleaved parts, write fp32 partials; a finish kernel sums them in a
+//             fixed order (and applies the inverse RoPE).  Deterministic, no atomics.
 // q, k, v live in the fused projection buffer [T, (H + 2 KV) hd] (q heads, k heads, v heads);
 // token t = b*S + s.
 #include "kernels.h"
@@ -277,30 +277,23 @@ struct BwdArgs {
   const float* lse;
   const float* dvec;
   int S, H, KV, B;
-  int W;     // sliding window (0 = none)
-  int n_kv;  // dK/dV work items (blocks [0, n_kv)); dQ items follow
+  int W;  // sliding window (0 = none)
   uint16_t* dqkv;
+  // split mode: every item cut into P parts, fp32 partials [slot][64][HD] (slots of dK, dV: (b, key
+  // block, query head, part); of dQ: (b, query block, head, part))
+  int P = 1;
+  float *wk = nullptr, *wv = nullptr, *wq = nullptr;
 };
 
-// dK, dV of one key block kb (output columns d0 .. d0 + DC), accumulated over the query blocks
-// kb .. that see the block.  Every dK/dV element is written once (no atomics, deterministic):
-//   CL = true : one item per query head h; the grp = H/KV query heads of a kv head form one
-//               thread-block cluster (rank j = head kvh*grp + j) whose fp32 partials are summed
-//               over distributed shared memory in head order (small grids);
-//   CL = false: one item per kv head, looping over its grp query heads (large grids).
-template <int HD, int DC, bool CL, bool WIN>
-__device__ __forceinline__ void dkdv_item(const BwdArgs& a, int idx, uint16_t* sm) {
-  constexpr int LD = HD + 8, NC = DC / 8, NCH = HD / DC;
+// dK, dV of key block kb, output columns d0 .. d0 + DC, accumulated over the (head, query block)
+// pairs that see the block — heads h_first .. h_first + h_count - 1, query blocks kb .. — taking
+// pairs it0, it0 + dit, ... of that list.  PART: write the fp32 sums (dK already scaled by
+// 1/sqrt(hd)) to pk / pv [64][HD]; else write fp16 into dqkv.
+template <int HD, int DC, bool PART, bool WIN>
+__device__ __forceinline__ void dkdv_run(const BwdArgs& a, int b, int kb, int kvh, int h_first, int h_count, int d0,
+                                         int it0, int dit, float* pk, float* pv, uint16_t* sm) {
+  constexpr int LD = HD + 8, NC = DC / 8;
   const int S = a.S, H = a.H, KV = a.KV;
-  const int grp = H / KV;
-  const int j = CL ? idx % grp : 0;
-  int rest = CL ? idx / grp : idx;
-  const int kvh = rest % KV;
-  rest /= KV;
-  const int nkb = (S + BKV - 1) / BKV;
-  const int kb = rest % nkb, bz = rest / nkb;
-  const int b = bz / NCH, d0 = (bz % NCH) * DC;
-  const int h_first = kvh * grp + j, h_count = CL ? 1 : grp;
   uint16_t* ks = sm;
   uint16_t* vs = ks + BKV * LD;
   // two (Q, dO, lse, dvec) buffers: the next query block loads while this one is used
@@ -324,28 +317,33 @@ __device__ __forceinline__ void dkdv_item(const BwdArgs& a, int idx, uint16_t* s
   // query blocks kb .. qb_end-1 see this key block (with a window, queries < k0 + BKV - 1 + W)
   const int qb_end = WIN ? min(nqb, (k0 + BKV - 1 + a.W - 1) / BQ + 1) : nqb;
   const int per_head = qb_end - kb;
-  const int n_it = h_count * per_head;
-  auto fetch = [&](int it, int buf) {
+  const int n_all = h_count * per_head;
+  const int n_it = it0 < n_all ? (n_all - it0 + dit - 1) / dit : 0;
+  auto fetch = [&](int i, int buf) {
+    const int it = it0 + i * dit;
     const int h = h_first + it / per_head, q0 = (kb + it % per_head) * BQ;
     load_tile<HD>(qs(buf), a.qkv, a.ld, tok0, q0, S, h * HD, tid);
     load_tile<HD>(dos(buf), a.dout, a.ldo, tok0, q0, S, h * HD, tid);
-    for (int i = tid; i < BQ; i += 128) {
-      const int q = q0 + i;
+    for (int r = tid; r < BQ; r += 128) {
+      const int q = q0 + r;
       const int64_t li = (static_cast<int64_t>(b) * H + h) * S + q;
-      lse_s(buf)[i] = q < S ? a.lse[li] * kLog2e : 0.0f;
-      dv_s(buf)[i] = q < S ? a.dvec[li] : 0.0f;
+      lse_s(buf)[r] = q < S ? a.lse[li] * kLog2e : 0.0f;
+      dv_s(buf)[r] = q < S ? a.dvec[li] : 0.0f;
     }
   };
-  load_tile<HD>(ks, a.qkv, a.ld, tok0, k0, S, (H + kvh) * HD, tid);
-  load_tile<HD>(vs, a.qkv, a.ld, tok0, k0, S, (H + KV + kvh) * HD, tid);
-  if (n_it > 0) fetch(0, 0);
+  if (n_it > 0) {
+    load_tile<HD>(ks, a.qkv, a.ld, tok0, k0, S, (H + kvh) * HD, tid);
+    load_tile<HD>(vs, a.qkv, a.ld, tok0, k0, S, (H + KV + kvh) * HD, tid);
+    fetch(0, 0);
+  }
   cp_async_commit();
 
-  for (int it = 0; it < n_it; ++it) {
-    const int buf = it & 1;
+  for (int i = 0; i < n_it; ++i) {
+    const int buf = i & 1;
+    const int it = it0 + i * dit;
     const int q0 = (kb + it % per_head) * BQ;
-    if (it + 1 < n_it) {
-      fetch(it + 1, buf ^ 1);
+    if (i + 1 < n_it) {
+      fetch(i + 1, buf ^ 1);
       cp_async_commit();
       cp_async_wait<1>();
     } else {
@@ -386,10 +384,18 @@ __device__ __forceinline__ void dkdv_item(const BwdArgs& a, int idx, uint16_t* s
 
   const float inv = rsqrtf(static_cast<float>(HD));
   const int c = 2 * (lane & 3);
-  if (!CL || grp == 1) {
 #pragma unroll
-    for (int i = 0; i < 2; ++i) {
-      const int key = key_a + 8 * i;
+  for (int i = 0; i < 2; ++i) {
+    const int kr = warp * 16 + (lane >> 2) + 8 * i;
+    if (PART) {
+#pragma unroll
+      for (int dt = 0; dt < NC; ++dt) {
+        __stcg(reinterpret_cast<float2*>(pk + kr * HD + d0 + dt * 8 + c),
+               make_float2(dk[dt][2 * i] * inv, dk[dt][2 * i + 1] * inv));
+        __stcg(reinterpret_cast<float2*>(pv + kr * HD + d0 + dt * 8 + c), make_float2(dv[dt][2 * i], dv[dt][2 * i + 1]));
+      }
+    } else {
+      const int key = k0 + kr;
       if (key >= S) continue;
       uint16_t* krow = a.dqkv + (tok0 + key) * a.ld + (H + kvh) * HD + d0;
       uint16_t* vrow = a.dqkv + (tok0 + key) * a.ld + (H + KV + kvh) * HD + d0;
@@ -399,61 +405,16 @@ __device__ __forceinline__ void dkdv_item(const BwdArgs& a, int idx, uint16_t* s
         *reinterpret_cast<uint32_t*>(vrow + dt * 8 + c) = pack_half2(dv[dt][2 * i], dv[dt][2 * i + 1]);
       }
     }
-    return;
   }
-  // partials [64 keys][DC] for dK then dV, fp32, in the idle tile buffers
-  constexpr int LDP = DC + 4;
-  static_assert(2 * BKV * LDP * 4 <= 6 * 64 * LD * 2, "partials fit in the tile buffers");
-  float* pk = reinterpret_cast<float*>(sm);
-  float* pv = pk + BKV * LDP;
-#pragma unroll
-  for (int i = 0; i < 2; ++i) {
-    const int kr = warp * 16 + (lane >> 2) + 8 * i;
-#pragma unroll
-    for (int dt = 0; dt < NC; ++dt) {
-      *reinterpret_cast<float2*>(pk + kr * LDP + dt * 8 + c) = make_float2(dk[dt][2 * i], dk[dt][2 * i + 1]);
-      *reinterpret_cast<float2*>(pv + kr * LDP + dt * 8 + c) = make_float2(dv[dt][2 * i], dv[dt][2 * i + 1]);
-    }
-  }
-  cluster_sync_all();
-  const int rpc = (BKV + grp - 1) / grp;
-  const int r0 = j * rpc, r1 = min(BKV, r0 + rpc);
-  constexpr int C4 = DC / 4;
-  const uint32_t base = smem_u32(sm);
-  for (int i = tid; i < 2 * (r1 - r0) * C4; i += 128) {
-    const int which = i / ((r1 - r0) * C4);  // 0: dK, 1: dV
-    const int e = i % ((r1 - r0) * C4);
-    const int kr = r0 + e / C4, cc = (e % C4) * 4;
-    const int key = k0 + kr;
-    if (key >= S) continue;
-    const uint32_t off = base + ((which * BKV + kr) * LDP + cc) * 4;
-    float4 v[8];
-#pragma unroll
-    for (int t = 0; t < 8; ++t)
-      if (t < grp) v[t] = ld_dsmem_f4(dsmem_addr(off, t));
-    float4 sum = v[0];
-#pragma unroll
-    for (int t = 1; t < 8; ++t)
-      if (t < grp) {
-        sum.x += v[t].x; sum.y += v[t].y; sum.z += v[t].z; sum.w += v[t].w;
-      }
-    const float m = which ? 1.0f : inv;
-    uint16_t* dst = a.dqkv + (tok0 + key) * a.ld + (H + which * KV + kvh) * HD + d0 + cc;
-    *reinterpret_cast<uint2*>(dst) = make_uint2(pack_half2(sum.x * m, sum.y * m), pack_half2(sum.z * m, sum.w * m));
-  }
-  cluster_sync_all();  // no CTA leaves while its partials are being read
 }
 
-// dQ for one query block of one head, output columns d0 .. d0 + DC.
-template <int HD, int DC, bool WIN>
-__device__ __forceinline__ void dq_item(const BwdArgs& a, int idx, uint16_t* sm) {
-  constexpr int LD = HD + 8, NC = DC / 8, NCH = HD / DC;
+// dQ of query block qb and head h, output columns d0 .. d0 + DC, from the key blocks kb_first + it0,
+// kb_first + it0 + dit, ... <= qb.  PART: fp32 (scaled by 1/sqrt(hd)) into pq [64][HD]; else fp16.
+template <int HD, int DC, bool PART, bool WIN>
+__device__ __forceinline__ void dq_run(const BwdArgs& a, int b, int qb, int h, int d0, int it0, int dit, float* pq,
+                                       uint16_t* sm) {
+  constexpr int LD = HD + 8, NC = DC / 8;
   const int S = a.S, H = a.H, KV = a.KV;
-  const int h = idx % H;
-  const int rest = idx / H;
-  const int nqb = (S + BQ - 1) / BQ;
-  const int qb = rest % nqb, bz = rest / nqb;
-  const int b = bz / NCH, d0 = (bz % NCH) * DC;
   uint16_t* qs = sm;
   uint16_t* dos = qs + BQ * LD;
   // two (K, V) buffers: the next key block loads while this one is used
@@ -464,12 +425,17 @@ __device__ __forceinline__ void dq_item(const BwdArgs& a, int idx, uint16_t* sm)
   const int64_t tok0 = static_cast<int64_t>(b) * S;
   const int q0 = qb * BQ;
   const float sc = kLog2e * rsqrtf(static_cast<float>(HD));
+  const int kb_first = WIN ? max(0, q0 - a.W + 1) / BKV : 0;  // first key block inside the window
+  const int n_all = qb - kb_first + 1;
+  const int n_it = it0 < n_all ? (n_all - it0 + dit - 1) / dit : 0;
 
-  const int kb0 = WIN ? max(0, q0 - a.W + 1) / BKV : 0;  // first key block inside the window
-  load_tile<HD>(qs, a.qkv, a.ld, tok0, q0, S, h * HD, tid);
-  load_tile<HD>(dos, a.dout, a.ldo, tok0, q0, S, h * HD, tid);
-  load_tile<HD>(ks(0), a.qkv, a.ld, tok0, kb0 * BKV, S, (H + kvh) * HD, tid);
-  load_tile<HD>(vs(0), a.qkv, a.ld, tok0, kb0 * BKV, S, (H + KV + kvh) * HD, tid);
+  if (n_it > 0) {
+    const int k0 = (kb_first + it0) * BKV;
+    load_tile<HD>(qs, a.qkv, a.ld, tok0, q0, S, h * HD, tid);
+    load_tile<HD>(dos, a.dout, a.ldo, tok0, q0, S, h * HD, tid);
+    load_tile<HD>(ks(0), a.qkv, a.ld, tok0, k0, S, (H + kvh) * HD, tid);
+    load_tile<HD>(vs(0), a.qkv, a.ld, tok0, k0, S, (H + KV + kvh) * HD, tid);
+  }
   cp_async_commit();
   const int ra = q0 + warp * 16 + (lane >> 2);
   float lse2[2], dvv[2];
@@ -484,11 +450,12 @@ __device__ __forceinline__ void dq_item(const BwdArgs& a, int idx, uint16_t* sm)
 #pragma unroll
   for (int i = 0; i < NC; ++i) dq[i][0] = dq[i][1] = dq[i][2] = dq[i][3] = 0.0f;
 
-  for (int kb = kb0; kb <= qb; ++kb) {
-    const int k0 = kb * BKV, buf = (kb - kb0) & 1;
-    if (kb < qb) {
-      load_tile<HD>(ks(buf ^ 1), a.qkv, a.ld, tok0, k0 + BKV, S, (H + kvh) * HD, tid);
-      load_tile<HD>(vs(buf ^ 1), a.qkv, a.ld, tok0, k0 + BKV, S, (H + KV + kvh) * HD, tid);
+  for (int i = 0; i < n_it; ++i) {
+    const int k0 = (kb_first + it0 + i * dit) * BKV, buf = i & 1;
+    if (i + 1 < n_it) {
+      const int k1 = k0 + dit * BKV;
+      load_tile<HD>(ks(buf ^ 1), a.qkv, a.ld, tok0, k1, S, (H + kvh) * HD, tid);
+      load_tile<HD>(vs(buf ^ 1), a.qkv, a.ld, tok0, k1, S, (H + KV + kvh) * HD, tid);
       cp_async_commit();
       cp_async_wait<1>();
     } else {
@@ -502,10 +469,10 @@ __device__ __forceinline__ void dq_item(const BwdArgs& a, int idx, uint16_t* sm)
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const int col = k0 + nt * 8 + 2 * (lane & 3) + (e & 1);
-        const int i = e >> 1;
-        const int row = ra + 8 * i;
+        const int ii = e >> 1;
+        const int row = ra + 8 * ii;
         const bool vis = col <= row && col < S && row < S && (!WIN || row - col < a.W);
-        p[nt][e] = vis ? exp2f(p[nt][e] * sc - lse2[i]) : 0.0f;
+        p[nt][e] = vis ? exp2f(p[nt][e] * sc - lse2[ii]) : 0.0f;
       }
     float dp[8][4];
     qk_tile<HD>(dp, smem_u32(dos), smem_u32(vs(buf)), warp, lane);
@@ -520,41 +487,130 @@ __device__ __forceinline__ void dq_item(const BwdArgs& a, int idx, uint16_t* sm)
   const int c = 2 * (lane & 3);
 #pragma unroll
   for (int i = 0; i < 2; ++i) {
-    const int row = ra + 8 * i;
-    if (row >= S) continue;
-    uint16_t* qrow = a.dqkv + (tok0 + row) * a.ld + h * HD + d0;
+    if (PART) {
+      const int rl = warp * 16 + (lane >> 2) + 8 * i;
 #pragma unroll
-    for (int dt = 0; dt < NC; ++dt)
-      *reinterpret_cast<uint32_t*>(qrow + dt * 8 + c) = pack_half2(dq[dt][2 * i] * inv, dq[dt][2 * i + 1] * inv);
+      for (int dt = 0; dt < NC; ++dt)
+        __stcg(reinterpret_cast<float2*>(pq + rl * HD + d0 + dt * 8 + c),
+               make_float2(dq[dt][2 * i] * inv, dq[dt][2 * i + 1] * inv));
+    } else {
+      const int row = ra + 8 * i;
+      if (row >= S) continue;
+      uint16_t* qrow = a.dqkv + (tok0 + row) * a.ld + h * HD + d0;
+#pragma unroll
+      for (int dt = 0; dt < NC; ++dt)
+        *reinterpret_cast<uint32_t*>(qrow + dt * 8 + c) = pack_half2(dq[dt][2 * i] * inv, dq[dt][2 * i + 1] * inv);
+    }
   }
 }
 
-// Small grids: one launch for both backward passes; blocks [0, n_kv) are dK/dV items (clusters
-// of the grp query heads of a kv head), the rest dQ items, and the two kinds run concurrently.
-// n_kv is a multiple of grp, so no cluster mixes the kinds.
-template <int HD, int DC, bool WIN>
-__global__ void __launch_bounds__(128, 1) bwd_kernel(const BwdArgs a) {
-  griddep_wait();
-  griddep_launch();
-  extern __shared__ __align__(16) uint16_t sm[];
-  if (static_cast<int>(blockIdx.x) < a.n_kv) dkdv_item<HD, DC, true, WIN>(a, blockIdx.x, sm);
-  else dq_item<HD, DC, WIN>(a, blockIdx.x - a.n_kv, sm);
-}
-
-// Large grids: dK/dV with one CTA per kv head, then dQ, as two launches.
+// Large grids: dK/dV with one CTA per (key block, kv head) looping over the group's query heads,
+// then dQ with one CTA per (query block, head), as two launches writing dqkv directly.
 template <int HD, int DC, bool WIN>
 __global__ void __launch_bounds__(128, 1) dkdv_kernel(const BwdArgs a) {
   griddep_wait();
   griddep_launch();
   extern __shared__ __align__(16) uint16_t sm[];
-  dkdv_item<HD, DC, false, WIN>(a, blockIdx.x, sm);
+  constexpr int NCH = HD / DC;
+  const int grp = a.H / a.KV, nkb = (a.S + BKV - 1) / BKV;
+  int rest = blockIdx.x;
+  const int kvh = rest % a.KV;
+  rest /= a.KV;
+  const int kb = rest % nkb;
+  rest /= nkb;
+  const int b = rest / NCH, d0 = (rest % NCH) * DC;
+  dkdv_run<HD, DC, false, WIN>(a, b, kb, kvh, kvh * grp, grp, d0, 0, 1, nullptr, nullptr, sm);
 }
 template <int HD, int DC, bool WIN>
 __global__ void __launch_bounds__(128, 1) dq_kernel(const BwdArgs a) {
   griddep_wait();
   griddep_launch();
   extern __shared__ __align__(16) uint16_t sm[];
-  dq_item<HD, DC, WIN>(a, blockIdx.x, sm);
+  constexpr int NCH = HD / DC;
+  const int nqb = (a.S + BQ - 1) / BQ;
+  int rest = blockIdx.x;
+  const int h = rest % a.H;
+  rest /= a.H;
+  const int qb = rest % nqb;
+  rest /= nqb;
+  const int b = rest / NCH, d0 = (rest % NCH) * DC;
+  dq_run<HD, DC, false, WIN>(a, b, qb, h, d0, 0, 1, nullptr, sm);
+}
+
+// Small grids: one launch of dK/dV items (key block, query head) and dQ items (query block, head),
+// each cut into P interleaved parts, longest first: group L holds the dK/dV items of key block L and
+// the dQ items of query block nqb-1-L (both see nqb-L blocks).  Partials go to the workspace;
+// bwd_finish_kernel sums them.
+template <int HD, int DC, bool WIN>
+__global__ void __launch_bounds__(128, 1) bwd_split_kernel(const BwdArgs a) {
+  griddep_wait();
+  griddep_launch();
+  extern __shared__ __align__(16) uint16_t sm[];
+  constexpr int NCH = HD / DC;
+  const int H = a.H, P = a.P, nb = (a.S + BQ - 1) / BQ;
+  const int G = H * a.B * NCH * P;
+  const int L = blockIdx.x / (2 * G), rem = blockIdx.x % (2 * G);
+  int r = rem % G;
+  const int p = r % P;
+  r /= P;
+  const int d0 = (r % NCH) * DC;
+  r /= NCH;
+  const int h = r % H, b = r / H;
+  if (rem < G) {
+    const int kb = L;
+    const int64_t slot = ((static_cast<int64_t>(b) * nb + kb) * H + h) * P + p;
+    dkdv_run<HD, DC, true, WIN>(a, b, kb, h / (H / a.KV), h, 1, d0, p, P, a.wk + slot * (64 * HD),
+                                a.wv + slot * (64 * HD), sm);
+  } else {
+    const int qb = nb - 1 - L;
+    const int64_t slot = ((static_cast<int64_t>(b) * nb + qb) * H + h) * P + p;
+    dq_run<HD, DC, true, WIN>(a, b, qb, h, d0, p, P, a.wq + slot * (64 * HD), sm);
+  }
+}
+
+// dqkv from the split partials: dQ = sum over parts; dK, dV = sum over the group's query heads and
+// parts (fixed order); q and k then rotated back by their RoPE angle when cs != null (the VJP of
+// the rotation: (d1, d2) -> (d1 c + d2 s, d2 c - d1 s)).  One thread per (token, head slot, pair j).
+template <int HD>
+__global__ void bwd_finish_kernel(const BwdArgs a, const float2* __restrict__ cs) {
+  griddep_wait();
+  griddep_launch();
+  constexpr int HALF = HD / 2;
+  const int H = a.H, KV = a.KV, S = a.S, P = a.P, nh = H + 2 * KV, grp = H / KV;
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  const int64_t T = static_cast<int64_t>(a.B) * S;
+  if (i >= T * nh * HALF) return;
+  const int j = static_cast<int>(i % HALF);
+  const int64_t r1 = i / HALF;
+  const int slot_h = static_cast<int>(r1 % nh);
+  const int64_t t = r1 / nh;
+  const int b = static_cast<int>(t / S), pos = static_cast<int>(t % S);
+  const int blk = pos / 64, row = pos % 64, nb = (S + 63) / 64;
+  const float* base;
+  int h0, hn;
+  if (slot_h < H) {
+    base = a.wq; h0 = slot_h; hn = 1;
+  } else if (slot_h < H + KV) {
+    base = a.wk; h0 = (slot_h - H) * grp; hn = grp;
+  } else {
+    base = a.wv; h0 = (slot_h - H - KV) * grp; hn = grp;
+  }
+  float x1 = 0.0f, x2 = 0.0f;
+  for (int h = h0; h < h0 + hn; ++h)
+    for (int p = 0; p < P; ++p) {
+      const float* pp = base + (((static_cast<int64_t>(b) * nb + blk) * H + h) * P + p) * (64 * HD) + row * HD;
+      x1 += __ldcg(pp + j);
+      x2 += __ldcg(pp + j + HALF);
+    }
+  if (cs && slot_h < H + KV) {
+    const float2 c = cs[static_cast<int64_t>(pos) * HALF + j];
+    const float y1 = x1 * c.x + x2 * c.y, y2 = x2 * c.x - x1 * c.y;
+    x1 = y1;
+    x2 = y2;
+  }
+  uint16_t* dst = a.dqkv + t * a.ld + static_cast<int64_t>(slot_h) * HD;
+  dst[j] = f_to_h(x1);
+  dst[j + HALF] = f_to_h(x2);
 }
 
 template <int HD, int NB, bool WIN, int NWG>
@@ -596,38 +652,48 @@ void fwd_launch(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, ui
   else fwd_launch_w<HD, false>(qkv, ld, B, S, H, KV, o, ldo, lse, 0, st);
 }
 
+// Returns true when the split mode ran (which also applied the inverse RoPE when cs != null).
 template <int HD, int DC, bool WIN>
-void bwd_launch_w(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t ldo, const float* lse,
-                const float* dvec, int B, int S, int H, int KV, int W, uint16_t* dqkv, cudaStream_t st) {
+bool bwd_launch_w(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t ldo, const float* lse,
+                  const float* dvec, int B, int S, int H, int KV, int W, uint16_t* dqkv, const float2* cs, float* ws,
+                  int64_t ws_floats, cudaStream_t st) {
   constexpr int smem = 6 * 64 * (HD + 8) * 2 + 4 * 64 * 4;  // 6 tiles (2 of them double-buffered) + lse, dvec x 2
   static_assert(smem <= 232448, "attention backward shared memory");
   static bool init = false;
   if (!init) {
-    cudaFuncSetAttribute(bwd_kernel<HD, DC, WIN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(bwd_split_kernel<HD, DC, WIN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     cudaFuncSetAttribute(dkdv_kernel<HD, DC, WIN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     cudaFuncSetAttribute(dq_kernel<HD, DC, WIN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     init = true;
   }
-  constexpr int NCH = HD / DC;
-  const int nkb = (S + BKV - 1) / BKV, nqb = (S + BQ - 1) / BQ;
-  const int grp = H / KV;
-  BwdArgs a{qkv, ld, dout, ldo, lse, dvec, S, H, KV, B, W, 0, dqkv};
-  const int n_q = nqb * H * B * NCH;      // a multiple of grp (H is)
-  const int n_grouped = nkb * KV * B * NCH;
-  if (n_grouped >= 2 * 152) {             // the per-kv-head items alone fill the GPU twice
-    a.n_kv = n_grouped;
-    launch_k(dkdv_kernel<HD, DC, WIN>, dim3(a.n_kv), 128, smem, st, a);
-    launch_k(dq_kernel<HD, DC, WIN>, dim3(n_q), 128, smem, st, a);
-    return;
+  constexpr int NCH = HD / DC, P = 2;
+  const int nb = (S + BKV - 1) / BKV;
+  BwdArgs a{qkv, ld, dout, ldo, lse, dvec, S, H, KV, B, W, dqkv};
+  const int64_t n_grouped = static_cast<int64_t>(nb) * KV * B * NCH;
+  const int64_t part_floats = static_cast<int64_t>(B) * nb * H * P * 64 * HD;  // per array
+  if (n_grouped < 2 * 152 && ws && 3 * part_floats <= ws_floats) {
+    a.P = P;
+    a.wk = ws;
+    a.wv = ws + part_floats;
+    a.wq = ws + 2 * part_floats;
+    launch_k(bwd_split_kernel<HD, DC, WIN>, dim3(static_cast<unsigned>(2LL * nb * H * B * NCH * P)), 128, smem, st,
+             a);
+    const int64_t n = static_cast<int64_t>(B) * S * (H + 2 * KV) * (HD / 2);
+    launch_k(bwd_finish_kernel<HD>, static_cast<unsigned>((n + 255) / 256), 256, 0, st, a, cs);
+    return true;
   }
-  a.n_kv = nkb * H * B * NCH;             // one item per (key block, query head, batch, column chunk)
-  launch_k_cluster(bwd_kernel<HD, DC, WIN>, dim3(a.n_kv + n_q), 128, smem, st, dim3(grp, 1, 1), a);
+  launch_k(dkdv_kernel<HD, DC, WIN>, dim3(static_cast<unsigned>(n_grouped)), 128, smem, st, a);
+  launch_k(dq_kernel<HD, DC, WIN>, dim3(static_cast<unsigned>(static_cast<int64_t>(nb) * H * B * NCH)), 128, smem, st,
+           a);
+  return false;
 }
 template <int HD, int DC>
-void bwd_launch(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t ldo, const float* lse,
-                const float* dvec, int B, int S, int H, int KV, int W, uint16_t* dqkv, cudaStream_t st) {
-  if (W > 0) bwd_launch_w<HD, DC, true>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, st);
-  else bwd_launch_w<HD, DC, false>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, 0, dqkv, st);
+bool bwd_launch(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t ldo, const float* lse,
+                const float* dvec, int B, int S, int H, int KV, int W, uint16_t* dqkv, const float2* cs, float* ws,
+                int64_t ws_floats, cudaStream_t st) {
+  if (W > 0)
+    return bwd_launch_w<HD, DC, true>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, cs, ws, ws_floats, st);
+  return bwd_launch_w<HD, DC, false>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, 0, dqkv, cs, ws, ws_floats, st);
 }
 
 }  // namespace attn
@@ -640,17 +706,18 @@ void launch_attn_fwd(const uint16_t* qkv, int64_t ld, int B, int S, int H, int K
   else attn::fwd_launch<256>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
 }
 
-void launch_attn_bwd(const uint16_t* qkv, int64_t ld, const uint16_t* o, const uint16_t* dout, int64_t ldo,
-                     const float* lse, int B, int S, int H, int KV, int hd, float* dvec, uint16_t* dqkv,
-                     int window, cudaStream_t st) {
+bool launch_attn_bwd(const uint16_t* qkv, int64_t ld, const uint16_t* o, const uint16_t* dout, int64_t ldo,
+                     const float* lse, int B, int S, int H, int KV, int hd, float* dvec, uint16_t* dqkv, int window,
+                     const float2* rope_cs, float* ws, int64_t ws_floats, cudaStream_t st) {
   const int W = window >= S ? 0 : window;
   const int64_t nw = static_cast<int64_t>(B) * S * H;
   launch_k(attn::dvec_kernel, static_cast<unsigned>((nw * 32 + 255) / 256), 256, 0, st, o, dout, ldo, B, S, H, hd,
            dvec);
-  if (hd == 64) attn::bwd_launch<64, 64>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, st);
-  else if (hd == 128)
-    attn::bwd_launch<128, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, st);
-  else attn::bwd_launch<256, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, st);
+  if (hd == 64)
+    return attn::bwd_launch<64, 64>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, rope_cs, ws, ws_floats, st);
+  if (hd == 128)
+    return attn::bwd_launch<128, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, rope_cs, ws, ws_floats, st);
+  return attn::bwd_launch<256, 128>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, rope_cs, ws, ws_floats, st);
 }
 
 }  // namespace mebp

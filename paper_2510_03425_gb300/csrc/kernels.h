@@ -204,8 +204,12 @@ void launch_attn_fwd(const uint16_t* qkv, int64_t ld, int B, int S, int H, int K
                      float* lse, int window, cudaStream_t st);
 void launch_adamw(float* p, const float* g, float* m, float* v, int64_t n, float lr, float b1, float b2, float eps,
                   float wd, float gs, double bc1, double bc2, cudaStream_t st);
-void launch_attn_bwd(const uint16_t* qkv, int64_t ld, const uint16_t* o, const uint16_t* dout, int64_t ldo,
-                     const float* lse, int B, int S, int H, int KV, int hd, float* dvec, uint16_t* dqkv,
-                     int window, cudaStream_t st);
+// Backward into dqkv.  Small grids run the split mode through the fp32 workspace ws (needs
+// 3 * B * ceil(S/64) * H * 2 * 64 * hd floats; a smaller or null ws falls back to the direct mode);
+// the split mode also rotates dq, dk back by rope_cs (when not null) and returns true — otherwise
+// the caller applies the inverse RoPE.
+bool launch_attn_bwd(const uint16_t* qkv, int64_t ld, const uint16_t* o, const uint16_t* dout, int64_t ldo,
+                     const float* lse, int B, int S, int H, int KV, int hd, float* dvec, uint16_t* dqkv, int window,
+                     const float2* rope_cs, float* ws, int64_t ws_floats, cudaStream_t st);
 
 }  // namespace mebp

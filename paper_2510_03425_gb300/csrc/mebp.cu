@@ -113,6 +113,8 @@ struct mebp_ctx {
   cudaEvent_t ev_grad[2] = {};     // reductions of a block of parity k finished
   uint16_t *dout = nullptr, *dy_h[3] = {nullptr, nullptr, nullptr};
   float *dm = nullptr, *dtmp = nullptr, *dh1 = nullptr, *dvec = nullptr, *gbuf[2] = {nullptr, nullptr};
+  float* attn_ws = nullptr;  // fp32 partials of the split attention backward (small grids)
+  int64_t attn_ws_floats = 0;
   float* red = nullptr;
   int64_t red_floats = 0;
   // LM head
@@ -480,12 +482,14 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   if ((rc = lin_grads(c, A, du[LIN_O], LIN_O, G.dh1_h, D, A.o, c->Na, T, grads, acc, grad_mult, st, tb))) return rc;
   // ---- attention, RoPE
   const Lin& lq = c->lin[LIN_QKV];
-  launch_attn_bwd(A.qkv, lq.N, A.o, c->dout, c->Na, A.lse_attn, B, Sq, c->H, c->KV, c->hd, c->dvec, G.dqkv,
-                  layer_window(c, layer), st);
+  const bool rope_done =
+      launch_attn_bwd(A.qkv, lq.N, A.o, c->dout, c->Na, A.lse_attn, B, Sq, c->H, c->KV, c->hd, c->dvec, G.dqkv,
+                      layer_window(c, layer), c->gemma ? nullptr : layer_rope(c, layer), c->attn_ws, c->attn_ws_floats,
+                      st);
   if (c->gemma)
     launch_qknorm_rope_bwd(G.dqkv, T, Sq, c->H, c->KV, c->hd, w->q_norm, w->k_norm, layer_rope(c, layer), A.qk_raw,
                            A.rqk, st);
-  else
+  else if (!rope_done)
     launch_rope(G.dqkv, T, Sq, c->H, c->KV, c->hd, layer_rope(c, layer), true, st);
   // ---- q, k, v projections
   if (lq.kx)
@@ -705,6 +709,10 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
   A(&c->dout, T * c->Na);
   for (int k = 0; k < (c->nsets == 2 ? 3 : 2); ++k) A(&c->dy_h[k], T * D);
   A(&c->dm, T * I); A(&c->dtmp, T * D); A(&c->dh1, T * D); A(&c->dvec, T * c->H);
+  // split attention backward: 3 arrays of B * ceil(S/64) * H * 2 parts * 64 * hd floats (<= 2 T rows
+  // per head and part when S >= 64), at most 192 MB; larger shapes take the direct mode
+  c->attn_ws_floats = std::min<int64_t>(3LL * 2 * c->H * c->hd * 2 * T, 48LL << 20);
+  A(&c->attn_ws, c->attn_ws_floats);
   A(&c->gbuf[0], T * D); A(&c->gbuf[1], T * D);
   c->red_floats = std::max<int64_t>(tall_reduce_scratch_floats(T, std::max<int64_t>(2 * I, c->Nqkv), 32),
                                     tall_reduce_scratch_floats(T, std::max<int64_t>(I, D), 32));
