@@ -1235,6 +1235,7 @@ int mebp_lora_step(mebp_ctx* c, const mebp_model_weights* model, const mebp_lora
     const mebp_block_weights& w = model->blocks[i];
     K(w.qkv.qpack); K(w.qkv.scales); K(w.o.qpack); K(w.o.scales); K(w.gate_up.qpack); K(w.gate_up.scales);
     K(w.down.qpack); K(w.down.scales); K(w.norm1); K(w.norm2);
+    K(w.q_norm); K(w.k_norm); K(w.post_attn_norm); K(w.post_ffn_norm);
     for (int t = 0; t < MEBP_N_TARGETS; ++t) {
       K(lora[i].A[t]); K(lora[i].B[t]);
       K(grads ? grads[i].dA[t] : nullptr); K(grads ? grads[i].dB[t] : nullptr);
