@@ -571,6 +571,7 @@ __global__ void __launch_bounds__(128, 1) bwd_split_kernel(const BwdArgs a) {
 // dqkv from the split partials: dQ = sum over parts; dK, dV = sum over the group's query heads and
 // parts (fixed order); q and k then rotated back by their RoPE angle when cs != null (the VJP of
 // the rotation: (d1, d2) -> (d1 c + d2 s, d2 c - d1 s)).  One thread per (token, head slot, pair j).
+constexpr int kFinishMax = 16;  // partials per element: query heads per kv head (<= 8) x parts (2)
 template <int HD>
 __global__ void bwd_finish_kernel(const BwdArgs a, const float2* __restrict__ cs) {
   griddep_wait();
@@ -595,13 +596,22 @@ __global__ void bwd_finish_kernel(const BwdArgs a, const float2* __restrict__ cs
   } else {
     base = a.wv; h0 = (slot_h - H - KV) * grp; hn = grp;
   }
+  // all loads first (up to kFinishMax independent L2 reads in flight), then the sums in
+  // (head, part) order
+  const int n = hn * P;
+  const float* pp0 = base + ((static_cast<int64_t>(b) * nb + blk) * H + h0) * P * (64 * HD) + row * HD + j;
+  float v1[kFinishMax], v2[kFinishMax];
+#pragma unroll
+  for (int k = 0; k < kFinishMax; ++k) {
+    v1[k] = k < n ? __ldcg(pp0 + static_cast<int64_t>(k) * (64 * HD)) : 0.0f;
+    v2[k] = k < n ? __ldcg(pp0 + static_cast<int64_t>(k) * (64 * HD) + HALF) : 0.0f;
+  }
   float x1 = 0.0f, x2 = 0.0f;
-  for (int h = h0; h < h0 + hn; ++h)
-    for (int p = 0; p < P; ++p) {
-      const float* pp = base + (((static_cast<int64_t>(b) * nb + blk) * H + h) * P + p) * (64 * HD) + row * HD;
-      x1 += __ldcg(pp + j);
-      x2 += __ldcg(pp + j + HALF);
-    }
+#pragma unroll
+  for (int k = 0; k < kFinishMax; ++k) {
+    x1 += v1[k];
+    x2 += v2[k];
+  }
   if (cs && slot_h < H + KV) {
     const float2 c = cs[static_cast<int64_t>(pos) * HALF + j];
     const float y1 = x1 * c.x + x2 * c.y, y2 = x2 * c.x - x1 * c.y;
@@ -671,7 +681,7 @@ bool bwd_launch_w(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t
   BwdArgs a{qkv, ld, dout, ldo, lse, dvec, S, H, KV, B, W, dqkv};
   const int64_t n_grouped = static_cast<int64_t>(nb) * KV * B * NCH;
   const int64_t part_floats = static_cast<int64_t>(B) * nb * H * P * 64 * HD;  // per array
-  if (n_grouped < 2 * 152 && ws && 3 * part_floats <= ws_floats) {
+  if (n_grouped < 2 * 152 && ws && 3 * part_floats <= ws_floats && (H / KV) * P <= kFinishMax) {
     a.P = P;
     a.wk = ws;
     a.wv = ws + part_floats;
