@@ -25,14 +25,23 @@ constexpr int A_BYTES = BM * BK * 2;
 constexpr int P_BYTES = BN * BK / 2;
 constexpr int S_BYTES = 128;
 constexpr int B_BYTES = BN * BK * 2;
-constexpr int TSTG = 4, BSTG = 3;
-constexpr int A_OFF = 0, P_OFF = A_BYTES, S_OFF = P_OFF + P_BYTES;
-constexpr int T_STRIDE = (S_OFF + S_BYTES + 1023) / 1024 * 1024;
-constexpr int B_BASE = TSTG * T_STRIDE;
-constexpr int BAR_OFF = B_BASE + BSTG * B_BYTES;
-constexpr int SMEM = BAR_OFF + 512 + 1024;
 constexpr uint32_t TMEM_COLS = 64;
-static_assert(2 * SMEM <= 232448, "two CTAs per SM");
+// Shared-memory layout for KCH chunks of 64 K per pipeline stage: a TMA slot holds KCH activation
+// tiles, then KCH packed weight tiles, then KCH scale rows; a decode slot holds KCH decoded tiles.
+// KCH = 1: four TMA slots and three decode slots, two CTAs per SM.  KCH = 2 (grids of at most one
+// CTA per SM): half as many stages, so half the barrier hand-offs for the same K.
+template <int KCH>
+struct Lay {
+  static constexpr int TSTG = KCH == 1 ? 4 : 3, BSTG = KCH == 1 ? 3 : 2;
+  static constexpr int A_OFF = 0, P_OFF = KCH * A_BYTES, S_OFF = P_OFF + KCH * P_BYTES;
+  static constexpr int T_STRIDE = (S_OFF + KCH * S_BYTES + 1023) / 1024 * 1024;
+  static constexpr int B_SLOT = KCH * B_BYTES;
+  static constexpr int B_BASE = TSTG * T_STRIDE;
+  static constexpr int BAR_OFF = B_BASE + BSTG * B_SLOT;
+  static constexpr int SMEM = BAR_OFF + 512 + 1024;
+};
+static_assert(2 * Lay<1>::SMEM <= 232448, "two CTAs per SM");
+static_assert(Lay<2>::SMEM <= 232448, "one CTA per SM");
 
 struct Params {
   int M, N, K;
@@ -144,14 +153,17 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
   }
 }
 
-template <bool TRANS>
-__global__ void __launch_bounds__(THREADS, 2)
+template <bool TRANS, int KCH>
+__global__ void __launch_bounds__(THREADS, KCH == 1 ? 2 : 1)
     dequant_gemm_narrow(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmP,
                         const __grid_constant__ CUtensorMap tmS, const __grid_constant__ CUtensorMap tmAx,
                         const Params p) {
+  using L = Lay<KCH>;
+  constexpr int TSTG = L::TSTG, BSTG = L::BSTG, T_STRIDE = L::T_STRIDE, B_BASE = L::B_BASE;
+  constexpr int A_OFF = L::A_OFF, P_OFF = L::P_OFF, S_OFF = L::S_OFF;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* wfull = reinterpret_cast<uint64_t*>(smem + BAR_OFF);  // packed weights + scales landed
+  uint64_t* wfull = reinterpret_cast<uint64_t*>(smem + L::BAR_OFF);  // packed weights + scales landed
   uint64_t* afull = wfull + TSTG;                                  // activation tile landed
   uint64_t* empty = afull + TSTG;                                  // MMA done with the TMA slot
   uint64_t* bfull = empty + TSTG;                                  // decoded tile ready
@@ -163,8 +175,14 @@ __global__ void __launch_bounds__(THREADS, 2)
   griddep_launch();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM;
-  const int num_main = p.K / BK;
-  const int total = num_main + (p.kx_steps + 3) / 4;  // LoRA block last
+  // chunks of 64 K: main ones, then the LoRA block's (each up to four k16 steps); stage it holds
+  // chunks it*KCH .. of the main sequence (it < num_main), then of the LoRA sequence
+  const int nch_main = p.K / BK, nch_lora = (p.kx_steps + 3) / 4;
+  const int num_main = (nch_main + KCH - 1) / KCH;
+  const int total = num_main + (nch_lora + KCH - 1) / KCH;
+  auto stage_chunks = [&](int it) {
+    return it < num_main ? min(KCH, nch_main - it * KCH) : min(KCH, nch_lora - (it - num_main) * KCH);
+  };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < TSTG; ++s) {
@@ -192,15 +210,18 @@ __global__ void __launch_bounds__(THREADS, 2)
       tma_prefetch_desc(&tmP);
       tma_prefetch_desc(&tmS);
       auto load_w = [&](int it) {
-        const int s = it % TSTG;
+        const int s = it % TSTG, nch = stage_chunks(it);
         uint8_t* st = smem + s * T_STRIDE;
-        mbar_arrive_expect_tx(&wfull[s], P_BYTES + S_BYTES);
-        if (!TRANS) {
-          tma_load_2d(st + P_OFF, &tmP, &wfull[s], it * (BK / 2), n0);  // packed [N, K/2]
-          tma_load_2d(st + S_OFF, &tmS, &wfull[s], n0, it);             // scales [K/64, N]
-        } else {
-          tma_load_2d(st + P_OFF, &tmP, &wfull[s], n0 / 2, it * BK);    // packed [K, N/2]
-          tma_load_2d(st + S_OFF, &tmS, &wfull[s], it * BK, n0 / 64);   // scales [N/64, K]
+        mbar_arrive_expect_tx(&wfull[s], nch * (P_BYTES + S_BYTES));
+        for (int c = 0; c < nch; ++c) {
+          const int kc = it * KCH + c;
+          if (!TRANS) {
+            tma_load_2d(st + P_OFF + c * P_BYTES, &tmP, &wfull[s], kc * (BK / 2), n0);  // packed [N, K/2]
+            tma_load_2d(st + S_OFF + c * S_BYTES, &tmS, &wfull[s], n0, kc);             // scales [K/64, N]
+          } else {
+            tma_load_2d(st + P_OFF + c * P_BYTES, &tmP, &wfull[s], n0 / 2, kc * BK);    // packed [K, N/2]
+            tma_load_2d(st + S_OFF + c * S_BYTES, &tmS, &wfull[s], kc * BK, n0 / 64);   // scales [N/64, K]
+          }
         }
       };
       // The packed weights are never written by a kernel of the same call (and the first kernel
@@ -213,9 +234,12 @@ __global__ void __launch_bounds__(THREADS, 2)
         if (it >= TSTG && !mbar_wait(&empty[s], ((it / TSTG) & 1) ^ 1, abort_flag, p.err)) break;
         if (it < num_main && it >= w_issued) load_w(w_issued++);
         uint8_t* st = smem + s * T_STRIDE;
-        mbar_arrive_expect_tx(&afull[s], A_BYTES);
-        if (it < num_main) tma_load_2d(st + A_OFF, &tmA, &afull[s], it * BK, m0);
-        else tma_load_2d(st + A_OFF, &tmAx, &afull[s], (it - num_main) * BK, m0);
+        const int nch = stage_chunks(it);
+        mbar_arrive_expect_tx(&afull[s], nch * A_BYTES);
+        for (int c = 0; c < nch; ++c) {
+          if (it < num_main) tma_load_2d(st + A_OFF + c * A_BYTES, &tmA, &afull[s], (it * KCH + c) * BK, m0);
+          else tma_load_2d(st + A_OFF + c * A_BYTES, &tmAx, &afull[s], ((it - num_main) * KCH + c) * BK, m0);
+        }
         a_issued = it + 1;
       }
       int dummy = 0;
@@ -232,19 +256,28 @@ __global__ void __launch_bounds__(THREADS, 2)
         if (!mbar_wait(&afull[s], (it / TSTG) & 1, abort_flag, p.err)) break;
         if (!mbar_wait(&bfull[b], (it / BSTG) & 1, abort_flag, p.err)) break;
         tc_fence_after();
-        // the stage's first-slice descriptors; later k16 slices advance the start-address field
+        // the stage's first-slice descriptors; later k16 slices advance the start-address field,
+        // later chunks start one tile further (A: A_BYTES, B: B_BYTES)
         const uint64_t ad0 = smem_desc_sw128(smem_u32(smem + s * T_STRIDE + A_OFF), 16, 1024);
-        const uint64_t bd0 = TRANS ? smem_desc_sw128(smem_u32(smem + B_BASE + b * B_BYTES), 8192, 1024)
-                                   : smem_desc_sw128(smem_u32(smem + B_BASE + b * B_BYTES), 16, 1024);
+        const uint64_t bd0 = TRANS ? smem_desc_sw128(smem_u32(smem + B_BASE + b * L::B_SLOT), 8192, 1024)
+                                   : smem_desc_sw128(smem_u32(smem + B_BASE + b * L::B_SLOT), 16, 1024);
         constexpr uint64_t A_K16 = 32 >> 4, B_K16 = (TRANS ? 2048 : 32) >> 4;
-        if (it < num_main) {
+        constexpr uint64_t A_CH = A_BYTES >> 4, B_CH = B_BYTES >> 4;
+        const int nch = stage_chunks(it);
+        if (it < num_main && nch == KCH) {
 #pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            tc_mma_f16(tmem, ad0 + kk * A_K16, bd0 + kk * B_K16, idesc, (it > 0 || kk > 0) ? 1u : 0u);
+          for (int c = 0; c < KCH; ++c)
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              tc_mma_f16(tmem, ad0 + c * A_CH + kk * A_K16, bd0 + c * B_CH + kk * B_K16, idesc,
+                         (it > 0 || c > 0 || kk > 0) ? 1u : 0u);
         } else {
-          const int nk = min(4, p.kx_steps - 4 * (it - num_main));
-          for (int kk = 0; kk < nk; ++kk)
-            tc_mma_f16(tmem, ad0 + kk * A_K16, bd0 + kk * B_K16, idesc, (it > 0 || kk > 0) ? 1u : 0u);
+          for (int c = 0; c < nch; ++c) {
+            const int nk = it < num_main ? 4 : min(4, p.kx_steps - 4 * ((it - num_main) * KCH + c));
+            for (int kk = 0; kk < nk; ++kk)
+              tc_mma_f16(tmem, ad0 + c * A_CH + kk * A_K16, bd0 + c * B_CH + kk * B_K16, idesc,
+                         (it > 0 || c > 0 || kk > 0) ? 1u : 0u);
+          }
         }
         tc_commit(&empty[s]);
         tc_commit(&bempty[b]);
@@ -257,15 +290,18 @@ __global__ void __launch_bounds__(THREADS, 2)
     for (int it = 0; it < total; ++it) {
       const int s = it % TSTG, b = it % BSTG;
       if (!mbar_wait(&bempty[b], ((it / BSTG) & 1) ^ 1, abort_flag, p.err)) break;
-      uint8_t* bt = smem + B_BASE + b * B_BYTES;
+      uint8_t* bt = smem + B_BASE + b * L::B_SLOT;
+      const int nch = stage_chunks(it);
       if (it < num_main) {
         if (!mbar_wait(&wfull[s], (it / TSTG) & 1, abort_flag, p.err)) break;
         const uint8_t* st = smem + s * T_STRIDE;
-        if (TRANS) convert_trans(st + P_OFF, st + S_OFF, bt, t);
-        else convert_fwd(st + P_OFF, st + S_OFF, bt, t);
+        for (int c = 0; c < nch; ++c) {
+          if (TRANS) convert_trans(st + P_OFF + c * P_BYTES, st + S_OFF + c * S_BYTES, bt + c * B_BYTES, t);
+          else convert_fwd(st + P_OFF + c * P_BYTES, st + S_OFF + c * S_BYTES, bt + c * B_BYTES, t);
+        }
       } else {
         griddep_wait();  // the LoRA operand comes from an earlier kernel
-        copy_lora_b<TRANS>(p, it - num_main, n0, bt, t);
+        for (int c = 0; c < nch; ++c) copy_lora_b<TRANS>(p, (it - num_main) * KCH + c, n0, bt + c * B_BYTES, t);
       }
       fence_proxy_async_smem();
       __syncwarp();
@@ -293,17 +329,18 @@ __global__ void __launch_bounds__(THREADS, 2)
 }  // namespace gemms
 
 namespace {
-template <bool TRANS>
+template <bool TRANS, int KCH>
 int launch_s(dim3 grid, const CUtensorMap& tA, const CUtensorMap& tP, const CUtensorMap& tS, const CUtensorMap& tAx,
              const gemms::Params& p, cudaStream_t st) {
+  constexpr int smem = gemms::Lay<KCH>::SMEM;
   static bool attr = false;
   if (!attr) {
-    if (cudaFuncSetAttribute(gemms::dequant_gemm_narrow<TRANS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             gemms::SMEM) != cudaSuccess)
+    if (cudaFuncSetAttribute(gemms::dequant_gemm_narrow<TRANS, KCH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             smem) != cudaSuccess)
       return MEBP_ERR_CUDA;
     attr = true;
   }
-  if (launch_k(gemms::dequant_gemm_narrow<TRANS>, grid, dim3(gemms::THREADS), gemms::SMEM, st, tA, tP, tS, tAx, p) !=
+  if (launch_k(gemms::dequant_gemm_narrow<TRANS, KCH>, grid, dim3(gemms::THREADS), smem, st, tA, tP, tS, tAx, p) !=
       cudaSuccess)
     return MEBP_ERR_CUDA;
   return MEBP_OK;
@@ -357,7 +394,11 @@ int launch_dequant_gemm_narrow(const GemmArgs& g, cudaStream_t st) {
   p.alpha = g.alpha;
   p.err = g.err;
   const dim3 grid(static_cast<unsigned>(g.N / BN), static_cast<unsigned>((g.M + BM - 1) / BM));
-  rc = g.trans ? launch_s<true>(grid, tA, tP, tS, tAx, p, st) : launch_s<false>(grid, tA, tP, tS, tAx, p, st);
+  // grids of at most one CTA per SM take two K chunks per stage
+  if (static_cast<int64_t>(grid.x) * grid.y <= 152)
+    rc = g.trans ? launch_s<true, 2>(grid, tA, tP, tS, tAx, p, st) : launch_s<false, 2>(grid, tA, tP, tS, tAx, p, st);
+  else
+    rc = g.trans ? launch_s<true, 1>(grid, tA, tP, tS, tAx, p, st) : launch_s<false, 1>(grid, tA, tP, tS, tAx, p, st);
   if (rc) return rc;
   return cudaGetLastError() == cudaSuccess ? MEBP_OK : MEBP_ERR_CUDA;
 }
