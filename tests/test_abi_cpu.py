@@ -52,6 +52,7 @@ def _cfg(binding, **kw):
     ("vocab_chunk", 100, 1),       # chunk not a multiple of 256
     ("max_tokens", 0, 1),
     ("act", 7, 1),
+    ("sliding_window", -1, 1),     # negative window
 ])
 def test_ctx_create_rejects_bad_configs_without_a_gpu(binding, field, value, code):
     cfg = _cfg(binding, **{field: value})
@@ -59,6 +60,22 @@ def test_ctx_create_rejects_bad_configs_without_a_gpu(binding, field, value, cod
     rc = binding.lib().mebp_ctx_create(ctypes.byref(cfg), 0, ctypes.byref(out))
     assert rc == code
     assert not out.value
+
+
+def test_ctx_create_rejects_a_window_without_global_layers_or_local_base(binding):
+    for kw in (dict(sliding_window=128, global_every=0), dict(sliding_window=128, rope_theta_local=0.0)):
+        cfg = _cfg(binding, **kw)
+        out = ctypes.c_void_p()
+        assert binding.lib().mebp_ctx_create(ctypes.byref(cfg), 0, ctypes.byref(out)) == 1
+        assert not out.value
+
+
+def test_model_cfg_carries_the_gemma3_options(binding):
+    from workload import synth
+    d = synth.preset(2).with_(gemma_norms=True, sliding_window=512, global_every=6, rope_theta_local=1e4)
+    c = binding.model_cfg(d)
+    assert (c.gemma_norms, c.sliding_window, c.global_every, c.rope_theta_local) == (1, 512, 6, 1e4)
+    assert binding.model_cfg(synth.preset(2)).gemma_norms == 0
 
 
 def test_null_context_is_rejected(binding):
