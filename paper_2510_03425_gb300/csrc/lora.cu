@@ -131,9 +131,100 @@ __global__ void __launch_bounds__(128) skinny_gemm_kernel(const uint16_t* __rest
   cluster_sync_all();  // no CTA leaves while its partial is being read
 }
 
+// Few tokens: one CTA per 16 rows holding the rows' whole K slab and all of W in shared memory
+// (one load, no pipeline), the four warps each taking a quarter of the k16 steps; the four fp32
+// partials are summed in warp order through shared memory.  No cluster, no second barrier round.
+template <int NT>
+__global__ void __launch_bounds__(128) skinny_slab_kernel(const uint16_t* __restrict__ X, int64_t ldx, int64_t M,
+                                                          int K, const uint16_t* __restrict__ W, int64_t ldw,
+                                                          float alpha, uint16_t* __restrict__ out, int64_t ldo) {
+  griddep_wait();
+  griddep_launch();
+  constexpr int JR = NT * 8, LDR = JR + 4;
+  extern __shared__ __align__(16) uint8_t sm[];
+  const int LDS = K + 8;
+  uint16_t* xs = reinterpret_cast<uint16_t*>(sm);
+  uint16_t* ws = xs + 16 * LDS;
+  float* red = reinterpret_cast<float*>(ws + JR * LDS);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int64_t m0 = static_cast<int64_t>(blockIdx.x) * 16;
+  const int kc = K / 8;
+  for (int c = tid; c < 16 * kc; c += 128) {
+    const int r = c / kc, cc = c % kc;
+    const int64_t gm = m0 + r;
+    const bool v = gm < M;
+    cp_async16(smem_u32(xs + r * LDS + cc * 8), X + (v ? gm : 0) * ldx + cc * 8, v);
+  }
+  for (int c = tid; c < JR * kc; c += 128) {
+    const int r = c / kc, cc = c % kc;
+    cp_async16(smem_u32(ws + r * LDS + cc * 8), W + r * ldw + cc * 8, true);
+  }
+  cp_async_commit();
+  cp_async_wait<0>();
+  __syncthreads();
+  float acc[NT][4];
+#pragma unroll
+  for (int i = 0; i < NT; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.0f;
+  const int nks = K / 16, ks0 = warp * nks / 4, ks1 = (warp + 1) * nks / 4;
+  const uint32_t xb = smem_u32(xs), wb = smem_u32(ws);
+  for (int ks = ks0; ks < ks1; ++ks) {
+    uint32_t a[4];
+    ldsm_x4(a, frag_a_addr(xb, LDS, 0, ks * 16, lane));
+#pragma unroll
+    for (int nt = 0; nt < NT; nt += 2) {
+      uint32_t b[4];
+      ldsm_x4(b, frag_bn_addr(wb, LDS, nt * 8, ks * 16, lane));
+      mma16816(acc[nt], a, b[0], b[1]);
+      mma16816(acc[nt + 1], a, b[2], b[3]);
+    }
+  }
+  const int r = lane >> 2, c = (lane & 3) * 2;
+  float* rw = red + warp * 16 * LDR;
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) {
+    *reinterpret_cast<float2*>(rw + r * LDR + nt * 8 + c) = make_float2(acc[nt][0], acc[nt][1]);
+    *reinterpret_cast<float2*>(rw + (r + 8) * LDR + nt * 8 + c) = make_float2(acc[nt][2], acc[nt][3]);
+  }
+  __syncthreads();
+  for (int i = tid; i < 16 * JR; i += 128) {
+    const int rr = i / JR, col = i % JR;
+    const int64_t row = m0 + rr;
+    if (row >= M) continue;
+    const float s = red[rr * LDR + col] + red[16 * LDR + rr * LDR + col] + red[32 * LDR + rr * LDR + col] +
+                    red[48 * LDR + rr * LDR + col];
+    out[row * ldo + col] = f_to_h(alpha * s);
+  }
+}
+
+template <int NT>
+int64_t skinny_slab_smem(int64_t K) {
+  return (16 + NT * 8) * (K + 8) * 2 + 4 * 16 * (NT * 8 + 4) * 4;
+}
+
+// The slab kernel when the token count is short and the slab fits; true if it was launched.
+template <int NT>
+bool skinny_slab_launch(const uint16_t* X, int64_t ldx, int64_t M, int64_t K, const uint16_t* W, int64_t ldw,
+                        float alpha, uint16_t* out, int64_t ldo, cudaStream_t st) {
+  const int64_t smem = skinny_slab_smem<NT>(K);
+  if (M > 1024 || smem > 200 * 1024 || K % 16) return false;
+  static int64_t set = 0;
+  if (smem > set) {
+    if (cudaFuncSetAttribute(skinny_slab_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(smem)) != cudaSuccess) {
+      cudaGetLastError();
+      return false;
+    }
+    set = smem;
+  }
+  launch_k(skinny_slab_kernel<NT>, static_cast<unsigned>((M + 15) / 16), 128, static_cast<size_t>(smem), st, X, ldx,
+           M, static_cast<int>(K), W, ldw, alpha, out, ldo);
+  return true;
+}
+
 template <int NT>
 void skinny_launch(const uint16_t* X, int64_t ldx, int64_t M, int64_t K, const uint16_t* W, int64_t ldw, float alpha,
                    uint16_t* out, int64_t ldo, cudaStream_t st) {
+  if (skinny_slab_launch<NT>(X, ldx, M, K, W, ldw, alpha, out, ldo, st)) return;
   const int gx = static_cast<int>((M + 63) / 64);
   const int nk = static_cast<int>(K / 64);
   // Split K over a cluster when the row blocks alone leave most of the SMs idle: up to 8 splits
