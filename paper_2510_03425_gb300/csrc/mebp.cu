@@ -112,7 +112,8 @@ struct mebp_ctx {
   cudaEvent_t ev_bwd = nullptr;    // backward of the current block issued (main stream)
   cudaEvent_t ev_grad[2] = {};     // reductions of a block of parity k finished
   uint16_t *dout = nullptr, *dy_h[3] = {nullptr, nullptr, nullptr};
-  float *dm = nullptr, *dtmp = nullptr, *dh1 = nullptr, *dvec = nullptr, *gbuf[2] = {nullptr, nullptr};
+  uint16_t* dm = nullptr;  // dE/dm of the gated MLP, fp16 (in the backward's working scale)
+  float *dtmp = nullptr, *dh1 = nullptr, *dvec = nullptr, *gbuf[2] = {nullptr, nullptr};
   float* attn_ws = nullptr;  // fp32 partials of the split attention backward (small grids)
   int64_t attn_ws_floats = 0;
   float* red = nullptr;
@@ -448,7 +449,7 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
     launch_skinny_gemm(ddn_h, D, T, D, A.sh->Bt_cat[LIN_DOWN], D, ld.kx, c->s, du[LIN_DOWN], ld.kxp, st);
     g.Ax = du[LIN_DOWN]; g.ldax = ld.kxp; g.kx = ld.kxp; g.Bx = A.sh->A_cat[LIN_DOWN]; g.ldbx = I;
   }
-  g.epi = EPI_F32; g.C = c->dm; g.ldc = I;
+  g.epi = EPI_F16; g.C = c->dm; g.ldc = I;
   if ((rc = run_gemm(c, g, st, "down dX"))) return rc;
   if ((rc = lin_grads(c, A, du[LIN_DOWN], LIN_DOWN, ddn_h, D, A.m, I, T, grads, acc, grad_mult, st, tb))) return rc;
   // ---- gated MLP

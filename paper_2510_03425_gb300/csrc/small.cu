@@ -357,7 +357,7 @@ __global__ void glu_fwd_kernel(const uint16_t* __restrict__ gu, int64_t T, int I
 }
 
 // dg = dm * u * act'(g), du = dm * act(g)
-__global__ void glu_bwd_kernel(const float* __restrict__ dm, const uint16_t* __restrict__ gu, int64_t T, int I, int act,
+__global__ void glu_bwd_kernel(const uint16_t* __restrict__ dm, const uint16_t* __restrict__ gu, int64_t T, int I, int act,
                                uint16_t* __restrict__ dgu) {
   griddep_wait();
   griddep_launch();
@@ -368,9 +368,9 @@ __global__ void glu_bwd_kernel(const float* __restrict__ dm, const uint16_t* __r
   const int c = static_cast<int>(i % per) * 8;
   const uint4 gv = *reinterpret_cast<const uint4*>(gu + t * 2 * I + c);
   const uint4 uv = *reinterpret_cast<const uint4*>(gu + t * 2 * I + I + c);
-  const float4 d0 = *reinterpret_cast<const float4*>(dm + t * I + c);
-  const float4 d1 = *reinterpret_cast<const float4*>(dm + t * I + c + 4);
-  const float dd[8] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
+  const uint4 dv = *reinterpret_cast<const uint4*>(dm + t * I + c);
+  const float dd[8] = {h2_lo(dv.x), h2_hi(dv.x), h2_lo(dv.y), h2_hi(dv.y),
+                       h2_lo(dv.z), h2_hi(dv.z), h2_lo(dv.w), h2_hi(dv.w)};
   const uint32_t ga[4] = {gv.x, gv.y, gv.z, gv.w}, ua[4] = {uv.x, uv.y, uv.z, uv.w};
   uint32_t og[4], ou[4];
 #pragma unroll
@@ -388,7 +388,7 @@ void launch_glu_fwd(const uint16_t* gu, int64_t T, int I, int act, uint16_t* m, 
   if (n <= 0) return;
   launch_k(glu_fwd_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, st, gu, T, I, act, m);
 }
-void launch_glu_bwd(const float* dm, const uint16_t* gu, int64_t T, int I, int act, uint16_t* dgu, cudaStream_t st) {
+void launch_glu_bwd(const uint16_t* dm, const uint16_t* gu, int64_t T, int I, int act, uint16_t* dgu, cudaStream_t st) {
   const int64_t n = T * (I / 8);
   if (n <= 0) return;
   launch_k(glu_bwd_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, st, dm, gu, T, I, act, dgu);
