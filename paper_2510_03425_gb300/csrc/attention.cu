@@ -88,7 +88,11 @@ __device__ __forceinline__ void pv_tile(float (&acc)[NC][4], const float (&p)[8]
 // buffers per group: 2 overlaps the next round's loads with this one; 1 saves shared memory.
 // WIN: sliding-window layer (window W); key blocks wholly before the window are skipped.  (Masking
 // only the blocks a mask cuts measured slower than masking every block.)
-template <int HD, int NB, bool WIN, int NWG>
+// C = 2: a query block's key blocks are shared by a cluster of two CTAs (grid.x = query blocks x 2,
+// rank = blockIdx.x % 2), key block i of the list going to group i % NWG of CTA (i / NWG) % 2; each
+// CTA merges its groups, then CTA r merges rows 32 r .. 32 r + 31 of both CTAs' (max, sum, o)
+// through distributed shared memory.  For grids whose doubled size still fits one CTA per SM.
+template <int HD, int NB, bool WIN, int NWG, int C = 1>
 __global__ void __launch_bounds__(128 * NWG, 1) fwd_kernel(const uint16_t* __restrict__ qkv, int64_t ld, int S,
                                                            int H, int KV, uint16_t* __restrict__ o, int64_t ldo,
                                                            float* __restrict__ lse, int W) {
@@ -101,18 +105,21 @@ __global__ void __launch_bounds__(128 * NWG, 1) fwd_kernel(const uint16_t* __res
   auto vs = [&](int buf, int g) { return qs + (2 + 2 * (buf * NWG + g)) * TILE; };
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int wg = warp >> 2, wr = warp & 3;
-  const int qb = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int crank = C > 1 ? static_cast<int>(blockIdx.x) % C : 0;
+  const int qb = static_cast<int>(blockIdx.x) / C, h = blockIdx.y, b = blockIdx.z;
   const int kvh = h / (H / KV);
   const int64_t tok0 = static_cast<int64_t>(b) * S;
   const int q0 = qb * BQ;
   const float sc = kLog2e * rsqrtf(static_cast<float>(HD));
   // visible key blocks: kb_first .. qb (window: from the first block inside it)
   const int kb_first = WIN ? max(0, q0 - W + 1) / BKV : 0;
-  const int nrounds = (qb - kb_first + NWG) / NWG;
+  const int nrounds = (qb - kb_first + C * NWG) / (C * NWG);
+  // key block of group g of this CTA in round t
+  auto kb_of = [&](int t, int g) { return kb_first + (t * C + crank) * NWG + g; };
   auto fetch = [&](int t, int buf) {  // the key/value blocks of round t, one per group
 #pragma unroll
     for (int g = 0; g < NWG; ++g) {
-      const int kb = kb_first + t * NWG + g;
+      const int kb = kb_of(t, g);
       if (kb > qb) break;
       load_tile<HD, NT>(ks(buf, g), qkv, ld, tok0, kb * BKV, S, (H + kvh) * HD, tid);
       load_tile<HD, NT>(vs(buf, g), qkv, ld, tok0, kb * BKV, S, (H + KV + kvh) * HD, tid);
@@ -142,7 +149,7 @@ __global__ void __launch_bounds__(128 * NWG, 1) fwd_kernel(const uint16_t* __res
       cp_async_wait<0>();
     }
     __syncthreads();
-    const int kb = kb_first + t * NWG + wg;
+    const int kb = kb_of(t, wg);
     if (kb <= qb) {  // uniform over the warp-group
       const int k0 = kb * BKV;
       float s[8][4];
@@ -208,9 +215,10 @@ __global__ void __launch_bounds__(128 * NWG, 1) fwd_kernel(const uint16_t* __res
       }
     }
     __syncthreads();
-    if (wg > 0) return;
+    if (C == 1 && wg > 0) return;  // (with a cluster every thread stays for its barriers)
 #pragma unroll
     for (int g = 1; g < NWG; ++g) {
+      if (wg > 0) break;
       const float* op = park + (g - 1) * PART;
       const float2* ml = reinterpret_cast<const float2*>(op + 64 * LDO);
 #pragma unroll
@@ -230,6 +238,57 @@ __global__ void __launch_bounds__(128 * NWG, 1) fwd_kernel(const uint16_t* __res
         }
       }
     }
+  }
+  if constexpr (C > 1) {
+    // group 0 of each CTA parks the CTA's (o, m, l) in its own shared memory; CTA r then merges
+    // rows r * 64/C .. of all C CTAs through distributed shared memory in rank order
+    constexpr int LDO = HD + 4, RPC = 64 / C, C4 = HD / 4;
+    static_assert(64 * LDO * 4 + 64 * 16 <= (1 + 2 * NB * NWG) * TILE * 2, "cluster merge buffers fit");
+    __syncthreads();  // the group merge has read the parked groups
+    float* op = reinterpret_cast<float*>(sm);
+    float4* ml = reinterpret_cast<float4*>(op + 64 * LDO);
+    if (wg == 0) {
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        const int rl = wr * 16 + (lane >> 2) + 8 * i;
+#pragma unroll
+        for (int dt = 0; dt < NO; ++dt)
+          *reinterpret_cast<float2*>(op + rl * LDO + dt * 8 + c) = make_float2(oacc[dt][2 * i], oacc[dt][2 * i + 1]);
+        if ((lane & 3) == 0) ml[rl] = make_float4(mrow[i], lrow[i], 0.0f, 0.0f);
+      }
+    }
+    cluster_sync_all();
+    const uint32_t op_u = smem_u32(op), ml_u = smem_u32(ml);
+    for (int e = tid; e < RPC * C4; e += NT) {
+      const int rl = crank * RPC + e / C4, cc = (e % C4) * 4;
+      const int row = q0 + rl;
+      float mj[C], lj[C];
+      float M = -INFINITY;
+#pragma unroll
+      for (int j = 0; j < C; ++j) {
+        const float4 v = ld_dsmem_f4(dsmem_addr(ml_u + rl * 16, j));
+        mj[j] = v.x;
+        lj[j] = v.y;
+        M = fmaxf(M, v.x);
+      }
+      float L = 0.0f;
+      float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll
+      for (int j = 0; j < C; ++j) {
+        const float w = mj[j] == -INFINITY ? 0.0f : exp2f(mj[j] - M);
+        L += w * lj[j];
+        const float4 q = ld_dsmem_f4(dsmem_addr(op_u + (rl * LDO + cc) * 4, j));
+        acc.x += w * q.x; acc.y += w * q.y; acc.z += w * q.z; acc.w += w * q.w;
+      }
+      if (row < S) {
+        const float inv = 1.0f / L;
+        *reinterpret_cast<uint2*>(o + (tok0 + row) * ldo + h * HD + cc) =
+            make_uint2(pack_half2(acc.x * inv, acc.y * inv), pack_half2(acc.z * inv, acc.w * inv));
+        if (cc == 0) lse[(static_cast<int64_t>(b) * H + h) * S + row] = (M + log2f(L)) / kLog2e;
+      }
+    }
+    cluster_sync_all();  // no CTA leaves while its partials are being read
+    return;
   }
 #pragma unroll
   for (int i = 0; i < 2; ++i) {
@@ -623,18 +682,21 @@ __global__ void bwd_finish_kernel(const BwdArgs a, const float2* __restrict__ cs
   dst[j + HALF] = f_to_h(x2);
 }
 
-template <int HD, int NB, bool WIN, int NWG>
+template <int HD, int NB, bool WIN, int NWG, int C = 1>
 void fwd_launch_g(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uint16_t* o, int64_t ldo, float* lse,
                   int W, cudaStream_t st) {
   constexpr int smem = (1 + 2 * NB * NWG) * 64 * (HD + 8) * 2;  // Q, NB x NWG x (K, V)
   static_assert(smem <= 232448, "attention forward shared memory");
   static bool init = false;
   if (!init) {
-    cudaFuncSetAttribute(fwd_kernel<HD, NB, WIN, NWG>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(fwd_kernel<HD, NB, WIN, NWG, C>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     init = true;
   }
-  dim3 grid((S + BQ - 1) / BQ, H, B);
-  launch_k(fwd_kernel<HD, NB, WIN, NWG>, grid, 128 * NWG, smem, st, qkv, ld, S, H, KV, o, ldo, lse, W);
+  dim3 grid((S + BQ - 1) / BQ * C, H, B);
+  if (C == 1) launch_k(fwd_kernel<HD, NB, WIN, NWG, C>, grid, 128 * NWG, smem, st, qkv, ld, S, H, KV, o, ldo, lse, W);
+  else
+    launch_k_cluster(fwd_kernel<HD, NB, WIN, NWG, C>, grid, 128 * NWG, smem, st, dim3(C, 1, 1), qkv, ld, S, H, KV, o,
+                     ldo, lse, W);
 }
 
 // Grids of at most one CTA per SM: several warp-groups per CTA — four at head_dim 64 when the
@@ -651,6 +713,9 @@ void fwd_launch_w(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, 
   if constexpr (HD == 64) {
     if (ctas <= 152 && nqb >= 4) return fwd_launch_g<HD, 2, WIN, 4>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
   }
+  // hd 128 / 256 on grids of at most half the SMs: also split the key blocks over a CTA pair
+  if (HD != 64 && ctas <= 76 && nqb > 1)
+    return fwd_launch_g<HD, HD == 256 ? 1 : 2, WIN, 2, 2>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
   if (ctas <= 152 && nqb > 1) fwd_launch_g<HD, HD == 256 ? 1 : 2, WIN, 2>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
   else if (HD == 256 && ctas > 2 * 152) fwd_launch_g<HD, 1, WIN, 1>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
   else fwd_launch_g<HD, 2, WIN, 1>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
