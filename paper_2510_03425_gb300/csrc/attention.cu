@@ -105,8 +105,11 @@ __global__ void __launch_bounds__(128 * NWG, 1) fwd_kernel(const uint16_t* __res
   auto vs = [&](int buf, int g) { return qs + (2 + 2 * (buf * NWG + g)) * TILE; };
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int wg = warp >> 2, wr = warp & 3;
+  // C = 1: grid (H, B, query blocks), the longest (last) query blocks launched first;
+  // C > 1: grid (query blocks x C, H, B), a cluster's CTAs adjacent in x
   const int crank = C > 1 ? static_cast<int>(blockIdx.x) % C : 0;
-  const int qb = static_cast<int>(blockIdx.x) / C, h = blockIdx.y, b = blockIdx.z;
+  const int qb = C > 1 ? static_cast<int>(blockIdx.x) / C : static_cast<int>(gridDim.z - 1 - blockIdx.z);
+  const int h = C > 1 ? blockIdx.y : blockIdx.x, b = C > 1 ? blockIdx.z : blockIdx.y;
   const int kvh = h / (H / KV);
   const int64_t tok0 = static_cast<int64_t>(b) * S;
   const int q0 = qb * BQ;
@@ -571,12 +574,13 @@ __global__ void __launch_bounds__(128, 1) dkdv_kernel(const BwdArgs a) {
   griddep_launch();
   extern __shared__ __align__(16) uint16_t sm[];
   constexpr int NCH = HD / DC;
-  const int grp = a.H / a.KV, nkb = (a.S + BKV - 1) / BKV;
-  int rest = blockIdx.x;
+  const int grp = a.H / a.KV;
+  // key block slowest-varying: the longest items (key block 0 sees every query block) first
+  const int per = a.KV * a.B * NCH;
+  const int kb = blockIdx.x / per;
+  int rest = blockIdx.x % per;
   const int kvh = rest % a.KV;
   rest /= a.KV;
-  const int kb = rest % nkb;
-  rest /= nkb;
   const int b = rest / NCH, d0 = (rest % NCH) * DC;
   dkdv_run<HD, DC, false, WIN>(a, b, kb, kvh, kvh * grp, grp, d0, 0, 1, nullptr, nullptr, sm);
 }
@@ -587,11 +591,12 @@ __global__ void __launch_bounds__(128, 1) dq_kernel(const BwdArgs a) {
   extern __shared__ __align__(16) uint16_t sm[];
   constexpr int NCH = HD / DC;
   const int nqb = (a.S + BQ - 1) / BQ;
-  int rest = blockIdx.x;
+  // query block slowest-varying, last first: the longest items first
+  const int per = a.H * a.B * NCH;
+  const int qb = nqb - 1 - static_cast<int>(blockIdx.x) / per;
+  int rest = blockIdx.x % per;
   const int h = rest % a.H;
   rest /= a.H;
-  const int qb = rest % nqb;
-  rest /= nqb;
   const int b = rest / NCH, d0 = (rest % NCH) * DC;
   dq_run<HD, DC, false, WIN>(a, b, qb, h, d0, 0, 1, nullptr, sm);
 }
@@ -692,7 +697,7 @@ void fwd_launch_g(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, 
     cudaFuncSetAttribute(fwd_kernel<HD, NB, WIN, NWG, C>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     init = true;
   }
-  dim3 grid((S + BQ - 1) / BQ * C, H, B);
+  const dim3 grid = C > 1 ? dim3((S + BQ - 1) / BQ * C, H, B) : dim3(H, B, (S + BQ - 1) / BQ);
   if (C == 1) launch_k(fwd_kernel<HD, NB, WIN, NWG, C>, grid, 128 * NWG, smem, st, qkv, ld, S, H, KV, o, ldo, lse, W);
   else
     launch_k_cluster(fwd_kernel<HD, NB, WIN, NWG, C>, grid, 128 * NWG, smem, st, dim3(C, 1, 1), qkv, ld, S, H, KV, o,
