@@ -619,7 +619,8 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
       f.vocab < 0 || f.vocab % 64 || f.lora_rank < 0 || f.lora_rank > 32)
     return MEBP_ERR_INVALID_ARG;
   if (!(f.head_dim == 64 || f.head_dim == 128 || f.head_dim == 256)) return MEBP_ERR_UNSUPPORTED;
-  if (f.n_heads / f.n_kv_heads > 8) return MEBP_ERR_UNSUPPORTED;  // query heads per kv head: one cluster
+  // query heads per kv head <= 8: the split attention backward sums at most 8 heads x 2 parts
+  if (f.n_heads / f.n_kv_heads > 8) return MEBP_ERR_UNSUPPORTED;
   if (f.lora_targets && (f.lora_rank % 8)) return MEBP_ERR_UNSUPPORTED;
   if (f.act != MEBP_ACT_SILU && f.act != MEBP_ACT_GELU_TANH) return MEBP_ERR_INVALID_ARG;
   if (f.vocab_chunk < 0 || f.vocab_chunk % 256) return MEBP_ERR_INVALID_ARG;
