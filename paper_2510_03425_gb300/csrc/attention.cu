@@ -381,7 +381,7 @@ __device__ __forceinline__ void dkdv_run(const BwdArgs& a, int b, int kb, int kv
   const int per_head = qb_end - kb;
   const int n_all = h_count * per_head;
   const int n_it = it0 < n_all ? (n_all - it0 + dit - 1) / dit : 0;
-  auto fetch = [&](int i, int buf) {
+  auto fetch = [&](int i, int buf, bool with_dvec) {
     const int it = it0 + i * dit;
     const int h = h_first + it / per_head, q0 = (kb + it % per_head) * BQ;
     load_tile<HD>(qs(buf), a.qkv, a.ld, tok0, q0, S, h * HD, tid);
@@ -390,22 +390,32 @@ __device__ __forceinline__ void dkdv_run(const BwdArgs& a, int b, int kb, int kv
       const int q = q0 + r;
       const int64_t li = (static_cast<int64_t>(b) * H + h) * S + q;
       lse_s(buf)[r] = q < S ? a.lse[li] * kLog2e : 0.0f;
-      dv_s(buf)[r] = q < S ? a.dvec[li] : 0.0f;
+      if (with_dvec) dv_s(buf)[r] = q < S ? a.dvec[li] : 0.0f;
     }
   };
+  // q, k, v, lse (the forward) and dO (two kernels back) are complete when this kernel starts;
+  // dvec comes from the kernel right before: the first tiles load before the wait
   if (n_it > 0) {
     load_tile<HD>(ks, a.qkv, a.ld, tok0, k0, S, (H + kvh) * HD, tid);
     load_tile<HD>(vs, a.qkv, a.ld, tok0, k0, S, (H + KV + kvh) * HD, tid);
-    fetch(0, 0);
+    fetch(0, 0, false);
   }
   cp_async_commit();
+  griddep_wait();
+  if (n_it > 0) {
+    const int h = h_first + it0 / per_head, q0 = (kb + it0 % per_head) * BQ;
+    for (int r = tid; r < BQ; r += 128) {
+      const int q = q0 + r;
+      dv_s(0)[r] = q < S ? a.dvec[(static_cast<int64_t>(b) * H + h) * S + q] : 0.0f;
+    }
+  }
 
   for (int i = 0; i < n_it; ++i) {
     const int buf = i & 1;
     const int it = it0 + i * dit;
     const int q0 = (kb + it % per_head) * BQ;
     if (i + 1 < n_it) {
-      fetch(i + 1, buf ^ 1);
+      fetch(i + 1, buf ^ 1, true);
       cp_async_commit();
       cp_async_wait<1>();
     } else {
@@ -504,9 +514,13 @@ __device__ __forceinline__ void dq_run(const BwdArgs& a, int b, int qb, int h, i
 #pragma unroll
   for (int i = 0; i < 2; ++i) {
     const int row = ra + 8 * i;
-    const int64_t li = (static_cast<int64_t>(b) * H + h) * S + row;
-    lse2[i] = row < S ? a.lse[li] * kLog2e : 0.0f;
-    dvv[i] = row < S ? a.dvec[li] : 0.0f;
+    lse2[i] = row < S ? a.lse[(static_cast<int64_t>(b) * H + h) * S + row] * kLog2e : 0.0f;
+  }
+  griddep_wait();  // dvec comes from the kernel right before (the tiles above are older)
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const int row = ra + 8 * i;
+    dvv[i] = row < S ? a.dvec[(static_cast<int64_t>(b) * H + h) * S + row] : 0.0f;
   }
   float dq[NC][4];
 #pragma unroll
@@ -570,8 +584,7 @@ __device__ __forceinline__ void dq_run(const BwdArgs& a, int b, int qb, int h, i
 // then dQ with one CTA per (query block, head), as two launches writing dqkv directly.
 template <int HD, int DC, bool WIN>
 __global__ void __launch_bounds__(128, 1) dkdv_kernel(const BwdArgs a) {
-  griddep_wait();
-  griddep_launch();
+  griddep_launch();  // the item functions wait (after issuing the loads of older data)
   extern __shared__ __align__(16) uint16_t sm[];
   constexpr int NCH = HD / DC;
   const int grp = a.H / a.KV;
@@ -586,8 +599,7 @@ __global__ void __launch_bounds__(128, 1) dkdv_kernel(const BwdArgs a) {
 }
 template <int HD, int DC, bool WIN>
 __global__ void __launch_bounds__(128, 1) dq_kernel(const BwdArgs a) {
-  griddep_wait();
-  griddep_launch();
+  griddep_launch();  // the item functions wait (after issuing the loads of older data)
   extern __shared__ __align__(16) uint16_t sm[];
   constexpr int NCH = HD / DC;
   const int nqb = (a.S + BQ - 1) / BQ;
@@ -607,8 +619,7 @@ __global__ void __launch_bounds__(128, 1) dq_kernel(const BwdArgs a) {
 // bwd_finish_kernel sums them.
 template <int HD, int DC, bool WIN>
 __global__ void __launch_bounds__(128, 1) bwd_split_kernel(const BwdArgs a) {
-  griddep_wait();
-  griddep_launch();
+  griddep_launch();  // the item functions wait (after issuing the loads of older data)
   extern __shared__ __align__(16) uint16_t sm[];
   constexpr int NCH = HD / DC;
   const int H = a.H, P = a.P, nb = (a.S + BQ - 1) / BQ;
