@@ -389,7 +389,7 @@ __device__ __forceinline__ void dkdv_run(const BwdArgs& a, int b, int kb, int kv
     for (int r = tid; r < BQ; r += 128) {
       const int q = q0 + r;
       const int64_t li = (static_cast<int64_t>(b) * H + h) * S + q;
-      lse_s(buf)[r] = q < S ? a.lse[li] * kLog2e : 0.0f;
+      lse_s(buf)[r] = q < S ? __ldcg(a.lse + li) * kLog2e : 0.0f;  // L2 only: may run before the wait
       if (with_dvec) dv_s(buf)[r] = q < S ? a.dvec[li] : 0.0f;
     }
   };
@@ -514,7 +514,7 @@ __device__ __forceinline__ void dq_run(const BwdArgs& a, int b, int qb, int h, i
 #pragma unroll
   for (int i = 0; i < 2; ++i) {
     const int row = ra + 8 * i;
-    lse2[i] = row < S ? a.lse[(static_cast<int64_t>(b) * H + h) * S + row] * kLog2e : 0.0f;
+    lse2[i] = row < S ? __ldcg(a.lse + (static_cast<int64_t>(b) * H + h) * S + row) * kLog2e : 0.0f;
   }
   griddep_wait();  // dvec comes from the kernel right before (the tiles above are older)
 #pragma unroll

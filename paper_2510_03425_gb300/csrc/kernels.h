@@ -20,11 +20,13 @@ inline void count_launch(int n = 1) { g_launches.fetch_add(n, std::memory_order_
 // is a normal launch (pdl_entry() marks it), so no kernel of one call overlaps an earlier call:
 // the fused GEMM may then read the packed weights before its wait (they are written only by
 // mebp_compress_weights, a separate call).
-// A kernel starts only after every CTA of its predecessor has triggered; a predecessor that waits
-// before it triggers has then seen everything before it complete.  Kernels whose predecessor is
-// such a kernel may therefore read, before their own wait, data written two or more kernels back
-// (the attention backward's q/k/v, lse and dO tiles; the skinny LoRA kernel's shadows), and read
-// after the wait only what the kernel right before wrote.
+// A kernel starts only after every CTA of its predecessor has triggered.  So, at its start,
+// everything written before the nearest preceding kernel that waits before it triggers is
+// complete.  Every kernel here waits first except the fused GEMMs (whose weight reads need no
+// wait) and the attention backward's dK/dV, dQ and split kernels; those issue their q/k/v, lse and
+// dO loads before the wait, relying on the dvec kernel (waits first) before them, and read dvec
+// after it.  Early reads go through L2 only (cp.async.cg, __ldcg): until the wait, L1 may still
+// hold lines of a reused buffer read by an earlier kernel on the same SM.
 void pdl_entry();   // the calling thread's next launch is a normal launch
 bool pdl_take();    // may this launch use PDL? (consumes the entry mark)
 

@@ -138,6 +138,7 @@ template <int NT>
 __global__ void __launch_bounds__(128) skinny_slab_kernel(const uint16_t* __restrict__ X, int64_t ldx, int64_t M,
                                                           int K, const uint16_t* __restrict__ W, int64_t ldw,
                                                           float alpha, uint16_t* __restrict__ out, int64_t ldo) {
+  griddep_wait();  // W may come from the kernel right before (a single linear builds its shadow first)
   griddep_launch();
   constexpr int JR = NT * 8, LDR = JR + 4;
   extern __shared__ __align__(16) uint8_t sm[];
@@ -148,13 +149,10 @@ __global__ void __launch_bounds__(128) skinny_slab_kernel(const uint16_t* __rest
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int64_t m0 = static_cast<int64_t>(blockIdx.x) * 16;
   const int kc = K / 8;
-  // W (a LoRA shadow, built before the step's first block) is complete when this kernel starts
-  // (the kernel two places back in the stream has finished): it loads before the wait for X
   for (int c = tid; c < JR * kc; c += 128) {
     const int r = c / kc, cc = c % kc;
     cp_async16(smem_u32(ws + r * LDS + cc * 8), W + r * ldw + cc * 8, true);
   }
-  griddep_wait();
   for (int c = tid; c < 16 * kc; c += 128) {
     const int r = c / kc, cc = c % kc;
     const int64_t gm = m0 + r;
