@@ -1,16 +1,17 @@
 """Benchmark of one MeBP LoRA training step (Algorithm 1) on GB300.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--config C] [--impl gb300|reference]
+                    [--per-block] [--min-memory] [--gemm-bench] [--table2] [--launch-list]
 
 A step = embed -> checkpointed forward loop over all blocks -> LM-head cross-entropy
 (forward + backward, vocabulary-chunked) -> reverse loop of block recompute + backward,
 producing the loss and every LoRA gradient (mebp_lora_step).  The default workload is the
-full Qwen2.5-0.5B-shaped model (24 blocks, vocab 151936, batch 1 x seq 512, LoRA r8 on
-q/k/v/o, 4-bit group-64 base weights).  Prints one JSON line (rank 0).
+largest preset, the Gemma3-4B-shaped model (34 blocks, vocab 262144, batch 8 x seq 2048, LoRA
+r32 on all seven linears, 4-bit group-64 base weights).  Prints one JSON line (rank 0).
 
---impl reference times the CPU oracle (plain numpy fp64) on the host cores, on a bounded
-sample of the same workload (one block's forward + recompute + backward and an LM-head
-token sample), extrapolated to the step.
+--impl reference times the CPU oracle (plain numpy fp64) on the host cores, each step one
+bounded sample of the same workload (one block's forward + recompute + backward on part of a
+sequence and an LM-head sample), extrapolated to the step.
 """
 from __future__ import annotations
 
@@ -61,38 +62,97 @@ def peaks():
 
 
 # ----------------------------------------------------------------------------- CPU oracle sample
-def oracle_sample(d, lm_tokens: int = 32):
-    """Time the oracle on one block (forward, recompute, backward) and an LM-head token
-    sample; return (tokens/s extrapolated to the whole step, description)."""
-    from oracle import model as OM
-    from oracle import quant
+def blas_threads() -> int:
+    """Threads the oracle's numpy BLAS uses (threadpoolctl when present, else the environment or
+    the core count)."""
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads", 0) for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+        if os.environ.get(k, "").isdigit():
+            return int(os.environ[k])
+    return os.cpu_count() or 1
 
-    W = synth.block_weights(d, 0)
-    L = OM.lora64(synth.lora_weights(d, 0))
-    x = synth.hidden_input(d).astype(np.float64)
-    G = synth.upstream_grad(d).astype(np.float64)
-    t0 = time.perf_counter()
-    pm = OM.PackedModel.compress([W])
-    Wd = pm.decompress_block(0)
-    OM.block_objective(x, Wd, L, G, d)
-    t_block = time.perf_counter() - t0
-    t_lm = 0.0
-    if d.vocab:
-        E, gf = synth.embedding(d)
-        qE = quant.compress(E)
-        t1 = time.perf_counter()
-        Ed = quant.dequant(*qE)
-        t_deq = time.perf_counter() - t1
-        h = x[:lm_tokens]
-        tg = synth.token_ids(d).reshape(-1)[:lm_tokens].astype(np.int64)
-        t2 = time.perf_counter()
-        OM.lm_head_ce(h, gf.astype(np.float64), Ed, tg, d.eps)
-        t_lm = t_deq + (time.perf_counter() - t2) * d.tokens / lm_tokens
-    t_step = d.n_layers * t_block + t_lm
-    desc = (f"oracle (numpy fp64) on 1 of {d.n_layers} blocks at the full {d.tokens} tokens (compress + decompress + "
-            f"forward + recompute + backward) and the LM head on {lm_tokens} of {d.tokens} tokens, extrapolated "
-            f"linearly to the step")
-    return d.tokens / t_step, desc
+
+class OracleSample:
+    """The oracle (numpy fp64) on a bounded sample of one training step, extrapolated to the step.
+
+    Sample: block 0 decompressed (LazyLoadAndDecompressWeights), its forward, then the recompute +
+    backward (block_objective) on the first `block_tokens` tokens of one sequence; and the LM head
+    (final norm + logits + CE + dE/dh) on `lm_tokens` tokens against a `lm_rows`-row slice of the
+    decompressed vocabulary.  Extrapolation is linear: blocks x L x (tokens / block_tokens), LM
+    head x (tokens / lm_tokens) x (V / lm_rows).  Attention's quadratic term is extrapolated
+    linearly too, which slightly flatters the CPU.  Compression (done once when a model is loaded)
+    is outside the timed sample.  full=True times the whole Algorithm 1 step instead (--cpu-full-step;
+    about 40 s on 8 cores for the Qwen2.5-0.5B shape, hours for the larger ones)."""
+
+    def __init__(self, d, block_tokens: int = 256, lm_tokens: int = 32, lm_rows: int = 16384, full: bool = False):
+        from oracle import model as OM
+        from oracle import quant
+        self.d = d
+        self.OM = OM
+        self.full = full and d.vocab > 0
+        if self.full:
+            self.blocks = [synth.block_weights(d, i) for i in range(d.n_layers)]
+            self.E, self.gf = synth.embedding(d)
+            self.pm = OM.PackedModel.compress(self.blocks, self.E, self.gf)
+            self.loras = [synth.lora_weights(d, i) for i in range(d.n_layers)]
+            self.ids = synth.token_ids(d)
+            self.desc = (f"oracle (numpy fp64) full Algorithm 1 step: {d.n_layers} blocks, {d.tokens} tokens, "
+                         f"vocab {d.vocab} (no extrapolation)")
+            return
+        bt = min(block_tokens, d.seq)
+        self.bt = bt
+        d1 = d.with_(batch=1, seq=bt)
+        self.d1 = d1
+        self.pm = OM.PackedModel.compress([synth.block_weights(d, 0)])
+        self.L = OM.lora64(synth.lora_weights(d, 0))
+        self.x = synth.hidden_input(d)[:bt].astype(np.float64)
+        self.G = synth.upstream_grad(d)[:bt].astype(np.float64)
+        self.lm = None
+        if d.vocab:
+            rows = min(lm_rows, d.vocab)
+            E, gf = synth.embedding(d, rows=rows)
+            self.qE = quant.compress(E)
+            self.gf = gf.astype(np.float64)
+            rng = np.random.default_rng(3)
+            self.h = rng.standard_normal((lm_tokens, d.hidden))
+            self.tg = rng.integers(0, rows, lm_tokens).astype(np.int64)
+            self.lm = (rows, lm_tokens)
+        self.desc = (f"oracle (numpy fp64): block 0 (decompress, forward, recompute + backward) on {bt} of the "
+                     f"{d.seq} tokens of one sequence, extrapolated x{d.n_layers} blocks x{d.tokens // bt}; LM head "
+                     f"(decompress, final norm, logits, CE, dE/dh) on {lm_tokens} tokens x {self.lm[0] if self.lm else 0}"
+                     f" vocabulary rows, extrapolated x{d.tokens // lm_tokens} x{d.vocab / max(1, self.lm[0] if self.lm else 1):.0f}")
+
+    def run(self):
+        """Returns (seconds the sample took, seconds of the whole step it stands for)."""
+        OM, d = self.OM, self.d
+        if self.full:
+            t0 = time.perf_counter()
+            OM.mebp_backpropagation(self.pm, self.loras, self.ids, d)
+            t = time.perf_counter() - t0
+            return t, t
+        from oracle import quant
+        t0 = time.perf_counter()
+        Wd = self.pm.decompress_block(0)
+        OM.block_forward(self.x, Wd, self.L, self.d1)
+        OM.block_objective(self.x, Wd, self.L, self.G, self.d1)
+        t_blk = time.perf_counter() - t0
+        t_lm = 0.0
+        if self.lm:
+            t1 = time.perf_counter()
+            Ed = quant.dequant(*self.qE)
+            OM.lm_head_ce(self.h, self.gf, Ed, self.tg, d.eps)
+            t_lm = time.perf_counter() - t1
+        sample = t_blk + t_lm
+        full = t_blk * d.n_layers * (d.tokens / self.bt)
+        if self.lm:
+            full += t_lm * (d.tokens / self.lm[1]) * (d.vocab / self.lm[0])
+        return sample, full
 
 
 # ----------------------------------------------------------------------------- clocks
@@ -162,6 +222,60 @@ def build_model(ctx, d, device):
     return DeviceModel(blocks, emb, gf)
 
 
+GEMM_SOURCES = ("gemm.cu", "gemm_s.cu", "dequant.cuh", "common.cuh")
+TRAFFIC_PROFILE = os.path.join(ROOT, "profiles", "dequant_gemm_gemma4b_step_traffic.md")
+
+
+def gemm_sources_sha() -> str:
+    import hashlib
+    h = hashlib.sha256()
+    for f in GEMM_SOURCES:
+        with open(os.path.join(ROOT, "paper_2510_03425_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def gemm_traffic(config: int):
+    """DRAM bytes per fused-GEMM launch of one step from the committed ncu summary, or None when
+    the summary is for another workload or the kernel sources changed since it was taken."""
+    import re
+    try:
+        with open(TRAFFIC_PROFILE) as f:
+            txt = f.read()
+    except OSError:
+        return None, "no ncu summary"
+    kv = dict(re.findall(r"^([a-z_]+):\s*(\S+)\s*$", txt, flags=re.M))
+    if kv.get("workload_config") != str(config):
+        return None, "ncu summary is for another workload"
+    if kv.get("kernel_sources_sha256") != gemm_sources_sha():
+        return None, "kernel changed since the ncu capture"
+    return float(kv["traffic_per_launch_bytes"]), os.path.relpath(TRAFFIC_PROFILE, ROOT)
+
+
+def make_step(M, ctx, mstruct, ls, ids, loss, st):
+    def step():
+        M.mebp_lora_step(ctx.handle, mstruct, ls.lora_array(), ids, loss, ls.grads_array(), False, st)
+    return step
+
+
+def time_steps(step, n, st):
+    import torch
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(st)
+    for _ in range(n):
+        step()
+    e1.record(st)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / 1e3
+
+
+def model_bytes(model, ls):
+    pw = sum(t.numel() * t.element_size() for b in model.blocks for lin in (b.qkv, b.o, b.gate_up, b.down)
+             for t in (lin.qpack, lin.scales))
+    pw += model.embed.qpack.numel() + model.embed.scales.numel() * 2
+    return pw, 2 * 4 * ls.n  # packed weights (+ scales); LoRA masters + gradients (fp32)
+
+
 def run_gpu(args, d, rank, world, local_rank):
     import torch
 
@@ -174,7 +288,7 @@ def run_gpu(args, d, rank, world, local_rank):
     if world > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
-    ctx = Context(d, device=local_rank)
+    ctx = Context(d, device=local_rank, min_memory=args.min_memory)
     model = build_model(ctx, d, device)
     ls = LoraSet([synth.lora_weights(d, i) for i in range(d.n_layers)], device=device)
     ids_host = torch.from_numpy(synth.token_ids(d, seed=2 + rank)).pin_memory()
@@ -185,93 +299,144 @@ def run_gpu(args, d, rank, world, local_rank):
     # a dedicated stream: mebp_lora_step replays a captured CUDA graph on non-default streams
     st = torch.cuda.Stream(device)
     torch.cuda.set_stream(st)
-
-    def step():
-        M.mebp_lora_step(ctx.handle, mstruct, ls.lora_array(), ids, loss, ls.grads_array(), False, st)
+    step = make_step(M, ctx, mstruct, ls, ids, loss, st)
 
     gpu_index = local_rank
     vis = os.environ.get("CUDA_VISIBLE_DEVICES")
     if vis and vis.split(",")[local_rank].strip().isdigit():
         gpu_index = int(vis.split(",")[local_rank])
-    clocks = ClockSampler(gpu_index)
+    torch.cuda.reset_peak_memory_stats(device)
     for _ in range(args.warmup):
         step()
     ctx.sync()
+    free0, total = torch.cuda.mem_get_info(device)
     # ---- timed region: K steps, inputs resident in HBM
+    clocks = ClockSampler(gpu_index)
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
     n0 = M.mebp_kernel_launches()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(st)
-    for _ in range(args.steps):
-        step()
-    e1.record(st)
-    torch.cuda.synchronize()
+    t = time_steps(step, args.steps, st)
     launches = M.mebp_kernel_launches() - n0
     if dist:
         dist.barrier()
     clk = clocks.stop()
     ctx.sync()
-    t = e0.elapsed_time(e1) / 1e3
+    free1, _ = torch.cuda.mem_get_info(device)
     if dist:
         tt = torch.tensor([t], device=device)
         dist.all_reduce(tt, op=dist.ReduceOp.MAX)
         t = float(tt.item())
     value = world * d.tokens * args.steps / t
 
-    # ---- GEMM roofline: CUDA events around every fused dequant-GEMM launch of K more steps
+    # ---- per-kernel CUDA events over K more steps (run eagerly: the events order each launch on
+    # its stream), the fused GEMMs' union of busy intervals, and the step's wall time meanwhile
+    kp = max(3, args.steps // 4)
     M.mebp_profile_begin(ctx.handle)
-    for _ in range(args.steps):
-        step()
+    t_prof = time_steps(step, kp, st)
     prof = M.mebp_profile_end(ctx.handle)
+    kstats = M.mebp_profile_kernels(ctx.handle)
 
     # ---- end to end through the public API: ids host->device, step, loss device->host
     ctx.sync()
     h2d = ids_host.numel() * ids_host.element_size()
     d2h = loss.numel() * loss.element_size()
-    e2, e3 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e2.record(st)
-    for _ in range(args.steps):
+
+    def e2e_step():
         ids.copy_(ids_host, non_blocking=True)
         step()
         loss_host.copy_(loss, non_blocking=True)
-    e3.record(st)
-    torch.cuda.synchronize()
-    te = e2.elapsed_time(e3) / 1e3
+    te = time_steps(e2e_step, args.steps, st)
     if dist:
         tt = torch.tensor([te], device=device)
         dist.all_reduce(tt, op=dist.ReduceOp.MAX)
         te = float(tt.item())
     ctx.sync()
+    peak_torch = torch.cuda.max_memory_allocated(device)
+    ws = M.mebp_workspace_bytes(ctx.handle)
+    breakdown, nsets = M.mebp_workspace_breakdown(ctx.handle)
+    pw_bytes, lora_bytes = model_bytes(model, ls)
+
+    mm = None
+    kstats_serial, kp_serial = None, 0
+    if rank == 0 and world == 1 and not args.min_memory and args.compare_min_memory:
+        # the paper's bound: one set of block intermediates (no recompute / backward overlap)
+        c2 = Context(d, device=local_rank, min_memory=True)
+        step2 = make_step(M, c2, mstruct, ls, ids, loss, st)
+        for _ in range(3):
+            step2()
+        c2.sync()
+        n2 = max(3, args.steps // 2)
+        t2 = time_steps(step2, n2, st)
+        c2.sync()
+        ws2 = M.mebp_workspace_bytes(c2.handle)
+        mm = {"workspace_bytes": ws2, "peak_device_bytes": peak_torch + ws2,
+              "workspace": M.mebp_workspace_breakdown(c2.handle)[0], "ms_per_step": 1e3 * t2 / n2,
+              "tokens_per_s": d.tokens * n2 / t2, "slowdown": (t2 / n2) / (t / args.steps)}
+        # one stream, nothing concurrent: per-kernel event times free of interference
+        kp_serial = 3
+        M.mebp_profile_begin(c2.handle)
+        time_steps(step2, kp_serial, st)
+        M.mebp_profile_end(c2.handle)
+        kstats_serial = M.mebp_profile_kernels(c2.handle)
+        c2.close()
 
     if rank != 0:
+        ctx.close()
         if dist:
             dist.destroy_process_group()
         return None
     pk, src = peaks()
-    long_step = t / args.steps > 1.0
-    peak = pk["bf16_tflops_sustained"] if long_step else pk["bf16_tflops"]
+    sustained = t > 1.0  # the GEMMs run inside a seconds-long loop of steps
+    peak = pk["bf16_tflops_sustained"] if sustained else pk["bf16_tflops"]
     achieved = prof.gemm_flops / (prof.gemm_ms / 1e3) / 1e12 if prof.gemm_ms > 0 else None
-    weights_mb = sum(b.qkv.qpack.numel() + b.o.qpack.numel() + b.gate_up.qpack.numel() + b.down.qpack.numel()
-                     for b in model.blocks) / 2**20 * (1 + 1 / 16)
+    busy_share = (prof.gemm_busy_ms / 1e3) / t_prof if t_prof > 0 else None
+    assert busy_share is None or busy_share <= 1.0 + 1e-6, busy_share
+    traffic, traffic_src = gemm_traffic(args.config) if not (args.gemma3 or args.min_memory) else (None, "n/a")
+    ks_src, ks_n = (kstats_serial, kp_serial) if kstats_serial else (kstats, kp)
+    tot_ms = sum(v["ms"] for v in ks_src.values()) or 1.0
+    kernels = {"how": ("CUDA events around every launch of " + str(ks_n) + " eager steps on one stream "
+                       "(min_memory context: nothing runs concurrently); bytes and flops algorithmic"
+                       if kstats_serial else
+                       "CUDA events around every launch of " + str(ks_n) + " eager steps (three streams: launches "
+                       "overlap, times include interference)")}
+    for name, v in sorted(ks_src.items(), key=lambda kv: -kv[1]["ms"]):
+        e = {"launches_per_step": v["launches"] / ks_n, "ms_per_step": v["ms"] / ks_n,
+             "share_of_kernel_time": v["ms"] / tot_ms}
+        if v["bytes"] and v["ms"]:
+            e["gbs"] = v["bytes"] / (v["ms"] / 1e3) / 1e9
+            e["hbm_frac"] = e["gbs"] / pk["hbm_gbs"]
+        if v["flops"] and v["ms"]:
+            e["tflops"] = v["flops"] / (v["ms"] / 1e3) / 1e12
+        kernels[name] = e
     out = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1e3 * t / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f16", "data": "synthetic",
         "config": {"workload": workload_name(d), "config_index": args.config, "global_batch": world * d.batch,
                    "seq_len": d.seq, "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-                   "l2": f"inputs larger than L2: {weights_mb:.0f} MB of packed block weights plus the "
-                         f"{d.vocab}x{d.hidden} packed LM head are streamed every step"},
-        "roofline": {"kernel": "dequant_gemm_kernel (fused 4-bit dequant GEMM, tcgen05)", "bound": "tensor",
-                     "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                     "frac": (achieved / peak) if achieved else None, "traffic": None,
-                     "peak_source": f"{src} {'sustained' if long_step else 'burst'} dense bf16 GEMM rate "
+                   "l2": f"inputs larger than L2: {pw_bytes / 2**20:.0f} MB of packed weights are streamed every "
+                         "step (no flush needed)"},
+        "roofline": {"kernel": "dequant_gemm_kernel (fused 4-bit dequant GEMM, tcgen05), every launch of the step",
+                     "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": (achieved / peak) if achieved else None, "traffic": traffic,
+                     "algorithmic_bytes": prof.gemm_bytes / max(prof.gemm_launches, 1),
+                     "traffic_source": traffic_src,
+                     "peak_source": f"{src} {'sustained' if sustained else 'burst'} dense bf16 GEMM rate "
                                     "(MEASURED_PEAKS.json); fp16 and bf16 share the kind::f16 rate (nominal ratio 1)",
-                     "launches_per_step": prof.gemm_launches / args.steps,
-                     "share_of_step": (prof.gemm_ms / 1e3) / t if t > 0 else None,
+                     "how": f"CUDA events on the launching stream around every fused-GEMM launch of {kp} eager "
+                            "steps; achieved = sum of algorithmic flops / sum of launch durations",
+                     "launches_per_step": prof.gemm_launches / kp,
+                     "busy_share_of_step": busy_share,
                      "fwd_tflops": prof.fwd_flops / max(prof.fwd_ms, 1e-9) / 1e9,
                      "dx_tflops": prof.dx_flops / max(prof.dx_ms, 1e-9) / 1e9},
+        "kernels": kernels,
+        "memory": {"peak_device_bytes": peak_torch + ws, "torch_peak_allocated_bytes": peak_torch,
+                   "library_workspace_bytes": ws, "workspace": breakdown, "intermediate_sets": nsets,
+                   "packed_weights_bytes": pw_bytes, "lora_masters_and_grads_bytes": lora_bytes,
+                   "device_used_bytes": total - free0,
+                   "step_allocates_nothing": free0 == free1,
+                   **({"min_memory": mm} if mm else {})},
         "e2e": {"value": world * d.tokens * args.steps / te, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": int(launches),
@@ -280,6 +445,90 @@ def run_gpu(args, d, rank, world, local_rank):
     ctx.close()
     if dist:
         dist.destroy_process_group()
+    return out
+
+
+def per_block(args, d, reps: int = 3):
+    """Analogue of the paper's Fig. 2 (per-layer time and memory): one eager step through the
+    public entry points, phase by phase (embedding, forward_i of every block, the LM head + CE,
+    backward_i of every block in reverse), each phase bracketed by CUDA events on the stream and
+    an NVTX range (emb, f_i, lm, b_i).  Memory per phase is the working set the phase touches
+    beyond the resident weights, LoRA state and checkpoints, from the workspace breakdown."""
+    import torch
+
+    from paper_2510_03425_gb300 import mebp as M
+    from paper_2510_03425_gb300.model import Context, LoraSet
+    device = torch.device("cuda", 0)
+    ctx = Context(d, device=0)
+    model = build_model(ctx, d, device)
+    ls = LoraSet([synth.lora_weights(d, i) for i in range(d.n_layers)], device=device)
+    ids = torch.from_numpy(synth.token_ids(d)).to(device)
+    tg = torch.cat([ids[:, 1:], torch.full((d.batch, 1), -1, dtype=ids.dtype, device=device)], 1).reshape(-1)
+    T, D, L = d.tokens, d.hidden, d.n_layers
+    ck = torch.empty((L + 1, T, D), device=device)
+    dy = torch.empty((T, D), device=device)
+    dx = torch.empty((T, D), device=device)
+    loss = torch.zeros(1, device=device)
+    st = torch.cuda.Stream(device)
+    torch.cuda.set_stream(st)
+    E = model.embed.struct()
+    blk = [b.struct() for b in model.blocks]
+    lor = [ls.layer(i) for i in range(L)]
+    grd = [ls.layer_grads(i) for i in range(L)]
+    names = ["emb"] + [f"f_{i}" for i in range(L)] + ["lm"] + [f"b_{i}" for i in reversed(range(L))]
+    times = {n: [] for n in names}
+    for rep in range(reps + 1):
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(names) + 1)]
+        k = 0
+        ev[0].record(st)
+
+        def mark(name):
+            nonlocal k
+            torch.cuda.nvtx.range_pop()
+            k += 1
+            ev[k].record(st)
+        torch.cuda.nvtx.range_push("emb")
+        M.mebp_embed(ctx.handle, E, ids.reshape(-1), ck[0], stream=st)
+        mark("emb")
+        for i in range(L):
+            torch.cuda.nvtx.range_push(f"f_{i}")
+            M.mebp_block_recompute_fwd(ctx.handle, i, blk[i], lor[i], ck[i], ck[i + 1], d.batch, d.seq, False, st)
+            mark(f"f_{i}")
+        torch.cuda.nvtx.range_push("lm")
+        M.mebp_lmhead_ce_fwd_bwd(ctx.handle, E, model.final_norm, ck[L], tg, loss, dy, stream=st)
+        mark("lm")
+        for i in reversed(range(L)):
+            torch.cuda.nvtx.range_push(f"b_{i}")
+            M.mebp_block_bwd(ctx.handle, i, blk[i], lor[i], ck[i], dy, dx, grd[i], d.batch, d.seq, False, st)
+            mark(f"b_{i}")
+            dy, dx = dx, dy
+        torch.cuda.synchronize()
+        ctx.sync(st)
+        if rep == 0:
+            continue  # warm-up
+        for j, n in enumerate(names):
+            times[n].append(ev[j].elapsed_time(ev[j + 1]))
+    br, nsets = M.mebp_workspace_breakdown(ctx.handle)
+    act = T * D * 4
+    fwd_set = br["forward_sets"] / nsets
+    mem = {"emb": act, "lm": br["lm_head"] + 2 * act}
+    for i in range(L):
+        mem[f"f_{i}"] = fwd_set + 2 * act
+        mem[f"b_{i}"] = fwd_set + br["backward"] + br["attention_split"] + 3 * act
+    pw, lb = model_bytes(model, ls)
+    ms = {n: statistics.median(v) for n, v in times.items()}
+    f_mean = statistics.mean(ms[f"f_{i}"] for i in range(L))
+    b_mean = statistics.mean(ms[f"b_{i}"] for i in range(L))
+    out = {"per_block": workload_name(d), "reps": reps, "ms": ms, "working_set_bytes": mem,
+           "resident_bytes": {"packed_weights": pw, "lora_masters_and_grads": lb,
+                              "checkpoints": br["checkpoints"], "lora_shadows": br["lora_shadows"]},
+           "summary": {"forward_block_ms": f_mean, "backward_block_ms": b_mean,
+                       "backward_over_forward_time": b_mean / f_mean,
+                       "backward_over_forward_memory": mem["b_0"] / mem["f_0"],
+                       "lm_head_ms": ms["lm"], "lm_head_over_backward_block": ms["lm"] / b_mean,
+                       "lm_head_working_set_over_backward_block": mem["lm"] / mem["b_0"],
+                       "step_ms": sum(ms.values())}}
+    ctx.close()
     return out
 
 
@@ -515,17 +764,26 @@ def gemm_bench(config: int, m_tokens=None, reps: int = 10, warmup: int = 3, shap
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=150)
+    ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--config", type=int, default=1, help="workload preset 0..4 (default 1)")
+    ap.add_argument("--config", type=int, default=4,
+                    help="workload preset 0..4 (default 4: the Gemma3-4B-shaped full step, the largest)")
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-full-step", action="store_true",
+                    help="the CPU oracle times the whole step instead of a bounded sample (small configs only)")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="only the step measurement (no isolated GEMM / AdamW figures, no min-memory comparison)")
+    ap.add_argument("--min-memory", action="store_true",
+                    help="run the step with one set of block intermediates (the paper's memory bound)")
     ap.add_argument("--gemm-bench", action="store_true",
                     help="time only the fused dequant-GEMMs at the config's projection shapes")
     ap.add_argument("--gemm-m", type=int, default=None, help="token count M for --gemm-bench")
     ap.add_argument("--gemm-shapes", default=None, help="comma list of qkv,o,gate_up,down for --gemm-bench")
     ap.add_argument("--table2", action="store_true",
                     help="decompression-overhead (Table 2) and sequence-length (Table 3) analogues")
+    ap.add_argument("--per-block", action="store_true",
+                    help="Fig. 2 analogue: per-phase time (CUDA events, NVTX emb / f_i / lm / b_i) and memory")
     ap.add_argument("--gemma3", action="store_true",
                     help="Gemma-shaped configs (2, 4) with the Gemma3 block options on")
     ap.add_argument("--launch-list", action="store_true",
@@ -541,6 +799,7 @@ def main():
         if d.act != "gelu_tanh":
             ap.error("--gemma3 applies to the Gemma-shaped configs 2 and 4")
         d = gemma3_extras(d)
+    args.compare_min_memory = not args.no_extras
 
     if args.gemm_bench:
         out = gemm_bench(args.config, args.gemm_m, reps=args.steps, warmup=args.warmup,
@@ -554,24 +813,35 @@ def main():
     if args.table2:
         print(json.dumps(table2()), flush=True)
         return
+    if args.per_block:
+        print(json.dumps(per_block(args, d)), flush=True)
+        return
 
     if args.impl == "reference":
+        # the CPU oracle as it stands, on the host cores: each step one bounded sample of the
+        # workload, its throughput extrapolated to the whole step (see OracleSample)
         if rank != 0:
             return
-        cores = os.cpu_count()
-        vals = []
+        smp = OracleSample(d, full=args.cpu_full_step)
+        samples, fulls = [], []
         for i in range(args.warmup + args.steps):
-            v, desc = oracle_sample(d)
+            ts, tf = smp.run()
             if i >= args.warmup:
-                vals.append(v)
-        v = statistics.mean(vals)
+                samples.append(ts)
+                fulls.append(tf)
+        tf = statistics.mean(fulls)
+        v = d.tokens / tf
+        cores = blas_threads()
         print(json.dumps({
             "metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": 1e3 * d.tokens / v, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "warmup": args.warmup, "ms_per_step": 1e3 * statistics.mean(samples),
+            "extrapolated_ms_per_full_step": 1e3 * tf, "extrapolated": not smp.full,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "impl": "reference",
             "config": {"workload": workload_name(d), "config_index": args.config, "global_batch": d.batch,
-                       "seq_len": d.seq, "parallelism": "host cores"},
-            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": desc},
+                       "seq_len": d.seq, "parallelism": "single GPU",
+                       "l2": "n/a (host cores; each step is one bounded sample of the workload)"},
+            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": smp.desc},
             "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
         }), flush=True)
         return
@@ -579,14 +849,15 @@ def main():
     out = run_gpu(args, d, rank, world, local_rank)
     if out is None:
         return
-    if world == 1:
+    if world == 1 and not args.no_extras:
         # second half of the metric: the fused dequant-GEMM alone at the largest workload's shapes
         out["fused_gemm_isolated"] = gemm_bench(4)
         out["adamw_isolated"] = adamw_bench(4)
     if world == 1 and not args.no_cpu_baseline:
-        v, desc = oracle_sample(d)
-        out["cpu_baseline"] = {"value": v, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
-                               "sample": desc}
+        smp = OracleSample(d, full=args.cpu_full_step)
+        ts, tf = smp.run()
+        out["cpu_baseline"] = {"value": d.tokens / tf, "unit": "tokens/s", "cores": blas_threads(), "kind": "oracle",
+                               "sample": smp.desc, "sample_seconds": ts, "extrapolated": not smp.full}
     print(json.dumps(out), flush=True)
 
 

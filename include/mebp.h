@@ -38,8 +38,11 @@ enum {
   MEBP_ERR_TIMEOUT = 4,      /* a device-side bounded wait expired (kernel returned early)       */
   MEBP_ERR_UNSUPPORTED = 5,  /* configuration outside what the kernels implement                 */
   MEBP_ERR_DEVICE = 6,       /* a kernel flagged bad input (e.g. token id out of range)          */
-  MEBP_ERR_SCRATCH = 7       /* mebp_linear_fwd_noalloc: the request needs more than the fixed
+  MEBP_ERR_SCRATCH = 7,      /* mebp_linear_fwd_noalloc: the request needs more than the fixed
                                 scratch array (MEBP_NOALLOC_SCRATCH_BYTES) holds                  */
+  MEBP_ERR_NONFINITE = 8     /* an fp16 intermediate (a GEMM output stored as fp16, the gated-MLP
+                                product or its gradient) overflowed the fp16 range (|x| > 65504)
+                                or was NaN; reported by mebp_sync()                                */
 };
 
 /* LoRA target index (bit i of mebp_model_cfg.lora_targets). */
@@ -77,6 +80,10 @@ typedef struct {
   int32_t sliding_window;
   int32_t global_every;
   float rope_theta_local;
+  /* min_memory != 0: one set of block intermediates (Section 3, "Runtime implementation": only
+   * one subgraph's intermediates are held at a time).  0: a second set lets mebp_lora_step run the
+   * recompute of block i-1 beside the backward of block i (same results, more memory). */
+  int32_t min_memory;
 } mebp_model_cfg;
 
 /* ---- compressed base weight (Section 3, "Base model weights compression") -------------------
@@ -150,8 +157,25 @@ const char* mebp_last_error(const mebp_ctx* ctx);
 /* Synchronises `stream`, then reads and clears the device error word: returns
  * MEBP_ERR_TIMEOUT / MEBP_ERR_DEVICE if a kernel flagged one since the last sync. */
 int mebp_sync(mebp_ctx* ctx, void* stream);
-/* Workspace bytes the context holds on the device (a high-water figure). */
+/* Workspace bytes the context holds on the device (allocated at creation; no call allocates
+ * more, so this is also the library's peak). */
 int64_t mebp_workspace_bytes(const mebp_ctx* ctx);
+
+/* The workspace by purpose (device bytes, except MEBP_WS_HOST_CKPT: pinned host bytes):
+ *   MEBP_WS_CKPT        block-boundary checkpoints (L+1 slots, or a 3-slot ring when spilling)
+ *   MEBP_WS_FWD_SETS    forward intermediates of one block, times the number of sets (*n_sets)
+ *   MEBP_WS_BWD         backward working buffers of one block (gradients of the intermediates)
+ *   MEBP_WS_ATTN_SPLIT  fp32 partials of the split attention backward (small grids)
+ *   MEBP_WS_LMHEAD      LM-head + CE buffers (one vocabulary chunk of the CE gradient)
+ *   MEBP_WS_LORA_SHADOW fp16 operand copies of the LoRA masters (every block)
+ *   MEBP_WS_OTHER       RoPE tables, device scalars, error word, reduction scratch
+ *   MEBP_WS_HOST_CKPT   pinned host checkpoints (spilling)
+ * bytes has MEBP_WS_N entries; n_sets may be NULL. */
+enum {
+  MEBP_WS_CKPT = 0, MEBP_WS_FWD_SETS, MEBP_WS_BWD, MEBP_WS_ATTN_SPLIT, MEBP_WS_LMHEAD, MEBP_WS_LORA_SHADOW,
+  MEBP_WS_OTHER, MEBP_WS_HOST_CKPT, MEBP_WS_N
+};
+int mebp_workspace_breakdown(const mebp_ctx* ctx, int64_t* bytes, int* n_sets);
 
 /* ---- Section 3 "Base model weights compression": quantise W fp32 [rows, cols] (device)
  * into qpack / scales (layout above).  group must be 64.  Ties round to even. */
@@ -173,6 +197,7 @@ int mebp_embed(mebp_ctx* ctx, const mebp_packed* embed, const int32_t* ids, int6
  * mebp_linear_fwd:  Y [M, N] = X [M, K] deq(W)^T + s (X A^T) B^T  (+ R if R != NULL)
  *   X fp16 [M, K] (bits), W packed [N, K], A fp32 [r, K] / B fp32 [N, r] or both NULL,
  *   Y fp32 [M, N] when y_f32 != NULL else fp16 bits into y_f16.  R fp32 [M, N] may alias y_f32.
+ *   X, the weight pointers, the outputs and R must be 16-byte aligned (MEBP_ERR_INVALID_ARG).
  * mebp_linear_dx:   dX [M, K] = dY [M, N] deq(W) + s (dY B) A  (+ R if R != NULL)
  *   dY fp16 [M, N] (bits), same W / A / B, dX fp32 [M, K].
  * Both use the tcgen05 fused dequant-GEMM kernels; r <= 32. */
@@ -191,13 +216,16 @@ int mebp_linear_dx(mebp_ctx* ctx, const uint16_t* dY, int64_t M, const mebp_pack
  * that is current when called.  Its scratch (the fp16 LoRA shadows, the rank-r product and an
  * error word) lives in one static device array of MEBP_NOALLOC_SCRATCH_BYTES per GPU that loads
  * the library, kept until the process exits:
- *   - the first call on a device looks up that array's address (cudaGetSymbolAddress) and must
- *     happen before any stream capture on that device;
+ *   - the first call in each CUDA context (the device's primary context, or one the caller made
+ *     current) looks up that array's address (cudaGetSymbolAddress) and must happen before any
+ *     stream capture in that context; after a device reset the next call looks it up again;
  *   - every call shares the array and leaves its contents behind: calls that can overlap on the
  *     GPU (different streams without ordering) race on it;
  *   - a request whose scratch (about 2 * (kx*K + 2*N*kx + M*kx) bytes, kx = r rounded up to 16;
  *     none without LoRA) exceeds the array returns MEBP_ERR_SCRATCH before doing anything;
- *   - device-side wait timeouts are not reported (there is no context to read them from).
+ *   - device-side wait timeouts are not reported (there is no context to read them from): the
+ *     output of a call whose bounded wait expired cannot be told apart from a good one;
+ *   - X, W's pointers, y_f32 / y_f16 and R must be 16-byte aligned (MEBP_ERR_INVALID_ARG).
  * Allocates nothing: no cudaMalloc, cudaFree or allocating library call. */
 #define MEBP_NOALLOC_SCRATCH_BYTES (8u << 20)
 int mebp_linear_fwd_noalloc(const uint16_t* X, int64_t M, const mebp_packed* W, const float* A,
@@ -262,24 +290,43 @@ typedef struct {
 int mebp_adamw_step(mebp_ctx* ctx, float* params, const float* grads, float* m, float* v, int64_t n,
                     const mebp_adamw_cfg* cfg, int64_t step, void* stream);
 
-/* ---- instrumentation (Section 4 reports per-layer time; here: device time of the fused GEMMs).
+/* ---- instrumentation (Section 4 reports per-layer time and memory; here: device time of every
+ * kernel, by kind, measured with CUDA events).
  * mebp_kernel_launches: process-wide number of kernel launches the library has issued.
  * mebp_profile_begin: from now on record a CUDA-event pair on the launching stream around every
- *   fused dequant-GEMM launch of this context.
- * mebp_profile_end: synchronise those events, stop recording and report the summed device time
- *   and algorithmic flops (2 M N K, plus 2 M N kx for the LoRA extra block) of the recorded
- *   launches, split into forward-mode (Y = X deq(W)^T, LM-head passes) and transposed (dX) ones. */
+ *   kernel launch of this context (mebp_lora_step then runs eagerly, not as a graph replay; the
+ *   events serialise each launch against its neighbours on that stream).
+ * mebp_profile_end: synchronise those events, stop recording and report the fused dequant-GEMM
+ *   launches: summed device time, algorithmic flops (2 M N K, plus 2 M N kx for the LoRA extra
+ *   block) and bytes (activation operand, packed weight and scales, output, residual and LoRA
+ *   operands, each once), split into forward-mode (Y = X deq(W)^T, LM-head passes) and transposed
+ *   (dX) launches.
+ * mebp_profile_kernels: after mebp_profile_end, one entry per kind of kernel (fused GEMM forward /
+ *   transposed, embedding, RMSNorm forward / backward, RoPE, gated-MLP forward / backward,
+ *   attention forward / backward, LoRA kernels, LM-head reductions, ...): launches, summed event
+ *   time, algorithmic HBM bytes and flops.  *n = the number of kinds; at most max are written.
+ *   name points to a static string. */
 typedef struct {
   int64_t gemm_launches;
-  double gemm_ms, gemm_flops;
+  double gemm_ms, gemm_flops;  /* summed per-launch device time (launches on concurrent streams
+                                  overlap, so this may exceed the wall time) and flops */
   double fwd_ms, fwd_flops;
   double dx_ms, dx_flops;
+  double gemm_busy_ms;         /* length of the union of the launches' [start, end] intervals:
+                                  wall time during which at least one fused GEMM ran */
+  double gemm_bytes;           /* algorithmic bytes of the launches */
 } mebp_profile;
+typedef struct {
+  const char* name;
+  int64_t launches;
+  double ms, bytes, flops;
+} mebp_kernel_stat;
 int64_t mebp_kernel_launches(void);
 /* Turn CUDA-graph replay of mebp_lora_step on (default) or off; drops any captured graph. */
 int mebp_enable_graphs(mebp_ctx* ctx, int on);
 int mebp_profile_begin(mebp_ctx* ctx);
 int mebp_profile_end(mebp_ctx* ctx, mebp_profile* out);
+int mebp_profile_kernels(const mebp_ctx* ctx, mebp_kernel_stat* out, int max, int* n);
 
 #ifdef __cplusplus
 }

@@ -14,6 +14,7 @@ namespace mebp {
 // Device error word codes (stored with atomicCAS so the first failure wins).
 constexpr int kErrTimeout = MEBP_ERR_TIMEOUT;
 constexpr int kErrDevice = MEBP_ERR_DEVICE;
+constexpr int kErrNonFinite = MEBP_ERR_NONFINITE;
 
 // Bounded waits give up after this many nanoseconds of %globaltimer.
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
@@ -30,13 +31,17 @@ MEBP_DEV uint64_t globaltimer_ns() {
 
 MEBP_DEV uint32_t smem_u32(const void* p) { return static_cast<uint32_t>(__cvta_generic_to_shared(p)); }
 
-// Tensor-core operands and stored activations are IEEE fp16 (kind::f16 runs fp16 and fp16 at
+// Tensor-core operands and stored activations are IEEE fp16 (kind::f16 runs fp16 and bf16 at
 // the same rate; fp16 keeps 3 more mantissa bits).
 MEBP_DEV uint32_t pack_half2(float lo, float hi) {
   // cvt.rn.f16x2.f32 d, a, b puts a in the upper half, b in the lower half.
   uint32_t r;
   asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
   return r;
+}
+// 1 when either fp16 half of v is inf or NaN (exponent field all ones), else 0.
+MEBP_DEV uint32_t h2_nonfinite(uint32_t v) {
+  return static_cast<uint32_t>((v & 0x7C00u) == 0x7C00u) | static_cast<uint32_t>((v & 0x7C000000u) == 0x7C000000u);
 }
 MEBP_DEV float h2_lo(uint32_t v) { return __half2float(__ushort_as_half(static_cast<uint16_t>(v & 0xFFFFu))); }
 MEBP_DEV float h2_hi(uint32_t v) { return __half2float(__ushort_as_half(static_cast<uint16_t>(v >> 16))); }

@@ -258,6 +258,7 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
     return;
   }
 
+  uint32_t bad = 0;  // an fp16 output overflowed (or is NaN)
 #pragma unroll 1
   for (int cc = 0; cc < NCH; ++cc) {
     float v[32];
@@ -269,9 +270,12 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
       uint4* dst = reinterpret_cast<uint4*>(C + static_cast<int64_t>(row) * p.ldc + c0);
 #pragma unroll
       for (int i = 0; i < 4; ++i)
-        if (c0 + 8 * i < p.N)
-          dst[i] = make_uint4(pack_half2(v[8 * i], v[8 * i + 1]), pack_half2(v[8 * i + 2], v[8 * i + 3]),
-                              pack_half2(v[8 * i + 4], v[8 * i + 5]), pack_half2(v[8 * i + 6], v[8 * i + 7]));
+        if (c0 + 8 * i < p.N) {
+          const uint4 o = make_uint4(pack_half2(v[8 * i], v[8 * i + 1]), pack_half2(v[8 * i + 2], v[8 * i + 3]),
+                                     pack_half2(v[8 * i + 4], v[8 * i + 5]), pack_half2(v[8 * i + 6], v[8 * i + 7]));
+          bad |= h2_nonfinite(o.x) | h2_nonfinite(o.y) | h2_nonfinite(o.z) | h2_nonfinite(o.w);
+          dst[i] = o;
+        }
     } else {  // EPI_F32 (+ residual)
       float4* dst = reinterpret_cast<float4*>(static_cast<float*>(p.C) + static_cast<int64_t>(row) * p.ldc + c0);
       const float4* res = p.R ? reinterpret_cast<const float4*>(p.R + static_cast<int64_t>(row) * p.ldr + c0) : nullptr;
@@ -288,6 +292,7 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
       }
     }
   }
+  if (bad) flag_error(p.err, kErrNonFinite);
 }
 
 // ---------------------------------------------------------------------------------- split-K
@@ -342,8 +347,9 @@ __device__ __forceinline__ void split_reduce(const Params& p, const uint8_t* sme
         s.x += v[j].x; s.y += v[j].y; s.z += v[j].z; s.w += v[j].w;
       }
     if (p.epi == EPI_F16) {
-      *reinterpret_cast<uint2*>(static_cast<uint16_t*>(p.C) + row * p.ldc + col) =
-          make_uint2(pack_half2(s.x, s.y), pack_half2(s.z, s.w));
+      const uint2 o = make_uint2(pack_half2(s.x, s.y), pack_half2(s.z, s.w));
+      if (h2_nonfinite(o.x) | h2_nonfinite(o.y)) flag_error(p.err, kErrNonFinite);
+      *reinterpret_cast<uint2*>(static_cast<uint16_t*>(p.C) + row * p.ldc + col) = o;
     } else {
       float4 o = make_float4(p.alpha * s.x, p.alpha * s.y, p.alpha * s.z, p.alpha * s.w);
       if (p.R) {

@@ -124,6 +124,7 @@ __device__ __forceinline__ void copy_lora_b(const Params& p, int e, int n0, uint
 __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int warp, int lane, int m0, int n0) {
   const int row = m0 + 32 * warp + lane;
   const uint32_t tb = tmem + (static_cast<uint32_t>(32 * warp) << 16);
+  uint32_t bad = 0;  // an fp16 output overflowed (or is NaN)
 #pragma unroll 1
   for (int cc = 0; cc < 2; ++cc) {
     float v[32];
@@ -133,9 +134,12 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
     if (p.epi == EPI_F16) {
       uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(p.C) + static_cast<int64_t>(row) * p.ldc + c0);
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
-        dst[i] = make_uint4(pack_half2(v[8 * i], v[8 * i + 1]), pack_half2(v[8 * i + 2], v[8 * i + 3]),
-                            pack_half2(v[8 * i + 4], v[8 * i + 5]), pack_half2(v[8 * i + 6], v[8 * i + 7]));
+      for (int i = 0; i < 4; ++i) {
+        const uint4 o = make_uint4(pack_half2(v[8 * i], v[8 * i + 1]), pack_half2(v[8 * i + 2], v[8 * i + 3]),
+                                   pack_half2(v[8 * i + 4], v[8 * i + 5]), pack_half2(v[8 * i + 6], v[8 * i + 7]));
+        bad |= h2_nonfinite(o.x) | h2_nonfinite(o.y) | h2_nonfinite(o.z) | h2_nonfinite(o.w);
+        dst[i] = o;
+      }
     } else {  // EPI_F32 (+ residual, which may alias C)
       float4* dst = reinterpret_cast<float4*>(static_cast<float*>(p.C) + static_cast<int64_t>(row) * p.ldc + c0);
       const float4* res = p.R ? reinterpret_cast<const float4*>(p.R + static_cast<int64_t>(row) * p.ldr + c0) : nullptr;
@@ -151,6 +155,7 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
       }
     }
   }
+  if (bad) flag_error(p.err, kErrNonFinite);
 }
 
 template <bool TRANS, int KCH>

@@ -147,9 +147,10 @@ void launch_add_norm2(const float* ao, const float* x, const float* gpa, const f
 void launch_add_norm(const float* dn, const float* h1, const float* gpf, int64_t T, int D, float eps, float* y,
                      float* rpf, cudaStream_t st);
 // Gated MLP: m = act(g) * u from gu = [g | u] (fp16 [T, 2I]); backward reads dm fp16 [T, I] and
-// writes dgu fp16 [T, 2I].
-void launch_glu_fwd(const uint16_t* gu, int64_t T, int I, int act, uint16_t* m, cudaStream_t st);
-void launch_glu_bwd(const uint16_t* dm, const uint16_t* gu, int64_t T, int I, int act, uint16_t* dgu, cudaStream_t st);
+// writes dgu fp16 [T, 2I].  A result outside the fp16 range sets MEBP_ERR_NONFINITE in *err.
+void launch_glu_fwd(const uint16_t* gu, int64_t T, int I, int act, uint16_t* m, int* err, cudaStream_t st);
+void launch_glu_bwd(const uint16_t* dm, const uint16_t* gu, int64_t T, int I, int act, uint16_t* dgu, int* err,
+                    cudaStream_t st);
 // y32 = x * (*scale), y16 = fp16(x * (*scale)); scale may be null (= 1), y32 may be null.
 void launch_scale_cast(const float* x, int64_t n, const float* scale, float* y32, uint16_t* y16, cudaStream_t st);
 // scal[0] = sigma = 2^-floor(log2(max|x|)) (1 if x == 0), scal[1] = 1/sigma; uses scal[2] as scratch.

@@ -7,6 +7,8 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -28,11 +30,45 @@ struct Lin {
 
 constexpr int kCkptSlots = 3;
 
+// Kinds of kernel the event profiler (mebp_profile_begin / _end / _kernels) tells apart.
+enum KKind {
+  KK_GEMM_FWD = 0, KK_GEMM_DX, KK_EMBED, KK_RMSNORM_FWD, KK_RMSNORM_BWD, KK_ADD_NORM, KK_ROPE, KK_QKNORM_ROPE,
+  KK_GLU_FWD, KK_GLU_BWD, KK_ATTN_FWD, KK_ATTN_BWD, KK_LORA_SKINNY, KK_LORA_REDUCE, KK_LORA_SHADOW, KK_LM_REDUCE,
+  KK_SCALE, KK_N
+};
+const char* const kKindName[KK_N] = {
+    "fused_gemm_fwd", "fused_gemm_dx", "embed", "rmsnorm_fwd", "rmsnorm_bwd", "add_norm", "rope", "qknorm_rope",
+    "glu_fwd", "glu_bwd", "attention_fwd", "attention_bwd", "lora_skinny", "lora_grad_reduce", "lora_shadow",
+    "lmhead_reduce", "grad_scale"};
+
+// One profiled launch: CUDA events on the launching stream around it, and its algorithmic work.
 struct ProfRec {
   cudaEvent_t a, b;
-  double flops;
-  bool trans;
+  int kind;
+  double flops, bytes;
 };
+
+// Algorithmic HBM bytes of the memory-bound kernels (each operand read or written once).
+double bytes_rms_fwd(int64_t T, int D) { return 6.0 * T * D + 4.0 * T + 4.0 * D; }
+double bytes_rms_bwd(int64_t T, int D, bool resid, bool dx, bool dxh) {
+  return T * static_cast<double>(D) * (8.0 + (resid ? 4 : 0) + (dx ? 4 : 0) + (dxh ? 2 : 0)) + 4.0 * T + 4.0 * D;
+}
+double bytes_rope(int64_t T, int S, int H, int KV, int hd) { return 4.0 * T * (H + KV) * hd + 8.0 * S * (hd / 2); }
+double bytes_qknorm(int64_t T, int S, int H, int KV, int hd) {
+  return 6.0 * T * (H + KV) * hd + 4.0 * T * (H + KV) + 8.0 * S * (hd / 2);
+}
+// Causal (window W > 0: sliding) attention flops of the forward: QK^T and PV over the visible keys.
+double attn_fwd_flops(int B, int S, int H, int hd, int W) {
+  double keys = 0.0;
+  for (int i = 0; i < S; ++i) keys += (W > 0 && W < i + 1) ? W : i + 1;
+  return 4.0 * hd * keys * B * H;
+}
+double bytes_attn_fwd(int64_t T, int H, int KV, int hd) { return 2.0 * T * (H + 2 * KV) * hd + 2.0 * T * H * hd + 4.0 * T * H; }
+double bytes_attn_bwd(int64_t T, int H, int KV, int hd) {
+  return 4.0 * T * (H + 2 * KV) * hd + 4.0 * T * H * hd + 12.0 * T * H;
+}
+double bytes_skinny(int64_t T, int64_t K, int kx, int kxp) { return 2.0 * T * K + 2.0 * kx * K + 2.0 * T * kxp; }
+double bytes_tall(int64_t M, int Pw, int Qw, bool acc) { return 2.0 * M * (Pw + Qw) + 4.0 * Pw * Qw * (acc ? 2 : 1); }
 
 }  // namespace
 
@@ -93,6 +129,8 @@ struct mebp_ctx {
   Lin lin[4];
   std::vector<void*> dev_allocs;
   int64_t ws_bytes = 0;
+  int64_t ws_cat[MEBP_WS_N] = {};  // bytes per purpose (mebp_workspace_breakdown)
+  int cur_cat = MEBP_WS_OTHER;     // purpose of the allocations being made
 
   float2* rope_cs = nullptr;
   float2* rope_cs_local = nullptr;  // RoPE table of the sliding-window layers (their own base)
@@ -137,9 +175,10 @@ struct mebp_ctx {
   long long graph_launches = 0;
   int graph_eager_runs = 0;
   cudaEvent_t copy_join = nullptr;
-  // GEMM event profiling
+  // event profiling of every launch (mebp_profile_begin / _end / _kernels)
   bool prof = false;
   std::vector<ProfRec> recs;
+  std::vector<mebp_kernel_stat> kstats;
   std::vector<cudaEvent_t> evpool;
   size_t evnext = 0;
 };
@@ -169,6 +208,7 @@ int dalloc(mebp_ctx* c, T** p, int64_t count) {
   }
   c->dev_allocs.push_back(q);
   c->ws_bytes += static_cast<int64_t>(bytes);
+  c->ws_cat[c->cur_cat] += static_cast<int64_t>(bytes);
   *p = static_cast<T*>(q);
   return MEBP_OK;
 }
@@ -255,21 +295,44 @@ cudaEvent_t pool_event(mebp_ctx* c) {
   return c->evpool[c->evnext++];
 }
 
+// Runs f() (one or more launches on st); when profiling, brackets it with an event pair on st and
+// records its kind and algorithmic work.
+template <class F>
+void KP(mebp_ctx* c, int kind, double bytes, double flops, cudaStream_t st, F&& f) {
+  if (!c->prof) {
+    f();
+    return;
+  }
+  ProfRec r{};
+  r.a = pool_event(c);
+  r.b = pool_event(c);
+  r.kind = kind;
+  r.bytes = bytes;
+  r.flops = flops;
+  cudaEventRecord(r.a, st);
+  f();
+  cudaEventRecord(r.b, st);
+  c->recs.push_back(r);
+}
+
+// Algorithmic bytes of a fused GEMM: the activation operand, the packed weight with its scales,
+// the output (and residual), the LoRA operands.
+double gemm_bytes(const GemmArgs& g) {
+  const double M = static_cast<double>(g.M), N = static_cast<double>(g.N), K = static_cast<double>(g.K);
+  double b = 2.0 * M * K + N * K / 2.0 + 2.0 * N * (K / 64.0);
+  if (g.epi == EPI_F32) b += 4.0 * M * N;
+  else if (g.epi == EPI_F16 || g.epi == EPI_CEGRAD) b += 2.0 * M * N;
+  else b += 8.0 * M * g.nparts / 2.0;  // LSE partials
+  if (g.R) b += 4.0 * M * N;
+  if (g.Ax) b += 2.0 * M * g.kx + 2.0 * N * g.kx;
+  return b;
+}
+
 int run_gemm(mebp_ctx* c, GemmArgs& g, cudaStream_t st, const char* what) {
   g.err = c->d_err;
-  ProfRec pr{};
-  if (c->prof) {
-    pr.a = pool_event(c);
-    pr.b = pool_event(c);
-    pr.trans = g.trans;
-    pr.flops = 2.0 * g.M * g.N * g.K + (g.Ax ? 2.0 * g.M * g.N * g.kx : 0.0);
-    cudaEventRecord(pr.a, st);
-  }
-  const int rc = launch_dequant_gemm(g, st);
-  if (c->prof) {
-    cudaEventRecord(pr.b, st);
-    c->recs.push_back(pr);
-  }
+  int rc = MEBP_OK;
+  KP(c, g.trans ? KK_GEMM_DX : KK_GEMM_FWD, gemm_bytes(g),
+     2.0 * g.M * g.N * g.K + (g.Ax ? 2.0 * g.M * g.N * g.kx : 0.0), st, [&] { rc = launch_dequant_gemm(g, st); });
   if (rc) return fail(c, rc, std::string(what) + ": fused GEMM launch failed (" + std::to_string(rc) + ")");
   return MEBP_OK;
 }
@@ -322,48 +385,70 @@ int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, 
   }
   A.sh = sh;
   // attention sub-block
-  launch_rmsnorm_fwd(x, w->norm1, T, D, c->cfg.rms_eps, A.a, A.r1, st);
+  KP(c, KK_RMSNORM_FWD, bytes_rms_fwd(T, D), 0, st,
+     [&] { launch_rmsnorm_fwd(x, w->norm1, T, D, c->cfg.rms_eps, A.a, A.r1, st); });
   const Lin& lq = c->lin[LIN_QKV];
   GemmArgs g = gemm_fwd(A.a, D, T, w->qkv, lq.N, lq.K);
   if (lq.kx) {
-    launch_skinny_gemm(A.a, D, T, D, A.sh->A_cat[LIN_QKV], D, lq.kx, c->s, A.us[LIN_QKV], lq.kxp, st);
+    KP(c, KK_LORA_SKINNY, bytes_skinny(T, D, lq.kx, lq.kxp), 2.0 * T * D * lq.kx, st, [&] {
+      launch_skinny_gemm(A.a, D, T, D, A.sh->A_cat[LIN_QKV], D, lq.kx, c->s, A.us[LIN_QKV], lq.kxp, st);
+    });
     g.Ax = A.us[LIN_QKV]; g.ldax = lq.kxp; g.kx = lq.kxp; g.Bx = A.sh->B_cat[LIN_QKV]; g.ldbx = lq.kxp;
   }
   g.epi = EPI_F16; g.C = A.qkv; g.ldc = lq.N;
   if ((rc = run_gemm(c, g, st, "qkv"))) return rc;
   if (c->gemma)
-    launch_qknorm_rope(A.qkv, T, Sq, c->H, c->KV, c->hd, w->q_norm, w->k_norm, c->cfg.rms_eps,
-                       layer_rope(c, layer), A.qk_raw, A.rqk, st);
+    KP(c, KK_QKNORM_ROPE, bytes_qknorm(T, Sq, c->H, c->KV, c->hd), 0, st, [&] {
+      launch_qknorm_rope(A.qkv, T, Sq, c->H, c->KV, c->hd, w->q_norm, w->k_norm, c->cfg.rms_eps,
+                         layer_rope(c, layer), A.qk_raw, A.rqk, st);
+    });
   else
-    launch_rope(A.qkv, T, Sq, c->H, c->KV, c->hd, layer_rope(c, layer), false, st);
-  launch_attn_fwd(A.qkv, lq.N, B, Sq, c->H, c->KV, c->hd, A.o, c->Na, A.lse_attn, layer_window(c, layer), st);
+    KP(c, KK_ROPE, bytes_rope(T, Sq, c->H, c->KV, c->hd), 0, st,
+       [&] { launch_rope(A.qkv, T, Sq, c->H, c->KV, c->hd, layer_rope(c, layer), false, st); });
+  {
+    const int win = layer_window(c, layer) >= Sq ? 0 : layer_window(c, layer);
+    KP(c, KK_ATTN_FWD, bytes_attn_fwd(T, c->H, c->KV, c->hd),
+       c->prof ? attn_fwd_flops(B, Sq, c->H, c->hd, win) : 0.0, st, [&] {
+         launch_attn_fwd(A.qkv, lq.N, B, Sq, c->H, c->KV, c->hd, A.o, c->Na, A.lse_attn, layer_window(c, layer), st);
+       });
+  }
   const Lin& lo = c->lin[LIN_O];
   g = gemm_fwd(A.o, c->Na, T, w->o, lo.N, lo.K);
   if (lo.kx) {
-    launch_skinny_gemm(A.o, c->Na, T, c->Na, A.sh->A_cat[LIN_O], c->Na, lo.kx, c->s, A.us[LIN_O], lo.kxp, st);
+    KP(c, KK_LORA_SKINNY, bytes_skinny(T, c->Na, lo.kx, lo.kxp), 2.0 * T * c->Na * lo.kx, st, [&] {
+      launch_skinny_gemm(A.o, c->Na, T, c->Na, A.sh->A_cat[LIN_O], c->Na, lo.kx, c->s, A.us[LIN_O], lo.kxp, st);
+    });
     g.Ax = A.us[LIN_O]; g.ldax = lo.kxp; g.kx = lo.kxp; g.Bx = A.sh->B_cat[LIN_O]; g.ldbx = lo.kxp;
   }
   if (c->gemma) {  // h1 = x + norm(ao) g_pa, b = norm(h1) g2
     g.epi = EPI_F32; g.C = A.ao; g.ldc = D;
     if ((rc = run_gemm(c, g, st, "o_proj"))) return rc;
-    launch_add_norm2(A.ao, x, w->post_attn_norm, w->norm2, T, D, c->cfg.rms_eps, A.h1, A.b, A.rpa, A.r2, st);
+    KP(c, KK_ADD_NORM, 14.0 * T * D + 8.0 * T + 8.0 * D, 0, st, [&] {
+      launch_add_norm2(A.ao, x, w->post_attn_norm, w->norm2, T, D, c->cfg.rms_eps, A.h1, A.b, A.rpa, A.r2, st);
+    });
   } else {
     g.epi = EPI_F32; g.C = A.h1; g.ldc = D; g.R = x; g.ldr = D;
     if ((rc = run_gemm(c, g, st, "o_proj"))) return rc;
-    launch_rmsnorm_fwd(A.h1, w->norm2, T, D, c->cfg.rms_eps, A.b, A.r2, st);
+    KP(c, KK_RMSNORM_FWD, bytes_rms_fwd(T, D), 0, st,
+       [&] { launch_rmsnorm_fwd(A.h1, w->norm2, T, D, c->cfg.rms_eps, A.b, A.r2, st); });
   }
   // MLP sub-block
   const Lin& lg = c->lin[LIN_GU];
   g = gemm_fwd(A.b, D, T, w->gate_up, lg.N, lg.K);
   if (lg.kx) {
-    launch_skinny_gemm(A.b, D, T, D, A.sh->A_cat[LIN_GU], D, lg.kx, c->s, A.us[LIN_GU], lg.kxp, st);
+    KP(c, KK_LORA_SKINNY, bytes_skinny(T, D, lg.kx, lg.kxp), 2.0 * T * D * lg.kx, st, [&] {
+      launch_skinny_gemm(A.b, D, T, D, A.sh->A_cat[LIN_GU], D, lg.kx, c->s, A.us[LIN_GU], lg.kxp, st);
+    });
     g.Ax = A.us[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = A.sh->B_cat[LIN_GU]; g.ldbx = lg.kxp;
   }
   g.epi = EPI_F16; g.C = A.gu; g.ldc = lg.N;
   if ((rc = run_gemm(c, g, st, "gate_up"))) return rc;
-  launch_glu_fwd(A.gu, T, I, c->cfg.act, A.m, st);
+  KP(c, KK_GLU_FWD, 6.0 * T * I, 0, st, [&] { launch_glu_fwd(A.gu, T, I, c->cfg.act, A.m, c->d_err, st); });
   const Lin& ld = c->lin[LIN_DOWN];
-  if (ld.kx) launch_skinny_gemm(A.m, I, T, I, A.sh->A_cat[LIN_DOWN], I, ld.kx, c->s, A.us[LIN_DOWN], ld.kxp, st);
+  if (ld.kx)
+    KP(c, KK_LORA_SKINNY, bytes_skinny(T, I, ld.kx, ld.kxp), 2.0 * T * I * ld.kx, st, [&] {
+      launch_skinny_gemm(A.m, I, T, I, A.sh->A_cat[LIN_DOWN], I, ld.kx, c->s, A.us[LIN_DOWN], ld.kxp, st);
+    });
   if (with_down || c->gemma) {
     g = gemm_fwd(A.m, I, T, w->down, ld.N, ld.K);
     if (ld.kx) {
@@ -372,7 +457,9 @@ int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, 
     if (c->gemma) {  // y = h1 + norm(dn) g_pf
       g.epi = EPI_F32; g.C = A.dn; g.ldc = D;
       if ((rc = run_gemm(c, g, st, "down"))) return rc;
-      launch_add_norm(A.dn, A.h1, w->post_ffn_norm, T, D, c->cfg.rms_eps, with_down ? y : nullptr, A.rpf, st);
+      KP(c, KK_ADD_NORM, (with_down ? 12.0 : 8.0) * T * D + 4.0 * T + 4.0 * D, 0, st, [&] {
+        launch_add_norm(A.dn, A.h1, w->post_ffn_norm, T, D, c->cfg.rms_eps, with_down ? y : nullptr, A.rpf, st);
+      });
     } else {
       g.epi = EPI_F32; g.C = y; g.ldc = D; g.R = A.h1; g.ldr = D;
       if ((rc = run_gemm(c, g, st, "down"))) return rc;
@@ -382,6 +469,16 @@ int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, 
   A.x = x;
   A.T = T;
   return cuda_check(c, "block forward");
+}
+
+// The batched LoRA-gradient reductions of one block (one launch).
+void run_tall_batch(mebp_ctx* c, const TallBatch& b, cudaStream_t st) {
+  double bytes = 0.0, flops = 0.0;
+  for (int i = 0; i < b.n; ++i) {
+    bytes += bytes_tall(b.M, b.p[i].Pw, b.p[i].Qw, b.p[i].acc != 0);
+    flops += 2.0 * b.M * b.p[i].Pw * b.p[i].Qw;
+  }
+  KP(c, KK_LORA_REDUCE, bytes, flops, st, [&] { launch_tall_reduce_batched(b, st); });
 }
 
 // Token counts below this run a block's LoRA-gradient reductions as one batched launch (each is a
@@ -400,14 +497,20 @@ int lin_grads(mebp_ctx* c, const Acts& A, const uint16_t* du, int li, const uint
     if (grads->dB[tg] &&
         !(tb && tall_batch_add(*tb, dY + l.no[t], ldy, A.us[li] + l.ro[t], l.kxp, l.nl[t], c->r, grads->dB[tg], c->r,
                                acc))) {
-      const int rc = launch_tall_reduce(dY + l.no[t], ldy, A.us[li] + l.ro[t], l.kxp, T, l.nl[t], c->r, grads->dB[tg],
-                                        c->r, acc, grad_mult, c->red, c->red_floats, st);
+      int rc = MEBP_OK;
+      KP(c, KK_LORA_REDUCE, bytes_tall(T, l.nl[t], c->r, acc), 2.0 * T * l.nl[t] * c->r, st, [&] {
+        rc = launch_tall_reduce(dY + l.no[t], ldy, A.us[li] + l.ro[t], l.kxp, T, l.nl[t], c->r, grads->dB[tg], c->r,
+                                acc, grad_mult, c->red, c->red_floats, st);
+      });
       if (rc) return fail(c, rc, "LoRA dB reduction");
     }
     if (grads->dA[tg] &&
         !(tb && tall_batch_add(*tb, X, ldx, du + l.ro[t], l.kxp, l.K, c->r, grads->dA[tg], -l.K, acc))) {
-      const int rc = launch_tall_reduce(X, ldx, du + l.ro[t], l.kxp, T, l.K, c->r, grads->dA[tg], -l.K, acc,
-                                        grad_mult, c->red, c->red_floats, st);
+      int rc = MEBP_OK;
+      KP(c, KK_LORA_REDUCE, bytes_tall(T, l.K, c->r, acc), 2.0 * T * l.K * c->r, st, [&] {
+        rc = launch_tall_reduce(X, ldx, du + l.ro[t], l.kxp, T, l.K, c->r, grads->dA[tg], -l.K, acc, grad_mult,
+                                c->red, c->red_floats, st);
+      });
       if (rc) return fail(c, rc, "LoRA dA reduction");
     }
   }
@@ -440,24 +543,31 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   // ---- down projection: y = h1 + m Wd^T (+ s (m Ad^T) Bd^T); Gemma3: y = h1 + norm(dn) g_pf
   const uint16_t* ddn_h = dy_h;
   if (c->gemma) {
-    launch_rmsnorm_bwd(dy, A.dn, w->post_ffn_norm, A.rpf, nullptr, T, D, nullptr, nullptr, G.ddn_h, st);
+    KP(c, KK_RMSNORM_BWD, bytes_rms_bwd(T, D, false, false, true), 0, st, [&] {
+      launch_rmsnorm_bwd(dy, A.dn, w->post_ffn_norm, A.rpf, nullptr, T, D, nullptr, nullptr, G.ddn_h, st);
+    });
     ddn_h = G.ddn_h;
   }
   const Lin& ld = c->lin[LIN_DOWN];
   GemmArgs g = gemm_dx(ddn_h, D, T, w->down);
   if (ld.kx) {
-    launch_skinny_gemm(ddn_h, D, T, D, A.sh->Bt_cat[LIN_DOWN], D, ld.kx, c->s, du[LIN_DOWN], ld.kxp, st);
+    KP(c, KK_LORA_SKINNY, bytes_skinny(T, D, ld.kx, ld.kxp), 2.0 * T * D * ld.kx, st, [&] {
+      launch_skinny_gemm(ddn_h, D, T, D, A.sh->Bt_cat[LIN_DOWN], D, ld.kx, c->s, du[LIN_DOWN], ld.kxp, st);
+    });
     g.Ax = du[LIN_DOWN]; g.ldax = ld.kxp; g.kx = ld.kxp; g.Bx = A.sh->A_cat[LIN_DOWN]; g.ldbx = I;
   }
   g.epi = EPI_F16; g.C = c->dm; g.ldc = I;
   if ((rc = run_gemm(c, g, st, "down dX"))) return rc;
   if ((rc = lin_grads(c, A, du[LIN_DOWN], LIN_DOWN, ddn_h, D, A.m, I, T, grads, acc, grad_mult, st, tb))) return rc;
   // ---- gated MLP
-  launch_glu_bwd(c->dm, A.gu, T, I, c->cfg.act, G.dgu, st);
+  KP(c, KK_GLU_BWD, 10.0 * T * I, 0, st,
+     [&] { launch_glu_bwd(c->dm, A.gu, T, I, c->cfg.act, G.dgu, c->d_err, st); });
   const Lin& lg = c->lin[LIN_GU];
   g = gemm_dx(G.dgu, 2 * I, T, w->gate_up);
   if (lg.kx) {
-    launch_skinny_gemm(G.dgu, 2 * I, T, 2 * I, A.sh->Bt_cat[LIN_GU], 2 * I, lg.kx, c->s, du[LIN_GU], lg.kxp, st);
+    KP(c, KK_LORA_SKINNY, bytes_skinny(T, 2 * I, lg.kx, lg.kxp), 4.0 * T * I * lg.kx, st, [&] {
+      launch_skinny_gemm(G.dgu, 2 * I, T, 2 * I, A.sh->Bt_cat[LIN_GU], 2 * I, lg.kx, c->s, du[LIN_GU], lg.kxp, st);
+    });
     g.Ax = du[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = A.sh->A_cat[LIN_GU]; g.ldbx = D;
   }
   g.epi = EPI_F32; g.C = c->dtmp; g.ldc = D;
@@ -466,16 +576,22 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   // dh1 = dy + RMSNorm2^T(db); the o projection's output gradient is dh1 (fp16 copy in dh1_h), for
   // Gemma3 the post-attention norm's VJP of it
   if (c->gemma) {
-    launch_rmsnorm_bwd(c->dtmp, A.h1, w->norm2, A.r2, dy, T, D, nullptr, c->dh1, nullptr, st);
-    launch_rmsnorm_bwd(c->dh1, A.ao, w->post_attn_norm, A.rpa, nullptr, T, D, nullptr, nullptr, G.dh1_h, st);
+    KP(c, KK_RMSNORM_BWD, bytes_rms_bwd(T, D, true, true, false), 0, st,
+       [&] { launch_rmsnorm_bwd(c->dtmp, A.h1, w->norm2, A.r2, dy, T, D, nullptr, c->dh1, nullptr, st); });
+    KP(c, KK_RMSNORM_BWD, bytes_rms_bwd(T, D, false, false, true), 0, st, [&] {
+      launch_rmsnorm_bwd(c->dh1, A.ao, w->post_attn_norm, A.rpa, nullptr, T, D, nullptr, nullptr, G.dh1_h, st);
+    });
   } else {
-    launch_rmsnorm_bwd(c->dtmp, A.h1, w->norm2, A.r2, dy, T, D, nullptr, c->dh1, G.dh1_h, st);
+    KP(c, KK_RMSNORM_BWD, bytes_rms_bwd(T, D, true, true, true), 0, st,
+       [&] { launch_rmsnorm_bwd(c->dtmp, A.h1, w->norm2, A.r2, dy, T, D, nullptr, c->dh1, G.dh1_h, st); });
   }
   // ---- o projection
   const Lin& lo = c->lin[LIN_O];
   g = gemm_dx(G.dh1_h, D, T, w->o);
   if (lo.kx) {
-    launch_skinny_gemm(G.dh1_h, D, T, D, A.sh->Bt_cat[LIN_O], D, lo.kx, c->s, du[LIN_O], lo.kxp, st);
+    KP(c, KK_LORA_SKINNY, bytes_skinny(T, D, lo.kx, lo.kxp), 2.0 * T * D * lo.kx, st, [&] {
+      launch_skinny_gemm(G.dh1_h, D, T, D, A.sh->Bt_cat[LIN_O], D, lo.kx, c->s, du[LIN_O], lo.kxp, st);
+    });
     g.Ax = du[LIN_O]; g.ldax = lo.kxp; g.kx = lo.kxp; g.Bx = A.sh->A_cat[LIN_O]; g.ldbx = c->Na;
   }
   g.epi = EPI_F16; g.C = c->dout; g.ldc = c->Na;
@@ -483,18 +599,29 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   if ((rc = lin_grads(c, A, du[LIN_O], LIN_O, G.dh1_h, D, A.o, c->Na, T, grads, acc, grad_mult, st, tb))) return rc;
   // ---- attention, RoPE
   const Lin& lq = c->lin[LIN_QKV];
-  const bool rope_done =
-      launch_attn_bwd(A.qkv, lq.N, A.o, c->dout, c->Na, A.lse_attn, B, Sq, c->H, c->KV, c->hd, c->dvec, G.dqkv,
-                      layer_window(c, layer), c->gemma ? nullptr : layer_rope(c, layer), c->attn_ws, c->attn_ws_floats,
-                      st);
+  bool rope_done = false;
+  {
+    const int win = layer_window(c, layer) >= Sq ? 0 : layer_window(c, layer);
+    KP(c, KK_ATTN_BWD, bytes_attn_bwd(T, c->H, c->KV, c->hd),
+       c->prof ? 2.5 * attn_fwd_flops(B, Sq, c->H, c->hd, win) : 0.0, st, [&] {
+         rope_done = launch_attn_bwd(A.qkv, lq.N, A.o, c->dout, c->Na, A.lse_attn, B, Sq, c->H, c->KV, c->hd, c->dvec,
+                                     G.dqkv, layer_window(c, layer), c->gemma ? nullptr : layer_rope(c, layer),
+                                     c->attn_ws, c->attn_ws_floats, st);
+       });
+  }
   if (c->gemma)
-    launch_qknorm_rope_bwd(G.dqkv, T, Sq, c->H, c->KV, c->hd, w->q_norm, w->k_norm, layer_rope(c, layer), A.qk_raw,
-                           A.rqk, st);
+    KP(c, KK_QKNORM_ROPE, bytes_qknorm(T, Sq, c->H, c->KV, c->hd), 0, st, [&] {
+      launch_qknorm_rope_bwd(G.dqkv, T, Sq, c->H, c->KV, c->hd, w->q_norm, w->k_norm, layer_rope(c, layer), A.qk_raw,
+                             A.rqk, st);
+    });
   else if (!rope_done)
-    launch_rope(G.dqkv, T, Sq, c->H, c->KV, c->hd, layer_rope(c, layer), true, st);
+    KP(c, KK_ROPE, bytes_rope(T, Sq, c->H, c->KV, c->hd), 0, st,
+       [&] { launch_rope(G.dqkv, T, Sq, c->H, c->KV, c->hd, layer_rope(c, layer), true, st); });
   // ---- q, k, v projections
   if (lq.kx)
-    launch_skinny_gemm(G.dqkv, lq.N, T, lq.N, A.sh->Bt_cat[LIN_QKV], lq.N, lq.kx, c->s, du[LIN_QKV], lq.kxp, st);
+    KP(c, KK_LORA_SKINNY, bytes_skinny(T, lq.N, lq.kx, lq.kxp), 2.0 * T * lq.N * lq.kx, st, [&] {
+      launch_skinny_gemm(G.dqkv, lq.N, T, lq.N, A.sh->Bt_cat[LIN_QKV], lq.N, lq.kx, c->s, du[LIN_QKV], lq.kxp, st);
+    });
   if ((rc = lin_grads(c, A, du[LIN_QKV], LIN_QKV, G.dqkv, lq.N, A.a, D, T, grads, acc, grad_mult, st, tb))) return rc;
   if (dx) {
     g = gemm_dx(G.dqkv, lq.N, T, w->qkv);
@@ -503,9 +630,10 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
     }
     g.epi = EPI_F32; g.C = c->dtmp; g.ldc = D;
     if ((rc = run_gemm(c, g, st, "qkv dX"))) return rc;
-    launch_rmsnorm_bwd(c->dtmp, x, w->norm1, A.r1, c->dh1, T, D, dx_mult, dx, dx_h, st);
+    KP(c, KK_RMSNORM_BWD, bytes_rms_bwd(T, D, true, dx != nullptr, dx_h != nullptr), 0, st,
+       [&] { launch_rmsnorm_bwd(c->dtmp, x, w->norm1, A.r1, c->dh1, T, D, dx_mult, dx, dx_h, st); });
   }
-  if (batch.n) launch_tall_reduce_batched(batch, st);
+  if (batch.n) run_tall_batch(c, batch, st);
   return cuda_check(c, "block backward");
 }
 
@@ -528,7 +656,7 @@ int block_lora_grads(mebp_ctx* c, int set, int bset, const uint16_t* dy_h, int64
   if ((rc = lin_grads(c, A, G.du[LIN_QKV], LIN_QKV, G.dqkv, c->lin[LIN_QKV].N, A.a, D, T, grads, acc, grad_mult, st,
                       tb)))
     return rc;
-  if (batch.n) launch_tall_reduce_batched(batch, st);
+  if (batch.n) run_tall_batch(c, batch, st);
   return MEBP_OK;
 }
 
@@ -538,14 +666,17 @@ int lmhead(mebp_ctx* c, const mebp_packed* E, const float* gf, const float* h, c
            float* loss, float* dh, uint16_t* dh_h, float* tok_loss, bool unscale_dh, cudaStream_t st) {
   const int D = c->D, V = c->V;
   int rc;
-  launch_rmsnorm_fwd(h, gf, T, D, c->cfg.rms_eps, c->hf, c->rf, st);
+  KP(c, KK_RMSNORM_FWD, bytes_rms_fwd(T, D), 0, st,
+     [&] { launch_rmsnorm_fwd(h, gf, T, D, c->cfg.rms_eps, c->hf, c->rf, st); });
   GemmArgs g = gemm_fwd(c->hf, D, T, *E, V, D);
   g.epi = EPI_LSE; g.targets = targets; g.col_offset = 0; g.n_valid = V; g.part = c->part; g.nparts = c->nparts;
   g.zt = c->zt;
   if ((rc = run_gemm(c, g, st, "LM head (log-sum-exp pass)"))) return rc;
   float* tl = tok_loss ? tok_loss : c->tok_loss;
-  launch_lse_combine(c->part, c->nparts, c->zt, targets, T, c->lse_tok, tl, st);
-  launch_loss_reduce(tl, targets, T, loss, c->scal, st);
+  KP(c, KK_LM_REDUCE, 8.0 * T * c->nparts + 20.0 * T, 0, st, [&] {
+    launch_lse_combine(c->part, c->nparts, c->zt, targets, T, c->lse_tok, tl, st);
+    launch_loss_reduce(tl, targets, T, loss, c->scal, st);
+  });
   for (int c0 = 0; c0 < V; c0 += c->vchunk) {
     const int n = std::min(c->vchunk, V - c0);
     mebp_packed Ec = *E;
@@ -564,7 +695,9 @@ int lmhead(mebp_ctx* c, const mebp_packed* E, const float* gf, const float* h, c
     t.epi = EPI_F32; t.C = c->dhf; t.ldc = D; t.R = c0 ? c->dhf : nullptr; t.ldr = D; t.alpha = 1.0f / kCeShift;
     if ((rc = run_gemm(c, t, st, "LM head (dH pass)"))) return rc;
   }
-  launch_rmsnorm_bwd(c->dhf, h, gf, c->rf, nullptr, T, D, unscale_dh ? c->scal + 1 : nullptr, dh, dh_h, st);
+  KP(c, KK_RMSNORM_BWD, bytes_rms_bwd(T, D, false, dh != nullptr, dh_h != nullptr), 0, st, [&] {
+    launch_rmsnorm_bwd(c->dhf, h, gf, c->rf, nullptr, T, D, unscale_dh ? c->scal + 1 : nullptr, dh, dh_h, st);
+  });
   return cuda_check(c, "LM head");
 }
 
@@ -649,15 +782,17 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
   auto A = [&](auto** p, int64_t n) {
     if (rc == MEBP_OK) rc = dalloc(c, p, n);
   };
+  c->cur_cat = MEBP_WS_OTHER;
   A(&c->d_err, 4);
   A(&c->scal, 8);
   A(&c->rope_cs, static_cast<int64_t>(f.max_seq) * (c->hd / 2));
   if (f.sliding_window > 0) A(&c->rope_cs_local, static_cast<int64_t>(f.max_seq) * (c->hd / 2));
   // a second intermediate set lets the step overlap recompute and backward (not when spilling:
   // then device memory is the constraint)
-  c->nsets = (!f.spill_ckpts && c->L > 1) ? 2 : 1;
+  c->nsets = (!f.spill_ckpts && !f.min_memory && c->L > 1) ? 2 : 1;
   for (int k = 0; k < c->nsets; ++k) {
     Acts& s = c->act[k];
+    c->cur_cat = MEBP_WS_FWD_SETS;
     A(&s.a, T * D); A(&s.b, T * D); A(&s.qkv, T * c->Nqkv); A(&s.o, T * c->Na); A(&s.gu, T * 2 * I);
     A(&s.m, T * I); A(&s.r1, T); A(&s.r2, T); A(&s.lse_attn, T * c->H); A(&s.h1, T * D);
     if (c->gemma) {
@@ -667,13 +802,16 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
     for (int li = 0; li < 4; ++li) {
       const Lin& l = c->lin[li];
       if (!l.kx) continue;
+      c->cur_cat = MEBP_WS_FWD_SETS;
       A(&s.us[li], T * l.kxp);
+      c->cur_cat = MEBP_WS_LORA_SHADOW;
       A(&s.own.A_cat[li], static_cast<int64_t>(l.kxp) * l.K);
       A(&s.own.B_cat[li], static_cast<int64_t>(l.N) * l.kxp);
       A(&s.own.Bt_cat[li], static_cast<int64_t>(l.N) * l.kxp);
     }
   }
   // the step's per-block shadows (one allocation per linear, blocks back to back)
+  c->cur_cat = MEBP_WS_LORA_SHADOW;
   c->layer_sh.assign(c->L, Shadow{});
   for (int li = 0; li < 4; ++li) {
     const Lin& l = c->lin[li];
@@ -688,6 +826,7 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
       c->layer_sh[i].Bt_cat[li] = pbt + i * nb;
     }
   }
+  c->cur_cat = MEBP_WS_BWD;
   for (int k = 0; k < c->nsets; ++k) {
     Grads2& g = c->bw[k];
     A(&g.dqkv, T * c->Nqkv); A(&g.dgu, T * 2 * I); A(&g.dh1_h, T * D);
@@ -708,17 +847,22 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
       rc = MEBP_ERR_CUDA;
     }
   }
+  c->cur_cat = MEBP_WS_BWD;
   A(&c->dout, T * c->Na);
   for (int k = 0; k < (c->nsets == 2 ? 3 : 2); ++k) A(&c->dy_h[k], T * D);
   A(&c->dm, T * I); A(&c->dtmp, T * D); A(&c->dh1, T * D); A(&c->dvec, T * c->H);
   // split attention backward: 3 arrays of B * ceil(S/64) * H * 2 parts * 64 * hd floats (<= 2 T rows
   // per head and part when S >= 64), at most 192 MB; larger shapes take the direct mode
   c->attn_ws_floats = std::min<int64_t>(3LL * 2 * c->H * c->hd * 2 * T, 48LL << 20);
+  c->cur_cat = MEBP_WS_ATTN_SPLIT;
   A(&c->attn_ws, c->attn_ws_floats);
+  c->cur_cat = MEBP_WS_BWD;
   A(&c->gbuf[0], T * D); A(&c->gbuf[1], T * D);
   c->red_floats = std::max<int64_t>(tall_reduce_scratch_floats(T, std::max<int64_t>(2 * I, c->Nqkv), 32),
                                     tall_reduce_scratch_floats(T, std::max<int64_t>(I, D), 32));
+  c->cur_cat = MEBP_WS_OTHER;
   A(&c->red, c->red_floats);
+  c->cur_cat = MEBP_WS_LMHEAD;
   if (c->V > 0) {
     c->nparts = 4 * ((c->V + 255) / 256);  // four (max, sum) parts per 256-column tile
     int64_t vc = f.vocab_chunk;
@@ -731,9 +875,11 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
     A(&c->tok_loss, T); A(&c->dz, T * c->vchunk); A(&c->dhf, T * D); A(&c->targets, T);
   }
   const int64_t nslots = f.spill_ckpts ? kCkptSlots : (c->L + 1);
+  c->cur_cat = MEBP_WS_CKPT;
   A(&c->ckpt, nslots * T * D);
   if (rc == MEBP_OK && f.spill_ckpts) {
     const size_t hb = static_cast<size_t>(c->L + 1) * T * D * sizeof(float);
+    c->ws_cat[MEBP_WS_HOST_CKPT] = static_cast<int64_t>(hb);
     if (cudaHostAlloc(reinterpret_cast<void**>(&c->h_ckpt), hb, cudaHostAllocDefault) != cudaSuccess) {
       cudaGetLastError();
       c->h_ckpt = nullptr;
@@ -811,6 +957,13 @@ const char* mebp_last_error(const mebp_ctx* c) { return c ? c->err_msg.c_str() :
 
 int64_t mebp_workspace_bytes(const mebp_ctx* c) { return c ? c->ws_bytes : 0; }
 
+int mebp_workspace_breakdown(const mebp_ctx* c, int64_t* bytes, int* n_sets) {
+  if (!c || !bytes) return MEBP_ERR_INVALID_ARG;
+  for (int i = 0; i < MEBP_WS_N; ++i) bytes[i] = c->ws_cat[i];
+  if (n_sets) *n_sets = c->nsets;
+  return MEBP_OK;
+}
+
 int mebp_sync(mebp_ctx* c, void* stream) {
   if (!c) return MEBP_ERR_INVALID_ARG;
   if (cudaStreamSynchronize(S(stream)) != cudaSuccess) return fail(c, MEBP_ERR_CUDA, cudaGetErrorString(cudaGetLastError()));
@@ -819,8 +972,9 @@ int mebp_sync(mebp_ctx* c, void* stream) {
     return fail(c, MEBP_ERR_CUDA, cudaGetErrorString(cudaGetLastError()));
   if (h) {
     cudaMemset(c->d_err, 0, sizeof(int));
-    return fail(c, h, h == MEBP_ERR_TIMEOUT ? "a device-side bounded wait expired"
-                                            : "a kernel flagged invalid input (e.g. token id out of range)");
+    return fail(c, h, h == MEBP_ERR_TIMEOUT     ? "a device-side bounded wait expired"
+                      : h == MEBP_ERR_NONFINITE ? "an fp16 intermediate overflowed the fp16 range or is NaN"
+                                                : "a kernel flagged invalid input (e.g. token id out of range)");
   }
   return MEBP_OK;
 }
@@ -849,14 +1003,29 @@ int mebp_profile_end(mebp_ctx* c, mebp_profile* out) {
   if (!c || !out) return MEBP_ERR_INVALID_ARG;
   c->prof = false;
   mebp_profile p{};
+  c->kstats.assign(KK_N, mebp_kernel_stat{});
+  for (int k = 0; k < KK_N; ++k) c->kstats[k].name = kKindName[k];
+  // [start, end] of every fused-GEMM launch relative to the first record's start event; their union
+  // is the time during which some fused GEMM ran (launches on concurrent streams overlap)
+  std::vector<std::pair<double, double>> iv;
+  iv.reserve(c->recs.size());
   for (const ProfRec& r : c->recs) {
     if (cudaEventSynchronize(r.b) != cudaSuccess) return fail(c, MEBP_ERR_CUDA, cudaGetErrorString(cudaGetLastError()));
-    float ms = 0.0f;
+    float ms = 0.0f, t0 = 0.0f;
     cudaEventElapsedTime(&ms, r.a, r.b);
+    mebp_kernel_stat& ks = c->kstats[r.kind];
+    ks.launches++;
+    ks.ms += ms;
+    ks.bytes += r.bytes;
+    ks.flops += r.flops;
+    if (r.kind != KK_GEMM_FWD && r.kind != KK_GEMM_DX) continue;
+    cudaEventElapsedTime(&t0, c->recs.front().a, r.a);
+    iv.emplace_back(t0, static_cast<double>(t0) + ms);
     p.gemm_launches++;
     p.gemm_ms += ms;
     p.gemm_flops += r.flops;
-    if (r.trans) {
+    p.gemm_bytes += r.bytes;
+    if (r.kind == KK_GEMM_DX) {
       p.dx_ms += ms;
       p.dx_flops += r.flops;
     } else {
@@ -864,10 +1033,31 @@ int mebp_profile_end(mebp_ctx* c, mebp_profile* out) {
       p.fwd_flops += r.flops;
     }
   }
+  std::sort(iv.begin(), iv.end());
+  double busy = 0.0, cs = 0.0, ce = -1e300;
+  for (const auto& v : iv) {
+    if (v.first > ce) {
+      if (ce > cs) busy += ce - cs;
+      cs = v.first;
+      ce = v.second;
+    } else {
+      ce = std::max(ce, v.second);
+    }
+  }
+  if (!iv.empty() && ce > cs) busy += ce - cs;
+  p.gemm_busy_ms = busy;
   c->recs.clear();
   c->evnext = 0;
   *out = p;
   return cuda_check(c, "profile");
+}
+
+int mebp_profile_kernels(const mebp_ctx* c, mebp_kernel_stat* out, int max, int* n) {
+  if (!c || (!out && max > 0) || !n) return MEBP_ERR_INVALID_ARG;
+  const int k = static_cast<int>(c->kstats.size());
+  for (int i = 0; i < k && i < max; ++i) out[i] = c->kstats[i];
+  *n = k;
+  return MEBP_OK;
 }
 
 int mebp_compress_weights(mebp_ctx* c, const float* W, int64_t rows, int64_t cols, int group, uint8_t* qpack,
@@ -911,7 +1101,9 @@ static int linear_common(mebp_ctx* c, bool dx_mode, const uint16_t* X, int64_t M
   if (!W || !W->qpack || !W->scales || !X) return fail(c, MEBP_ERR_INVALID_ARG, "NULL pointer");
   const int64_t N = W->rows, K = W->cols;
   if (N % 64 || K % 64 || N <= 0 || K <= 0) return fail(c, MEBP_ERR_INVALID_ARG, "W dims must be multiples of 64");
-  if (!aligned16(X) || !aligned16(W->qpack) || !aligned16(W->scales))
+  // TMA reads X and the weights; the epilogue stores y and reads R as 16-byte vectors
+  if (!aligned16(X) || !aligned16(W->qpack) || !aligned16(W->scales) || !aligned16(y32) || !aligned16(y16) ||
+      !aligned16(R))
     return fail(c, MEBP_ERR_INVALID_ARG, "pointers must be 16-byte aligned");
   if ((A == nullptr) != (Bm == nullptr)) return fail(c, MEBP_ERR_INVALID_ARG, "A and B must both be set or both NULL");
   if (A && (r <= 0 || r > 32 || r % 8)) return fail(c, MEBP_ERR_UNSUPPORTED, "rank must be 8, 16, 24 or 32");
@@ -1102,7 +1294,12 @@ static int lora_step_body(mebp_ctx* c, const mebp_model_weights* model, const me
     wait_free(sl);
     x0 = dev_ckpt(sl);
   }
-  launch_embed(model->embed.qpack, model->embed.scales, c->V, D, ids, T, x0, c->d_err, embed_scale(c), st);
+  char rname[32];
+  nvtxRangePushA("emb");
+  KP(c, KK_EMBED, T * D * (0.5 + 1.0 / 16.0 + 4.0) + 4.0 * T, 0, st, [&] {
+    launch_embed(model->embed.qpack, model->embed.scales, c->V, D, ids, T, x0, c->d_err, embed_scale(c), st);
+  });
+  nvtxRangePop();
   if (spill) spill_out(0);
   // ---- forward loop: store only block-boundary checkpoints
   for (int i = 0; i < L; ++i) {
@@ -1113,17 +1310,21 @@ static int lora_step_body(mebp_ctx* c, const mebp_model_weights* model, const me
       wait_free(sl);  // its previous contents reached the host
       yout = dev_ckpt(sl);
     }
-    if ((rc = block_forward(c, i % c->nsets, i, &model->blocks[i], &lora[i], xin, yout, B, Sq, true, st,
-                            &c->layer_sh[i])))
-      return rc;
+    std::snprintf(rname, sizeof(rname), "f_%d", i);
+    nvtxRangePushA(rname);
+    rc = block_forward(c, i % c->nsets, i, &model->blocks[i], &lora[i], xin, yout, B, Sq, true, st, &c->layer_sh[i]);
+    nvtxRangePop();
+    if (rc) return rc;
     if (spill && i + 1 < L) spill_out(i + 1);
   }
   // ---- loss subgraph: final norm + LM head + CE
   const float* hL = spill ? dev_ckpt(slot_of[L]) : dev_ckpt(L);
   int cur = 0;
-  if ((rc = lmhead(c, &model->embed, model->final_norm, hL, c->targets, T, loss, c->gbuf[cur], c->dy_h[cur], nullptr,
-                   false, st)))
-    return rc;
+  nvtxRangePushA("lm");
+  rc = lmhead(c, &model->embed, model->final_norm, hL, c->targets, T, loss, c->gbuf[cur], c->dy_h[cur], nullptr, false,
+              st);
+  nvtxRangePop();
+  if (rc) return rc;
   if (spill) release(L);
   // ---- backward loop in reverse order: recompute block i from ckpt_i, apply its VJP.  With two
   // intermediate sets (no spilling) three streams share the work: the recompute of block i-1
@@ -1145,6 +1346,11 @@ static int lora_step_body(mebp_ctx* c, const mebp_model_weights* model, const me
     const float* xin = spill ? dev_ckpt(slot_of[i]) : dev_ckpt(i);
     const int set = i % c->nsets;
     const int nxt = cur ^ 1;
+    std::snprintf(rname, sizeof(rname), "b_%d", i);
+    nvtxRangePushA(rname);
+    struct PopOnExit {
+      ~PopOnExit() { nvtxRangePop(); }
+    } pop_on_exit;
     if (!overlap) {
       if ((rc = block_backward(c, set, 0, i, &model->blocks[i], &lora[i], xin, c->gbuf[cur], c->dy_h[cur],
                                i > 0 ? c->gbuf[nxt] : nullptr, i > 0 ? c->dy_h[nxt] : nullptr, &grads[i], B, Sq,

@@ -8,40 +8,70 @@
 // takes stream-ordered temporaries for the fp16 LoRA shadows and the rank-r product.
 //
 // Here that scratch is one file-scope device array of fixed size, present on every GPU that
-// loads the library for the life of the process.  Its device address is looked up once per
-// device (on the first call made while that device is current) and reused afterwards.
+// loads the library for the life of the process.  Its device address is looked up once per CUDA
+// context (on the first call made while that context is current) and reused afterwards; keying
+// by context rather than by device ordinal means a context created after a device reset, or a
+// non-primary context made current by the caller, gets its own lookup instead of a stale address.
+#include <cudaTypedefs.h>
+
 #include <mutex>
 
 #include "../../include/mebp.h"
 #include "kernels.h"
 
-#define MEBP_NOALLOC_MAX_DEVICES 64
+#define MEBP_NOALLOC_MAX_CONTEXTS 64
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[MEBP_NOALLOC_SCRATCH_BYTES];
 
 namespace {
 
 std::mutex g_noalloc_mu;
-void* g_noalloc_addr[MEBP_NOALLOC_MAX_DEVICES] = {};
+struct ScratchEntry {
+  CUcontext ctx;
+  void* addr;
+};
+ScratchEntry g_noalloc_cache[MEBP_NOALLOC_MAX_CONTEXTS] = {};
+int g_noalloc_n = 0;
 
-// Device address of g_noalloc_scratch on the current device (set up on first use).
+PFN_cuCtxGetCurrent_v4000 ctx_get_current() {
+  static PFN_cuCtxGetCurrent_v4000 fn = nullptr;
+  static bool tried = false;
+  if (!tried) {
+    tried = true;
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 4000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(f);
+    else
+      cudaGetLastError();
+  }
+  return fn;
+}
+
+// Device address of g_noalloc_scratch in the current context (looked up on first use).
 int noalloc_scratch(unsigned char** out) {
-  int dev = -1;
-  if (cudaGetDevice(&dev) != cudaSuccess) {
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  PFN_cuCtxGetCurrent_v4000 get = ctx_get_current();
+  if (!get) return MEBP_ERR_CUDA;
+  CUcontext cur = nullptr;
+  if (get(&cur) != CUDA_SUCCESS) return MEBP_ERR_CUDA;
+  if (cur)
+    for (int i = 0; i < g_noalloc_n; ++i)
+      if (g_noalloc_cache[i].ctx == cur) {
+        *out = static_cast<unsigned char*>(g_noalloc_cache[i].addr);
+        return MEBP_OK;
+      }
+  // Not cached (or no context current yet: the runtime makes the device's primary context
+  // current here).
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) {
     cudaGetLastError();
     return MEBP_ERR_CUDA;
   }
-  if (dev < 0 || dev >= MEBP_NOALLOC_MAX_DEVICES) return MEBP_ERR_UNSUPPORTED;
-  std::lock_guard<std::mutex> lock(g_noalloc_mu);
-  if (!g_noalloc_addr[dev]) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) {
-      cudaGetLastError();
-      return MEBP_ERR_CUDA;
-    }
-    g_noalloc_addr[dev] = p;
-  }
-  *out = static_cast<unsigned char*>(g_noalloc_addr[dev]);
+  if (!cur && get(&cur) != CUDA_SUCCESS) return MEBP_ERR_CUDA;
+  if (cur && g_noalloc_n < MEBP_NOALLOC_MAX_CONTEXTS) g_noalloc_cache[g_noalloc_n++] = {cur, p};
+  *out = static_cast<unsigned char*>(p);
   return MEBP_OK;
 }
 
@@ -56,8 +86,11 @@ extern "C" int mebp_linear_fwd_noalloc(const uint16_t* X, int64_t M, const mebp_
   if (!X || !W || !W->qpack || !W->scales || (!y_f32 && !y_f16)) return MEBP_ERR_INVALID_ARG;
   const int64_t N = W->rows, K = W->cols;
   if (N <= 0 || K <= 0 || N % 64 || K % 64) return MEBP_ERR_INVALID_ARG;
+  // 16-byte alignment: TMA reads X and the weights; the epilogue stores y and reads R as 16-byte
+  // vectors.
   if ((reinterpret_cast<uintptr_t>(X) | reinterpret_cast<uintptr_t>(W->qpack) |
-       reinterpret_cast<uintptr_t>(W->scales)) & 15)
+       reinterpret_cast<uintptr_t>(W->scales) | reinterpret_cast<uintptr_t>(y_f32) |
+       reinterpret_cast<uintptr_t>(y_f16) | reinterpret_cast<uintptr_t>(R)) & 15)
     return MEBP_ERR_INVALID_ARG;
   if ((A == nullptr) != (B == nullptr)) return MEBP_ERR_INVALID_ARG;
   if (A && (r <= 0 || r > 32 || r % 8)) return MEBP_ERR_UNSUPPORTED;

@@ -338,7 +338,9 @@ __device__ __forceinline__ float act_grad(float x, int act) {
 }
 
 // m = act(g) * u; gu row = [g (I) | u (I)].  8 elements per thread.
-__global__ void glu_fwd_kernel(const uint16_t* __restrict__ gu, int64_t T, int I, int act, uint16_t* __restrict__ m) {
+// A product outside the fp16 range (or NaN) sets MEBP_ERR_NONFINITE in *err.
+__global__ void glu_fwd_kernel(const uint16_t* __restrict__ gu, int64_t T, int I, int act, uint16_t* __restrict__ m,
+                               int* err) {
   griddep_wait();
   griddep_launch();
   const int per = I / 8;
@@ -353,12 +355,13 @@ __global__ void glu_fwd_kernel(const uint16_t* __restrict__ gu, int64_t T, int I
 #pragma unroll
   for (int k = 0; k < 4; ++k)
     o[k] = pack_half2(act_f(h2_lo(ga[k]), act) * h2_lo(ua[k]), act_f(h2_hi(ga[k]), act) * h2_hi(ua[k]));
+  if (h2_nonfinite(o[0]) | h2_nonfinite(o[1]) | h2_nonfinite(o[2]) | h2_nonfinite(o[3])) flag_error(err, kErrNonFinite);
   *reinterpret_cast<uint4*>(m + t * I + c) = make_uint4(o[0], o[1], o[2], o[3]);
 }
 
 // dg = dm * u * act'(g), du = dm * act(g)
 __global__ void glu_bwd_kernel(const uint16_t* __restrict__ dm, const uint16_t* __restrict__ gu, int64_t T, int I, int act,
-                               uint16_t* __restrict__ dgu) {
+                               uint16_t* __restrict__ dgu, int* err) {
   griddep_wait();
   griddep_launch();
   const int per = I / 8;
@@ -379,19 +382,24 @@ __global__ void glu_bwd_kernel(const uint16_t* __restrict__ dm, const uint16_t* 
     og[k] = pack_half2(dd[2 * k] * u0 * act_grad(g0, act), dd[2 * k + 1] * u1 * act_grad(g1, act));
     ou[k] = pack_half2(dd[2 * k] * act_f(g0, act), dd[2 * k + 1] * act_f(g1, act));
   }
+  uint32_t bad = 0;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) bad |= h2_nonfinite(og[k]) | h2_nonfinite(ou[k]);
+  if (bad) flag_error(err, kErrNonFinite);
   *reinterpret_cast<uint4*>(dgu + t * 2 * I + c) = make_uint4(og[0], og[1], og[2], og[3]);
   *reinterpret_cast<uint4*>(dgu + t * 2 * I + I + c) = make_uint4(ou[0], ou[1], ou[2], ou[3]);
 }
 
-void launch_glu_fwd(const uint16_t* gu, int64_t T, int I, int act, uint16_t* m, cudaStream_t st) {
+void launch_glu_fwd(const uint16_t* gu, int64_t T, int I, int act, uint16_t* m, int* err, cudaStream_t st) {
   const int64_t n = T * (I / 8);
   if (n <= 0) return;
-  launch_k(glu_fwd_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, st, gu, T, I, act, m);
+  launch_k(glu_fwd_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, st, gu, T, I, act, m, err);
 }
-void launch_glu_bwd(const uint16_t* dm, const uint16_t* gu, int64_t T, int I, int act, uint16_t* dgu, cudaStream_t st) {
+void launch_glu_bwd(const uint16_t* dm, const uint16_t* gu, int64_t T, int I, int act, uint16_t* dgu, int* err,
+                    cudaStream_t st) {
   const int64_t n = T * (I / 8);
   if (n <= 0) return;
-  launch_k(glu_bwd_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, st, dm, gu, T, I, act, dgu);
+  launch_k(glu_bwd_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, st, dm, gu, T, I, act, dgu, err);
 }
 
 // ------------------------------------------------------------------------------------ casts

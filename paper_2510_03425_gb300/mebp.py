@@ -17,9 +17,11 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "libmebp.so")
 HEADER = os.path.join(os.path.dirname(HERE), "include", "mebp.h")
 
-OK, ERR_INVALID_ARG, ERR_CUDA, ERR_OOM, ERR_TIMEOUT, ERR_UNSUPPORTED, ERR_DEVICE, ERR_SCRATCH = range(8)
+OK, ERR_INVALID_ARG, ERR_CUDA, ERR_OOM, ERR_TIMEOUT, ERR_UNSUPPORTED, ERR_DEVICE, ERR_SCRATCH, ERR_NONFINITE = range(9)
 NOALLOC_SCRATCH_BYTES = 8 << 20
 T_Q, T_K, T_V, T_O, T_GATE, T_UP, T_DOWN = range(7)
+WS_NAMES = ("checkpoints", "forward_sets", "backward", "attention_split", "lm_head", "lora_shadows", "other",
+            "host_checkpoints")
 TARGET_NAMES = ("q", "k", "v", "o", "gate", "up", "down")
 ACT = {"silu": 0, "gelu_tanh": 1}
 
@@ -36,7 +38,8 @@ class ModelCfg(ctypes.Structure):
                 ("rope_theta", c_float), ("rms_eps", c_float), ("lora_rank", c_int32), ("lora_scale", c_float),
                 ("lora_targets", c_uint32), ("max_tokens", c_int32), ("max_seq", c_int32),
                 ("spill_ckpts", c_int32), ("vocab_chunk", c_int32), ("gemma_norms", c_int32),
-                ("sliding_window", c_int32), ("global_every", c_int32), ("rope_theta_local", c_float)]
+                ("sliding_window", c_int32), ("global_every", c_int32), ("rope_theta_local", c_float),
+                ("min_memory", c_int32)]
 
 
 class Packed(ctypes.Structure):
@@ -60,7 +63,13 @@ class LoraGrads(ctypes.Structure):
 class Profile(ctypes.Structure):
     _fields_ = [("gemm_launches", c_int64), ("gemm_ms", ctypes.c_double), ("gemm_flops", ctypes.c_double),
                 ("fwd_ms", ctypes.c_double), ("fwd_flops", ctypes.c_double),
-                ("dx_ms", ctypes.c_double), ("dx_flops", ctypes.c_double)]
+                ("dx_ms", ctypes.c_double), ("dx_flops", ctypes.c_double), ("gemm_busy_ms", ctypes.c_double),
+                ("gemm_bytes", ctypes.c_double)]
+
+
+class KernelStat(ctypes.Structure):
+    _fields_ = [("name", c_char_p), ("launches", c_int64), ("ms", ctypes.c_double), ("bytes", ctypes.c_double),
+                ("flops", ctypes.c_double)]
 
 
 class AdamWCfg(ctypes.Structure):
@@ -78,6 +87,7 @@ _SIGS = {
     "mebp_last_error": (c_char_p, [c_void_p]),
     "mebp_sync": (c_int, [c_void_p, c_void_p]),
     "mebp_workspace_bytes": (c_int64, [c_void_p]),
+    "mebp_workspace_breakdown": (c_int, [c_void_p, POINTER(c_int64), POINTER(c_int)]),
     "mebp_compress_weights": (c_int, [c_void_p, c_void_p, c_int64, c_int64, c_int, c_void_p, c_void_p, c_void_p]),
     "mebp_decode_weights": (c_int, [c_void_p, POINTER(Packed), c_void_p, c_void_p]),
     "mebp_embed": (c_int, [c_void_p, POINTER(Packed), c_void_p, c_int64, c_void_p, c_void_p]),
@@ -97,6 +107,7 @@ _SIGS = {
     "mebp_enable_graphs": (c_int, [c_void_p, c_int]),
     "mebp_profile_begin": (c_int, [c_void_p]),
     "mebp_profile_end": (c_int, [c_void_p, POINTER(Profile)]),
+    "mebp_profile_kernels": (c_int, [c_void_p, POINTER(KernelStat), c_int, POINTER(c_int)]),
     "mebp_lora_step": (c_int, [c_void_p, POINTER(ModelWeights), POINTER(Lora), c_void_p, c_int, c_int, c_void_p,
                                POINTER(LoraGrads), c_int, c_void_p]),
     "mebp_adamw_step": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_int64, POINTER(AdamWCfg), c_int64,
@@ -179,7 +190,7 @@ def grads_struct(tensors: dict) -> LoraGrads:
     return G
 
 
-def model_cfg(dims, max_tokens=None, max_seq=None, spill=None, vocab_chunk=0) -> ModelCfg:
+def model_cfg(dims, max_tokens=None, max_seq=None, spill=None, vocab_chunk=0, min_memory=False) -> ModelCfg:
     """ModelCfg from a ``workload.ModelDims``-like object."""
     mask = sum(1 << TARGET_NAMES.index(t) for t in dims.targets)
     return ModelCfg(dims.hidden, dims.n_heads, dims.n_kv_heads, dims.head_dim, dims.intermediate, dims.vocab,
@@ -187,7 +198,8 @@ def model_cfg(dims, max_tokens=None, max_seq=None, spill=None, vocab_chunk=0) ->
                     mask, max_tokens or dims.batch * dims.seq, max_seq or dims.seq,
                     int(dims.spill if spill is None else spill), vocab_chunk,
                     int(getattr(dims, "gemma_norms", False)), int(getattr(dims, "sliding_window", 0)),
-                    int(getattr(dims, "global_every", 1)), float(getattr(dims, "rope_theta_local", 1e4)))
+                    int(getattr(dims, "global_every", 1)), float(getattr(dims, "rope_theta_local", 1e4)),
+                    int(min_memory))
 
 
 # ----------------------------------------------------------------------------- C entry points
@@ -213,6 +225,14 @@ def mebp_sync(ctx, stream=None):
 
 def mebp_workspace_bytes(ctx) -> int:
     return _lib.mebp_workspace_bytes(ctx)
+
+
+def mebp_workspace_breakdown(ctx) -> tuple:
+    """({purpose: bytes} in the order of WS_NAMES, number of intermediate sets)."""
+    arr = (c_int64 * len(WS_NAMES))()
+    n = c_int()
+    _check(ctx, _lib.mebp_workspace_breakdown(ctx, arr, ctypes.byref(n)))
+    return dict(zip(WS_NAMES, list(arr))), n.value
 
 
 def mebp_compress_weights(ctx, W, qpack, scales, group: int = 64, stream=None):
@@ -287,6 +307,15 @@ def mebp_profile_end(ctx) -> Profile:
     p = Profile()
     _check(ctx, _lib.mebp_profile_end(ctx, ctypes.byref(p)))
     return p
+
+
+def mebp_profile_kernels(ctx) -> dict:
+    """{kind: {"launches", "ms", "bytes", "flops"}} of the last profiled interval (kinds with launches)."""
+    arr = (KernelStat * 64)()
+    n = c_int()
+    _check(ctx, _lib.mebp_profile_kernels(ctx, arr, 64, ctypes.byref(n)))
+    return {arr[i].name.decode(): {"launches": arr[i].launches, "ms": arr[i].ms, "bytes": arr[i].bytes,
+                                   "flops": arr[i].flops} for i in range(min(n.value, 64)) if arr[i].launches}
 
 
 def mebp_enable_graphs(ctx, on: bool = True):

@@ -18,9 +18,11 @@ LINEARS = ("q", "k", "v", "o", "gate", "up", "down")
 class Context:
     """Owns one ``mebp_ctx``."""
 
-    def __init__(self, dims, device: int = 0, max_tokens=None, max_seq=None, spill=None, vocab_chunk=0):
+    def __init__(self, dims, device: int = 0, max_tokens=None, max_seq=None, spill=None, vocab_chunk=0,
+                 min_memory=False):
         self.dims = dims
-        self.cfg = M.model_cfg(dims, max_tokens=max_tokens, max_seq=max_seq, spill=spill, vocab_chunk=vocab_chunk)
+        self.cfg = M.model_cfg(dims, max_tokens=max_tokens, max_seq=max_seq, spill=spill, vocab_chunk=vocab_chunk,
+                               min_memory=min_memory)
         self.handle = M.mebp_ctx_create(self.cfg, device)
 
     def close(self):

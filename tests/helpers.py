@@ -35,3 +35,17 @@ def np_of(t):
 
 def dense_blocks(dims, n=None, seed=0, **kw):
     return [synth.block_weights(dims, i, seed=seed, **kw) for i in range(n if n is not None else dims.n_layers)]
+
+
+def rowblock_err(got, ref, rows: int = 64) -> float:
+    """Worst element-wise error of a row block relative to that block's largest reference value:
+    max over blocks of max|got - ref| / max|ref|, blocks of `rows` consecutive rows (the
+    kernels' tile height).  A wrong ragged tile or sequence boundary that touches a few rows
+    shows here even when a norm over thousands of rows hides it."""
+    a = np.asarray(got, np.float64).reshape(np.shape(got)[0], -1)
+    b = np.asarray(ref, np.float64).reshape(a.shape)
+    worst = 0.0
+    for r0 in range(0, a.shape[0], rows):
+        d = np.abs(a[r0:r0 + rows] - b[r0:r0 + rows]).max()
+        worst = max(worst, float(d / max(np.abs(b[r0:r0 + rows]).max(), 1e-30)))
+    return worst

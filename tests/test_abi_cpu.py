@@ -83,3 +83,19 @@ def test_null_context_is_rejected(binding):
     assert lib.mebp_sync(None, None) == binding.ERR_INVALID_ARG
     assert lib.mebp_lora_step(None, None, None, None, 1, 1, None, None, 0, None) == binding.ERR_INVALID_ARG
     assert lib.mebp_last_error(None) == b"NULL context"
+
+
+@pytest.mark.parametrize("which", ["X", "qpack", "scales", "y_f32", "y_f16", "R"])
+def test_noalloc_rejects_misaligned_pointers_before_touching_cuda(binding, which):
+    """The fused GEMM reads X and the weights by TMA and stores y / reads R as 16-byte vectors:
+    a pointer off a 16-byte boundary is refused on the host, before any CUDA call (the
+    addresses below are never dereferenced)."""
+    ptrs = dict(X=0x10000, qpack=0x20000, scales=0x30000, y_f32=0x40000, y_f16=None, R=0x50000)
+    if which == "y_f16":
+        ptrs["y_f32"] = None
+        ptrs["y_f16"] = 0x40000
+    ptrs[which] += 8
+    W = binding.Packed(ptrs["qpack"], ptrs["scales"], 64, 128)
+    rc = binding.lib().mebp_linear_fwd_noalloc(ptrs["X"], 16, ctypes.byref(W), None, None, 0, 1.0, ptrs["R"],
+                                                ptrs["y_f32"], ptrs["y_f16"], None)
+    assert rc == binding.ERR_INVALID_ARG

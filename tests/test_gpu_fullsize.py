@@ -3,9 +3,10 @@ on outputs the oracle can compute one sample at a time:
 
 * fused GEMMs at M = 16384 (Gemma3-4B-shaped projections): sampled rows;
 * one decoder block of the Gemma3-1B / Qwen2.5-1.5B / Gemma3-4B-shaped models run over the
-  full batch, with the upstream gradient non-zero on sequence 0 only — sequences do not
-  interact, so y and dE/dx of sequence 0 and every LoRA gradient equal the oracle's block
-  run on sequence 0 alone;
+  full batch, with the upstream gradient non-zero on the first and the last sequence only —
+  sequences do not interact, so y of every sequence equals the oracle's block run on that
+  sequence alone (element-wise), dE/dx of the two graded sequences equals the oracle's, dE/dx
+  of the others is zero, and every LoRA gradient is the sum over the two graded sequences;
 * the LM head over the full vocabulary: per-token loss and dE/dh on sampled tokens.
 """
 import numpy as np
@@ -15,8 +16,8 @@ from oracle import model as OM
 from oracle import quant
 from workload import synth
 
-from .helpers import f16_round, np_of, rel_fro, to_gpu
-from .test_gpu_block import oracle_dense
+from .helpers import f16_round, np_of, rel_fro, rowblock_err, to_gpu
+from .test_gpu_block import ELEM_TOL, oracle_dense
 
 pytestmark = [pytest.mark.gpu, pytest.mark.slow]
 
@@ -57,34 +58,56 @@ def test_gemm_rows_at_full_size(name, N, K):
 
 
 @pytest.mark.parametrize("cfg", [2, 3, 4])
-def test_block_at_full_batch_against_sequence_zero(cfg):
+def test_block_at_full_batch_against_per_sequence_oracle(cfg):
     dims = synth.preset(cfg)
     W = synth.block_weights(dims, 0)
     L = synth.lora_weights(dims, 0)
     x = synth.hidden_input(dims)
     G = synth.upstream_grad(dims)
-    G[dims.seq:] = 0.0                        # only sequence 0 carries gradient
+    S, B = dims.seq, dims.batch
+    graded = sorted({0, B - 1})               # the first and the last sequence carry gradient
+    for b in range(B):
+        if b not in graded:
+            G[b * S:(b + 1) * S] = 0.0
     ctx = Context(dims)
     blk = DeviceBlock(ctx, {k: to_gpu(v) for k, v in W.items()})
     ls = LoraSet([L])
     xg, Gg = to_gpu(x), to_gpu(G)
     y = torch.empty_like(xg)
     dx = torch.empty_like(xg)
-    M.mebp_block_recompute_fwd(ctx.handle, 0, blk.struct(), ls.layer(0), xg, y, dims.batch, dims.seq, False)
-    M.mebp_block_bwd(ctx.handle, 0, blk.struct(), ls.layer(0), xg, Gg, dx, ls.layer_grads(0), dims.batch, dims.seq)
+    M.mebp_block_recompute_fwd(ctx.handle, 0, blk.struct(), ls.layer(0), xg, y, B, S, False)
+    M.mebp_block_bwd(ctx.handle, 0, blk.struct(), ls.layer(0), xg, Gg, dx, ls.layer_grads(0), B, S)
     ctx.sync()
-    S = dims.seq
+    y_np, dx_np = np_of(y), np_of(dx)
     d1 = dims.with_(batch=1)
     Wd = oracle_dense(W)
     Lo = OM.lora64(L)
-    x0 = x[:S].astype(np.float64)
-    yo, _ = OM.block_forward(x0, Wd, Lo, d1)
-    _, dxo, go = OM.block_objective(x0, Wd, Lo, G[:S].astype(np.float64), d1)
-    assert rel_fro(np_of(y[:S]) - x0, yo - x0) < 2e-2
-    assert rel_fro(np_of(dx[:S]), dxo) < 2e-2
-    if dims.batch > 1:
-        assert float(dx[S:].abs().max()) == 0.0
-    for n, (dA, dB) in go.items():
+    # sequences do not interact: the oracle runs each one alone
+    for b in range(B):
+        rows = slice(b * S, (b + 1) * S)
+        xb = x[rows].astype(np.float64)
+        if b in graded:
+            continue
+        yo, _ = OM.block_forward(xb, Wd, Lo, d1)
+        e = rowblock_err(y_np[rows] - xb, yo - xb)
+        assert e < ELEM_TOL, (b, "y", e)
+        assert float(np.abs(dx_np[rows]).max()) == 0.0, b
+    grads = {}
+    for b in graded:
+        rows = slice(b * S, (b + 1) * S)
+        xb = x[rows].astype(np.float64)
+        yo, _ = OM.block_forward(xb, Wd, Lo, d1)
+        _, dxo, go = OM.block_objective(xb, Wd, Lo, G[rows].astype(np.float64), d1)
+        ey, ed = rowblock_err(y_np[rows] - xb, yo - xb), rowblock_err(dx_np[rows], dxo)
+        print(f"sequence {b}: element-wise row-block error y - x {ey:.2e}, dx {ed:.2e}")
+        assert rel_fro(y_np[rows] - xb, yo - xb) < 2e-2
+        assert rel_fro(dx_np[rows], dxo) < 2e-2
+        assert ey < ELEM_TOL and ed < ELEM_TOL, (b, ey, ed)
+        for n, (dA, dB) in go.items():
+            pa, pb = grads.get(n, (0.0, 0.0))
+            grads[n] = (pa + dA, pb + dB)
+    # LoRA gradients of the batch = the sum over the graded sequences
+    for n, (dA, dB) in grads.items():
         a, b = ls.grads[0][n]
         assert rel_fro(np_of(a), dA) < 2e-2, (n, "dA", rel_fro(np_of(a), dA))
         assert rel_fro(np_of(b), dB) < 2e-2, (n, "dB", rel_fro(np_of(b), dB))

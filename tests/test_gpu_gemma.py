@@ -12,7 +12,7 @@ from oracle import model as OM
 from oracle import quant
 from workload import synth
 
-from .helpers import dense_blocks, np_of, rel_fro, to_gpu
+from .helpers import dense_blocks, np_of, rel_fro, rowblock_err, to_gpu
 
 pytestmark = pytest.mark.gpu
 
@@ -25,6 +25,7 @@ from paper_2510_03425_gb300.model import (Context, DeviceBlock, DeviceModel, Lor
                                           compress)
 
 TOL = 2e-2  # relative Frobenius error (fp16 operands, fp32 accumulate), as for the plain block
+ELEM_TOL = 2e-2  # element-wise, per 64-row block relative to the block's largest value (as for the plain block)
 
 
 def oracle_dense(W):
@@ -57,6 +58,9 @@ def run_block(dims, layer):
     _, dxo, go = OM.block_objective(xo, Wd, Lo, G.astype(np.float64), dims, layer=layer)
     assert rel_fro(np_of(y) - xo, yo - xo) < TOL
     assert rel_fro(np_of(dx), dxo) < TOL, rel_fro(np_of(dx), dxo)
+    ey, ed = rowblock_err(np_of(y) - xo, yo - xo), rowblock_err(np_of(dx), dxo)
+    print(f"element-wise row-block error: y - x {ey:.2e}, dx {ed:.2e}")
+    assert ey < ELEM_TOL and ed < ELEM_TOL, (ey, ed)
     for n, (dA, dB) in go.items():
         a, b = ls.grads[0][n]
         assert rel_fro(np_of(b), dB) < TOL, (n, "dB", rel_fro(np_of(b), dB))

@@ -184,3 +184,70 @@ def test_linear_rejects_bad_shapes(ctx):
     with pytest.raises(M.MebpError) as ei:
         M.mebp_linear_fwd(ctx.handle, X, M.packed(q, s), y_f32=y)
     assert ei.value.code == M.ERR_INVALID_ARG
+
+
+def test_linear_rejects_misaligned_outputs_and_residual(ctx):
+    """y and R are stored / read as 16-byte vectors: views off a 16-byte boundary are refused on
+    the host with MEBP_ERR_INVALID_ARG (nothing is launched)."""
+    Mr, N, K = 4, 64, 64
+    qo, so = quant.compress(_w(N, K, 1))
+    Wp = M.packed(to_gpu(qo), to_gpu(so))
+    X = torch.zeros((Mr, K), dtype=torch.float16, device="cuda")
+    buf = torch.zeros(Mr * N + 4, device="cuda")
+    off = buf[2:2 + Mr * N].view(Mr, N)          # 8 bytes past a 16-byte boundary
+    good = torch.zeros((Mr, N), device="cuda")
+    buf16 = torch.zeros(Mr * N + 8, dtype=torch.float16, device="cuda")
+    off16 = buf16[4:4 + Mr * N].view(Mr, N)
+    for kw in (dict(y_f32=off), dict(y_f16=off16), dict(y_f32=good, R=off)):
+        with pytest.raises(M.MebpError) as ei:
+            M.mebp_linear_fwd(ctx.handle, X, Wp, **kw)
+        assert ei.value.code == M.ERR_INVALID_ARG
+    with pytest.raises(M.MebpError) as ei:
+        M.mebp_linear_dx(ctx.handle, torch.zeros((Mr, N), dtype=torch.float16, device="cuda"), Wp, dx=off)
+    assert ei.value.code == M.ERR_INVALID_ARG
+    ctx.sync()
+
+
+def test_fp16_overflow_is_reported_not_silent(ctx):
+    """A GEMM output stored as fp16 that leaves the fp16 range (|y| > 65504) sets MEBP_ERR_NONFINITE,
+    reported by mebp_sync; the fp32 output of the same product is fine, and the error word is
+    cleared afterwards (inputs chosen on the host so that |y| ~ 1e5: only an inf is produced)."""
+    Mr, N, K = 64, 128, 256
+    W = np.full((N, K), 0.25, np.float32)
+    qo, so = quant.compress(W)
+    Wp = M.packed(to_gpu(qo), to_gpu(so))
+    X = torch.full((Mr, K), 2000.0, device="cuda", dtype=torch.float16)   # y = 256 * 2000 * 0.25 = 128000
+    y32 = torch.empty((Mr, N), device="cuda")
+    M.mebp_linear_fwd(ctx.handle, X, Wp, y_f32=y32)
+    ctx.sync()
+    assert float(y32.max()) == pytest.approx(128000.0, rel=1e-3)
+    y16 = torch.empty((Mr, N), device="cuda", dtype=torch.float16)
+    M.mebp_linear_fwd(ctx.handle, X, Wp, y_f16=y16)
+    with pytest.raises(M.MebpError) as ei:
+        ctx.sync()
+    assert ei.value.code == M.ERR_NONFINITE
+    X.fill_(1.0)
+    M.mebp_linear_fwd(ctx.handle, X, Wp, y_f16=y16)
+    ctx.sync()                                     # the error word was cleared; in range now
+    assert torch.isfinite(y16.float()).all()
+
+
+def test_gated_mlp_overflow_is_reported():
+    """The gated-MLP product m = act(g) u is stored as fp16: a block whose gate / up outputs are
+    large enough that m leaves the fp16 range reports MEBP_ERR_NONFINITE at mebp_sync."""
+    from paper_2510_03425_gb300.model import DeviceBlock, LoraSet
+    dims = synth.tiny(hidden=256, n_heads=4, n_kv_heads=2, head_dim=64, intermediate=256, n_layers=1, vocab=0,
+                      batch=1, seq=64, rank=8, alpha=16.0, targets=())
+    W = synth.block_weights(dims, 0)
+    W["gate"] = np.full_like(W["gate"], 0.06)      # b = norm(h1) * 24 ~ 24, so g = u ~ 0.06 * 256 * 24 = 369
+    W["up"] = np.full_like(W["up"], 0.06)          # and m = silu(g) u ~ 1.4e5 > 65504 (g, u themselves fit)
+    W["norm2"] = np.full_like(W["norm2"], 24.0)
+    c = Context(dims)
+    blk = DeviceBlock(c, {k: to_gpu(v) for k, v in W.items()})
+    x = to_gpu(np.ones((dims.tokens, dims.hidden), np.float32))
+    y = torch.empty_like(x)
+    M.mebp_block_recompute_fwd(c.handle, 0, blk.struct(), LoraSet([{}]).layer(0), x, y, 1, dims.seq, False)
+    with pytest.raises(M.MebpError) as ei:
+        c.sync()
+    assert ei.value.code == M.ERR_NONFINITE
+    c.close()

@@ -141,9 +141,10 @@ def block_weights(d: ModelDims, layer: int, seed: int = 0, norm_jitter: float = 
     return out
 
 
-def embedding(d: ModelDims, seed: int = 0, std: float = 0.02, norm_jitter: float = 0.0):
-    """Tied embedding / LM-head matrix E [V, D] and the final RMSNorm gain [D]."""
-    E = _normal(seed, (10_000, 0), (d.vocab, d.hidden), std)
+def embedding(d: ModelDims, seed: int = 0, std: float = 0.02, norm_jitter: float = 0.0, rows: int = 0):
+    """Tied embedding / LM-head matrix E [V, D] and the final RMSNorm gain [D]; rows > 0 draws only
+    the first `rows` rows (the same values as E[:rows])."""
+    E = _normal(seed, (10_000, 0), (rows if rows > 0 else d.vocab, d.hidden), std)
     g = np.ones(d.hidden, np.float32)
     if norm_jitter:
         g += _normal(seed, (10_000, 1), (d.hidden,), norm_jitter)
