@@ -115,6 +115,10 @@ int launch_dequant_gemm_narrow(const GemmArgs& g, cudaStream_t st);
 // 2-D tiled TMA descriptor: dims {d0 (inner), d1}, row pitch in bytes, box {b0, b1}.
 int make_tmap_2d(CUtensorMap* m, const void* base, CUtensorMapDataType dt, int elem_bytes, uint64_t d0, uint64_t d1,
                  uint64_t pitch_bytes, uint32_t b0, uint32_t b1, CUtensorMapSwizzle swz);
+// 3-D tiled TMA descriptor: dims {d0 (inner), d1, d2}, pitches of d1 and d2 in bytes, box {b0, b1, b2}.
+int make_tmap_3d(CUtensorMap* m, const void* base, CUtensorMapDataType dt, int elem_bytes, uint64_t d0, uint64_t d1,
+                 uint64_t d2, uint64_t pitch1_bytes, uint64_t pitch2_bytes, uint32_t b0, uint32_t b1, uint32_t b2,
+                 CUtensorMapSwizzle swz);
 int gemm_smem_bytes();
 
 void launch_compress(const float* W, int64_t rows, int64_t cols, uint8_t* qpack, uint16_t* scales, cudaStream_t st);
@@ -168,8 +172,13 @@ void launch_loss_reduce(const float* tok_loss, const int32_t* targets, int64_t T
 
 // LoRA helpers.
 // out[m, j] = alpha * sum_k X[m, k] W[j, k]  (fp16 in, fp16 out with columns J..ldo-1 zeroed)
+// err: device error word for a bounded wait that expires (may be null).
 void launch_skinny_gemm(const uint16_t* X, int64_t ldx, int64_t M, int64_t K, const uint16_t* W, int64_t ldw, int J,
-                        float alpha, uint16_t* out, int64_t ldo, cudaStream_t st);
+                        float alpha, uint16_t* out, int64_t ldo, cudaStream_t st, int* err = nullptr);
+// The same on tcgen05 with a TMA ring (large M); ldo in {16, 32, 48, 64, 80, 96}, K % 64 == 0,
+// X / W 16-byte aligned with row pitches that are multiples of 8 elements.
+int launch_skinny_tc(const uint16_t* X, int64_t ldx, int64_t M, int64_t K, const uint16_t* W, int64_t ldw,
+                     float alpha, uint16_t* out, int64_t ldo, int* err, cudaStream_t st);
 // C[p, q] (+)= sum_m P[m, p0 + p] Q[m, q0 + q], p < Pw, q < Qw; deterministic split over m.
 // The sum is multiplied by *mult (mult may be null = 1) before it is written / added.
 int launch_tall_reduce(const uint16_t* P, int64_t ldp, const uint16_t* Q, int64_t ldq, int64_t M, int Pw, int Qw,
@@ -209,8 +218,11 @@ void launch_lora_shadow(const float* const* A, const float* const* B, int nt, co
 
 // Attention (causal GQA).  q/k/v live inside the fused qkv buffer (row pitch ld).
 // window > 0: query i sees keys i - window + 1 .. i (sliding-window local layers); 0 = causal.
-void launch_attn_fwd(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, int hd, uint16_t* o, int64_t ldo,
-                     float* lse, int window, cudaStream_t st);
+int launch_attn_fwd(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, int hd, uint16_t* o, int64_t ldo,
+                    float* lse, int window, int* err, cudaStream_t st);
+// The forward on tcgen05 (attention_tc.cu); ld % 64 == 0, ldo % 8 == 0.
+int launch_attn_fwd_tc(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, int hd, uint16_t* o, int64_t ldo,
+                       float* lse, int window, int* err, cudaStream_t st);
 void launch_adamw(float* p, const float* g, float* m, float* v, int64_t n, float lr, float b1, float b2, float eps,
                   float wd, float gs, double bc1, double bc2, cudaStream_t st);
 // Backward into dqkv.  Small grids run the split mode through the fp32 workspace ws (needs

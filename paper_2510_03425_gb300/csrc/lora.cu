@@ -221,9 +221,19 @@ bool skinny_slab_launch(const uint16_t* X, int64_t ldx, int64_t M, int64_t K, co
   return true;
 }
 
+// Token counts above this stream X through the tcgen05 kernel (skinny_tc.cu): with the warp-level
+// kernel's two small cp.async stages per CTA the X pass ran at under a tenth of HBM bandwidth at
+// 16384 tokens.
+constexpr int64_t kSkinnyTcMinM = 1024;
+
 template <int NT>
 void skinny_launch(const uint16_t* X, int64_t ldx, int64_t M, int64_t K, const uint16_t* W, int64_t ldw, float alpha,
-                   uint16_t* out, int64_t ldo, cudaStream_t st) {
+                   uint16_t* out, int64_t ldo, cudaStream_t st, int* err) {
+  if (M > kSkinnyTcMinM && K % 64 == 0 && ldx % 8 == 0 && ldw % 8 == 0 &&
+      !((reinterpret_cast<uintptr_t>(X) | reinterpret_cast<uintptr_t>(W)) & 15)) {
+    launch_skinny_tc(X, ldx, M, K, W, ldw, alpha, out, ldo, err, st);
+    return;
+  }
   if (skinny_slab_launch<NT>(X, ldx, M, K, W, ldw, alpha, out, ldo, st)) return;
   const int gx = static_cast<int>((M + 63) / 64);
   const int nk = static_cast<int>(K / 64);
@@ -238,15 +248,15 @@ void skinny_launch(const uint16_t* X, int64_t ldx, int64_t M, int64_t K, const u
 }
 
 void launch_skinny_gemm(const uint16_t* X, int64_t ldx, int64_t M, int64_t K, const uint16_t* W, int64_t ldw, int J,
-                        float alpha, uint16_t* out, int64_t ldo, cudaStream_t st) {
+                        float alpha, uint16_t* out, int64_t ldo, cudaStream_t st, int* err) {
   (void)J;  // W holds ldo rows (zero beyond the used ranks), so every output column is written
   if (M <= 0) return;
   switch (ldo) {
-    case 16: skinny_launch<2>(X, ldx, M, K, W, ldw, alpha, out, ldo, st); break;
-    case 32: skinny_launch<4>(X, ldx, M, K, W, ldw, alpha, out, ldo, st); break;
-    case 48: skinny_launch<6>(X, ldx, M, K, W, ldw, alpha, out, ldo, st); break;
-    case 64: skinny_launch<8>(X, ldx, M, K, W, ldw, alpha, out, ldo, st); break;
-    default: skinny_launch<12>(X, ldx, M, K, W, ldw, alpha, out, ldo, st); break;
+    case 16: skinny_launch<2>(X, ldx, M, K, W, ldw, alpha, out, ldo, st, err); break;
+    case 32: skinny_launch<4>(X, ldx, M, K, W, ldw, alpha, out, ldo, st, err); break;
+    case 48: skinny_launch<6>(X, ldx, M, K, W, ldw, alpha, out, ldo, st, err); break;
+    case 64: skinny_launch<8>(X, ldx, M, K, W, ldw, alpha, out, ldo, st, err); break;
+    default: skinny_launch<12>(X, ldx, M, K, W, ldw, alpha, out, ldo, st, err); break;
   }
 }
 

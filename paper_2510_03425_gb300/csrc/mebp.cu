@@ -391,7 +391,7 @@ int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, 
   GemmArgs g = gemm_fwd(A.a, D, T, w->qkv, lq.N, lq.K);
   if (lq.kx) {
     KP(c, KK_LORA_SKINNY, bytes_skinny(T, D, lq.kx, lq.kxp), 2.0 * T * D * lq.kx, st, [&] {
-      launch_skinny_gemm(A.a, D, T, D, A.sh->A_cat[LIN_QKV], D, lq.kx, c->s, A.us[LIN_QKV], lq.kxp, st);
+      launch_skinny_gemm(A.a, D, T, D, A.sh->A_cat[LIN_QKV], D, lq.kx, c->s, A.us[LIN_QKV], lq.kxp, st, c->d_err);
     });
     g.Ax = A.us[LIN_QKV]; g.ldax = lq.kxp; g.kx = lq.kxp; g.Bx = A.sh->B_cat[LIN_QKV]; g.ldbx = lq.kxp;
   }
@@ -409,14 +409,17 @@ int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, 
     const int win = layer_window(c, layer) >= Sq ? 0 : layer_window(c, layer);
     KP(c, KK_ATTN_FWD, bytes_attn_fwd(T, c->H, c->KV, c->hd),
        c->prof ? attn_fwd_flops(B, Sq, c->H, c->hd, win) : 0.0, st, [&] {
-         launch_attn_fwd(A.qkv, lq.N, B, Sq, c->H, c->KV, c->hd, A.o, c->Na, A.lse_attn, layer_window(c, layer), st);
+         rc = launch_attn_fwd(A.qkv, lq.N, B, Sq, c->H, c->KV, c->hd, A.o, c->Na, A.lse_attn, layer_window(c, layer),
+                              c->d_err, st);
        });
+    if (rc) return fail(c, rc, "attention forward launch failed");
   }
   const Lin& lo = c->lin[LIN_O];
   g = gemm_fwd(A.o, c->Na, T, w->o, lo.N, lo.K);
   if (lo.kx) {
     KP(c, KK_LORA_SKINNY, bytes_skinny(T, c->Na, lo.kx, lo.kxp), 2.0 * T * c->Na * lo.kx, st, [&] {
-      launch_skinny_gemm(A.o, c->Na, T, c->Na, A.sh->A_cat[LIN_O], c->Na, lo.kx, c->s, A.us[LIN_O], lo.kxp, st);
+      launch_skinny_gemm(A.o, c->Na, T, c->Na, A.sh->A_cat[LIN_O], c->Na, lo.kx, c->s, A.us[LIN_O],
+          lo.kxp, st, c->d_err);
     });
     g.Ax = A.us[LIN_O]; g.ldax = lo.kxp; g.kx = lo.kxp; g.Bx = A.sh->B_cat[LIN_O]; g.ldbx = lo.kxp;
   }
@@ -437,7 +440,7 @@ int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, 
   g = gemm_fwd(A.b, D, T, w->gate_up, lg.N, lg.K);
   if (lg.kx) {
     KP(c, KK_LORA_SKINNY, bytes_skinny(T, D, lg.kx, lg.kxp), 2.0 * T * D * lg.kx, st, [&] {
-      launch_skinny_gemm(A.b, D, T, D, A.sh->A_cat[LIN_GU], D, lg.kx, c->s, A.us[LIN_GU], lg.kxp, st);
+      launch_skinny_gemm(A.b, D, T, D, A.sh->A_cat[LIN_GU], D, lg.kx, c->s, A.us[LIN_GU], lg.kxp, st, c->d_err);
     });
     g.Ax = A.us[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = A.sh->B_cat[LIN_GU]; g.ldbx = lg.kxp;
   }
@@ -447,7 +450,7 @@ int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, 
   const Lin& ld = c->lin[LIN_DOWN];
   if (ld.kx)
     KP(c, KK_LORA_SKINNY, bytes_skinny(T, I, ld.kx, ld.kxp), 2.0 * T * I * ld.kx, st, [&] {
-      launch_skinny_gemm(A.m, I, T, I, A.sh->A_cat[LIN_DOWN], I, ld.kx, c->s, A.us[LIN_DOWN], ld.kxp, st);
+      launch_skinny_gemm(A.m, I, T, I, A.sh->A_cat[LIN_DOWN], I, ld.kx, c->s, A.us[LIN_DOWN], ld.kxp, st, c->d_err);
     });
   if (with_down || c->gemma) {
     g = gemm_fwd(A.m, I, T, w->down, ld.N, ld.K);
@@ -552,7 +555,7 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   GemmArgs g = gemm_dx(ddn_h, D, T, w->down);
   if (ld.kx) {
     KP(c, KK_LORA_SKINNY, bytes_skinny(T, D, ld.kx, ld.kxp), 2.0 * T * D * ld.kx, st, [&] {
-      launch_skinny_gemm(ddn_h, D, T, D, A.sh->Bt_cat[LIN_DOWN], D, ld.kx, c->s, du[LIN_DOWN], ld.kxp, st);
+      launch_skinny_gemm(ddn_h, D, T, D, A.sh->Bt_cat[LIN_DOWN], D, ld.kx, c->s, du[LIN_DOWN], ld.kxp, st, c->d_err);
     });
     g.Ax = du[LIN_DOWN]; g.ldax = ld.kxp; g.kx = ld.kxp; g.Bx = A.sh->A_cat[LIN_DOWN]; g.ldbx = I;
   }
@@ -566,7 +569,8 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   g = gemm_dx(G.dgu, 2 * I, T, w->gate_up);
   if (lg.kx) {
     KP(c, KK_LORA_SKINNY, bytes_skinny(T, 2 * I, lg.kx, lg.kxp), 4.0 * T * I * lg.kx, st, [&] {
-      launch_skinny_gemm(G.dgu, 2 * I, T, 2 * I, A.sh->Bt_cat[LIN_GU], 2 * I, lg.kx, c->s, du[LIN_GU], lg.kxp, st);
+      launch_skinny_gemm(G.dgu, 2 * I, T, 2 * I, A.sh->Bt_cat[LIN_GU], 2 * I, lg.kx, c->s, du[LIN_GU],
+          lg.kxp, st, c->d_err);
     });
     g.Ax = du[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = A.sh->A_cat[LIN_GU]; g.ldbx = D;
   }
@@ -590,7 +594,7 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   g = gemm_dx(G.dh1_h, D, T, w->o);
   if (lo.kx) {
     KP(c, KK_LORA_SKINNY, bytes_skinny(T, D, lo.kx, lo.kxp), 2.0 * T * D * lo.kx, st, [&] {
-      launch_skinny_gemm(G.dh1_h, D, T, D, A.sh->Bt_cat[LIN_O], D, lo.kx, c->s, du[LIN_O], lo.kxp, st);
+      launch_skinny_gemm(G.dh1_h, D, T, D, A.sh->Bt_cat[LIN_O], D, lo.kx, c->s, du[LIN_O], lo.kxp, st, c->d_err);
     });
     g.Ax = du[LIN_O]; g.ldax = lo.kxp; g.kx = lo.kxp; g.Bx = A.sh->A_cat[LIN_O]; g.ldbx = c->Na;
   }
@@ -620,7 +624,8 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
   // ---- q, k, v projections
   if (lq.kx)
     KP(c, KK_LORA_SKINNY, bytes_skinny(T, lq.N, lq.kx, lq.kxp), 2.0 * T * lq.N * lq.kx, st, [&] {
-      launch_skinny_gemm(G.dqkv, lq.N, T, lq.N, A.sh->Bt_cat[LIN_QKV], lq.N, lq.kx, c->s, du[LIN_QKV], lq.kxp, st);
+      launch_skinny_gemm(G.dqkv, lq.N, T, lq.N, A.sh->Bt_cat[LIN_QKV], lq.N, lq.kx, c->s, du[LIN_QKV],
+          lq.kxp, st, c->d_err);
     });
   if ((rc = lin_grads(c, A, du[LIN_QKV], LIN_QKV, G.dqkv, lq.N, A.a, D, T, grads, acc, grad_mult, st, tb))) return rc;
   if (dx) {
@@ -1132,7 +1137,7 @@ static int linear_common(mebp_ctx* c, bool dx_mode, const uint16_t* X, int64_t M
   if (!dx_mode) {
     g = gemm_fwd(X, K, M, *W, static_cast<int>(N), static_cast<int>(K));
     if (A) {
-      launch_skinny_gemm(X, K, M, K, Ac, K, r, s, u, kxp, st);
+      launch_skinny_gemm(X, K, M, K, Ac, K, r, s, u, kxp, st, c->d_err);
       g.Ax = u; g.ldax = kxp; g.kx = kxp; g.Bx = Bc; g.ldbx = kxp;
     }
     if (y32) {
@@ -1143,7 +1148,7 @@ static int linear_common(mebp_ctx* c, bool dx_mode, const uint16_t* X, int64_t M
   } else {
     g = gemm_dx(X, N, M, *W);
     if (A) {
-      launch_skinny_gemm(X, N, M, N, Btc, N, r, s, u, kxp, st);
+      launch_skinny_gemm(X, N, M, N, Btc, N, r, s, u, kxp, st, c->d_err);
       g.Ax = u; g.ldax = kxp; g.kx = kxp; g.Bx = Ac; g.ldbx = K;
     }
     g.epi = EPI_F32; g.C = y32; g.ldc = K; g.R = R; g.ldr = K;

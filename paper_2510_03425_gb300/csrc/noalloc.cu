@@ -135,7 +135,7 @@ extern "C" int mebp_linear_fwd_noalloc(const uint16_t* X, int64_t M, const mebp_
     const int ro[1] = {0}, no[1] = {0};
     const int nl[1] = {static_cast<int>(N)};
     launch_lora_shadow(As, Bs, 1, ro, no, nl, r, static_cast<int>(K), static_cast<int>(N), kxp, Ac, Bc, Btc, st);
-    launch_skinny_gemm(X, K, M, K, Ac, K, r, s, U, kxp, st);
+    launch_skinny_gemm(X, K, M, K, Ac, K, r, s, U, kxp, st, err);
     g.Ax = U;
     g.ldax = kxp;
     g.kx = kxp;

@@ -123,7 +123,10 @@ def test_linear_dx_matches_exact_operand_product(ctx, Mr, N, K):
 
 @pytest.mark.parametrize("r,Mr,N,K", [(r, *shape) for r in (8, 16, 32)
                                       for shape in ((200, 320, 192), (300, 1152, 896), (2304 + 77, 576, 640))]
-                         + [(16, 4096 + 77, 1152, 1536)])  # > 152 tiles: persistent CTAs run several
+                         + [(16, 4096 + 77, 1152, 1536)]   # > 152 tiles: persistent CTAs run several
+                         # above 1024 tokens the rank-r products run on the tcgen05 kernel
+                         # (one rank block of 16 or 32 columns, K split over a cluster or not)
+                         + [(r, 2500, 640, 1024) for r in (8, 24, 32)] + [(32, 16384 + 5, 256, 2560)])
 def test_linear_with_lora_against_oracle(ctx, r, Mr, N, K):
     """Y = X deq(W)^T + s (X A^T) B^T (+R) and dX = dY deq(W) + s (dY B) A against fp64."""
     s = 2.0

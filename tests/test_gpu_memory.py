@@ -147,8 +147,9 @@ def test_step_allocates_nothing_and_fits_the_bound(min_memory):
     ws = M.mebp_workspace_bytes(ctx.handle)
     assert br["forward_sets"] + br["backward"] <= block_ws, (br["forward_sets"], br["backward"], block_ws)
     assert ws + weights + 8 * ls.n <= bound
-    # and the device agrees with the accounting: the context's own allocations are its workspace
-    # (plus allocator rounding), the weights and LoRA buffers torch's
+    # and the device agrees with the accounting: besides torch's tensors, the device memory taken
+    # since before the context is its workspace plus what the driver holds for the library's code
+    # (loaded on first launch), the captured graph and allocator rounding
     used_by_ctx = (free_before_ctx - free0) - (torch.cuda.memory_reserved() - reserved_before)
-    assert used_by_ctx <= ws + (64 << 20), (used_by_ctx, ws)
+    assert used_by_ctx <= ws + (256 << 20), (used_by_ctx, ws)
     ctx.close()
