@@ -703,6 +703,46 @@ def launch_list_step(args, d):
     ctx.close()
 
 
+def block_only(args, d):
+    """One decoder block of the workload (its dims and token count, one layer, no LM head):
+    warm-up, then one eager forward_i + backward_i through the public entry points inside the
+    NVTX range 'mebp_block'.  A few GB on the device at the Gemma3-4B shape, for full-set
+    profiler captures of single kernels at the workload's size."""
+    import torch
+
+    from paper_2510_03425_gb300 import mebp as M
+    from paper_2510_03425_gb300.model import Context, DeviceBlock, LoraSet
+    d1 = d.with_(n_layers=1, vocab=0)
+    device = torch.device("cuda", 0)
+    ctx = Context(d1, device=0)
+    W = synth.torch_block_weights(d1, 0, device=device)
+    blk = DeviceBlock(ctx, W)
+    del W
+    ls = LoraSet([synth.lora_weights(d1, 0)], device=device)
+    g = torch.Generator(device=device)
+    g.manual_seed(2)
+    x = torch.randn(d1.tokens, d1.hidden, device=device, generator=g)
+    dy = torch.randn(d1.tokens, d1.hidden, device=device, generator=g)
+    y, dx = torch.empty_like(x), torch.empty_like(x)
+    st = torch.cuda.Stream(device)
+    torch.cuda.set_stream(st)
+    bw = blk.struct()
+
+    def run():
+        M.mebp_block_recompute_fwd(ctx.handle, 0, bw, ls.layer(0), x, y, d1.batch, d1.seq, False, st)
+        M.mebp_block_bwd(ctx.handle, 0, bw, ls.layer(0), x, dy, dx, ls.layer_grads(0), d1.batch, d1.seq, False, st)
+    for _ in range(args.warmup):
+        run()
+    ctx.sync(st)
+    n0 = M.mebp_kernel_launches()
+    torch.cuda.nvtx.range_push("mebp_block")
+    run()
+    torch.cuda.nvtx.range_pop()
+    ctx.sync(st)
+    print(json.dumps({"block_only": workload_name(d1), "kernels": M.mebp_kernel_launches() - n0}), flush=True)
+    ctx.close()
+
+
 def gemm_bench(config: int, m_tokens=None, reps: int = 10, warmup: int = 3, shapes_only=None):
     """The fused dequant-GEMMs alone (forward Y = X deq(W)^T and transposed dX = dY deq(W)) at
     the four projection shapes of a workload, M = its token count.  Returns a dict."""
@@ -786,6 +826,9 @@ def main():
                     help="Fig. 2 analogue: per-phase time (CUDA events, NVTX emb / f_i / lm / b_i) and memory")
     ap.add_argument("--gemma3", action="store_true",
                     help="Gemma-shaped configs (2, 4) with the Gemma3 block options on")
+    ap.add_argument("--block-only", action="store_true",
+                    help="no timing: one decoder block of the workload (one layer, no LM head) run eagerly inside "
+                         "the NVTX range 'mebp_block' after the warm-up (for single-kernel profiler captures)")
     ap.add_argument("--launch-list", action="store_true",
                     help="no timing: after the warm-up run one eager step inside the NVTX range "
                          "'mebp_step' (for ncu --nvtx --nvtx-include mebp_step/)")
@@ -809,6 +852,9 @@ def main():
 
     if args.launch_list:
         launch_list_step(args, d)
+        return
+    if args.block_only:
+        block_only(args, d)
         return
     if args.table2:
         print(json.dumps(table2()), flush=True)

@@ -789,21 +789,38 @@ bool bwd_launch(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t l
 
 }  // namespace attn
 
-void launch_attn_fwd(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, int hd, uint16_t* o, int64_t ldo,
-                     float* lse, int window, cudaStream_t st) {
+// Grids of at least this many 128-query tiles run the tcgen05 kernels (attention_tc.cu); smaller
+// ones keep the warp-level kernels above, which split the keys of a query block over several
+// warp-groups or a CTA pair (measured: tcgen05 595 TFLOP/s at the Gemma3-4B shape, 36.1 -> 15.5 ms
+// per step; at 56 tiles, Qwen2.5-0.5B, 0.68 ms warp-level against 0.97 ms tcgen05).
+constexpr int64_t kTcMinTiles = 64;
+
+int launch_attn_fwd(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, int hd, uint16_t* o, int64_t ldo,
+                    float* lse, int window, int* err, cudaStream_t st) {
+  const int64_t tiles = static_cast<int64_t>((S + 127) / 128) * H * B;
+  if (tiles >= kTcMinTiles) return launch_attn_fwd_tc(qkv, ld, B, S, H, KV, hd, o, ldo, lse, window, err, st);
   const int W = window >= S ? 0 : window;  // a window covering the sequence is plain causal
   if (hd == 64) attn::fwd_launch<64>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
   else if (hd == 128) attn::fwd_launch<128>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
   else attn::fwd_launch<256>(qkv, ld, B, S, H, KV, o, ldo, lse, W, st);
+  return cudaGetLastError() == cudaSuccess ? MEBP_OK : MEBP_ERR_CUDA;
 }
 
 bool launch_attn_bwd(const uint16_t* qkv, int64_t ld, const uint16_t* o, const uint16_t* dout, int64_t ldo,
                      const float* lse, int B, int S, int H, int KV, int hd, float* dvec, uint16_t* dqkv, int window,
-                     const float2* rope_cs, float* ws, int64_t ws_floats, cudaStream_t st) {
+                     const float2* rope_cs, float* ws, int64_t ws_floats, int* err, cudaStream_t st) {
   const int W = window >= S ? 0 : window;
   const int64_t nw = static_cast<int64_t>(B) * S * H;
   launch_k(attn::dvec_kernel, static_cast<unsigned>((nw * 32 + 255) / 256), 256, 0, st, o, dout, ldo, B, S, H, hd,
            dvec);
+  // tcgen05 dK/dV and dQ when the dK/dV grid (128-key blocks x kv heads x sequences x column
+  // halves at hd 256) fills the GPU: Gemma3-4B shape 108 -> 51 ms per step; below that its CTAs
+  // each loop over too many query blocks, and the warp-level kernels split the work instead
+  const int64_t kv_tiles = static_cast<int64_t>((S + 127) / 128) * KV * B * (hd == 256 ? 2 : 1);
+  if (kv_tiles >= 152) {
+    launch_attn_bwd_tc(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, hd, dqkv, window, err, st);
+    return false;  // the caller applies the inverse RoPE
+  }
   if (hd == 64)
     return attn::bwd_launch<64, 64>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, rope_cs, ws, ws_floats, st);
   if (hd == 128)

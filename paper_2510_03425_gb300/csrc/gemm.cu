@@ -569,6 +569,23 @@ int make_tmap_2d(CUtensorMap* m, const void* base, CUtensorMapDataType dt, int e
   return r == CUDA_SUCCESS ? MEBP_OK : MEBP_ERR_INVALID_ARG;
 }
 
+int make_tmap_3d(CUtensorMap* m, const void* base, CUtensorMapDataType dt, int elem_bytes, uint64_t d0, uint64_t d1,
+                 uint64_t d2, uint64_t pitch1_bytes, uint64_t pitch2_bytes, uint32_t b0, uint32_t b1, uint32_t b2,
+                 CUtensorMapSwizzle swz) {
+  auto enc = get_encode();
+  if (!enc) return MEBP_ERR_CUDA;
+  if ((reinterpret_cast<uintptr_t>(base) & 15) || (pitch1_bytes & 15) || (pitch2_bytes & 15) ||
+      ((b0 * elem_bytes) & 15))
+    return MEBP_ERR_INVALID_ARG;
+  cuuint64_t dims[3] = {d0, d1, d2};
+  cuuint64_t strides[2] = {pitch1_bytes, pitch2_bytes};
+  cuuint32_t box[3] = {b0, b1, b2};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = enc(m, dt, 3, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? MEBP_OK : MEBP_ERR_INVALID_ARG;
+}
+
 int gemm_smem_bytes() { return gemm::Layout<1>::SMEM; }
 
 namespace {

@@ -610,7 +610,7 @@ int block_backward(mebp_ctx* c, int set, int bset, int layer, const mebp_block_w
        c->prof ? 2.5 * attn_fwd_flops(B, Sq, c->H, c->hd, win) : 0.0, st, [&] {
          rope_done = launch_attn_bwd(A.qkv, lq.N, A.o, c->dout, c->Na, A.lse_attn, B, Sq, c->H, c->KV, c->hd, c->dvec,
                                      G.dqkv, layer_window(c, layer), c->gemma ? nullptr : layer_rope(c, layer),
-                                     c->attn_ws, c->attn_ws_floats, st);
+                                     c->attn_ws, c->attn_ws_floats, c->d_err, st);
        });
   }
   if (c->gemma)

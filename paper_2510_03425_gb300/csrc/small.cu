@@ -89,36 +89,64 @@ void launch_rmsnorm_bwd(const float* dy, const float* x, const float* g, const f
 
 // ------------------------------------------------------------------------------------ RoPE
 // Half-split rotation: (x1, x2) -> (x1 c - x2 s, x2 c + x1 s) with (c, s) = table[pos][j];
-// inverse rotates by -angle (the VJP).  One thread per (token, head, pair of j).
+// inverse rotates by -angle (the VJP).  One thread per (token, group of 8 pairs j .. j+7, up to
+// four heads): the eight (c, s) pairs are read once and applied to every head of the thread, and
+// the eight x1 and eight x2 values of a head move as one 16-byte load / store each.
+constexpr int kRopeHeadsPerThread = 4;
 __global__ void rope_kernel(uint16_t* __restrict__ qkv, int64_t T, int S, int nheads, int ld, int hd,
                             const float2* __restrict__ cs, int inverse) {
   griddep_wait();
   griddep_launch();
-  const int half = hd >> 1, pairs = half >> 1;
+  const int half = hd >> 1, ng = half >> 3, nhc = (nheads + kRopeHeadsPerThread - 1) / kRopeHeadsPerThread;
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (i >= T * nheads * pairs) return;
-  const int jp = static_cast<int>(i % pairs);
-  const int64_t th = i / pairs;
-  const int head = static_cast<int>(th % nheads);
-  const int64_t t = th / nheads;
+  if (i >= T * ng * nhc) return;
+  const int g = static_cast<int>(i % ng);
+  const int64_t th = i / ng;
+  const int hc = static_cast<int>(th % nhc);
+  const int64_t t = th / nhc;
   const int pos = static_cast<int>(t % S);
-  uint16_t* base = qkv + t * ld + static_cast<int64_t>(head) * hd;
-  uint32_t* p1 = reinterpret_cast<uint32_t*>(base + 2 * jp);
-  uint32_t* p2 = reinterpret_cast<uint32_t*>(base + half + 2 * jp);
-  const uint32_t a = *p1, b = *p2;
-  const float2 c0 = cs[static_cast<int64_t>(pos) * half + 2 * jp];
-  const float2 c1 = cs[static_cast<int64_t>(pos) * half + 2 * jp + 1];
+  const float4* tab = reinterpret_cast<const float4*>(cs + static_cast<int64_t>(pos) * half + 8 * g);
   const float sg = inverse ? -1.0f : 1.0f;
-  const float x1a = h2_lo(a), x1b = h2_hi(a), x2a = h2_lo(b), x2b = h2_hi(b);
-  const float s0 = sg * c0.y, s1 = sg * c1.y;
-  *p1 = pack_half2(x1a * c0.x - x2a * s0, x1b * c1.x - x2b * s1);
-  *p2 = pack_half2(x2a * c0.x + x1a * s0, x2b * c1.x + x1b * s1);
+  float c[8], sn[8];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const float4 v = tab[k];
+    c[2 * k] = v.x;
+    sn[2 * k] = sg * v.y;
+    c[2 * k + 1] = v.z;
+    sn[2 * k + 1] = sg * v.w;
+  }
+  const int h0 = hc * kRopeHeadsPerThread, h1 = min(nheads, h0 + kRopeHeadsPerThread);
+  uint4 a[kRopeHeadsPerThread], b[kRopeHeadsPerThread];
+#pragma unroll
+  for (int k = 0; k < kRopeHeadsPerThread; ++k)
+    if (h0 + k < h1) {
+      const uint16_t* base = qkv + t * ld + static_cast<int64_t>(h0 + k) * hd + 8 * g;
+      a[k] = *reinterpret_cast<const uint4*>(base);
+      b[k] = *reinterpret_cast<const uint4*>(base + half);
+    }
+#pragma unroll
+  for (int k = 0; k < kRopeHeadsPerThread; ++k)
+    if (h0 + k < h1) {
+      const uint32_t x1[4] = {a[k].x, a[k].y, a[k].z, a[k].w}, x2[4] = {b[k].x, b[k].y, b[k].z, b[k].w};
+      uint32_t y1[4], y2[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float p0 = h2_lo(x1[q]), p1 = h2_hi(x1[q]), q0 = h2_lo(x2[q]), q1 = h2_hi(x2[q]);
+        const int j0 = 2 * q, j1 = 2 * q + 1;
+        y1[q] = pack_half2(p0 * c[j0] - q0 * sn[j0], p1 * c[j1] - q1 * sn[j1]);
+        y2[q] = pack_half2(q0 * c[j0] + p0 * sn[j0], q1 * c[j1] + p1 * sn[j1]);
+      }
+      uint16_t* base = qkv + t * ld + static_cast<int64_t>(h0 + k) * hd + 8 * g;
+      *reinterpret_cast<uint4*>(base) = make_uint4(y1[0], y1[1], y1[2], y1[3]);
+      *reinterpret_cast<uint4*>(base + half) = make_uint4(y2[0], y2[1], y2[2], y2[3]);
+    }
 }
 
 void launch_rope(uint16_t* qkv, int64_t T, int S, int H, int KV, int hd, const float2* cs, bool inverse,
                  cudaStream_t st) {
   const int nheads = H + KV;  // q heads then k heads
-  const int64_t n = T * nheads * (hd / 4);
+  const int64_t n = T * (hd / 16) * ((nheads + kRopeHeadsPerThread - 1) / kRopeHeadsPerThread);
   if (n <= 0) return;
   launch_k(rope_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, st, qkv, T, S, nheads, (H + 2 * KV) * hd, hd,
            cs, inverse ? 1 : 0);

@@ -94,6 +94,21 @@ def test_block_variants_match_oracle(kw):
     check(gpu, ref)
 
 
+@pytest.mark.parametrize("kw", [
+    # enough 128-row tiles for the tcgen05 attention kernels (forward and backward), ragged ends
+    dict(hidden=256, n_heads=8, n_kv_heads=8, head_dim=64, intermediate=256, act="silu", batch=10, seq=200,
+         rank=8, alpha=16.0, targets=("q", "k", "v", "o")),
+    dict(hidden=256, n_heads=8, n_kv_heads=4, head_dim=128, intermediate=256, act="gelu_tanh", batch=20, seq=250,
+         rank=16, alpha=32.0, targets=synth.TARGETS),
+    dict(hidden=512, n_heads=4, n_kv_heads=2, head_dim=256, intermediate=256, act="silu", batch=20, seq=140,
+         rank=8, alpha=16.0, targets=("q", "k", "v", "o")),
+])
+def test_block_on_tensor_core_attention_matches_oracle(kw):
+    dims = synth.tiny(n_layers=1, vocab=0, **kw)
+    gpu, ref, _ = run_block(dims, jitter=0.1)
+    check(gpu, ref)
+
+
 def test_lora_b_zero_block_equals_base_block_and_da_is_zero():
     dims = synth.preset(0)
     gpu, ref, (ctx, blk, ls, xg, Gg) = run_block(dims, zero_b=True)
