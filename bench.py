@@ -244,7 +244,7 @@ def gemm_traffic(config: int):
             txt = f.read()
     except OSError:
         return None, "no ncu summary"
-    kv = dict(re.findall(r"^([a-z_]+):\s*(\S+)\s*$", txt, flags=re.M))
+    kv = dict(re.findall(r"^([a-z0-9_]+):\s*(\S+)\s*$", txt, flags=re.M))
     if kv.get("workload_config") != str(config):
         return None, "ncu summary is for another workload"
     if kv.get("kernel_sources_sha256") != gemm_sources_sha():
