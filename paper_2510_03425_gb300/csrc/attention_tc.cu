@@ -53,7 +53,10 @@ struct Fwd {
   static constexpr uint32_t TM_O = 0, TM_S = 256;  // TMEM columns: O [0, HD), scores 256 + 128 b
 };
 
-template <int HD, bool WIN>
+// CL > 1 (grids under one wave): the key blocks of a query tile are dealt round-robin to the CL
+// CTAs of a cluster; each keeps its own (m, l, O) and the cluster merges them through
+// distributed shared memory, CTA c normalising and writing rows c*128/CL .. (c+1)*128/CL - 1.
+template <int HD, bool WIN, int CL>
 __global__ void __launch_bounds__(FWD_THREADS, 1)
     fwd_tc_kernel(const __grid_constant__ CUtensorMap tm, int S, int H, int KV, uint16_t* __restrict__ o, int64_t ldo,
                   float* __restrict__ lse, int W, int* err) {
@@ -76,13 +79,15 @@ __global__ void __launch_bounds__(FWD_THREADS, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int h = blockIdx.x, b = blockIdx.y;
+  const int h = static_cast<int>(blockIdx.x) / CL, crank = static_cast<int>(blockIdx.x) % CL, b = blockIdx.y;
   const int qb = static_cast<int>(gridDim.z) - 1 - static_cast<int>(blockIdx.z);  // longest rows first
   const int kvh = h / (H / KV);
   const int q0 = qb * BQ;
   const int kend = min(S, q0 + BQ);                          // keys below kend are seen by some row
   const int kb0 = WIN ? max(0, q0 - W + 1) / BKV : 0;        // first key block inside the window
-  const int nkb = (kend + BKV - 1) / BKV - kb0;
+  const int nkb_all = (kend + BKV - 1) / BKV - kb0;
+  const int nkb = (nkb_all - crank + CL - 1) / CL;           // this CTA's blocks: crank, crank + CL, ...
+  auto kblock = [&](int j) { return kb0 + crank + j * CL; };
 
   if (threadIdx.x == 0) {
     mbar_init(qfull, 1);
@@ -122,7 +127,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1)
         mbar_arrive_expect_tx(&kfull[s], C::KV_BYTES);
         for (int c = 0; c < C::NCH; ++c)
           tma_load_3d(sm + C::K_OFF + s * C::KV_BYTES + c * BKV * 128, &tm, &kfull[s], (H + kvh) * HD + c * 64,
-                      (kb0 + j) * BKV, b);
+                      kblock(j) * BKV, b);
         issued = j + 1;
       }
       int dummy = 0;  // never leave with copies in flight
@@ -140,7 +145,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1)
         mbar_arrive_expect_tx(&vfull[s], C::KV_BYTES);
         for (int c = 0; c < C::NCH; ++c)
           tma_load_3d(sm + C::V_OFF + s * C::KV_BYTES + c * BKV * 128, &tm, &vfull[s],
-                      (H + KV + kvh) * HD + c * 64, (kb0 + j) * BKV, b);
+                      (H + KV + kvh) * HD + c * 64, kblock(j) * BKV, b);
         issued = j + 1;
       }
       int dummy = 0;
@@ -203,7 +208,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1)
       if (!ok) break;
       tc_fence_after();
       // pass 1: the row max of this block (scores scaled to log2 units, masked)
-      const int k0 = (kb0 + j) * BKV;
+      const int k0 = kblock(j) * BKV;
       const uint32_t ts = tmem + lane_off + C::TM_S + (j & 1) * BKV;
       auto masked = [&](float (&t)[32], int c) {
 #pragma unroll
@@ -281,7 +286,23 @@ __global__ void __launch_bounds__(FWD_THREADS, 1)
     }
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(ofull, 0, abort_flag, err));
     tc_fence_after();
-    if (ok) {
+    if (CL > 1) {
+      // park the unnormalised row of O and (m, l) in this CTA's shared memory (every load and
+      // MMA of the CTA has completed, so the tiles are free); a CTA without key blocks parks zeros
+      float* po = reinterpret_cast<float*>(sm) + r * (HD + 4);
+#pragma unroll 1
+      for (int c = 0; c < HD / 32; ++c) {
+        float t[32];
+        tmem_ld32(tmem + lane_off + C::TM_O + 32 * c, t);
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          *reinterpret_cast<float4*>(po + 32 * c + 4 * i) =
+              (ok && nkb > 0) ? make_float4(t[4 * i], t[4 * i + 1], t[4 * i + 2], t[4 * i + 3])
+                              : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+      }
+      reinterpret_cast<float4*>(sm + BQ * (HD + 4) * 4)[r] =
+          make_float4((ok && nkb > 0) ? m_used : -INFINITY, (ok && nkb > 0) ? l : 0.0f, 0.0f, 0.0f);
+    } else if (ok) {
       const float inv = l > 0.0f ? 1.0f / l : 0.0f;
       const int64_t tok = static_cast<int64_t>(b) * S + row;
 #pragma unroll 1
@@ -313,29 +334,79 @@ __global__ void __launch_bounds__(FWD_THREADS, 1)
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
+  if constexpr (CL > 1) {
+    // every thread of every CTA of the cluster passes both barriers (no wait above is unbounded)
+    cluster_sync_all();
+    constexpr int RPC = BQ / CL, C4 = HD / 4;
+    const uint32_t o_base = smem_u32(sm), ml_base = smem_u32(sm + BQ * (HD + 4) * 4);
+    for (int e = threadIdx.x; e < RPC * C4; e += FWD_THREADS) {
+      const int rl = crank * RPC + e / C4, cc = (e % C4) * 4, row = q0 + rl;
+      float mj[CL], lj[CL];
+      float Mx = -INFINITY;
+#pragma unroll
+      for (int j = 0; j < CL; ++j) {
+        const float4 v = ld_dsmem_f4(dsmem_addr(ml_base + rl * 16, j));
+        mj[j] = v.x;
+        lj[j] = v.y;
+        Mx = fmaxf(Mx, v.x);
+      }
+      float L = 0.0f;
+      float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll
+      for (int j = 0; j < CL; ++j) {
+        if (mj[j] == -INFINITY) continue;
+        const float w = exp2f(mj[j] - Mx);
+        L += w * lj[j];
+        const float4 q = ld_dsmem_f4(dsmem_addr(o_base + (rl * (HD + 4) + cc) * 4, j));
+        acc.x += w * q.x; acc.y += w * q.y; acc.z += w * q.z; acc.w += w * q.w;
+      }
+      if (row < S) {
+        const float inv = L > 0.0f ? 1.0f / L : 0.0f;
+        *reinterpret_cast<uint2*>(o + (static_cast<int64_t>(b) * S + row) * ldo + h * HD + cc) =
+            make_uint2(pack_half2(acc.x * inv, acc.y * inv), pack_half2(acc.z * inv, acc.w * inv));
+        if (cc == 0) lse[(static_cast<int64_t>(b) * H + h) * S + row] = (Mx + log2f(L)) / kLog2e;
+      }
+    }
+    cluster_sync_all();  // no CTA leaves while its partials are being read
+  }
 }
 
-template <int HD, bool WIN>
-int fwd_launch(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uint16_t* o, int64_t ldo, float* lse,
-               int W, int* err, cudaStream_t st) {
+template <int HD, bool WIN, int CL>
+int fwd_launch_cl(const CUtensorMap& tm, int B, int S, int H, int KV, uint16_t* o, int64_t ldo, float* lse, int W,
+                  int* err, cudaStream_t st) {
   using C = Fwd<HD>;
+  static_assert(BQ * (HD + 4) * 4 + BQ * 16 <= C::BAR_OFF, "parked O and (m, l) fit below the barriers");
   static bool attr = false;
   if (!attr) {
-    if (cudaFuncSetAttribute(fwd_tc_kernel<HD, WIN>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM) !=
+    if (cudaFuncSetAttribute(fwd_tc_kernel<HD, WIN, CL>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM) !=
         cudaSuccess) {
       cudaGetLastError();
       return MEBP_ERR_CUDA;
     }
     attr = true;
   }
+  const dim3 grid(H * CL, B, (S + BQ - 1) / BQ);
+  if (CL == 1) launch_k(fwd_tc_kernel<HD, WIN, CL>, grid, FWD_THREADS, C::SMEM, st, tm, S, H, KV, o, ldo, lse, W, err);
+  else
+    launch_k_cluster(fwd_tc_kernel<HD, WIN, CL>, grid, FWD_THREADS, C::SMEM, st, dim3(CL, 1, 1), tm, S, H, KV, o, ldo,
+                     lse, W, err);
+  return cudaGetLastError() == cudaSuccess ? MEBP_OK : MEBP_ERR_CUDA;
+}
+
+template <int HD, bool WIN>
+int fwd_launch(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uint16_t* o, int64_t ldo, float* lse,
+               int W, int* err, cudaStream_t st) {
   CUtensorMap tm;
   // {columns of the fused projection buffer, positions, sequences}, 64 x 128 x 1 boxes
   int rc = make_tmap_3d(&tm, qkv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, ld, S, B, ld * 2, static_cast<uint64_t>(S) * ld * 2,
                         64, BQ, 1, CU_TENSOR_MAP_SWIZZLE_128B);
   if (rc) return rc;
-  const dim3 grid(H, B, (S + BQ - 1) / BQ);
-  launch_k(fwd_tc_kernel<HD, WIN>, grid, FWD_THREADS, C::SMEM, st, tm, S, H, KV, o, ldo, lse, W, err);
-  return cudaGetLastError() == cudaSuccess ? MEBP_OK : MEBP_ERR_CUDA;
+  // grids under one wave share each query tile's key blocks among a cluster of 2 or 4 CTAs
+  const int64_t tiles = static_cast<int64_t>((S + BQ - 1) / BQ) * H * B;
+  const int nkb_max = (S + BKV - 1) / BKV;
+  if (tiles * 4 <= 152 && nkb_max >= 4) return fwd_launch_cl<HD, WIN, 4>(tm, B, S, H, KV, o, ldo, lse, W, err, st);
+  if (tiles * 2 <= 152 && nkb_max >= 2) return fwd_launch_cl<HD, WIN, 2>(tm, B, S, H, KV, o, ldo, lse, W, err, st);
+  return fwd_launch_cl<HD, WIN, 1>(tm, B, S, H, KV, o, ldo, lse, W, err, st);
 }
 
 // ================================================================================== backward
@@ -356,6 +427,16 @@ int fwd_launch(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uin
 constexpr int BWD_THREADS = 192;  // warps 0-3 elementwise + epilogue, 4 TMA, 5 MMA
 constexpr int BQB = 64;           // queries per dK/dV iteration, keys per dQ iteration
 
+// Split mode (grids under one wave): a dK/dV item is one (128 keys, query head, part) and takes
+// every P-th query block of that head; a dQ item is one (128 queries, head, part) and takes every
+// P-th key block.  Items write fp32 partials (dK and dQ already times 1/sqrt(hd)) into slots of
+// [64 rows][hd] floats indexed ((b * nb64 + 64-row block) * H + query head) * P + part, which the
+// finish kernel sums over parts and the query heads of a group.  P == 0: direct mode.
+struct SplitOut {
+  int P;
+  float *wk, *wv, *wq;
+};
+
 template <int HD>
 struct DkDv {
   static constexpr int DC = HD == 256 ? 128 : HD;  // output columns per CTA
@@ -375,11 +456,13 @@ struct DkDv {
   static constexpr uint32_t TM_DK = 0, TM_DV = DC, TM_S = 256;  // S^T / dP^T buffer b: 256 + 128 b (+64)
 };
 
+// One dK/dV item: item = (((kb * B + b) * heads + head) * NCOL + col) * P + part, heads = KV (direct,
+// P = 1) or H (split).
 template <int HD, bool WIN>
-__global__ void __launch_bounds__(BWD_THREADS, 1)
-    dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmKV, const __grid_constant__ CUtensorMap tmQ,
-                   const __grid_constant__ CUtensorMap tmDO, int S, int H, int KV, const float* __restrict__ lse,
-                   const float* __restrict__ dvec, uint16_t* __restrict__ dqkv, int64_t ld, int W, int* err) {
+__device__ __forceinline__ void dkdv_body(const CUtensorMap& tmKV, const CUtensorMap& tmQ, const CUtensorMap& tmDO,
+                                          int S, int H, int KV, const float* __restrict__ lse,
+                                          const float* __restrict__ dvec, uint16_t* __restrict__ dqkv, int64_t ld,
+                                          int W, int* err, const SplitOut& so, int item, int B) {
   using C = DkDv<HD>;
   constexpr int NS = C::NS, NPB = C::NPB, DC = C::DC;
   static_assert(C::SMEM <= 232448, "shared memory");
@@ -400,22 +483,31 @@ __global__ void __launch_bounds__(BWD_THREADS, 1)
   float* vec = reinterpret_cast<float*>(sm + C::VEC_OFF);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // blockIdx.x = ((kb * B + b) * KV + kvh) * NCOL + col, key block slowest and first (longest)
-  int t = blockIdx.x;
+  // direct: blockIdx.x = ((kb * B + b) * KV + kvh) * NCOL + col; split: (((kb * B + b) * H + h) * NCOL +
+  // col) * P + p; key block slowest and first (the longest items)
+  const bool split = so.P > 0;
+  const int P = split ? so.P : 1;
+  const int heads = split ? H : KV;
+  int t = item;
+  const int part = t % P;
+  t /= P;
   const int col = t % C::NCOL;
   t /= C::NCOL;
-  const int kvh = t % KV;
-  t /= KV;
-  const int B = static_cast<int>(gridDim.x) / (C::NCOL * KV * ((S + BKV - 1) / BKV));
+  const int hsel = t % heads;
+  t /= heads;
   const int b = t % B, kb = t / B;
+  const int grp = H / KV;
+  const int kvh = split ? hsel / grp : hsel;
+  const int h_first = split ? hsel : kvh * grp;
   const int c0 = col * DC;
   const int k0 = kb * BKV;
-  const int grp = H / KV, h_first = kvh * grp;
   const int nqb = (S + BQB - 1) / BQB;
   const int qb_first = k0 / BQB;
   const int qb_end = WIN ? min(nqb, (k0 + BKV - 1 + W - 1) / BQB + 1) : nqb;
   const int per_head = qb_end - qb_first;
-  const int n_it = grp * per_head;
+  const int n_all = split ? per_head : grp * per_head;
+  const int n_it = part < n_all ? (n_all - part + P - 1) / P : 0;
+  auto g_of = [&](int j) { return part + j * P; };  // iteration j covers (head, query block) number g
 
   if (threadIdx.x == 0) {
     mbar_init(kvfull, 1);
@@ -458,7 +550,7 @@ __global__ void __launch_bounds__(BWD_THREADS, 1)
       for (int it = 0; it < n_it; ++it) {
         const int s = it % NS;
         if (it >= NS && !mbar_wait(&qempty[s], ((it / NS) & 1) ^ 1, abort_flag, err)) break;
-        const int hh = h_first + it / per_head, q0 = (qb_first + it % per_head) * BQB;
+        const int g = g_of(it), hh = h_first + g / per_head, q0 = (qb_first + g % per_head) * BQB;
         uint8_t* qs = sm + C::Q_OFF + s * 2 * C::Q_BYTES;
         mbar_arrive_expect_tx(&qfull[s], 2 * C::Q_BYTES);
         for (int c = 0; c < C::NCH; ++c) {
@@ -531,15 +623,20 @@ __global__ void __launch_bounds__(BWD_THREADS, 1)
     const int r = threadIdx.x, kr = k0 + r;
     const uint32_t lane_off = static_cast<uint32_t>(32 * warp) << 16;
     const float sc = kLog2e * rsqrtf(static_cast<float>(HD));
+    // thread r < 64 carries lse * log2e of query q0 + r, thread r >= 64 D of query q0 + r - 64;
+    // the value of iteration j + 1 is loaded while iteration j runs
+    auto vec_load = [&](int j) -> float {
+      const int g = g_of(j), hh = h_first + g / per_head, q = (qb_first + g % per_head) * BQB + (r & 63);
+      const int64_t li = (static_cast<int64_t>(b) * H + hh) * S + q;
+      return q < S ? (r < 64 ? lse[li] * kLog2e : dvec[li]) : 0.0f;
+    };
+    float vnext = n_it > 0 ? vec_load(0) : 0.0f;
     bool ok = true;
     for (int j = 0; j < n_it; ++j) {
-      const int hh = h_first + j / per_head, q0 = (qb_first + j % per_head) * BQB;
+      const int q0 = (qb_first + g_of(j) % per_head) * BQB;
       float* lv = vec + (j & 1) * 2 * BQB;  // [64] lse * log2e, then [64] D
-      {
-        const int qi = r & 63, q = q0 + qi;
-        const int64_t li = (static_cast<int64_t>(b) * H + hh) * S + q;
-        lv[r] = q < S ? (r < 64 ? lse[li] * kLog2e : dvec[li]) : 0.0f;
-      }
+      lv[r] = vnext;
+      if (j + 1 < n_it) vnext = vec_load(j + 1);
       // every thread of the four warps has written its entry (and, by the same token, finished
       // reading this buffer two iterations ago): a bounded mbarrier, never a named barrier, so an
       // aborting warp cannot leave the others waiting
@@ -556,22 +653,23 @@ __global__ void __launch_bounds__(BWD_THREADS, 1)
       tc_fence_after();
       const uint32_t ts = tmem + lane_off + C::TM_S + 128 * (j & 1);
       uint8_t* prow = sm + C::P_OFF + (j % NPB) * 2 * C::P_BYTES + r * 128;
-#pragma unroll 1
-      for (int c = 0; c < BQB / 32; ++c) {
-        float sv[32], dp[32];
-        tmem_ld32(ts + 32 * c, sv);
-        tmem_ld32(ts + 64 + 32 * c, dp);
+      {
+        static_assert(BQB == 64, "one 64-column TMEM load per score row");
+        constexpr int c = 0;
+        float sv[64], dp[64];
+        tmem_ld64(ts, sv);
+        tmem_ld64(ts + 64, dp);
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          const int qi = 32 * c + e, q = q0 + qi;
+        for (int e = 0; e < 64; ++e) {
+          const int qi = e, q = q0 + qi;
           const bool vis = kr <= q && q < S && kr < S && (!WIN || q - kr < W);
           const float pv = vis ? exp2f(sv[e] * sc - lv[qi]) : 0.0f;
           sv[e] = pv;
           dp[e] = pv * (dp[e] - lv[BQB + qi]);
         }
 #pragma unroll
-        for (int qd = 0; qd < 4; ++qd) {  // 8 queries per 16-byte unit
-          const int w = 4 * c + qd, off = (w ^ (r & 7)) << 4;
+        for (int qd = 0; qd < 8; ++qd) {  // 8 queries per 16-byte unit
+          const int w = 8 * c + qd, off = (w ^ (r & 7)) << 4;
           *reinterpret_cast<uint4*>(prow + off) =
               make_uint4(pack_half2(sv[8 * qd], sv[8 * qd + 1]), pack_half2(sv[8 * qd + 2], sv[8 * qd + 3]),
                          pack_half2(sv[8 * qd + 4], sv[8 * qd + 5]), pack_half2(sv[8 * qd + 6], sv[8 * qd + 7]));
@@ -590,7 +688,32 @@ __global__ void __launch_bounds__(BWD_THREADS, 1)
     }
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(dfull, 0, abort_flag, err));
     tc_fence_after();
-    if (ok) {
+    if (ok && split) {
+      // fp32 partials of this (head, part); an item without query blocks writes zeros
+      const float inv = rsqrtf(static_cast<float>(HD));
+      const int nb64 = (S + 63) / 64;
+      const int64_t slot = ((static_cast<int64_t>(b) * nb64 + 2 * kb + r / 64) * H + hsel) * P + part;
+      float* pk = so.wk + slot * (64 * HD) + (r % 64) * HD + c0;
+      float* pv = so.wv + slot * (64 * HD) + (r % 64) * HD + c0;
+#pragma unroll 1
+      for (int c = 0; c < DC / 32; ++c) {
+        float dk[32], dv[32];
+        tmem_ld32(tmem + lane_off + C::TM_DK + 32 * c, dk);
+        tmem_ld32(tmem + lane_off + C::TM_DV + 32 * c, dv);
+        if (kr < S) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const bool z = n_it == 0;
+            __stcg(reinterpret_cast<float4*>(pk + 32 * c + 4 * i),
+                   z ? make_float4(0.0f, 0.0f, 0.0f, 0.0f)
+                     : make_float4(dk[4 * i] * inv, dk[4 * i + 1] * inv, dk[4 * i + 2] * inv, dk[4 * i + 3] * inv));
+            __stcg(reinterpret_cast<float4*>(pv + 32 * c + 4 * i),
+                   z ? make_float4(0.0f, 0.0f, 0.0f, 0.0f)
+                     : make_float4(dv[4 * i], dv[4 * i + 1], dv[4 * i + 2], dv[4 * i + 3]));
+          }
+        }
+      }
+    } else if (ok) {
       const float inv = rsqrtf(static_cast<float>(HD));
       const int64_t tok = static_cast<int64_t>(b) * S + kr;
       // every key block below S is seen by at least its own query block, so n_it >= 1
@@ -645,11 +768,12 @@ struct Dq {
   static constexpr uint32_t TM_DQ = 0, TM_S = 256;  // S / dP buffer b: 256 + 128 b (+64)
 };
 
+// One dQ item: x = head * P + part, sequence b, query tile nqb - 1 - z (the longest first).
 template <int HD, bool WIN>
-__global__ void __launch_bounds__(BWD_THREADS, 1)
-    dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKV,
-                 const __grid_constant__ CUtensorMap tmDO, int S, int H, int KV, const float* __restrict__ lse,
-                 const float* __restrict__ dvec, uint16_t* __restrict__ dqkv, int64_t ld, int W, int* err) {
+__device__ __forceinline__ void dq_body(const CUtensorMap& tmQ, const CUtensorMap& tmKV, const CUtensorMap& tmDO,
+                                        int S, int H, int KV, const float* __restrict__ lse,
+                                        const float* __restrict__ dvec, uint16_t* __restrict__ dqkv, int64_t ld,
+                                        int W, int* err, const SplitOut& so, int x, int b, int z) {
   using C = Dq<HD>;
   constexpr int NS = C::NS, NPB = C::NPB;
   static_assert(C::SMEM <= 232448, "shared memory");
@@ -668,13 +792,17 @@ __global__ void __launch_bounds__(BWD_THREADS, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int h = blockIdx.x, b = blockIdx.y;
-  const int qb = static_cast<int>(gridDim.z) - 1 - static_cast<int>(blockIdx.z);  // longest rows first
+  const bool split = so.P > 0;
+  const int P = split ? so.P : 1;
+  const int h = x / P, part = x % P;
+  const int qb = (S + BQ - 1) / BQ - 1 - z;  // longest rows first
   const int kvh = h / (H / KV);
   const int q0 = qb * BQ;
   const int kend = min(S, q0 + BQ);
   const int kb0 = WIN ? max(0, q0 - W + 1) / BQB : 0;
-  const int nkb = (kend + BQB - 1) / BQB - kb0;
+  const int nkb_all = (kend + BQB - 1) / BQB - kb0;
+  const int nkb = part < nkb_all ? (nkb_all - part + P - 1) / P : 0;  // key blocks part, part + P, ...
+  auto kblock = [&](int j) { return kb0 + part + j * P; };
 
   if (threadIdx.x == 0) {
     mbar_init(qfull, 1);
@@ -719,9 +847,9 @@ __global__ void __launch_bounds__(BWD_THREADS, 1)
         uint8_t* ks = sm + C::K_OFF + s * 2 * C::K_BYTES;
         mbar_arrive_expect_tx(&kfull[s], 2 * C::K_BYTES);
         for (int c = 0; c < C::NCH; ++c) {
-          tma_load_3d(ks + c * BQB * 128, &tmKV, &kfull[s], (H + kvh) * HD + c * 64, (kb0 + j) * BQB, b);
+          tma_load_3d(ks + c * BQB * 128, &tmKV, &kfull[s], (H + kvh) * HD + c * 64, kblock(j) * BQB, b);
           tma_load_3d(ks + C::K_BYTES + c * BQB * 128, &tmKV, &kfull[s], (H + KV + kvh) * HD + c * 64,
-                      (kb0 + j) * BQB, b);
+                      kblock(j) * BQB, b);
         }
         issued = j + 1;
       }
@@ -799,22 +927,22 @@ __global__ void __launch_bounds__(BWD_THREADS, 1)
       tc_fence_after();
       const uint32_t ts = tmem + lane_off + C::TM_S + 128 * (j & 1);
       uint8_t* drow = sm + C::P_OFF + (j % NPB) * C::P_BYTES + r * 128;
-      const int k0 = (kb0 + j) * BQB;
-#pragma unroll 1
-      for (int c = 0; c < BQB / 32; ++c) {
-        float sv[32], dp[32];
-        tmem_ld32(ts + 32 * c, sv);
-        tmem_ld32(ts + 64 + 32 * c, dp);
+      const int k0 = kblock(j) * BQB;
+      {
+        constexpr int c = 0;
+        float sv[64], dp[64];
+        tmem_ld64(ts, sv);
+        tmem_ld64(ts + 64, dp);
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          const int key = k0 + 32 * c + e;
+        for (int e = 0; e < 64; ++e) {
+          const int key = k0 + e;
           const bool vis = key <= row && row < S && (!WIN || row - key < W);
           const float pv = vis ? exp2f(sv[e] * sc - l2) : 0.0f;
           dp[e] = pv * (dp[e] - dr);
         }
 #pragma unroll
-        for (int kd = 0; kd < 4; ++kd) {
-          const int w = 4 * c + kd;
+        for (int kd = 0; kd < 8; ++kd) {
+          const int w = 8 * c + kd;
           *reinterpret_cast<uint4*>(drow + ((w ^ (r & 7)) << 4)) =
               make_uint4(pack_half2(dp[8 * kd], dp[8 * kd + 1]), pack_half2(dp[8 * kd + 2], dp[8 * kd + 3]),
                          pack_half2(dp[8 * kd + 4], dp[8 * kd + 5]), pack_half2(dp[8 * kd + 6], dp[8 * kd + 7]));
@@ -830,7 +958,24 @@ __global__ void __launch_bounds__(BWD_THREADS, 1)
     }
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(dfull, 0, abort_flag, err));
     tc_fence_after();
-    if (ok) {
+    if (ok && split) {
+      const float inv = rsqrtf(static_cast<float>(HD));
+      const int nb64 = (S + 63) / 64;
+      const int64_t slot = ((static_cast<int64_t>(b) * nb64 + 2 * qb + r / 64) * H + h) * P + part;
+      float* pq = so.wq + slot * (64 * HD) + (r % 64) * HD;
+#pragma unroll 1
+      for (int c = 0; c < HD / 32; ++c) {
+        float t[32];
+        tmem_ld32(tmem + lane_off + C::TM_DQ + 32 * c, t);
+        if (row < S) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            __stcg(reinterpret_cast<float4*>(pq + 32 * c + 4 * i),
+                   nkb == 0 ? make_float4(0.0f, 0.0f, 0.0f, 0.0f)
+                            : make_float4(t[4 * i] * inv, t[4 * i + 1] * inv, t[4 * i + 2] * inv, t[4 * i + 3] * inv));
+        }
+      }
+    } else if (ok) {
       const float inv = rsqrtf(static_cast<float>(HD));
       const int64_t tok = static_cast<int64_t>(b) * S + row;
 #pragma unroll 1
@@ -864,14 +1009,55 @@ __global__ void __launch_bounds__(BWD_THREADS, 1)
 }
 
 template <int HD, bool WIN>
+__global__ void __launch_bounds__(BWD_THREADS, 1)
+    dkdv_tc_kernel(const __grid_constant__ CUtensorMap tmKV, const __grid_constant__ CUtensorMap tmQ,
+                   const __grid_constant__ CUtensorMap tmDO, int S, int H, int KV, const float* __restrict__ lse,
+                   const float* __restrict__ dvec, uint16_t* __restrict__ dqkv, int64_t ld, int W, int* err,
+                   const SplitOut so, int B) {
+  dkdv_body<HD, WIN>(tmKV, tmQ, tmDO, S, H, KV, lse, dvec, dqkv, ld, W, err, so, blockIdx.x, B);
+}
+
+template <int HD, bool WIN>
+__global__ void __launch_bounds__(BWD_THREADS, 1)
+    dq_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKV,
+                 const __grid_constant__ CUtensorMap tmDO, int S, int H, int KV, const float* __restrict__ lse,
+                 const float* __restrict__ dvec, uint16_t* __restrict__ dqkv, int64_t ld, int W, int* err,
+                 const SplitOut so) {
+  dq_body<HD, WIN>(tmQ, tmKV, tmDO, S, H, KV, lse, dvec, dqkv, ld, W, err, so, blockIdx.x, blockIdx.y, blockIdx.z);
+}
+
+// Split mode as one launch: group L holds the dK/dV items of key tile L and the dQ items of query
+// tile nqb - 1 - L (both see nqb - L tiles of the other kind), groups in order, so the longest
+// items of both kinds start first and the two kinds run side by side.
+template <int HD, bool WIN>
+__global__ void __launch_bounds__(BWD_THREADS, 1)
+    bwd_split_tc_kernel(const __grid_constant__ CUtensorMap kv128, const __grid_constant__ CUtensorMap q64,
+                        const __grid_constant__ CUtensorMap do64, const __grid_constant__ CUtensorMap q128,
+                        const __grid_constant__ CUtensorMap kv64, const __grid_constant__ CUtensorMap do128, int S,
+                        int H, int KV, const float* __restrict__ lse, const float* __restrict__ dvec,
+                        uint16_t* __restrict__ dqkv, int64_t ld, int W, int* err, const SplitOut so, int B) {
+  const int nd = B * H * DkDv<HD>::NCOL * so.P, nq = H * so.P * B;
+  const int L = static_cast<int>(blockIdx.x) / (nd + nq), r = static_cast<int>(blockIdx.x) % (nd + nq);
+  if (r < nd)
+    dkdv_body<HD, WIN>(kv128, q64, do64, S, H, KV, lse, dvec, dqkv, ld, W, err, so, L * nd + r, B);
+  else
+    dq_body<HD, WIN>(q128, kv64, do128, S, H, KV, lse, dvec, dqkv, ld, W, err, so, (r - nd) % (H * so.P),
+                     (r - nd) / (H * so.P), L);
+}
+
+template <int HD, bool WIN>
 int bwd_launch(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t ldo, const float* lse,
-               const float* dvec, int B, int S, int H, int KV, int W, uint16_t* dqkv, int* err, cudaStream_t st) {
+               const float* dvec, int B, int S, int H, int KV, int W, uint16_t* dqkv, int* err, const SplitOut& so,
+               cudaStream_t st) {
+  constexpr int SPLIT_SMEM = DkDv<HD>::SMEM > Dq<HD>::SMEM ? DkDv<HD>::SMEM : Dq<HD>::SMEM;
   static bool attr = false;
   if (!attr) {
     if (cudaFuncSetAttribute(dkdv_tc_kernel<HD, WIN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              DkDv<HD>::SMEM) != cudaSuccess ||
         cudaFuncSetAttribute(dq_tc_kernel<HD, WIN>, cudaFuncAttributeMaxDynamicSharedMemorySize, Dq<HD>::SMEM) !=
-            cudaSuccess) {
+            cudaSuccess ||
+        cudaFuncSetAttribute(bwd_split_tc_kernel<HD, WIN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             SPLIT_SMEM) != cudaSuccess) {
       cudaGetLastError();
       return MEBP_ERR_CUDA;
     }
@@ -894,10 +1080,17 @@ int bwd_launch(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t ld
                          CU_TENSOR_MAP_SWIZZLE_128B)))
     return rc;
   const int nkb = (S + BKV - 1) / BKV;
-  launch_k(dkdv_tc_kernel<HD, WIN>, dim3(static_cast<unsigned>(nkb * B * KV * DkDv<HD>::NCOL)), BWD_THREADS,
-           DkDv<HD>::SMEM, st, kv128, q64, do64, S, H, KV, lse, dvec, dqkv, ld, W, err);
-  launch_k(dq_tc_kernel<HD, WIN>, dim3(H, B, (S + BQ - 1) / BQ), BWD_THREADS, Dq<HD>::SMEM, st, q128, kv64, do128, S,
-           H, KV, lse, dvec, dqkv, ld, W, err);
+  if (so.P > 0) {  // 128-key and 128-query tiles pair up group by group (nkb of each)
+    const int64_t n = static_cast<int64_t>(nkb) * (B * H * DkDv<HD>::NCOL * so.P + H * so.P * B);
+    launch_k(bwd_split_tc_kernel<HD, WIN>, dim3(static_cast<unsigned>(n)), BWD_THREADS, SPLIT_SMEM, st, kv128, q64,
+             do64, q128, kv64, do128, S, H, KV, lse, dvec, dqkv, ld, W, err, so, B);
+  } else {
+    const int64_t n_dkdv = static_cast<int64_t>(nkb) * B * KV * DkDv<HD>::NCOL;
+    launch_k(dkdv_tc_kernel<HD, WIN>, dim3(static_cast<unsigned>(n_dkdv)), BWD_THREADS, DkDv<HD>::SMEM, st, kv128,
+             q64, do64, S, H, KV, lse, dvec, dqkv, ld, W, err, so, B);
+    launch_k(dq_tc_kernel<HD, WIN>, dim3(H, B, (S + BQ - 1) / BQ), BWD_THREADS, Dq<HD>::SMEM, st, q128, kv64, do128,
+             S, H, KV, lse, dvec, dqkv, ld, W, err, so);
+  }
   return cudaGetLastError() == cudaSuccess ? MEBP_OK : MEBP_ERR_CUDA;
 }
 
@@ -922,17 +1115,18 @@ int launch_attn_fwd_tc(const uint16_t* qkv, int64_t ld, int B, int S, int H, int
 
 namespace mebp {
 int launch_attn_bwd_tc(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t ldo, const float* lse,
-                       const float* dvec, int B, int S, int H, int KV, int hd, uint16_t* dqkv, int window, int* err,
-                       cudaStream_t st) {
+                       const float* dvec, int B, int S, int H, int KV, int hd, uint16_t* dqkv, int window, int parts,
+                       float* wk, float* wv, float* wq, int* err, cudaStream_t st) {
   const int W = window >= S ? 0 : window;
   if (ld % 64 || ldo % 64) return MEBP_ERR_INVALID_ARG;
+  const atc::SplitOut so{parts, wk, wv, wq};
   switch (hd) {
-    case 64: return W ? atc::bwd_launch<64, true>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, err, st)
-                      : atc::bwd_launch<64, false>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, 0, dqkv, err, st);
-    case 128: return W ? atc::bwd_launch<128, true>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, err, st)
-                       : atc::bwd_launch<128, false>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, 0, dqkv, err, st);
-    case 256: return W ? atc::bwd_launch<256, true>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, err, st)
-                       : atc::bwd_launch<256, false>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, 0, dqkv, err, st);
+    case 64: return W ? atc::bwd_launch<64, true>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, err, so, st)
+                      : atc::bwd_launch<64, false>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, 0, dqkv, err, so, st);
+    case 128: return W ? atc::bwd_launch<128, true>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, err, so, st)
+                       : atc::bwd_launch<128, false>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, 0, dqkv, err, so, st);
+    case 256: return W ? atc::bwd_launch<256, true>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, W, dqkv, err, so, st)
+                       : atc::bwd_launch<256, false>(qkv, ld, dout, ldo, lse, dvec, B, S, H, KV, 0, dqkv, err, so, st);
     default: return MEBP_ERR_UNSUPPORTED;
   }
 }

@@ -232,9 +232,11 @@ void launch_adamw(float* p, const float* g, float* m, float* v, int64_t n, float
 bool launch_attn_bwd(const uint16_t* qkv, int64_t ld, const uint16_t* o, const uint16_t* dout, int64_t ldo,
                      const float* lse, int B, int S, int H, int KV, int hd, float* dvec, uint16_t* dqkv, int window,
                      const float2* rope_cs, float* ws, int64_t ws_floats, int* err, cudaStream_t st);
-// dK/dV and dQ on tcgen05 (attention_tc.cu) from dvec = rowsum(dO o); writes dqkv (no RoPE inverse).
+// dK/dV and dQ on tcgen05 (attention_tc.cu) from dvec = rowsum(dO o).  parts == 0: writes dqkv
+// (no RoPE inverse); parts = P > 0: fp32 partials into wk / wv / wq (see attention.cu) for the
+// finish kernel.
 int launch_attn_bwd_tc(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t ldo, const float* lse,
-                       const float* dvec, int B, int S, int H, int KV, int hd, uint16_t* dqkv, int window, int* err,
-                       cudaStream_t st);
+                       const float* dvec, int B, int S, int H, int KV, int hd, uint16_t* dqkv, int window, int parts,
+                       float* wk, float* wv, float* wq, int* err, cudaStream_t st);
 
 }  // namespace mebp
