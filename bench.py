@@ -84,8 +84,10 @@ class OracleSample:
     Sample: block 0 decompressed (LazyLoadAndDecompressWeights), its forward, then the recompute +
     backward (block_objective) on the first `block_tokens` tokens of one sequence; and the LM head
     (final norm + logits + CE + dE/dh) on `lm_tokens` tokens against a `lm_rows`-row slice of the
-    decompressed vocabulary.  Extrapolation is linear: blocks x L x (tokens / block_tokens), LM
-    head x (tokens / lm_tokens) x (V / lm_rows).  Attention's quadratic term is extrapolated
+    decompressed vocabulary.  Extrapolation is linear in what each part scales with: a block's
+    decompression x 2 L (forward and recompute), its forward + backward x L x tokens / block_tokens,
+    the embedding's decompression x V / lm_rows, the LM head x tokens / lm_tokens x V / lm_rows.
+    Attention's quadratic term is extrapolated
     linearly too, which slightly flatters the CPU.  Compression (done once when a model is loaded)
     is outside the timed sample.  full=True times the whole Algorithm 1 step instead (--cpu-full-step;
     about 40 s on 8 cores for the Qwen2.5-0.5B shape, hours for the larger ones)."""
@@ -123,10 +125,13 @@ class OracleSample:
             self.h = rng.standard_normal((lm_tokens, d.hidden))
             self.tg = rng.integers(0, rows, lm_tokens).astype(np.int64)
             self.lm = (rows, lm_tokens)
-        self.desc = (f"oracle (numpy fp64): block 0 (decompress, forward, recompute + backward) on {bt} of the "
-                     f"{d.seq} tokens of one sequence, extrapolated x{d.n_layers} blocks x{d.tokens // bt}; LM head "
-                     f"(decompress, final norm, logits, CE, dE/dh) on {lm_tokens} tokens x {self.lm[0] if self.lm else 0}"
-                     f" vocabulary rows, extrapolated x{d.tokens // lm_tokens} x{d.vocab / max(1, self.lm[0] if self.lm else 1):.0f}")
+        rows = self.lm[0] if self.lm else 0
+        self.desc = (f"oracle (numpy fp64): block 0 decompressed (x{2 * d.n_layers}: every block, forward and "
+                     f"recompute) and its forward + recompute + backward on {bt} of the {d.seq} tokens of one "
+                     f"sequence (x{d.n_layers} blocks x{d.tokens // bt}); the embedding's first {rows} rows "
+                     f"decompressed (x{d.vocab / max(1, rows):.0f}) and the LM head (final norm, logits, CE, dE/dh) "
+                     f"on {lm_tokens} tokens against them (x{d.tokens // lm_tokens} x{d.vocab / max(1, rows):.0f}); "
+                     f"extrapolated linearly to the step")
 
     def run(self):
         """Returns (seconds the sample took, seconds of the whole step it stands for)."""
@@ -138,20 +143,25 @@ class OracleSample:
             return t, t
         from oracle import quant
         t0 = time.perf_counter()
-        Wd = self.pm.decompress_block(0)
+        Wd = self.pm.decompress_block(0)            # once per block and pass: x L x 2 (forward, recompute)
+        t1 = time.perf_counter()
         OM.block_forward(self.x, Wd, self.L, self.d1)
-        OM.block_objective(self.x, Wd, self.L, self.G, self.d1)
-        t_blk = time.perf_counter() - t0
-        t_lm = 0.0
+        OM.block_objective(self.x, Wd, self.L, self.G, self.d1)  # per token: x L x tokens / bt
+        t2 = time.perf_counter()
+        t_dec, t_blk = t1 - t0, t2 - t1
+        t_dec_e = t_ce = 0.0
         if self.lm:
-            t1 = time.perf_counter()
-            Ed = quant.dequant(*self.qE)
-            OM.lm_head_ce(self.h, self.gf, Ed, self.tg, d.eps)
-            t_lm = time.perf_counter() - t1
-        sample = t_blk + t_lm
-        full = t_blk * d.n_layers * (d.tokens / self.bt)
+            t3 = time.perf_counter()
+            Ed = quant.dequant(*self.qE)            # once per step: x V / rows
+            t4 = time.perf_counter()
+            OM.lm_head_ce(self.h, self.gf, Ed, self.tg, d.eps)  # per token and row: x tokens / lm_tokens x V / rows
+            t5 = time.perf_counter()
+            t_dec_e, t_ce = t4 - t3, t5 - t4
+        sample = t_dec + t_blk + t_dec_e + t_ce
+        full = d.n_layers * (2 * t_dec + t_blk * d.tokens / self.bt)
         if self.lm:
-            full += t_lm * (d.tokens / self.lm[1]) * (d.vocab / self.lm[0])
+            vr = d.vocab / self.lm[0]
+            full += t_dec_e * vr + t_ce * (d.tokens / self.lm[1]) * vr
         return sample, full
 
 

@@ -38,19 +38,22 @@ constexpr float kRescale = 8.0f;  // log2 units
 
 template <int HD>
 struct Fwd {
+  // keys per block (64 at hd 256, with two K/V stages and two P buffers, measured 7 % slower than
+  // 128 with one of each: more blocks, more hand-offs)
+  static constexpr int BK = BKV;
   static constexpr int NST = HD == 256 ? 1 : (HD == 128 ? 2 : 3);  // key ring = value ring depth
   static constexpr int NP = HD == 256 ? 1 : 2;                      // probability buffers
   static constexpr int NCH = HD / 64;                               // 64-column (128-byte) chunks
   static constexpr int Q_BYTES = BQ * HD * 2;
-  static constexpr int KV_BYTES = BKV * HD * 2;
-  static constexpr int P_BYTES = BQ * BKV * 2;
+  static constexpr int KV_BYTES = BK * HD * 2;
+  static constexpr int P_BYTES = BQ * BK * 2;
   static constexpr int Q_OFF = 0;
   static constexpr int K_OFF = Q_OFF + Q_BYTES;
   static constexpr int V_OFF = K_OFF + NST * KV_BYTES;
   static constexpr int P_OFF = V_OFF + NST * KV_BYTES;
   static constexpr int BAR_OFF = P_OFF + NP * P_BYTES;
   static constexpr int SMEM = BAR_OFF + 256 + 1024;
-  static constexpr uint32_t TM_O = 0, TM_S = 256;  // TMEM columns: O [0, HD), scores 256 + 128 b
+  static constexpr uint32_t TM_O = 0, TM_S = 256;  // TMEM columns: O [0, HD), scores 256 + BK b
 };
 
 // CL > 1 (grids under one wave): the key blocks of a query tile are dealt round-robin to the CL
@@ -58,9 +61,10 @@ struct Fwd {
 // distributed shared memory, CTA c normalising and writing rows c*128/CL .. (c+1)*128/CL - 1.
 template <int HD, bool WIN, int CL>
 __global__ void __launch_bounds__(FWD_THREADS, 1)
-    fwd_tc_kernel(const __grid_constant__ CUtensorMap tm, int S, int H, int KV, uint16_t* __restrict__ o, int64_t ldo,
-                  float* __restrict__ lse, int W, int* err) {
+    fwd_tc_kernel(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtensorMap tmkv, int S, int H, int KV,
+                  uint16_t* __restrict__ o, int64_t ldo, float* __restrict__ lse, int W, int* err) {
   using C = Fwd<HD>;
+  constexpr int BKV = C::BK;  // keys per block in this kernel
   constexpr int NST = C::NST, NP = C::NP;
   static_assert(C::SMEM <= 232448, "shared memory");
   static_assert(C::SMEM > 232448 / 2, "one CTA per SM (512 TMEM columns each)");
@@ -118,6 +122,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1)
     // ---------------------------------------------------------------- query + key tiles
     if (lane == 0) {
       tma_prefetch_desc(&tm);
+      tma_prefetch_desc(&tmkv);
       mbar_arrive_expect_tx(qfull, C::Q_BYTES);
       for (int c = 0; c < C::NCH; ++c) tma_load_3d(sm + C::Q_OFF + c * BQ * 128, &tm, qfull, h * HD + c * 64, q0, b);
       int issued = 0;
@@ -126,7 +131,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1)
         if (j >= NST && !mbar_wait(&kempty[s], ((j / NST) & 1) ^ 1, abort_flag, err)) break;
         mbar_arrive_expect_tx(&kfull[s], C::KV_BYTES);
         for (int c = 0; c < C::NCH; ++c)
-          tma_load_3d(sm + C::K_OFF + s * C::KV_BYTES + c * BKV * 128, &tm, &kfull[s], (H + kvh) * HD + c * 64,
+          tma_load_3d(sm + C::K_OFF + s * C::KV_BYTES + c * BKV * 128, &tmkv, &kfull[s], (H + kvh) * HD + c * 64,
                       kblock(j) * BKV, b);
         issued = j + 1;
       }
@@ -144,7 +149,7 @@ __global__ void __launch_bounds__(FWD_THREADS, 1)
         if (j >= NST && !mbar_wait(&vempty[s], ((j / NST) & 1) ^ 1, abort_flag, err)) break;
         mbar_arrive_expect_tx(&vfull[s], C::KV_BYTES);
         for (int c = 0; c < C::NCH; ++c)
-          tma_load_3d(sm + C::V_OFF + s * C::KV_BYTES + c * BKV * 128, &tm, &vfull[s],
+          tma_load_3d(sm + C::V_OFF + s * C::KV_BYTES + c * BKV * 128, &tmkv, &vfull[s],
                       (H + KV + kvh) * HD + c * 64, kblock(j) * BKV, b);
         issued = j + 1;
       }
@@ -372,8 +377,8 @@ __global__ void __launch_bounds__(FWD_THREADS, 1)
 }
 
 template <int HD, bool WIN, int CL>
-int fwd_launch_cl(const CUtensorMap& tm, int B, int S, int H, int KV, uint16_t* o, int64_t ldo, float* lse, int W,
-                  int* err, cudaStream_t st) {
+int fwd_launch_cl(const CUtensorMap& tm, const CUtensorMap& tmkv, int B, int S, int H, int KV, uint16_t* o,
+                  int64_t ldo, float* lse, int W, int* err, cudaStream_t st) {
   using C = Fwd<HD>;
   static_assert(BQ * (HD + 4) * 4 + BQ * 16 <= C::BAR_OFF, "parked O and (m, l) fit below the barriers");
   static bool attr = false;
@@ -386,27 +391,35 @@ int fwd_launch_cl(const CUtensorMap& tm, int B, int S, int H, int KV, uint16_t* 
     attr = true;
   }
   const dim3 grid(H * CL, B, (S + BQ - 1) / BQ);
-  if (CL == 1) launch_k(fwd_tc_kernel<HD, WIN, CL>, grid, FWD_THREADS, C::SMEM, st, tm, S, H, KV, o, ldo, lse, W, err);
+  if (CL == 1)
+    launch_k(fwd_tc_kernel<HD, WIN, CL>, grid, FWD_THREADS, C::SMEM, st, tm, tmkv, S, H, KV, o, ldo, lse, W, err);
   else
-    launch_k_cluster(fwd_tc_kernel<HD, WIN, CL>, grid, FWD_THREADS, C::SMEM, st, dim3(CL, 1, 1), tm, S, H, KV, o, ldo,
-                     lse, W, err);
+    launch_k_cluster(fwd_tc_kernel<HD, WIN, CL>, grid, FWD_THREADS, C::SMEM, st, dim3(CL, 1, 1), tm, tmkv, S, H, KV, o,
+                     ldo, lse, W, err);
   return cudaGetLastError() == cudaSuccess ? MEBP_OK : MEBP_ERR_CUDA;
 }
 
 template <int HD, bool WIN>
 int fwd_launch(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uint16_t* o, int64_t ldo, float* lse,
                int W, int* err, cudaStream_t st) {
-  CUtensorMap tm;
-  // {columns of the fused projection buffer, positions, sequences}, 64 x 128 x 1 boxes
-  int rc = make_tmap_3d(&tm, qkv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, ld, S, B, ld * 2, static_cast<uint64_t>(S) * ld * 2,
-                        64, BQ, 1, CU_TENSOR_MAP_SWIZZLE_128B);
+  CUtensorMap tm, tmkv;
+  // {columns of the fused projection buffer, positions, sequences}: 64 x 128 x 1 boxes for the
+  // query tile, 64 x BK x 1 for key / value blocks
+  const uint64_t seq = static_cast<uint64_t>(S) * ld * 2;
+  int rc = make_tmap_3d(&tm, qkv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, ld, S, B, ld * 2, seq, 64, BQ, 1,
+                        CU_TENSOR_MAP_SWIZZLE_128B);
+  if (!rc)
+    rc = make_tmap_3d(&tmkv, qkv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, ld, S, B, ld * 2, seq, 64, Fwd<HD>::BK, 1,
+                      CU_TENSOR_MAP_SWIZZLE_128B);
   if (rc) return rc;
   // grids under one wave share each query tile's key blocks among a cluster of 2 or 4 CTAs
   const int64_t tiles = static_cast<int64_t>((S + BQ - 1) / BQ) * H * B;
-  const int nkb_max = (S + BKV - 1) / BKV;
-  if (tiles * 4 <= 152 && nkb_max >= 4) return fwd_launch_cl<HD, WIN, 4>(tm, B, S, H, KV, o, ldo, lse, W, err, st);
-  if (tiles * 2 <= 152 && nkb_max >= 2) return fwd_launch_cl<HD, WIN, 2>(tm, B, S, H, KV, o, ldo, lse, W, err, st);
-  return fwd_launch_cl<HD, WIN, 1>(tm, B, S, H, KV, o, ldo, lse, W, err, st);
+  const int nkb_max = (S + Fwd<HD>::BK - 1) / Fwd<HD>::BK;
+  if (tiles * 4 <= 152 && nkb_max >= 4)
+    return fwd_launch_cl<HD, WIN, 4>(tm, tmkv, B, S, H, KV, o, ldo, lse, W, err, st);
+  if (tiles * 2 <= 152 && nkb_max >= 2)
+    return fwd_launch_cl<HD, WIN, 2>(tm, tmkv, B, S, H, KV, o, ldo, lse, W, err, st);
+  return fwd_launch_cl<HD, WIN, 1>(tm, tmkv, B, S, H, KV, o, ldo, lse, W, err, st);
 }
 
 // ================================================================================== backward
@@ -425,7 +438,12 @@ int fwd_launch(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uin
 // the scores of block j (the stage is reused); otherwise the scores of block j go first so the
 // tensor cores run while the softmax warps work.
 constexpr int BWD_THREADS = 192;  // warps 0-3 elementwise + epilogue, 4 TMA, 5 MMA
-constexpr int BQB = 64;           // queries per dK/dV iteration, keys per dQ iteration
+// Queries per dK/dV iteration and keys per dQ iteration.  (At hd 256 the resident 128-row tiles,
+// K and V or Q and dO, take 128 KB and leave room for one operand stage of 64-row blocks; 32-row
+// blocks with two stages measured 18 % slower: more iterations, more hand-offs.)  The P^T / dS^T /
+// dS tiles have 128-byte rows (64 columns).
+template <int HD>
+constexpr int bwd_block() { return 64; }
 
 // Split mode (grids under one wave): a dK/dV item is one (128 keys, query head, part) and takes
 // every P-th query block of that head; a dQ item is one (128 queries, head, part) and takes every
@@ -439,19 +457,20 @@ struct SplitOut {
 
 template <int HD>
 struct DkDv {
+  static constexpr int QB = bwd_block<HD>();       // queries per iteration
   static constexpr int DC = HD == 256 ? 128 : HD;  // output columns per CTA
   static constexpr int NCOL = HD / DC;
   static constexpr int NS = HD == 256 ? 1 : (HD == 128 ? 3 : 4);  // (Q, dO) stages
   static constexpr int NPB = HD == 256 ? 1 : 2;                   // (P^T, dS^T) buffers
   static constexpr int NCH = HD / 64;
   static constexpr int KV_BYTES = BKV * HD * 2;   // one of K, V
-  static constexpr int Q_BYTES = BQB * HD * 2;    // one of Q_i, dO_i
-  static constexpr int P_BYTES = BKV * BQB * 2;   // one of P^T, dS^T
+  static constexpr int Q_BYTES = QB * HD * 2;     // one of Q_i, dO_i
+  static constexpr int P_BYTES = BKV * 64 * 2;    // one of P^T, dS^T (128-byte rows)
   static constexpr int K_OFF = 0, V_OFF = KV_BYTES;
   static constexpr int Q_OFF = 2 * KV_BYTES;      // stage s: Q at Q_OFF + 2 s Q_BYTES, dO after it
   static constexpr int P_OFF = Q_OFF + NS * 2 * Q_BYTES;  // buffer p: P^T, then dS^T
   static constexpr int VEC_OFF = P_OFF + NPB * 2 * P_BYTES;  // [2][2][64] floats: lse*log2e, D
-  static constexpr int BAR_OFF = VEC_OFF + 2 * 2 * BQB * 4;
+  static constexpr int BAR_OFF = VEC_OFF + 2 * 2 * 64 * 4;
   static constexpr int SMEM = BAR_OFF + 256 + 1024;
   static constexpr uint32_t TM_DK = 0, TM_DV = DC, TM_S = 256;  // S^T / dP^T buffer b: 256 + 128 b (+64)
 };
@@ -464,7 +483,7 @@ __device__ __forceinline__ void dkdv_body(const CUtensorMap& tmKV, const CUtenso
                                           const float* __restrict__ dvec, uint16_t* __restrict__ dqkv, int64_t ld,
                                           int W, int* err, const SplitOut& so, int item, int B) {
   using C = DkDv<HD>;
-  constexpr int NS = C::NS, NPB = C::NPB, DC = C::DC;
+  constexpr int NS = C::NS, NPB = C::NPB, DC = C::DC, BQB = C::QB;
   static_assert(C::SMEM <= 232448, "shared memory");
   static_assert(C::SMEM > 232448 / 2, "one CTA per SM (512 TMEM columns each)");
   extern __shared__ uint8_t smem_raw[];
@@ -626,16 +645,16 @@ __device__ __forceinline__ void dkdv_body(const CUtensorMap& tmKV, const CUtenso
     // thread r < 64 carries lse * log2e of query q0 + r, thread r >= 64 D of query q0 + r - 64;
     // the value of iteration j + 1 is loaded while iteration j runs
     auto vec_load = [&](int j) -> float {
-      const int g = g_of(j), hh = h_first + g / per_head, q = (qb_first + g % per_head) * BQB + (r & 63);
+      const int g = g_of(j), hh = h_first + g / per_head, q = (qb_first + g % per_head) * BQB + (r % BQB);
       const int64_t li = (static_cast<int64_t>(b) * H + hh) * S + q;
-      return q < S ? (r < 64 ? lse[li] * kLog2e : dvec[li]) : 0.0f;
+      return (q < S && r < 2 * BQB) ? (r < BQB ? lse[li] * kLog2e : dvec[li]) : 0.0f;
     };
     float vnext = n_it > 0 ? vec_load(0) : 0.0f;
     bool ok = true;
     for (int j = 0; j < n_it; ++j) {
       const int q0 = (qb_first + g_of(j) % per_head) * BQB;
-      float* lv = vec + (j & 1) * 2 * BQB;  // [64] lse * log2e, then [64] D
-      lv[r] = vnext;
+      float* lv = vec + (j & 1) * 2 * 64;  // [BQB] lse * log2e, then [BQB] D
+      if (r < 2 * BQB) lv[r] = vnext;
       if (j + 1 < n_it) vnext = vec_load(j + 1);
       // every thread of the four warps has written its entry (and, by the same token, finished
       // reading this buffer two iterations ago): a bounded mbarrier, never a named barrier, so an
@@ -645,46 +664,46 @@ __device__ __forceinline__ void dkdv_body(const CUtensorMap& tmKV, const CUtenso
       if (!ok) break;
       ok = __all_sync(0xffffffffu, mbar_wait(&sfull[j & 1], (j >> 1) & 1, abort_flag, err));
       if (!ok) break;
-      if (j >= NPB) {
+      tc_fence_after();
+      const uint32_t ts = tmem + lane_off + C::TM_S + 128 * (j & 1);
+      float sv[BQB], dp[BQB];
+      if constexpr (BQB == 64) {
+        tmem_ld64(ts, sv);
+        tmem_ld64(ts + 64, dp);
+      } else {
+        tmem_ld32(ts, sv);
+        tmem_ld32(ts + 64, dp);
+      }
+      tc_fence_before();  // the score buffer may be overwritten once every warp has read it
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sfree[j & 1]);
+#pragma unroll
+      for (int e = 0; e < BQB; ++e) {
+        const int q = q0 + e;
+        const bool vis = kr <= q && q < S && kr < S && (!WIN || q - kr < W);
+        const float pv = vis ? exp2f(sv[e] * sc - lv[e]) : 0.0f;
+        sv[e] = pv;
+        dp[e] = pv * (dp[e] - lv[BQB + e]);
+      }
+      if (j >= NPB) {  // the P^T / dS^T buffer is free once the products of block j - NPB retired
         const int i = j - NPB;
         ok = __all_sync(0xffffffffu, mbar_wait(&pdone[i % NPB], (i / NPB) & 1, abort_flag, err));
         if (!ok) break;
       }
-      tc_fence_after();
-      const uint32_t ts = tmem + lane_off + C::TM_S + 128 * (j & 1);
       uint8_t* prow = sm + C::P_OFF + (j % NPB) * 2 * C::P_BYTES + r * 128;
-      {
-        static_assert(BQB == 64, "one 64-column TMEM load per score row");
-        constexpr int c = 0;
-        float sv[64], dp[64];
-        tmem_ld64(ts, sv);
-        tmem_ld64(ts + 64, dp);
 #pragma unroll
-        for (int e = 0; e < 64; ++e) {
-          const int qi = e, q = q0 + qi;
-          const bool vis = kr <= q && q < S && kr < S && (!WIN || q - kr < W);
-          const float pv = vis ? exp2f(sv[e] * sc - lv[qi]) : 0.0f;
-          sv[e] = pv;
-          dp[e] = pv * (dp[e] - lv[BQB + qi]);
-        }
-#pragma unroll
-        for (int qd = 0; qd < 8; ++qd) {  // 8 queries per 16-byte unit
-          const int w = 8 * c + qd, off = (w ^ (r & 7)) << 4;
-          *reinterpret_cast<uint4*>(prow + off) =
-              make_uint4(pack_half2(sv[8 * qd], sv[8 * qd + 1]), pack_half2(sv[8 * qd + 2], sv[8 * qd + 3]),
-                         pack_half2(sv[8 * qd + 4], sv[8 * qd + 5]), pack_half2(sv[8 * qd + 6], sv[8 * qd + 7]));
-          *reinterpret_cast<uint4*>(prow + C::P_BYTES + off) =
-              make_uint4(pack_half2(dp[8 * qd], dp[8 * qd + 1]), pack_half2(dp[8 * qd + 2], dp[8 * qd + 3]),
-                         pack_half2(dp[8 * qd + 4], dp[8 * qd + 5]), pack_half2(dp[8 * qd + 6], dp[8 * qd + 7]));
-        }
+      for (int qd = 0; qd < BQB / 8; ++qd) {  // 8 queries per 16-byte unit
+        const int off = (qd ^ (r & 7)) << 4;
+        *reinterpret_cast<uint4*>(prow + off) =
+            make_uint4(pack_half2(sv[8 * qd], sv[8 * qd + 1]), pack_half2(sv[8 * qd + 2], sv[8 * qd + 3]),
+                       pack_half2(sv[8 * qd + 4], sv[8 * qd + 5]), pack_half2(sv[8 * qd + 6], sv[8 * qd + 7]));
+        *reinterpret_cast<uint4*>(prow + C::P_BYTES + off) =
+            make_uint4(pack_half2(dp[8 * qd], dp[8 * qd + 1]), pack_half2(dp[8 * qd + 2], dp[8 * qd + 3]),
+                       pack_half2(dp[8 * qd + 4], dp[8 * qd + 5]), pack_half2(dp[8 * qd + 6], dp[8 * qd + 7]));
       }
       fence_proxy_async_smem();  // the MMA (async proxy) reads P^T and dS^T
-      tc_fence_before();         // the TMEM reads are ordered before the arrivals
       __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(&sfree[j & 1]);
-        mbar_arrive(&pready[j % NPB]);
-      }
+      if (lane == 0) mbar_arrive(&pready[j % NPB]);
     }
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(dfull, 0, abort_flag, err));
     tc_fence_after();
@@ -754,12 +773,13 @@ __device__ __forceinline__ void dkdv_body(const CUtensorMap& tmKV, const CUtenso
 
 template <int HD>
 struct Dq {
+  static constexpr int QB = bwd_block<HD>();                      // keys per iteration
   static constexpr int NS = HD == 256 ? 1 : (HD == 128 ? 3 : 4);  // (K_j, V_j) stages
   static constexpr int NPB = 2;                                   // dS buffers
   static constexpr int NCH = HD / 64;
   static constexpr int Q_BYTES = BQ * HD * 2;    // one of Q, dO
-  static constexpr int K_BYTES = BQB * HD * 2;   // one of K_j, V_j
-  static constexpr int P_BYTES = BQ * BQB * 2;   // one dS buffer
+  static constexpr int K_BYTES = QB * HD * 2;    // one of K_j, V_j
+  static constexpr int P_BYTES = BQ * 64 * 2;    // one dS buffer (128-byte rows)
   static constexpr int Q_OFF = 0, DO_OFF = Q_BYTES;
   static constexpr int K_OFF = 2 * Q_BYTES;      // stage s: K at K_OFF + 2 s K_BYTES, V after it
   static constexpr int P_OFF = K_OFF + NS * 2 * K_BYTES;
@@ -775,7 +795,7 @@ __device__ __forceinline__ void dq_body(const CUtensorMap& tmQ, const CUtensorMa
                                         const float* __restrict__ dvec, uint16_t* __restrict__ dqkv, int64_t ld,
                                         int W, int* err, const SplitOut& so, int x, int b, int z) {
   using C = Dq<HD>;
-  constexpr int NS = C::NS, NPB = C::NPB;
+  constexpr int NS = C::NS, NPB = C::NPB, BQB = C::QB;
   static_assert(C::SMEM <= 232448, "shared memory");
   static_assert(C::SMEM > 232448 / 2, "one CTA per SM (512 TMEM columns each)");
   extern __shared__ uint8_t smem_raw[];
@@ -929,24 +949,26 @@ __device__ __forceinline__ void dq_body(const CUtensorMap& tmQ, const CUtensorMa
       uint8_t* drow = sm + C::P_OFF + (j % NPB) * C::P_BYTES + r * 128;
       const int k0 = kblock(j) * BQB;
       {
-        constexpr int c = 0;
-        float sv[64], dp[64];
-        tmem_ld64(ts, sv);
-        tmem_ld64(ts + 64, dp);
+        float sv[BQB], dp[BQB];
+        if constexpr (BQB == 64) {
+          tmem_ld64(ts, sv);
+          tmem_ld64(ts + 64, dp);
+        } else {
+          tmem_ld32(ts, sv);
+          tmem_ld32(ts + 64, dp);
+        }
 #pragma unroll
-        for (int e = 0; e < 64; ++e) {
+        for (int e = 0; e < BQB; ++e) {
           const int key = k0 + e;
           const bool vis = key <= row && row < S && (!WIN || row - key < W);
           const float pv = vis ? exp2f(sv[e] * sc - l2) : 0.0f;
           dp[e] = pv * (dp[e] - dr);
         }
 #pragma unroll
-        for (int kd = 0; kd < 8; ++kd) {
-          const int w = 8 * c + kd;
-          *reinterpret_cast<uint4*>(drow + ((w ^ (r & 7)) << 4)) =
+        for (int kd = 0; kd < BQB / 8; ++kd)
+          *reinterpret_cast<uint4*>(drow + ((kd ^ (r & 7)) << 4)) =
               make_uint4(pack_half2(dp[8 * kd], dp[8 * kd + 1]), pack_half2(dp[8 * kd + 2], dp[8 * kd + 3]),
                          pack_half2(dp[8 * kd + 4], dp[8 * kd + 5]), pack_half2(dp[8 * kd + 6], dp[8 * kd + 7]));
-        }
       }
       fence_proxy_async_smem();
       tc_fence_before();
@@ -1064,17 +1086,18 @@ int bwd_launch(const uint16_t* qkv, int64_t ld, const uint16_t* dout, int64_t ld
     attr = true;
   }
   const uint64_t seq_q = static_cast<uint64_t>(S) * ld * 2, seq_o = static_cast<uint64_t>(S) * ldo * 2;
+  constexpr int QB = bwd_block<HD>();  // box rows of the 32 / 64-row operand blocks
   CUtensorMap kv128, q64, do64, q128, kv64, do128;
   int rc;
   if ((rc = make_tmap_3d(&kv128, qkv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, ld, S, B, ld * 2, seq_q, 64, BKV, 1,
                          CU_TENSOR_MAP_SWIZZLE_128B)) ||
-      (rc = make_tmap_3d(&q64, qkv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, ld, S, B, ld * 2, seq_q, 64, BQB, 1,
+      (rc = make_tmap_3d(&q64, qkv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, ld, S, B, ld * 2, seq_q, 64, QB, 1,
                          CU_TENSOR_MAP_SWIZZLE_128B)) ||
-      (rc = make_tmap_3d(&do64, dout, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, ldo, S, B, ldo * 2, seq_o, 64, BQB, 1,
+      (rc = make_tmap_3d(&do64, dout, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, ldo, S, B, ldo * 2, seq_o, 64, QB, 1,
                          CU_TENSOR_MAP_SWIZZLE_128B)) ||
       (rc = make_tmap_3d(&q128, qkv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, ld, S, B, ld * 2, seq_q, 64, BQ, 1,
                          CU_TENSOR_MAP_SWIZZLE_128B)) ||
-      (rc = make_tmap_3d(&kv64, qkv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, ld, S, B, ld * 2, seq_q, 64, BQB, 1,
+      (rc = make_tmap_3d(&kv64, qkv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, ld, S, B, ld * 2, seq_q, 64, QB, 1,
                          CU_TENSOR_MAP_SWIZZLE_128B)) ||
       (rc = make_tmap_3d(&do128, dout, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, ldo, S, B, ldo * 2, seq_o, 64, BQ, 1,
                          CU_TENSOR_MAP_SWIZZLE_128B)))
