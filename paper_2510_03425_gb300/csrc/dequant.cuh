@@ -11,7 +11,8 @@
 //   q   = t - (1032, 1032)                          exact small integers
 //   out = q * (s, s)                                one IEEE fp16 multiplication = fp16_rne(q * s)
 // i.e. 1 shift, 1 LOP3 and 2 half2 FP ops per two elements, and the scale is used as the
-// fp16 bits it is stored in.
+// fp16 bits it is stored in.  (The OR-into-the-mantissa conversion of small integers to fp16 is
+// the published "magic number" method of Kim et al., 2022, "Who Says Elephants Can't Run".)
 #pragma once
 #include "common.cuh"
 
