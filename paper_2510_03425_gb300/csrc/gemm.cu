@@ -63,6 +63,8 @@ static_assert(Layout<1>::SMEM <= 232448 && Layout<2>::SMEM <= 232448, "shared me
 // the idle rings.
 static_assert(Layout<1>::SMEM > 232448 / 2 && Layout<2>::SMEM > 232448 / 2, "one CTA per SM");
 static_assert(Layout<1>::BAR_OFF >= BM * BN * 4, "partial tile fits below the barriers");
+static_assert(Layout<1>::BAR_OFF >= Warps<1>::CONV * 8192 && Layout<2>::BAR_OFF >= Warps<2>::CONV * 8192,
+              "epilogue staging slots fit below the barriers");
 
 struct Params {
   int M, N, K;
@@ -178,8 +180,16 @@ __device__ __forceinline__ void copy_lora_b(const Params& p, int e, int n0, uint
 // of a quarter split the NACC x 256 accumulator columns into column groups cg = w >> 2:
 // NACC = 1 (16 warps): columns 64*cg .. +63 of the single accumulator;
 // NACC = 2 (8 warps):  accumulator cg (tile rows 128*cg + ...), all 256 columns.
+// Stored outputs go through the warp's 8 KB slot `stage` of shared memory (the rings are idle
+// once the accumulator is final), 64 columns per round.  tcgen05.ld hands each thread one row, so
+// written straight to global memory every store instruction would touch 32 rows (32 lines); that
+// made the epilogue a quarter of a CTA's life.  Phase 1: thread = row writes its values to the
+// slot, 16-byte chunk c of row r at chunk c ^ (r & 7) within its 128-byte half (no bank
+// conflicts).  Phase 2: the warp copies the slot out with consecutive lanes on consecutive chunks
+// of a row, so each instruction writes (and, for the residual, reads) whole 128-byte lines.
 template <int NACC>
-__device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int warp, int lane, int m0, int n0) {
+__device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int warp, int lane, int m0, int n0,
+                                         uint8_t* stage) {
   const int q = warp & 3, cg = warp >> 2;
   constexpr int NCG = Warps<NACC>::CONV / 4;            // column groups
   constexpr int COLS = NACC * 256 / NCG;                // columns per group
@@ -229,68 +239,82 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
     return;
   }
 
-  if (p.epi == EPI_CEGRAD) {
-    const float lse = row_ok ? p.lse[row] : 0.0f;
-    const int tgt = row_ok ? p.targets[row] : -1;
-    const float w = (tgt >= 0) ? *p.ce_w : 0.0f;
-    const int tl = tgt - p.col_offset;
-    uint16_t* C = static_cast<uint16_t*>(p.C);
-#pragma unroll 1
-    for (int cc = 0; cc < NCH; ++cc) {
-      float v[32];
-      tmem_ld32(tbase + 32 * cc, v);
-      const int c0 = cbase + 32 * cc;
-      if (!row_ok || c0 >= p.N) continue;
-      uint32_t o[16];
-#pragma unroll
-      for (int i = 0; i < 32; i += 2) {
-        float a = (c0 + i < p.n_valid) ? __expf(v[i] - lse) * w : 0.0f;
-        float b = (c0 + i + 1 < p.n_valid) ? __expf(v[i + 1] - lse) * w : 0.0f;
-        if (c0 + i == tl) a -= w;
-        if (c0 + i + 1 == tl) b -= w;
-        o[i / 2] = pack_half2(a, b);
-      }
-      uint4* dst = reinterpret_cast<uint4*>(C + static_cast<int64_t>(row) * p.ldc + c0);
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-        if (c0 + 8 * i < p.N) dst[i] = make_uint4(o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
-    }
-    return;
-  }
-
+  // EPI_F16, EPI_CEGRAD (fp16 rows of 128 bytes per round) and EPI_F32 (fp32, 256 bytes)
+  const bool f32 = p.epi == EPI_F32, ce = p.epi == EPI_CEGRAD;
+  const float lse = (ce && row_ok) ? p.lse[row] : 0.0f;
+  const int tgt = (ce && row_ok) ? p.targets[row] : -1;
+  const float cw = (tgt >= 0) ? *p.ce_w : 0.0f;
+  const int tl = tgt - p.col_offset;
+  const int row0 = row - lane;
   uint32_t bad = 0;  // an fp16 output overflowed (or is NaN)
 #pragma unroll 1
-  for (int cc = 0; cc < NCH; ++cc) {
-    float v[32];
-    tmem_ld32(tbase + 32 * cc, v);
-    const int c0 = cbase + 32 * cc;
-    if (!row_ok || c0 >= p.N) continue;
-    if (p.epi == EPI_F16) {
-      uint16_t* C = static_cast<uint16_t*>(p.C);
-      uint4* dst = reinterpret_cast<uint4*>(C + static_cast<int64_t>(row) * p.ldc + c0);
+  for (int rd = 0; rd < COLS / 64; ++rd) {
+    const int c0 = cbase + 64 * rd;
+    if (c0 >= p.N) break;  // warp-uniform (N is a multiple of 64)
+    float v[64];
+    {
+      float lo[32], hi[32];
+      tmem_ld32(tbase + 64 * rd, lo);
+      tmem_ld32(tbase + 64 * rd + 32, hi);
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
-        if (c0 + 8 * i < p.N) {
-          const uint4 o = make_uint4(pack_half2(v[8 * i], v[8 * i + 1]), pack_half2(v[8 * i + 2], v[8 * i + 3]),
-                                     pack_half2(v[8 * i + 4], v[8 * i + 5]), pack_half2(v[8 * i + 6], v[8 * i + 7]));
-          bad |= h2_nonfinite(o.x) | h2_nonfinite(o.y) | h2_nonfinite(o.z) | h2_nonfinite(o.w);
-          dst[i] = o;
-        }
-    } else {  // EPI_F32 (+ residual)
-      float4* dst = reinterpret_cast<float4*>(static_cast<float*>(p.C) + static_cast<int64_t>(row) * p.ldc + c0);
-      const float4* res = p.R ? reinterpret_cast<const float4*>(p.R + static_cast<int64_t>(row) * p.ldr + c0) : nullptr;
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        if (c0 + 4 * i >= p.N) break;
-        float4 o = make_float4(p.alpha * v[4 * i], p.alpha * v[4 * i + 1], p.alpha * v[4 * i + 2],
-                               p.alpha * v[4 * i + 3]);
-        if (res) {
-          const float4 r = res[i];
-          o.x += r.x; o.y += r.y; o.z += r.z; o.w += r.w;
-        }
-        dst[i] = o;
+      for (int i = 0; i < 32; ++i) {
+        v[i] = lo[i];
+        v[32 + i] = hi[i];
       }
     }
+    // ---- phase 1: this thread's row into the slot
+    if (f32) {
+      uint8_t* srow = stage + lane * 256;
+#pragma unroll
+      for (int j = 0; j < 16; ++j)
+        *reinterpret_cast<float4*>(srow + (((j & 8) | ((j ^ lane) & 7)) << 4)) =
+            make_float4(p.alpha * v[4 * j], p.alpha * v[4 * j + 1], p.alpha * v[4 * j + 2], p.alpha * v[4 * j + 3]);
+    } else {
+      if (ce) {
+#pragma unroll
+        for (int i = 0; i < 64; ++i) {
+          float a = (c0 + i < p.n_valid) ? __expf(v[i] - lse) * cw : 0.0f;
+          if (c0 + i == tl) a -= cw;
+          v[i] = a;
+        }
+      }
+      uint8_t* srow = stage + lane * 128;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const uint4 o = make_uint4(pack_half2(v[8 * j], v[8 * j + 1]), pack_half2(v[8 * j + 2], v[8 * j + 3]),
+                                   pack_half2(v[8 * j + 4], v[8 * j + 5]), pack_half2(v[8 * j + 6], v[8 * j + 7]));
+        if (!ce && row_ok) bad |= h2_nonfinite(o.x) | h2_nonfinite(o.y) | h2_nonfinite(o.z) | h2_nonfinite(o.w);
+        *reinterpret_cast<uint4*>(srow + (((j ^ lane) & 7) << 4)) = o;
+      }
+    }
+    __syncwarp();
+    // ---- phase 2: whole lines out (rows past M skipped)
+    if (f32) {
+      float* C = static_cast<float*>(p.C);
+      const int c = lane & 15;
+#pragma unroll 4
+      for (int i = 0; i < 16; ++i) {
+        const int rr = 2 * i + (lane >> 4), r = row0 + rr;
+        float4 o = *reinterpret_cast<const float4*>(stage + rr * 256 + (((c & 8) | ((c ^ rr) & 7)) << 4));
+        if (r < p.M) {
+          if (p.R) {
+            const float4 res = *reinterpret_cast<const float4*>(p.R + static_cast<int64_t>(r) * p.ldr + c0 + 4 * c);
+            o.x += res.x; o.y += res.y; o.z += res.z; o.w += res.w;
+          }
+          *reinterpret_cast<float4*>(C + static_cast<int64_t>(r) * p.ldc + c0 + 4 * c) = o;
+        }
+      }
+    } else {
+      uint16_t* C = static_cast<uint16_t*>(p.C);
+      const int c = lane & 7;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int rr = 4 * i + (lane >> 3), r = row0 + rr;
+        const uint4 o = *reinterpret_cast<const uint4*>(stage + rr * 128 + (((c ^ rr) & 7) << 4));
+        if (r < p.M) *reinterpret_cast<uint4*>(C + static_cast<int64_t>(r) * p.ldc + c0 + 8 * c) = o;
+      }
+    }
+    __syncwarp();  // the slot is rewritten by the next round
   }
   if (bad) flag_error(p.err, kErrNonFinite);
 }
@@ -516,7 +540,7 @@ __global__ void __launch_bounds__(Warps<NACC>::THREADS, 1)
     const bool acc_ok = __all_sync(0xffffffffu, mbar_wait(accf, 0, abort_flag, p.err));
     tc_fence_after();
     if (split) stash_partial(tmem, acc_ok && total > 0, warp, lane, smem);
-    else if (acc_ok && total > 0) epilogue<NACC>(p, tmem, warp, lane, m0, n0);
+    else if (acc_ok && total > 0) epilogue<NACC>(p, tmem, warp, lane, m0, n0, smem + warp * 8192);
   }
 
   tc_fence_before();
