@@ -17,7 +17,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(HERE, "libmebp.so")
-SOURCES = ["quant.cu", "gemm.cu", "gemm_s.cu", "small.cu", "lora.cu", "skinny_tc.cu", "attention.cu", "attention_tc.cu", "mebp.cu", "noalloc.cu", "optim.cu"]
+SOURCES = ["quant.cu", "gemm.cu", "gemm_s.cu", "small.cu", "lora.cu", "skinny_tc.cu", "tall_tc.cu", "attention.cu", "attention_tc.cu", "mebp.cu", "noalloc.cu", "optim.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ARCH + ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-fno-strict-aliasing",
                 "--expt-relaxed-constexpr", "-I" + os.path.join(ROOT, "include")]

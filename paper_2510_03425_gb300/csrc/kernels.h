@@ -183,7 +183,20 @@ int launch_skinny_tc(const uint16_t* X, int64_t ldx, int64_t M, int64_t K, const
 // The sum is multiplied by *mult (mult may be null = 1) before it is written / added.
 int launch_tall_reduce(const uint16_t* P, int64_t ldp, const uint16_t* Q, int64_t ldq, int64_t M, int Pw, int Qw,
                        float* C, int64_t ldc, bool accumulate, const float* mult, float* scratch,
-                       int64_t scratch_floats, cudaStream_t st);
+                       int64_t scratch_floats, int* err, cudaStream_t st);
+// Several reductions over the same P at once: C[j][p, q] (+)= mult * sum_m P[m, p] Q[m, j r + q],
+// j < nq (ldc shared); on tcgen05 (tall_tc.cu) where tall_tc_takes() says so, else nq calls of the
+// above.
+int launch_tall_reduce_multi(const uint16_t* P, int64_t ldp, const uint16_t* Q, int64_t ldq, int64_t M, int Pw,
+                             int nq, int r, float* const* C, int64_t ldc, bool accumulate, const float* mult,
+                             float* scratch, int64_t scratch_floats, int* err, cudaStream_t st);
+bool tall_tc_takes(int64_t M, int Pw, int nq, int r);
+// The tcgen05 reduction; MEBP_ERR_UNSUPPORTED for shapes it does not take.
+int launch_tall_tc(const uint16_t* P, int64_t ldp, const uint16_t* Q, int64_t ldq, int64_t M, int Pw, int nq, int r,
+                   float* const* C, int64_t ldc, bool accumulate, const float* mult, int* err, cudaStream_t st);
+// C[p * sp + q * sq] (+)= mult * sum over splits of part[z][p][q], in split order.
+void launch_split_sum(const float* part, int splits, int Pw, int Qw, float* C, int64_t sp, int64_t sq, bool accumulate,
+                      const float* mult, cudaStream_t st);
 int64_t tall_reduce_scratch_floats(int64_t M, int Pw, int Qw);
 // Up to kTallMaxProbs single-pass reductions C (+)= mult * P^T Q over the same M rows in one launch
 // (Qw <= 32, Pw and Qw multiples of 8).  tall_batch_add returns false for a problem it cannot take.

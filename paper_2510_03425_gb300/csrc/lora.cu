@@ -374,6 +374,40 @@ __global__ void split_sum_kernel(const float* __restrict__ part, int splits, int
   *dst = accumulate ? *dst + s : s;
 }
 
+void launch_split_sum(const float* part, int splits, int Pw, int Qw, float* C, int64_t sp, int64_t sq, bool accumulate,
+                      const float* mult, cudaStream_t st) {
+  const int64_t n = static_cast<int64_t>(Pw) * Qw;
+  launch_k(split_sum_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, st, part, splits, Pw, Qw, C, sp, sq,
+           accumulate ? 1 : 0, mult);
+}
+
+// Token counts from this on take the tcgen05 kernel (tall_tc.cu) where the shapes allow.
+constexpr int64_t kTallTcMinM = 2048;
+
+bool tall_tc_takes(int64_t M, int Pw, int nq, int r) {
+  const int qw = nq * r;
+  return M >= kTallTcMinM && Pw % 64 == 0 && r % 16 == 0 && (qw == 16 || qw == 32 || qw == 64 || qw == 96);
+}
+
+int launch_tall_reduce_multi(const uint16_t* P, int64_t ldp, const uint16_t* Q, int64_t ldq, int64_t M, int Pw,
+                             int nq, int r, float* const* C, int64_t ldc, bool accumulate, const float* mult,
+                             float* scratch, int64_t scratch_floats, int* err, cudaStream_t st) {
+  if (Pw <= 0 || M <= 0) return MEBP_OK;
+  if (tall_tc_takes(M, Pw, nq, r) && ldp % 8 == 0 && ldq % 8 == 0 &&
+      !((reinterpret_cast<uintptr_t>(P) | reinterpret_cast<uintptr_t>(Q)) & 15)) {
+    const int rc = launch_tall_tc(P, ldp, Q, ldq, M, Pw, nq, r, C, ldc, accumulate, mult, err, st);
+    if (rc != MEBP_ERR_UNSUPPORTED) return rc;
+  }
+  for (int j = 0; j < nq; ++j) {  // one target at a time (the tensor-core kernel where it takes one)
+    const int rc = nq > 1 ? launch_tall_reduce_multi(P, ldp, Q + j * r, ldq, M, Pw, 1, r, C + j, ldc, accumulate, mult,
+                                                     scratch, scratch_floats, err, st)
+                          : launch_tall_reduce(P, ldp, Q, ldq, M, Pw, r, C[0], ldc, accumulate, mult, scratch,
+                                               scratch_floats, err, st);
+    if (rc) return rc;
+  }
+  return MEBP_OK;
+}
+
 int64_t tall_reduce_scratch_floats(int64_t M, int Pw, int Qw) {
   (void)M;
   return static_cast<int64_t>(Pw) * Qw * 16;
@@ -383,7 +417,8 @@ int64_t tall_reduce_scratch_floats(int64_t M, int Pw, int Qw) {
 // (transposed output).
 int launch_tall_reduce(const uint16_t* P, int64_t ldp, const uint16_t* Q, int64_t ldq, int64_t M, int Pw, int Qw,
                        float* C, int64_t ldc, bool accumulate, const float* mult, float* scratch,
-                       int64_t scratch_floats, cudaStream_t st) {
+                       int64_t scratch_floats, int* err, cudaStream_t st) {
+  (void)err;
   if (Pw <= 0 || Qw <= 0) return MEBP_OK;
   if ((Pw % 8) || (Qw % 8) || Qw > 96) return MEBP_ERR_UNSUPPORTED;
   const int nq = Qw <= 32 ? 4 : (Qw <= 64 ? 8 : 12);

@@ -494,6 +494,26 @@ int lin_grads(mebp_ctx* c, const Acts& A, const uint16_t* du, int li, const uint
               const uint16_t* X, int64_t ldx, int64_t T, const mebp_lora_grads* grads, bool acc,
               const float* grad_mult, cudaStream_t st, TallBatch* tb = nullptr) {
   const Lin& l = c->lin[li];
+  // dA of all the linear's targets in one pass over X when they sit side by side in dU (their rank
+  // blocks consecutive) and the tensor-core reduction takes the shape
+  bool dA_fused = false;
+  if (grads && !tb && l.nt > 1) {
+    bool ok = true;
+    float* Cs[3] = {nullptr, nullptr, nullptr};
+    for (int t = 0; t < l.nt; ++t) {
+      ok = ok && grads->dA[l.tgt[t]] && l.ro[t] == l.ro[0] + t * c->r;
+      Cs[t] = grads->dA[l.tgt[t]];
+    }
+    if (ok && tall_tc_takes(T, l.K, l.nt, c->r)) {
+      int rc = MEBP_OK;
+      KP(c, KK_LORA_REDUCE, bytes_tall(T, l.K, l.nt * c->r, acc), 2.0 * T * l.K * l.nt * c->r, st, [&] {
+        rc = launch_tall_reduce_multi(X, ldx, du + l.ro[0], l.kxp, T, l.K, l.nt, c->r, Cs, -l.K, acc, grad_mult,
+                                      c->red, c->red_floats, c->d_err, st);
+      });
+      if (rc) return fail(c, rc, "LoRA dA reduction");
+      dA_fused = true;
+    }
+  }
   for (int t = 0; t < l.nt; ++t) {
     const int tg = l.tgt[t];
     if (!grads) break;
@@ -502,17 +522,19 @@ int lin_grads(mebp_ctx* c, const Acts& A, const uint16_t* du, int li, const uint
                                acc))) {
       int rc = MEBP_OK;
       KP(c, KK_LORA_REDUCE, bytes_tall(T, l.nl[t], c->r, acc), 2.0 * T * l.nl[t] * c->r, st, [&] {
-        rc = launch_tall_reduce(dY + l.no[t], ldy, A.us[li] + l.ro[t], l.kxp, T, l.nl[t], c->r, grads->dB[tg], c->r,
-                                acc, grad_mult, c->red, c->red_floats, st);
+        float* C1[1] = {grads->dB[tg]};
+        rc = launch_tall_reduce_multi(dY + l.no[t], ldy, A.us[li] + l.ro[t], l.kxp, T, l.nl[t], 1, c->r, C1, c->r,
+                                      acc, grad_mult, c->red, c->red_floats, c->d_err, st);
       });
       if (rc) return fail(c, rc, "LoRA dB reduction");
     }
-    if (grads->dA[tg] &&
+    if (grads->dA[tg] && !dA_fused &&
         !(tb && tall_batch_add(*tb, X, ldx, du + l.ro[t], l.kxp, l.K, c->r, grads->dA[tg], -l.K, acc))) {
       int rc = MEBP_OK;
       KP(c, KK_LORA_REDUCE, bytes_tall(T, l.K, c->r, acc), 2.0 * T * l.K * c->r, st, [&] {
-        rc = launch_tall_reduce(X, ldx, du + l.ro[t], l.kxp, T, l.K, c->r, grads->dA[tg], -l.K, acc, grad_mult,
-                                c->red, c->red_floats, st);
+        float* C1[1] = {grads->dA[tg]};
+        rc = launch_tall_reduce_multi(X, ldx, du + l.ro[t], l.kxp, T, l.K, 1, c->r, C1, -l.K, acc, grad_mult, c->red,
+                                      c->red_floats, c->d_err, st);
       });
       if (rc) return fail(c, rc, "LoRA dA reduction");
     }
