@@ -73,6 +73,8 @@ struct Params {
   const uint16_t* Bx;  // LoRA B operand (FWD [N, kx], TRANS [kx, N]), row pitch ldbx
   int64_t ldbx;
   int kt_split;        // main 64-wide K tiles per split (blockIdx.z)
+  int m_group;         // > 0: grouped tile order over a 1-D grid (see the host), else (n, m) = blockIdx
+  int tiles_m, tiles_n;
   int epi;             // GemmEpi
   void* C;
   int64_t ldc;
@@ -228,7 +230,7 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
       }
     }
     if (row_ok) {  // four (max, sum) parts per 256-column tile and row; unused parts are empty
-      float2* pr = reinterpret_cast<float2*>(p.lse_part) + static_cast<int64_t>(row) * p.nparts + blockIdx.x * 4;
+      float2* pr = reinterpret_cast<float2*>(p.lse_part) + static_cast<int64_t>(row) * p.nparts + (n0 / BN) * 4;
       constexpr int GPR = 256 / COLS;      // column groups per row (1 or 4)
       const int part = col0 / COLS;
       pr[part] = make_float2(mx, sum);
@@ -410,7 +412,14 @@ __global__ void __launch_bounds__(Warps<NACC>::THREADS, 1)
 
   griddep_launch();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM * NACC;
+  int n_tile = blockIdx.x, m_tile = blockIdx.y;
+  if (p.m_group > 0) {  // groups of m_group row tiles, row-fastest within a group
+    const int per = p.m_group * p.tiles_n, g = static_cast<int>(blockIdx.x) / per, idx = static_cast<int>(blockIdx.x) % per;
+    const int rows = min(p.m_group, p.tiles_m - g * p.m_group);
+    m_tile = g * p.m_group + idx % rows;
+    n_tile = idx / rows;
+  }
+  const int n0 = n_tile * BN, m0 = m_tile * BM * NACC;
   // K range of this split: main tiles [kt0, kt1); the LoRA block rides with the last split.
   const int num_k = p.K / BK;
   const int kt0 = blockIdx.z * p.kt_split;
@@ -775,6 +784,17 @@ int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st) {
   splits = (num_k + kt_split - 1) / kt_split;  // every split gets >= 1 K tile
   p.kt_split = kt_split;
   dim3 grid(tiles_n, tiles_m, splits);
+  // Consecutive CTAs share their row tile of A and walk through the weight tiles, so a weight
+  // operand larger than the L2 (the LM head's whole vocabulary) would be streamed once per row
+  // tile.  Then run the tiles in groups of 16 row tiles, row-fastest within a group: the weights
+  // stream once per group and the group's rows of A stay in L2.
+  const double w_bytes = static_cast<double>(g.N) * g.K * (0.5 + 1.0 / 32);
+  if (w_bytes > 64.0 * (1 << 20) && tiles_m > 1 && splits == 1) {
+    p.m_group = 16;
+    p.tiles_m = tiles_m;
+    p.tiles_n = tiles_n;
+    grid = dim3(static_cast<unsigned>(tiles_m) * static_cast<unsigned>(tiles_n), 1, 1);
+  }
   if (g.trans)
     rc = nacc == 2 ? launch_variant<true, 2>(grid, tA, tP, tS, tAx, p, st)
                    : launch_variant<true, 1>(grid, tA, tP, tS, tAx, p, st);
