@@ -457,23 +457,42 @@ struct SplitOut {
 
 template <int HD>
 struct DkDv {
+  // hd 256: V lives in TMEM as the A operand of dP^T = V dO^T (tcgen05 reads A from TMEM), which
+  // frees its 64 KB of shared memory for a second (Q, dO) stage; V lands in that stage's slot once
+  // and the elementwise warps copy it row by row into TMEM before the loop.
+  static constexpr bool VT = HD == 256;
   static constexpr int QB = bwd_block<HD>();       // queries per iteration
   static constexpr int DC = HD == 256 ? 128 : HD;  // output columns per CTA
   static constexpr int NCOL = HD / DC;
-  static constexpr int NS = HD == 256 ? 1 : (HD == 128 ? 3 : 4);  // (Q, dO) stages
+  static constexpr int NS = HD == 256 ? 2 : (HD == 128 ? 3 : 4);  // (Q, dO) stages
   static constexpr int NPB = HD == 256 ? 1 : 2;                   // (P^T, dS^T) buffers
+  static constexpr int NSB = VT ? 1 : 2;                          // S^T / dP^T buffers in TMEM
   static constexpr int NCH = HD / 64;
   static constexpr int KV_BYTES = BKV * HD * 2;   // one of K, V
   static constexpr int Q_BYTES = QB * HD * 2;     // one of Q_i, dO_i
   static constexpr int P_BYTES = BKV * 64 * 2;    // one of P^T, dS^T (128-byte rows)
-  static constexpr int K_OFF = 0, V_OFF = KV_BYTES;
-  static constexpr int Q_OFF = 2 * KV_BYTES;      // stage s: Q at Q_OFF + 2 s Q_BYTES, dO after it
-  static constexpr int P_OFF = Q_OFF + NS * 2 * Q_BYTES;  // buffer p: P^T, then dS^T
-  static constexpr int VEC_OFF = P_OFF + NPB * 2 * P_BYTES;  // [2][2][64] floats: lse*log2e, D
+  static constexpr int K_OFF = 0, V_OFF = KV_BYTES;  // (V_OFF unused when VT)
+  static constexpr int Q_OFF = VT ? KV_BYTES : 2 * KV_BYTES;  // stage s: Q at Q_OFF + 2 s Q_BYTES, dO after it
+  static constexpr int V_LAND = Q_OFF + 2 * Q_BYTES;          // VT: V passes through stage 1
+  static constexpr int P_OFF = Q_OFF + NS * 2 * Q_BYTES;      // buffer p: P^T, then dS^T
+  static constexpr int VEC_OFF = P_OFF + NPB * 2 * P_BYTES;   // [2][2][64] floats: lse*log2e, D
   static constexpr int BAR_OFF = VEC_OFF + 2 * 2 * 64 * 4;
   static constexpr int SMEM = BAR_OFF + 256 + 1024;
-  static constexpr uint32_t TM_DK = 0, TM_DV = DC, TM_S = 256;  // S^T / dP^T buffer b: 256 + 128 b (+64)
+  // S^T / dP^T buffer b: TM_S + 128 b (+64); V (VT): 256 fp16 per key row packed in 128 columns
+  static constexpr uint32_t TM_DK = 0, TM_DV = DC, TM_V = 256, TM_S = VT ? 384 : 256;
+  static_assert(!VT || 2 * Q_BYTES == KV_BYTES, "V fits the second stage");
 };
+
+// tcgen05.mma with the A operand in TMEM (K-major: TMEM lane = row of A, each 32-bit column two
+// consecutive K elements): D[tmem] (+)= A[a_tmem] * B[smem desc]^T.
+__device__ __forceinline__ void tc_mma_f16_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                              uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
 
 // One dK/dV item: item = (((kb * B + b) * heads + head) * NCOL + col) * P + part, heads = KV (direct,
 // P = 1) or H (split).
@@ -483,7 +502,8 @@ __device__ __forceinline__ void dkdv_body(const CUtensorMap& tmKV, const CUtenso
                                           const float* __restrict__ dvec, uint16_t* __restrict__ dqkv, int64_t ld,
                                           int W, int* err, const SplitOut& so, int item, int B) {
   using C = DkDv<HD>;
-  constexpr int NS = C::NS, NPB = C::NPB, DC = C::DC, BQB = C::QB;
+  constexpr int NS = C::NS, NPB = C::NPB, DC = C::DC, BQB = C::QB, NSB = C::NSB;
+  constexpr bool VT = C::VT;
   static_assert(C::SMEM <= 232448, "shared memory");
   static_assert(C::SMEM > 232448 / 2, "one CTA per SM (512 TMEM columns each)");
   extern __shared__ uint8_t smem_raw[];
@@ -497,7 +517,9 @@ __device__ __forceinline__ void dkdv_body(const CUtensorMap& tmKV, const CUtenso
   uint64_t* pdone = pready + NPB;  // [NPB]
   uint64_t* dfull = pdone + NPB;
   uint64_t* vready = dfull + 1;    // [2] the lse / D vectors of an iteration are in shared memory
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(vready + 2);
+  uint64_t* vland = vready + 2;    // VT: V landed in stage 1's slot
+  uint64_t* vmoved = vland + 1;    // VT: V copied into TMEM (stage 1's slot is free again)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(vmoved + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   float* vec = reinterpret_cast<float*>(sm + C::VEC_OFF);
 
@@ -544,6 +566,8 @@ __device__ __forceinline__ void dkdv_body(const CUtensorMap& tmKV, const CUtenso
     }
     mbar_init(dfull, 1);
     for (int i = 0; i < 2; ++i) mbar_init(&vready[i], 128);
+    mbar_init(vland, 1);
+    mbar_init(vmoved, 4);  // one arrival per elementwise warp
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -560,15 +584,22 @@ __device__ __forceinline__ void dkdv_body(const CUtensorMap& tmKV, const CUtenso
       tma_prefetch_desc(&tmKV);
       tma_prefetch_desc(&tmQ);
       tma_prefetch_desc(&tmDO);
-      mbar_arrive_expect_tx(kvfull, 2 * C::KV_BYTES);
+      mbar_arrive_expect_tx(kvfull, (VT ? 1 : 2) * C::KV_BYTES);
+      if (VT) mbar_arrive_expect_tx(vland, C::KV_BYTES);
       for (int c = 0; c < C::NCH; ++c) {
         tma_load_3d(sm + C::K_OFF + c * BKV * 128, &tmKV, kvfull, (H + kvh) * HD + c * 64, k0, b);
-        tma_load_3d(sm + C::V_OFF + c * BKV * 128, &tmKV, kvfull, (H + KV + kvh) * HD + c * 64, k0, b);
+        if (VT) tma_load_3d(sm + C::V_LAND + c * BKV * 128, &tmKV, vland, (H + KV + kvh) * HD + c * 64, k0, b);
+        else tma_load_3d(sm + C::V_OFF + c * BKV * 128, &tmKV, kvfull, (H + KV + kvh) * HD + c * 64, k0, b);
       }
       int issued = 0;
+      bool v_out = !VT;  // stage 1's slot holds V until the elementwise warps have moved it
       for (int it = 0; it < n_it; ++it) {
         const int s = it % NS;
         if (it >= NS && !mbar_wait(&qempty[s], ((it / NS) & 1) ^ 1, abort_flag, err)) break;
+        if (!v_out && s == 1) {
+          if (!mbar_wait(vmoved, 0, abort_flag, err)) break;
+          v_out = true;
+        }
         const int g = g_of(it), hh = h_first + g / per_head, q0 = (qb_first + g % per_head) * BQB;
         uint8_t* qs = sm + C::Q_OFF + s * 2 * C::Q_BYTES;
         mbar_arrive_expect_tx(&qfull[s], 2 * C::Q_BYTES);
@@ -580,6 +611,7 @@ __device__ __forceinline__ void dkdv_body(const CUtensorMap& tmKV, const CUtenso
       }
       int dummy = 0;  // never leave with copies in flight
       mbar_wait(kvfull, 0, &dummy, err);
+      if (VT) mbar_wait(vland, 0, &dummy, err);
       for (int it = (issued > NS ? issued - NS : 0); it < issued; ++it)
         mbar_wait(&qfull[it % NS], (it / NS) & 1, &dummy, err);
     }
@@ -590,9 +622,10 @@ __device__ __forceinline__ void dkdv_body(const CUtensorMap& tmKV, const CUtenso
       bool ok = mbar_wait(kvfull, 0, abort_flag, err);
       const uint32_t k_addr = smem_u32(sm + C::K_OFF), v_addr = smem_u32(sm + C::V_OFF);
       auto scores = [&](int j) -> bool {
-        const int s = j % NS, bf = j & 1;
+        const int s = j % NS, bf = j % NSB;
         if (!mbar_wait(&qfull[s], (j / NS) & 1, abort_flag, err)) return false;
-        if (j >= 2 && !mbar_wait(&sfree[bf], ((j >> 1) & 1) ^ 1, abort_flag, err)) return false;
+        if (j >= NSB && !mbar_wait(&sfree[bf], ((j / NSB) & 1) ^ 1, abort_flag, err)) return false;
+        if (VT && j == 0 && !mbar_wait(vmoved, 0, abort_flag, err)) return false;  // V is in TMEM
         tc_fence_after();
         const uint32_t q_addr = smem_u32(sm + C::Q_OFF + s * 2 * C::Q_BYTES), do_addr = q_addr + C::Q_BYTES;
         const uint32_t ts = tmem + C::TM_S + 128 * bf;
@@ -601,8 +634,12 @@ __device__ __forceinline__ void dkdv_body(const CUtensorMap& tmKV, const CUtenso
           const uint32_t ka = (kk >> 2) * (BKV * 128) + (kk & 3) * 32, qa = (kk >> 2) * (BQB * 128) + (kk & 3) * 32;
           tc_mma_f16(ts, smem_desc_sw128(k_addr + ka, 16, 1024), smem_desc_sw128(q_addr + qa, 16, 1024), id_s,
                      kk > 0 ? 1u : 0u);
-          tc_mma_f16(ts + 64, smem_desc_sw128(v_addr + ka, 16, 1024), smem_desc_sw128(do_addr + qa, 16, 1024), id_s,
-                     kk > 0 ? 1u : 0u);
+          if (VT)  // 16 hd elements of V = 8 TMEM columns
+            tc_mma_f16_ta(ts + 64, tmem + C::TM_V + 8 * kk, smem_desc_sw128(do_addr + qa, 16, 1024), id_s,
+                          kk > 0 ? 1u : 0u);
+          else
+            tc_mma_f16(ts + 64, smem_desc_sw128(v_addr + ka, 16, 1024), smem_desc_sw128(do_addr + qa, 16, 1024), id_s,
+                       kk > 0 ? 1u : 0u);
         }
         tc_commit(&sfull[bf]);
         return true;
@@ -651,7 +688,32 @@ __device__ __forceinline__ void dkdv_body(const CUtensorMap& tmKV, const CUtenso
     };
     float vnext = n_it > 0 ? vec_load(0) : 0.0f;
     bool ok = true;
-    for (int j = 0; j < n_it; ++j) {
+    if (VT) {
+      // thread r copies key row r of V from stage 1's slot (128-byte swizzled chunks of 64 columns)
+      // into TMEM lane r: the 16-byte unit u of chunk c (columns 64 c + 8 u ..) is TMEM columns
+      // 32 c + 4 u .. + 3 (two fp16 per column)
+      ok = __all_sync(0xffffffffu, mbar_wait(vland, 0, abort_flag, err));
+      if (ok) {
+#pragma unroll 1
+        for (int c = 0; c < C::NCH; ++c) {
+          float w[32];
+          const uint8_t* row = sm + C::V_LAND + c * BKV * 128 + r * 128;
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const uint4 x = *reinterpret_cast<const uint4*>(row + ((u ^ (r & 7)) << 4));
+            w[4 * u] = __uint_as_float(x.x);
+            w[4 * u + 1] = __uint_as_float(x.y);
+            w[4 * u + 2] = __uint_as_float(x.z);
+            w[4 * u + 3] = __uint_as_float(x.w);
+          }
+          tmem_st32(tmem + lane_off + C::TM_V + 32 * c, w);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(vmoved);  // also after an abort: the waiters do not sit out their limit
+    }
+    for (int j = 0; ok && j < n_it; ++j) {
       const int q0 = (qb_first + g_of(j) % per_head) * BQB;
       float* lv = vec + (j & 1) * 2 * 64;  // [BQB] lse * log2e, then [BQB] D
       if (r < 2 * BQB) lv[r] = vnext;
@@ -662,10 +724,10 @@ __device__ __forceinline__ void dkdv_body(const CUtensorMap& tmKV, const CUtenso
       mbar_arrive(&vready[j & 1]);
       ok = __all_sync(0xffffffffu, mbar_wait(&vready[j & 1], (j >> 1) & 1, abort_flag, err));
       if (!ok) break;
-      ok = __all_sync(0xffffffffu, mbar_wait(&sfull[j & 1], (j >> 1) & 1, abort_flag, err));
+      ok = __all_sync(0xffffffffu, mbar_wait(&sfull[j % NSB], (j / NSB) & 1, abort_flag, err));
       if (!ok) break;
       tc_fence_after();
-      const uint32_t ts = tmem + lane_off + C::TM_S + 128 * (j & 1);
+      const uint32_t ts = tmem + lane_off + C::TM_S + 128 * (j % NSB);
       float sv[BQB], dp[BQB];
       if constexpr (BQB == 64) {
         tmem_ld64(ts, sv);
@@ -676,7 +738,7 @@ __device__ __forceinline__ void dkdv_body(const CUtensorMap& tmKV, const CUtenso
       }
       tc_fence_before();  // the score buffer may be overwritten once every warp has read it
       __syncwarp();
-      if (lane == 0) mbar_arrive(&sfree[j & 1]);
+      if (lane == 0) mbar_arrive(&sfree[j % NSB]);
 #pragma unroll
       for (int e = 0; e < BQB; ++e) {
         const int q = q0 + e;
