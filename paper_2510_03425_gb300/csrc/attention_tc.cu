@@ -835,19 +835,27 @@ __device__ __forceinline__ void dkdv_body(const CUtensorMap& tmKV, const CUtenso
 
 template <int HD>
 struct Dq {
+  // hd 256: dO lives in TMEM as the A operand of dP = dO V^T (as V does in the dK/dV kernel),
+  // freeing 64 KB for a second (K, V) stage; dO lands in that stage's slot once and the dS warps
+  // copy it row by row into TMEM before the loop.
+  static constexpr bool DT = HD == 256;
   static constexpr int QB = bwd_block<HD>();                      // keys per iteration
-  static constexpr int NS = HD == 256 ? 1 : (HD == 128 ? 3 : 4);  // (K_j, V_j) stages
+  static constexpr int NS = HD == 256 ? 2 : (HD == 128 ? 3 : 4);  // (K_j, V_j) stages
   static constexpr int NPB = 2;                                   // dS buffers
+  static constexpr int NSB = DT ? 1 : 2;                          // S / dP buffers in TMEM
   static constexpr int NCH = HD / 64;
   static constexpr int Q_BYTES = BQ * HD * 2;    // one of Q, dO
   static constexpr int K_BYTES = QB * HD * 2;    // one of K_j, V_j
   static constexpr int P_BYTES = BQ * 64 * 2;    // one dS buffer (128-byte rows)
-  static constexpr int Q_OFF = 0, DO_OFF = Q_BYTES;
-  static constexpr int K_OFF = 2 * Q_BYTES;      // stage s: K at K_OFF + 2 s K_BYTES, V after it
+  static constexpr int Q_OFF = 0, DO_OFF = Q_BYTES;  // (DO_OFF unused when DT)
+  static constexpr int K_OFF = DT ? Q_BYTES : 2 * Q_BYTES;  // stage s: K at K_OFF + 2 s K_BYTES, V after it
+  static constexpr int D_LAND = K_OFF + 2 * K_BYTES;        // DT: dO passes through stage 1
   static constexpr int P_OFF = K_OFF + NS * 2 * K_BYTES;
   static constexpr int BAR_OFF = P_OFF + NPB * P_BYTES;
   static constexpr int SMEM = BAR_OFF + 256 + 1024;
-  static constexpr uint32_t TM_DQ = 0, TM_S = 256;  // S / dP buffer b: 256 + 128 b (+64)
+  // S / dP buffer b: TM_S + 128 b (+64); dO (DT): 256 fp16 per query row packed in 128 columns
+  static constexpr uint32_t TM_DQ = 0, TM_DO = 256, TM_S = DT ? 384 : 256;
+  static_assert(!DT || 2 * K_BYTES == Q_BYTES, "dO fits the second stage");
 };
 
 // One dQ item: x = head * P + part, sequence b, query tile nqb - 1 - z (the longest first).
@@ -857,7 +865,8 @@ __device__ __forceinline__ void dq_body(const CUtensorMap& tmQ, const CUtensorMa
                                         const float* __restrict__ dvec, uint16_t* __restrict__ dqkv, int64_t ld,
                                         int W, int* err, const SplitOut& so, int x, int b, int z) {
   using C = Dq<HD>;
-  constexpr int NS = C::NS, NPB = C::NPB, BQB = C::QB;
+  constexpr int NS = C::NS, NPB = C::NPB, BQB = C::QB, NSB = C::NSB;
+  constexpr bool DT = C::DT;
   static_assert(C::SMEM <= 232448, "shared memory");
   static_assert(C::SMEM > 232448 / 2, "one CTA per SM (512 TMEM columns each)");
   extern __shared__ uint8_t smem_raw[];
@@ -870,7 +879,9 @@ __device__ __forceinline__ void dq_body(const CUtensorMap& tmQ, const CUtensorMa
   uint64_t* pready = sfree + 2;   // [NPB]
   uint64_t* pdone = pready + NPB; // [NPB]
   uint64_t* dfull = pdone + NPB;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(dfull + 1);
+  uint64_t* dland = dfull + 1;    // DT: dO landed in stage 1's slot
+  uint64_t* dmoved = dland + 1;   // DT: dO copied into TMEM (stage 1's slot is free again)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(dmoved + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -901,6 +912,8 @@ __device__ __forceinline__ void dq_body(const CUtensorMap& tmQ, const CUtensorMa
       mbar_init(&pdone[i], 1);
     }
     mbar_init(dfull, 1);
+    mbar_init(dland, 1);
+    mbar_init(dmoved, 4);  // one arrival per dS warp
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -917,15 +930,22 @@ __device__ __forceinline__ void dq_body(const CUtensorMap& tmQ, const CUtensorMa
       tma_prefetch_desc(&tmQ);
       tma_prefetch_desc(&tmKV);
       tma_prefetch_desc(&tmDO);
-      mbar_arrive_expect_tx(qfull, 2 * C::Q_BYTES);
+      mbar_arrive_expect_tx(qfull, (DT ? 1 : 2) * C::Q_BYTES);
+      if (DT) mbar_arrive_expect_tx(dland, C::Q_BYTES);
       for (int c = 0; c < C::NCH; ++c) {
         tma_load_3d(sm + C::Q_OFF + c * BQ * 128, &tmQ, qfull, h * HD + c * 64, q0, b);
-        tma_load_3d(sm + C::DO_OFF + c * BQ * 128, &tmDO, qfull, h * HD + c * 64, q0, b);
+        if (DT) tma_load_3d(sm + C::D_LAND + c * BQ * 128, &tmDO, dland, h * HD + c * 64, q0, b);
+        else tma_load_3d(sm + C::DO_OFF + c * BQ * 128, &tmDO, qfull, h * HD + c * 64, q0, b);
       }
       int issued = 0;
+      bool d_out = !DT;  // stage 1's slot holds dO until the dS warps have moved it
       for (int j = 0; j < nkb; ++j) {
         const int s = j % NS;
         if (j >= NS && !mbar_wait(&kempty[s], ((j / NS) & 1) ^ 1, abort_flag, err)) break;
+        if (!d_out && s == 1) {
+          if (!mbar_wait(dmoved, 0, abort_flag, err)) break;
+          d_out = true;
+        }
         uint8_t* ks = sm + C::K_OFF + s * 2 * C::K_BYTES;
         mbar_arrive_expect_tx(&kfull[s], 2 * C::K_BYTES);
         for (int c = 0; c < C::NCH; ++c) {
@@ -937,6 +957,7 @@ __device__ __forceinline__ void dq_body(const CUtensorMap& tmQ, const CUtensorMa
       }
       int dummy = 0;
       mbar_wait(qfull, 0, &dummy, err);
+      if (DT) mbar_wait(dland, 0, &dummy, err);
       for (int j = (issued > NS ? issued - NS : 0); j < issued; ++j)
         mbar_wait(&kfull[j % NS], (j / NS) & 1, &dummy, err);
     }
@@ -947,9 +968,10 @@ __device__ __forceinline__ void dq_body(const CUtensorMap& tmQ, const CUtensorMa
       bool ok = mbar_wait(qfull, 0, abort_flag, err);
       const uint32_t q_addr = smem_u32(sm + C::Q_OFF), do_addr = smem_u32(sm + C::DO_OFF);
       auto scores = [&](int j) -> bool {
-        const int s = j % NS, bf = j & 1;
+        const int s = j % NS, bf = j % NSB;
         if (!mbar_wait(&kfull[s], (j / NS) & 1, abort_flag, err)) return false;
-        if (j >= 2 && !mbar_wait(&sfree[bf], ((j >> 1) & 1) ^ 1, abort_flag, err)) return false;
+        if (j >= NSB && !mbar_wait(&sfree[bf], ((j / NSB) & 1) ^ 1, abort_flag, err)) return false;
+        if (DT && j == 0 && !mbar_wait(dmoved, 0, abort_flag, err)) return false;  // dO is in TMEM
         tc_fence_after();
         const uint32_t k_addr = smem_u32(sm + C::K_OFF + s * 2 * C::K_BYTES), v_addr = k_addr + C::K_BYTES;
         const uint32_t ts = tmem + C::TM_S + 128 * bf;
@@ -958,8 +980,12 @@ __device__ __forceinline__ void dq_body(const CUtensorMap& tmQ, const CUtensorMa
           const uint32_t qa = (kk >> 2) * (BQ * 128) + (kk & 3) * 32, ka = (kk >> 2) * (BQB * 128) + (kk & 3) * 32;
           tc_mma_f16(ts, smem_desc_sw128(q_addr + qa, 16, 1024), smem_desc_sw128(k_addr + ka, 16, 1024), id_s,
                      kk > 0 ? 1u : 0u);
-          tc_mma_f16(ts + 64, smem_desc_sw128(do_addr + qa, 16, 1024), smem_desc_sw128(v_addr + ka, 16, 1024), id_s,
-                     kk > 0 ? 1u : 0u);
+          if (DT)  // 16 hd elements of dO = 8 TMEM columns
+            tc_mma_f16_ta(ts + 64, tmem + C::TM_DO + 8 * kk, smem_desc_sw128(v_addr + ka, 16, 1024), id_s,
+                          kk > 0 ? 1u : 0u);
+          else
+            tc_mma_f16(ts + 64, smem_desc_sw128(do_addr + qa, 16, 1024), smem_desc_sw128(v_addr + ka, 16, 1024),
+                       id_s, kk > 0 ? 1u : 0u);
         }
         tc_commit(&sfull[bf]);
         return true;
@@ -998,8 +1024,31 @@ __device__ __forceinline__ void dq_body(const CUtensorMap& tmQ, const CUtensorMa
     const float l2 = row < S ? lse[li] * kLog2e : 0.0f;
     const float dr = row < S ? dvec[li] : 0.0f;
     bool ok = true;
-    for (int j = 0; j < nkb; ++j) {
-      ok = __all_sync(0xffffffffu, mbar_wait(&sfull[j & 1], (j >> 1) & 1, abort_flag, err));
+    if (DT) {
+      // thread r copies query row r of dO from stage 1's slot into TMEM lane r (as V in dK/dV)
+      ok = __all_sync(0xffffffffu, mbar_wait(dland, 0, abort_flag, err));
+      if (ok) {
+#pragma unroll 1
+        for (int c = 0; c < C::NCH; ++c) {
+          float w[32];
+          const uint8_t* src = sm + C::D_LAND + c * BQ * 128 + r * 128;
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const uint4 x = *reinterpret_cast<const uint4*>(src + ((u ^ (r & 7)) << 4));
+            w[4 * u] = __uint_as_float(x.x);
+            w[4 * u + 1] = __uint_as_float(x.y);
+            w[4 * u + 2] = __uint_as_float(x.z);
+            w[4 * u + 3] = __uint_as_float(x.w);
+          }
+          tmem_st32(tmem + lane_off + C::TM_DO + 32 * c, w);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(dmoved);  // also after an abort: the waiters do not sit out their limit
+    }
+    for (int j = 0; ok && j < nkb; ++j) {
+      ok = __all_sync(0xffffffffu, mbar_wait(&sfull[j % NSB], (j / NSB) & 1, abort_flag, err));
       if (!ok) break;
       if (j >= NPB) {
         const int i = j - NPB;
@@ -1007,7 +1056,7 @@ __device__ __forceinline__ void dq_body(const CUtensorMap& tmQ, const CUtensorMa
         if (!ok) break;
       }
       tc_fence_after();
-      const uint32_t ts = tmem + lane_off + C::TM_S + 128 * (j & 1);
+      const uint32_t ts = tmem + lane_off + C::TM_S + 128 * (j % NSB);
       uint8_t* drow = sm + C::P_OFF + (j % NPB) * C::P_BYTES + r * 128;
       const int k0 = kblock(j) * BQB;
       {
@@ -1019,6 +1068,9 @@ __device__ __forceinline__ void dq_body(const CUtensorMap& tmQ, const CUtensorMa
           tmem_ld32(ts, sv);
           tmem_ld32(ts + 64, dp);
         }
+        tc_fence_before();  // the score buffer may be overwritten once every warp has read it
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sfree[j % NSB]);
 #pragma unroll
         for (int e = 0; e < BQB; ++e) {
           const int key = k0 + e;
@@ -1035,10 +1087,7 @@ __device__ __forceinline__ void dq_body(const CUtensorMap& tmQ, const CUtensorMa
       fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(&sfree[j & 1]);
-        mbar_arrive(&pready[j % NPB]);
-      }
+      if (lane == 0) mbar_arrive(&pready[j % NPB]);
     }
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(dfull, 0, abort_flag, err));
     tc_fence_after();
