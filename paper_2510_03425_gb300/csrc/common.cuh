@@ -252,6 +252,31 @@ MEBP_DEV float4 ld_dsmem_f4(uint32_t addr) {
 MEBP_DEV void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 MEBP_DEV void griddep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
+// ------------------------------------------------------------------------------------ activations
+// Gated-MLP activations (SiLU, or GELU with the tanh approximation) and their derivatives; the GLU
+// kernels and the gate|up GEMM's fused epilogue use these same functions.  tanh is the hardware
+// approximation (tanh.approx.f32, relative error about 2^-11, the size of the fp16 rounding that
+// the stored activations get anyway): in the fused epilogue the activation is on the GEMM's path.
+MEBP_DEV float tanh_fast(float x) {
+  float y;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+MEBP_DEV float act_f(float x, int act) {
+  if (act == MEBP_ACT_SILU) return x / (1.0f + __expf(-x));
+  const float k0 = 0.7978845608028654f;  // sqrt(2/pi)
+  return 0.5f * x * (1.0f + tanh_fast(k0 * (x + 0.044715f * x * x * x)));
+}
+MEBP_DEV float act_grad(float x, int act) {
+  if (act == MEBP_ACT_SILU) {
+    const float sg = 1.0f / (1.0f + __expf(-x));
+    return sg * (1.0f + x * (1.0f - sg));
+  }
+  const float k0 = 0.7978845608028654f;
+  const float th = tanh_fast(k0 * (x + 0.044715f * x * x * x));
+  return 0.5f * (1.0f + th) + 0.5f * x * (1.0f - th * th) * k0 * (1.0f + 3.0f * 0.044715f * x * x);
+}
+
 // ------------------------------------------------------------------------------------ misc
 MEBP_DEV float warp_sum(float v) {
 #pragma unroll

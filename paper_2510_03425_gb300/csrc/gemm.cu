@@ -90,6 +90,10 @@ struct Params {
   float* zt;               // EPI_LSE: target logit [M]
   const float* lse;        // EPI_CEGRAD: [M]
   const float* ce_w;       // EPI_CEGRAD: device scalar weight of a valid row
+  void* C2;                // EPI_GLU: gate and up outputs (fp16), or null
+  int64_t ldc2;
+  int glu_half;            // EPI_GLU: rows of the gate half of the fused weight
+  int act;                 // EPI_GLU: activation
   int* err;
 };
 
@@ -154,7 +158,9 @@ __device__ __forceinline__ void copy_lora_b(const Params& p, int e, int n0, uint
   constexpr int NW = 8 / TPR;
   const uint4 zero = make_uint4(0, 0, 0, 0);
   if (!TRANS) {  // K-major: row r, chunk j = 8 columns of the rank axis
-    const int r = t / TPR, h = t % TPR, n = n0 + r;
+    const int r = t / TPR, h = t % TPR;
+    // EPI_GLU: tile rows 0-127 are gate rows n0/2 + r, rows 128-255 the up rows glu_half + n0/2 + r - 128
+    const int n = p.epi != EPI_GLU ? n0 + r : (r < BN / 2 ? n0 / 2 + r : p.glu_half + n0 / 2 + r - BN / 2);
 #pragma unroll
     for (int w = 0; w < NW; ++w) {
       const int j = NW * h + w;
@@ -239,6 +245,64 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
       if (has_t) p.zt[row] = zt;
     }
     return;
+  }
+
+  if constexpr (NACC == 2) {
+    if (p.epi == EPI_GLU) {
+      // The warp's accumulator holds the gate (columns 0-127) and up (128-255) pre-activations of
+      // hidden units j0 .. j0 + 127, j0 = n0 / 2.  Per round of 32 units: gate and up rounded to
+      // fp16 (the values the unfused path stores), m = act(gate) up from those, as the GLU kernel
+      // computes it (bit-identical), all three staged at 64 bytes per row (16-byte chunk c of row
+      // r at chunk c ^ ((r >> 1) & 3): conflict-free) and written out 8 rows per instruction.
+      const int j0 = n0 / 2, row0 = row - lane;
+      const uint32_t tacc = tmem + (static_cast<uint32_t>(32 * q) << 16) + 256 * acc;
+      // slots of 2 KB in the staging area: m at +0, gate at +2048, up at +4096
+      const int nout = p.C2 ? 3 : 1;
+      uint32_t bad = 0;
+#pragma unroll 1
+      for (int u0 = 0; u0 < 128; u0 += 32) {
+        const int j = j0 + u0;
+        if (j >= p.glu_half) break;  // warp-uniform
+        float gv[32], uv[32];
+        tmem_ld32(tacc + u0, gv);
+        tmem_ld32(tacc + 128 + u0, uv);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {  // 8 units per 16-byte chunk
+          uint32_t mo[4], go[4], uo[4];
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const int e = 8 * c + 2 * k;
+            go[k] = pack_half2(gv[e], gv[e + 1]);
+            uo[k] = pack_half2(uv[e], uv[e + 1]);
+            mo[k] = pack_half2(act_f(h2_lo(go[k]), p.act) * h2_lo(uo[k]), act_f(h2_hi(go[k]), p.act) * h2_hi(uo[k]));
+            if (row_ok) bad |= h2_nonfinite(mo[k]) | (p.C2 ? h2_nonfinite(go[k]) | h2_nonfinite(uo[k]) : 0u);
+          }
+          const int off = lane * 64 + ((c ^ ((lane >> 1) & 3)) << 4);
+          *reinterpret_cast<uint4*>(stage + off) = make_uint4(mo[0], mo[1], mo[2], mo[3]);
+          if (p.C2) {
+            *reinterpret_cast<uint4*>(stage + 2048 + off) = make_uint4(go[0], go[1], go[2], go[3]);
+            *reinterpret_cast<uint4*>(stage + 4096 + off) = make_uint4(uo[0], uo[1], uo[2], uo[3]);
+          }
+        }
+        __syncwarp();
+        const int c = lane & 3;
+#pragma unroll 1
+        for (int o = 0; o < nout; ++o) {
+          uint16_t* dst = o == 0 ? static_cast<uint16_t*>(p.C) + j
+                                 : static_cast<uint16_t*>(p.C2) + (o == 1 ? j : p.glu_half + j);
+          const int64_t ld = o == 0 ? p.ldc : p.ldc2;
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int rr = 8 * i + (lane >> 2), r = row0 + rr;
+            const uint4 v = *reinterpret_cast<const uint4*>(stage + o * 2048 + rr * 64 + ((c ^ ((rr >> 1) & 3)) << 4));
+            if (r < p.M) *reinterpret_cast<uint4*>(dst + static_cast<int64_t>(r) * ld + 8 * c) = v;
+          }
+        }
+        __syncwarp();  // the slots are rewritten by the next round
+      }
+      if (bad) flag_error(p.err, kErrNonFinite);
+      return;
+    }
   }
 
   // EPI_F16, EPI_CEGRAD (fp16 rows of 128 bytes per round) and EPI_F32 (fp32, 256 bytes)
@@ -460,7 +524,13 @@ __global__ void __launch_bounds__(Warps<NACC>::THREADS, 1)
         const int s = it % TSTG, kt = kt0 + it;
         uint8_t* st = smem + s * Ly::T_STRIDE;
         mbar_arrive_expect_tx(&wfull[s], P_BYTES + S_BYTES);
-        if (!TRANS) {
+        if (!TRANS && p.epi == EPI_GLU) {  // 128 gate rows, then the matching 128 up rows
+          const int j0 = n0 / 2;
+          tma_load_2d(st + Ly::P_OFF, &tmP, &wfull[s], kt * (BK / 2), j0);
+          tma_load_2d(st + Ly::P_OFF + (BN / 2) * (BK / 2), &tmP, &wfull[s], kt * (BK / 2), p.glu_half + j0);
+          tma_load_2d(st + Ly::S_OFF, &tmS, &wfull[s], j0, kt);
+          tma_load_2d(st + Ly::S_OFF + BN, &tmS, &wfull[s], p.glu_half + j0, kt);  // BN / 2 fp16 scales
+        } else if (!TRANS) {
           tma_load_2d(st + Ly::P_OFF, &tmP, &wfull[s], kt * (BK / 2), n0);  // packed [N, K/2]
           tma_load_2d(st + Ly::S_OFF, &tmS, &wfull[s], n0, kt);             // scales [K/64, N]
         } else {
@@ -697,6 +767,8 @@ int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st) {
   using namespace gemm;
   if (g.M <= 0 || g.N <= 0) return MEBP_OK;
   if (g.K % 64 || g.N % 64 || g.K <= 0) return MEBP_ERR_INVALID_ARG;
+  const bool glu = g.epi == EPI_GLU;
+  if (glu && (g.trans || g.glu_half <= 0 || g.glu_half % 128 || g.N != 2 * g.glu_half)) return MEBP_ERR_UNSUPPORTED;
   // Two 128-row accumulators per CTA (half the decode work per flop) once 256-row tiles alone give
   // at least two waves on the 152 SMs (large M, or a large N such as the LM head).
   const int64_t tiles_n256 = (g.N + BN - 1) / BN;
@@ -704,6 +776,7 @@ int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st) {
   const int bm = BM * nacc;
   // Few tokens and a short K: 128 x 256 tiles would leave most SMs idle; narrow 128 x 64 tiles
   // instead of a K split (a long K keeps the split: its serial chain would dominate).
+  if (glu && nacc != 2) return MEBP_ERR_UNSUPPORTED;  // the fused GLU epilogue is the two-accumulator one
   if (nacc == 1 && (g.epi == EPI_F32 || g.epi == EPI_F16) && g.K <= 2560 &&
       ((g.N + BN - 1) / BN) * ((g.M + BM - 1) / BM) <= 76)
     return launch_dequant_gemm_narrow(g, st);
@@ -716,11 +789,13 @@ int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st) {
     return rc;
   if (!g.trans) {
     // packed [N, K/2] bytes, scales [K/64, N] (pitch = scale_pitch elements)
-    if ((rc = make_tmap_2d(&tP, g.qpack, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, g.K / 2, g.N, g.K / 2, 32, BN,
+    // (EPI_GLU: two boxes of 128 rows per tile, the gate rows and the matching up rows)
+    const uint32_t wbox = glu ? BN / 2 : BN;
+    if ((rc = make_tmap_2d(&tP, g.qpack, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, g.K / 2, g.N, g.K / 2, 32, wbox,
                            CU_TENSOR_MAP_SWIZZLE_NONE)))
       return rc;
-    if ((rc = make_tmap_2d(&tS, g.scales, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, g.N, g.K / 64, g.scale_pitch * 2, BN, 1,
-                           CU_TENSOR_MAP_SWIZZLE_NONE)))
+    if ((rc = make_tmap_2d(&tS, g.scales, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, g.N, g.K / 64, g.scale_pitch * 2, wbox,
+                           1, CU_TENSOR_MAP_SWIZZLE_NONE)))
       return rc;
   } else {
     // packed [K, N/2] bytes, scales [N/64, K]
@@ -763,6 +838,10 @@ int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st) {
   p.zt = g.zt;
   p.lse = g.lse;
   p.ce_w = g.ce_w;
+  p.C2 = g.C2;
+  p.ldc2 = g.ldc2;
+  p.glu_half = g.glu_half;
+  p.act = g.act;
   p.err = g.err;
 
   const int tiles_n = static_cast<int>((g.N + BN - 1) / BN), tiles_m = static_cast<int>((g.M + bm - 1) / bm);

@@ -76,7 +76,10 @@ inline cudaError_t launch_k_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 bl
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
-enum GemmEpi { EPI_F16 = 0, EPI_F32 = 1, EPI_LSE = 2, EPI_CEGRAD = 3 };
+// EPI_GLU (forward, two accumulators): the weight is the fused [gate; up] matrix of 2 glu_half rows;
+// 256-column tile t holds gate rows 128 t .. 128 t + 127 and the matching up rows, and the epilogue
+// writes m = act(gate) * up (fp16, C [M, glu_half]) and, with C2, gate and up (fp16, [M, 2 glu_half]).
+enum GemmEpi { EPI_F16 = 0, EPI_F32 = 1, EPI_LSE = 2, EPI_CEGRAD = 3, EPI_GLU = 4 };
 
 struct GemmArgs {
   bool trans = false;            // false: C = A deq(W)^T (W [N,K]);  true: C = A deq(W) (W [K,N])
@@ -105,6 +108,10 @@ struct GemmArgs {
   float* zt = nullptr;
   const float* lse = nullptr;
   const float* ce_w = nullptr;   // EPI_CEGRAD: device scalar weight of a valid row
+  void* C2 = nullptr;            // EPI_GLU: gate and up as well (fp16 [M, 2 glu_half]), or null
+  int64_t ldc2 = 0;
+  int glu_half = 0;              // EPI_GLU: rows of the gate (= of the up) half of the weight
+  int act = 0;                   // EPI_GLU: MEBP_ACT_*
   int* err = nullptr;
 };
 

@@ -322,6 +322,7 @@ double gemm_bytes(const GemmArgs& g) {
   double b = 2.0 * M * K + N * K / 2.0 + 2.0 * N * (K / 64.0);
   if (g.epi == EPI_F32) b += 4.0 * M * N;
   else if (g.epi == EPI_F16 || g.epi == EPI_CEGRAD) b += 2.0 * M * N;
+  else if (g.epi == EPI_GLU) b += M * N + (g.C2 ? 2.0 * M * N : 0.0);  // m (N / 2 columns), gate and up
   else b += 8.0 * M * g.nparts / 2.0;  // LSE partials
   if (g.R) b += 4.0 * M * N;
   if (g.Ax) b += 2.0 * M * g.kx + 2.0 * N * g.kx;
@@ -373,8 +374,11 @@ const float2* layer_rope(const mebp_ctx* c, int layer) {
 // y = F(x) for one block.  with_down == false stops after the MLP activation (what the
 // backward consumes), so y is not produced; the Gemma3 block still runs the down projection,
 // whose output the backward of its sandwich norm reads.
+// keep_gu: the gate and up pre-activations are stored in the set (a backward reads them from it); a
+// forward whose intermediates are recomputed before any backward can skip them.
 int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, const mebp_lora* lora, const float* x,
-                  float* y, int B, int Sq, bool with_down, cudaStream_t st, const Shadow* sh = nullptr) {
+                  float* y, int B, int Sq, bool with_down, cudaStream_t st, const Shadow* sh = nullptr,
+                  bool keep_gu = true) {
   Acts& A = c->act[set];
   const int64_t T = static_cast<int64_t>(B) * Sq;
   const int D = c->D, I = c->I;
@@ -444,9 +448,18 @@ int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, 
     });
     g.Ax = A.us[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = A.sh->B_cat[LIN_GU]; g.ldbx = lg.kxp;
   }
-  g.epi = EPI_F16; g.C = A.gu; g.ldc = lg.N;
-  if ((rc = run_gemm(c, g, st, "gate_up"))) return rc;
-  KP(c, KK_GLU_FWD, 6.0 * T * I, 0, st, [&] { launch_glu_fwd(A.gu, T, I, c->cfg.act, A.m, c->d_err, st); });
+  // From 2048 tokens the gate|up GEMM's epilogue applies the activation itself (EPI_GLU, the
+  // two-accumulator kernel): it writes m and, when a backward will read them, gate and up.
+  const bool fuse_glu = T >= 2048 && I % 128 == 0 && lg.N == 2 * I;
+  if (fuse_glu) {
+    g.epi = EPI_GLU; g.C = A.m; g.ldc = I; g.C2 = keep_gu ? A.gu : nullptr; g.ldc2 = lg.N; g.glu_half = I;
+    g.act = c->cfg.act;
+    if ((rc = run_gemm(c, g, st, "gate_up"))) return rc;
+  } else {
+    g.epi = EPI_F16; g.C = A.gu; g.ldc = lg.N;
+    if ((rc = run_gemm(c, g, st, "gate_up"))) return rc;
+    KP(c, KK_GLU_FWD, 6.0 * T * I, 0, st, [&] { launch_glu_fwd(A.gu, T, I, c->cfg.act, A.m, c->d_err, st); });
+  }
   const Lin& ld = c->lin[LIN_DOWN];
   if (ld.kx)
     KP(c, KK_LORA_SKINNY, bytes_skinny(T, I, ld.kx, ld.kxp), 2.0 * T * I * ld.kx, st, [&] {
@@ -468,7 +481,7 @@ int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, 
       if ((rc = run_gemm(c, g, st, "down"))) return rc;
     }
   }
-  A.layer = layer;
+  A.layer = (fuse_glu && !keep_gu) ? -1 : layer;  // without gate and up the set cannot serve a backward
   A.x = x;
   A.T = T;
   return cuda_check(c, "block forward");
@@ -1339,7 +1352,9 @@ static int lora_step_body(mebp_ctx* c, const mebp_model_weights* model, const me
     }
     std::snprintf(rname, sizeof(rname), "f_%d", i);
     nvtxRangePushA(rname);
-    rc = block_forward(c, i % c->nsets, i, &model->blocks[i], &lora[i], xin, yout, B, Sq, true, st, &c->layer_sh[i]);
+    // only the last nsets blocks' intermediates survive to their backward; the others are recomputed
+    rc = block_forward(c, i % c->nsets, i, &model->blocks[i], &lora[i], xin, yout, B, Sq, true, st, &c->layer_sh[i],
+                       i >= L - c->nsets);
     nvtxRangePop();
     if (rc) return rc;
     if (spill && i + 1 < L) spill_out(i + 1);

@@ -350,20 +350,6 @@ void launch_add_norm(const float* dn, const float* h1, const float* gpf, int64_t
 }
 
 // ------------------------------------------------------------------------------------ gated MLP
-__device__ __forceinline__ float act_f(float x, int act) {
-  if (act == MEBP_ACT_SILU) return x / (1.0f + __expf(-x));
-  const float k0 = 0.7978845608028654f;  // sqrt(2/pi)
-  return 0.5f * x * (1.0f + tanhf(k0 * (x + 0.044715f * x * x * x)));
-}
-__device__ __forceinline__ float act_grad(float x, int act) {
-  if (act == MEBP_ACT_SILU) {
-    const float sg = 1.0f / (1.0f + __expf(-x));
-    return sg * (1.0f + x * (1.0f - sg));
-  }
-  const float k0 = 0.7978845608028654f;
-  const float th = tanhf(k0 * (x + 0.044715f * x * x * x));
-  return 0.5f * (1.0f + th) + 0.5f * x * (1.0f - th * th) * k0 * (1.0f + 3.0f * 0.044715f * x * x);
-}
 
 // m = act(g) * u; gu row = [g (I) | u (I)].  8 elements per thread.
 // A product outside the fp16 range (or NaN) sets MEBP_ERR_NONFINITE in *err.

@@ -65,6 +65,28 @@ def _small():
     return dims, blocks, E, gf, loras, synth.token_ids(dims)
 
 
+def test_step_at_2048_tokens_matches_oracle():
+    """The large-token path of the step: from 2048 tokens the gate|up GEMM applies the gated
+    activation in its epilogue (and skips storing gate and up for blocks that are recomputed
+    before their backward), the fused GEMMs use two accumulators and the LoRA-gradient
+    reductions run on the tensor cores; four blocks, rank 16 on all seven linears."""
+    dims = synth.tiny(hidden=256, n_heads=4, n_kv_heads=2, head_dim=64, intermediate=512, n_layers=4, vocab=2048,
+                      batch=2, seq=1024, rank=16, alpha=32.0, targets=synth.TARGETS)
+    blocks = dense_blocks(dims)
+    E, gf = synth.embedding(dims)
+    loras = [synth.lora_weights(dims, i) for i in range(dims.n_layers)]
+    ids = synth.token_ids(dims)
+    ctx, model = build(dims, blocks, E, gf)
+    ls = LoraSet(loras)
+    loss = step(ctx, model, ls, to_gpu(ids))
+    lo, go = OM.mebp_backpropagation(OM.PackedModel.compress(blocks, E, gf), loras, ids, dims)
+    assert abs(loss - lo) < 1e-3, (loss, lo)
+    for i in range(dims.n_layers):
+        for n, (dA, dB) in go[i].items():
+            a, b = ls.grads[i][n]
+            assert rel_fro(np_of(a), dA) < 2e-2 and rel_fro(np_of(b), dB) < 2e-2, (i, n)
+
+
 def test_small_model_step_matches_oracle():
     dims, blocks, E, gf, loras, ids = _small()
     ctx, model = build(dims, blocks, E, gf)
