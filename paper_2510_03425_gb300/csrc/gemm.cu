@@ -319,40 +319,38 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
   for (int rd = 0; rd < COLS / 64; ++rd) {
     const int c0 = cbase + 64 * rd;
     if (c0 >= p.N) break;  // warp-uniform (N is a multiple of 64)
-    float v[64];
-    {
-      float lo[32], hi[32];
-      tmem_ld32(tbase + 64 * rd, lo);
-      tmem_ld32(tbase + 64 * rd + 32, hi);
+    // ---- phase 1: this thread's row into the slot, 32 columns at a time (registers)
+#pragma unroll 1
+    for (int hh = 0; hh < 2; ++hh) {
+      float v[32];
+      tmem_ld32(tbase + 64 * rd + 32 * hh, v);
+      if (f32) {
+        uint8_t* srow = stage + lane * 256;
 #pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        v[i] = lo[i];
-        v[32 + i] = hi[i];
-      }
-    }
-    // ---- phase 1: this thread's row into the slot
-    if (f32) {
-      uint8_t* srow = stage + lane * 256;
-#pragma unroll
-      for (int j = 0; j < 16; ++j)
-        *reinterpret_cast<float4*>(srow + (((j & 8) | ((j ^ lane) & 7)) << 4)) =
-            make_float4(p.alpha * v[4 * j], p.alpha * v[4 * j + 1], p.alpha * v[4 * j + 2], p.alpha * v[4 * j + 3]);
-    } else {
-      if (ce) {
-#pragma unroll
-        for (int i = 0; i < 64; ++i) {
-          float a = (c0 + i < p.n_valid) ? __expf(v[i] - lse) * cw : 0.0f;
-          if (c0 + i == tl) a -= cw;
-          v[i] = a;
+        for (int jj = 0; jj < 8; ++jj) {
+          const int j = 8 * hh + jj;
+          *reinterpret_cast<float4*>(srow + (((j & 8) | ((j ^ lane) & 7)) << 4)) =
+              make_float4(p.alpha * v[4 * jj], p.alpha * v[4 * jj + 1], p.alpha * v[4 * jj + 2], p.alpha * v[4 * jj + 3]);
         }
-      }
-      uint8_t* srow = stage + lane * 128;
+      } else {
+        if (ce) {
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const uint4 o = make_uint4(pack_half2(v[8 * j], v[8 * j + 1]), pack_half2(v[8 * j + 2], v[8 * j + 3]),
-                                   pack_half2(v[8 * j + 4], v[8 * j + 5]), pack_half2(v[8 * j + 6], v[8 * j + 7]));
-        if (!ce && row_ok) bad |= h2_nonfinite(o.x) | h2_nonfinite(o.y) | h2_nonfinite(o.z) | h2_nonfinite(o.w);
-        *reinterpret_cast<uint4*>(srow + (((j ^ lane) & 7) << 4)) = o;
+          for (int i = 0; i < 32; ++i) {
+            const int col = c0 + 32 * hh + i;
+            float a = (col < p.n_valid) ? __expf(v[i] - lse) * cw : 0.0f;
+            if (col == tl) a -= cw;
+            v[i] = a;
+          }
+        }
+        uint8_t* srow = stage + lane * 128;
+#pragma unroll
+        for (int jj = 0; jj < 4; ++jj) {
+          const int j = 4 * hh + jj;
+          const uint4 o = make_uint4(pack_half2(v[8 * jj], v[8 * jj + 1]), pack_half2(v[8 * jj + 2], v[8 * jj + 3]),
+                                     pack_half2(v[8 * jj + 4], v[8 * jj + 5]), pack_half2(v[8 * jj + 6], v[8 * jj + 7]));
+          if (!ce && row_ok) bad |= h2_nonfinite(o.x) | h2_nonfinite(o.y) | h2_nonfinite(o.z) | h2_nonfinite(o.w);
+          *reinterpret_cast<uint4*>(srow + (((j ^ lane) & 7) << 4)) = o;
+        }
       }
     }
     __syncwarp();
