@@ -873,6 +873,11 @@ def main():
         print(json.dumps(per_block(args, d)), flush=True)
         return
 
+    if d.vocab == 0:  # a single block without a vocabulary: parity workload of the GPU tests
+        raise SystemExit(f"preset {args.config} ({workload_name(d)}) has no vocabulary and no training step to "
+                         "time: it is the single-block parity case of tests/test_gpu_block.py (--block-only and "
+                         "--gemm-bench take it)")
+
     if args.impl == "reference":
         # the CPU oracle as it stands, on the host cores: each step one bounded sample of the
         # workload, its throughput extrapolated to the whole step (see OracleSample)
