@@ -168,7 +168,8 @@ int64_t mebp_workspace_bytes(const mebp_ctx* ctx);
  *   MEBP_WS_ATTN_SPLIT  fp32 partials of the split attention backward (small grids)
  *   MEBP_WS_LMHEAD      LM-head + CE buffers (one vocabulary chunk of the CE gradient)
  *   MEBP_WS_LORA_SHADOW fp16 operand copies of the LoRA masters (every block)
- *   MEBP_WS_OTHER       RoPE tables, device scalars, error word, reduction scratch
+ *   MEBP_WS_OTHER       RoPE tables, device scalars, error word, reduction scratch, the fp32
+ *                       partials of fused GEMMs split over K through memory
  *   MEBP_WS_HOST_CKPT   pinned host checkpoints (spilling)
  * bytes has MEBP_WS_N entries; n_sets may be NULL. */
 enum {

@@ -23,6 +23,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <cstdint>
 
 #include "dequant.cuh"
 #include "kernels.h"
@@ -96,6 +97,8 @@ struct Params {
   int64_t ldc2;
   int glu_half;            // EPI_GLU: rows of the gate half of the fused weight
   int act;                 // EPI_GLU: activation
+  int64_t zstride;         // > 0: K split through memory (no cluster): CTA z stores its fp32 partial
+                           // tile with the EPI_F32 epilogue at C + z * zstride
   int* err;
 };
 
@@ -249,20 +252,24 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
     return;
   }
 
-  if constexpr (NACC == 2) {
+  {
     if (p.epi == EPI_GLU) {
-      // The warp's accumulator holds the gate (columns 0-127) and up (128-255) pre-activations of
-      // hidden units j0 .. j0 + 127, j0 = n0 / 2.  Per round of 32 units: gate and up rounded to
-      // fp16 (the values the unfused path stores), m = act(gate) up from those, as the GLU kernel
-      // computes it (bit-identical), all three staged at 64 bytes per row (16-byte chunk c of row
-      // r at chunk c ^ ((r >> 1) & 3): conflict-free) and written out 8 rows per instruction.
+      // The accumulator holds the gate (columns 0-127) and up (128-255) pre-activations of hidden
+      // units j0 .. j0 + 127, j0 = n0 / 2.  NACC = 2: the warp takes all 128 units of its
+      // accumulator; NACC = 1: column group cg takes units 32 cg .. +31 (gate and up columns of
+      // the same units, not the group's own 64 columns).  Per round of 32 units: gate and up
+      // rounded to fp16 (the values the unfused path stores), m = act(gate) up from those, as the
+      // GLU kernel computes it (bit-identical), all three staged at 64 bytes per row (16-byte chunk
+      // c of row r at chunk c ^ ((r >> 1) & 3): conflict-free) and written out 8 rows per
+      // instruction.
       const int j0 = n0 / 2, row0 = row - lane;
+      const int u_beg = col0 / 2, u_end = u_beg + COLS / 2;
       const uint32_t tacc = tmem + (static_cast<uint32_t>(32 * q) << 16) + 256 * acc;
       // slots of 2 KB in the staging area: m at +0, gate at +2048, up at +4096
       const int nout = p.C2 ? 3 : 1;
       uint32_t bad = 0;
 #pragma unroll 1
-      for (int u0 = 0; u0 < 128; u0 += 32) {
+      for (int u0 = u_beg; u0 < u_end; u0 += 32) {
         const int j = j0 + u0;
         if (j >= p.glu_half) break;  // warp-uniform
         float gv[32], uv[32];
@@ -356,7 +363,7 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
     __syncwarp();
     // ---- phase 2: whole lines out (rows past M skipped)
     if (f32) {
-      float* C = static_cast<float*>(p.C);
+      float* C = static_cast<float*>(p.C) + blockIdx.z * p.zstride;
       const int c = lane & 15;
 #pragma unroll 4
       for (int i = 0; i < 16; ++i) {
@@ -451,6 +458,38 @@ __device__ __forceinline__ void split_reduce(const Params& p, const uint8_t* sme
   }
 }
 
+// A K split through memory: partial tiles [S][M][N] (fp32, pitch N, split z at z * zstride) are
+// summed in split order (deterministic) and given the epilogue the split replaced: C = alpha *
+// sum (+ R, which may alias C) in fp32, or the sum rounded to fp16 with the overflow check.  One
+// thread per 4 columns.
+__global__ void ksplit_sum_kernel(const float* __restrict__ part, int S, int64_t zstride, int M, int N, float alpha,
+                                  const float* R, int64_t ldr, void* C, int64_t ldc, int f16, int* err) {
+  griddep_wait();  // the partials come from the GEMM right before
+  griddep_launch();
+  const int nq = N / 4;
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= static_cast<int64_t>(M) * nq) return;
+  const int64_t row = i / nq, col = 4 * (i % nq);
+  const float* src = part + row * N + col;
+  float4 s = *reinterpret_cast<const float4*>(src);
+  for (int z = 1; z < S; ++z) {
+    const float4 v = *reinterpret_cast<const float4*>(src + z * zstride);
+    s.x += v.x; s.y += v.y; s.z += v.z; s.w += v.w;
+  }
+  if (f16) {
+    const uint2 o = make_uint2(pack_half2(s.x, s.y), pack_half2(s.z, s.w));
+    if (h2_nonfinite(o.x) | h2_nonfinite(o.y)) flag_error(err, kErrNonFinite);
+    *reinterpret_cast<uint2*>(static_cast<uint16_t*>(C) + row * ldc + col) = o;
+  } else {
+    float4 o = make_float4(alpha * s.x, alpha * s.y, alpha * s.z, alpha * s.w);
+    if (R) {
+      const float4 rr = *reinterpret_cast<const float4*>(R + row * ldr + col);
+      o.x += rr.x; o.y += rr.y; o.z += rr.z; o.w += rr.w;
+    }
+    *reinterpret_cast<float4*>(static_cast<float*>(C) + row * ldc + col) = o;
+  }
+}
+
 // ---------------------------------------------------------------------------------- kernel
 // Launched with programmatic stream serialization: the prologue and the weight loads and decodes
 // of the first ring slots overlap the previous kernel; everything that reads an activation or
@@ -489,7 +528,7 @@ __global__ void __launch_bounds__(Warps<NACC>::THREADS, 1)
   const int kt0 = blockIdx.z * p.kt_split;
   const int kt1 = min(num_k, kt0 + p.kt_split);
   const int num_main = max(0, kt1 - kt0);
-  const bool split = gridDim.z > 1;  // NACC == 1 only (host)
+  const bool split = gridDim.z > 1 && p.zstride == 0;  // cluster split: NACC == 1 only (host)
   const bool last_split = blockIdx.z == gridDim.z - 1;
   const int num_x = last_split ? (p.kx_steps + 3) / 4 : 0;
   const int total = num_main + num_x;
@@ -747,7 +786,7 @@ int launch_variant(dim3 grid, const CUtensorMap& tA, const CUtensorMap& tP, cons
     at[na].val.programmaticStreamSerializationAllowed = 1;
     ++na;
   }
-  if (grid.z > 1) {
+  if (grid.z > 1 && p.zstride == 0) {
     at[na].id = cudaLaunchAttributeClusterDimension;
     at[na].val.clusterDim.x = 1;
     at[na].val.clusterDim.y = 1;
@@ -763,21 +802,76 @@ int launch_variant(dim3 grid, const CUtensorMap& tA, const CUtensorMap& tP, cons
 }
 }  // namespace
 
+namespace gemm {
+// Two 128-row accumulators per CTA (half the decode work per flop) once 256-row tiles alone give
+// at least two waves on the 152 SMs (large M, or a large N such as the LM head).
+int pick_nacc(int64_t M, int64_t N) {
+  const int64_t tiles_n256 = (N + BN - 1) / BN;
+  return (M >= 2048 || (M >= 256 && tiles_n256 * ((M + 255) / 256) >= 2 * 152)) ? 2 : 1;
+}
+}  // namespace gemm
+
+namespace gemm {
+// K split through memory for few output tiles over a long K (the LM head's dH pass and long-K
+// input gradients at a few hundred tokens).  A cluster split is limited by how many clusters fit
+// at once (with one CTA per SM, 16 clusters of 7 or more do not), so 16 tiles got at most 96 of
+// the 152 SMs; unbound CTAs fill them.  The accumulator count and the split count minimise a
+// per-SM time model: K steps per split x the measured time of a 64-deep step (0.60 us with one
+// accumulator, 0.72 with two), plus storing the fp32 partial tile, plus the sum kernel reading
+// every partial (at 4 TB/s).  Used from 128 K steps on and with at most 76 one-accumulator tiles
+// (below that the cluster split or the narrow kernel serve); never more partials than ws_floats.
+struct KSplitPlan {
+  int nacc = 0, splits = 0;
+};
+KSplitPlan plan_ksplit(int64_t M, int64_t N, int64_t K, int64_t ws_floats) {
+  KSplitPlan best;
+  const int64_t num_k = K / BK, tn = (N + BN - 1) / BN;
+  if (M <= 0 || num_k < 128 || tn * ((M + BM - 1) / BM) > 76) return best;
+  double best_t = 0.0;
+  for (int nacc = 1; nacc <= 2; ++nacc) {
+    const int64_t tiles = tn * ((M + BM * nacc - 1) / (BM * nacc));
+    const double tk = nacc == 1 ? 0.60 : 0.72;
+    for (int64_t s = 2; s * tiles <= 152 && s * M * N <= ws_floats; ++s) {
+      const int64_t ks = (num_k + s - 1) / s;
+      const double t = ks * tk + 1.0 * nacc + static_cast<double>(s) * M * N * 4.0 / 4.0e6;
+      if (best.splits == 0 || t < best_t) {
+        best.nacc = nacc;
+        best.splits = static_cast<int>(s);
+        best_t = t;
+      }
+    }
+  }
+  return best;
+}
+}  // namespace gemm
+
+int64_t gemm_ksplit_floats(int64_t M, int64_t N, int64_t K) {
+  const gemm::KSplitPlan k = gemm::plan_ksplit(M, N, K, INT64_MAX);
+  return k.splits ? k.splits * M * N : 0;
+}
+
+// Whether the [M, N] x K GEMM runs on the wide kernel without a K split (the form that can apply
+// the gated activation in its epilogue): two accumulators, or more one-accumulator tiles than
+// the narrow kernel and the K split take.
+bool gemm_glu_fusable(int64_t M, int64_t N, int64_t K) {
+  using namespace gemm;
+  if (M <= 0 || N <= 0 || K <= 0) return false;
+  return pick_nacc(M, N) == 2 || ((N + BN - 1) / BN) * ((M + BM - 1) / BM) > 76;
+}
+
 int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st) {
   using namespace gemm;
   if (g.M <= 0 || g.N <= 0) return MEBP_OK;
   if (g.K % 64 || g.N % 64 || g.K <= 0) return MEBP_ERR_INVALID_ARG;
   const bool glu = g.epi == EPI_GLU;
   if (glu && (g.trans || g.glu_half <= 0 || g.glu_half % 128 || g.N != 2 * g.glu_half)) return MEBP_ERR_UNSUPPORTED;
-  // Two 128-row accumulators per CTA (half the decode work per flop) once 256-row tiles alone give
-  // at least two waves on the 152 SMs (large M, or a large N such as the LM head).
-  const int64_t tiles_n256 = (g.N + BN - 1) / BN;
-  const int nacc = (g.M >= 2048 || (g.M >= 256 && tiles_n256 * ((g.M + 255) / 256) >= 2 * 152)) ? 2 : 1;
+  const bool plain = g.epi == EPI_F32 || g.epi == EPI_F16;
+  const KSplitPlan ks = (plain && g.ksplit_ws) ? plan_ksplit(g.M, g.N, g.K, g.ksplit_floats) : KSplitPlan{};
+  const int nacc = ks.splits ? ks.nacc : pick_nacc(g.M, g.N);
   const int bm = BM * nacc;
   // Few tokens and a short K: 128 x 256 tiles would leave most SMs idle; narrow 128 x 64 tiles
   // instead of a K split (a long K keeps the split: its serial chain would dominate).
-  if (glu && nacc != 2) return MEBP_ERR_UNSUPPORTED;  // the fused GLU epilogue is the two-accumulator one
-  if (nacc == 1 && (g.epi == EPI_F32 || g.epi == EPI_F16) && g.K <= 2560 &&
+  if (!ks.splits && nacc == 1 && plain && g.K <= 2560 &&
       ((g.N + BN - 1) / BN) * ((g.M + BM - 1) / BM) <= 76)
     return launch_dequant_gemm_narrow(g, st);
 
@@ -850,7 +944,15 @@ int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st) {
   // size S <= 8 with >= 2 K tiles per split whose clusters all fit on the GPU at once.
   int splits = 1;
   const int grid_mn = tiles_n * tiles_m;
-  if ((g.epi == EPI_F32 || g.epi == EPI_F16) && nacc == 1 && grid_mn <= 76 && num_k >= 4) {
+  if (ks.splits) {  // through memory: partial tiles in the workspace, summed by ksplit_sum_kernel
+    splits = ks.splits;
+    p.epi = EPI_F32;
+    p.C = g.ksplit_ws;
+    p.ldc = g.N;
+    p.R = nullptr;
+    p.alpha = 1.0f;
+    p.zstride = g.M * g.N;
+  } else if (plain && nacc == 1 && grid_mn <= 76 && num_k >= 4) {
     for (int s = std::min(8, num_k / 2); s >= 2; --s) {
       const int mac = g.trans ? max_active_clusters<true>(s) : max_active_clusters<false>(s);
       if (grid_mn <= mac) {
@@ -881,6 +983,12 @@ int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st) {
     rc = nacc == 2 ? launch_variant<false, 2>(grid, tA, tP, tS, tAx, p, st)
                    : launch_variant<false, 1>(grid, tA, tP, tS, tAx, p, st);
   if (rc) return rc;
+  if (ks.splits) {
+    const int64_t n4 = g.M * (g.N / 4);
+    launch_k(ksplit_sum_kernel, dim3(static_cast<unsigned>((n4 + 255) / 256)), 256, 0, st,
+             static_cast<const float*>(g.ksplit_ws), splits, p.zstride, static_cast<int>(g.M), static_cast<int>(g.N),
+             g.alpha, g.R, g.ldr, g.C, g.ldc, g.epi == EPI_F16 ? 1 : 0, g.err);
+  }
   return cudaGetLastError() == cudaSuccess ? MEBP_OK : MEBP_ERR_CUDA;
 }
 

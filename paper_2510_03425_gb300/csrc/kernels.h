@@ -112,10 +112,20 @@ struct GemmArgs {
   int64_t ldc2 = 0;
   int glu_half = 0;              // EPI_GLU: rows of the gate (= of the up) half of the weight
   int act = 0;                   // EPI_GLU: MEBP_ACT_*
+  // fp32 scratch for a K split through memory (EPI_F32 / EPI_F16 with few output tiles over a
+  // long K); null = cluster splits only.  Not shared between GEMMs that may overlap on the GPU.
+  float* ksplit_ws = nullptr;
+  int64_t ksplit_floats = 0;
   int* err = nullptr;
 };
 
 int launch_dequant_gemm(const GemmArgs& g, cudaStream_t st);
+// True when launch_dequant_gemm runs an [M, N] x K GEMM on the wide kernel without a K split:
+// then EPI_GLU (the gated activation in the epilogue) costs no parallelism.
+bool gemm_glu_fusable(int64_t M, int64_t N, int64_t K);
+// fp32 scratch (floats) the K split through memory wants for an [M, N] x K GEMM; 0 when that
+// shape does not split through memory.
+int64_t gemm_ksplit_floats(int64_t M, int64_t N, int64_t K);
 // The 128 x 64-tile variant for few-token GEMMs (EPI_F16 / EPI_F32); launch_dequant_gemm routes
 // to it when the 128 x 256 tiles would leave most SMs idle.
 int launch_dequant_gemm_narrow(const GemmArgs& g, cudaStream_t st);

@@ -156,6 +156,10 @@ struct mebp_ctx {
   int64_t attn_ws_floats = 0;
   float* red = nullptr;
   int64_t red_floats = 0;
+  // fp32 partials of fused GEMMs split over K through memory: [0] for GEMMs on the caller's
+  // stream, [1] for the recompute stream (the two overlap on the GPU)
+  float* ksplit[2] = {nullptr, nullptr};
+  int64_t ksplit_floats = 0;
   // LM head
   uint16_t *hf = nullptr, *dz = nullptr;
   float *rf = nullptr, *part = nullptr, *zt = nullptr, *lse_tok = nullptr, *tok_loss = nullptr,
@@ -331,6 +335,8 @@ double gemm_bytes(const GemmArgs& g) {
 
 int run_gemm(mebp_ctx* c, GemmArgs& g, cudaStream_t st, const char* what) {
   g.err = c->d_err;
+  g.ksplit_ws = (st == c->fstream && c->fstream) ? c->ksplit[1] : c->ksplit[0];
+  g.ksplit_floats = g.ksplit_ws ? c->ksplit_floats : 0;
   int rc = MEBP_OK;
   KP(c, g.trans ? KK_GEMM_DX : KK_GEMM_FWD, gemm_bytes(g),
      2.0 * g.M * g.N * g.K + (g.Ax ? 2.0 * g.M * g.N * g.kx : 0.0), st, [&] { rc = launch_dequant_gemm(g, st); });
@@ -448,9 +454,13 @@ int block_forward(mebp_ctx* c, int set, int layer, const mebp_block_weights* w, 
     });
     g.Ax = A.us[LIN_GU]; g.ldax = lg.kxp; g.kx = lg.kxp; g.Bx = A.sh->B_cat[LIN_GU]; g.ldbx = lg.kxp;
   }
-  // From 2048 tokens the gate|up GEMM's epilogue applies the activation itself (EPI_GLU, the
-  // two-accumulator kernel): it writes m and, when a backward will read them, gate and up.
-  const bool fuse_glu = T >= 2048 && I % 128 == 0 && lg.N == 2 * I;
+  // When the gate|up GEMM runs on the wide kernel without a K split, its epilogue applies the
+  // activation itself (EPI_GLU): it writes m and, when a backward will read them, gate and up.
+  // Below 2048 tokens (one-accumulator tiles) only when gate and up need not be kept: storing
+  // all three from the epilogue lengthened each tile more than the separate GLU launch cost
+  // (Gemma3-1B shape, 1024 tokens: 13.59 vs 13.49 ms per step).
+  const bool fuse_glu =
+      I % 128 == 0 && lg.N == 2 * I && gemm_glu_fusable(T, lg.N, lg.K) && (T >= 2048 || !keep_gu);
   if (fuse_glu) {
     g.epi = EPI_GLU; g.C = A.m; g.ldc = I; g.C2 = keep_gu ? A.gu : nullptr; g.ldc2 = lg.N; g.glu_half = I;
     g.act = c->cfg.act;
@@ -914,6 +924,21 @@ int mebp_ctx_create(const mebp_model_cfg* cfg, int device, mebp_ctx** out) {
     A(&c->hf, T * D); A(&c->rf, T); A(&c->part, T * c->nparts * 2); A(&c->zt, T); A(&c->lse_tok, T);
     A(&c->tok_loss, T); A(&c->dz, T * c->vchunk); A(&c->dhf, T * D); A(&c->targets, T);
   }
+  // K-split partials: the largest any of the step's fused GEMMs wants at T tokens (forward and
+  // input-gradient shapes of the four linears, the LM head's dH pass over one vocabulary chunk)
+  {
+    int64_t kf = c->V > 0 ? gemm_ksplit_floats(T, D, c->vchunk) : 0;
+    for (int li = 0; li < 4; ++li) {
+      kf = std::max(kf, gemm_ksplit_floats(T, c->lin[li].N, c->lin[li].K));
+      kf = std::max(kf, gemm_ksplit_floats(T, c->lin[li].K, c->lin[li].N));
+    }
+    c->ksplit_floats = kf;
+    c->cur_cat = MEBP_WS_OTHER;
+    if (kf > 0) {
+      A(&c->ksplit[0], kf);
+      if (c->nsets == 2) A(&c->ksplit[1], kf);
+    }
+  }
   const int64_t nslots = f.spill_ckpts ? kCkptSlots : (c->L + 1);
   c->cur_cat = MEBP_WS_CKPT;
   A(&c->ckpt, nslots * T * D);
@@ -1216,7 +1241,8 @@ int mebp_block_recompute_fwd(mebp_ctx* c, int layer, const mebp_block_weights* w
   if (!x || !y || !aligned16(x) || !aligned16(y)) return fail(c, MEBP_ERR_INVALID_ARG, "x / y must be 16-byte aligned");
   if (x == y) return fail(c, MEBP_ERR_INVALID_ARG, "x and y must not alias");
   pdl_entry();
-  rc = block_forward(c, 0, layer, w, lora, x, y, B, Sq, true, S(stream));
+  // without save_for_bwd gate and up need not be kept (the gate|up GEMM may store m alone)
+  rc = block_forward(c, 0, layer, w, lora, x, y, B, Sq, true, S(stream), nullptr, save_for_bwd != 0);
   if (!save_for_bwd) c->act[0].layer = -1;
   return rc;
 }

@@ -140,6 +140,29 @@ def test_saved_intermediates_give_the_same_backward_as_recompute():
         np.testing.assert_array_equal(np_of(b), gpu["grads"][n][1])
 
 
+@pytest.mark.parametrize("tokens,act", [(512, "silu"), (1024, "gelu_tanh"), (2048, "silu")])
+def test_gated_activation_in_the_gemm_epilogue_is_bit_identical(tokens, act):
+    """Without save_for_bwd the gate|up GEMM applies the gated activation in its epilogue and
+    stores m alone (one-accumulator tiles below 2048 tokens, two from 2048); with it, gate and up
+    are stored for the backward and, below 2048 tokens, a separate kernel computes m.  Both round
+    gate and up to fp16 first, so the block outputs agree bit for bit."""
+    dims = synth.tiny(hidden=256, n_heads=4, n_kv_heads=2, head_dim=64, intermediate=2560, act=act, n_layers=1,
+                      vocab=0, batch=1, seq=tokens, rank=16)
+    W = synth.block_weights(dims, 0)
+    L = synth.lora_weights(dims, 0)
+    ctx = Context(dims)
+    blk = DeviceBlock(ctx, {k: to_gpu(v) for k, v in W.items()})
+    ls = LoraSet([L])
+    xg = to_gpu(synth.hidden_input(dims))
+    y0, y1 = torch.empty_like(xg), torch.empty_like(xg)
+    M.mebp_block_recompute_fwd(ctx.handle, 0, blk.struct(), ls.layer(0), xg, y0, 1, tokens, False)
+    M.mebp_block_recompute_fwd(ctx.handle, 0, blk.struct(), ls.layer(0), xg, y1, 1, tokens, True)
+    ctx.sync()
+    assert torch.isfinite(y0).all()
+    assert torch.equal(y0, y1)
+    ctx.close()
+
+
 def test_gradient_accumulation_adds():
     dims = synth.preset(0)
     gpu, _, (ctx, blk, ls, xg, Gg) = run_block(dims)

@@ -157,6 +157,92 @@ def test_linear_with_lora_against_oracle(ctx, r, Mr, N, K):
     assert rel_fro(got_term, lora_term) < 1e-2
 
 
+# K split through memory.  A context sized for the Qwen2.5-0.5B-shaped step (512 tokens) holds
+# fp32 partial-tile scratch (its gate|up dX and LM-head dH passes want it); a GEMM with few output
+# tiles over a long K then runs as tiles x splits CTAs not bound to clusters, and a second launch
+# sums the partials in split order.  (trans, M, N, K) in GEMM terms: an M x N output over K; the
+# comments give the plan (accumulators per CTA, splits).
+KSPLIT = [(True, 512, 896, 9728),     # the gate|up dX shape: one accumulator, 9 splits
+          (True, 300, 640, 8256),     # ragged rows, 129 K steps
+          (False, 200, 576, 16384),   # forward: one accumulator, 25 splits
+          (True, 512, 896, 32768)]    # two accumulators, 19 splits (152 CTAs)
+
+
+@pytest.fixture(scope="module")
+def kctx():
+    c = Context(synth.preset(1), max_tokens=512, max_seq=512)
+    yield c
+    c.close()
+
+
+@pytest.mark.parametrize("trans,Mr,N,K", KSPLIT)
+def test_ksplit_through_memory_matches_exact_operand_product(kctx, trans, Mr, N, K):
+    """No LoRA: the split GEMM equals the operand product up to fp32 accumulation (fp32 and, in
+    the forward, fp16 outputs and a residual), is deterministic, and ran as two launches."""
+    rng = np.random.default_rng(K + Mr)
+    W = _w(K, N, 31) if trans else _w(N, K, 31)        # dX = dY W with W [K_gemm, N_gemm]
+    qo, so = quant.compress(W)
+    Wd = quant.f16_bits_to_f64(quant.dequant_f16_bits(qo, so))
+    X = _x(Mr, K, 7)
+    ref = X @ Wd if trans else X @ Wd.T
+    Wp = M.packed(to_gpu(qo), to_gpu(so))
+    Xg = to_gpu(X.astype(np.float32)).to(torch.float16)
+    y = torch.empty((Mr, N), dtype=torch.float32, device="cuda")
+    y2 = torch.empty_like(y)
+    run = (lambda out: M.mebp_linear_dx(kctx.handle, Xg, Wp, dx=out)) if trans else \
+        (lambda out: M.mebp_linear_fwd(kctx.handle, Xg, Wp, y_f32=out))
+    n0 = M.mebp_kernel_launches()
+    run(y)
+    assert M.mebp_kernel_launches() - n0 == 2          # the GEMM and the split sum
+    run(y2)
+    kctx.sync()
+    scale = np.abs(ref).max()
+    assert np.abs(np_of(y) - ref).max() <= 2e-5 * scale + 1e-6
+    assert torch.equal(y, y2)
+    if not trans:
+        R = rng.standard_normal((Mr, N)).astype(np.float32)
+        yr = torch.empty_like(y)
+        yb = torch.empty((Mr, N), dtype=torch.float16, device="cuda")
+        M.mebp_linear_fwd(kctx.handle, Xg, Wp, R=to_gpu(R), y_f32=yr)
+        M.mebp_linear_fwd(kctx.handle, Xg, Wp, y_f16=yb)
+        kctx.sync()
+        assert np.abs(np_of(yr) - (ref + R)).max() <= 2e-5 * (scale + np.abs(R).max()) + 1e-6
+        assert np.abs(np_of(yb) - ref).max() <= 1e-3 * scale + 1e-6
+
+
+@pytest.mark.parametrize("trans", [False, True])
+def test_ksplit_through_memory_with_lora_against_oracle(kctx, trans):
+    """The LoRA block rides with the last split: Y = X deq(W)^T + s (X A^T) B^T + R and
+    dX = dY deq(W) + s (dY B) A against fp64 at split shapes."""
+    s, r = 2.0, 16
+    rng = np.random.default_rng(5)
+    Mr, Nl, Kl = (300, 9728, 896) if trans else (300, 576, 16384)   # the layer's W is [Nl, Kl]
+    qo, so = quant.compress(_w(Nl, Kl, 12))
+    Wd = quant.dequant(qo, so)
+    A = (rng.standard_normal((r, Kl)) * 0.05).astype(np.float32)
+    B = (rng.standard_normal((Nl, r)) * 0.05).astype(np.float32)
+    Wp = M.packed(to_gpu(qo), to_gpu(so))
+    Ag, Bg = to_gpu(A), to_gpu(B)
+    if trans:
+        dY = _x(Mr, Nl, 8)
+        ref = dY @ Wd + s * (dY @ B.astype(np.float64)) @ A.astype(np.float64)
+        out = torch.empty((Mr, Kl), dtype=torch.float32, device="cuda")
+        M.mebp_linear_dx(kctx.handle, to_gpu(dY.astype(np.float32)).to(torch.float16), Wp, Ag, Bg, r, s, dx=out)
+        kctx.sync()
+        assert rel_fro(np_of(out), ref) < 2e-3
+    else:
+        X = _x(Mr, Kl, 9)
+        R = rng.standard_normal((Mr, Nl)).astype(np.float32)
+        ref = X @ Wd.T + s * (X @ A.T.astype(np.float64)) @ B.T.astype(np.float64) + R
+        out = torch.empty((Mr, Nl), dtype=torch.float32, device="cuda")
+        M.mebp_linear_fwd(kctx.handle, to_gpu(X.astype(np.float32)).to(torch.float16), Wp, Ag, Bg, r, s,
+                          R=to_gpu(R), y_f32=out)
+        kctx.sync()
+        assert rel_fro(np_of(out) - R, ref - R) < 2e-3
+        base = X @ Wd.T
+        assert rel_fro(np_of(out).astype(np.float64) - R - base, ref - R - base) < 1e-2
+
+
 def test_lora_b_zero_is_bit_identical_to_base(ctx):
     Mr, N, K, r = 257, 512, 384, 16
     W = _w(N, K, 21)
