@@ -56,7 +56,7 @@ struct BwdArgs {
 // dqkv from the split partials: dQ = sum over parts; dK, dV = sum over the group's query heads and
 // parts (fixed order); q and k then rotated back by their RoPE angle when cs != null (the VJP of
 // the rotation: (d1, d2) -> (d1 c + d2 s, d2 c - d1 s)).  One thread per (token, head slot, pair j).
-constexpr int kFinishMax = 16;  // partials per element: query heads per kv head (<= 8) x parts (2)
+constexpr int kFinishMax = 16;  // partials per element: query heads per kv head (<= 8) x parts (<= 2)
 template <int HD>
 __global__ void bwd_finish_kernel(const BwdArgs a, const float2* __restrict__ cs) {
   griddep_wait();
@@ -126,7 +126,10 @@ bool launch_attn_bwd(const uint16_t* qkv, int64_t ld, const uint16_t* o, const u
   // over every query head of its group and every query block, so the work is split into
   // (query head, part) items instead, summed by the finish kernel.
   const int64_t kv_tiles = static_cast<int64_t>((S + 127) / 128) * KV * B * (hd == 256 ? 2 : 1);
-  constexpr int P = 2;
+  // query blocks of a head split in P parts: two at hd 64 / 128, one at hd 256 (measured per
+  // step: Gemma3-1B shape, hd 256, 1024 tokens, 13.19 ms with one part, 13.56 with two;
+  // Qwen2.5-0.5B shape, hd 64, 512 tokens, 5.44 with two, 5.48 with one)
+  const int P = hd == 256 ? 1 : 2;
   const int nb = (S + 63) / 64;
   const int64_t part_floats = static_cast<int64_t>(B) * nb * H * P * 64 * hd;  // per array
   if (kv_tiles < 152 && ws && 3 * part_floats <= ws_floats && (H / KV) * P <= attn::kFinishMax) {

@@ -412,12 +412,15 @@ int fwd_launch(const uint16_t* qkv, int64_t ld, int B, int S, int H, int KV, uin
     rc = make_tmap_3d(&tmkv, qkv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, ld, S, B, ld * 2, seq, 64, Fwd<HD>::BK, 1,
                       CU_TENSOR_MAP_SWIZZLE_128B);
   if (rc) return rc;
-  // grids under one wave share each query tile's key blocks among a cluster of 2 or 4 CTAs
+  // grids under one wave whose longest query tiles see at least 8 key blocks share each tile's
+  // key blocks among a cluster of 2 or 4 CTAs (Gemma3-1B shape, 1024 tokens).  With fewer blocks
+  // the cluster merge costs more than the shorter chain saves (Qwen2.5-0.5B shape, 512 tokens:
+  // 5.36 ms per step without the split, 5.44 with pairs).
   const int64_t tiles = static_cast<int64_t>((S + BQ - 1) / BQ) * H * B;
   const int nkb_max = (S + Fwd<HD>::BK - 1) / Fwd<HD>::BK;
-  if (tiles * 4 <= 152 && nkb_max >= 4)
+  if (tiles * 4 <= 152 && nkb_max >= 8)
     return fwd_launch_cl<HD, WIN, 4>(tm, tmkv, B, S, H, KV, o, ldo, lse, W, err, st);
-  if (tiles * 2 <= 152 && nkb_max >= 2)
+  if (tiles * 2 <= 152 && nkb_max >= 8)
     return fwd_launch_cl<HD, WIN, 2>(tm, tmkv, B, S, H, KV, o, ldo, lse, W, err, st);
   return fwd_launch_cl<HD, WIN, 1>(tm, tmkv, B, S, H, KV, o, ldo, lse, W, err, st);
 }
