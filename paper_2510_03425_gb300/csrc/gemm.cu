@@ -200,7 +200,7 @@ __device__ __forceinline__ void copy_lora_b(const Params& p, int e, int n0, uint
 // slot, 16-byte chunk c of row r at chunk c ^ (r & 7) within its 128-byte half (no bank
 // conflicts).  Phase 2: the warp copies the slot out with consecutive lanes on consecutive chunks
 // of a row, so each instruction writes (and, for the residual, reads) whole 128-byte lines.
-template <int NACC>
+template <bool TRANS, int NACC>
 __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int warp, int lane, int m0, int n0,
                                          uint8_t* stage) {
   const int q = warp & 3, cg = warp >> 2;
@@ -215,14 +215,14 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
   const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * q) << 16) + 256 * acc + col0;
   const int cbase = n0 + col0;  // first GEMM column of this thread's range
 
-  if (p.epi == EPI_LSE) {
+  if (!TRANS && p.epi == EPI_LSE) {  // the LM-head epilogues run on forward GEMMs only
     float mx = -INFINITY, sum = 0.0f, zt = 0.0f;
     bool has_t = false;
     const int tgt = row_ok ? p.targets[row] - p.col_offset : -1;
-#pragma unroll 1
-    for (int cc = 0; cc < NCH; ++cc) {
+    auto chunk = [&](const uint32_t (&r)[32], int cc) {
       float v[32];
-      tmem_ld32(tbase + 32 * cc, v);
+#pragma unroll
+      for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
       const int c0 = cbase + 32 * cc;
       float cm = -INFINITY;
 #pragma unroll
@@ -239,6 +239,28 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
         sum = sum * __expf(mx - nm) + acc;
         mx = nm;
       }
+    };
+    static_assert(NCH % 2 == 0, "chunks are processed in pairs");
+    uint32_t ra[32];
+    if constexpr (NACC == 2) {  // the TMEM loads run one chunk ahead of the arithmetic
+      uint32_t rb[32];
+      tmem_ld32_issue(tbase, ra);
+#pragma unroll 1
+      for (int cc = 0; cc < NCH; cc += 2) {
+        tmem_wait_ld32(ra);
+        tmem_ld32_issue(tbase + 32 * (cc + 1), rb);
+        chunk(ra, cc);
+        tmem_wait_ld32(rb);
+        if (cc + 2 < NCH) tmem_ld32_issue(tbase + 32 * (cc + 2), ra);
+        chunk(rb, cc + 1);
+      }
+    } else {  // 96 registers a thread: one load at a time
+#pragma unroll 1
+      for (int cc = 0; cc < NCH; ++cc) {
+        tmem_ld32_issue(tbase + 32 * cc, ra);
+        tmem_wait_ld32(ra);
+        chunk(ra, cc);
+      }
     }
     if (row_ok) {  // four (max, sum) parts per 256-column tile and row; unused parts are empty
       float2* pr = reinterpret_cast<float2*>(p.lse_part) + static_cast<int64_t>(row) * p.nparts + (n0 / BN) * 4;
@@ -253,7 +275,7 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
   }
 
   {
-    if (p.epi == EPI_GLU) {
+    if (!TRANS && p.epi == EPI_GLU) {
       // The accumulator holds the gate (columns 0-127) and up (128-255) pre-activations of hidden
       // units j0 .. j0 + 127, j0 = n0 / 2.  NACC = 2: the warp takes all 128 units of its
       // accumulator; NACC = 1: column group cg takes units 32 cg .. +31 (gate and up columns of
@@ -273,8 +295,15 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
         const int j = j0 + u0;
         if (j >= p.glu_half) break;  // warp-uniform
         float gv[32], uv[32];
-        tmem_ld32(tacc + u0, gv);
-        tmem_ld32(tacc + 128 + u0, uv);
+        {  // both loads in flight at once
+          uint32_t rg[32], ru[32];
+          tmem_ld32x2(tacc + u0, tacc + 128 + u0, rg, ru);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            gv[i] = __uint_as_float(rg[i]);
+            uv[i] = __uint_as_float(ru[i]);
+          }
+        }
 #pragma unroll
         for (int c = 0; c < 4; ++c) {  // 8 units per 16-byte chunk
           uint32_t mo[4], go[4], uo[4];
@@ -284,7 +313,7 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
             go[k] = pack_half2(gv[e], gv[e + 1]);
             uo[k] = pack_half2(uv[e], uv[e + 1]);
             mo[k] = pack_half2(act_f(h2_lo(go[k]), p.act) * h2_lo(uo[k]), act_f(h2_hi(go[k]), p.act) * h2_hi(uo[k]));
-            if (row_ok) bad |= h2_nonfinite(mo[k]) | (p.C2 ? h2_nonfinite(go[k]) | h2_nonfinite(uo[k]) : 0u);
+            if (row_ok) bad |= h2_exp_probe(mo[k]) | (p.C2 ? h2_exp_probe(go[k]) | h2_exp_probe(uo[k]) : 0u);
           }
           const int off = lane * 64 + ((c ^ ((lane >> 1) & 3)) << 4);
           *reinterpret_cast<uint4*>(stage + off) = make_uint4(mo[0], mo[1], mo[2], mo[3]);
@@ -309,56 +338,75 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
         }
         __syncwarp();  // the slots are rewritten by the next round
       }
-      if (bad) flag_error(p.err, kErrNonFinite);
+      if (bad & kH2Bad) flag_error(p.err, kErrNonFinite);
       return;
     }
   }
 
   // EPI_F16, EPI_CEGRAD (fp16 rows of 128 bytes per round) and EPI_F32 (fp32, 256 bytes)
-  const bool f32 = p.epi == EPI_F32, ce = p.epi == EPI_CEGRAD;
+  const bool f32 = p.epi == EPI_F32, ce = !TRANS && p.epi == EPI_CEGRAD;
   const float lse = (ce && row_ok) ? p.lse[row] : 0.0f;
   const int tgt = (ce && row_ok) ? p.targets[row] : -1;
   const float cw = (tgt >= 0) ? *p.ce_w : 0.0f;
   const int tl = tgt - p.col_offset;
   const int row0 = row - lane;
-  uint32_t bad = 0;  // an fp16 output overflowed (or is NaN)
+  uint32_t bad = 0;  // OR of h2_exp_probe over the fp16 outputs (an overflow or NaN sets kH2Bad bits)
+  // Phase 1 for one 32-column chunk: half hh of round rd (first column c0 of the round).
+  auto stage32 = [&](float (&v)[32], int hh, int c0) {
+    if (f32) {
+      uint8_t* srow = stage + lane * 256;
+#pragma unroll
+      for (int jj = 0; jj < 8; ++jj) {
+        const int j = 8 * hh + jj;
+        *reinterpret_cast<float4*>(srow + (((j & 8) | ((j ^ lane) & 7)) << 4)) =
+            make_float4(p.alpha * v[4 * jj], p.alpha * v[4 * jj + 1], p.alpha * v[4 * jj + 2], p.alpha * v[4 * jj + 3]);
+      }
+    } else {
+      if (ce) {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const int col = c0 + 32 * hh + i;
+          float a = (col < p.n_valid) ? __expf(v[i] - lse) * cw : 0.0f;
+          if (col == tl) a -= cw;
+          v[i] = a;
+        }
+      }
+      uint8_t* srow = stage + lane * 128;
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj) {
+        const int j = 4 * hh + jj;
+        const uint4 o = make_uint4(pack_half2(v[8 * jj], v[8 * jj + 1]), pack_half2(v[8 * jj + 2], v[8 * jj + 3]),
+                                   pack_half2(v[8 * jj + 4], v[8 * jj + 5]), pack_half2(v[8 * jj + 6], v[8 * jj + 7]));
+        if (!ce && row_ok) bad |= h2_exp_probe(o.x) | h2_exp_probe(o.y) | h2_exp_probe(o.z) | h2_exp_probe(o.w);
+        *reinterpret_cast<uint4*>(srow + (((j ^ lane) & 7) << 4)) = o;
+      }
+    }
+  };
 #pragma unroll 1
   for (int rd = 0; rd < COLS / 64; ++rd) {
     const int c0 = cbase + 64 * rd;
     if (c0 >= p.N) break;  // warp-uniform (N is a multiple of 64)
-    // ---- phase 1: this thread's row into the slot, 32 columns at a time (registers)
+    // ---- phase 1: this thread's row into the slot.  Forward GEMMs with fp16 outputs: both
+    // 32-column loads of the round in flight at once (loading one round ahead as well needs more
+    // than the 168 registers a thread has); otherwise one load at a time (the transposed kernel
+    // keeps its 122 registers: with the forward's paths compiled in it ran 2-4 % slower)
+    if (f32 || TRANS) {
 #pragma unroll 1
-    for (int hh = 0; hh < 2; ++hh) {
-      float v[32];
-      tmem_ld32(tbase + 64 * rd + 32 * hh, v);
-      if (f32) {
-        uint8_t* srow = stage + lane * 256;
-#pragma unroll
-        for (int jj = 0; jj < 8; ++jj) {
-          const int j = 8 * hh + jj;
-          *reinterpret_cast<float4*>(srow + (((j & 8) | ((j ^ lane) & 7)) << 4)) =
-              make_float4(p.alpha * v[4 * jj], p.alpha * v[4 * jj + 1], p.alpha * v[4 * jj + 2], p.alpha * v[4 * jj + 3]);
-        }
-      } else {
-        if (ce) {
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const int col = c0 + 32 * hh + i;
-            float a = (col < p.n_valid) ? __expf(v[i] - lse) * cw : 0.0f;
-            if (col == tl) a -= cw;
-            v[i] = a;
-          }
-        }
-        uint8_t* srow = stage + lane * 128;
-#pragma unroll
-        for (int jj = 0; jj < 4; ++jj) {
-          const int j = 4 * hh + jj;
-          const uint4 o = make_uint4(pack_half2(v[8 * jj], v[8 * jj + 1]), pack_half2(v[8 * jj + 2], v[8 * jj + 3]),
-                                     pack_half2(v[8 * jj + 4], v[8 * jj + 5]), pack_half2(v[8 * jj + 6], v[8 * jj + 7]));
-          if (!ce && row_ok) bad |= h2_nonfinite(o.x) | h2_nonfinite(o.y) | h2_nonfinite(o.z) | h2_nonfinite(o.w);
-          *reinterpret_cast<uint4*>(srow + (((j ^ lane) & 7) << 4)) = o;
-        }
+      for (int hh = 0; hh < 2; ++hh) {
+        float v[32];
+        tmem_ld32(tbase + 64 * rd + 32 * hh, v);
+        stage32(v, hh, c0);
       }
+    } else {
+      uint32_t ra[32], rb[32];
+      tmem_ld32x2(tbase + 64 * rd, tbase + 64 * rd + 32, ra, rb);
+      float v[32];
+#pragma unroll
+      for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(ra[i]);
+      stage32(v, 0, c0);
+#pragma unroll
+      for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(rb[i]);
+      stage32(v, 1, c0);
     }
     __syncwarp();
     // ---- phase 2: whole lines out (rows past M skipped)
@@ -389,7 +437,7 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
     }
     __syncwarp();  // the slot is rewritten by the next round
   }
-  if (bad) flag_error(p.err, kErrNonFinite);
+  if (bad & kH2Bad) flag_error(p.err, kErrNonFinite);
 }
 
 // ---------------------------------------------------------------------------------- split-K
@@ -658,7 +706,7 @@ __global__ void __launch_bounds__(Warps<NACC>::THREADS, 1)
     const bool acc_ok = __all_sync(0xffffffffu, mbar_wait(accf, 0, abort_flag, p.err));
     tc_fence_after();
     if (split) stash_partial(tmem, acc_ok && total > 0, warp, lane, smem);
-    else if (acc_ok && total > 0) epilogue<NACC>(p, tmem, warp, lane, m0, n0, smem + warp * 8192);
+    else if (acc_ok && total > 0) epilogue<TRANS, NACC>(p, tmem, warp, lane, m0, n0, smem + warp * 8192);
   }
 
   tc_fence_before();
