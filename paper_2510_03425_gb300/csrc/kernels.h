@@ -76,7 +76,7 @@ inline cudaError_t launch_k_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 bl
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
-// EPI_GLU (forward, two accumulators): the weight is the fused [gate; up] matrix of 2 glu_half rows;
+// EPI_GLU (forward, wide kernel, no K split): the weight is the fused [gate; up] matrix of 2 glu_half rows;
 // 256-column tile t holds gate rows 128 t .. 128 t + 127 and the matching up rows, and the epilogue
 // writes m = act(gate) * up (fp16, C [M, glu_half]) and, with C2, gate and up (fp16, [M, 2 glu_half]).
 enum GemmEpi { EPI_F16 = 0, EPI_F32 = 1, EPI_LSE = 2, EPI_CEGRAD = 3, EPI_GLU = 4 };
