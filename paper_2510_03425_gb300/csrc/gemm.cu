@@ -388,8 +388,9 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t tmem, int war
     if (c0 >= p.N) break;  // warp-uniform (N is a multiple of 64)
     // ---- phase 1: this thread's row into the slot.  Forward GEMMs with fp16 outputs: both
     // 32-column loads of the round in flight at once (loading one round ahead as well needs more
-    // than the 168 registers a thread has); otherwise one load at a time (the transposed kernel
-    // keeps its 122 registers: with the forward's paths compiled in it ran 2-4 % slower)
+    // than the 168 registers a thread has); otherwise one load at a time (the transposed kernel,
+    // without the forward-only paths, stays at 106 registers: with them compiled in, at 168, it
+    // ran 2-4 % slower)
     if (f32 || TRANS) {
 #pragma unroll 1
       for (int hh = 0; hh < 2; ++hh) {
