@@ -286,6 +286,23 @@ def model_bytes(model, ls):
     return pw, 2 * 4 * ls.n  # packed weights (+ scales); LoRA masters + gradients (fp32)
 
 
+def max_over_ranks(x: float, dist, device=None) -> float:
+    """The largest of every rank's x (a job's time is its slowest rank's); x itself when there is
+    no process group.  NCCL reduces a device tensor, gloo a host one."""
+    if dist is None:
+        return x
+    import torch
+    dev = device if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tokens_per_s(tokens_per_rank: int, steps: int, world: int, seconds: float) -> float:
+    """Whole-job throughput: the tokens every rank processed over the slowest rank's time."""
+    return world * tokens_per_rank * steps / seconds
+
+
 def run_gpu(args, d, rank, world, local_rank):
     import torch
 
@@ -333,11 +350,8 @@ def run_gpu(args, d, rank, world, local_rank):
     clk = clocks.stop()
     ctx.sync()
     free1, _ = torch.cuda.mem_get_info(device)
-    if dist:
-        tt = torch.tensor([t], device=device)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        t = float(tt.item())
-    value = world * d.tokens * args.steps / t
+    t = max_over_ranks(t, dist, device)
+    value = job_tokens_per_s(d.tokens, args.steps, world, t)
 
     # ---- per-kernel CUDA events over K more steps (run eagerly: the events order each launch on
     # its stream), the fused GEMMs' union of busy intervals, and the step's wall time meanwhile
@@ -356,11 +370,7 @@ def run_gpu(args, d, rank, world, local_rank):
         ids.copy_(ids_host, non_blocking=True)
         step()
         loss_host.copy_(loss, non_blocking=True)
-    te = time_steps(e2e_step, args.steps, st)
-    if dist:
-        tt = torch.tensor([te], device=device)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        te = float(tt.item())
+    te = max_over_ranks(time_steps(e2e_step, args.steps, st), dist, device)
     ctx.sync()
     peak_torch = torch.cuda.max_memory_allocated(device)
     ws = M.mebp_workspace_bytes(ctx.handle)
@@ -447,8 +457,8 @@ def run_gpu(args, d, rank, world, local_rank):
                    "device_used_bytes": total - free0,
                    "step_allocates_nothing": free0 == free1,
                    **({"min_memory": mm} if mm else {})},
-        "e2e": {"value": world * d.tokens * args.steps / te, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h},
+        "e2e": {"value": job_tokens_per_s(d.tokens, args.steps, world, te), "unit": "tokens/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": int(launches),
         "clocks": clk,
     }

@@ -58,3 +58,38 @@ def test_gpu_arm_fails_loudly_without_cuda():
                        capture_output=True, text=True, timeout=600)
     assert r.returncode != 0
     assert not any(ln.startswith("{") and '"value"' in ln for ln in r.stdout.splitlines())
+
+
+def _rank_worker(rank, world, port, out):
+    import torch.distributed as dist
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        # each rank's own time; the job's is the slowest rank's, on every rank
+        t = bench.max_over_ranks(1.5 + rank, dist)
+        out[rank] = (t, bench.job_tokens_per_s(16384, 20, world, t))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_ranks_report_the_slowest_rank_and_the_whole_job():
+    """The N > 1 path's host logic over two gloo ranks: every rank gets the maximum time, and the
+    value counts the tokens of both ranks over it (weak scaling: fixed work per rank)."""
+    import socket
+
+    import torch.multiprocessing as mp
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        port = s.getsockname()[1]
+    out = mp.Manager().dict()
+    mp.spawn(_rank_worker, args=(2, port, out), nprocs=2, join=True)
+    assert dict(out) == {0: (2.5, 2 * 16384 * 20 / 2.5), 1: (2.5, 2 * 16384 * 20 / 2.5)}
+    assert bench.max_over_ranks(3.0, None) == 3.0
+
+
+def test_reference_arm_on_a_second_rank_exits_without_work():
+    env = dict(os.environ, RANK="1", WORLD_SIZE="2", LOCAL_RANK="1")
+    r = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--config", "1", "--steps", "1",
+                        "--warmup", "3"], cwd=ROOT, capture_output=True, text=True, timeout=120, env=env)
+    assert r.returncode == 0, r.stderr[-2000:]
+    assert r.stdout.strip() == ""
