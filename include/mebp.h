@@ -11,6 +11,9 @@
  *    void*; NULL = the legacy default stream).  Device-side failures (a
  *    bounded wait that expired, a bad token id) are recorded in the context's
  *    device error word and reported by mebp_sync().
+ *  - A context's workspace (intermediates, split partials, LM-head buffers) is
+ *    shared by its calls: issue the calls of one context on one stream, or
+ *    order the streams they use; calls that overlap on the GPU race on it.
  *  - Every call returns an int status (MEBP_OK on success).  No exception or
  *    abort crosses the ABI; mebp_last_error() gives a message.
  *  - Dense activations are row-major [tokens, features]; token t = b*S + s.
